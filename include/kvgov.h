@@ -1,0 +1,205 @@
+/*
+ * kvgov.h -- C ABI of libkvgov: the salted block-hash chain and block
+ * prefix-cache probe of KVGov (arxiv 2608.09225), on one GB300 (sm_103a).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Pointers named d_* are DEVICE pointers owned by the caller.  Nothing
+ *    here allocates device or host memory, synchronises, or keeps a pointer
+ *    after returning.  Every call only enqueues kernels on `stream` (a
+ *    cudaStream_t; NULL is the legacy default stream) and returns.
+ *  - Return value: KVGOV_OK, or a host-detected error (KVGOV_EINVAL for a bad
+ *    argument, KVGOV_ECUDA when a launch fails).  On a host-detected error
+ *    nothing is enqueued.
+ *  - Errors that only the device can see (a bad per-request index, a
+ *    reserved key, a full table, a wait that ran out) are OR-ed as
+ *    KVGOV_F_* bits into the u32 at d_status.  The caller zeroes it before
+ *    the call and reads it after synchronising.  Where d_status may be NULL
+ *    the flags are dropped.
+ *  - A token is an int32; the hashed bytes of a token are its 4 bytes in
+ *    little-endian order.  A block is KVGOV_BLOCK = 16 consecutive tokens of
+ *    one request; only full blocks are hashed (a request of len tokens has
+ *    n_b = floor(len / 16) blocks; the tail is not hashed).  A digest is the
+ *    32-byte SHA-256 output.
+ *  - Requests are given in CSR form: request r is tokens
+ *    d_tokens[d_tok_off[r] .. d_tok_off[r+1]), d_tok_off non-decreasing,
+ *    int64.  Block-level outputs are request-major: block j of request r is
+ *    row d_blk_off[r] + j, with d_blk_off the exclusive prefix sum of n_b
+ *    (see kvgov_block_offsets).
+ */
+#ifndef KVGOV_H
+#define KVGOV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t / CUstream. */
+typedef struct CUstream_st *kvgov_stream_t;
+
+#define KVGOV_BLOCK 16             /* tokens per block, B in the paper        */
+#define KVGOV_DIGEST_BYTES 32      /* SHA-256 digest and table key size       */
+#define KVGOV_MAX_SECRET 1024      /* longest HMAC key kvgov_derive_salts takes */
+#define KVGOV_MIN_CAPACITY 32      /* smallest table capacity (slots)         */
+
+/* Return codes (host-detected). */
+#define KVGOV_OK 0
+#define KVGOV_EINVAL 1             /* bad argument; nothing was enqueued      */
+#define KVGOV_ECUDA 2              /* a kernel launch failed                  */
+
+/* Device-detected flags, OR-ed into *d_status. */
+#define KVGOV_F_BADINDEX 0x10u     /* a principal index, boundary offset or
+                                      offset array entry was out of range; the
+                                      affected request produced no output     */
+#define KVGOV_F_SENTINEL 0x20u     /* a key whose first 8 bytes are all 0x00 or
+                                      all 0xFF was given to kvgov_insert; it is
+                                      skipped (these values mark empty and
+                                      claimed slots)                          */
+#define KVGOV_F_TABLE_FULL 0x40u   /* kvgov_insert found no free slot for a key */
+#define KVGOV_F_TIMEOUT 0x80u      /* kvgov_insert gave up waiting for another
+                                      thread's claimed slot to be published   */
+
+/* Salt placement (paper section 2.1 equation, section 4.1, section 4.2). */
+#define KVGOV_UNSALTED 0           /* h_0 = H(T_0), h_j = H(h_{j-1} || T_j)   */
+#define KVGOV_ROOT 1               /* h_0 = H(sigma_p || T_0), then chained   */
+#define KVGOV_BOUNDARY 2           /* salt injected at block k = floor(b/16)  */
+
+/*
+ * kvgov_status_string -- a static, human-readable name for a return code or
+ * for a single KVGOV_F_* flag.  Never NULL.
+ */
+const char *kvgov_status_string(int status);
+
+/*
+ * kvgov_block_offsets -- blocking, paper section 2.1 (keys are per B-token
+ * block; only full blocks are keyed).
+ *
+ *   d_tok_off [n_req + 1] int64, non-decreasing token offsets (CSR).
+ *   d_blk_off [n_req + 1] int64 output: d_blk_off[0] = 0 and
+ *             d_blk_off[r+1] = d_blk_off[r] + floor(len_r / 16).
+ *   d_status  nullable; KVGOV_F_BADINDEX if some len_r < 0 (that request
+ *             then counts 0 blocks).
+ * n_req = 0 writes d_blk_off[0] = 0.  EINVAL: n_req < 0 or a NULL array.
+ */
+int kvgov_block_offsets(const int64_t *d_tok_off, int32_t n_req, int64_t *d_blk_off,
+                        uint32_t *d_status, kvgov_stream_t stream);
+
+/*
+ * kvgov_derive_salts -- per-principal salt, paper section 4.1:
+ * sigma_p = HMAC_K(secret, principal_id), HMAC per RFC 2104 with SHA-256.
+ *
+ *   secret, secret_len  HOST bytes of the server secret K, the HMAC key
+ *                       (0 <= secret_len <= KVGOV_MAX_SECRET; keys longer
+ *                       than 64 bytes are first hashed, as RFC 2104 says).
+ *                       Copied into the launch; the host buffer may be
+ *                       reused as soon as the call returns.
+ *   d_ids, d_id_off     the principal ids as byte strings in CSR form:
+ *                       principal p is d_ids[d_id_off[p] .. d_id_off[p+1]).
+ *   d_salts             [n_principals][32] u8 output.
+ *   d_status            nullable; KVGOV_F_BADINDEX for a negative or
+ *                       decreasing id offset (that salt is left untouched).
+ * n_principals = 0 is a no-op.  EINVAL: secret_len too large, secret NULL
+ * with secret_len > 0, n_principals < 0, a NULL device array.
+ */
+int kvgov_derive_salts(const uint8_t *secret, size_t secret_len, const uint8_t *d_ids,
+                       const int64_t *d_id_off, int32_t n_principals, uint8_t *d_salts,
+                       uint32_t *d_status, kvgov_stream_t stream);
+
+/*
+ * kvgov_chain_hash -- the chained block digests of every request:
+ *   UNSALTED (paper section 2.1):  h_0 = H(T_0), h_j = H(h_{j-1} || T_j);
+ *   ROOT     (section 4.1):        h_0 = H(sigma_p || T_0), h_j as above;
+ *   BOUNDARY (section 4.2): with k = floor(b_r / 16) for the request's
+ *     boundary token offset b_r, blocks j < k follow UNSALTED, block k is
+ *     H(sigma_p || h_{k-1} || T_k) (H(sigma_p || T_0) when k = 0), and
+ *     blocks j > k are chained as usual.  k >= n_b leaves the chain unsalted.
+ * H is SHA-256, T_j the 64 bytes of block j, || byte concatenation.
+ *
+ *   mode            KVGOV_UNSALTED, KVGOV_ROOT or KVGOV_BOUNDARY.
+ *   d_tokens        int32 tokens; must be 16-byte aligned (blocks are staged
+ *                   with aligned 16-byte copies; no byte outside
+ *                   [d_tokens, d_tokens + d_tok_off[n_req]) is read).
+ *   d_tok_off       [n_req + 1] int64 token offsets.
+ *   d_principal     [n_req] int32 row of d_salts per request; unused (may be
+ *                   NULL) for UNSALTED.
+ *   d_salts         [n_principals][32] u8 salts (kvgov_derive_salts); unused
+ *                   for UNSALTED.
+ *   d_boundary_tok  [n_req] int32 boundary token offset b_r >= 0; used (and
+ *                   required) only for BOUNDARY.
+ *   d_blk_off       [n_req + 1] int64 from kvgov_block_offsets.
+ *   d_digests       [d_blk_off[n_req]][32] u8 output, 16-byte aligned.
+ *   d_status        nullable; KVGOV_F_BADINDEX for a principal outside
+ *                   [0, n_principals), a negative b_r, or a malformed token
+ *                   offset (that request's digests are not written).
+ * n_req = 0 is a no-op.  EINVAL: bad mode, misaligned or NULL array.
+ */
+int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                     const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                     const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                     uint32_t *d_status, kvgov_stream_t stream);
+
+/*
+ * The prefix-cache index (paper section 2.1 and Table 1, row 1: a block
+ * prefix cache keyed by chained block hashes).  The caller owns a table of
+ * `capacity` 32-byte slots (capacity a power of two >= KVGOV_MIN_CAPACITY,
+ * d_slots 16-byte aligned).  A slot is empty when its first 8 bytes are zero;
+ * a key's home slot is its first 8 bytes read as a little-endian u64, modulo
+ * capacity, with linear probing.  Keys are stored verbatim, so keys whose
+ * first 8 bytes are all 0x00 or all 0xFF cannot be stored (KVGOV_F_SENTINEL);
+ * for SHA-256 digests that happens with probability 2^-63.
+ */
+
+/* kvgov_table_init -- mark every slot empty.  EINVAL: bad capacity/pointer. */
+int kvgov_table_init(uint8_t *d_slots, uint64_t capacity, kvgov_stream_t stream);
+
+/*
+ * kvgov_insert -- add d_keys[n_keys][32] (16-byte aligned) to the set.
+ * Duplicates, within the batch or with the table, are no-ops, so the
+ * resulting set does not depend on order.  Calls on the same table must not
+ * overlap in time with each other or with kvgov_probe (stream order them).
+ *   d_n_new   nullable; the number of keys newly stored is ADDED to it.
+ *   d_status  required; KVGOV_F_SENTINEL, KVGOV_F_TABLE_FULL and
+ *             KVGOV_F_TIMEOUT as above.  A wait for a concurrently claimed
+ *             slot is bounded (kvgov_set_spin_limit); on timeout the key is
+ *             not inserted.
+ * n_keys = 0 is a no-op.  EINVAL: bad capacity, NULL or misaligned pointer,
+ * n_keys < 0.
+ */
+int kvgov_insert(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_keys, int64_t n_keys,
+                 unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream);
+
+/*
+ * kvgov_probe -- block prefix-cache lookup, paper section 2.1 (a lookup
+ * matches the longest common prefix from position 0, truncated to a block
+ * boundary), Table 1 row 1 (the probe learns the first k matched blocks) and
+ * section 5.7 (a divergence at token i invalidates blocks floor(i/B) on):
+ *   d_prefix_blocks[r] = min { j : h_j(r) not in table }, or n_b(r) if every
+ *   block of request r is present.  Tokens served from cache = 16 * that.
+ *
+ *   d_digests       [d_blk_off[n_req]][32] u8 (kvgov_chain_hash output).
+ *   d_blk_off       [n_req + 1] int64.
+ *   d_prefix_blocks [n_req] int32 output.
+ *   d_status        nullable; KVGOV_F_BADINDEX for decreasing d_blk_off.
+ * n_req = 0 is a no-op.  EINVAL: bad capacity, NULL or misaligned pointer.
+ */
+int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,
+                const int64_t *d_blk_off, int32_t n_req, int32_t *d_prefix_blocks,
+                uint32_t *d_status, kvgov_stream_t stream);
+
+/*
+ * kvgov_set_spin_limit -- bound on how many times an inserting thread
+ * re-reads a slot that another thread has claimed but not yet published
+ * before it gives up with KVGOV_F_TIMEOUT (about 100 ns per re-read).
+ * Process-wide; applies to launches made after the call.  0 restores the
+ * default (2^23, about a second).  Returns the previous value.
+ */
+uint32_t kvgov_set_spin_limit(uint32_t limit);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVGOV_H */

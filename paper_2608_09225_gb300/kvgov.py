@@ -1,0 +1,211 @@
+"""ctypes binding of libkvgov (include/kvgov.h).
+
+Argument marshalling only: every function checks tensor devices, dtypes and
+contiguity, passes raw device pointers and the current torch CUDA stream to the
+C entry point of the same name, and raises KVGovError on a non-zero return.
+All work runs in the library's CUDA kernels; there is no CPU path.  If the
+library is missing or CUDA is unavailable the first call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+UNSALTED, ROOT, BOUNDARY = 0, 1, 2
+BLOCK = 16
+DIGEST_BYTES = 32
+MAX_SECRET = 1024
+MIN_CAPACITY = 32
+
+OK, EINVAL, ECUDA = 0, 1, 2
+F_BADINDEX, F_SENTINEL, F_TABLE_FULL, F_TIMEOUT = 0x10, 0x20, 0x40, 0x80
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libkvgov.so")
+_lock = threading.Lock()
+_lib = None
+
+_p = ctypes.c_void_p
+
+
+class KVGovError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status) if _lib is not None else status}")
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not torch.cuda.is_available():
+            raise RuntimeError("libkvgov needs a CUDA device; none is available (no CPU fallback)")
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"libkvgov.so is not built ({LIB_PATH}); run __graft_entry__.build()")
+        L = ctypes.CDLL(LIB_PATH)
+        L.kvgov_status_string.argtypes = [ctypes.c_int]
+        L.kvgov_status_string.restype = ctypes.c_char_p
+        L.kvgov_block_offsets.argtypes = [_p, ctypes.c_int32, _p, _p, _p]
+        L.kvgov_derive_salts.argtypes = [_p, ctypes.c_size_t, _p, _p, ctypes.c_int32, _p, _p, _p]
+        L.kvgov_chain_hash.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p, _p,
+                                       _p, _p]
+        L.kvgov_table_init.argtypes = [_p, ctypes.c_uint64, _p]
+        L.kvgov_insert.argtypes = [_p, ctypes.c_uint64, _p, ctypes.c_int64, _p, _p, _p]
+        L.kvgov_probe.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p]
+        L.kvgov_set_spin_limit.argtypes = [ctypes.c_uint32]
+        L.kvgov_set_spin_limit.restype = ctypes.c_uint32
+        for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
+                   "kvgov_insert", "kvgov_probe"):
+            getattr(L, fn).restype = ctypes.c_int
+        _lib = L
+        return L
+
+
+def lib():
+    return _lib if _lib is not None else _load()
+
+
+def status_string(status: int) -> str:
+    return lib().kvgov_status_string(int(status)).decode()
+
+
+def _check(rc: int, where: str):
+    if rc != OK:
+        raise KVGovError(rc, where)
+
+
+def _dev(t: torch.Tensor | None, dtype, name: str, allow_none: bool = False):
+    if t is None:
+        if allow_none:
+            return None
+        raise ValueError(f"{name} is required")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr() if t.numel() else None
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def block_offsets(tok_off: torch.Tensor, blk_off: torch.Tensor | None = None,
+                  status: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """blk_off[r+1] - blk_off[r] = floor(len_r / 16) (paper section 2.1)."""
+    L = lib()
+    n = tok_off.numel() - 1
+    if blk_off is None:
+        blk_off = torch.empty(n + 1, dtype=torch.int64, device=tok_off.device)
+    _check(L.kvgov_block_offsets(_dev(tok_off, torch.int64, "tok_off"), n,
+                                 _dev(blk_off, torch.int64, "blk_off"),
+                                 _dev(status, torch.int32, "status", True), _stream(stream)),
+           "kvgov_block_offsets")
+    return blk_off
+
+
+def derive_salts(secret: bytes, ids: torch.Tensor, id_off: torch.Tensor, salts: torch.Tensor | None = None,
+                 status: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """sigma_p = HMAC-SHA-256(secret, id_p) for every principal (paper section 4.1)."""
+    L = lib()
+    n = id_off.numel() - 1
+    if salts is None:
+        salts = torch.empty((n, 32), dtype=torch.uint8, device=id_off.device)
+    if ids.numel() == 0:   # every id is empty: hand the kernel a valid (unread) buffer
+        ids = torch.zeros(1, dtype=torch.uint8, device=id_off.device)
+    sec = bytes(secret)
+    buf = ctypes.create_string_buffer(sec, len(sec)) if sec else None
+    _check(L.kvgov_derive_salts(ctypes.cast(buf, _p) if buf is not None else None, len(sec),
+                                _dev(ids, torch.uint8, "ids"), _dev(id_off, torch.int64, "id_off"), n,
+                                _dev(salts, torch.uint8, "salts"),
+                                _dev(status, torch.int32, "status", True), _stream(stream)),
+           "kvgov_derive_salts")
+    return salts
+
+
+def chain_hash(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, blk_off: torch.Tensor,
+               principal: torch.Tensor | None = None, salts: torch.Tensor | None = None,
+               boundary_tok: torch.Tensor | None = None, digests: torch.Tensor | None = None,
+               n_blocks: int | None = None, status: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Chained block digests, request-major [sum n_b, 32] (paper sections 2.1, 4.1, 4.2).
+
+    digests (or n_blocks = blk_off[-1]) sizes the output; with neither, the
+    total is read back from the device, which synchronises.
+    """
+    L = lib()
+    n = tok_off.numel() - 1
+    if digests is None:
+        if n_blocks is None:
+            n_blocks = int(blk_off[-1].item())
+        digests = torch.empty((n_blocks, 32), dtype=torch.uint8, device=tokens.device)
+    if tokens.numel() == 0:
+        tokens = torch.zeros(4, dtype=torch.int32, device=tok_off.device)
+    n_p = 0 if salts is None else salts.shape[0]
+    _check(L.kvgov_chain_hash(int(mode), _dev(tokens, torch.int32, "tokens"), _dev(tok_off, torch.int64, "tok_off"),
+                              n, _dev(principal, torch.int32, "principal", True),
+                              _dev(salts, torch.uint8, "salts", True), n_p,
+                              _dev(boundary_tok, torch.int32, "boundary_tok", True),
+                              _dev(blk_off, torch.int64, "blk_off"),
+                              _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(tokens),
+                              _dev(status, torch.int32, "status", True), _stream(stream)),
+           "kvgov_chain_hash")
+    return digests
+
+
+def _dummy(like: torch.Tensor):
+    global _dummy_buf
+    if _dummy_buf is None or _dummy_buf.device != like.device:
+        _dummy_buf = torch.zeros(64, dtype=torch.uint8, device=like.device)
+    return _dummy_buf.data_ptr()
+
+
+_dummy_buf = None
+
+
+def table_init(slots: torch.Tensor, stream=None) -> torch.Tensor:
+    """Mark every slot of a [capacity, 32] u8 table empty."""
+    _check(lib().kvgov_table_init(_dev(slots, torch.uint8, "slots"), slots.shape[0], _stream(stream)),
+           "kvgov_table_init")
+    return slots
+
+
+def new_table(capacity: int, device="cuda", stream=None) -> torch.Tensor:
+    slots = torch.empty((capacity, 32), dtype=torch.uint8, device=device)
+    return table_init(slots, stream)
+
+
+def insert(slots: torch.Tensor, keys: torch.Tensor, status: torch.Tensor, n_new: torch.Tensor | None = None,
+           stream=None):
+    """Set-insert [n, 32] u8 keys; adds the number stored to n_new (int64[1])."""
+    _check(lib().kvgov_insert(_dev(slots, torch.uint8, "slots"), slots.shape[0],
+                              _dev(keys, torch.uint8, "keys"), keys.shape[0] if keys.dim() == 2 else 0,
+                              _dev(n_new, torch.int64, "n_new", True), _dev(status, torch.int32, "status"),
+                              _stream(stream)),
+           "kvgov_insert")
+
+
+def probe(slots: torch.Tensor, digests: torch.Tensor, blk_off: torch.Tensor,
+          prefix_blocks: torch.Tensor | None = None, status: torch.Tensor | None = None,
+          stream=None) -> torch.Tensor:
+    """prefix_blocks[r] = first j with h_j(r) not cached, or n_b(r) (paper section 2.1, Table 1)."""
+    n = blk_off.numel() - 1
+    if prefix_blocks is None:
+        prefix_blocks = torch.empty(n, dtype=torch.int32, device=blk_off.device)
+    _check(lib().kvgov_probe(_dev(slots, torch.uint8, "slots"), slots.shape[0],
+                             _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(blk_off),
+                             _dev(blk_off, torch.int64, "blk_off"), n,
+                             _dev(prefix_blocks, torch.int32, "prefix_blocks"),
+                             _dev(status, torch.int32, "status", True), _stream(stream)),
+           "kvgov_probe")
+    return prefix_blocks
+
+
+def set_spin_limit(limit: int) -> int:
+    return int(lib().kvgov_set_spin_limit(int(limit)))

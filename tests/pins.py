@@ -1,0 +1,377 @@
+"""Pins for the CPU oracle: checks against things other than the oracle itself.
+
+Every check here compares the oracle with an independent implementation of a
+special case (Python's hashlib / hmac, i.e. OpenSSL), with an invariant the
+paper states, with a number the paper prints for a worked example
+(tests/golden/paper_examples.json), with a closed form of a synthetic
+workload, or with brute force on tiny inputs.  They are plain functions so
+that tests/test_oracle_pins.py can also run them against copies of the oracle
+with a planted mistake and show that some pin fails.
+"""
+from __future__ import annotations
+
+import hashlib
+import hmac
+import json
+import os
+import struct
+
+import numpy as np
+
+import oracle
+from paper_2608_09225_gb300 import workloads as W
+
+UNSALTED, ROOT, BOUNDARY = oracle.UNSALTED, oracle.ROOT, oracle.BOUNDARY
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def H(b: bytes) -> bytes:
+    return hashlib.sha256(b).digest()
+
+
+def block_le(tokens) -> bytes:
+    """Little-endian int32 serialisation, written with struct (not numpy)."""
+    return struct.pack("<%di" % len(tokens), *[int(t) for t in tokens])
+
+
+def _batch(lengths, seed=3):
+    return W.ragged(seed, lengths)
+
+
+def _rows(blk_off, r):
+    return range(int(blk_off[r]), int(blk_off[r + 1]))
+
+
+# --------------------------------------------------------------- SHA-256 / HMAC
+def pin_sha256_every_length():
+    """FIPS 180-4 SHA-256 == hashlib on every length 0..300 (all padding edges)."""
+    rng = np.random.default_rng(11)
+    for n in range(301):
+        m = rng.integers(0, 256, n, dtype=np.uint8).tobytes()
+        assert oracle.sha256(m) == H(m), f"length {n}"
+
+
+def pin_sha256_long_and_classic():
+    """Multi-block messages: short ASCII, a two-block 56-byte message, 1 MB."""
+    for m in (b"abc", b"abcdbcdecdefdefgefghfghighijhijkijkljklmklmnlmnomnopnopq",
+              b"a" * 1_000_000, bytes(range(256)) * 17):
+        assert oracle.sha256(m) == H(m)
+
+
+def pin_hmac():
+    """RFC 2104 HMAC-SHA-256 == Python hmac for keys shorter than, equal to and
+    longer than the 64-byte block, and messages across the padding edges."""
+    rng = np.random.default_rng(12)
+    for kl in (0, 1, 20, 32, 63, 64, 65, 131, 1024):
+        key = rng.integers(0, 256, kl, dtype=np.uint8).tobytes()
+        for ml in (0, 4, 50, 55, 56, 64, 119, 152, 1000):
+            msg = rng.integers(0, 256, ml, dtype=np.uint8).tobytes()
+            assert oracle.hmac_sha256(key, msg) == hmac.new(key, msg, "sha256").digest(), (kl, ml)
+
+
+def pin_salts():
+    """sigma_p = HMAC_K(secret, principal_id) (section 4.1) == Python hmac,
+    for 4-byte ids and for variable-length ids including the empty one."""
+    secret = bytes(range(32))
+    ids, id_off = W.principal_ids(64)
+    s = oracle.derive_salts(secret, ids, id_off)
+    for p in range(64):
+        assert s[p].tobytes() == hmac.new(secret, struct.pack("<I", p), "sha256").digest()
+    rng = np.random.default_rng(13)
+    lens = [0, 1, 55, 56, 64, 100, 200]
+    raw = [rng.integers(0, 256, L, dtype=np.uint8).tobytes() for L in lens]
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    buf = np.frombuffer(b"".join(raw), np.uint8)
+    long_key = bytes(rng.integers(0, 256, 100, dtype=np.uint8))
+    s = oracle.derive_salts(long_key, buf, off)
+    for i, m in enumerate(raw):
+        assert s[i].tobytes() == hmac.new(long_key, m, "sha256").digest()
+
+
+# ----------------------------------------------------------------- the chain
+def pin_token_serialisation():
+    """A token's hashed bytes are its int32 little-endian bytes; a block of
+    16 tokens hashes as H(T_0) (section 2.1, j = 0)."""
+    toks = np.array([0x04030201, -1, -(2 ** 31), 2 ** 31 - 1, 0, 1, 256, 65536,
+                     152063, 7, 0x7F00FF00, -2, 3, 4, 5, 6], dtype=np.int32)
+    d = oracle.chain_hash(UNSALTED, toks, np.array([0, 16]))
+    assert d[0].tobytes() == H(block_le(toks))
+    assert block_le(toks[:1]) == b"\x01\x02\x03\x04"
+
+
+def pin_chain_unsalted():
+    """Section 2.1: h_0 = H(T_0), h_j = H(h_{j-1} || T_j); partial tails unhashed."""
+    b = _batch([16, 33, 48, 0, 15, 16 * 9 + 5])
+    d = oracle.chain_hash(UNSALTED, b.tokens, b.tok_off)
+    blk = oracle.block_offsets(b.tok_off)
+    assert list(np.diff(blk)) == [1, 2, 3, 0, 0, 9]
+    for r in range(b.n):
+        t = b.tokens[b.tok_off[r]:b.tok_off[r + 1]]
+        prev = None
+        for j, row in enumerate(_rows(blk, r)):
+            T = block_le(t[16 * j:16 * j + 16])
+            want = H(T) if j == 0 else H(prev + T)
+            assert d[row].tobytes() == want, (r, j)
+            prev = want
+
+
+def pin_chain_root():
+    """Section 4.1: h_0 = H(sigma_p || T_0); later blocks chained as before."""
+    b = _batch([16, 40, 64, 16 * 7])
+    salts = np.random.default_rng(5).integers(0, 256, (8, 32), dtype=np.uint8)
+    d = oracle.chain_hash(ROOT, b.tokens, b.tok_off, b.principal, salts)
+    blk = oracle.block_offsets(b.tok_off)
+    for r in range(b.n):
+        t = b.tokens[b.tok_off[r]:b.tok_off[r + 1]]
+        sig = salts[b.principal[r]].tobytes()
+        prev = None
+        for j, row in enumerate(_rows(blk, r)):
+            T = block_le(t[16 * j:16 * j + 16])
+            want = H(sig + T) if j == 0 else H(prev + T)
+            assert d[row].tobytes() == want, (r, j)
+            prev = want
+
+
+def pin_chain_boundary():
+    """Section 4.2: blocks j < k unsalted; h_k = H(sigma_p || h_{k-1} || T_k)
+    (H(sigma_p || T_0) at k = 0); j > k chained; k = floor(b / 16)."""
+    bounds = [0, 1, 15, 16, 17, 31, 32, 47, 48, 63, 64, 100, 10 ** 6]
+    n = len(bounds)
+    rng = np.random.default_rng(6)
+    toks = rng.integers(0, W.VOCAB, (n, 16 * 6), dtype=np.int32)
+    tok_off = np.arange(n + 1, dtype=np.int64) * 96
+    principal = np.arange(n, dtype=np.int32) % 4
+    salts = rng.integers(0, 256, (4, 32), dtype=np.uint8)
+    bt = np.array(bounds, dtype=np.int32)
+    d = oracle.chain_hash(BOUNDARY, toks.reshape(-1), tok_off, principal, salts, bt)
+    for r in range(n):
+        k = bounds[r] // 16
+        sig = salts[principal[r]].tobytes()
+        prev = None
+        for j in range(6):
+            T = block_le(toks[r, 16 * j:16 * j + 16])
+            if j == k:
+                want = H(sig + T) if j == 0 else H(sig + prev + T)
+            else:
+                want = H(T) if j == 0 else H(prev + T)
+            assert d[6 * r + j].tobytes() == want, (r, j)
+            prev = want
+
+
+def pin_boundary_invariants():
+    """Section 4.2: for j < k the digests are principal-independent and equal
+    to the unsalted chain (shared, routable); for j >= k they differ across
+    principals and from the unsalted chain; BOUNDARY with b < 16 is ROOT."""
+    rng = np.random.default_rng(8)
+    toks = rng.integers(0, W.VOCAB, 16 * 8, dtype=np.int32)
+    n_p = 6
+    tokens = np.tile(toks, n_p)
+    tok_off = np.arange(n_p + 1, dtype=np.int64) * 128
+    principal = np.arange(n_p, dtype=np.int32)
+    salts = oracle.derive_salts(b"k" * 32, *W.principal_ids(n_p))
+    un = oracle.chain_hash(UNSALTED, toks, np.array([0, 128]))
+    for b in (16 * 3, 16 * 3 + 9):
+        d = oracle.chain_hash(BOUNDARY, tokens, tok_off, principal, salts, np.full(n_p, b, np.int32))
+        d = d.reshape(n_p, 8, 32)
+        for j in range(3):
+            for p in range(n_p):
+                assert (d[p, j] == un[j]).all()
+        for j in range(3, 8):
+            rows = {d[p, j].tobytes() for p in range(n_p)}
+            assert len(rows) == n_p and un[j].tobytes() not in rows
+    root = oracle.chain_hash(ROOT, tokens, tok_off, principal, salts)
+    for b in (0, 7, 15):
+        d = oracle.chain_hash(BOUNDARY, tokens, tok_off, principal, salts, np.full(n_p, b, np.int32))
+        assert (d == root).all()
+
+
+def pin_disjoint_and_deterministic():
+    """Section 4.1: over identical tokens, ROOT chains of different principals
+    share no digest at any position; the same (principal, tokens) gives the
+    same chain at any batch position."""
+    rng = np.random.default_rng(9)
+    n_p, per = 8, 8
+    base = rng.integers(0, W.VOCAB, (per, 64), dtype=np.int32)
+    tokens = np.tile(base.reshape(-1), n_p)
+    tok_off = np.arange(n_p * per + 1, dtype=np.int64) * 64
+    principal = np.repeat(np.arange(n_p, dtype=np.int32), per)
+    salts = oracle.derive_salts(b"s" * 32, *W.principal_ids(n_p))
+    d = oracle.chain_hash(ROOT, tokens, tok_off, principal, salts).reshape(n_p, per, 4, 32)
+    seen = {}
+    for p in range(n_p):
+        for q in range(per):
+            for j in range(4):
+                key = d[p, q, j].tobytes()
+                assert seen.setdefault(key, (p, q, j)) == (p, q, j)
+    # same chain at another batch position (request reordered)
+    perm = np.random.default_rng(10).permutation(n_p * per)
+    t2 = tokens.reshape(-1, 64)[perm].reshape(-1)
+    d2 = oracle.chain_hash(ROOT, t2, tok_off, principal[perm], salts).reshape(-1, 4, 32)
+    assert (d2 == d.reshape(-1, 4, 32)[perm]).all()
+
+
+# ------------------------------------------------------------------- lookup
+def _prefix(mode, fill_tokens, fill_principal, probe_tokens, probe_principal, salts=None, b=0, L=None):
+    """Fill a set with one request's chain, probe another; returns hit blocks."""
+    L = L or len(fill_tokens)
+    ks = oracle.KeySet(1)
+    d = oracle.chain_hash(mode, fill_tokens, np.array([0, L]), np.array([fill_principal]), salts,
+                          np.array([b], np.int32))
+    ks.insert(d)
+    q = oracle.chain_hash(mode, probe_tokens, np.array([0, L]), np.array([probe_principal]), salts,
+                          np.array([b], np.int32))
+    return int(ks.prefix_blocks(q, oracle.block_offsets(np.array([0, L])))[0])
+
+
+def _paper():
+    with open(os.path.join(GOLDEN, "paper_examples.json")) as f:
+        return json.load(f)
+
+
+def pin_paper_divergence_layout():
+    """Section 5.7: a 2119-token shared preamble diverging at token 1990 keeps
+    124 block hits; diverging at token 5 keeps none."""
+    ex = _paper()["divergence_layout"]
+    n = ex["prompt_tokens"]
+    rng = np.random.default_rng(14)
+    a = rng.integers(0, W.VOCAB, n, dtype=np.int32)
+    for i, want in zip(ex["diverge_at_token"], ex["hit_blocks"]):
+        bq = a.copy()
+        bq[i] = (bq[i] + 1) % W.VOCAB
+        assert _prefix(UNSALTED, a, 0, bq, 0) == want
+
+
+def pin_paper_boundary_efficiency():
+    """Section 4.2: with the salt at the end of a 2000-token shared preamble of
+    a 2119-token prompt, another principal reuses the preamble's full blocks
+    and prefills 8 blocks (7 full + the partial tail) instead of 133."""
+    ex = _paper()["boundary_salting_efficiency"]
+    n, pre = ex["prompt_tokens"], ex["shared_preamble_tokens"]
+    total_blocks = -(-n // 16)
+    rng = np.random.default_rng(15)
+    a = rng.integers(0, W.VOCAB, n, dtype=np.int32)
+    salts = oracle.derive_salts(b"x" * 32, *W.principal_ids(2))
+    hits_b = _prefix(BOUNDARY, a, 0, a, 1, salts, b=pre)
+    hits_r = _prefix(ROOT, a, 0, a, 1, salts)
+    assert total_blocks - hits_b == ex["blocks_to_prefill_boundary"]
+    assert total_blocks - hits_r == ex["blocks_to_prefill_root"]
+    assert _prefix(BOUNDARY, a, 1, a, 1, salts, b=pre) == n // 16   # same principal: all full blocks
+
+
+def pin_cross_principal_all_miss():
+    """Section 4.1: a prober on another principal sees all-MISS on the victim's
+    cached prompt; the same principal hits every full block."""
+    rng = np.random.default_rng(16)
+    salts = oracle.derive_salts(b"y" * 32, *W.principal_ids(4))
+    for L in (16, 100, 512):
+        a = rng.integers(0, W.VOCAB, L, dtype=np.int32)
+        assert _prefix(ROOT, a, 2, a, 3, salts) == 0
+        assert _prefix(ROOT, a, 2, a, 2, salts) == L // 16
+        assert _prefix(UNSALTED, a, 2, a, 3) == L // 16
+
+
+def pin_prefix_brute_force():
+    """Lookup == a Python-set brute force: first missing block, later hits
+    ignored (section 2.1 longest common prefix from position 0)."""
+    rng = np.random.default_rng(17)
+    for trial in range(20):
+        nb = rng.integers(0, 12, 30)
+        off = np.concatenate([[0], np.cumsum(nb)]).astype(np.int64)
+        pool = rng.integers(0, 256, (8, 32), dtype=np.uint8)
+        pool[:, 0] |= 1                                   # no reserved keys
+        digests = pool[rng.integers(0, 8, int(off[-1]))]
+        member = rng.random(8) < 0.6
+        ks = oracle.KeySet(1)
+        ks.insert(pool[member])
+        S = {pool[i].tobytes() for i in range(8) if member[i]}
+        got = ks.prefix_blocks(digests, off)
+        for r in range(30):
+            L = 0
+            while L < nb[r] and digests[off[r] + L].tobytes() in S:
+                L += 1
+            assert got[r] == L
+
+
+def pin_set_semantics():
+    """Set insert: duplicates are no-ops in any order; reserved first words
+    (all 0x00 / all 0xFF) are refused and flagged."""
+    rng = np.random.default_rng(18)
+    keys = rng.integers(0, 256, (50, 32), dtype=np.uint8)
+    keys[:, 0] |= 1
+    batch = np.concatenate([keys, keys[::-1], keys[:10]])
+    ks = oracle.KeySet(1)
+    n_new, flag = ks.insert(batch)
+    assert n_new == 50 and not flag
+    n_new, flag = ks.insert(keys[:20])
+    assert n_new == 0 and not flag
+    bad = np.zeros((3, 32), np.uint8)
+    bad[1, :8] = 255
+    bad[2, 8:] = 7            # first 8 bytes zero, rest not
+    n_new, flag = ks.insert(bad)
+    assert n_new == 0 and flag and ks.n == 50
+    ks2 = oracle.KeySet(1)
+    ks2.insert(batch[rng.permutation(len(batch))])
+    assert (ks2.contents() == ks.contents()).all()
+
+
+# ------------------------------------------------------ workload closed forms
+def run_workload_oracle(w, mode):
+    """Salts, chains, table fill and probe of a workload, all with the oracle."""
+    salts = oracle.derive_salts(w.secret, w.ids, w.id_off)
+    b = w.batch
+    d = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+    blk = oracle.block_offsets(b.tok_off)
+    ks = oracle.KeySet(1)
+    if w.fill_from == "prior":
+        p = w.prior
+        dp = oracle.chain_hash(mode, p.tokens, p.tok_off, p.principal, salts, p.boundary_tok)
+        ks.insert(dp)
+    else:
+        f0, f1 = w.fill
+        ks.insert(d[blk[f0]:blk[f1]])
+    if w.random_keys is not None:
+        ks.insert(w.random_keys)
+    p0, p1 = w.probe
+    L = ks.prefix_blocks(d, blk[p0:p1 + 1])
+    return salts, d, blk, ks, L
+
+
+def pin_tiny_closed_form():
+    """Tiny workload: the table holds requests 0-15; requests 16-31 share the
+    128-token template (8 blocks) with request r-16 of the same principal;
+    requests 32-63 share nothing."""
+    w = W.make("tiny")
+    _, _, _, _, L = run_workload_oracle(w, ROOT)
+    assert list(L) == [16] * 16 + [8] * 16 + [0] * 32
+
+
+def pin_sysprompt_closed_form():
+    """Shared system prompt (reduced): filled requests hit all 132 blocks;
+    others hit the 64 system-prefix blocks iff their principal filled."""
+    w = W.sysprompt(n_req=96, fill_n=24)
+    _, _, _, _, L = run_workload_oracle(w, ROOT)
+    filled = set(w.batch.principal[:24].tolist())
+    want = [132] * 24 + [64 if int(p) in filled else 0 for p in w.batch.principal[24:]]
+    assert list(L) == want
+
+
+def pin_probe_closed_form():
+    """Probe-heavy (reduced): a request reusing c blocks of a prior request
+    (with that request's principal) hits exactly c; a fresh one hits 0."""
+    w = W.probe(n_req=512, n_prior=64, capacity=1 << 12, n_random=1000)
+    _, _, _, _, L = run_workload_oracle(w, ROOT)
+    assert (L == w.info["cut"]).all()
+
+
+def pin_template_ordering():
+    """Template workload (reduced): per request, hits under UNSALTED >=
+    BOUNDARY >= ROOT; BOUNDARY (k = 6) keeps the 6 template blocks before the
+    first field for every request."""
+    w = W.template(n_req=1024)
+    Ls = {m: run_workload_oracle(w, m)[4] for m in (UNSALTED, ROOT, BOUNDARY)}
+    assert (Ls[UNSALTED] >= Ls[BOUNDARY]).all() and (Ls[BOUNDARY] >= Ls[ROOT]).all()
+    assert (Ls[BOUNDARY] >= 6).all() and (Ls[UNSALTED] >= 6).all()
+    assert Ls[UNSALTED].mean() > Ls[BOUNDARY].mean()
+
+
+PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]
