@@ -1,0 +1,447 @@
+#!/usr/bin/env python3
+"""Benchmark: KVGov salted block-hash chain + prefix-cache probe on GB300.
+
+One step = one serving batch through the whole hot path, every step a
+libkvgov kernel: per-principal salts (HMAC-SHA-256, 4096 principals) ->
+blocking (block offsets) -> BOUNDARY-salted chain hash (salt at token 64,
+block 4) -> probe of the resident prefix-cache table -> insert of the batch's
+digests.  Workload: 131,072 requests x 128 tokens (8 blocks each; the
+largest batch), a 64-token prefix shared by all requests, 4096 principals.
+
+Timed region: `--steps` steps after `--warmup` untimed ones, bracketed by a
+barrier and cuda synchronize, CUDA events on the launching stream, max over
+ranks.  A pool of distinct batches (inputs already resident in HBM) is cycled,
+and the table is pre-filled with every pool batch's chains before timing, so
+every step re-serves a cached batch: each probe walks all 8 blocks (all hit)
+and each insert finds its 8 keys present.
+
+Prints ONE JSON line (rank 0).  `--impl reference` times the CPU oracle
+(plain C, the bounded sample described in its line) as the reference arm.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, HERE)
+
+METRIC = "salted block digests/s and tokens hashed/s on 1 GB300; % of INT32 issue peak"
+UNIT = "block digests/s"
+WORKLOAD = {"workload": "wide: 131072 requests x 128 tokens, BOUNDARY salt at token 64, 4096 principals",
+            "requests": 131072, "tokens_per_request": 128, "block": 16, "blocks_per_step": 131072 * 8,
+            "principals": 4096, "mode": "BOUNDARY (k=4)"}
+N_SM_NOMINAL = 152
+SM_MAX_MHZ = 2070.0
+
+
+# --------------------------------------------------------------------------- helpers
+def nominal_chain_ops(nb: np.ndarray, mode: int, k: np.ndarray | None) -> int:
+    """Nominal integer ops of the chain kernel: 1384 per scheduled compression,
+    904 per compression whose schedule is a compile-time constant (padding
+    block).  Per block: 64-byte message 1384 + 904; 96-byte 2 x 1384;
+    128-byte (boundary block, k >= 1) 2 x 1384 + 904."""
+    nb = np.asarray(nb, dtype=np.int64)
+    m64, m96, m128 = 1384 + 904, 2 * 1384, 2 * 1384 + 904
+    if mode == 0:
+        return int(np.where(nb > 0, m64 + (nb - 1) * m96, 0).sum())
+    if mode == 1:
+        return int((nb * m96).sum())
+    k = np.asarray(k, dtype=np.int64)
+    salted = k < nb
+    tot = np.zeros_like(nb)
+    # k = 0: ROOT chain; k >= 1 inside: 64 + (nb-2) x 96 + one 128; k >= nb: UNSALTED
+    tot = np.where(salted & (k == 0), nb * m96, tot)
+    tot = np.where(salted & (k > 0), m64 + (nb - 2) * m96 + m128, tot)
+    tot = np.where(~salted & (nb > 0), m64 + (nb - 1) * m96, tot)
+    return int(tot.sum())
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.t.join(timeout=2)
+
+    def summary(self):
+        sm, mx, pw, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+                pw.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "power_w_max": max(pw),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def measure_int_peak(torch, peak_lib_path):
+    """Thread-ops per SM clock for SHA-256's op mix, from libkvgov_peak."""
+    import ctypes
+    L = ctypes.CDLL(peak_lib_path)
+    L.kvgov_peak_int.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                 ctypes.c_void_p, ctypes.c_void_p]
+    L.kvgov_peak_ops_per_iter.argtypes = [ctypes.c_int]
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    out = {}
+    for kind, name, threads, blocks_per_sm, iters in ((0, "lop3", 256, 8, 4000), (1, "shf", 256, 8, 4000),
+                                                      (2, "iadd3", 256, 8, 4000), (3, "sha256", 256, 4, 200)):
+        blocks = n_sm * blocks_per_sm
+        sink = torch.zeros(1, dtype=torch.int32, device="cuda")
+        clocks = torch.zeros(blocks * 3, dtype=torch.int64, device="cuda")
+        for _ in range(2):
+            rc = L.kvgov_peak_int(kind, iters, blocks, threads, sink.data_ptr(), clocks.data_ptr(),
+                                  torch.cuda.current_stream().cuda_stream)
+            assert rc == 0, rc
+        torch.cuda.synchronize()
+        c = clocks.view(blocks, 3).cpu().numpy()
+        per_sm = {}
+        for sm, t0, t1 in c:
+            lo, hi, cnt = per_sm.get(int(sm), (t0, t1, 0))
+            per_sm[int(sm)] = (min(lo, t0), max(hi, t1), cnt + 1)
+        ops_iter = L.kvgov_peak_ops_per_iter(kind)
+        rates = [cnt * threads * iters * ops_iter / max(hi - lo, 1) for lo, hi, cnt in per_sm.values()]
+        out[name] = float(np.median(rates))
+    out["n_sm"] = n_sm
+    return out
+
+
+# --------------------------------------------------------------------------- reference arm
+def cpu_oracle_step(w, sample_req, n_threads, keyset):
+    """The oracle on a sample: salts, chain (threaded over request chunks),
+    probe and insert.  Returns blocks hashed."""
+    import concurrent.futures as cf
+
+    import oracle
+    b = w.batch
+    salts = oracle.derive_salts(w.secret, w.ids, w.id_off)
+    n = sample_req
+    chunks = np.array_split(np.arange(n), n_threads)
+
+    def run(ix):
+        if len(ix) == 0:
+            return np.zeros((0, 32), np.uint8)
+        lo, hi = int(ix[0]), int(ix[-1]) + 1
+        off = b.tok_off[lo:hi + 1] - b.tok_off[lo]
+        toks = b.tokens[b.tok_off[lo]:b.tok_off[hi]]
+        return oracle.chain_hash(oracle.BOUNDARY, toks, off, b.principal[lo:hi], salts, b.boundary_tok[lo:hi])
+
+    with cf.ThreadPoolExecutor(n_threads) as ex:
+        parts = list(ex.map(run, chunks))
+    d = np.concatenate(parts)
+    blk = oracle.block_offsets(b.tok_off[:n + 1])
+    keyset.prefix_blocks(d, blk)
+    keyset.insert(d)
+    return int(blk[-1])
+
+
+def reference_arm(args):
+    import oracle
+    from paper_2608_09225_gb300 import workloads as W
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    oracle.build()
+    cores = len(os.sched_getaffinity(0))
+    w = W.make("wide", seed=args.seed)
+    sample = args.cpu_sample
+    ks = oracle.KeySet(1)
+    cpu_oracle_step(w, sample, cores, ks)          # pre-fill: the sample is cached, as on the GPU
+    for _ in range(args.warmup):
+        cpu_oracle_step(w, sample, cores, ks)
+    t0 = time.perf_counter()
+    blocks = 0
+    for _ in range(args.steps):
+        blocks += cpu_oracle_step(w, sample, cores, ks)
+    dt = time.perf_counter() - t0
+    value = blocks / dt
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
+            "config": dict(WORKLOAD, sample_requests=sample),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"first {sample} requests of the batch per step: salts, chain, "
+                                       f"probe, insert (set already holding them)"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "tokens_per_s": 16 * value}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# --------------------------------------------------------------------------- GPU arm
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="kvgov", choices=["kvgov", "reference"])
+    ap.add_argument("--pool", type=int, default=16, help="distinct resident batches cycled by the steps")
+    ap.add_argument("--e2e-steps", type=int, default=100)
+    ap.add_argument("--seed", type=int, default=None, help="base seed (default: fresh per run)")
+    ap.add_argument("--cpu-sample", type=int, default=16384, help="requests per oracle step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.seed is None:
+        args.seed = int.from_bytes(os.urandom(4), "little")
+    args.warmup = max(args.warmup, 3)
+    if args.impl == "reference":
+        return reference_arm(args)
+
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_09225_gb300 import build as kbuild
+    from paper_2608_09225_gb300 import kvgov as K
+    from paper_2608_09225_gb300 import workloads as W
+    from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache, next_pow2
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    kbuild.build()
+    K.lib()
+
+    # ---- inputs: a pool of distinct batches, resident in HBM (weak scaling: per-rank seeds)
+    base = args.seed + 1000003 * rank
+    pool_host = [W.make("wide", seed=base + i) for i in range(args.pool)]
+    w0 = pool_host[0]
+    n_req = w0.batch.n
+    n_blocks = int((w0.batch.lengths() // 16).sum())
+    pool = [DeviceBatch.from_host(w.batch.tokens, w.batch.tok_off, w.batch.principal, w.batch.boundary_tok)
+            for w in pool_host]
+    cache = PrefixCache(next_pow2(4 * args.pool * n_blocks // 2), w0.secret, w0.ids, w0.id_off)
+    bufs = {"blk_off": torch.empty(n_req + 1, dtype=torch.int64, device="cuda"),
+            "digests": torch.empty((n_blocks, 32), dtype=torch.uint8, device="cuda"),
+            "prefix": torch.empty(n_req, dtype=torch.int32, device="cuda")}
+    for db in pool:                                          # pre-fill: every pool batch is cached
+        cache.serve(W.BOUNDARY, db, bufs)
+    torch.cuda.synchronize()
+    cache.check_status()
+
+    # ---- parity gate on a sample (oracle) before timing
+    gate = parity_gate(cache, pool_host[0], pool[0], bufs)
+
+    stream = torch.cuda.current_stream()
+
+    def step(db, ev=None):
+        K.derive_salts(cache.secret, cache.ids, cache.id_off, cache.salts, cache.status)
+        K.block_offsets(db.tok_off, bufs["blk_off"], cache.status)
+        if ev is not None:
+            ev[0].record(stream)
+        K.chain_hash(W.BOUNDARY, db.tokens, db.tok_off, bufs["blk_off"], db.principal, cache.salts,
+                     db.boundary_tok, bufs["digests"], status=cache.status)
+        if ev is not None:
+            ev[1].record(stream)
+        K.probe(cache.slots, bufs["digests"], bufs["blk_off"], bufs["prefix"], cache.status)
+        K.insert(cache.slots, bufs["digests"], cache.status, cache.n_new)
+
+    kernels_per_step = 1 + (1 if n_req <= 4096 else 3) + 1 + 1 + 1
+    for i in range(args.warmup):
+        step(pool[i % args.pool])
+    torch.cuda.synchronize()
+
+    chain_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                for _ in range(args.steps)]
+    t_start, t_stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        t_start.record(stream)
+        for i in range(args.steps):
+            step(pool[i % args.pool], chain_ev[i])
+        t_stop.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+    cache.check_status()
+    ms = t_start.elapsed_time(t_stop)
+    chain_ms = float(np.mean([a.elapsed_time(b) for a, b in chain_ev]))
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * args.steps * n_blocks / (ms / 1e3)
+
+    # ---- end to end through the public API with host buffers
+    e2e = e2e_leg(torch, K, W, cache, pool_host[: min(4, args.pool)], args.e2e_steps, bufs, world, dist)
+
+    # ---- roofline of the chain kernel (integer issue bound)
+    peak = measure_int_peak(torch, kbuild.PEAK_LIB)
+    nb = (w0.batch.lengths() // 16)
+    ops = nominal_chain_ops(nb, 2, w0.batch.boundary_tok // 16)
+    achieved = ops / (chain_ms / 1e3) / 1e12
+    clock = clk.summary()
+    peak_ops_clk = peak["sha256"]
+    peak_tops = peak["n_sm"] * peak_ops_clk * SM_MAX_MHZ * 1e6 / 1e12
+    roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s (int32)",
+                "frac": achieved / peak_tops, "traffic": None,
+                "kernel": "chain_kernel<BOUNDARY>", "ops_per_launch": ops, "kernel_ms": chain_ms,
+                "peak_basis": f"{peak['n_sm']} SMs x {peak_ops_clk:.1f} SHA-256 thread-ops/clk/SM "
+                              f"(measured, libkvgov_peak) x {SM_MAX_MHZ:.0f} MHz",
+                "int_ops_per_clk_per_sm": {k: round(v, 2) for k, v in peak.items() if k != "n_sm"}}
+    if clock.get("sm_mhz"):
+        roofline["frac_at_run_clock"] = achieved / (peak["n_sm"] * peak_ops_clk * clock["sm_mhz"] * 1e6 / 1e12)
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "u32", "data": "synthetic",
+            "config": dict(WORKLOAD, pool_batches=args.pool, seed=args.seed,
+                           l2=f"{args.pool} distinct resident batches cycled (each re-read after "
+                              f"{args.pool - 1} others); table {cache.capacity * 32 >> 20} MiB",
+                           table_slots=cache.capacity),
+            "tokens_per_s": 16 * value, "chain_digests_per_s": world * n_blocks / (chain_ms / 1e3),
+            "e2e": e2e, "gpu_launches": kernels_per_step * args.steps, "clocks": clock, "roofline": roofline,
+            "parity_gate": gate}
+    if rank == 0 and not args.no_cpu_baseline and world == 1:
+        line["cpu_baseline"] = cpu_baseline(pool_host[0], args.cpu_sample)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def parity_gate(cache, w, db, bufs):
+    """Before timing: a sample of digests and every prefix length of one
+    batch against the oracle and the closed form (all 8 blocks cached)."""
+    import torch
+
+    import oracle
+    from paper_2608_09225_gb300 import workloads as W
+    prefix, digests, blk = cache.serve(W.BOUNDARY, db, bufs)
+    torch.cuda.synchronize()
+    b = w.batch
+    rng = np.random.default_rng(0)
+    rows = np.sort(rng.choice(b.n, size=256, replace=False))
+    salts = oracle.derive_salts(w.secret, w.ids, w.id_off)
+    got = digests.cpu().numpy().reshape(b.n, -1, 32)[rows]
+    for r, g in zip(rows, got):
+        lo, hi = b.tok_off[r], b.tok_off[r + 1]
+        ref = oracle.chain_hash(oracle.BOUNDARY, b.tokens[lo:hi], np.array([0, hi - lo]), b.principal[r:r + 1],
+                                salts, b.boundary_tok[r:r + 1])
+        if not (ref == g).all():
+            raise SystemExit(f"parity gate: request {r} digests differ from the oracle")
+    if not (cache.salts.cpu().numpy() == salts).all():
+        raise SystemExit("parity gate: salts differ from the oracle")
+    pre = prefix.cpu().numpy()
+    if not (pre == 8).all():
+        raise SystemExit("parity gate: cached batch must hit all 8 blocks")
+    return {"sampled_requests": 256, "digests": "bit-exact", "prefix_blocks": "all 8 (closed form)"}
+
+
+def e2e_leg(torch, K, W, cache, hosts, steps, bufs, world, dist):
+    """Same metric with host buffers: pinned H2D of each step's inputs and
+    D2H of its prefix lengths inside the timed region."""
+    from paper_2608_09225_gb300.pipeline import DeviceBatch
+    pinned = []
+    for w in hosts:
+        b = w.batch
+        pinned.append(tuple(torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+                            for a in (b.tokens, b.tok_off, b.principal, b.boundary_tok)))
+    n_req = hosts[0].batch.n
+    n_blocks = int((hosts[0].batch.lengths() // 16).sum())
+    out = torch.empty(n_req, dtype=torch.int32).pin_memory()
+    dev = [torch.empty_like(t, device="cuda") for t in pinned[0]]
+    h2d = sum(t.numel() * t.element_size() for t in pinned[0])
+    d2h = out.numel() * out.element_size()
+
+    def one(i):
+        src = pinned[i % len(pinned)]
+        for d, s in zip(dev, src):
+            d.copy_(s, non_blocking=True)
+        db = DeviceBatch(dev[0], dev[1], dev[2], dev[3], n_blocks)
+        prefix, _, _ = cache.serve(W.BOUNDARY, db, bufs)
+        out.copy_(prefix, non_blocking=True)
+
+    for i in range(3):
+        one(i)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    a.record()
+    for i in range(steps):
+        one(i)
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b)
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return {"value": world * steps * n_blocks / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": steps}
+
+
+def cpu_baseline(w, sample):
+    """The oracle, as it stands, on the machine's host cores: a bounded sample."""
+    import oracle
+    oracle.build()
+    cores = len(os.sched_getaffinity(0))
+    ks = oracle.KeySet(1)
+    cpu_oracle_step(w, sample, cores, ks)
+    reps, blocks, t0 = 0, 0, time.perf_counter()
+    while reps < 2 or time.perf_counter() - t0 < 5.0:
+        blocks += cpu_oracle_step(w, sample, cores, ks)
+        reps += 1
+    dt = time.perf_counter() - t0
+    return {"value": blocks / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{reps} steps over the first {sample} requests of one batch "
+                      f"(salts, chain on {cores} threads, probe, insert); {dt:.1f} s"}
+
+
+if __name__ == "__main__":
+    sys.exit(main())

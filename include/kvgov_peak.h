@@ -1,0 +1,41 @@
+/*
+ * kvgov_peak.h -- C ABI of libkvgov_peak: the integer issue-rate
+ * microbenchmark that sets the roofline denominator for the hashing kernels.
+ * It is a measurement tool beside libkvgov, not part of the method.
+ *
+ * The hashing path of the paper (SHA-256 block keys and HMAC salts, section
+ * 4.1; Table 9) is integer work: rotates, three-input booleans and adds.
+ * Its roofline is the rate at which an SM can issue those instructions.
+ */
+#ifndef KVGOV_PEAK_H
+#define KVGOV_PEAK_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *kvgov_stream_t;
+
+/*
+ * kvgov_peak_int -- launch `blocks` CTAs of `threads` threads, each running
+ * `iters` iterations of the instruction body of `kind`:
+ *   0 LOP3, 1 SHF (funnel shift), 2 IADD3, 3 SHA-256 compression (FIPS 180-4).
+ * d_clocks [blocks][3] u64 receives, per CTA, its SM id and its clock64()
+ * at start and end.  d_sink [1] u32 is written only in a case that never
+ * happens (keeps results live).  Asynchronous on `stream`.
+ * Returns 0, 1 for a bad argument (nothing launched), 2 for a launch error.
+ */
+int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint32_t *d_sink,
+                   unsigned long long *d_clocks, kvgov_stream_t stream);
+
+/* Thread-operations one thread executes per iteration of `kind` (nominal
+ * SHA-256 count of 1384 per compression for kind 3), or 0 for a bad kind. */
+int kvgov_peak_ops_per_iter(int kind);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVGOV_PEAK_H */

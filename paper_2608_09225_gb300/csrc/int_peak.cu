@@ -1,0 +1,116 @@
+// int_peak.cu -- integer issue-rate microbenchmark for the roofline of the
+// hashing kernels (libkvgov_peak.so; header include/kvgov_peak.h).
+//
+// Every thread runs `iters` iterations of a fixed body of integer
+// instructions over register-resident values (no memory traffic).  Each CTA
+// records its SM id and clock64() at start and end; the host divides the
+// thread-operations an SM executed by the SM clock cycles it took, which
+// gives thread-ops per SM clock, independent of the clock frequency.
+//
+// Kinds (ops per thread per iteration in kvgov_peak_ops_per_iter):
+//   0  LOP3   x_s = lop3(x_s, x_{s+1}, x_{s+2})    over 8 streams
+//   1  SHF    x_s = shf.r.wrap(x_s, x_{s+1}, n_s)   over 8 streams
+//   2  IADD3  x_s = x_s + x_{s+1} + x_{s+2}         over 8 streams
+//   3  SHA-256: one FIPS 180-4 compression (1384 nominal ops: 64 rounds x 14
+//      + 48 schedule words x 10 + 8) on each of 2 independent chains
+// Each update reads two other streams' latest values, so no chain of updates
+// collapses into fewer instructions (a three-input boolean of three fixed
+// inputs would fold into one LOP3; these never have three fixed inputs).
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "../../include/kvgov_peak.h"
+#include "sha256_dev.cuh"
+
+namespace {
+
+constexpr int kStreams = 8;
+constexpr int kShaChains = 2;
+
+__device__ __forceinline__ uint32_t smid() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
+    return r;
+}
+
+template <int KIND>
+__global__ void peak_kernel(int iters, uint32_t seed, uint32_t *sink, unsigned long long *clocks) {
+    __shared__ unsigned long long t_start;
+    uint32_t x[kStreams];
+#pragma unroll
+    for (int s = 0; s < kStreams; ++s) x[s] = (seed ^ (threadIdx.x * 0x9e3779b9u)) + 0x85ebca6bu * (s + 1);
+    __syncthreads();
+    if (threadIdx.x == 0) t_start = clock64();
+    __syncthreads();
+    if (KIND == 3) {
+        uint32_t st[kShaChains][8], w[kShaChains][16];
+#pragma unroll
+        for (int c = 0; c < kShaChains; ++c) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) st[c][i] = x[i] + c;
+        }
+        for (int it = 0; it < iters; ++it) {
+#pragma unroll
+            for (int c = 0; c < kShaChains; ++c) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) w[c][i] = st[c][i & 7] ^ (uint32_t)i;
+                kvgov_dev::sha_compress(st[c], w[c]);
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) x[i] = st[0][i] ^ st[1][i];
+    } else {
+        for (int it = 0; it < iters; ++it) {
+#pragma unroll
+            for (int rep = 0; rep < 4; ++rep) {
+#pragma unroll
+                for (int s = 0; s < kStreams; ++s) {
+                    const uint32_t a = x[(s + 1) % kStreams], b = x[(s + 2) % kStreams];
+                    if (KIND == 0)
+                        asm("lop3.b32 %0, %0, %1, %2, 0x96;" : "+r"(x[s]) : "r"(a), "r"(b));
+                    else if (KIND == 1)
+                        x[s] = __funnelshift_r(x[s], a, (s * 5 + rep * 3 + 1) & 31);
+                    else
+                        x[s] = x[s] + a + b;
+                }
+            }
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const unsigned long long t_end = clock64();
+        clocks[3 * blockIdx.x + 0] = smid();
+        clocks[3 * blockIdx.x + 1] = t_start;
+        clocks[3 * blockIdx.x + 2] = t_end;
+    }
+    uint32_t acc = 0;
+#pragma unroll
+    for (int s = 0; s < kStreams; ++s) acc ^= x[s];
+    if (acc == 0x12345678u) sink[0] = acc;   // keeps every stream live
+}
+
+}  // namespace
+
+extern "C" int kvgov_peak_ops_per_iter(int kind) {
+    switch (kind) {
+    case 0: case 1: return 4 * kStreams;   // one instruction per update; IADD3 counts as one op
+    case 2: return 4 * kStreams;
+    case 3: return kShaChains * 1384;
+    default: return 0;
+    }
+}
+
+extern "C" int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint32_t *d_sink,
+                              unsigned long long *d_clocks, kvgov_stream_t stream) {
+    if (kind < 0 || kind > 3 || iters <= 0 || blocks <= 0 || threads <= 0 || threads > 1024 || !d_sink ||
+        !d_clocks)
+        return 1;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    switch (kind) {
+    case 0: peak_kernel<0><<<blocks, threads, 0, s>>>(iters, 1u, d_sink, d_clocks); break;
+    case 1: peak_kernel<1><<<blocks, threads, 0, s>>>(iters, 1u, d_sink, d_clocks); break;
+    case 2: peak_kernel<2><<<blocks, threads, 0, s>>>(iters, 1u, d_sink, d_clocks); break;
+    default: peak_kernel<3><<<blocks, threads, 0, s>>>(iters, 1u, d_sink, d_clocks); break;
+    }
+    return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}

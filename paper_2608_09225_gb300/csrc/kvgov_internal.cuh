@@ -1,0 +1,43 @@
+// kvgov_internal.cuh -- helpers shared by the libkvgov translation units.
+#pragma once
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "../../include/kvgov.h"
+
+namespace kvgov_dev {
+
+__device__ __forceinline__ void raise_flag(uint32_t *status, uint32_t flag) {
+    if (status) atomicOr(status, flag);
+}
+
+// 16-byte asynchronous global->shared copy (LDGSTS, L2 only).  src_bytes < 16
+// reads only that many bytes and zero-fills the rest of the destination.
+__device__ __forceinline__ void cp_async16(void *smem_dst, const void *gmem_src, int src_bytes) {
+    const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(gmem_src), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+}  // namespace kvgov_dev
+
+namespace kvgov_host {
+
+inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline bool pow2_capacity(uint64_t cap) { return cap >= KVGOV_MIN_CAPACITY && (cap & (cap - 1)) == 0; }
+
+inline int launch_status() {
+    return cudaGetLastError() == cudaSuccess ? KVGOV_OK : KVGOV_ECUDA;
+}
+
+inline int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 152;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 152;
+    return n;
+}
+
+}  // namespace kvgov_host

@@ -1,0 +1,165 @@
+// sha256_dev.cuh -- register-resident SHA-256 compression for sm_103a.
+//
+// SHA-256 as FIPS 180-4 defines it (section 4.1.2 functions, section 4.2.2
+// constants, section 6.2.2 compression).  The paper fixes H = SHA-256 for
+// block keys and for the HMAC salt (section 4.1; Table 9).
+//
+// Mapping onto the SM's integer pipes:
+//   * every rotate is one funnel shift (SHF.R.W) via __funnelshift_r;
+//   * the three-input boolean functions -- Ch, Maj and the XOR that closes
+//     each Sigma / sigma -- are single LOP3 instructions, written as inline
+//     PTX lop3.b32 with the truth table of the function;
+//   * the 16-word message schedule is a rolling window in registers; with the
+//     rounds fully unrolled every index is a compile-time constant, and the
+//     round constants are immediates, so blocks whose schedule is known at
+//     compile time (the final padding block of a fixed-length message) fold
+//     to constants.
+#pragma once
+#include <cstdint>
+
+namespace kvgov_dev {
+
+// FIPS 180-4 section 4.2.2: K_0 .. K_63.  Returned through a switch so that,
+// after unrolling, each use is an immediate operand.
+__device__ __forceinline__ uint32_t sha_k(int t) {
+    switch (t) {
+    case 0: return 0x428a2f98u; case 1: return 0x71374491u; case 2: return 0xb5c0fbcfu; case 3: return 0xe9b5dba5u;
+    case 4: return 0x3956c25bu; case 5: return 0x59f111f1u; case 6: return 0x923f82a4u; case 7: return 0xab1c5ed5u;
+    case 8: return 0xd807aa98u; case 9: return 0x12835b01u; case 10: return 0x243185beu; case 11: return 0x550c7dc3u;
+    case 12: return 0x72be5d74u; case 13: return 0x80deb1feu; case 14: return 0x9bdc06a7u; case 15: return 0xc19bf174u;
+    case 16: return 0xe49b69c1u; case 17: return 0xefbe4786u; case 18: return 0x0fc19dc6u; case 19: return 0x240ca1ccu;
+    case 20: return 0x2de92c6fu; case 21: return 0x4a7484aau; case 22: return 0x5cb0a9dcu; case 23: return 0x76f988dau;
+    case 24: return 0x983e5152u; case 25: return 0xa831c66du; case 26: return 0xb00327c8u; case 27: return 0xbf597fc7u;
+    case 28: return 0xc6e00bf3u; case 29: return 0xd5a79147u; case 30: return 0x06ca6351u; case 31: return 0x14292967u;
+    case 32: return 0x27b70a85u; case 33: return 0x2e1b2138u; case 34: return 0x4d2c6dfcu; case 35: return 0x53380d13u;
+    case 36: return 0x650a7354u; case 37: return 0x766a0abbu; case 38: return 0x81c2c92eu; case 39: return 0x92722c85u;
+    case 40: return 0xa2bfe8a1u; case 41: return 0xa81a664bu; case 42: return 0xc24b8b70u; case 43: return 0xc76c51a3u;
+    case 44: return 0xd192e819u; case 45: return 0xd6990624u; case 46: return 0xf40e3585u; case 47: return 0x106aa070u;
+    case 48: return 0x19a4c116u; case 49: return 0x1e376c08u; case 50: return 0x2748774cu; case 51: return 0x34b0bcb5u;
+    case 52: return 0x391c0cb3u; case 53: return 0x4ed8aa4au; case 54: return 0x5b9cca4fu; case 55: return 0x682e6ff3u;
+    case 56: return 0x748f82eeu; case 57: return 0x78a5636fu; case 58: return 0x84c87814u; case 59: return 0x8cc70208u;
+    case 60: return 0x90befffau; case 61: return 0xa4506cebu; case 62: return 0xbef9a3f7u; default: return 0xc67178f2u;
+    }
+}
+
+// FIPS 180-4 section 5.3.3: initial hash value H(0).
+__device__ __forceinline__ void sha_iv(uint32_t s[8]) {
+    s[0] = 0x6a09e667u; s[1] = 0xbb67ae85u; s[2] = 0x3c6ef372u; s[3] = 0xa54ff53au;
+    s[4] = 0x510e527fu; s[5] = 0x9b05688cu; s[6] = 0x1f83d9abu; s[7] = 0x5be0cd19u;
+}
+
+__device__ __forceinline__ uint32_t rotr(uint32_t x, int n) { return __funnelshift_r(x, x, n); }
+
+// LOP3 truth tables over (a = 0xF0, b = 0xCC, c = 0xAA).
+#ifndef KVGOV_PLAIN_BOOL
+__device__ __forceinline__ uint32_t xor3(uint32_t a, uint32_t b, uint32_t c) {
+    uint32_t r;
+    asm("lop3.b32 %0, %1, %2, %3, 0x96;" : "=r"(r) : "r"(a), "r"(b), "r"(c));
+    return r;
+}
+// Ch(x, y, z) = (x & y) ^ (~x & z)
+__device__ __forceinline__ uint32_t ch(uint32_t x, uint32_t y, uint32_t z) {
+    uint32_t r;
+    asm("lop3.b32 %0, %1, %2, %3, 0xCA;" : "=r"(r) : "r"(x), "r"(y), "r"(z));
+    return r;
+}
+// Maj(x, y, z) = (x & y) ^ (x & z) ^ (y & z)
+__device__ __forceinline__ uint32_t maj(uint32_t x, uint32_t y, uint32_t z) {
+    uint32_t r;
+    asm("lop3.b32 %0, %1, %2, %3, 0xE8;" : "=r"(r) : "r"(x), "r"(y), "r"(z));
+    return r;
+}
+#else
+__device__ __forceinline__ uint32_t xor3(uint32_t a, uint32_t b, uint32_t c) { return a ^ b ^ c; }
+__device__ __forceinline__ uint32_t ch(uint32_t x, uint32_t y, uint32_t z) { return (x & y) ^ (~x & z); }
+__device__ __forceinline__ uint32_t maj(uint32_t x, uint32_t y, uint32_t z) { return (x & y) | (z & (x | y)); }
+#endif
+
+__device__ __forceinline__ uint32_t bsig0(uint32_t x) { return xor3(rotr(x, 2), rotr(x, 13), rotr(x, 22)); }
+__device__ __forceinline__ uint32_t bsig1(uint32_t x) { return xor3(rotr(x, 6), rotr(x, 11), rotr(x, 25)); }
+__device__ __forceinline__ uint32_t ssig0(uint32_t x) { return xor3(rotr(x, 7), rotr(x, 18), x >> 3); }
+__device__ __forceinline__ uint32_t ssig1(uint32_t x) { return xor3(rotr(x, 17), rotr(x, 19), x >> 10); }
+
+// Big-endian word from 4 little-endian-loaded bytes, and back.
+__device__ __forceinline__ uint32_t bswap32(uint32_t x) { return __byte_perm(x, 0u, 0x0123u); }
+
+// One compression (FIPS 180-4 section 6.2.2, steps 1-4) of the 512-bit block
+// w[0..15] (big-endian words) into the chaining state s.  w is overwritten by
+// the message schedule.
+__device__ __forceinline__ void sha_compress(uint32_t s[8], uint32_t w[16]) {
+    uint32_t a = s[0], b = s[1], c = s[2], d = s[3];
+    uint32_t e = s[4], f = s[5], g = s[6], h = s[7];
+#pragma unroll
+    for (int t = 0; t < 64; ++t) {
+        if (t >= 16)
+            w[t & 15] += ssig1(w[(t - 2) & 15]) + w[(t - 7) & 15] + ssig0(w[(t - 15) & 15]);
+        const uint32_t t1 = h + (sha_k(t) + w[t & 15]) + ch(e, f, g) + bsig1(e);
+        const uint32_t t2 = bsig0(a) + maj(a, b, c);
+        h = g; g = f; f = e; e = d + t1;
+        d = c; c = b; b = a; a = t1 + t2;
+    }
+    s[0] += a; s[1] += b; s[2] += c; s[3] += d;
+    s[4] += e; s[5] += f; s[6] += g; s[7] += h;
+}
+
+// Fixed-length messages of the chain (section 2.1 / 4.1 / 4.2 equations).
+// Arguments are big-endian message words; out gets the digest's state words
+// (digest byte 4i.. 4i+3 = out[i] big-endian).  SHA-256 padding (section
+// 5.1.1) appends 0x80, zeros and the 64-bit bit length; for these lengths the
+// padding words are compile-time constants.
+
+// H(T): 64-byte message = one data block + one constant padding block.
+__device__ __forceinline__ void sha256_msg64(const uint32_t tw[16], uint32_t out[8]) {
+    uint32_t s[8], w[16];
+    sha_iv(s);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) w[i] = tw[i];
+    sha_compress(s, w);
+    w[0] = 0x80000000u;
+#pragma unroll
+    for (int i = 1; i < 15; ++i) w[i] = 0u;
+    w[15] = 64u * 8u;
+    sha_compress(s, w);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) out[i] = s[i];
+}
+
+// H(P || T): 32-byte prefix P (parent digest or salt) + 64-byte block.
+__device__ __forceinline__ void sha256_msg96(const uint32_t pw[8], const uint32_t tw[16], uint32_t out[8]) {
+    uint32_t s[8], w[16];
+    sha_iv(s);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) { w[i] = pw[i]; w[8 + i] = tw[i]; }
+    sha_compress(s, w);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) w[i] = tw[8 + i];
+    w[8] = 0x80000000u;
+#pragma unroll
+    for (int i = 9; i < 15; ++i) w[i] = 0u;
+    w[15] = 96u * 8u;
+    sha_compress(s, w);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) out[i] = s[i];
+}
+
+// H(S || P || T): salt, parent digest, block (the boundary block of 4.2).
+__device__ __forceinline__ void sha256_msg128(const uint32_t sw[8], const uint32_t pw[8], const uint32_t tw[16],
+                                              uint32_t out[8]) {
+    uint32_t s[8], w[16];
+    sha_iv(s);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) { w[i] = sw[i]; w[8 + i] = pw[i]; }
+    sha_compress(s, w);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) w[i] = tw[i];
+    sha_compress(s, w);
+    w[0] = 0x80000000u;
+#pragma unroll
+    for (int i = 1; i < 15; ++i) w[i] = 0u;
+    w[15] = 128u * 8u;
+    sha_compress(s, w);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) out[i] = s[i];
+}
+
+}  // namespace kvgov_dev

@@ -1,0 +1,110 @@
+"""The hot path as one call sequence: salts -> blocking -> chain -> probe -> insert.
+
+``PrefixCache`` owns the device-resident state of one KVGov prefix-cache
+index (the slot table and the per-principal salts) and runs a batch of
+requests through the library's kernels on one CUDA stream.  Nothing here
+computes; every step is a libkvgov entry point (include/kvgov.h).
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+import torch
+
+from . import kvgov as K
+
+
+def next_pow2(n: int) -> int:
+    return 1 << max(int(n) - 1, 0).bit_length()
+
+
+@dataclass
+class DeviceBatch:
+    """Device copies of one batch of requests (CSR tokens)."""
+    tokens: torch.Tensor        # int32 [T]
+    tok_off: torch.Tensor       # int64 [n + 1]
+    principal: torch.Tensor     # int32 [n]
+    boundary_tok: torch.Tensor  # int32 [n]
+    n_blocks: int               # sum of floor(len / 16), known on the host
+
+    @property
+    def n(self) -> int:
+        return self.tok_off.numel() - 1
+
+    @staticmethod
+    def from_host(tokens, tok_off, principal, boundary_tok, device="cuda", non_blocking=False) -> "DeviceBatch":
+        tok_off_np = np.asarray(tok_off, dtype=np.int64)
+        n_blocks = int((np.diff(tok_off_np) // K.BLOCK).sum())
+
+        def put(a, dt):
+            t = a if isinstance(a, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(a, dtype=dt))
+            return t.to(device, non_blocking=non_blocking)
+
+        return DeviceBatch(put(tokens, np.int32), put(tok_off_np, np.int64), put(principal, np.int32),
+                           put(boundary_tok, np.int32), n_blocks)
+
+
+class PrefixCache:
+    """A GPU-resident block prefix-cache index with per-principal salts.
+
+    capacity   table slots (power of two, >= 32), 32 bytes each.
+    secret     the server secret K (HMAC key of section 4.1).
+    ids/id_off principal-id bytes in CSR form (host numpy or device tensors).
+    """
+
+    def __init__(self, capacity: int, secret: bytes, ids, id_off, device="cuda", stream=None):
+        self.device = torch.device(device)
+        self.stream = stream
+        self.capacity = int(capacity)
+        self.secret = bytes(secret)
+        self.ids = torch.as_tensor(np.asarray(ids, dtype=np.uint8)).to(self.device)
+        self.id_off = torch.as_tensor(np.asarray(id_off, dtype=np.int64)).to(self.device)
+        self.n_principals = self.id_off.numel() - 1
+        self.salts = torch.empty((self.n_principals, 32), dtype=torch.uint8, device=self.device)
+        self.slots = torch.empty((self.capacity, 32), dtype=torch.uint8, device=self.device)
+        self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
+        self.n_new = torch.zeros(1, dtype=torch.int64, device=self.device)
+        K.table_init(self.slots, self.stream)
+        self.derive_salts()
+
+    # -- individual steps ------------------------------------------------
+    def derive_salts(self):
+        K.derive_salts(self.secret, self.ids, self.id_off, self.salts, self.status, self.stream)
+        return self.salts
+
+    def hash(self, mode: int, b: DeviceBatch, blk_off=None, digests=None):
+        if blk_off is None:
+            blk_off = torch.empty(b.n + 1, dtype=torch.int64, device=self.device)
+        K.block_offsets(b.tok_off, blk_off, self.status, self.stream)
+        if digests is None:
+            digests = torch.empty((b.n_blocks, 32), dtype=torch.uint8, device=self.device)
+        salted = mode != K.UNSALTED
+        K.chain_hash(mode, b.tokens, b.tok_off, blk_off, b.principal if salted else None,
+                     self.salts if salted else None, b.boundary_tok if mode == K.BOUNDARY else None,
+                     digests, status=self.status, stream=self.stream)
+        return blk_off, digests
+
+    def insert(self, keys: torch.Tensor):
+        K.insert(self.slots, keys, self.status, self.n_new, self.stream)
+
+    def probe(self, digests, blk_off, prefix_blocks=None):
+        return K.probe(self.slots, digests, blk_off, prefix_blocks, self.status, self.stream)
+
+    # -- one serving step -------------------------------------------------
+    def serve(self, mode: int, b: DeviceBatch, bufs: dict | None = None, derive_salts: bool = True):
+        """Salts, blocking, chain, probe, insert for one batch.  Returns
+        (prefix_blocks, digests, blk_off), all on the device."""
+        bufs = bufs if bufs is not None else {}
+        if derive_salts:
+            self.derive_salts()
+        blk_off, digests = self.hash(mode, b, bufs.get("blk_off"), bufs.get("digests"))
+        prefix = self.probe(digests, blk_off, bufs.get("prefix"))
+        self.insert(digests)
+        return prefix, digests, blk_off
+
+    def check_status(self):
+        s = int(self.status.item()) & 0xFFFFFFFF
+        if s:
+            raise K.KVGovError(s, "device status")
+        return s

@@ -1,0 +1,281 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle,
+bit-exact on every salt, block offset, digest, prefix length and insert
+count; plus the device-detected error flags.  Marked gpu."""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_09225_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+DEV = "cuda"
+
+
+def dev(a, dtype=None):
+    t = torch.from_numpy(np.ascontiguousarray(a if dtype is None else np.asarray(a, dtype=dtype)))
+    return t.to(DEV)
+
+
+def status_tensor():
+    return torch.zeros(1, dtype=torch.int32, device=DEV)
+
+
+def gpu_chain(kv, mode, b: W.Batch, salts_np, status=None):
+    toks = dev(b.tokens, np.int32)
+    tok_off = dev(b.tok_off, np.int64)
+    blk = kv.block_offsets(tok_off, status=status)
+    n_blocks = int((np.diff(b.tok_off) // 16).sum())
+    d = kv.chain_hash(mode, toks, tok_off, blk, dev(b.principal, np.int32), dev(salts_np, np.uint8),
+                      dev(b.boundary_tok, np.int32), n_blocks=n_blocks, status=status)
+    torch.cuda.synchronize()
+    return blk.cpu().numpy(), d.cpu().numpy()
+
+
+# ----------------------------------------------------------------- salts
+@pytest.mark.parametrize("secret_len", [0, 1, 32, 63, 64, 65, 200, 1024])
+def test_salts_match_oracle(kv, secret_len):
+    rng = np.random.default_rng(secret_len)
+    secret = rng.integers(0, 256, secret_len, dtype=np.uint8).tobytes()
+    ids, id_off = W.principal_ids(4096)
+    s = kv.derive_salts(secret, dev(ids), dev(id_off))
+    torch.cuda.synchronize()
+    assert (s.cpu().numpy() == oracle.derive_salts(secret, ids, id_off)).all()
+
+
+def test_salts_variable_length_ids(kv):
+    rng = np.random.default_rng(21)
+    lens = rng.integers(0, 300, 777)
+    lens[:10] = [0, 1, 55, 56, 63, 64, 119, 120, 0, 200]
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    ids = rng.integers(0, 256, int(off[-1]), dtype=np.uint8)
+    secret = b"server secret"
+    s = kv.derive_salts(secret, dev(ids), dev(off))
+    torch.cuda.synchronize()
+    assert (s.cpu().numpy() == oracle.derive_salts(secret, ids, off)).all()
+
+
+def test_salts_bad_offsets_flagged(kv):
+    ids, off = W.principal_ids(4)
+    off = off.copy()
+    off[2] = 1          # principal 1 has a decreasing range
+    st = status_tensor()
+    salts = torch.zeros((4, 32), dtype=torch.uint8, device=DEV)
+    kv.derive_salts(b"k", dev(ids), dev(off), salts, st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & kv.F_BADINDEX
+    ref = oracle.derive_salts(b"k", ids, W.principal_ids(4)[1])
+    assert (salts.cpu().numpy()[[0, 3]] == ref[[0, 3]]).all()
+
+
+# --------------------------------------------------------- block offsets
+@pytest.mark.parametrize("n", [0, 1, 5, 127, 4095, 4096, 4097, 10000, 131073])
+def test_block_offsets(kv, n):
+    rng = np.random.default_rng(n)
+    lens = rng.integers(0, 200, n)
+    tok_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    st = status_tensor()
+    blk = kv.block_offsets(dev(tok_off), status=st)
+    torch.cuda.synchronize()
+    assert (blk.cpu().numpy() == oracle.block_offsets(tok_off)).all()
+    assert int(st.item()) == 0
+
+
+def test_block_offsets_negative_length_flagged(kv):
+    tok_off = np.array([0, 16, 8, 40], dtype=np.int64)
+    st = status_tensor()
+    kv.block_offsets(dev(tok_off), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & kv.F_BADINDEX
+
+
+# ------------------------------------------------------------------ chain
+RAGGED = [0, 15, 16, 17, 31, 32, 33, 2119, 64, 100, 7, 48, 3, 19, 257, 1, 128, 129, 130, 131]
+
+
+@pytest.mark.parametrize("mode", [0, 1, 2])
+@pytest.mark.parametrize("lengths", [RAGGED, RAGGED * 17, [3, 16], [1, 16 * 9 + 2], [5] * 300],
+                         ids=["ragged", "ragged_many_ctas", "tail_at_array_end", "tail2", "all_short"])
+def test_chain_matches_oracle(kv, mode, lengths):
+    b = W.ragged(31 + len(lengths), lengths)
+    salts = oracle.derive_salts(b"salt key", *W.principal_ids(8))
+    st = status_tensor()
+    blk, d = gpu_chain(kv, mode, b, salts, st)
+    assert int(st.item()) == 0
+    ref = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+    assert (blk == oracle.block_offsets(b.tok_off)).all()
+    assert d.shape == ref.shape
+    bad = np.nonzero((d != ref).any(axis=1))[0]
+    assert len(bad) == 0, f"{len(bad)} digests differ, first rows {bad[:5]}"
+
+
+@pytest.mark.parametrize("boundary", [0, 15, 16, 17, 100, 16 * 20, 16 * 39, 16 * 40, 16 * 41, 10 ** 9])
+def test_chain_boundary_positions(kv, boundary):
+    """k = 0, interior, last block (k = n_b - 1), past the end."""
+    b = W.ragged(5, [16 * 40] * 150)
+    b.boundary_tok[:] = boundary
+    salts = oracle.derive_salts(b"B", *W.principal_ids(8))
+    _, d = gpu_chain(kv, 2, b, salts)
+    ref = oracle.chain_hash(2, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+    assert (d == ref).all()
+
+
+def test_chain_against_golden_file(kv):
+    with open(os.path.join(GOLDEN, "oracle_small.json")) as f:
+        g = json.load(f)
+    b = W.ragged(g["seed"], g["lengths"])
+    ids, id_off = W.principal_ids(g["n_principals"])
+    s = kv.derive_salts(bytes.fromhex(g["secret_hex"]), dev(ids), dev(id_off))
+    torch.cuda.synchronize()
+    salts = s.cpu().numpy()
+    assert [x.tobytes().hex() for x in salts] == g["salts"]
+    for name, mode in (("unsalted", 0), ("root", 1), ("boundary", 2)):
+        blk, d = gpu_chain(kv, mode, b, salts)
+        assert blk.tolist() == g["blk_off"]
+        assert [x.tobytes().hex() for x in d] == g["digests_" + name]
+
+
+def test_chain_bad_principal_flagged(kv):
+    b = W.ragged(9, [64, 64, 64])
+    b.principal[:] = [0, 99, 1]
+    salts = oracle.derive_salts(b"k", *W.principal_ids(8))
+    st = status_tensor()
+    _, d = gpu_chain(kv, 1, b, salts, st)
+    assert int(st.item()) & kv.F_BADINDEX
+    good = b.principal.copy()
+    good[1] = 0
+    ref = oracle.chain_hash(1, b.tokens, b.tok_off, good, salts)
+    assert (d[:4] == ref[:4]).all() and (d[8:] == ref[8:]).all()
+
+
+def test_chain_negative_boundary_flagged(kv):
+    b = W.ragged(9, [64, 64])
+    b.boundary_tok[:] = [-5, 16]
+    st = status_tensor()
+    gpu_chain(kv, 2, b, oracle.derive_salts(b"k", *W.principal_ids(8)), st)
+    assert int(st.item()) & kv.F_BADINDEX
+
+
+# ------------------------------------------------------------------ table
+def keys_np(n, seed):
+    k = np.random.default_rng(seed).integers(0, 256, (n, 32), dtype=np.uint8)
+    k[:, 0] |= 1
+    return k
+
+
+def table_contents(slots):
+    s = slots.cpu().numpy()
+    w0 = s[:, :8].view(np.uint64).reshape(-1)
+    full = s[(w0 != 0) & (w0 != np.uint64(0xFFFFFFFFFFFFFFFF))]
+    return {r.tobytes() for r in full}
+
+
+def test_insert_set_semantics(kv):
+    k = keys_np(5000, 1)
+    batch = np.concatenate([k, k[::-1], k[:100], k[:100]])
+    slots = kv.new_table(1 << 14)
+    st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
+    kv.insert(slots, dev(batch), st, n_new)
+    kv.insert(slots, dev(k[:777]), st, n_new)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0 and int(n_new.item()) == 5000
+    assert table_contents(slots) == {r.tobytes() for r in k}
+
+
+def test_insert_heavy_in_batch_duplicates(kv):
+    """One key repeated 100,000 times plus 64 keys each 512 times: every
+    concurrent claim of the same key stores it once."""
+    k = keys_np(65, 2)
+    batch = np.concatenate([np.repeat(k[:1], 100000, axis=0), np.tile(k[1:], (512, 1))])
+    batch = batch[np.random.default_rng(3).permutation(len(batch))]
+    slots = kv.new_table(1 << 10)
+    st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
+    kv.insert(slots, dev(batch), st, n_new)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0 and int(n_new.item()) == 65
+    assert table_contents(slots) == {r.tobytes() for r in k}
+
+
+def test_insert_reserved_keys(kv):
+    k = keys_np(10, 4)
+    k[3, :] = 0                 # all zero
+    k[5, :8] = 255              # first word all ones
+    k[7, :8] = 0                # first word zero, rest not
+    slots = kv.new_table(64)
+    st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
+    kv.insert(slots, dev(k), st, n_new)
+    torch.cuda.synchronize()
+    assert int(st.item()) == kv.F_SENTINEL
+    ks = oracle.KeySet(1)
+    n_ref, flagged = ks.insert(k)
+    assert flagged and int(n_new.item()) == n_ref == 7
+    assert table_contents(slots) == {r.tobytes() for r in ks.contents()}
+
+
+def test_table_full(kv):
+    k = keys_np(40, 5)
+    slots = kv.new_table(32)
+    st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
+    kv.insert(slots, dev(k), st, n_new)
+    torch.cuda.synchronize()
+    assert int(st.item()) & kv.F_TABLE_FULL
+    assert int(n_new.item()) == 32 and len(table_contents(slots)) == 32
+
+
+def test_insert_wait_times_out_on_a_claim_nobody_publishes(kv):
+    """A slot left claimed (first word all ones) by an insert that never
+    publishes: a later insert homed there waits a bounded number of times,
+    reports KVGOV_F_TIMEOUT and returns; probes treat the slot as occupied."""
+    cap = 64
+    k = keys_np(1, 6)
+    home = int(k[0, :8].view(np.uint64)[0]) & (cap - 1)
+    slots = kv.new_table(cap)
+    slots[home, :8] = 255
+    st = status_tensor()
+    prev = kv.set_spin_limit(1000)
+    try:
+        kv.insert(slots, dev(k), st)
+        torch.cuda.synchronize()
+    finally:
+        kv.set_spin_limit(prev)
+    assert int(st.item()) == kv.F_TIMEOUT
+    blk = dev(np.array([0, 1], np.int64))
+    pre = kv.probe(slots, dev(k), blk)
+    torch.cuda.synchronize()
+    assert int(pre.item()) == 0
+
+
+@pytest.mark.parametrize("cap_log2", [5, 10, 16])
+def test_probe_matches_oracle(kv, cap_log2):
+    """Random chains of known digests against a table holding a random subset:
+    prefix length = first missing block (later hits ignored)."""
+    rng = np.random.default_rng(cap_log2)
+    pool = keys_np(min(1 << (cap_log2 - 1), 4000), cap_log2 + 100)
+    nb = rng.integers(0, 70, 3000)
+    nb[:5] = [0, 1, 33, 64, 69]
+    off = np.concatenate([[0], np.cumsum(nb)]).astype(np.int64)
+    digests = pool[rng.integers(0, len(pool), int(off[-1]))]
+    member = rng.random(len(pool)) < 0.85
+    slots = kv.new_table(1 << cap_log2)
+    st = status_tensor()
+    kv.insert(slots, dev(pool[member]), st)
+    pre = kv.probe(slots, dev(digests), dev(off), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    ks = oracle.KeySet(1)
+    ks.insert(pool[member])
+    assert (pre.cpu().numpy() == ks.prefix_blocks(digests, off)).all()
+
+
+def test_probe_empty_and_bad_offsets(kv):
+    slots = kv.new_table(64)
+    st = status_tensor()
+    pre = kv.probe(slots, dev(keys_np(4, 7)), dev(np.array([0, 4, 2], np.int64)), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & kv.F_BADINDEX
+    empty = kv.probe(slots, dev(keys_np(1, 7)), dev(np.array([0], np.int64)))
+    assert empty.numel() == 0

@@ -1,0 +1,140 @@
+"""The five workloads through the CUDA path, bit-exact against the oracle:
+reduced sizes, then the full sizes in the launch configuration bench.py
+times (PrefixCache.serve: salts, blocking, chain, probe, insert).  Marked gpu."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_09225_gb300 import workloads as W
+from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache, next_pow2
+from tests.pins import run_workload_oracle
+
+pytestmark = pytest.mark.gpu
+
+
+def run_gpu(kv, w: W.Workload, mode: int):
+    """Salts, chains, table fill (same content as the oracle's) and probe."""
+    cap = w.capacity or 1024
+    cache = PrefixCache(cap, w.secret, w.ids, w.id_off)
+    b = w.batch
+    db = DeviceBatch.from_host(b.tokens, b.tok_off, b.principal, b.boundary_tok)
+    blk, d = cache.hash(mode, db)
+    blk_np = blk.cpu().numpy()
+    if w.fill_from == "prior":
+        p = w.prior
+        dp = DeviceBatch.from_host(p.tokens, p.tok_off, p.principal, p.boundary_tok)
+        _, dpd = cache.hash(mode, dp)
+        cache.insert(dpd)
+    else:
+        f0, f1 = w.fill
+        if f1 > f0:
+            cache.insert(d[blk_np[f0]:blk_np[f1]])
+    if w.random_keys is not None:
+        cache.insert(torch.from_numpy(w.random_keys).cuda())
+    p0, p1 = w.probe
+    pre = cache.probe(d, blk[p0:p1 + 1])
+    torch.cuda.synchronize()
+    cache.check_status()
+    return cache, blk_np, d.cpu().numpy(), pre.cpu().numpy()
+
+
+def check(kv, w, mode):
+    cache, blk, d, pre = run_gpu(kv, w, mode)
+    salts, dref, bref, ks, pref = run_workload_oracle(w, mode)
+    assert (cache.salts.cpu().numpy() == salts).all()
+    assert (blk == bref).all()
+    bad = np.nonzero((d != dref).any(axis=1))[0]
+    assert len(bad) == 0, f"{len(bad)} of {len(d)} digests differ"
+    assert (pre == pref).all(), f"{int((pre != pref).sum())} prefix lengths differ"
+    assert int(cache.n_new.item()) == ks.n
+    return pre
+
+
+def test_tiny_full(kv):
+    pre = check(kv, W.make("tiny"), W.ROOT)
+    assert list(pre) == [16] * 16 + [8] * 16 + [0] * 32
+
+
+def test_sysprompt_reduced(kv):
+    check(kv, W.sysprompt(n_req=128, fill_n=32), W.ROOT)
+
+
+@pytest.mark.parametrize("mode", [W.UNSALTED, W.ROOT, W.BOUNDARY])
+def test_template_reduced(kv, mode):
+    check(kv, W.template(n_req=1024), mode)
+
+
+def test_probe_reduced(kv):
+    w = W.probe(n_req=2048, n_prior=256, capacity=1 << 16)
+    pre = check(kv, w, W.ROOT)
+    assert (pre == w.info["cut"]).all()
+
+
+def test_long_reduced(kv):
+    w = W.long(seed=11, n_req=8)
+    w.capacity, w.fill, w.probe = 1 << 16, (0, 4), (0, 8)
+    check(kv, w, W.BOUNDARY)
+
+
+def test_wide_reduced(kv):
+    w = W.wide(seed=12, n_req=4096)
+    w.capacity, w.fill, w.probe = 1 << 16, (0, 2048), (0, 4096)
+    pre = check(kv, w, W.BOUNDARY)
+    assert (pre[:2048] == 8).all() and (pre[2048:] == 4).all()
+
+
+# ------------------------------------------------------------- full sizes
+def test_full_sysprompt(kv):
+    w = W.make("sysprompt")
+    pre = check(kv, w, W.ROOT)
+    filled = set(w.batch.principal[:256].tolist())
+    assert list(pre) == [132] * 256 + [64 if int(p) in filled else 0 for p in w.batch.principal[256:]]
+
+
+@pytest.mark.parametrize("mode", [W.UNSALTED, W.ROOT, W.BOUNDARY])
+def test_full_template(kv, mode):
+    check(kv, W.make("template"), mode)
+
+
+def test_full_probe(kv):
+    w = W.make("probe")
+    pre = check(kv, w, W.ROOT)
+    assert (pre == w.info["cut"]).all()
+
+
+def test_full_long(kv):
+    w = W.make("long", seed=77)
+    w.capacity, w.fill, w.probe = 1 << 20, (0, 128), (0, 256)
+    pre = check(kv, w, W.BOUNDARY)
+    assert (pre[:128] == 2048).all() and (pre[128:] == 4).all()
+
+
+def test_full_wide_serving_steps(kv):
+    """The bench's step (PrefixCache.serve) on the full 131,072 x 128 batch,
+    three times: batch A into an empty cache, a fresh batch B, then A again.
+    Every salt, digest and prefix length is compared with the oracle."""
+    wa, wb = W.make("wide", seed=101), W.make("wide", seed=102)
+    wb.secret, wb.ids, wb.id_off = wa.secret, wa.ids, wa.id_off
+    n_blocks = wa.batch.n * 8
+    cache = PrefixCache(next_pow2(4 * 3 * n_blocks), wa.secret, wa.ids, wa.id_off)
+    salts = oracle.derive_salts(wa.secret, wa.ids, wa.id_off)
+    ks = oracle.KeySet(1)
+    seen = []
+    for w in (wa, wb, wa):
+        b = w.batch
+        db = DeviceBatch.from_host(b.tokens, b.tok_off, b.principal, b.boundary_tok)
+        pre, d, blk = cache.serve(W.BOUNDARY, db)
+        torch.cuda.synchronize()
+        cache.check_status()
+        dref = oracle.chain_hash(W.BOUNDARY, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+        bref = oracle.block_offsets(b.tok_off)
+        assert (cache.salts.cpu().numpy() == salts).all()
+        assert (blk.cpu().numpy() == bref).all()
+        assert (d.cpu().numpy() == dref).all()
+        pref = ks.prefix_blocks(dref, bref)
+        assert (pre.cpu().numpy() == pref).all()
+        ks.insert(dref)
+        assert int(cache.n_new.item()) == ks.n
+        seen.append(int(pref.min()))
+    assert seen == [0, 4, 8]

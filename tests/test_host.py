@@ -1,0 +1,162 @@
+"""CPU-only checks: the C-ABI library builds, loads and exports every symbol
+the header declares; host-side argument validation; the golden file is still
+what the oracle computes; the seeded workloads have the structure they claim.
+No GPU and no kernel launch is involved."""
+import ctypes
+import json
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_09225_gb300 import build as kbuild
+from paper_2608_09225_gb300 import workloads as W
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "kvgov.h")
+
+
+@pytest.fixture(scope="module")
+def libkv():
+    path = kbuild.build()
+    return ctypes.CDLL(path)
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(kvgov_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for want in ("kvgov_derive_salts", "kvgov_block_offsets", "kvgov_chain_hash", "kvgov_table_init",
+                 "kvgov_insert", "kvgov_probe", "kvgov_status_string", "kvgov_set_spin_limit"):
+        assert want in names
+
+
+def test_library_exports_every_declared_symbol(libkv):
+    for name in declared_functions():
+        assert hasattr(libkv, name), name
+
+
+def test_status_strings(libkv):
+    f = libkv.kvgov_status_string
+    f.restype = ctypes.c_char_p
+    f.argtypes = [ctypes.c_int]
+    assert f(0) == b"KVGOV_OK"
+    assert b"EINVAL" in f(1)
+    for flag, word in ((0x10, b"BADINDEX"), (0x20, b"SENTINEL"), (0x40, b"FULL"), (0x80, b"TIMEOUT")):
+        assert word in f(flag)
+    assert f(12345)
+
+
+def test_spin_limit_roundtrip(libkv):
+    f = libkv.kvgov_set_spin_limit
+    f.restype = ctypes.c_uint32
+    f.argtypes = [ctypes.c_uint32]
+    prev = f(77)
+    assert f(0) == 77
+    assert f(prev) == 1 << 23
+
+
+def test_host_validation_rejects_bad_arguments(libkv):
+    """Arguments the host can check are refused with KVGOV_EINVAL before any
+    CUDA call (these calls never reach the GPU)."""
+    p = ctypes.c_void_p
+    fake = p(1 << 20)          # never dereferenced: every call below fails validation first
+    odd = p((1 << 20) + 4)     # not 16-byte aligned
+    ch = libkv.kvgov_chain_hash
+    ch.argtypes = [ctypes.c_int, p, p, ctypes.c_int32, p, p, ctypes.c_int32, p, p, p, p, p]
+    assert ch(7, fake, fake, 4, fake, fake, 1, fake, fake, fake, None, None) == 1          # bad mode
+    assert ch(0, odd, fake, 4, None, None, 0, None, fake, fake, None, None) == 1            # misaligned tokens
+    assert ch(0, fake, fake, 4, None, None, 0, None, fake, odd, None, None) == 1            # misaligned digests
+    assert ch(1, fake, fake, 4, None, fake, 1, None, fake, fake, None, None) == 1           # ROOT without principal
+    assert ch(2, fake, fake, 4, fake, fake, 1, None, fake, fake, None, None) == 1           # BOUNDARY without offsets
+    assert ch(0, fake, fake, -1, None, None, 0, None, fake, fake, None, None) == 1          # negative n_req
+    assert ch(0, fake, fake, 0, None, None, 0, None, fake, fake, None, None) == 0           # empty batch: no-op
+    ti = libkv.kvgov_table_init
+    ti.argtypes = [p, ctypes.c_uint64, p]
+    for cap in (0, 16, 48, 1000):
+        assert ti(fake, cap, None) == 1
+    ins = libkv.kvgov_insert
+    ins.argtypes = [p, ctypes.c_uint64, p, ctypes.c_int64, p, p, p]
+    assert ins(fake, 64, fake, 5, None, None, None) == 1      # status is required
+    assert ins(fake, 64, fake, -1, None, fake, None) == 1
+    assert ins(fake, 64, None, 0, None, fake, None) == 0      # nothing to insert
+    pr = libkv.kvgov_probe
+    pr.argtypes = [p, ctypes.c_uint64, p, p, ctypes.c_int32, p, p, p]
+    assert pr(fake, 100, fake, fake, 3, fake, None, None) == 1
+    assert pr(fake, 64, odd, fake, 3, fake, None, None) == 1
+    sa = libkv.kvgov_derive_salts
+    sa.argtypes = [p, ctypes.c_size_t, p, p, ctypes.c_int32, p, p, p]
+    assert sa(None, 1025, fake, fake, 3, fake, None, None) == 1
+    assert sa(None, 5, fake, fake, 3, fake, None, None) == 1
+    assert sa(None, 0, fake, fake, 0, fake, None, None) == 0
+    bo = libkv.kvgov_block_offsets
+    bo.argtypes = [p, ctypes.c_int32, p, p, p]
+    assert bo(fake, -2, fake, None, None) == 1
+
+
+def test_golden_file_is_what_the_oracle_computes():
+    import importlib.util
+    spec = importlib.util.spec_from_file_location("make_golden", os.path.join(ROOT, "tests", "golden",
+                                                                              "make_golden.py"))
+    mg = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mg)
+    with open(mg.OUT) as f:
+        stored = json.load(f)
+    assert mg.compute() == stored
+
+
+# ----------------------------------------------------------------- workloads
+def test_workloads_are_deterministic():
+    a, b = W.make("template", n_req=64), W.make("template", n_req=64)
+    assert a.secret == b.secret and (a.batch.tokens == b.batch.tokens).all()
+    c = W.make("wide", seed=5, n_req=32)
+    d = W.make("wide", seed=6, n_req=32)
+    assert not (c.batch.tokens == d.batch.tokens).all()
+
+
+def test_workload_structure():
+    w = W.make("tiny")
+    t = w.batch.tokens.reshape(64, 256)
+    assert (t[:32, :128] == t[0, :128]).all() and not (t[32:, :128] == t[0, :128]).all(axis=1).any()
+    assert t.min() >= 0 and t.max() < W.VOCAB
+    s = W.sysprompt(n_req=64)
+    ts = s.batch.tokens.reshape(64, 2119)
+    assert (ts[:, :1024] == ts[0, :1024]).all()
+    assert 0.4 < s.info["gini"] < 0.9
+    tp = W.template(n_req=128)
+    tt = tp.batch.tokens.reshape(128, 512)
+    mask = np.ones(512, bool)
+    for off in W.FIELD_OFFSETS:
+        mask[off:off + 8] = False
+    assert (tt[:, mask] == tt[0, mask]).all()
+    assert (tp.batch.boundary_tok == 96).all()
+    pw = W.probe(n_req=256, n_prior=32, capacity=1 << 12, n_random=100)
+    reuse, src, cut = pw.info["reuse"], pw.info["src"], pw.info["cut"]
+    pt, prt = pw.batch.tokens.reshape(256, 512), pw.prior.tokens.reshape(32, 512)
+    for r in np.nonzero(reuse)[0]:
+        c = 16 * int(cut[r])
+        assert (pt[r, :c] == prt[src[r], :c]).all()
+        assert pw.batch.principal[r] == pw.prior.principal[src[r]]
+    keys = pw.random_keys
+    assert not (np.all(keys[:, :8] == 0, axis=1) | np.all(keys[:, :8] == 255, axis=1)).any()
+    lw = W.make("long", n_req=4)
+    assert lw.batch.tokens.shape[0] == 4 * 32768 and (lw.batch.boundary_tok == 64).all()
+
+
+def test_full_size_shapes():
+    """The full-size definitions (sizes only; generation is cheap except probe)."""
+    assert W.make("wide").batch.n == 131072
+    assert W.make("sysprompt").batch.lengths()[0] == 2119
+
+
+def test_oracle_key_reserved_rule():
+    assert oracle.key_reserved(bytes(32))
+    assert oracle.key_reserved(b"\xff" * 8 + b"\x01" * 24)
+    assert oracle.key_reserved(bytes(8) + b"\x01" * 24)
+    assert not oracle.key_reserved(b"\x01" + bytes(31))
