@@ -39,11 +39,54 @@ UNIT = "block digests/s"
 WORKLOAD = {"workload": "wide: 131072 requests x 128 tokens, BOUNDARY salt at token 64, 4096 principals",
             "requests": 131072, "tokens_per_request": 128, "block": 16, "blocks_per_step": 131072 * 8,
             "principals": 4096, "mode": "BOUNDARY (k=4)"}
-N_SM_NOMINAL = 152
-SM_MAX_MHZ = 2070.0
+SM_MAX_MHZ = 2070.0            # maximum SM clock of a GB300 (profiling recipe)
+INT32_LANES_PER_SM = 64        # 4 SMSPs x 16 lanes of the integer pipe (LOP3/SHF/IMAD microbench: 64.0/clk/SM)
+CHAIN_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_chain.cu", "paper_2608_09225_gb300/csrc/sha256_dev.cuh",
+                 "paper_2608_09225_gb300/csrc/kvgov_internal.cuh", "include/kvgov.h"]
+CHAIN_PROFILE = "profiles/chain_kernel_wide.md"
+
+
+def chain_source_hash() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for rel in CHAIN_SOURCES:
+        with open(os.path.join(HERE, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def profiled_traffic():
+    """DRAM bytes per chain-kernel launch from the committed ncu summary, if
+    that capture was taken of the chain kernel's current sources; else None."""
+    path = os.path.join(HERE, CHAIN_PROFILE)
+    try:
+        text = open(path).read()
+    except OSError:
+        return None, "no profile"
+    vals = dict(line.split(":", 1) for line in text.splitlines() if line.startswith(("traffic_bytes_per_launch:",
+                                                                                       "source_sha256:")))
+    if vals.get("source_sha256:".rstrip(":"), "").strip() != chain_source_hash():
+        return None, f"{CHAIN_PROFILE} was captured from other sources"
+    return int(vals["traffic_bytes_per_launch"].strip()), CHAIN_PROFILE
 
 
 # --------------------------------------------------------------------------- helpers
+def rank_seed(seed: int, rank: int, i: int) -> int:
+    """Seed of batch i on rank `rank`: ranks draw disjoint streams of batches
+    (weak scaling: requests are sharded, nothing is exchanged)."""
+    return seed + 1000003 * rank + i
+
+
+def max_over_ranks(ms: float, world: int, dist, device) -> float:
+    """Slowest rank's time (the whole job finishes when it does)."""
+    if world <= 1:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def nominal_chain_ops(nb: np.ndarray, mode: int, k: np.ndarray | None) -> int:
     """Nominal integer ops of the chain kernel: 1384 per scheduled compression,
     904 per compression whose schedule is a compile-time constant (padding
@@ -125,7 +168,8 @@ class ClockSampler:
 
 
 def measure_int_peak(torch, peak_lib_path):
-    """Thread-ops per SM clock for SHA-256's op mix, from libkvgov_peak."""
+    """Thread-ops per SM clock of LOP3, SHF, IADD3, IMAD and SHA-256 (adds on
+    the ALU / as IMAD), from libkvgov_peak."""
     import ctypes
     L = ctypes.CDLL(peak_lib_path)
     L.kvgov_peak_int.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
@@ -134,7 +178,8 @@ def measure_int_peak(torch, peak_lib_path):
     n_sm = torch.cuda.get_device_properties(0).multi_processor_count
     out = {}
     for kind, name, threads, blocks_per_sm, iters in ((0, "lop3", 256, 8, 4000), (1, "shf", 256, 8, 4000),
-                                                      (2, "iadd3", 256, 8, 4000), (3, "sha256", 256, 4, 200)):
+                                                      (2, "iadd3", 256, 8, 4000), (3, "sha_alu", 256, 4, 200),
+                                                      (4, "sha_fma", 256, 4, 200), (5, "imad", 256, 8, 4000)):
         blocks = n_sm * blocks_per_sm
         sink = torch.zeros(1, dtype=torch.int32, device="cuda")
         clocks = torch.zeros(blocks * 3, dtype=torch.int64, device="cuda")
@@ -254,8 +299,7 @@ def main():
     K.lib()
 
     # ---- inputs: a pool of distinct batches, resident in HBM (weak scaling: per-rank seeds)
-    base = args.seed + 1000003 * rank
-    pool_host = [W.make("wide", seed=base + i) for i in range(args.pool)]
+    pool_host = [W.make("wide", seed=rank_seed(args.seed, rank, i)) for i in range(args.pool)]
     w0 = pool_host[0]
     n_req = w0.batch.n
     n_blocks = int((w0.batch.lengths() // 16).sum())
@@ -287,7 +331,7 @@ def main():
         K.probe(cache.slots, bufs["digests"], bufs["blk_off"], bufs["prefix"], cache.status)
         K.insert(cache.slots, bufs["digests"], cache.status, cache.n_new)
 
-    kernels_per_step = 1 + (1 if n_req <= 4096 else 3) + 1 + 1 + 1
+    kernels_per_step = 5   # salts, block offsets, chain, probe, insert
     for i in range(args.warmup):
         step(pool[i % args.pool])
     torch.cuda.synchronize()
@@ -309,31 +353,33 @@ def main():
     cache.check_status()
     ms = t_start.elapsed_time(t_stop)
     chain_ms = float(np.mean([a.elapsed_time(b) for a, b in chain_ev]))
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, world, dist, "cuda")
     value = world * args.steps * n_blocks / (ms / 1e3)
 
     # ---- end to end through the public API with host buffers
     e2e = e2e_leg(torch, K, W, cache, pool_host[: min(4, args.pool)], args.e2e_steps, bufs, world, dist)
 
-    # ---- roofline of the chain kernel (integer issue bound)
-    peak = measure_int_peak(torch, kbuild.PEAK_LIB)
+    # ---- roofline of the chain kernel (integer-pipe bound)
+    micro = measure_int_peak(torch, kbuild.PEAK_LIB)
     nb = (w0.batch.lengths() // 16)
     ops = nominal_chain_ops(nb, 2, w0.batch.boundary_tok // 16)
     achieved = ops / (chain_ms / 1e3) / 1e12
     clock = clk.summary()
-    peak_ops_clk = peak["sha256"]
-    peak_tops = peak["n_sm"] * peak_ops_clk * SM_MAX_MHZ * 1e6 / 1e12
+    n_sm = micro["n_sm"]
+    peak_tops = n_sm * INT32_LANES_PER_SM * SM_MAX_MHZ * 1e6 / 1e12
+    traffic, traffic_src = profiled_traffic()
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s (int32)",
-                "frac": achieved / peak_tops, "traffic": None,
+                "frac": achieved / peak_tops, "traffic": traffic,
                 "kernel": "chain_kernel<BOUNDARY>", "ops_per_launch": ops, "kernel_ms": chain_ms,
-                "peak_basis": f"{peak['n_sm']} SMs x {peak_ops_clk:.1f} SHA-256 thread-ops/clk/SM "
-                              f"(measured, libkvgov_peak) x {SM_MAX_MHZ:.0f} MHz",
-                "int_ops_per_clk_per_sm": {k: round(v, 2) for k, v in peak.items() if k != "n_sm"}}
+                "algorithmic_bytes_per_launch": 96 * n_blocks,
+                "peak_basis": f"{n_sm} SMs x 4 SMSPs x 16 int32 lanes x {SM_MAX_MHZ:.0f} MHz; every SHF, LOP3, "
+                              f"IADD3 and IMAD of SHA-256 issues to that one 16-lane pipe per SMSP",
+                "int_ops_per_clk_per_sm_measured": {k: round(v, 2) for k, v in micro.items() if k != "n_sm"},
+                "frac_of_sha256_microbench": achieved / (n_sm * micro["sha_alu"] * SM_MAX_MHZ * 1e6 / 1e12),
+                "frac_of_issue_peak": achieved / (n_sm * 128 * SM_MAX_MHZ * 1e6 / 1e12),
+                "traffic_source": traffic_src}
     if clock.get("sm_mhz"):
-        roofline["frac_at_run_clock"] = achieved / (peak["n_sm"] * peak_ops_clk * clock["sm_mhz"] * 1e6 / 1e12)
+        roofline["frac_at_run_clock"] = achieved / (n_sm * INT32_LANES_PER_SM * clock["sm_mhz"] * 1e6 / 1e12)
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
@@ -417,11 +463,7 @@ def e2e_leg(torch, K, W, cache, hosts, steps, bufs, world, dist):
         one(i)
     b.record()
     torch.cuda.synchronize()
-    ms = a.elapsed_time(b)
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(a.elapsed_time(b), world, dist, "cuda")
     return {"value": world * steps * n_blocks / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps}
 

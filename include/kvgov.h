@@ -182,7 +182,8 @@ int kvgov_insert(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_keys, int
  *   d_digests       [d_blk_off[n_req]][32] u8 (kvgov_chain_hash output).
  *   d_blk_off       [n_req + 1] int64.
  *   d_prefix_blocks [n_req] int32 output.
- *   d_status        nullable; KVGOV_F_BADINDEX for decreasing d_blk_off.
+ *   d_status        nullable; KVGOV_F_BADINDEX for a request whose rows are
+ *                   not inside [d_blk_off[r], d_blk_off[n_req]) (it gets 0).
  * n_req = 0 is a no-op.  EINVAL: bad capacity, NULL or misaligned pointer.
  */
 int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,

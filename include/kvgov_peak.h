@@ -21,7 +21,8 @@ typedef struct CUstream_st *kvgov_stream_t;
 /*
  * kvgov_peak_int -- launch `blocks` CTAs of `threads` threads, each running
  * `iters` iterations of the instruction body of `kind`:
- *   0 LOP3, 1 SHF (funnel shift), 2 IADD3, 3 SHA-256 compression (FIPS 180-4).
+ *   0 LOP3, 1 SHF (funnel shift), 2 IADD3, 3 SHA-256 compression (FIPS 180-4)
+ *   with ALU adds, 4 the same with every add as IMAD (FMA pipe), 5 IMAD.
  * d_clocks [blocks][3] u64 receives, per CTA, its SM id and its clock64()
  * at start and end.  d_sink [1] u32 is written only in a case that never
  * happens (keeps results live).  Asynchronous on `stream`.
@@ -31,7 +32,8 @@ int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint32_t *d_sin
                    unsigned long long *d_clocks, kvgov_stream_t stream);
 
 /* Thread-operations one thread executes per iteration of `kind` (nominal
- * SHA-256 count of 1384 per compression for kind 3), or 0 for a bad kind. */
+ * SHA-256 count of 1384 per compression for kinds 3 and 4), or 0 for a bad
+ * kind. */
 int kvgov_peak_ops_per_iter(int kind);
 
 #ifdef __cplusplus

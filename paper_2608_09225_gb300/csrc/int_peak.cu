@@ -12,7 +12,10 @@
 //   1  SHF    x_s = shf.r.wrap(x_s, x_{s+1}, n_s)   over 8 streams
 //   2  IADD3  x_s = x_s + x_{s+1} + x_{s+2}         over 8 streams
 //   3  SHA-256: one FIPS 180-4 compression (1384 nominal ops: 64 rounds x 14
-//      + 48 schedule words x 10 + 8) on each of 2 independent chains
+//      + 48 schedule words x 10 + 8) on each of 2 independent chains, adds on
+//      the ALU pipe
+//   4  the same with every add issued as IMAD on the FMA pipe
+//   5  IMAD  x_s = x_s * one + x_{s+1}   (one = 1 at run time)
 // Each update reads two other streams' latest values, so no chain of updates
 // collapses into fewer instructions (a three-input boolean of three fixed
 // inputs would fold into one LOP3; these never have three fixed inputs).
@@ -34,7 +37,7 @@ __device__ __forceinline__ uint32_t smid() {
 }
 
 template <int KIND>
-__global__ void peak_kernel(int iters, uint32_t seed, uint32_t *sink, unsigned long long *clocks) {
+__global__ void peak_kernel(int iters, uint32_t seed, uint32_t one, uint32_t *sink, unsigned long long *clocks) {
     __shared__ unsigned long long t_start;
     uint32_t x[kStreams];
 #pragma unroll
@@ -42,7 +45,7 @@ __global__ void peak_kernel(int iters, uint32_t seed, uint32_t *sink, unsigned l
     __syncthreads();
     if (threadIdx.x == 0) t_start = clock64();
     __syncthreads();
-    if (KIND == 3) {
+    if (KIND == 3 || KIND == 4) {
         uint32_t st[kShaChains][8], w[kShaChains][16];
 #pragma unroll
         for (int c = 0; c < kShaChains; ++c) {
@@ -54,7 +57,8 @@ __global__ void peak_kernel(int iters, uint32_t seed, uint32_t *sink, unsigned l
             for (int c = 0; c < kShaChains; ++c) {
 #pragma unroll
                 for (int i = 0; i < 16; ++i) w[c][i] = st[c][i & 7] ^ (uint32_t)i;
-                kvgov_dev::sha_compress(st[c], w[c]);
+                if (KIND == 3) kvgov_dev::sha_compress(st[c], w[c], kvgov_dev::AddAlu{});
+                else kvgov_dev::sha_compress(st[c], w[c], kvgov_dev::AddFma{one});
             }
         }
 #pragma unroll
@@ -70,8 +74,10 @@ __global__ void peak_kernel(int iters, uint32_t seed, uint32_t *sink, unsigned l
                         asm("lop3.b32 %0, %0, %1, %2, 0x96;" : "+r"(x[s]) : "r"(a), "r"(b));
                     else if (KIND == 1)
                         x[s] = __funnelshift_r(x[s], a, (s * 5 + rep * 3 + 1) & 31);
-                    else
+                    else if (KIND == 2)
                         x[s] = x[s] + a + b;
+                    else
+                        asm("mad.lo.u32 %0, %0, %1, %2;" : "+r"(x[s]) : "r"(one), "r"(a));
                 }
             }
         }
@@ -95,22 +101,25 @@ extern "C" int kvgov_peak_ops_per_iter(int kind) {
     switch (kind) {
     case 0: case 1: return 4 * kStreams;   // one instruction per update; IADD3 counts as one op
     case 2: return 4 * kStreams;
-    case 3: return kShaChains * 1384;
+    case 3: case 4: return kShaChains * 1384;
+    case 5: return 4 * kStreams;
     default: return 0;
     }
 }
 
 extern "C" int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint32_t *d_sink,
                               unsigned long long *d_clocks, kvgov_stream_t stream) {
-    if (kind < 0 || kind > 3 || iters <= 0 || blocks <= 0 || threads <= 0 || threads > 1024 || !d_sink ||
+    if (kind < 0 || kind > 5 || iters <= 0 || blocks <= 0 || threads <= 0 || threads > 1024 || !d_sink ||
         !d_clocks)
         return 1;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     switch (kind) {
-    case 0: peak_kernel<0><<<blocks, threads, 0, s>>>(iters, 1u, d_sink, d_clocks); break;
-    case 1: peak_kernel<1><<<blocks, threads, 0, s>>>(iters, 1u, d_sink, d_clocks); break;
-    case 2: peak_kernel<2><<<blocks, threads, 0, s>>>(iters, 1u, d_sink, d_clocks); break;
-    default: peak_kernel<3><<<blocks, threads, 0, s>>>(iters, 1u, d_sink, d_clocks); break;
+    case 0: peak_kernel<0><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 1: peak_kernel<1><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 2: peak_kernel<2><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 3: peak_kernel<3><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 4: peak_kernel<4><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    default: peak_kernel<5><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
     }
     return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }

@@ -15,6 +15,8 @@
 // then reads its 16 tokens from shared memory, byte-swaps them into
 // big-endian SHA words and runs the 2 (or 3) compressions of its message in
 // registers.
+#include <cooperative_groups.h>
+
 #include "kvgov_internal.cuh"
 #include "sha256_dev.cuh"
 
@@ -23,16 +25,19 @@ namespace {
 using namespace kvgov_dev;
 
 // ---------------------------------------------------------------------------
-// Block offsets: exclusive scan of floor(len_r / 16), three small kernels
-// (tile scan, scan of tile totals, add tile bases).
+// Block offsets: exclusive scan of floor(len_r / 16) in one cooperative
+// launch.  CTA c owns a contiguous range of requests.  Phase 1: each CTA sums
+// its range and posts the total at the position of its last request (a slot
+// it alone will overwrite later).  Grid sync.  Phase 2: each CTA adds the
+// totals posted by the CTAs before it.  Grid sync (every total has been read).
+// Phase 3: each CTA rescans its range and writes base + running count.
 // ---------------------------------------------------------------------------
 
 constexpr int kScanThreads = 1024;
-constexpr int kScanItems = 4;
-constexpr int kScanTile = kScanThreads * kScanItems;
 
-// Inclusive scan of one value per thread across a 1024-thread CTA.
-__device__ __forceinline__ long long cta_inclusive_scan(long long v, long long *warp_sums) {
+// Inclusive scan of one value per thread across a 1024-thread CTA; also
+// returns the CTA total through *total.
+__device__ __forceinline__ long long cta_inclusive_scan(long long v, long long *warp_sums, long long *total) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
     for (int d = 1; d < 32; d <<= 1) {
@@ -52,77 +57,91 @@ __device__ __forceinline__ long long cta_inclusive_scan(long long v, long long *
     }
     __syncthreads();
     if (warp > 0) v += warp_sums[warp - 1];
+    *total = warp_sums[31];
+    __syncthreads();   // warp_sums is reused by the next call
     return v;
 }
 
-// Tile c covers requests [c*T, min((c+1)*T, n)).  Writes the tile-local
-// inclusive counts to blk_off[r+1]; blk_off[0] = 0.
-__global__ void __launch_bounds__(kScanThreads) blkoff_tile_kernel(const int64_t *__restrict__ tok_off, int32_t n,
-                                                                   int64_t *__restrict__ blk_off, uint32_t *status) {
+__device__ __forceinline__ long long blocks_of(const int64_t *tok_off, long long r, bool *bad) {
+    const long long len = tok_off[r + 1] - tok_off[r];
+    if (len < 0) { *bad = true; return 0; }
+    return len / KVGOV_BLOCK;
+}
+
+__global__ void __launch_bounds__(kScanThreads) blkoff_kernel(const int64_t *__restrict__ tok_off, int32_t n,
+                                                              int64_t *blk_off, uint32_t *status, long long per_cta) {
     __shared__ long long warp_sums[32];
-    const long long base = (long long)blockIdx.x * kScanTile + (long long)threadIdx.x * kScanItems;
-    long long cnt[kScanItems];
-    long long sum = 0;
+    __shared__ long long s_base;
+    namespace cg = cooperative_groups;
+    cg::grid_group grid = cg::this_grid();
+    const long long lo = (long long)blockIdx.x * per_cta;
+    const long long hi = lo + per_cta < n ? lo + per_cta : (long long)n;
     bool bad = false;
-#pragma unroll
-    for (int q = 0; q < kScanItems; ++q) {
-        const long long r = base + q;
-        cnt[q] = 0;
-        if (r < n) {
-            const long long len = tok_off[r + 1] - tok_off[r];
-            if (len < 0) bad = true;
-            else cnt[q] = len / KVGOV_BLOCK;
-        }
-        sum += cnt[q];
-    }
+
+    // phase 1: this CTA's total, posted at blk_off[hi]
+    long long part = 0;
+    for (long long r = lo + threadIdx.x; r < hi; r += kScanThreads) part += blocks_of(tok_off, r, &bad);
+    long long total;
+    cta_inclusive_scan(part, warp_sums, &total);
+    if (threadIdx.x == 0 && hi > lo) blk_off[hi] = total;
     if (bad) raise_flag(status, KVGOV_F_BADINDEX);
-    long long run = cta_inclusive_scan(sum, warp_sums) - sum;
-#pragma unroll
-    for (int q = 0; q < kScanItems; ++q) {
-        const long long r = base + q;
-        run += cnt[q];
-        if (r < n) blk_off[r + 1] = run;
+    grid.sync();
+
+    // phase 2: base = totals of the CTAs before this one
+    long long v = 0;
+    for (long long c = threadIdx.x; c < blockIdx.x; c += kScanThreads) {
+        const long long clo = c * per_cta, chi = clo + per_cta < n ? clo + per_cta : (long long)n;
+        if (chi > clo) v += blk_off[chi];
     }
+    long long base;
+    cta_inclusive_scan(v, warp_sums, &base);
+    grid.sync();
+
+    // phase 3: rescan the range and write the final prefix sums
     if (blockIdx.x == 0 && threadIdx.x == 0) blk_off[0] = 0;
-}
-
-// One CTA: turn the tile totals at positions min((c+1)*T, n) into global
-// inclusive prefixes.
-__global__ void __launch_bounds__(kScanThreads) blkoff_carry_kernel(int32_t n, int64_t *__restrict__ blk_off) {
-    __shared__ long long warp_sums[32];
-    const long long n_tiles = ((long long)n + kScanTile - 1) / kScanTile;
-    long long carry = 0;
-    for (long long c0 = 0; c0 < n_tiles; c0 += kScanThreads) {
-        const long long c = c0 + threadIdx.x;
-        long long end = 0, v = 0;
-        if (c < n_tiles) {
-            end = (c + 1) * kScanTile;
-            if (end > n) end = n;
-            v = blk_off[end];
-        }
-        const long long inc = cta_inclusive_scan(v, warp_sums);
-        const long long total = warp_sums[31];
-        if (c < n_tiles) blk_off[end] = carry + inc;
-        carry += total;
-        __syncthreads();   // warp_sums is rewritten by the next round
+    if (threadIdx.x == 0) s_base = base;
+    __syncthreads();
+    long long carry = s_base;
+    for (long long r0 = lo; r0 < hi; r0 += kScanThreads) {
+        const long long r = r0 + threadIdx.x;
+        bool ignored = false;
+        const long long cnt = r < hi ? blocks_of(tok_off, r, &ignored) : 0;
+        long long chunk;
+        const long long inc = cta_inclusive_scan(cnt, warp_sums, &chunk);
+        if (r < hi) blk_off[r + 1] = carry + inc;
+        carry += chunk;
     }
 }
 
-// Add the global base of tile c (now at blk_off[c*T]) to the tile's interior.
-__global__ void __launch_bounds__(kScanThreads) blkoff_add_kernel(int32_t n, int64_t *__restrict__ blk_off) {
-    const long long c = blockIdx.x + 1;
-    const long long lo = c * kScanTile;
-    long long hi = lo + kScanTile;
-    if (hi > n) hi = n;
-    const long long add = blk_off[lo];
-    for (long long p = lo + 1 + threadIdx.x; p < hi; p += kScanThreads) blk_off[p] += add;
+struct DeviceInfo {
+    int sms = 0, coop_blocks_per_sm = 0;
+};
+
+// SM count and cooperative residency of blkoff_kernel on the current device,
+// looked up once per device.
+DeviceInfo device_info() {
+    static DeviceInfo cache[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return DeviceInfo{};
+    DeviceInfo &d = cache[dev];
+    if (d.sms == 0) {
+        int sms = 0, per = 0;
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, blkoff_kernel, kScanThreads, 0);
+        d.coop_blocks_per_sm = per;
+        d.sms = sms;
+    }
+    return d;
 }
 
 // ---------------------------------------------------------------------------
 // Chain kernel
 // ---------------------------------------------------------------------------
 
-constexpr int kR = 128;           // requests (threads) per CTA
+#ifndef KVGOV_CHAIN_R
+#define KVGOV_CHAIN_R 128
+#endif
+constexpr int kR = KVGOV_CHAIN_R;   // requests (threads) per CTA
 constexpr int kStages = 2;        // shared-memory buffers for token blocks
 constexpr int kChunks = 5;        // 16-byte chunks that can cover one 64-byte block
 constexpr int kSlotWords = kChunks * 4;
@@ -138,7 +157,15 @@ struct ChainParams {
     uint32_t *status;
     int32_t n_req;
     int32_t n_principals;
+    uint32_t one;   // 1, opaque to the compiler (see AddFma)
 };
+
+// Which adder the SHA-256 rounds use.  Measured on GB300: IMAD shares the
+// integer pipe with SHF/LOP3/IADD3 (libkvgov_peak kinds 3-5), so AddFma
+// only adds instructions; plain adds are the default.
+#ifndef KVGOV_FMA_ADDS
+#define KVGOV_FMA_ADDS 0
+#endif
 
 // Big-endian words of principal pi's 32-byte salt.
 __device__ __forceinline__ void load_salt(const uint8_t *salts, int pi, uint32_t sw[8]) {
@@ -213,6 +240,11 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
         cp_async_commit();
     }
 
+#if KVGOV_FMA_ADDS
+    const AddFma add{p.one};
+#else
+    const AddAlu add{};
+#endif
     const int sh = (int)(t0 & 3);   // word offset of the block inside its first chunk
     uint32_t h[8];
 #pragma unroll
@@ -232,8 +264,8 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
             for (int i = 0; i < 16; ++i) tw[i] = bswap32(src[i]);
 
             if (MODE == KVGOV_UNSALTED) {
-                if (j == 0) sha256_msg64(tw, h);
-                else sha256_msg96(h, tw, h);
+                if (j == 0) sha256_msg64(tw, h, add);
+                else sha256_msg96(h, tw, h, add);
             } else if (MODE == KVGOV_ROOT) {
                 uint32_t pw[8];
                 if (j == 0) load_salt(p.salts, pi, pw);
@@ -241,14 +273,14 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
 #pragma unroll
                     for (int i = 0; i < 8; ++i) pw[i] = h[i];
                 }
-                sha256_msg96(pw, tw, h);
+                sha256_msg96(pw, tw, h, add);
             } else {
                 if (j == k && j > 0) {
                     uint32_t sw[8];
                     load_salt(p.salts, pi, sw);
-                    sha256_msg128(sw, h, tw, h);
+                    sha256_msg128(sw, h, tw, h, add);
                 } else if (j == 0 && k != 0) {
-                    sha256_msg64(tw, h);
+                    sha256_msg64(tw, h, add);
                 } else {
                     uint32_t pw[8];
                     if (j == k) load_salt(p.salts, pi, pw);
@@ -256,7 +288,7 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
 #pragma unroll
                         for (int i = 0; i < 8; ++i) pw[i] = h[i];
                     }
-                    sha256_msg96(pw, tw, h);
+                    sha256_msg96(pw, tw, h, add);
                 }
             }
 
@@ -274,13 +306,22 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
 extern "C" int kvgov_block_offsets(const int64_t *d_tok_off, int32_t n_req, int64_t *d_blk_off,
                                    uint32_t *d_status, kvgov_stream_t stream) {
     if (n_req < 0 || !d_tok_off || !d_blk_off) return KVGOV_EINVAL;
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    const long long n_tiles = n_req == 0 ? 1 : ((long long)n_req + kScanTile - 1) / kScanTile;
-    blkoff_tile_kernel<<<(unsigned)n_tiles, kScanThreads, 0, s>>>(d_tok_off, n_req, d_blk_off, d_status);
-    if (n_tiles > 1) {
-        blkoff_carry_kernel<<<1, kScanThreads, 0, s>>>(n_req, d_blk_off);
-        blkoff_add_kernel<<<(unsigned)(n_tiles - 1), kScanThreads, 0, s>>>(n_req, d_blk_off);
-    }
+    const DeviceInfo d = device_info();
+    if (d.sms <= 0 || d.coop_blocks_per_sm <= 0) return KVGOV_ECUDA;
+    long long grid = ((long long)n_req + kScanThreads - 1) / kScanThreads;
+    const long long max_grid = (long long)d.sms * d.coop_blocks_per_sm;
+    if (grid > max_grid) grid = max_grid;
+    if (grid < 1) grid = 1;
+    long long per_cta = ((long long)n_req + grid - 1) / grid;
+    if (per_cta < 1) per_cta = 1;
+    const int64_t *tok_off = d_tok_off;
+    int64_t *blk_off = d_blk_off;
+    uint32_t *status = d_status;
+    int32_t n = n_req;
+    void *args[] = {(void *)&tok_off, (void *)&n, (void *)&blk_off, (void *)&status, (void *)&per_cta};
+    if (cudaLaunchCooperativeKernel((const void *)blkoff_kernel, dim3((unsigned)grid), dim3(kScanThreads), args, 0,
+                                    reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return KVGOV_ECUDA;
     return kvgov_host::launch_status();
 }
 
@@ -301,7 +342,7 @@ extern "C" int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t
     ChainParams p;
     p.tokens = d_tokens; p.tok_off = d_tok_off; p.principal = d_principal; p.salts = d_salts;
     p.boundary_tok = d_boundary_tok; p.blk_off = d_blk_off; p.digests = d_digests; p.status = d_status;
-    p.n_req = n_req; p.n_principals = n_principals;
+    p.n_req = n_req; p.n_principals = n_principals; p.one = 1u;
     const unsigned grid = (unsigned)(((long long)n_req + kR - 1) / kR);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     switch (mode) {

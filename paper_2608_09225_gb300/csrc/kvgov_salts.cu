@@ -15,7 +15,7 @@ namespace {
 
 using namespace kvgov_dev;
 
-constexpr int kSaltThreads = 128;
+constexpr int kSaltThreads = 64;
 
 struct SaltParams {
     uint8_t secret[KVGOV_MAX_SECRET];
@@ -51,7 +51,7 @@ __device__ void sha_absorb_finish(uint32_t s[8], unsigned long long prior, unsig
             w[14] = (uint32_t)(total_bits >> 32);
             w[15] = (uint32_t)total_bits;
         }
-        sha_compress(s, w);
+        sha_compress_small(s, w);
     }
 }
 
@@ -75,11 +75,11 @@ __global__ void __launch_bounds__(kSaltThreads) salts_kernel(const SaltParams p)
         sha_iv(si);
 #pragma unroll
         for (int i = 0; i < 16; ++i) w[i] = k0[i] ^ 0x36363636u;
-        sha_compress(si, w);
+        sha_compress_small(si, w);
         sha_iv(so);
 #pragma unroll
         for (int i = 0; i < 16; ++i) w[i] = k0[i] ^ 0x5c5c5c5cu;
-        sha_compress(so, w);
+        sha_compress_small(so, w);
 #pragma unroll
         for (int i = 0; i < 8; ++i) { s_ipad[i] = si[i]; s_opad[i] = so[i]; }
     }
@@ -106,7 +106,7 @@ __global__ void __launch_bounds__(kSaltThreads) salts_kernel(const SaltParams p)
 #pragma unroll
         for (int i = 9; i < 15; ++i) w[i] = 0u;
         w[15] = (64u + 32u) * 8u;
-        sha_compress(s, w);
+        sha_compress_small(s, w);
 
         uint4 *dst = reinterpret_cast<uint4 *>(p.salts + 32ll * pr);
         dst[0] = make_uint4(bswap32(s[0]), bswap32(s[1]), bswap32(s[2]), bswap32(s[3]));
@@ -128,7 +128,7 @@ extern "C" int kvgov_derive_salts(const uint8_t *secret, size_t secret_len, cons
     p.ids = d_ids; p.id_off = d_id_off; p.salts = d_salts; p.status = d_status;
     p.secret_len = (uint32_t)secret_len; p.n = n_principals;
     long long grid = ((long long)n_principals + kSaltThreads - 1) / kSaltThreads;
-    if (grid > 1024) grid = 1024;
+    if (grid > 4096) grid = 4096;
     salts_kernel<<<(unsigned)grid, kSaltThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(p);
     return kvgov_host::launch_status();
 }

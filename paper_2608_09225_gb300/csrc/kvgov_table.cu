@@ -21,11 +21,12 @@
 // duplicate, done; different = keep probing).  Two inserts of one key in one
 // batch therefore store it once.
 //
-// Probe: G lanes of a warp serve one request.  The lanes look up a window of
+// Probe: G lanes of a warp serve one request.  The lanes look up the next G
 // consecutive blocks in parallel; a ballot over the window's misses gives the
-// first miss (the prefix length) and ends the request.  The window starts at
-// one block and doubles up to G, so a request that misses at block 0 costs a
-// single lookup and a long hit run costs O(log) rounds.
+// first miss (the prefix length) and ends the request, else the window moves
+// on.  A request of n_b blocks takes ceil((L+1)/G) rounds of two dependent
+// memory accesses (digest, slot); lookups past the first miss inside the last
+// window are wasted, which costs bandwidth but not latency.
 #include <atomic>
 
 #include "kvgov_internal.cuh"
@@ -46,6 +47,11 @@ __device__ __forceinline__ unsigned long long ld_acquire(const unsigned long lon
 __device__ __forceinline__ unsigned long long ld_relaxed(const unsigned long long *p) {
     unsigned long long v;
     asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];\n" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ ulonglong2 ld_relaxed2(const unsigned long long *p) {
+    ulonglong2 v;
+    asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];\n" : "=l"(v.x), "=l"(v.y) : "l"(p) : "memory");
     return v;
 }
 __device__ __forceinline__ void st_relaxed(unsigned long long *p, unsigned long long v) {
@@ -76,7 +82,12 @@ __device__ InsertResult insert_one(unsigned long long *slots, unsigned long long
     unsigned long long pos = k[0] & mask;
     for (unsigned long long n = 0; n <= mask; ++n, pos = (pos + 1) & mask) {
         unsigned long long *slot = slots + 4 * pos;
-        unsigned long long w0 = ld_acquire(slot);
+        // One 32-byte look at the slot.  A slot is written once (claim, tail,
+        // publish) and never changes afterwards, so a full match on these
+        // unordered reads can only be the key itself: a duplicate.
+        const ulonglong2 lo = ld_relaxed2(slot), hi = ld_relaxed2(slot + 2);
+        unsigned long long w0 = lo.x;
+        if (w0 == k[0] && lo.y == k[1] && hi.x == k[2] && hi.y == k[3]) return kDuplicate;
         if (w0 == 0ull) {
             const unsigned long long old = atomicCAS(slot, 0ull, kClaimed);
             if (old == 0ull) {
@@ -88,15 +99,20 @@ __device__ InsertResult insert_one(unsigned long long *slots, unsigned long long
             }
             w0 = old;
         }
-        if (w0 == kClaimed) {
+        if (w0 == kClaimed || w0 == k[0]) {
+            // claimed but not yet published, or our first word with a tail
+            // that may have been read before it was written: wait for the
+            // publication (bounded) and compare again with acquire ordering
             uint32_t spins = 0;
             while ((w0 = ld_acquire(slot)) == kClaimed) {
                 if (++spins >= spin_limit) return kTimeout;
                 __nanosleep(100);
             }
+            if (w0 == k[0]) {
+                const ulonglong2 t = ld_relaxed2(slot + 2);
+                if (ld_relaxed(slot + 1) == k[1] && t.x == k[2] && t.y == k[3]) return kDuplicate;
+            }
         }
-        if (w0 == k[0] && ld_relaxed(slot + 1) == k[1] && ld_relaxed(slot + 2) == k[2] && ld_relaxed(slot + 3) == k[3])
-            return kDuplicate;
     }
     return kFull;
 }
@@ -106,13 +122,11 @@ __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long lo
                                                                 const uint4 *__restrict__ keys, long long n_keys,
                                                                 unsigned long long *n_new, uint32_t *status,
                                                                 uint32_t spin_limit) {
-    __shared__ unsigned int s_new;
-    __shared__ uint32_t s_flags;
-    if (threadIdx.x == 0) { s_new = 0; s_flags = 0; }
+    __shared__ unsigned int s_new, s_flags, s_done;
+    if (threadIdx.x == 0) { s_new = 0; s_flags = 0; s_done = 0; }
     __syncthreads();
     const long long stride = (long long)gridDim.x * kInsertThreads;
-    unsigned int my_new = 0;
-    uint32_t my_flags = 0;
+    unsigned int my_new = 0, my_flags = 0;
     for (long long i = (long long)blockIdx.x * kInsertThreads + threadIdx.x; i < n_keys; i += stride) {
         const uint4 a = __ldg(keys + 2 * i), b = __ldg(keys + 2 * i + 1);
         const unsigned long long k[4] = {u64_of(a.x, a.y), u64_of(a.z, a.w), u64_of(b.x, b.y), u64_of(b.z, b.w)};
@@ -127,12 +141,19 @@ __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long lo
         default: my_flags |= KVGOV_F_TIMEOUT; break;
         }
     }
-    if (my_new) atomicAdd(&s_new, my_new);
-    if (my_flags) atomicOr(&s_flags, my_flags);
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        if (s_new && n_new) atomicAdd(n_new, (unsigned long long)s_new);
-        if (s_flags) atomicOr(status, s_flags);
+    // Counts: warp reduction, shared-memory accumulation, and the CTA's last
+    // warp to finish publishes them (no barrier: early warps just exit).
+    const unsigned w_new = __reduce_add_sync(0xffffffffu, my_new);
+    const unsigned w_flags = __reduce_or_sync(0xffffffffu, my_flags);
+    if ((threadIdx.x & 31) == 0) {
+        if (w_new) atomicAdd(&s_new, w_new);
+        if (w_flags) atomicOr(&s_flags, w_flags);
+        __threadfence_block();
+        if (atomicAdd(&s_done, 1u) == kInsertThreads / 32 - 1) {
+            const unsigned t_new = atomicAdd(&s_new, 0u), t_flags = atomicOr(&s_flags, 0u);
+            if (t_new && n_new) atomicAdd(n_new, (unsigned long long)t_new);
+            if (t_flags) atomicOr(status, t_flags);
+        }
     }
 }
 
@@ -174,14 +195,14 @@ __global__ void __launch_bounds__(kProbeThreads) probe_kernel(const uint4 *__res
         if (r < n_req) {
             base = blk_off[r];
             nb = blk_off[r + 1] - base;
-            if (nb < 0 || base < 0) {
+            if (nb < 0 || base < 0 || base + nb > blk_off[n_req]) {
                 if (sl == 0) raise_flag(status, KVGOV_F_BADINDEX);
                 nb = 0;
             }
             active = nb > 0;
         }
         long long L = 0;
-        int win = 1;
+        const int win = G;
         while (__any_sync(0xffffffffu, active)) {
             const long long j = L + sl;
             const bool mine = active && sl < win && j < nb;
@@ -198,7 +219,6 @@ __global__ void __launch_bounds__(kProbeThreads) probe_kernel(const uint4 *__res
                 } else {
                     L += (nb - L < win) ? (nb - L) : win;
                     if (L >= nb) active = false;
-                    win = win * 2 < G ? win * 2 : G;
                 }
             }
         }

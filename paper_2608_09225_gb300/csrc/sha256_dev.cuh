@@ -83,23 +83,128 @@ __device__ __forceinline__ uint32_t ssig1(uint32_t x) { return xor3(rotr(x, 17),
 // Big-endian word from 4 little-endian-loaded bytes, and back.
 __device__ __forceinline__ uint32_t bswap32(uint32_t x) { return __byte_perm(x, 0u, 0x0123u); }
 
+// Adders.  Every 32-bit add of the compression goes through one of these.
+// AddAlu is a plain add (the compiler emits IADD3 on the integer ALU pipe,
+// the pipe that also carries every SHF and LOP3).  AddFma issues the add as
+// IMAD a * one + b on the FMA pipe, which SHA-256 otherwise leaves idle;
+// `one` is a runtime 1 from the launch parameters, so the compiler cannot
+// turn the multiply-add back into an ALU add.
+struct AddAlu {
+    __device__ __forceinline__ uint32_t operator()(uint32_t a, uint32_t b) const { return a + b; }
+};
+struct AddFma {
+    uint32_t one;
+    __device__ __forceinline__ uint32_t operator()(uint32_t a, uint32_t b) const {
+        uint32_t r;
+        asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(one), "r"(b));
+        return r;
+    }
+};
+
 // One compression (FIPS 180-4 section 6.2.2, steps 1-4) of the 512-bit block
 // w[0..15] (big-endian words) into the chaining state s.  w is overwritten by
-// the message schedule.
-__device__ __forceinline__ void sha_compress(uint32_t s[8], uint32_t w[16]) {
+// the message schedule.  CONST_W: w is a compile-time constant (a padding
+// block), so its schedule and K_t + W_t are computed with plain operations
+// and fold to immediates.  FROM_IV: s is the initial hash value, so round 0
+// (all state words constant) also folds.
+template <bool CONST_W, bool FROM_IV, class Add>
+__device__ __forceinline__ void sha_compress_t(uint32_t s[8], uint32_t w[16], Add add) {
     uint32_t a = s[0], b = s[1], c = s[2], d = s[3];
     uint32_t e = s[4], f = s[5], g = s[6], h = s[7];
 #pragma unroll
     for (int t = 0; t < 64; ++t) {
-        if (t >= 16)
-            w[t & 15] += ssig1(w[(t - 2) & 15]) + w[(t - 7) & 15] + ssig0(w[(t - 15) & 15]);
-        const uint32_t t1 = h + (sha_k(t) + w[t & 15]) + ch(e, f, g) + bsig1(e);
-        const uint32_t t2 = bsig0(a) + maj(a, b, c);
-        h = g; g = f; f = e; e = d + t1;
-        d = c; c = b; b = a; a = t1 + t2;
+        const int i = t & 15;
+        if (t >= 16) {
+            if (CONST_W)
+                w[i] += ssig1(w[(t - 2) & 15]) + w[(t - 7) & 15] + ssig0(w[(t - 15) & 15]);
+            else
+                w[i] = add(add(w[i], w[(t - 7) & 15]), add(ssig0(w[(t - 15) & 15]), ssig1(w[(t - 2) & 15])));
+        }
+        uint32_t t1, t2;
+        if (FROM_IV && t == 0) {            // every state word is a constant
+            t1 = h + sha_k(0) + ch(e, f, g) + bsig1(e) + w[0];
+            t2 = bsig0(a) + maj(a, b, c);
+            h = g; g = f; f = e; e = d + t1;
+            d = c; c = b; b = a; a = t1 + t2;
+            continue;
+        }
+        const uint32_t kw = CONST_W ? sha_k(t) + w[i] : add(w[i], sha_k(t));
+        t1 = add(add(add(h, kw), ch(e, f, g)), bsig1(e));
+        t2 = add(bsig0(a), maj(a, b, c));
+        h = g; g = f; f = e; e = add(d, t1);
+        d = c; c = b; b = a; a = add(t1, t2);
     }
-    s[0] += a; s[1] += b; s[2] += c; s[3] += d;
-    s[4] += e; s[5] += f; s[6] += g; s[7] += h;
+    s[0] = add(s[0], a); s[1] = add(s[1], b); s[2] = add(s[2], c); s[3] = add(s[3], d);
+    s[4] = add(s[4], e); s[5] = add(s[5], f); s[6] = add(s[6], g); s[7] = add(s[7], h);
+}
+
+template <class Add = AddAlu>
+__device__ __forceinline__ void sha_compress(uint32_t s[8], uint32_t w[16], Add add = Add()) {
+    sha_compress_t<false, false>(s, w, add);
+}
+
+// FIPS 180-4 K_t in constant memory, for the compact compression below.
+static __constant__ uint32_t c_sha_k[64] = {
+    0x428a2f98u, 0x71374491u, 0xb5c0fbcfu, 0xe9b5dba5u, 0x3956c25bu, 0x59f111f1u, 0x923f82a4u, 0xab1c5ed5u,
+    0xd807aa98u, 0x12835b01u, 0x243185beu, 0x550c7dc3u, 0x72be5d74u, 0x80deb1feu, 0x9bdc06a7u, 0xc19bf174u,
+    0xe49b69c1u, 0xefbe4786u, 0x0fc19dc6u, 0x240ca1ccu, 0x2de92c6fu, 0x4a7484aau, 0x5cb0a9dcu, 0x76f988dau,
+    0x983e5152u, 0xa831c66du, 0xb00327c8u, 0xbf597fc7u, 0xc6e00bf3u, 0xd5a79147u, 0x06ca6351u, 0x14292967u,
+    0x27b70a85u, 0x2e1b2138u, 0x4d2c6dfcu, 0x53380d13u, 0x650a7354u, 0x766a0abbu, 0x81c2c92eu, 0x92722c85u,
+    0xa2bfe8a1u, 0xa81a664bu, 0xc24b8b70u, 0xc76c51a3u, 0xd192e819u, 0xd6990624u, 0xf40e3585u, 0x106aa070u,
+    0x19a4c116u, 0x1e376c08u, 0x2748774cu, 0x34b0bcb5u, 0x391c0cb3u, 0x4ed8aa4au, 0x5b9cca4fu, 0x682e6ff3u,
+    0x748f82eeu, 0x78a5636fu, 0x84c87814u, 0x8cc70208u, 0x90befffau, 0xa4506cebu, 0xbef9a3f7u, 0xc67178f2u};
+
+// The same compression with a small instruction footprint: rounds 0-15 are
+// unrolled, rounds 16-63 run as three passes of one unrolled 16-round body
+// (after 16 rounds the eight working variables are back in their original
+// roles, so the loop carries them without moves), with K_t read from
+// constant memory.  About a quarter of the code of sha_compress, for kernels
+// whose time goes to instruction fetch rather than to the integer pipe.
+template <class Add = AddAlu>
+__device__ __forceinline__ void sha_compress_small(uint32_t s[8], uint32_t w[16], Add add = Add()) {
+    uint32_t v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = s[i];
+#pragma unroll
+    for (int t = 0; t < 16; ++t) {
+        uint32_t &a = v[(8 - t % 8) % 8], &b = v[(9 - t % 8) % 8], &c = v[(10 - t % 8) % 8], &d = v[(11 - t % 8) % 8];
+        uint32_t &e = v[(12 - t % 8) % 8], &f = v[(13 - t % 8) % 8], &g = v[(14 - t % 8) % 8], &h = v[(15 - t % 8) % 8];
+        const uint32_t t1 = add(add(add(h, add(w[t], sha_k(t))), ch(e, f, g)), bsig1(e));
+        const uint32_t t2 = add(bsig0(a), maj(a, b, c));
+        d = add(d, t1);
+        h = add(t1, t2);
+    }
+#pragma unroll 1
+    for (int base = 16; base < 64; base += 16) {
+#pragma unroll
+        for (int t = 0; t < 16; ++t) {
+            w[t] = add(add(w[t], w[(t + 9) & 15]), add(ssig0(w[(t + 1) & 15]), ssig1(w[(t + 14) & 15])));
+            uint32_t &a = v[(8 - t % 8) % 8], &b = v[(9 - t % 8) % 8], &c = v[(10 - t % 8) % 8], &d = v[(11 - t % 8) % 8];
+            uint32_t &e = v[(12 - t % 8) % 8], &f = v[(13 - t % 8) % 8], &g = v[(14 - t % 8) % 8], &h = v[(15 - t % 8) % 8];
+            const uint32_t t1 = add(add(add(h, add(w[t], c_sha_k[base + t])), ch(e, f, g)), bsig1(e));
+            const uint32_t t2 = add(bsig0(a), maj(a, b, c));
+            d = add(d, t1);
+            h = add(t1, t2);
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s[i] = add(s[i], v[i]);
+}
+
+// Compression of a data block inside the fixed-length messages below:
+// compact (default; measured faster for the chain kernel on GB300, whose
+// fully unrolled form stalls on instruction fetch) or fully unrolled
+// (KVGOV_COMPACT_ROUNDS=0).
+#ifndef KVGOV_COMPACT_ROUNDS
+#define KVGOV_COMPACT_ROUNDS 1
+#endif
+template <bool FROM_IV, class Add>
+__device__ __forceinline__ void sha_compress_data(uint32_t s[8], uint32_t w[16], Add add) {
+#if KVGOV_COMPACT_ROUNDS
+    sha_compress_small(s, w, add);
+#else
+    sha_compress_t<false, FROM_IV>(s, w, add);
+#endif
 }
 
 // Fixed-length messages of the chain (section 2.1 / 4.1 / 4.2 equations).
@@ -108,56 +213,60 @@ __device__ __forceinline__ void sha_compress(uint32_t s[8], uint32_t w[16]) {
 // 5.1.1) appends 0x80, zeros and the 64-bit bit length; for these lengths the
 // padding words are compile-time constants.
 
+__device__ __forceinline__ void pad_block(uint32_t w[16], int first, uint32_t bits) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) w[i] = 0u;
+    w[first] = 0x80000000u;
+    w[15] = bits;
+}
+
 // H(T): 64-byte message = one data block + one constant padding block.
-__device__ __forceinline__ void sha256_msg64(const uint32_t tw[16], uint32_t out[8]) {
+template <class Add>
+__device__ __forceinline__ void sha256_msg64(const uint32_t tw[16], uint32_t out[8], Add add) {
     uint32_t s[8], w[16];
     sha_iv(s);
 #pragma unroll
     for (int i = 0; i < 16; ++i) w[i] = tw[i];
-    sha_compress(s, w);
-    w[0] = 0x80000000u;
-#pragma unroll
-    for (int i = 1; i < 15; ++i) w[i] = 0u;
-    w[15] = 64u * 8u;
-    sha_compress(s, w);
+    sha_compress_data<true>(s, w, add);
+    pad_block(w, 0, 64u * 8u);
+    sha_compress_t<true, false>(s, w, add);
 #pragma unroll
     for (int i = 0; i < 8; ++i) out[i] = s[i];
 }
 
 // H(P || T): 32-byte prefix P (parent digest or salt) + 64-byte block.
-__device__ __forceinline__ void sha256_msg96(const uint32_t pw[8], const uint32_t tw[16], uint32_t out[8]) {
+template <class Add>
+__device__ __forceinline__ void sha256_msg96(const uint32_t pw[8], const uint32_t tw[16], uint32_t out[8], Add add) {
     uint32_t s[8], w[16];
     sha_iv(s);
 #pragma unroll
     for (int i = 0; i < 8; ++i) { w[i] = pw[i]; w[8 + i] = tw[i]; }
-    sha_compress(s, w);
+    sha_compress_data<true>(s, w, add);
 #pragma unroll
     for (int i = 0; i < 8; ++i) w[i] = tw[8 + i];
     w[8] = 0x80000000u;
 #pragma unroll
     for (int i = 9; i < 15; ++i) w[i] = 0u;
     w[15] = 96u * 8u;
-    sha_compress(s, w);
+    sha_compress_data<false>(s, w, add);
 #pragma unroll
     for (int i = 0; i < 8; ++i) out[i] = s[i];
 }
 
 // H(S || P || T): salt, parent digest, block (the boundary block of 4.2).
+template <class Add>
 __device__ __forceinline__ void sha256_msg128(const uint32_t sw[8], const uint32_t pw[8], const uint32_t tw[16],
-                                              uint32_t out[8]) {
+                                              uint32_t out[8], Add add) {
     uint32_t s[8], w[16];
     sha_iv(s);
 #pragma unroll
     for (int i = 0; i < 8; ++i) { w[i] = sw[i]; w[8 + i] = pw[i]; }
-    sha_compress(s, w);
+    sha_compress_data<true>(s, w, add);
 #pragma unroll
     for (int i = 0; i < 16; ++i) w[i] = tw[i];
-    sha_compress(s, w);
-    w[0] = 0x80000000u;
-#pragma unroll
-    for (int i = 1; i < 15; ++i) w[i] = 0u;
-    w[15] = 128u * 8u;
-    sha_compress(s, w);
+    sha_compress_data<false>(s, w, add);
+    pad_block(w, 0, 128u * 8u);
+    sha_compress_t<true, false>(s, w, add);
 #pragma unroll
     for (int i = 0; i < 8; ++i) out[i] = s[i];
 }

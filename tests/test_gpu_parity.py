@@ -73,7 +73,7 @@ def test_salts_bad_offsets_flagged(kv):
 
 
 # --------------------------------------------------------- block offsets
-@pytest.mark.parametrize("n", [0, 1, 5, 127, 4095, 4096, 4097, 10000, 131073])
+@pytest.mark.parametrize("n", [0, 1, 5, 127, 1024, 1025, 4097, 10000, 131073, 1000003])
 def test_block_offsets(kv, n):
     rng = np.random.default_rng(n)
     lens = rng.integers(0, 200, n)

@@ -112,10 +112,13 @@ def test_full_long(kv):
 
 def test_full_wide_serving_steps(kv):
     """The bench's step (PrefixCache.serve) on the full 131,072 x 128 batch,
-    three times: batch A into an empty cache, a fresh batch B, then A again.
+    three times: batch A into an empty cache, a fresh batch B with the same
+    shared prefix (its 4 unsalted blocks hit), then A again (all 8 hit).
     Every salt, digest and prefix length is compared with the oracle."""
     wa, wb = W.make("wide", seed=101), W.make("wide", seed=102)
     wb.secret, wb.ids, wb.id_off = wa.secret, wa.ids, wa.id_off
+    # B shares A's 64-token prefix (the prefix every request of the service starts with)
+    wb.batch.tokens.reshape(-1, 128)[:, :64] = wa.batch.tokens[:64]
     n_blocks = wa.batch.n * 8
     cache = PrefixCache(next_pow2(4 * 3 * n_blocks), wa.secret, wa.ids, wa.id_off)
     salts = oracle.derive_salts(wa.secret, wa.ids, wa.id_off)
