@@ -4,19 +4,21 @@
 One step = one serving batch through the whole hot path, every step a
 libkvgov kernel: per-principal salts (HMAC-SHA-256, 4096 principals) ->
 blocking (block offsets) -> BOUNDARY-salted chain hash (salt at token 64,
-block 4) -> probe of the resident prefix-cache table -> insert of the batch's
-digests.  Workload: 131,072 requests x 128 tokens (8 blocks each; the
-largest batch), a 64-token prefix shared by all requests, 4096 principals.
+block 4) -> probe of the resident prefix-cache table -> insert of each
+request's uncached blocks.  Workload: 131,072 requests x 128 tokens (8 blocks
+each; the largest batch), a 64-token prefix shared by all requests, 4096
+principals.
+
+Serving regime: a pool of distinct batches (inputs resident in HBM) is
+cycled, and every step runs under a new secret epoch, so each step is new
+traffic: the 4 unsalted shared-prefix blocks of every request hit the cache,
+the 4 salted blocks miss and are inserted (524,288 new keys per step).  The
+table is sized so that its load factor stays at or below 0.5 at the end.
 
 Timed region: `--steps` steps after `--warmup` untimed ones, bracketed by a
 barrier and cuda synchronize, CUDA events on the launching stream, max over
-ranks.  A pool of distinct batches (inputs already resident in HBM) is cycled,
-and the table is pre-filled with every pool batch's chains before timing, so
-every step re-serves a cached batch: each probe walks all 8 blocks (all hit)
-and each insert finds its 8 keys present.
-
-Prints ONE JSON line (rank 0).  `--impl reference` times the CPU oracle
-(plain C, the bounded sample described in its line) as the reference arm.
+ranks.  Prints ONE JSON line (rank 0).  `--impl reference` times the CPU
+oracle (plain C) on a bounded sample of the same step as the reference arm.
 """
 from __future__ import annotations
 
@@ -201,14 +203,53 @@ def measure_int_peak(torch, peak_lib_path):
 
 
 # --------------------------------------------------------------------------- reference arm
-def cpu_oracle_step(w, sample_req, n_threads, keyset):
-    """The oracle on a sample: salts, chain (threaded over request chunks),
-    probe and insert.  Returns blocks hashed."""
+def epoch_secret(base: bytes, step: int) -> bytes:
+    """The server secret of step `step` (an input of the step, not a hash)."""
+    return base[:24] + int(step).to_bytes(8, "little")
+
+
+def share_prefix(pool_host):
+    """Give every pool batch the first batch's 64-token prefix (the prefix
+    every request of the service starts with)."""
+    p0 = pool_host[0].batch.tokens.reshape(-1, 128)[0, :64].copy()
+    for w in pool_host:
+        w.batch.tokens.reshape(-1, 128)[:, :64] = p0
+
+
+class FlushPolicy:
+    """Host bookkeeping of the cache's flush policy and the closed-form key
+    counts: after a flush the next batch misses everywhere (it inserts the 4
+    shared-prefix blocks once plus 4 salted blocks per request); later batches
+    hit the shared prefix and insert their 4 salted blocks."""
+
+    def __init__(self, capacity: int, new_per_step: int):
+        self.capacity, self.new_per_step = capacity, new_per_step
+        self.in_table, self.expected_new, self.flushes, self.last_prefix = 0, 0, 0, 0
+        self.fresh = True
+
+    def before_step(self) -> bool:
+        flushed = False
+        if not self.fresh and self.in_table + self.new_per_step > self.capacity // 2:
+            self.in_table, self.fresh, flushed = 0, True, True
+            self.flushes += 1
+        add = self.new_per_step + (4 if self.fresh else 0)
+        self.last_prefix = 0 if self.fresh else 4
+        self.in_table += add
+        self.expected_new += add
+        self.fresh = False
+        return flushed
+
+
+def cpu_oracle_step(w, sample_req, n_threads, secret):
+    """The oracle on the first `sample_req` requests of one step: salts under
+    `secret`, the chain (threaded over request chunks), the probe against a
+    set holding the shared prefix's 4 blocks, and the insert of the uncached
+    blocks.  Returns (blocks hashed, digests)."""
     import concurrent.futures as cf
 
     import oracle
     b = w.batch
-    salts = oracle.derive_salts(w.secret, w.ids, w.id_off)
+    salts = oracle.derive_salts(secret, w.ids, w.id_off)
     n = sample_req
     chunks = np.array_split(np.arange(n), n_threads)
 
@@ -221,12 +262,14 @@ def cpu_oracle_step(w, sample_req, n_threads, keyset):
         return oracle.chain_hash(oracle.BOUNDARY, toks, off, b.principal[lo:hi], salts, b.boundary_tok[lo:hi])
 
     with cf.ThreadPoolExecutor(n_threads) as ex:
-        parts = list(ex.map(run, chunks))
-    d = np.concatenate(parts)
+        d = np.concatenate(list(ex.map(run, chunks)))
     blk = oracle.block_offsets(b.tok_off[:n + 1])
-    keyset.prefix_blocks(d, blk)
-    keyset.insert(d)
-    return int(blk[-1])
+    ks = oracle.KeySet(1)
+    ks.insert(d[:4])                     # the shared prefix's blocks are cached
+    pre = ks.prefix_blocks(d, blk)
+    suffix = np.concatenate([d[blk[r] + pre[r]:blk[r + 1]] for r in range(n)])
+    ks.insert(suffix)
+    return int(blk[-1]), d
 
 
 def reference_arm(args):
@@ -239,14 +282,12 @@ def reference_arm(args):
     cores = len(os.sched_getaffinity(0))
     w = W.make("wide", seed=args.seed)
     sample = args.cpu_sample
-    ks = oracle.KeySet(1)
-    cpu_oracle_step(w, sample, cores, ks)          # pre-fill: the sample is cached, as on the GPU
-    for _ in range(args.warmup):
-        cpu_oracle_step(w, sample, cores, ks)
+    for i in range(args.warmup):
+        cpu_oracle_step(w, sample, cores, epoch_secret(w.secret, i))
     t0 = time.perf_counter()
     blocks = 0
-    for _ in range(args.steps):
-        blocks += cpu_oracle_step(w, sample, cores, ks)
+    for i in range(args.steps):
+        blocks += cpu_oracle_step(w, sample, cores, epoch_secret(w.secret, args.warmup + i))[0]
     dt = time.perf_counter() - t0
     value = blocks / dt
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
@@ -254,8 +295,8 @@ def reference_arm(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
             "config": dict(WORKLOAD, sample_requests=sample),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                             "sample": f"first {sample} requests of the batch per step: salts, chain, "
-                                       f"probe, insert (set already holding them)"},
+                             "sample": f"first {sample} requests of the batch per step (salts for all 4096 "
+                                       f"principals, chain on {cores} threads, probe, insert of the uncached blocks)"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "tokens_per_s": 16 * value}
     print(json.dumps(line), flush=True)
@@ -271,6 +312,7 @@ def main():
     ap.add_argument("--impl", default="kvgov", choices=["kvgov", "reference"])
     ap.add_argument("--pool", type=int, default=16, help="distinct resident batches cycled by the steps")
     ap.add_argument("--e2e-steps", type=int, default=100)
+    ap.add_argument("--table-slots", type=int, default=1 << 25, help="cache capacity (power of two)")
     ap.add_argument("--seed", type=int, default=None, help="base seed (default: fresh per run)")
     ap.add_argument("--cpu-sample", type=int, default=16384, help="requests per oracle step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -287,7 +329,7 @@ def main():
     from paper_2608_09225_gb300 import build as kbuild
     from paper_2608_09225_gb300 import kvgov as K
     from paper_2608_09225_gb300 import workloads as W
-    from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache, next_pow2
+    from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -300,27 +342,41 @@ def main():
 
     # ---- inputs: a pool of distinct batches, resident in HBM (weak scaling: per-rank seeds)
     pool_host = [W.make("wide", seed=rank_seed(args.seed, rank, i)) for i in range(args.pool)]
+    share_prefix(pool_host)
     w0 = pool_host[0]
     n_req = w0.batch.n
     n_blocks = int((w0.batch.lengths() // 16).sum())
+    new_per_step = 4 * n_req                       # the salted blocks 4..7 of every request
     pool = [DeviceBatch.from_host(w.batch.tokens, w.batch.tok_off, w.batch.principal, w.batch.boundary_tok)
             for w in pool_host]
-    cache = PrefixCache(next_pow2(4 * args.pool * n_blocks // 2), w0.secret, w0.ids, w0.id_off)
+    cache = PrefixCache(args.table_slots, w0.secret, w0.ids, w0.id_off)
+    flush = FlushPolicy(args.table_slots, new_per_step)
     bufs = {"blk_off": torch.empty(n_req + 1, dtype=torch.int64, device="cuda"),
             "digests": torch.empty((n_blocks, 32), dtype=torch.uint8, device="cuda"),
             "prefix": torch.empty(n_req, dtype=torch.int32, device="cuda")}
-    for db in pool:                                          # pre-fill: every pool batch is cached
-        cache.serve(W.BOUNDARY, db, bufs)
+
+    # ---- gate before timing: the first serve into the empty table (closed forms)
+    cache.set_secret(epoch_secret(w0.secret, 0))
+    flush.before_step()
+    prefix, digests, _ = cache.serve(W.BOUNDARY, pool[0], bufs)
     torch.cuda.synchronize()
     cache.check_status()
-
-    # ---- parity gate on a sample (oracle) before timing
-    gate = parity_gate(cache, pool_host[0], pool[0], bufs)
+    gate_digests = digests.view(n_req, -1, 32)[: args.cpu_sample].cpu().numpy().reshape(-1, 32)
+    gate = {"prefix_all_zero_on_empty_table": bool((prefix == 0).all().item()),
+            "n_new": int(cache.n_new.item()), "n_new_expected": flush.expected_new}
+    if not gate["prefix_all_zero_on_empty_table"] or gate["n_new"] != gate["n_new_expected"]:
+        raise SystemExit(f"gate failed: {gate}")
 
     stream = torch.cuda.current_stream()
+    epoch = [1]
+    launches = [0]
 
     def step(db, ev=None):
-        K.derive_salts(cache.secret, cache.ids, cache.id_off, cache.salts, cache.status)
+        if flush.before_step():                   # load factor would pass 0.5: flush the cache
+            K.table_init(cache.slots)
+            launches[0] += 1
+        K.derive_salts(epoch_secret(cache.secret, epoch[0]), cache.ids, cache.id_off, cache.salts, cache.status)
+        epoch[0] += 1
         K.block_offsets(db.tok_off, bufs["blk_off"], cache.status)
         if ev is not None:
             ev[0].record(stream)
@@ -329,35 +385,45 @@ def main():
         if ev is not None:
             ev[1].record(stream)
         K.probe(cache.slots, bufs["digests"], bufs["blk_off"], bufs["prefix"], cache.status)
-        K.insert(cache.slots, bufs["digests"], cache.status, cache.n_new)
+        K.insert_uncached(cache.slots, bufs["digests"], bufs["blk_off"], bufs["prefix"], cache.status, cache.n_new)
+        launches[0] += 5   # salts, block offsets, chain, probe, insert
 
-    kernels_per_step = 5   # salts, block offsets, chain, probe, insert
     for i in range(args.warmup):
-        step(pool[i % args.pool])
+        step(pool[(1 + i) % args.pool])
     torch.cuda.synchronize()
 
     chain_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                 for _ in range(args.steps)]
     t_start, t_stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    launches[0] = 0
+    flushes_before = flush.flushes
     with ClockSampler(local) as clk:
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize()
         t_start.record(stream)
         for i in range(args.steps):
-            step(pool[i % args.pool], chain_ev[i])
+            step(pool[(1 + args.warmup + i) % args.pool], chain_ev[i])
         t_stop.record(stream)
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
     cache.check_status()
+    gate["n_new_total"] = int(cache.n_new.item())
+    gate["n_new_total_expected"] = flush.expected_new
+    gate["flushes_in_timed_steps"] = flush.flushes - flushes_before
+    gate["last_step_prefix_expected"] = flush.last_prefix
+    gate["last_step_prefix_ok"] = bool((bufs["prefix"] == flush.last_prefix).all().item())
+    if gate["n_new_total"] != gate["n_new_total_expected"] or not gate["last_step_prefix_ok"]:
+        raise SystemExit(f"gate failed: {gate}")
+    kernel_launches = launches[0]
     ms = t_start.elapsed_time(t_stop)
     chain_ms = float(np.mean([a.elapsed_time(b) for a, b in chain_ev]))
     ms = max_over_ranks(ms, world, dist, "cuda")
     value = world * args.steps * n_blocks / (ms / 1e3)
 
     # ---- end to end through the public API with host buffers
-    e2e = e2e_leg(torch, K, W, cache, pool_host[: min(4, args.pool)], args.e2e_steps, bufs, world, dist)
+    e2e = e2e_leg(torch, K, W, w0, pool_host[: min(4, args.pool)], args.e2e_steps, world, dist, args.table_slots)
 
     # ---- roofline of the chain kernel (integer-pipe bound)
     micro = measure_int_peak(torch, kbuild.PEAK_LIB)
@@ -387,12 +453,17 @@ def main():
             "config": dict(WORKLOAD, pool_batches=args.pool, seed=args.seed,
                            l2=f"{args.pool} distinct resident batches cycled (each re-read after "
                               f"{args.pool - 1} others); table {cache.capacity * 32 >> 20} MiB",
-                           table_slots=cache.capacity),
+                           table_slots=cache.capacity,
+                           regime="new secret epoch per step: the 4 shared-prefix blocks hit, the 4 salted blocks "
+                                  "miss and are inserted; the cache is flushed (table re-initialised, inside the "
+                                  "timed steps) whenever the next step would take it past load factor 0.5"),
             "tokens_per_s": 16 * value, "chain_digests_per_s": world * n_blocks / (chain_ms / 1e3),
-            "e2e": e2e, "gpu_launches": kernels_per_step * args.steps, "clocks": clock, "roofline": roofline,
-            "parity_gate": gate}
+            "e2e": e2e, "gpu_launches": kernel_launches, "clocks": clock, "roofline": roofline,
+            "gate": gate}
     if rank == 0 and not args.no_cpu_baseline and world == 1:
-        line["cpu_baseline"] = cpu_baseline(pool_host[0], args.cpu_sample)
+        line["cpu_baseline"] = cpu_baseline(pool_host[0], args.cpu_sample, gate_digests)
+        if not line["cpu_baseline"]["gate_sample_digests_equal_gpu"]:
+            raise SystemExit("parity: GPU digests of the gate step differ from the oracle's")
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -400,38 +471,11 @@ def main():
     return 0
 
 
-def parity_gate(cache, w, db, bufs):
-    """Before timing: a sample of digests and every prefix length of one
-    batch against the oracle and the closed form (all 8 blocks cached)."""
-    import torch
-
-    import oracle
-    from paper_2608_09225_gb300 import workloads as W
-    prefix, digests, blk = cache.serve(W.BOUNDARY, db, bufs)
-    torch.cuda.synchronize()
-    b = w.batch
-    rng = np.random.default_rng(0)
-    rows = np.sort(rng.choice(b.n, size=256, replace=False))
-    salts = oracle.derive_salts(w.secret, w.ids, w.id_off)
-    got = digests.cpu().numpy().reshape(b.n, -1, 32)[rows]
-    for r, g in zip(rows, got):
-        lo, hi = b.tok_off[r], b.tok_off[r + 1]
-        ref = oracle.chain_hash(oracle.BOUNDARY, b.tokens[lo:hi], np.array([0, hi - lo]), b.principal[r:r + 1],
-                                salts, b.boundary_tok[r:r + 1])
-        if not (ref == g).all():
-            raise SystemExit(f"parity gate: request {r} digests differ from the oracle")
-    if not (cache.salts.cpu().numpy() == salts).all():
-        raise SystemExit("parity gate: salts differ from the oracle")
-    pre = prefix.cpu().numpy()
-    if not (pre == 8).all():
-        raise SystemExit("parity gate: cached batch must hit all 8 blocks")
-    return {"sampled_requests": 256, "digests": "bit-exact", "prefix_blocks": "all 8 (closed form)"}
-
-
-def e2e_leg(torch, K, W, cache, hosts, steps, bufs, world, dist):
-    """Same metric with host buffers: pinned H2D of each step's inputs and
-    D2H of its prefix lengths inside the timed region."""
-    from paper_2608_09225_gb300.pipeline import DeviceBatch
+def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots):
+    """Same step with host buffers: pinned H2D of each step's inputs and D2H
+    of its prefix lengths inside the timed region, through PrefixCache.serve
+    on a cache of its own."""
+    from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache
     pinned = []
     for w in hosts:
         b = w.batch
@@ -439,6 +483,12 @@ def e2e_leg(torch, K, W, cache, hosts, steps, bufs, world, dist):
                             for a in (b.tokens, b.tok_off, b.principal, b.boundary_tok)))
     n_req = hosts[0].batch.n
     n_blocks = int((hosts[0].batch.lengths() // 16).sum())
+    warm = 3
+    cache = PrefixCache(table_slots, w0.secret, w0.ids, w0.id_off)
+    flush = FlushPolicy(table_slots, 4 * n_req)
+    bufs = {"blk_off": torch.empty(n_req + 1, dtype=torch.int64, device="cuda"),
+            "digests": torch.empty((n_blocks, 32), dtype=torch.uint8, device="cuda"),
+            "prefix": torch.empty(n_req, dtype=torch.int32, device="cuda")}
     out = torch.empty(n_req, dtype=torch.int32).pin_memory()
     dev = [torch.empty_like(t, device="cuda") for t in pinned[0]]
     h2d = sum(t.numel() * t.element_size() for t in pinned[0])
@@ -448,11 +498,13 @@ def e2e_leg(torch, K, W, cache, hosts, steps, bufs, world, dist):
         src = pinned[i % len(pinned)]
         for d, s in zip(dev, src):
             d.copy_(s, non_blocking=True)
-        db = DeviceBatch(dev[0], dev[1], dev[2], dev[3], n_blocks)
-        prefix, _, _ = cache.serve(W.BOUNDARY, db, bufs)
+        cache.set_secret(epoch_secret(w0.secret, i))
+        if flush.before_step():
+            K.table_init(cache.slots)
+        prefix, _, _ = cache.serve(W.BOUNDARY, DeviceBatch(dev[0], dev[1], dev[2], dev[3], n_blocks), bufs)
         out.copy_(prefix, non_blocking=True)
 
-    for i in range(3):
+    for i in range(warm):
         one(i)
     torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -460,29 +512,32 @@ def e2e_leg(torch, K, W, cache, hosts, steps, bufs, world, dist):
         dist.barrier()
     a.record()
     for i in range(steps):
-        one(i)
+        one(warm + i)
     b.record()
     torch.cuda.synchronize()
+    cache.check_status()
     ms = max_over_ranks(a.elapsed_time(b), world, dist, "cuda")
     return {"value": world * steps * n_blocks / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps}
 
 
-def cpu_baseline(w, sample):
-    """The oracle, as it stands, on the machine's host cores: a bounded sample."""
+def cpu_baseline(w, sample, gpu_digests):
+    """The oracle, as it stands, on the machine's host cores: a bounded sample of
+    the step.  Its digests of the gate step are compared with the GPU's."""
     import oracle
     oracle.build()
     cores = len(os.sched_getaffinity(0))
-    ks = oracle.KeySet(1)
-    cpu_oracle_step(w, sample, cores, ks)
+    _, d0 = cpu_oracle_step(w, sample, cores, epoch_secret(w.secret, 0))
+    same = bool(d0.shape == gpu_digests.shape and (d0 == gpu_digests).all())
     reps, blocks, t0 = 0, 0, time.perf_counter()
     while reps < 2 or time.perf_counter() - t0 < 5.0:
-        blocks += cpu_oracle_step(w, sample, cores, ks)
+        blocks += cpu_oracle_step(w, sample, cores, epoch_secret(w.secret, 1 + reps))[0]
         reps += 1
     dt = time.perf_counter() - t0
     return {"value": blocks / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"{reps} steps over the first {sample} requests of one batch "
-                      f"(salts, chain on {cores} threads, probe, insert); {dt:.1f} s"}
+            "sample": f"{reps} steps over the first {sample} requests of one batch (salts for 4096 principals, "
+                      f"chain on {cores} threads, probe, insert of the uncached blocks); {dt:.1f} s",
+            "gate_sample_digests_equal_gpu": same}
 
 
 if __name__ == "__main__":

@@ -54,13 +54,13 @@ typedef struct CUstream_st *kvgov_stream_t;
 #define KVGOV_F_BADINDEX 0x10u     /* a principal index, boundary offset or
                                       offset array entry was out of range; the
                                       affected request produced no output     */
-#define KVGOV_F_SENTINEL 0x20u     /* a key whose first 8 bytes are all 0x00 or
-                                      all 0xFF was given to kvgov_insert; it is
-                                      skipped (these values mark empty and
-                                      claimed slots)                          */
+#define KVGOV_F_SENTINEL 0x20u     /* a reserved key (bytes 0-15, 16-23 or
+                                      24-31 all zero) was given to an insert; it
+                                      is skipped (these values mark empty slots
+                                      and keys still being written)           */
 #define KVGOV_F_TABLE_FULL 0x40u   /* kvgov_insert found no free slot for a key */
-#define KVGOV_F_TIMEOUT 0x80u      /* kvgov_insert gave up waiting for another
-                                      thread's claimed slot to be published   */
+#define KVGOV_F_TIMEOUT 0x80u      /* an insert gave up waiting for another
+                                      thread to finish writing a slot's key   */
 
 /* Salt placement (paper section 2.1 equation, section 4.1, section 4.2). */
 #define KVGOV_UNSALTED 0           /* h_0 = H(T_0), h_j = H(h_{j-1} || T_j)   */
@@ -145,11 +145,13 @@ int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t *d_tok_off
  * The prefix-cache index (paper section 2.1 and Table 1, row 1: a block
  * prefix cache keyed by chained block hashes).  The caller owns a table of
  * `capacity` 32-byte slots (capacity a power of two >= KVGOV_MIN_CAPACITY,
- * d_slots 16-byte aligned).  A slot is empty when its first 8 bytes are zero;
- * a key's home slot is its first 8 bytes read as a little-endian u64, modulo
- * capacity, with linear probing.  Keys are stored verbatim, so keys whose
- * first 8 bytes are all 0x00 or all 0xFF cannot be stored (KVGOV_F_SENTINEL);
- * for SHA-256 digests that happens with probability 2^-63.
+ * d_slots 16-byte aligned).  A slot is empty when its first 16 bytes are
+ * zero; a key's home slot is its first 8 bytes read as a little-endian u64,
+ * modulo capacity, with linear probing.  Keys are stored verbatim and claimed
+ * with a 128-bit compare-and-swap of their first 16 bytes, so keys whose
+ * bytes 0-15, 16-23 or 24-31 are all zero cannot be stored
+ * (KVGOV_F_SENTINEL); for SHA-256 digests that happens with probability
+ * about 2^-63.
  */
 
 /* kvgov_table_init -- mark every slot empty.  EINVAL: bad capacity/pointer. */
@@ -162,9 +164,9 @@ int kvgov_table_init(uint8_t *d_slots, uint64_t capacity, kvgov_stream_t stream)
  * overlap in time with each other or with kvgov_probe (stream order them).
  *   d_n_new   nullable; the number of keys newly stored is ADDED to it.
  *   d_status  required; KVGOV_F_SENTINEL, KVGOV_F_TABLE_FULL and
- *             KVGOV_F_TIMEOUT as above.  A wait for a concurrently claimed
- *             slot is bounded (kvgov_set_spin_limit); on timeout the key is
- *             not inserted.
+ *             KVGOV_F_TIMEOUT as above.  A wait for another thread to finish
+ *             writing a slot with the same first 16 bytes is bounded
+ *             (kvgov_set_spin_limit); on timeout the key is not inserted.
  * n_keys = 0 is a no-op.  EINVAL: bad capacity, NULL or misaligned pointer,
  * n_keys < 0.
  */
@@ -191,9 +193,28 @@ int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_dige
                 uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * kvgov_insert_uncached -- insert a probed batch: for every request r, its
+ * blocks j >= d_prefix_blocks[r] (the output of kvgov_probe on the same
+ * table, digests and offsets).  The blocks before that were found in the
+ * table, and a table only grows, so the resulting set and *d_n_new are those
+ * of inserting every digest with kvgov_insert.  In the serving step of the
+ * paper's block prefix cache (section 2.1: lookup, then the uncached blocks
+ * are computed and cached) this is the insert after the probe.
+ *   d_digests, d_blk_off, n_req  as for kvgov_probe.
+ *   d_prefix_blocks  [n_req] int32 from kvgov_probe (values < 0 read as 0).
+ *   d_n_new, d_status  as for kvgov_insert (d_status required); also
+ *                    KVGOV_F_BADINDEX for rows outside [d_blk_off[r], d_blk_off[n_req]).
+ * Must not overlap in time with other calls on the same table.
+ * n_req = 0 is a no-op.  EINVAL: bad capacity, NULL or misaligned pointer.
+ */
+int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,
+                          const int64_t *d_blk_off, int32_t n_req, const int32_t *d_prefix_blocks,
+                          unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream);
+
+/*
  * kvgov_set_spin_limit -- bound on how many times an inserting thread
- * re-reads a slot that another thread has claimed but not yet published
- * before it gives up with KVGOV_F_TIMEOUT (about 100 ns per re-read).
+ * re-reads a slot whose key another thread is still writing before it gives
+ * up with KVGOV_F_TIMEOUT (about 100 ns per re-read).
  * Process-wide; applies to launches made after the call.  0 restores the
  * default (2^23, about a second).  Returns the previous value.
  */

@@ -32,9 +32,10 @@
  *
  * The cache index is modelled as a mathematical set of 32-byte keys, kept as
  * a sorted array searched with bsearch; it has nothing in common with the
- * GPU's open-addressing table except the keys it holds.  Keys whose first 8
- * bytes are all 0x00 or all 0xFF are reserved by the GPU table encoding
- * (empty slot and in-flight claim); the set refuses them the same way.
+ * GPU's open-addressing table except the keys it holds.  Keys whose bytes
+ * 0..15, 16..23 or 24..31 are all zero are reserved by the GPU table
+ * encoding (empty slot, key still being written); the set refuses them the
+ * same way.
  *
  * Parity pins (tests/test_oracle_pins.py): SHA-256 against Python hashlib on
  * every message length 0..300 and random messages; HMAC against Python hmac;
@@ -322,15 +323,19 @@ int oracle_chain_hash(int mode, const int32_t *tokens, const int64_t *tok_off,
 
 static int key_cmp(const void *a, const void *b) { return memcmp(a, b, 32); }
 
-/* First 8 bytes all 0x00 or all 0xFF: not storable (see header). */
+/* Keys the GPU table cannot store (see header): bytes 0..15 all zero (an
+ * empty slot), or bytes 16..23 or 24..31 all zero (a key still being
+ * written). */
 int oracle_key_reserved(const uint8_t *key)
 {
-    int zeros = 1, ones = 1;
-    for (int i = 0; i < 8; i++) {
-        if (key[i] != 0x00) zeros = 0;
-        if (key[i] != 0xFF) ones = 0;
-    }
-    return zeros || ones;
+    int lo = 1, mid = 1, hi = 1;
+    for (int i = 0; i < 16; i++)
+        if (key[i] != 0) lo = 0;
+    for (int i = 16; i < 24; i++)
+        if (key[i] != 0) mid = 0;
+    for (int i = 24; i < 32; i++)
+        if (key[i] != 0) hi = 0;
+    return lo || mid || hi;
 }
 
 int oracle_set_contains(const uint8_t *set_keys, int64_t n_set, const uint8_t *key)

@@ -55,35 +55,43 @@ __device__ void sha_absorb_finish(uint32_t s[8], unsigned long long prior, unsig
     }
 }
 
+// K0 of RFC 2104 as 16 big-endian words: the key zero-padded to 64 bytes, or
+// SHA-256(key) zero-padded when the key is longer than 64 bytes.
+__device__ __forceinline__ void hmac_k0(const SaltParams &p, uint32_t k0[16]) {
+    if (p.secret_len > 64) {
+        uint32_t hk[8];
+        sha_iv(hk);
+        sha_absorb_finish(hk, 0ull, p.secret_len, [&](unsigned long long i) { return p.secret[i]; });
+#pragma unroll
+        for (int i = 0; i < 16; ++i) k0[i] = i < 8 ? hk[i] : 0u;
+        return;
+    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        uint32_t v = 0;
+#pragma unroll
+        for (int b = 0; b < 4; ++b) v = (v << 8) | (4u * i + b < p.secret_len ? (uint32_t)p.secret[4 * i + b] : 0u);
+        k0[i] = v;
+    }
+}
+
 __global__ void __launch_bounds__(kSaltThreads) salts_kernel(const SaltParams p) {
-    __shared__ uint32_t s_ipad[8], s_opad[8];
-    if (threadIdx.x == 0) {
-        uint32_t k0[16];
+    // The (K0 ^ ipad) and (K0 ^ opad) midstates are computed once per CTA,
+    // by the first thread of warp 0 and of warp 1 in parallel.
+    __shared__ uint32_t s_mid[2][8];
+    if ((threadIdx.x & 31) == 0 && threadIdx.x < 64) {
+        const uint32_t pad = threadIdx.x == 0 ? 0x36363636u : 0x5c5c5c5cu;
+        uint32_t k0[16], st[8];
+        hmac_k0(p, k0);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) k0[i] = 0u;
-        if (p.secret_len > 64) {
-            uint32_t hk[8];
-            sha_iv(hk);
-            sha_absorb_finish(hk, 0ull, p.secret_len, [&](unsigned long long i) { return p.secret[i]; });
+        for (int i = 0; i < 16; ++i) k0[i] ^= pad;
+        sha_iv(st);
+        sha_compress_small(st, k0);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) k0[i] = hk[i];
-        } else {
-            for (uint32_t i = 0; i < p.secret_len; ++i)
-                k0[i >> 2] |= (uint32_t)p.secret[i] << (24 - 8 * (i & 3));
-        }
-        uint32_t si[8], so[8], w[16];
-        sha_iv(si);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) w[i] = k0[i] ^ 0x36363636u;
-        sha_compress_small(si, w);
-        sha_iv(so);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) w[i] = k0[i] ^ 0x5c5c5c5cu;
-        sha_compress_small(so, w);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) { s_ipad[i] = si[i]; s_opad[i] = so[i]; }
+        for (int i = 0; i < 8; ++i) s_mid[threadIdx.x >> 5][i] = st[i];
     }
     __syncthreads();
+    uint32_t *s_ipad = s_mid[0], *s_opad = s_mid[1];
 
     for (long long pr = (long long)blockIdx.x * kSaltThreads + threadIdx.x; pr < p.n;
          pr += (long long)gridDim.x * kSaltThreads) {

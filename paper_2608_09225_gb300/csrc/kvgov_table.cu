@@ -8,18 +8,24 @@
 // adversary's probes only populate its own namespace), section 5.7 (a
 // divergence at token i invalidates every block from floor(i/B) on).
 //
-// Slot encoding: four little-endian u64 words w0..w3 = the key verbatim.
-// w0 == 0 marks an empty slot and w0 == ~0 a slot claimed by an insert that
-// has not yet published the key; keys with those first words are refused.
-// Home slot = w0 & (capacity - 1); collisions go to the next slot (linear
-// probing, wrapping).
+// Slot encoding: the key verbatim as four little-endian u64 words w0..w3.
+// (w0, w1) == 0 marks an empty slot.  Home slot = w0 & (capacity - 1);
+// collisions go to the next slot (linear probing, wrapping).  Keys with
+// (w0, w1) == 0, w2 == 0 or w3 == 0 are refused (reserved): the first marks
+// empty slots, the other two mark a key still being written.
 //
-// Insert protocol (one key per thread): CAS w0 from 0 to the claim marker,
-// store w1..w3, then store w0 = key with release semantics.  A thread that
-// meets a claimed slot re-reads it with acquire loads, a bounded number of
-// times, until the owner publishes; then it compares the full key (equal =
-// duplicate, done; different = keep probing).  Two inserts of one key in one
-// batch therefore store it once.
+// Insert protocol (one key per thread, no fences): walk the slots with a
+// 128-bit compare-and-swap of (w0, w1) from (0, 0) to the key's first half.
+// The CAS either claims an empty slot -- then the thread stores w2 and w3 --
+// or returns the occupant's first half atomically.  If that equals the key's,
+// the thread waits, a bounded number of re-reads, until w2 and w3 are both
+// non-zero (written), then compares them: equal is a duplicate, different is
+// another key with the same first half, and the walk goes on.  Two inserts of
+// one key in one batch therefore store it once, and no reader can act on a
+// half-written slot.
+//
+// Insert of a probed batch (kvgov_insert_uncached): only the blocks at and
+// after each request's first miss, with the same per-key protocol.
 //
 // Probe: G lanes of a warp serve one request.  The lanes look up the next G
 // consecutive blocks in parallel; a ballot over the window's misses gives the
@@ -35,30 +41,30 @@ namespace {
 
 using namespace kvgov_dev;
 
-constexpr unsigned long long kClaimed = ~0ull;
 constexpr uint32_t kDefaultSpin = 1u << 23;
 std::atomic<uint32_t> g_spin_limit{kDefaultSpin};
 
-__device__ __forceinline__ unsigned long long ld_acquire(const unsigned long long *p) {
-    unsigned long long v;
-    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];\n" : "=l"(v) : "l"(p) : "memory");
-    return v;
-}
 __device__ __forceinline__ unsigned long long ld_relaxed(const unsigned long long *p) {
     unsigned long long v;
     asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];\n" : "=l"(v) : "l"(p) : "memory");
     return v;
 }
-__device__ __forceinline__ ulonglong2 ld_relaxed2(const unsigned long long *p) {
-    ulonglong2 v;
-    asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];\n" : "=l"(v.x), "=l"(v.y) : "l"(p) : "memory");
-    return v;
-}
 __device__ __forceinline__ void st_relaxed(unsigned long long *p, unsigned long long v) {
     asm volatile("st.relaxed.gpu.global.u64 [%0], %1;\n" ::"l"(p), "l"(v) : "memory");
 }
-__device__ __forceinline__ void st_release(unsigned long long *p, unsigned long long v) {
-    asm volatile("st.release.gpu.global.u64 [%0], %1;\n" ::"l"(p), "l"(v) : "memory");
+// 128-bit compare-and-swap of the 16-byte-aligned pair p[0..1]: if it holds
+// (c0, c1) it becomes (n0, n1); the previous value is returned in (o0, o1).
+__device__ __forceinline__ void cas128(unsigned long long *p, unsigned long long c0, unsigned long long c1,
+                                       unsigned long long n0, unsigned long long n1, unsigned long long &o0,
+                                       unsigned long long &o1) {
+    asm volatile("{\n\t.reg .b128 c, n, o;\n\t"
+                 "mov.b128 c, {%2, %3};\n\t"
+                 "mov.b128 n, {%4, %5};\n\t"
+                 "atom.relaxed.gpu.global.cas.b128 o, [%6], c, n;\n\t"
+                 "mov.b128 {%0, %1}, o;\n\t}"
+                 : "=l"(o0), "=l"(o1)
+                 : "l"(c0), "l"(c1), "l"(n0), "l"(n1), "l"(p)
+                 : "memory");
 }
 
 __device__ __forceinline__ unsigned long long u64_of(uint32_t lo, uint32_t hi) {
@@ -77,44 +83,60 @@ constexpr int kInsertThreads = 256;
 
 enum InsertResult { kNew = 0, kDuplicate = 1, kFull = 2, kTimeout = 3 };
 
-__device__ InsertResult insert_one(unsigned long long *slots, unsigned long long mask, const unsigned long long k[4],
+__device__ __forceinline__ InsertResult insert_one(unsigned long long *slots, unsigned long long mask, const unsigned long long k[4],
                                    uint32_t spin_limit) {
     unsigned long long pos = k[0] & mask;
     for (unsigned long long n = 0; n <= mask; ++n, pos = (pos + 1) & mask) {
         unsigned long long *slot = slots + 4 * pos;
-        // One 32-byte look at the slot.  A slot is written once (claim, tail,
-        // publish) and never changes afterwards, so a full match on these
-        // unordered reads can only be the key itself: a duplicate.
-        const ulonglong2 lo = ld_relaxed2(slot), hi = ld_relaxed2(slot + 2);
-        unsigned long long w0 = lo.x;
-        if (w0 == k[0] && lo.y == k[1] && hi.x == k[2] && hi.y == k[3]) return kDuplicate;
-        if (w0 == 0ull) {
-            const unsigned long long old = atomicCAS(slot, 0ull, kClaimed);
-            if (old == 0ull) {
-                st_relaxed(slot + 1, k[1]);
-                st_relaxed(slot + 2, k[2]);
-                st_relaxed(slot + 3, k[3]);
-                st_release(slot, k[0]);
-                return kNew;
-            }
-            w0 = old;
+        unsigned long long o0, o1;
+        cas128(slot, 0ull, 0ull, k[0], k[1], o0, o1);
+        if ((o0 | o1) == 0ull) {                 // claimed: write the second half
+            st_relaxed(slot + 2, k[2]);
+            st_relaxed(slot + 3, k[3]);
+            return kNew;
         }
-        if (w0 == kClaimed || w0 == k[0]) {
-            // claimed but not yet published, or our first word with a tail
-            // that may have been read before it was written: wait for the
-            // publication (bounded) and compare again with acquire ordering
-            uint32_t spins = 0;
-            while ((w0 = ld_acquire(slot)) == kClaimed) {
-                if (++spins >= spin_limit) return kTimeout;
-                __nanosleep(100);
-            }
-            if (w0 == k[0]) {
-                const ulonglong2 t = ld_relaxed2(slot + 2);
-                if (ld_relaxed(slot + 1) == k[1] && t.x == k[2] && t.y == k[3]) return kDuplicate;
-            }
+        if (o0 != k[0] || o1 != k[1]) continue;  // another key
+        unsigned long long w2 = ld_relaxed(slot + 2), w3 = ld_relaxed(slot + 3);
+        for (uint32_t spins = 0; w2 == 0ull || w3 == 0ull; ++spins) {
+            if (spins >= spin_limit) return kTimeout;
+            __nanosleep(100);
+            w2 = ld_relaxed(slot + 2);
+            w3 = ld_relaxed(slot + 3);
         }
+        if (w2 == k[2] && w3 == k[3]) return kDuplicate;
     }
     return kFull;
+}
+
+// Insert counts: warp reduction, shared-memory accumulation, and the CTA's
+// last warp to finish publishes them (no barrier: early warps just exit).
+__device__ __forceinline__ void publish_counts(unsigned my_new, unsigned my_flags, unsigned *s_new, unsigned *s_flags,
+                                               unsigned *s_done, unsigned long long *n_new, uint32_t *status) {
+    const unsigned w_new = __reduce_add_sync(0xffffffffu, my_new);
+    const unsigned w_flags = __reduce_or_sync(0xffffffffu, my_flags);
+    if ((threadIdx.x & 31) == 0) {
+        if (w_new) atomicAdd(s_new, w_new);
+        if (w_flags) atomicOr(s_flags, w_flags);
+        __threadfence_block();
+        if (atomicAdd(s_done, 1u) == blockDim.x / 32 - 1) {
+            const unsigned t_new = atomicAdd(s_new, 0u), t_flags = atomicOr(s_flags, 0u);
+            if (t_new && n_new) atomicAdd(n_new, (unsigned long long)t_new);
+            if (t_flags && status) atomicOr(status, t_flags);
+        }
+    }
+}
+
+__device__ __forceinline__ void count_insert(InsertResult res, unsigned &my_new, unsigned &my_flags) {
+    switch (res) {
+    case kNew: ++my_new; break;
+    case kDuplicate: break;
+    case kFull: my_flags |= KVGOV_F_TABLE_FULL; break;
+    default: my_flags |= KVGOV_F_TIMEOUT; break;
+    }
+}
+
+__device__ __forceinline__ bool key_reserved(const unsigned long long k[4]) {
+    return (k[0] | k[1]) == 0ull || k[2] == 0ull || k[3] == 0ull;
 }
 
 __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long long *__restrict__ slots,
@@ -130,31 +152,13 @@ __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long lo
     for (long long i = (long long)blockIdx.x * kInsertThreads + threadIdx.x; i < n_keys; i += stride) {
         const uint4 a = __ldg(keys + 2 * i), b = __ldg(keys + 2 * i + 1);
         const unsigned long long k[4] = {u64_of(a.x, a.y), u64_of(a.z, a.w), u64_of(b.x, b.y), u64_of(b.z, b.w)};
-        if (k[0] == 0ull || k[0] == kClaimed) {
+        if (key_reserved(k)) {
             my_flags |= KVGOV_F_SENTINEL;
             continue;
         }
-        switch (insert_one(slots, mask, k, spin_limit)) {
-        case kNew: ++my_new; break;
-        case kDuplicate: break;
-        case kFull: my_flags |= KVGOV_F_TABLE_FULL; break;
-        default: my_flags |= KVGOV_F_TIMEOUT; break;
-        }
+        count_insert(insert_one(slots, mask, k, spin_limit), my_new, my_flags);
     }
-    // Counts: warp reduction, shared-memory accumulation, and the CTA's last
-    // warp to finish publishes them (no barrier: early warps just exit).
-    const unsigned w_new = __reduce_add_sync(0xffffffffu, my_new);
-    const unsigned w_flags = __reduce_or_sync(0xffffffffu, my_flags);
-    if ((threadIdx.x & 31) == 0) {
-        if (w_new) atomicAdd(&s_new, w_new);
-        if (w_flags) atomicOr(&s_flags, w_flags);
-        __threadfence_block();
-        if (atomicAdd(&s_done, 1u) == kInsertThreads / 32 - 1) {
-            const unsigned t_new = atomicAdd(&s_new, 0u), t_flags = atomicOr(&s_flags, 0u);
-            if (t_new && n_new) atomicAdd(n_new, (unsigned long long)t_new);
-            if (t_flags) atomicOr(status, t_flags);
-        }
-    }
+    publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
 }
 
 // ---------------------------------------------------------------------------
@@ -163,14 +167,14 @@ constexpr int kProbeThreads = 256;
 // Is the 32-byte key q in the table?  Reads slots through the read-only path:
 // the table does not change during a probe.
 __device__ __forceinline__ bool lookup(const uint4 *__restrict__ slots, unsigned long long mask, uint4 q0, uint4 q1) {
-    const unsigned long long k0 = u64_of(q0.x, q0.y);
-    if (k0 == 0ull || k0 == kClaimed) return false;   // such keys are never stored
+    const unsigned long long k0 = u64_of(q0.x, q0.y), k1 = u64_of(q0.z, q0.w);
+    if ((k0 | k1) == 0ull || u64_of(q1.x, q1.y) == 0ull || u64_of(q1.z, q1.w) == 0ull)
+        return false;                               // reserved keys are never stored
     unsigned long long pos = k0 & mask;
     for (unsigned long long n = 0; n <= mask; ++n, pos = (pos + 1) & mask) {
         const uint4 a = __ldg(slots + 2 * pos);
-        const unsigned long long w0 = u64_of(a.x, a.y);
-        if (w0 == 0ull) return false;
-        if (w0 == k0 && a.z == q0.z && a.w == q0.w) {
+        if ((a.x | a.y | a.z | a.w) == 0u) return false;   // empty slot ends the walk
+        if (a.x == q0.x && a.y == q0.y && a.z == q0.z && a.w == q0.w) {
             const uint4 b = __ldg(slots + 2 * pos + 1);
             if (b.x == q1.x && b.y == q1.y && b.z == q1.z && b.w == q1.w) return true;
         }
@@ -226,6 +230,43 @@ __global__ void __launch_bounds__(kProbeThreads) probe_kernel(const uint4 *__res
     }
 }
 
+// Insert every request's blocks from its cached-prefix length on (the output
+// of kvgov_probe): the blocks before it were found in the table, and a table
+// only grows, so inserting them would change nothing.  G lanes per request.
+template <int G>
+__global__ void __launch_bounds__(kInsertThreads) insert_uncached_kernel(
+    unsigned long long *__restrict__ slots, unsigned long long mask, const uint4 *__restrict__ digests,
+    const int64_t *__restrict__ blk_off, int32_t n_req, const int32_t *__restrict__ prefix_blocks,
+    unsigned long long *n_new, uint32_t *status, uint32_t spin_limit) {
+    __shared__ unsigned int s_new, s_flags, s_done;
+    if (threadIdx.x == 0) { s_new = 0; s_flags = 0; s_done = 0; }
+    __syncthreads();
+    constexpr int kSegs = 32 / G;
+    const int sl = (threadIdx.x & 31) % G;
+    const long long total_segs = (long long)gridDim.x * (kInsertThreads / G);
+    unsigned my_new = 0, my_flags = 0;
+    for (long long r = ((long long)blockIdx.x * kInsertThreads + threadIdx.x) / G; r < n_req; r += total_segs) {
+        const long long base = blk_off[r], nb = blk_off[r + 1] - base;
+        if (nb < 0 || base < 0 || base + nb > blk_off[n_req]) {
+            if (sl == 0) my_flags |= KVGOV_F_BADINDEX;
+            continue;
+        }
+        long long L = prefix_blocks[r];
+        if (L < 0) L = 0;
+        for (long long j = L + sl; j < nb; j += G) {
+            const uint4 a = __ldg(digests + 2 * (base + j)), b = __ldg(digests + 2 * (base + j) + 1);
+            const unsigned long long k[4] = {u64_of(a.x, a.y), u64_of(a.z, a.w), u64_of(b.x, b.y), u64_of(b.z, b.w)};
+            if (key_reserved(k)) {
+                my_flags |= KVGOV_F_SENTINEL;
+                continue;
+            }
+            count_insert(insert_one(slots, mask, k, spin_limit), my_new, my_flags);
+        }
+    }
+    (void)kSegs;
+    publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
+}
+
 }  // namespace
 
 extern "C" int kvgov_table_init(uint8_t *d_slots, uint64_t capacity, kvgov_stream_t stream) {
@@ -270,6 +311,23 @@ extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint
     return kvgov_host::launch_status();
 }
 
+extern "C" int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,
+                                     const int64_t *d_blk_off, int32_t n_req, const int32_t *d_prefix_blocks,
+                                     unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream) {
+    using kvgov_host::aligned16;
+    if (!d_slots || !aligned16(d_slots) || !kvgov_host::pow2_capacity(capacity) || n_req < 0 || !d_status)
+        return KVGOV_EINVAL;
+    if (n_req == 0) return KVGOV_OK;
+    if (!d_digests || !aligned16(d_digests) || !d_blk_off || !d_prefix_blocks) return KVGOV_EINVAL;
+    constexpr int G = 8;
+    long long grid = ((long long)n_req * G + kInsertThreads - 1) / kInsertThreads;
+    if (grid > 152ll * 64) grid = 152ll * 64;
+    insert_uncached_kernel<G><<<(unsigned)grid, kInsertThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+        reinterpret_cast<unsigned long long *>(d_slots), capacity - 1, reinterpret_cast<const uint4 *>(d_digests),
+        d_blk_off, n_req, d_prefix_blocks, d_n_new, d_status, g_spin_limit.load());
+    return kvgov_host::launch_status();
+}
+
 extern "C" uint32_t kvgov_set_spin_limit(uint32_t limit) {
     return g_spin_limit.exchange(limit == 0 ? kDefaultSpin : limit);
 }
@@ -280,9 +338,9 @@ extern "C" const char *kvgov_status_string(int status) {
     case KVGOV_EINVAL: return "KVGOV_EINVAL: invalid argument";
     case KVGOV_ECUDA: return "KVGOV_ECUDA: kernel launch failed";
     case (int)KVGOV_F_BADINDEX: return "KVGOV_F_BADINDEX: index or offset out of range";
-    case (int)KVGOV_F_SENTINEL: return "KVGOV_F_SENTINEL: reserved key (first 8 bytes all 0x00 or all 0xFF)";
+    case (int)KVGOV_F_SENTINEL: return "KVGOV_F_SENTINEL: reserved key (bytes 0-15, 16-23 or 24-31 all zero)";
     case (int)KVGOV_F_TABLE_FULL: return "KVGOV_F_TABLE_FULL: no free slot";
-    case (int)KVGOV_F_TIMEOUT: return "KVGOV_F_TIMEOUT: gave up waiting for a claimed slot";
+    case (int)KVGOV_F_TIMEOUT: return "KVGOV_F_TIMEOUT: gave up waiting for a slot's key to be written";
     default: return "KVGOV: unknown status";
     }
 }

@@ -56,10 +56,11 @@ def _load():
         L.kvgov_table_init.argtypes = [_p, ctypes.c_uint64, _p]
         L.kvgov_insert.argtypes = [_p, ctypes.c_uint64, _p, ctypes.c_int64, _p, _p, _p]
         L.kvgov_probe.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p]
+        L.kvgov_insert_uncached.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p, _p]
         L.kvgov_set_spin_limit.argtypes = [ctypes.c_uint32]
         L.kvgov_set_spin_limit.restype = ctypes.c_uint32
         for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
-                   "kvgov_insert", "kvgov_probe"):
+                   "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached"):
             getattr(L, fn).restype = ctypes.c_int
         _lib = L
         return L
@@ -205,6 +206,19 @@ def probe(slots: torch.Tensor, digests: torch.Tensor, blk_off: torch.Tensor,
                              _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_probe")
     return prefix_blocks
+
+
+def insert_uncached(slots: torch.Tensor, digests: torch.Tensor, blk_off: torch.Tensor, prefix_blocks: torch.Tensor,
+                    status: torch.Tensor, n_new: torch.Tensor | None = None, stream=None):
+    """Insert each request's blocks from prefix_blocks[r] on (after probe)."""
+    n = blk_off.numel() - 1
+    _check(lib().kvgov_insert_uncached(_dev(slots, torch.uint8, "slots"), slots.shape[0],
+                                       _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(blk_off),
+                                       _dev(blk_off, torch.int64, "blk_off"), n,
+                                       _dev(prefix_blocks, torch.int32, "prefix_blocks"),
+                                       _dev(n_new, torch.int64, "n_new", True), _dev(status, torch.int32, "status"),
+                                       _stream(stream)),
+           "kvgov_insert_uncached")
 
 
 def set_spin_limit(limit: int) -> int:

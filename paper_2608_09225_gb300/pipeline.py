@@ -68,6 +68,10 @@ class PrefixCache:
         K.table_init(self.slots, self.stream)
         self.derive_salts()
 
+    def set_secret(self, secret: bytes):
+        """Change the server secret; salts are derived again on the next serve."""
+        self.secret = bytes(secret)
+
     # -- individual steps ------------------------------------------------
     def derive_salts(self):
         K.derive_salts(self.secret, self.ids, self.id_off, self.salts, self.status, self.stream)
@@ -91,16 +95,19 @@ class PrefixCache:
     def probe(self, digests, blk_off, prefix_blocks=None):
         return K.probe(self.slots, digests, blk_off, prefix_blocks, self.status, self.stream)
 
+    def insert_uncached(self, digests, blk_off, prefix_blocks):
+        K.insert_uncached(self.slots, digests, blk_off, prefix_blocks, self.status, self.n_new, self.stream)
+
     # -- one serving step -------------------------------------------------
     def serve(self, mode: int, b: DeviceBatch, bufs: dict | None = None, derive_salts: bool = True):
-        """Salts, blocking, chain, probe, insert for one batch.  Returns
-        (prefix_blocks, digests, blk_off), all on the device."""
+        """Salts, blocking, chain, probe, and insert of the uncached blocks for
+        one batch.  Returns (prefix_blocks, digests, blk_off), on the device."""
         bufs = bufs if bufs is not None else {}
         if derive_salts:
             self.derive_salts()
         blk_off, digests = self.hash(mode, b, bufs.get("blk_off"), bufs.get("digests"))
         prefix = self.probe(digests, blk_off, bufs.get("prefix"))
-        self.insert(digests)
+        self.insert_uncached(digests, blk_off, prefix)
         return prefix, digests, blk_off
 
     def check_status(self):

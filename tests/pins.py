@@ -293,8 +293,8 @@ def pin_prefix_brute_force():
 
 
 def pin_set_semantics():
-    """Set insert: duplicates are no-ops in any order; reserved first words
-    (all 0x00 / all 0xFF) are refused and flagged."""
+    """Set insert: duplicates are no-ops in any order; reserved keys (bytes
+    0-15, 16-23 or 24-31 all zero) are refused and flagged."""
     rng = np.random.default_rng(18)
     keys = rng.integers(0, 256, (50, 32), dtype=np.uint8)
     keys[:, 0] |= 1
@@ -304,13 +304,21 @@ def pin_set_semantics():
     assert n_new == 50 and not flag
     n_new, flag = ks.insert(keys[:20])
     assert n_new == 0 and not flag
-    bad = np.zeros((3, 32), np.uint8)
-    bad[1, :8] = 255
-    bad[2, 8:] = 7            # first 8 bytes zero, rest not
+    bad = np.full((4, 32), 7, np.uint8)
+    bad[0, :] = 0               # all zero
+    bad[1, :16] = 0             # first half zero
+    bad[2, 16:24] = 0           # third word zero
+    bad[3, 24:] = 0             # fourth word zero
     n_new, flag = ks.insert(bad)
     assert n_new == 0 and flag and ks.n == 50
+    ok = np.full((3, 32), 7, np.uint8)
+    ok[0, :8] = 0               # a zero first word alone is storable
+    ok[1, 8:16] = 0
+    ok[2, :8] = 255
+    n_new, flag = ks.insert(ok)
+    assert n_new == 3 and not flag and ks.n == 53
     ks2 = oracle.KeySet(1)
-    ks2.insert(batch[rng.permutation(len(batch))])
+    ks2.insert(np.concatenate([ok, batch])[rng.permutation(len(batch) + 3)])
     assert (ks2.contents() == ks.contents()).all()
 
 

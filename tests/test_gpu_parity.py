@@ -169,8 +169,7 @@ def keys_np(n, seed):
 
 def table_contents(slots):
     s = slots.cpu().numpy()
-    w0 = s[:, :8].view(np.uint64).reshape(-1)
-    full = s[(w0 != 0) & (w0 != np.uint64(0xFFFFFFFFFFFFFFFF))]
+    full = s[s[:, :16].any(axis=1)]          # first 16 bytes zero = empty slot
     return {r.tobytes() for r in full}
 
 
@@ -201,10 +200,13 @@ def test_insert_heavy_in_batch_duplicates(kv):
 
 
 def test_insert_reserved_keys(kv):
-    k = keys_np(10, 4)
+    k = keys_np(12, 4)
     k[3, :] = 0                 # all zero
-    k[5, :8] = 255              # first word all ones
-    k[7, :8] = 0                # first word zero, rest not
+    k[5, :16] = 0               # first half zero
+    k[7, 16:24] = 0             # third word zero
+    k[9, 24:] = 0               # fourth word zero
+    k[10, :8] = 0               # first word zero alone: storable
+    k[11, :8] = 255             # first word all ones: storable
     slots = kv.new_table(64)
     st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
     kv.insert(slots, dev(k), st, n_new)
@@ -212,8 +214,11 @@ def test_insert_reserved_keys(kv):
     assert int(st.item()) == kv.F_SENTINEL
     ks = oracle.KeySet(1)
     n_ref, flagged = ks.insert(k)
-    assert flagged and int(n_new.item()) == n_ref == 7
+    assert flagged and int(n_new.item()) == n_ref == 8
     assert table_contents(slots) == {r.tobytes() for r in ks.contents()}
+    pre = kv.probe(slots, dev(k), dev(np.arange(13, dtype=np.int64)))
+    torch.cuda.synchronize()
+    assert list(pre.cpu().numpy()) == [0 if oracle.key_reserved(r.tobytes()) else 1 for r in k]
 
 
 def test_table_full(kv):
@@ -226,15 +231,16 @@ def test_table_full(kv):
     assert int(n_new.item()) == 32 and len(table_contents(slots)) == 32
 
 
-def test_insert_wait_times_out_on_a_claim_nobody_publishes(kv):
-    """A slot left claimed (first word all ones) by an insert that never
-    publishes: a later insert homed there waits a bounded number of times,
-    reports KVGOV_F_TIMEOUT and returns; probes treat the slot as occupied."""
+def test_insert_wait_times_out_on_a_slot_nobody_finishes(kv):
+    """A slot holding a key's first 16 bytes whose second half is never
+    written (as if its writer stopped): an insert of that key waits a bounded
+    number of times, reports KVGOV_F_TIMEOUT and returns; a probe of the key
+    does not match the half-written slot."""
     cap = 64
     k = keys_np(1, 6)
     home = int(k[0, :8].view(np.uint64)[0]) & (cap - 1)
     slots = kv.new_table(cap)
-    slots[home, :8] = 255
+    slots[home, :16] = torch.from_numpy(k[0, :16].copy()).to(DEV)
     st = status_tensor()
     prev = kv.set_spin_limit(1000)
     try:
@@ -269,6 +275,42 @@ def test_probe_matches_oracle(kv, cap_log2):
     ks = oracle.KeySet(1)
     ks.insert(pool[member])
     assert (pre.cpu().numpy() == ks.prefix_blocks(digests, off)).all()
+
+
+@pytest.mark.parametrize("cap_log2", [6, 12, 16])
+def test_insert_uncached_after_probe_matches_insert_all(kv, cap_log2):
+    """Probe, then insert each request's suffix from its prefix length: the
+    set and the count of new keys equal those of inserting every digest."""
+    rng = np.random.default_rng(100 + cap_log2)
+    pool = keys_np(min(1 << (cap_log2 - 1), 3000), cap_log2 + 200)
+    nb = rng.integers(0, 40, 2000)
+    nb[:4] = [0, 1, 39, 16]
+    off = np.concatenate([[0], np.cumsum(nb)]).astype(np.int64)
+    digests = pool[rng.integers(0, len(pool), int(off[-1]))]
+    member = rng.random(len(pool)) < 0.5
+    slots = kv.new_table(1 << cap_log2)
+    st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
+    kv.insert(slots, dev(pool[member]), st)
+    d_dig, d_off = dev(digests), dev(off)
+    pre = kv.probe(slots, d_dig, d_off, status=st)
+    kv.insert_uncached(slots, d_dig, d_off, pre, st, n_new)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    ks = oracle.KeySet(1)
+    ks.insert(pool[member])
+    assert (pre.cpu().numpy() == ks.prefix_blocks(digests, off)).all()
+    n_ref, _ = ks.insert(digests)
+    assert int(n_new.item()) == n_ref
+    assert table_contents(slots) == {r.tobytes() for r in ks.contents()}
+
+
+def test_insert_uncached_bad_offsets_flagged(kv):
+    slots = kv.new_table(64)
+    st = status_tensor()
+    kv.insert_uncached(slots, dev(keys_np(4, 7)), dev(np.array([0, 4, 2], np.int64)),
+                       dev(np.zeros(2, np.int32)), st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & kv.F_BADINDEX
 
 
 def test_probe_empty_and_bad_offsets(kv):

@@ -33,7 +33,8 @@ def declared_functions():
 def test_header_declares_the_boundary():
     names = declared_functions()
     for want in ("kvgov_derive_salts", "kvgov_block_offsets", "kvgov_chain_hash", "kvgov_table_init",
-                 "kvgov_insert", "kvgov_probe", "kvgov_status_string", "kvgov_set_spin_limit"):
+                 "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_status_string",
+                 "kvgov_set_spin_limit"):
         assert want in names
 
 
@@ -90,6 +91,11 @@ def test_host_validation_rejects_bad_arguments(libkv):
     pr.argtypes = [p, ctypes.c_uint64, p, p, ctypes.c_int32, p, p, p]
     assert pr(fake, 100, fake, fake, 3, fake, None, None) == 1
     assert pr(fake, 64, odd, fake, 3, fake, None, None) == 1
+    iu = libkv.kvgov_insert_uncached
+    iu.argtypes = [p, ctypes.c_uint64, p, p, ctypes.c_int32, p, p, p, p]
+    assert iu(fake, 64, fake, fake, 3, fake, None, None, None) == 1     # status is required
+    assert iu(fake, 64, odd, fake, 3, fake, None, fake, None) == 1      # misaligned digests
+    assert iu(fake, 64, fake, fake, 0, None, None, fake, None) == 0     # empty batch
     sa = libkv.kvgov_derive_salts
     sa.argtypes = [p, ctypes.c_size_t, p, p, ctypes.c_int32, p, p, p]
     assert sa(None, 1025, fake, fake, 3, fake, None, None) == 1
@@ -144,7 +150,7 @@ def test_workload_structure():
         assert (pt[r, :c] == prt[src[r], :c]).all()
         assert pw.batch.principal[r] == pw.prior.principal[src[r]]
     keys = pw.random_keys
-    assert not (np.all(keys[:, :8] == 0, axis=1) | np.all(keys[:, :8] == 255, axis=1)).any()
+    assert not any(oracle.key_reserved(k.tobytes()) for k in keys)
     lw = W.make("long", n_req=4)
     assert lw.batch.tokens.shape[0] == 4 * 32768 and (lw.batch.boundary_tok == 64).all()
 
@@ -156,7 +162,10 @@ def test_full_size_shapes():
 
 
 def test_oracle_key_reserved_rule():
+    one = b"\x01" * 8
     assert oracle.key_reserved(bytes(32))
-    assert oracle.key_reserved(b"\xff" * 8 + b"\x01" * 24)
-    assert oracle.key_reserved(bytes(8) + b"\x01" * 24)
-    assert not oracle.key_reserved(b"\x01" + bytes(31))
+    assert oracle.key_reserved(bytes(16) + one + one)
+    assert oracle.key_reserved(one + one + bytes(8) + one)
+    assert oracle.key_reserved(one + one + one + bytes(8))
+    assert not oracle.key_reserved(bytes(8) + one + one + one)
+    assert not oracle.key_reserved(b"\xff" * 8 + one + one + one)
