@@ -44,6 +44,8 @@ typedef struct CUstream_st *kvgov_stream_t;
 #define KVGOV_DIGEST_BYTES 32      /* SHA-256 digest and table key size       */
 #define KVGOV_MAX_SECRET 1024      /* longest HMAC key kvgov_derive_salts takes */
 #define KVGOV_MIN_CAPACITY 32      /* smallest table capacity (slots)         */
+#define KVGOV_PROBE_WINDOW 1024    /* a key lives within this many slots of its
+                                      home slot (fewer if the table is smaller) */
 
 /* Return codes (host-detected). */
 #define KVGOV_OK 0
@@ -58,7 +60,8 @@ typedef struct CUstream_st *kvgov_stream_t;
                                       24-31 all zero) was given to an insert; it
                                       is skipped (these values mark empty slots
                                       and keys still being written)           */
-#define KVGOV_F_TABLE_FULL 0x40u   /* kvgov_insert found no free slot for a key */
+#define KVGOV_F_TABLE_FULL 0x40u   /* an insert found no free slot in a key's
+                                      probe window; the key is not stored     */
 #define KVGOV_F_TIMEOUT 0x80u      /* an insert gave up waiting for another
                                       thread to finish writing a slot's key   */
 
@@ -147,7 +150,11 @@ int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t *d_tok_off
  * `capacity` 32-byte slots (capacity a power of two >= KVGOV_MIN_CAPACITY,
  * d_slots 16-byte aligned).  A slot is empty when its first 16 bytes are
  * zero; a key's home slot is its first 8 bytes read as a little-endian u64,
- * modulo capacity, with linear probing.  Keys are stored verbatim and claimed
+ * modulo capacity, with linear probing inside a window of
+ * min(capacity, KVGOV_PROBE_WINDOW) slots: an insert that finds no free slot
+ * in its window reports KVGOV_F_TABLE_FULL (at load factor 0.5 a walk longer
+ * than a few dozen slots practically never happens), and lookups stop at the
+ * end of the window.  Keys are stored verbatim and claimed
  * with a 128-bit compare-and-swap of their first 16 bytes, so keys whose
  * bytes 0-15, 16-23 or 24-31 are all zero cannot be stored
  * (KVGOV_F_SENTINEL); for SHA-256 digests that happens with probability

@@ -10,14 +10,20 @@
 //
 // Slot encoding: the key verbatim as four little-endian u64 words w0..w3.
 // (w0, w1) == 0 marks an empty slot.  Home slot = w0 & (capacity - 1);
-// collisions go to the next slot (linear probing, wrapping).  Keys with
+// collisions go to the next slot (linear probing, wrapping) within a window
+// of min(capacity, KVGOV_PROBE_WINDOW) slots: an insert that finds no free
+// slot in its key's window fails (table full), so a lookup can stop at the
+// end of the window too.  Every walk is bounded, even in a full table.  Keys with
 // (w0, w1) == 0, w2 == 0 or w3 == 0 are refused (reserved): the first marks
 // empty slots, the other two mark a key still being written.
 //
-// Insert protocol (one key per thread, no fences): walk the slots with a
-// 128-bit compare-and-swap of (w0, w1) from (0, 0) to the key's first half.
-// The CAS either claims an empty slot -- then the thread stores w2 and w3 --
-// or returns the occupant's first half atomically.  If that equals the key's,
+// Insert protocol (one key per thread, no fences): walk the slots.  A plain
+// read whose two first-half words are both non-zero is final (the half is
+// written once, from zero, so a torn read shows a zero word): another key
+// means walk on, the key's own first half means compare the second half.
+// Any other slot gets a 128-bit compare-and-swap of (w0, w1) from (0, 0) to
+// the key's first half, which either claims an empty slot -- then the thread
+// stores w2 and w3 -- or returns the occupant's first half atomically.  If that equals the key's,
 // the thread waits, a bounded number of re-reads, until w2 and w3 are both
 // non-zero (written), then compares them: equal is a duplicate, different is
 // another key with the same first half, and the walk goes on.  Two inserts of
@@ -41,6 +47,20 @@ namespace {
 
 using namespace kvgov_dev;
 
+// Insert variants, chosen at build time (python -m
+// paper_2608_09225_gb300.variants --insert times them): KVGOV_INSERT_LOOK
+// reads a slot before using an atomic on it (default: it turns the step after
+// a cache flush, where every request inserts the same shared-prefix blocks,
+// from ~377 to ~70 us for +5 us on an ordinary step); KVGOV_INSERT_DEDUP
+// elects one lane per distinct key within a warp (off: it costs more on an
+// ordinary step than it saves after a flush).
+#ifndef KVGOV_INSERT_LOOK
+#define KVGOV_INSERT_LOOK 1
+#endif
+#ifndef KVGOV_INSERT_DEDUP
+#define KVGOV_INSERT_DEDUP 0
+#endif
+
 constexpr uint32_t kDefaultSpin = 1u << 23;
 std::atomic<uint32_t> g_spin_limit{kDefaultSpin};
 
@@ -49,6 +69,13 @@ __device__ __forceinline__ unsigned long long ld_relaxed(const unsigned long lon
     asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];\n" : "=l"(v) : "l"(p) : "memory");
     return v;
 }
+#if KVGOV_INSERT_LOOK
+__device__ __forceinline__ ulonglong2 ld_relaxed2(const unsigned long long *p) {
+    ulonglong2 v;
+    asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];\n" : "=l"(v.x), "=l"(v.y) : "l"(p) : "memory");
+    return v;
+}
+#endif
 __device__ __forceinline__ void st_relaxed(unsigned long long *p, unsigned long long v) {
     asm volatile("st.relaxed.gpu.global.u64 [%0], %1;\n" ::"l"(p), "l"(v) : "memory");
 }
@@ -67,6 +94,10 @@ __device__ __forceinline__ void cas128(unsigned long long *p, unsigned long long
                  : "memory");
 }
 
+__device__ __forceinline__ unsigned long long probe_window(unsigned long long mask) {
+    return mask < KVGOV_PROBE_WINDOW - 1 ? mask + 1 : (unsigned long long)KVGOV_PROBE_WINDOW;
+}
+
 __device__ __forceinline__ unsigned long long u64_of(uint32_t lo, uint32_t hi) {
     return (unsigned long long)lo | ((unsigned long long)hi << 32);
 }
@@ -83,19 +114,32 @@ constexpr int kInsertThreads = 256;
 
 enum InsertResult { kNew = 0, kDuplicate = 1, kFull = 2, kTimeout = 3 };
 
-__device__ __forceinline__ InsertResult insert_one(unsigned long long *slots, unsigned long long mask, const unsigned long long k[4],
-                                   uint32_t spin_limit) {
+__device__ __forceinline__ InsertResult insert_one(unsigned long long *slots, unsigned long long mask,
+                                                   const unsigned long long k[4], uint32_t spin_limit) {
+    const unsigned long long window = probe_window(mask);
     unsigned long long pos = k[0] & mask;
-    for (unsigned long long n = 0; n <= mask; ++n, pos = (pos + 1) & mask) {
+    for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
         unsigned long long *slot = slots + 4 * pos;
-        unsigned long long o0, o1;
-        cas128(slot, 0ull, 0ull, k[0], k[1], o0, o1);
-        if ((o0 | o1) == 0ull) {                 // claimed: write the second half
-            st_relaxed(slot + 2, k[2]);
-            st_relaxed(slot + 3, k[3]);
-            return kNew;
+        unsigned long long o0 = 0ull, o1 = 0ull;
+#if KVGOV_INSERT_LOOK
+        // Look first.  A slot's first half is written once, from (0, 0) to
+        // its final value, so a plain read racing that write can only show a
+        // zero word; a read with both words non-zero is the final value and
+        // needs no atomic (another key: walk on; our first half: compare).
+        const ulonglong2 seen = ld_relaxed2(slot);
+        o0 = seen.x;
+        o1 = seen.y;
+        if (o0 == 0ull || o1 == 0ull)
+#endif
+        {
+            cas128(slot, 0ull, 0ull, k[0], k[1], o0, o1);
+            if ((o0 | o1) == 0ull) {                 // claimed: write the second half
+                st_relaxed(slot + 2, k[2]);
+                st_relaxed(slot + 3, k[3]);
+                return kNew;
+            }
         }
-        if (o0 != k[0] || o1 != k[1]) continue;  // another key
+        if (o0 != k[0] || o1 != k[1]) continue;      // another key
         unsigned long long w2 = ld_relaxed(slot + 2), w3 = ld_relaxed(slot + 3);
         for (uint32_t spins = 0; w2 == 0ull || w3 == 0ull; ++spins) {
             if (spins >= spin_limit) return kTimeout;
@@ -106,6 +150,22 @@ __device__ __forceinline__ InsertResult insert_one(unsigned long long *slots, un
         if (w2 == k[2] && w3 == k[3]) return kDuplicate;
     }
     return kFull;
+}
+
+// Insert from the lanes of a warp named in `inserting` (all of which make
+// this call together): lanes holding the same 32 bytes elect their lowest
+// lane to insert; the others are duplicates of that insert.
+__device__ __forceinline__ InsertResult insert_warp_dedup(unsigned long long *slots, unsigned long long mask,
+                                                         const unsigned long long k[4], uint32_t spin_limit,
+                                                         unsigned inserting) {
+#if KVGOV_INSERT_DEDUP
+    const unsigned same = __match_any_sync(inserting, k[0]) & __match_any_sync(inserting, k[1]) &
+                          __match_any_sync(inserting, k[2]) & __match_any_sync(inserting, k[3]);
+    if ((threadIdx.x & 31) != (unsigned)(__ffs(same) - 1)) return kDuplicate;
+#else
+    (void)inserting;
+#endif
+    return insert_one(slots, mask, k, spin_limit);
 }
 
 // Insert counts: warp reduction, shared-memory accumulation, and the CTA's
@@ -148,15 +208,24 @@ __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long lo
     if (threadIdx.x == 0) { s_new = 0; s_flags = 0; s_done = 0; }
     __syncthreads();
     const long long stride = (long long)gridDim.x * kInsertThreads;
+    const int lane = threadIdx.x & 31;
     unsigned int my_new = 0, my_flags = 0;
-    for (long long i = (long long)blockIdx.x * kInsertThreads + threadIdx.x; i < n_keys; i += stride) {
-        const uint4 a = __ldg(keys + 2 * i), b = __ldg(keys + 2 * i + 1);
-        const unsigned long long k[4] = {u64_of(a.x, a.y), u64_of(a.z, a.w), u64_of(b.x, b.y), u64_of(b.z, b.w)};
-        if (key_reserved(k)) {
-            my_flags |= KVGOV_F_SENTINEL;
-            continue;
+    // warp-uniform trip count, so that the lanes inserting in one iteration
+    // are known exactly (the ballot) and meet in insert_warp_dedup
+    for (long long i0 = (long long)blockIdx.x * kInsertThreads + (threadIdx.x & ~31); i0 < n_keys; i0 += stride) {
+        const long long i = i0 + lane;
+        unsigned long long k[4] = {0ull, 0ull, 0ull, 0ull};
+        bool mine = i < n_keys;
+        if (mine) {
+            const uint4 a = __ldg(keys + 2 * i), b = __ldg(keys + 2 * i + 1);
+            k[0] = u64_of(a.x, a.y); k[1] = u64_of(a.z, a.w); k[2] = u64_of(b.x, b.y); k[3] = u64_of(b.z, b.w);
+            if (key_reserved(k)) {
+                my_flags |= KVGOV_F_SENTINEL;
+                mine = false;
+            }
         }
-        count_insert(insert_one(slots, mask, k, spin_limit), my_new, my_flags);
+        const unsigned inserting = __ballot_sync(0xffffffffu, mine);
+        if (mine) count_insert(insert_warp_dedup(slots, mask, k, spin_limit, inserting), my_new, my_flags);
     }
     publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
 }
@@ -170,8 +239,9 @@ __device__ __forceinline__ bool lookup(const uint4 *__restrict__ slots, unsigned
     const unsigned long long k0 = u64_of(q0.x, q0.y), k1 = u64_of(q0.z, q0.w);
     if ((k0 | k1) == 0ull || u64_of(q1.x, q1.y) == 0ull || u64_of(q1.z, q1.w) == 0ull)
         return false;                               // reserved keys are never stored
+    const unsigned long long window = probe_window(mask);
     unsigned long long pos = k0 & mask;
-    for (unsigned long long n = 0; n <= mask; ++n, pos = (pos + 1) & mask) {
+    for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
         const uint4 a = __ldg(slots + 2 * pos);
         if ((a.x | a.y | a.z | a.w) == 0u) return false;   // empty slot ends the walk
         if (a.x == q0.x && a.y == q0.y && a.z == q0.z && a.w == q0.w) {
@@ -242,28 +312,42 @@ __global__ void __launch_bounds__(kInsertThreads) insert_uncached_kernel(
     if (threadIdx.x == 0) { s_new = 0; s_flags = 0; s_done = 0; }
     __syncthreads();
     constexpr int kSegs = 32 / G;
-    const int sl = (threadIdx.x & 31) % G;
-    const long long total_segs = (long long)gridDim.x * (kInsertThreads / G);
+    const int lane = threadIdx.x & 31, seg = lane / G, sl = lane % G;
+    const long long warps_total = (long long)gridDim.x * (kInsertThreads / 32);
     unsigned my_new = 0, my_flags = 0;
-    for (long long r = ((long long)blockIdx.x * kInsertThreads + threadIdx.x) / G; r < n_req; r += total_segs) {
-        const long long base = blk_off[r], nb = blk_off[r + 1] - base;
-        if (nb < 0 || base < 0 || base + nb > blk_off[n_req]) {
-            if (sl == 0) my_flags |= KVGOV_F_BADINDEX;
-            continue;
-        }
-        long long L = prefix_blocks[r];
-        if (L < 0) L = 0;
-        for (long long j = L + sl; j < nb; j += G) {
-            const uint4 a = __ldg(digests + 2 * (base + j)), b = __ldg(digests + 2 * (base + j) + 1);
-            const unsigned long long k[4] = {u64_of(a.x, a.y), u64_of(a.z, a.w), u64_of(b.x, b.y), u64_of(b.z, b.w)};
-            if (key_reserved(k)) {
-                my_flags |= KVGOV_F_SENTINEL;
-                continue;
+    for (long long w = ((long long)blockIdx.x * kInsertThreads + threadIdx.x) / 32; w * kSegs < n_req;
+         w += warps_total) {                                   // warp-uniform
+        const long long r = w * kSegs + seg;
+        long long base = 0, nb = 0, L = 0;
+        if (r < n_req) {
+            base = blk_off[r];
+            nb = blk_off[r + 1] - base;
+            if (nb < 0 || base < 0 || base + nb > blk_off[n_req]) {
+                if (sl == 0) my_flags |= KVGOV_F_BADINDEX;
+                nb = 0;
             }
-            count_insert(insert_one(slots, mask, k, spin_limit), my_new, my_flags);
+            L = prefix_blocks[r];
+            if (L < 0) L = 0;
+        }
+        const long long left = nb - L - sl;
+        const int iters = left > 0 ? (int)((left + G - 1) / G) : 0;
+        const int wmax = __reduce_max_sync(0xffffffffu, iters);
+        for (int it = 0; it < wmax; ++it) {
+            unsigned long long k[4] = {0ull, 0ull, 0ull, 0ull};
+            bool mine = it < iters;
+            if (mine) {
+                const long long row = base + L + sl + (long long)it * G;
+                const uint4 a = __ldg(digests + 2 * row), b = __ldg(digests + 2 * row + 1);
+                k[0] = u64_of(a.x, a.y); k[1] = u64_of(a.z, a.w); k[2] = u64_of(b.x, b.y); k[3] = u64_of(b.z, b.w);
+                if (key_reserved(k)) {
+                    my_flags |= KVGOV_F_SENTINEL;
+                    mine = false;
+                }
+            }
+            const unsigned inserting = __ballot_sync(0xffffffffu, mine);
+            if (mine) count_insert(insert_warp_dedup(slots, mask, k, spin_limit, inserting), my_new, my_flags);
         }
     }
-    (void)kSegs;
     publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
 }
 

@@ -1,13 +1,25 @@
-"""Build-time variants of libkvgov's chain kernel, timed side by side.
+"""Build-time variants of libkvgov, timed side by side.
 
     python -m paper_2608_09225_gb300.variants [name:flags ...]
+    python -m paper_2608_09225_gb300.variants --insert [name:flags ...]
 
-Each variant is the library compiled with extra nvcc -D flags (for example
-KVGOV_COMPACT_ROUNDS=0|1, KVGOV_CHAIN_R=64|128|256, KVGOV_FMA_ADDS=0|1) into
-_build/variants/<name>/libkvgov.so.  kvgov_chain_hash is timed on three
-workload shapes (15 launches each, CUDA events, median) and every variant's
-digests must equal the first variant's, byte for byte.  Prints one JSON line
-per variant.  Needs a GPU.
+Each variant is the library compiled with extra nvcc -D flags into
+_build/variants/<name>/libkvgov.so.
+
+Chain mode (default; flags such as KVGOV_COMPACT_ROUNDS=0|1,
+KVGOV_CHAIN_R=64|128|256, KVGOV_FMA_ADDS=0|1): kvgov_chain_hash is timed on
+three workload shapes (15 launches each, CUDA events, median) and every
+variant's digests must equal the first variant's, byte for byte.
+
+Insert mode (flags KVGOV_INSERT_LOOK=0|1, KVGOV_INSERT_DEDUP=0|1): 80 serving
+steps of the wide batch (131,072 x 128 tokens, BOUNDARY at token 64) against
+a 2^25-slot table under a new secret epoch per step, flushed before a step
+would take it past load factor 0.5; CUDA events around every kernel.  Reports
+the median steady-state insert, the insert of the first step after a flush
+(where every request's shared-prefix blocks are new, a hot key), probe and
+step times; the number of keys inserted must equal the closed form.
+
+Prints one JSON line per variant.  Needs a GPU.
 """
 from __future__ import annotations
 
@@ -47,8 +59,96 @@ def build_variant(name: str, flags: list[str]) -> str:
     return lib
 
 
+INSERT_DEFAULT = ["look1_dedup1:-DKVGOV_INSERT_LOOK=1 -DKVGOV_INSERT_DEDUP=1",
+                  "look0_dedup0:-DKVGOV_INSERT_LOOK=0 -DKVGOV_INSERT_DEDUP=0",
+                  "look1_dedup0:-DKVGOV_INSERT_LOOK=1 -DKVGOV_INSERT_DEDUP=0",
+                  "look0_dedup1:-DKVGOV_INSERT_LOOK=0 -DKVGOV_INSERT_DEDUP=1"]
+
+
+def _bind(L):
+    p = ctypes.c_void_p
+    L.kvgov_block_offsets.argtypes = [p, ctypes.c_int32, p, p, p]
+    L.kvgov_derive_salts.argtypes = [p, ctypes.c_size_t, p, p, ctypes.c_int32, p, p, p]
+    L.kvgov_chain_hash.argtypes = [ctypes.c_int, p, p, ctypes.c_int32, p, p, ctypes.c_int32, p, p, p, p, p]
+    L.kvgov_table_init.argtypes = [p, ctypes.c_uint64, p]
+    L.kvgov_probe.argtypes = [p, ctypes.c_uint64, p, p, ctypes.c_int32, p, p, p]
+    L.kvgov_insert_uncached.argtypes = [p, ctypes.c_uint64, p, p, ctypes.c_int32, p, p, p, p]
+    return L
+
+
+def insert_mode(specs):
+    import torch
+    n_pool, steps, cap = 4, 80, 1 << 25
+    pool = [W.make("wide", seed=300 + i) for i in range(n_pool)]
+    p0 = pool[0].batch.tokens.reshape(-1, 128)[0, :64].copy()
+    for w in pool:                               # one service-wide 64-token prefix
+        w.batch.tokens.reshape(-1, 128)[:, :64] = p0
+    w0 = pool[0]
+    n = w0.batch.n
+    nblk = n * 8
+
+    def dev(a):
+        return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+    dp = [(dev(w.batch.tokens), dev(w.batch.tok_off), dev(w.batch.principal), dev(w.batch.boundary_tok))
+          for w in pool]
+    ids, id_off = dev(w0.ids), dev(w0.id_off)
+    stream = torch.cuda.current_stream().cuda_stream
+    for spec in specs:
+        name, _, flags = spec.partition(":")
+        L = _bind(ctypes.CDLL(build_variant(name, flags.split())))
+        slots = torch.empty((cap, 32), dtype=torch.uint8, device="cuda")
+        salts = torch.empty((4096, 32), dtype=torch.uint8, device="cuda")
+        blk = torch.empty(n + 1, dtype=torch.int64, device="cuda")
+        dig = torch.empty((nblk, 32), dtype=torch.uint8, device="cuda")
+        pre = torch.empty(n, dtype=torch.int32, device="cuda")
+        st = torch.zeros(1, dtype=torch.int32, device="cuda")
+        n_new = torch.zeros(1, dtype=torch.int64, device="cuda")
+        in_table, expect, fresh = 0, 0, True
+        t = {"insert_steady": [], "insert_after_flush": [], "probe": [], "step": []}
+        assert L.kvgov_table_init(slots.data_ptr(), cap, stream) == 0
+        for s_i in range(steps):
+            if not fresh and in_table + 4 * n > cap // 2:
+                assert L.kvgov_table_init(slots.data_ptr(), cap, stream) == 0
+                in_table, fresh = 0, True
+            add = 4 * n + (4 if fresh else 0)
+            first = fresh
+            in_table, expect, fresh = in_table + add, expect + add, False
+            toks, toff, prin, bt = dp[s_i % n_pool]
+            sec = w0.secret[:24] + s_i.to_bytes(8, "little")
+            buf = ctypes.create_string_buffer(sec, len(sec))
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+            ev[0].record()
+            assert L.kvgov_derive_salts(ctypes.cast(buf, ctypes.c_void_p), len(sec), ids.data_ptr(),
+                                        id_off.data_ptr(), 4096, salts.data_ptr(), st.data_ptr(), stream) == 0
+            assert L.kvgov_block_offsets(toff.data_ptr(), n, blk.data_ptr(), st.data_ptr(), stream) == 0
+            assert L.kvgov_chain_hash(2, toks.data_ptr(), toff.data_ptr(), n, prin.data_ptr(), salts.data_ptr(),
+                                      4096, bt.data_ptr(), blk.data_ptr(), dig.data_ptr(), st.data_ptr(),
+                                      stream) == 0
+            ev[1].record()
+            assert L.kvgov_probe(slots.data_ptr(), cap, dig.data_ptr(), blk.data_ptr(), n, pre.data_ptr(),
+                                 st.data_ptr(), stream) == 0
+            ev[2].record()
+            assert L.kvgov_insert_uncached(slots.data_ptr(), cap, dig.data_ptr(), blk.data_ptr(), n, pre.data_ptr(),
+                                           n_new.data_ptr(), st.data_ptr(), stream) == 0
+            ev[3].record()
+            torch.cuda.synchronize()
+            if s_i >= 2:
+                t["insert_after_flush" if first else "insert_steady"].append(ev[2].elapsed_time(ev[3]))
+                t["probe"].append(ev[1].elapsed_time(ev[2]))
+                t["step"].append(ev[0].elapsed_time(ev[3]))
+        ok = int(st.item()) == 0 and int(n_new.item()) == expect
+        res = {k: round(float(np.median(v)) * 1e3, 1) for k, v in t.items() if v}
+        print(json.dumps({"variant": name, "flags": flags, "us_median": res, "keys_inserted": int(n_new.item()),
+                          "keys_expected": expect, "ok": ok}), flush=True)
+        del slots
+    return 0
+
+
 def main(argv):
     import torch
+    if argv and argv[0] == "--insert":
+        return insert_mode(argv[1:] or INSERT_DEFAULT)
     specs = argv or DEFAULT
     p = ctypes.c_void_p
     cases = []

@@ -231,6 +231,29 @@ def test_table_full(kv):
     assert int(n_new.item()) == 32 and len(table_contents(slots)) == 32
 
 
+def test_full_table_inserts_and_lookups_stay_bounded(kv):
+    """A table filled to the end: further inserts report TABLE_FULL after at
+    most one probe window of slots, and lookups of absent keys end."""
+    cap = 4096
+    k = keys_np(cap + 500, 8)
+    slots = kv.new_table(cap)
+    st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
+    kv.insert(slots, dev(k), st, n_new)
+    torch.cuda.synchronize()
+    assert int(st.item()) & kv.F_TABLE_FULL
+    stored = table_contents(slots)
+    # with the probe window a nearly full table may refuse a key before the
+    # last slot is taken; every refusal is flagged and every store counted
+    assert int(n_new.item()) == len(stored) and len(stored) > 0.9 * cap
+    assert stored <= {r.tobytes() for r in k}
+    absent = keys_np(300, 9)
+    pre = kv.probe(slots, dev(absent), dev(np.arange(301, dtype=np.int64)))
+    pre_k = kv.probe(slots, dev(k), dev(np.arange(cap + 501, dtype=np.int64)))
+    torch.cuda.synchronize()
+    assert (pre.cpu().numpy() == 0).all()
+    assert list(pre_k.cpu().numpy()) == [int(r.tobytes() in stored) for r in k]
+
+
 def test_insert_wait_times_out_on_a_slot_nobody_finishes(kv):
     """A slot holding a key's first 16 bytes whose second half is never
     written (as if its writer stopped): an insert of that key waits a bounded
