@@ -145,6 +145,23 @@ int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t *d_tok_off
                      uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * kvgov_chain_hash_probe -- kvgov_chain_hash and kvgov_probe in one launch:
+ * writes the same d_digests as kvgov_chain_hash and the same
+ * d_prefix_blocks as kvgov_probe on the table (d_slots, capacity) would
+ * (paper section 2.1: the block keys of a request and its longest cached
+ * prefix).  Each thread looks up a block's digest as soon as it has computed
+ * it, while other warps go on hashing; the table must not change during the
+ * call (run inserts after it).  Arguments as for those two calls;
+ * d_prefix_blocks [n_req] int32 output, required.  EINVAL: as for
+ * kvgov_chain_hash, plus a NULL or misaligned d_slots or a bad capacity.
+ */
+int kvgov_chain_hash_probe(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                           const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                           const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                           const uint8_t *d_slots, uint64_t capacity, int32_t *d_prefix_blocks,
+                           uint32_t *d_status, kvgov_stream_t stream);
+
+/*
  * The prefix-cache index (paper section 2.1 and Table 1, row 1: a block
  * prefix cache keyed by chained block hashes).  The caller owns a table of
  * `capacity` 32-byte slots (capacity a power of two >= KVGOV_MIN_CAPACITY,

@@ -18,6 +18,7 @@
 #include <cooperative_groups.h>
 
 #include "kvgov_internal.cuh"
+#include "kvgov_lookup.cuh"
 #include "sha256_dev.cuh"
 
 namespace {
@@ -158,6 +159,10 @@ struct ChainParams {
     int32_t n_req;
     int32_t n_principals;
     uint32_t one;   // 1, opaque to the compiler (see AddFma)
+    // fused probe (kvgov_chain_hash_probe) only
+    const uint4 *slots;
+    unsigned long long mask;
+    int32_t *prefix_blocks;
 };
 
 // Which adder the SHA-256 rounds use.  Measured on GB300: IMAD shares the
@@ -175,7 +180,11 @@ __device__ __forceinline__ void load_salt(const uint8_t *salts, int pi, uint32_t
     sw[4] = bswap32(b.x); sw[5] = bswap32(b.y); sw[6] = bswap32(b.z); sw[7] = bswap32(b.w);
 }
 
-template <int MODE>
+// PROBE: after storing block j's digest, a thread whose blocks 0..j-1 were
+// all found in the table looks block j up too (kvgov_probe's definition),
+// and at the end writes its request's cached-prefix length.  The lookup's
+// memory latency is covered by the other warps' hashing.
+template <int MODE, bool PROBE>
 __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
     __shared__ __align__(16) uint32_t stage[kStages][kR * kSlotWords];
     __shared__ long long s_tok[kR];
@@ -249,6 +258,7 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
     uint32_t h[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) h[i] = 0u;
+    int hits = 0;   // PROBE: leading blocks found in the table so far
 
     for (int j = 0; j < jmax; ++j) {
         const int jn = j + kStages - 1;
@@ -293,12 +303,16 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
             }
 
             uint4 *dst = reinterpret_cast<uint4 *>(p.digests + (row + j) * 32);
-            dst[0] = make_uint4(bswap32(h[0]), bswap32(h[1]), bswap32(h[2]), bswap32(h[3]));
-            dst[1] = make_uint4(bswap32(h[4]), bswap32(h[5]), bswap32(h[6]), bswap32(h[7]));
+            const uint4 q0 = make_uint4(bswap32(h[0]), bswap32(h[1]), bswap32(h[2]), bswap32(h[3]));
+            const uint4 q1 = make_uint4(bswap32(h[4]), bswap32(h[5]), bswap32(h[6]), bswap32(h[7]));
+            dst[0] = q0;
+            dst[1] = q1;
+            if (PROBE && hits == j && lookup(p.slots, p.mask, q0, q1)) hits = j + 1;
         }
         __syncthreads();
     }
     cp_async_wait<0>();
+    if (PROBE && r < p.n_req) p.prefix_blocks[r] = hits;
 }
 
 }  // namespace
@@ -325,10 +339,12 @@ extern "C" int kvgov_block_offsets(const int64_t *d_tok_off, int32_t n_req, int6
     return kvgov_host::launch_status();
 }
 
-extern "C" int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
-                                const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
-                                const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
-                                uint32_t *d_status, kvgov_stream_t stream) {
+namespace {
+
+int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                 const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                 const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests, uint32_t *d_status,
+                 const uint8_t *d_slots, uint64_t capacity, int32_t *d_prefix_blocks, kvgov_stream_t stream) {
     using kvgov_host::aligned16;
     if (mode != KVGOV_UNSALTED && mode != KVGOV_ROOT && mode != KVGOV_BOUNDARY) return KVGOV_EINVAL;
     if (n_req < 0) return KVGOV_EINVAL;
@@ -337,18 +353,51 @@ extern "C" int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t
     if (mode != KVGOV_UNSALTED && (!d_principal || !d_salts || !aligned16(d_salts) || n_principals <= 0))
         return KVGOV_EINVAL;
     if (mode == KVGOV_BOUNDARY && !d_boundary_tok) return KVGOV_EINVAL;
+    const bool probe = d_prefix_blocks != nullptr;
+    if (probe && (!d_slots || !aligned16(d_slots) || !kvgov_host::pow2_capacity(capacity))) return KVGOV_EINVAL;
     if (n_req == 0) return KVGOV_OK;
 
     ChainParams p;
     p.tokens = d_tokens; p.tok_off = d_tok_off; p.principal = d_principal; p.salts = d_salts;
     p.boundary_tok = d_boundary_tok; p.blk_off = d_blk_off; p.digests = d_digests; p.status = d_status;
     p.n_req = n_req; p.n_principals = n_principals; p.one = 1u;
+    p.slots = reinterpret_cast<const uint4 *>(d_slots);
+    p.mask = probe ? capacity - 1 : 0;
+    p.prefix_blocks = d_prefix_blocks;
     const unsigned grid = (unsigned)(((long long)n_req + kR - 1) / kR);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    switch (mode) {
-    case KVGOV_UNSALTED: chain_kernel<KVGOV_UNSALTED><<<grid, kR, 0, s>>>(p); break;
-    case KVGOV_ROOT: chain_kernel<KVGOV_ROOT><<<grid, kR, 0, s>>>(p); break;
-    default: chain_kernel<KVGOV_BOUNDARY><<<grid, kR, 0, s>>>(p); break;
+    if (probe) {
+        switch (mode) {
+        case KVGOV_UNSALTED: chain_kernel<KVGOV_UNSALTED, true><<<grid, kR, 0, s>>>(p); break;
+        case KVGOV_ROOT: chain_kernel<KVGOV_ROOT, true><<<grid, kR, 0, s>>>(p); break;
+        default: chain_kernel<KVGOV_BOUNDARY, true><<<grid, kR, 0, s>>>(p); break;
+        }
+    } else {
+        switch (mode) {
+        case KVGOV_UNSALTED: chain_kernel<KVGOV_UNSALTED, false><<<grid, kR, 0, s>>>(p); break;
+        case KVGOV_ROOT: chain_kernel<KVGOV_ROOT, false><<<grid, kR, 0, s>>>(p); break;
+        default: chain_kernel<KVGOV_BOUNDARY, false><<<grid, kR, 0, s>>>(p); break;
+        }
     }
     return kvgov_host::launch_status();
+}
+
+}  // namespace
+
+extern "C" int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                                const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                                const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                                uint32_t *d_status, kvgov_stream_t stream) {
+    return launch_chain(mode, d_tokens, d_tok_off, n_req, d_principal, d_salts, n_principals, d_boundary_tok,
+                        d_blk_off, d_digests, d_status, nullptr, 0, nullptr, stream);
+}
+
+extern "C" int kvgov_chain_hash_probe(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                                      const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                                      const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                                      const uint8_t *d_slots, uint64_t capacity, int32_t *d_prefix_blocks,
+                                      uint32_t *d_status, kvgov_stream_t stream) {
+    if (!d_prefix_blocks) return KVGOV_EINVAL;
+    return launch_chain(mode, d_tokens, d_tok_off, n_req, d_principal, d_salts, n_principals, d_boundary_tok,
+                        d_blk_off, d_digests, d_status, d_slots, capacity, d_prefix_blocks, stream);
 }

@@ -1,0 +1,40 @@
+// kvgov_lookup.cuh -- read-only lookup of a 32-byte key in the prefix-cache
+// table (slot encoding and probe window as described in kvgov_table.cu and
+// include/kvgov.h), shared by the probe kernel and the fused chain + probe
+// kernel.  The table must not change while a lookup runs.
+#pragma once
+#include <cstdint>
+
+#include "../../include/kvgov.h"
+
+namespace kvgov_dev {
+
+__device__ __forceinline__ unsigned long long u64_of(uint32_t lo, uint32_t hi) {
+    return (unsigned long long)lo | ((unsigned long long)hi << 32);
+}
+
+// Slots a key may occupy past its home slot: min(capacity, KVGOV_PROBE_WINDOW).
+__device__ __forceinline__ unsigned long long probe_window(unsigned long long mask) {
+    return mask < KVGOV_PROBE_WINDOW - 1 ? mask + 1 : (unsigned long long)KVGOV_PROBE_WINDOW;
+}
+
+// Is the key q0 || q1 (bytes 0-15, 16-31, as stored) in the table?  Slots are
+// read through the read-only path.
+__device__ __forceinline__ bool lookup(const uint4 *__restrict__ slots, unsigned long long mask, uint4 q0, uint4 q1) {
+    const unsigned long long k0 = u64_of(q0.x, q0.y), k1 = u64_of(q0.z, q0.w);
+    if ((k0 | k1) == 0ull || u64_of(q1.x, q1.y) == 0ull || u64_of(q1.z, q1.w) == 0ull)
+        return false;                               // reserved keys are never stored
+    const unsigned long long window = probe_window(mask);
+    unsigned long long pos = k0 & mask;
+    for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
+        const uint4 a = __ldg(slots + 2 * pos);
+        if ((a.x | a.y | a.z | a.w) == 0u) return false;   // empty slot ends the walk
+        if (a.x == q0.x && a.y == q0.y && a.z == q0.z && a.w == q0.w) {
+            const uint4 b = __ldg(slots + 2 * pos + 1);
+            if (b.x == q1.x && b.y == q1.y && b.z == q1.z && b.w == q1.w) return true;
+        }
+    }
+    return false;
+}
+
+}  // namespace kvgov_dev

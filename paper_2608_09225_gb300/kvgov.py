@@ -53,6 +53,8 @@ def _load():
         L.kvgov_derive_salts.argtypes = [_p, ctypes.c_size_t, _p, _p, ctypes.c_int32, _p, _p, _p]
         L.kvgov_chain_hash.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p, _p,
                                        _p, _p]
+        L.kvgov_chain_hash_probe.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p,
+                                             _p, _p, ctypes.c_uint64, _p, _p, _p]
         L.kvgov_table_init.argtypes = [_p, ctypes.c_uint64, _p]
         L.kvgov_insert.argtypes = [_p, ctypes.c_uint64, _p, ctypes.c_int64, _p, _p, _p]
         L.kvgov_probe.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p]
@@ -60,7 +62,7 @@ def _load():
         L.kvgov_set_spin_limit.argtypes = [ctypes.c_uint32]
         L.kvgov_set_spin_limit.restype = ctypes.c_uint32
         for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
-                   "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached"):
+                   "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe"):
             getattr(L, fn).restype = ctypes.c_int
         _lib = L
         return L
@@ -158,6 +160,37 @@ def chain_hash(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, blk_off: 
                               _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_chain_hash")
     return digests
+
+
+def chain_hash_probe(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, blk_off: torch.Tensor,
+                     slots: torch.Tensor, principal: torch.Tensor | None = None, salts: torch.Tensor | None = None,
+                     boundary_tok: torch.Tensor | None = None, digests: torch.Tensor | None = None,
+                     prefix_blocks: torch.Tensor | None = None, n_blocks: int | None = None,
+                     status: torch.Tensor | None = None, stream=None):
+    """chain_hash and probe in one launch; returns (digests, prefix_blocks)."""
+    L = lib()
+    n = tok_off.numel() - 1
+    if digests is None:
+        if n_blocks is None:
+            n_blocks = int(blk_off[-1].item())
+        digests = torch.empty((n_blocks, 32), dtype=torch.uint8, device=tokens.device)
+    if prefix_blocks is None:
+        prefix_blocks = torch.empty(n, dtype=torch.int32, device=tok_off.device)
+    if tokens.numel() == 0:
+        tokens = torch.zeros(4, dtype=torch.int32, device=tok_off.device)
+    n_p = 0 if salts is None else salts.shape[0]
+    _check(L.kvgov_chain_hash_probe(int(mode), _dev(tokens, torch.int32, "tokens"),
+                                    _dev(tok_off, torch.int64, "tok_off"), n,
+                                    _dev(principal, torch.int32, "principal", True),
+                                    _dev(salts, torch.uint8, "salts", True), n_p,
+                                    _dev(boundary_tok, torch.int32, "boundary_tok", True),
+                                    _dev(blk_off, torch.int64, "blk_off"),
+                                    _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(tokens),
+                                    _dev(slots, torch.uint8, "slots"), slots.shape[0],
+                                    _dev(prefix_blocks, torch.int32, "prefix_blocks") if n else _dummy(tokens),
+                                    _dev(status, torch.int32, "status", True), _stream(stream)),
+           "kvgov_chain_hash_probe")
+    return digests, prefix_blocks
 
 
 def _dummy(like: torch.Tensor):

@@ -100,13 +100,22 @@ class PrefixCache:
 
     # -- one serving step -------------------------------------------------
     def serve(self, mode: int, b: DeviceBatch, bufs: dict | None = None, derive_salts: bool = True):
-        """Salts, blocking, chain, probe, and insert of the uncached blocks for
-        one batch.  Returns (prefix_blocks, digests, blk_off), on the device."""
+        """Salts, blocking, chain hash with the probe fused in, and insert of
+        the uncached blocks for one batch.  Returns (prefix_blocks, digests,
+        blk_off), on the device."""
         bufs = bufs if bufs is not None else {}
         if derive_salts:
             self.derive_salts()
-        blk_off, digests = self.hash(mode, b, bufs.get("blk_off"), bufs.get("digests"))
-        prefix = self.probe(digests, blk_off, bufs.get("prefix"))
+        blk_off = bufs.get("blk_off")
+        if blk_off is None:
+            blk_off = torch.empty(b.n + 1, dtype=torch.int64, device=self.device)
+        K.block_offsets(b.tok_off, blk_off, self.status, self.stream)
+        salted = mode != K.UNSALTED
+        digests, prefix = K.chain_hash_probe(mode, b.tokens, b.tok_off, blk_off, self.slots,
+                                             b.principal if salted else None, self.salts if salted else None,
+                                             b.boundary_tok if mode == K.BOUNDARY else None, bufs.get("digests"),
+                                             bufs.get("prefix"), n_blocks=b.n_blocks, status=self.status,
+                                             stream=self.stream)
         self.insert_uncached(digests, blk_off, prefix)
         return prefix, digests, blk_off
 

@@ -336,6 +336,36 @@ def test_insert_uncached_bad_offsets_flagged(kv):
     assert int(st.item()) & kv.F_BADINDEX
 
 
+@pytest.mark.parametrize("mode", [0, 1, 2])
+@pytest.mark.parametrize("fill", [0.0, 0.5, 1.0])
+def test_chain_hash_probe_matches_separate_calls(kv, mode, fill):
+    """The fused launch writes the digests of kvgov_chain_hash and the prefix
+    lengths of kvgov_probe; both equal the oracle's."""
+    b = W.ragged(77, RAGGED * 9)
+    salts = oracle.derive_salts(b"fused", *W.principal_ids(8))
+    ref = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+    blk_ref = oracle.block_offsets(b.tok_off)
+    rng = np.random.default_rng(int(fill * 10) + mode)
+    member = rng.random(len(ref)) < fill
+    member[blk_ref[5]:blk_ref[9]] = True          # some requests fully cached
+    slots = kv.new_table(1 << 14)
+    st = status_tensor()
+    if member.any():
+        kv.insert(slots, dev(ref[member]), st)
+    toks, tok_off = dev(b.tokens, np.int32), dev(b.tok_off, np.int64)
+    blk = kv.block_offsets(tok_off, status=st)
+    d, pre = kv.chain_hash_probe(mode, toks, tok_off, blk, slots, dev(b.principal, np.int32), dev(salts),
+                                 dev(b.boundary_tok, np.int32), n_blocks=len(ref), status=st)
+    pre_sep = kv.probe(slots, d, blk, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert (d.cpu().numpy() == ref).all()
+    ks = oracle.KeySet(1)
+    ks.insert(ref[member])
+    pref = ks.prefix_blocks(ref, blk_ref)
+    assert (pre.cpu().numpy() == pref).all() and (pre_sep.cpu().numpy() == pref).all()
+
+
 def test_probe_empty_and_bad_offsets(kv):
     slots = kv.new_table(64)
     st = status_tensor()

@@ -33,7 +33,8 @@ def declared_functions():
 def test_header_declares_the_boundary():
     names = declared_functions()
     for want in ("kvgov_derive_salts", "kvgov_block_offsets", "kvgov_chain_hash", "kvgov_table_init",
-                 "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_status_string",
+                 "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
+                 "kvgov_status_string",
                  "kvgov_set_spin_limit"):
         assert want in names
 
@@ -78,6 +79,12 @@ def test_host_validation_rejects_bad_arguments(libkv):
     assert ch(2, fake, fake, 4, fake, fake, 1, None, fake, fake, None, None) == 1           # BOUNDARY without offsets
     assert ch(0, fake, fake, -1, None, None, 0, None, fake, fake, None, None) == 1          # negative n_req
     assert ch(0, fake, fake, 0, None, None, 0, None, fake, fake, None, None) == 0           # empty batch: no-op
+    cp = libkv.kvgov_chain_hash_probe
+    cp.argtypes = [ctypes.c_int, p, p, ctypes.c_int32, p, p, ctypes.c_int32, p, p, p, p, ctypes.c_uint64, p, p, p]
+    assert cp(0, fake, fake, 4, None, None, 0, None, fake, fake, fake, 64, None, None, None) == 1   # no output
+    assert cp(0, fake, fake, 4, None, None, 0, None, fake, fake, fake, 100, fake, None, None) == 1  # capacity
+    assert cp(0, fake, fake, 4, None, None, 0, None, fake, fake, odd, 64, fake, None, None) == 1    # misaligned
+    assert cp(0, fake, fake, 0, None, None, 0, None, fake, fake, fake, 64, fake, None, None) == 0   # empty batch
     ti = libkv.kvgov_table_init
     ti.argtypes = [p, ctypes.c_uint64, p]
     for cap in (0, 16, 48, 1000):
