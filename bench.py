@@ -473,53 +473,48 @@ def main():
 
 
 def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots):
-    """Same step with host buffers: pinned H2D of each step's inputs and D2H
-    of its prefix lengths inside the timed region, through PrefixCache.serve
-    on a cache of its own."""
-    from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache
+    """Same step with host buffers, through the public HostPipeline: each
+    step's inputs are copied from pinned host memory (a copy stream, which
+    overlaps the previous step's serving) and its prefix lengths are copied
+    back to pinned host memory, all inside the timed region."""
+    from paper_2608_09225_gb300.pipeline import HostPipeline, PrefixCache
     pinned = []
     for w in hosts:
         b = w.batch
         pinned.append(tuple(torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
                             for a in (b.tokens, b.tok_off, b.principal, b.boundary_tok)))
     n_req = hosts[0].batch.n
+    n_tok = int(hosts[0].batch.tok_off[-1])
     n_blocks = int((hosts[0].batch.lengths() // 16).sum())
-    warm = 3
     cache = PrefixCache(table_slots, w0.secret, w0.ids, w0.id_off)
+    pipe = HostPipeline(cache, W.BOUNDARY, n_req, n_tok)
     flush = FlushPolicy(table_slots, 4 * n_req)
-    bufs = {"blk_off": torch.empty(n_req + 1, dtype=torch.int64, device="cuda"),
-            "digests": torch.empty((n_blocks, 32), dtype=torch.uint8, device="cuda"),
-            "prefix": torch.empty(n_req, dtype=torch.int32, device="cuda")}
-    out = torch.empty(n_req, dtype=torch.int32).pin_memory()
-    dev = [torch.empty_like(t, device="cuda") for t in pinned[0]]
     h2d = sum(t.numel() * t.element_size() for t in pinned[0])
-    d2h = out.numel() * out.element_size()
+    d2h = n_req * 4
 
     def one(i):
-        src = pinned[i % len(pinned)]
-        for d, s in zip(dev, src):
-            d.copy_(s, non_blocking=True)
         cache.set_secret(epoch_secret(w0.secret, i))
-        if flush.before_step():
-            K.table_init(cache.slots)
-        prefix, _, _ = cache.serve(W.BOUNDARY, DeviceBatch(dev[0], dev[1], dev[2], dev[3], n_blocks), bufs)
-        out.copy_(prefix, non_blocking=True)
+        before = (lambda: K.table_init(cache.slots, pipe.compute_stream)) if flush.before_step() else None
+        return pipe.submit(*pinned[i % len(pinned)], n_blocks, before)
 
+    warm = 3
     for i in range(warm):
         one(i)
     torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         dist.barrier()
-    a.record()
+    a.record(pipe.copy_stream)
     for i in range(steps):
-        one(warm + i)
-    b.record()
+        out, ev = one(warm + i)
+    b.record(pipe.compute_stream)
     torch.cuda.synchronize()
     cache.check_status()
+    last_ok = bool((out == 4).all()) if flush.last_prefix == 4 else bool((out == 0).all())
     ms = max_over_ranks(a.elapsed_time(b), world, dist, "cuda")
     return {"value": world * steps * n_blocks / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "steps": steps}
+            "d2h_bytes_per_step": d2h, "steps": steps, "last_step_prefix_ok": last_ok,
+            "api": "paper_2608_09225_gb300.pipeline.HostPipeline (copy of step i+1 overlaps serving of step i)"}
 
 
 def cpu_baseline(w, sample, gpu_digests):

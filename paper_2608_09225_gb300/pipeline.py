@@ -124,3 +124,70 @@ class PrefixCache:
         if s:
             raise K.KVGovError(s, "device status")
         return s
+
+
+class HostPipeline:
+    """Serve batches that live in pinned host memory, overlapping each batch's
+    host-to-device copy with the serving of the previous one.
+
+    Two device input slots alternate: ``submit`` copies the batch into the next
+    slot on a copy stream, and the compute stream serves it (salts, blocking,
+    chain hash with the fused probe, insert) once that copy has landed, then
+    copies the prefix lengths back into a pinned host buffer.  A slot is reused
+    only after the compute stream has finished with it.
+
+    submit() returns (prefix_host, event): prefix_host is valid once event has
+    completed (event.synchronize()) and is overwritten two submits later.
+    Every step runs on the GPU; nothing here computes.
+    """
+
+    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_tokens: int, device="cuda"):
+        self.cache, self.mode = cache, mode
+        dev = torch.device(device)
+        self.copy_stream = torch.cuda.Stream(dev)
+        self.compute_stream = torch.cuda.Stream(dev)
+        cache.stream = self.compute_stream
+        max_blocks = max_tokens // K.BLOCK
+        self.slots = []
+        for _ in range(2):
+            self.slots.append({
+                "tokens": torch.empty(max(max_tokens, 4), dtype=torch.int32, device=dev),
+                "tok_off": torch.empty(max_req + 1, dtype=torch.int64, device=dev),
+                "principal": torch.empty(max(max_req, 1), dtype=torch.int32, device=dev),
+                "boundary_tok": torch.empty(max(max_req, 1), dtype=torch.int32, device=dev),
+                "blk_off": torch.empty(max_req + 1, dtype=torch.int64, device=dev),
+                "digests": torch.empty((max(max_blocks, 1), 32), dtype=torch.uint8, device=dev),
+                "prefix": torch.empty(max(max_req, 1), dtype=torch.int32, device=dev),
+                "out": torch.empty(max(max_req, 1), dtype=torch.int32).pin_memory(),
+                "copied": torch.cuda.Event(), "free": torch.cuda.Event(), "used": False,
+            })
+        self.i = 0
+
+    def submit(self, tokens, tok_off, principal, boundary_tok, n_blocks: int, before_serve=None):
+        """Queue one batch given as pinned host tensors (int32 tokens, int64
+        offsets, int32 principal rows and boundary offsets).  before_serve, if
+        given, is called with the compute stream current just before serving
+        (for instance to flush the cache)."""
+        s = self.slots[self.i % 2]
+        self.i += 1
+        n, t = tok_off.numel() - 1, tokens.numel()
+        with torch.cuda.stream(self.copy_stream):
+            if s["used"]:
+                self.copy_stream.wait_event(s["free"])
+            s["tokens"][:t].copy_(tokens, non_blocking=True)
+            s["tok_off"][:n + 1].copy_(tok_off, non_blocking=True)
+            s["principal"][:n].copy_(principal, non_blocking=True)
+            s["boundary_tok"][:n].copy_(boundary_tok, non_blocking=True)
+            s["copied"].record(self.copy_stream)
+        s["used"] = True
+        with torch.cuda.stream(self.compute_stream):
+            self.compute_stream.wait_event(s["copied"])
+            if before_serve is not None:
+                before_serve()
+            db = DeviceBatch(s["tokens"][:max(t, 4)], s["tok_off"][:n + 1], s["principal"][:n],
+                             s["boundary_tok"][:n], n_blocks)
+            bufs = {"blk_off": s["blk_off"][:n + 1], "digests": s["digests"][:n_blocks], "prefix": s["prefix"][:n]}
+            prefix, _, _ = self.cache.serve(self.mode, db, bufs)
+            s["out"][:n].copy_(prefix, non_blocking=True)
+            s["free"].record(self.compute_stream)
+        return s["out"][:n], s["free"]

@@ -7,7 +7,7 @@ import torch
 
 import oracle
 from paper_2608_09225_gb300 import workloads as W
-from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache, next_pow2
+from paper_2608_09225_gb300.pipeline import DeviceBatch, HostPipeline, PrefixCache, next_pow2
 from tests.pins import run_workload_oracle
 
 pytestmark = pytest.mark.gpu
@@ -141,3 +141,39 @@ def test_full_wide_serving_steps(kv):
         assert int(cache.n_new.item()) == ks.n
         seen.append(int(pref.min()))
     assert seen == [0, 4, 8]
+
+
+def test_host_pipeline_matches_device_serving(kv):
+    """Batches served from pinned host memory through HostPipeline (copies
+    overlapping the previous batch's serving) give the prefix lengths of the
+    same batches served from device memory, and the same cache contents."""
+    ws = [W.make("wide", seed=200 + i, n_req=8192) for i in range(4)]
+    for w in ws[1:]:
+        w.batch.tokens.reshape(-1, 128)[:, :64] = ws[0].batch.tokens[:64]
+    w0 = ws[0]
+    dev_cache = PrefixCache(1 << 18, w0.secret, w0.ids, w0.id_off)
+    host_cache = PrefixCache(1 << 18, w0.secret, w0.ids, w0.id_off)
+    n_tok = int(w0.batch.tok_off[-1])
+    pipe = HostPipeline(host_cache, W.BOUNDARY, w0.batch.n, n_tok)
+    order = [0, 1, 2, 0, 3, 1]
+    got, want = [], []
+    for i, k in enumerate(order):
+        b = ws[k].batch
+        secret = w0.secret[:24] + (0 if i < 4 else 1).to_bytes(8, "little")   # a new epoch from batch 4 on
+        dev_cache.set_secret(secret)
+        host_cache.set_secret(secret)
+        pre, _, _ = dev_cache.serve(W.BOUNDARY, DeviceBatch.from_host(b.tokens, b.tok_off, b.principal,
+                                                                       b.boundary_tok))
+        want.append(pre.cpu().numpy())
+        host = [torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+                for a in (b.tokens, b.tok_off, b.principal, b.boundary_tok)]
+        out, ev = pipe.submit(*host, b.n * 8)
+        ev.synchronize()
+        got.append(out.numpy().copy())
+    torch.cuda.synchronize()
+    dev_cache.check_status()
+    host_cache.check_status()
+    for g, w in zip(got, want):
+        assert (g == w).all()
+    assert int(dev_cache.n_new.item()) == int(host_cache.n_new.item())
+    assert [int(x.min()) for x in want] == [0, 4, 4, 8, 4, 4]
