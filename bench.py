@@ -317,12 +317,16 @@ def main():
     ap.add_argument("--seed", type=int, default=None, help="base seed (default: fresh per run)")
     ap.add_argument("--cpu-sample", type=int, default=16384, help="requests per oracle step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--configs", action="store_true",
+                    help="instead of the timed serving step: per-kernel rates on every workload, one JSON line each")
     args = ap.parse_args()
     if args.seed is None:
         args.seed = int.from_bytes(os.urandom(4), "little")
     args.warmup = max(args.warmup, 3)
     if args.impl == "reference":
         return reference_arm(args)
+    if args.configs:
+        return run_configs(args)
 
     import torch
     import torch.distributed as dist
@@ -534,6 +538,144 @@ def cpu_baseline(w, sample, gpu_digests):
             "sample": f"{reps} steps over the first {sample} requests of one batch (salts for 4096 principals, "
                       f"chain on {cores} threads, probe, insert of the uncached blocks); {dt:.1f} s",
             "gate_sample_digests_equal_gpu": same}
+
+
+# --------------------------------------------------------------------------- per-workload rates
+def _time(torch, fn, reps=10, warm=3):
+    """Median CUDA-event time of fn() in ms (fn enqueues on the current stream)."""
+    for _ in range(warm):
+        fn()
+    torch.cuda.synchronize()
+    ts = []
+    for _ in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        fn()
+        b.record()
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    return float(np.median(ts))
+
+
+def _oracle_rate(w, mode, cores, budget_s=3.0):
+    """Oracle digests/s on 1 thread and on `cores` threads over request chunks."""
+    import concurrent.futures as cf
+
+    import oracle
+    b = w.batch
+    salts = oracle.derive_salts(w.secret, w.ids, w.id_off)
+
+    def run(lo, hi):
+        off = b.tok_off[lo:hi + 1] - b.tok_off[lo]
+        return len(oracle.chain_hash(mode, b.tokens[b.tok_off[lo]:b.tok_off[hi]], off, b.principal[lo:hi], salts,
+                                     b.boundary_tok[lo:hi]))
+
+    out = {}
+    for threads in (1, cores):
+        n = 1
+        while True:                                 # grow the sample until it takes ~budget/4
+            t0 = time.perf_counter()
+            step = max(1, n // threads)
+            with cf.ThreadPoolExecutor(threads) as ex:
+                blocks = sum(ex.map(lambda i: run(i, min(i + step, n)), range(0, n, step)))
+            dt = time.perf_counter() - t0
+            if dt > budget_s / 4 or n >= b.n:
+                break
+            n = min(b.n, n * 4)
+        out[f"oracle_digests_per_s_{threads}_threads"] = blocks / dt
+    return out
+
+
+def run_configs(args):
+    """Per-kernel GPU rates (and the oracle's) on every workload at full size."""
+    import torch
+
+    import oracle
+    from paper_2608_09225_gb300 import build as kbuild
+    from paper_2608_09225_gb300 import kvgov as K
+    from paper_2608_09225_gb300 import workloads as W
+    from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache, next_pow2
+    kbuild.build()
+    oracle.build()
+    K.lib()
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    peak = n_sm * INT32_LANES_PER_SM * SM_MAX_MHZ * 1e6
+    cores = len(os.sched_getaffinity(0))
+    l2 = torch.cuda.get_device_properties(0).L2_cache_size
+    seed = args.seed
+    plan = [("tiny", W.make("tiny"), W.ROOT), ("sysprompt", W.make("sysprompt"), W.ROOT)]
+    tmpl = W.make("template")
+    plan += [("template", tmpl, m) for m in (W.UNSALTED, W.ROOT, W.BOUNDARY)]
+    plan += [("probe", W.make("probe"), W.ROOT), ("long", W.make("long", seed=seed), W.BOUNDARY),
+             ("wide", W.make("wide", seed=seed + 1), W.BOUNDARY)]
+    names = {W.UNSALTED: "UNSALTED", W.ROOT: "ROOT", W.BOUNDARY: "BOUNDARY"}
+    for name, w, mode in plan:
+        b = w.batch
+        cap = w.capacity or next_pow2(4 * int((b.lengths() // 16).sum()))
+        cache = PrefixCache(cap, w.secret, w.ids, w.id_off)
+        db = DeviceBatch.from_host(b.tokens, b.tok_off, b.principal, b.boundary_tok)
+        n_blocks = db.n_blocks
+        blk = torch.empty(b.n + 1, dtype=torch.int64, device="cuda")
+        dig = torch.empty((n_blocks, 32), dtype=torch.uint8, device="cuda")
+        pre = torch.empty(b.n, dtype=torch.int32, device="cuda")
+        salted = mode != W.UNSALTED
+        pr, sl, bt = (db.principal if salted else None), (cache.salts if salted else None), \
+            (db.boundary_tok if mode == W.BOUNDARY else None)
+        K.block_offsets(db.tok_off, blk)
+        t_salts = _time(torch, lambda: K.derive_salts(w.secret, cache.ids, cache.id_off, cache.salts))
+        t_blk = _time(torch, lambda: K.block_offsets(db.tok_off, blk))
+        t_chain = _time(torch, lambda: K.chain_hash(mode, db.tokens, db.tok_off, blk, pr, sl, bt, dig))
+        # the workload's table content
+        blk_np = blk.cpu().numpy()
+        fill_keys = []
+        if w.fill_from == "prior":
+            p = w.prior
+            dp = DeviceBatch.from_host(p.tokens, p.tok_off, p.principal, p.boundary_tok)
+            pblk = torch.empty(p.n + 1, dtype=torch.int64, device="cuda")
+            K.block_offsets(dp.tok_off, pblk)
+            pd = K.chain_hash(mode, dp.tokens, dp.tok_off, pblk, dp.principal if salted else None, sl,
+                              dp.boundary_tok if mode == W.BOUNDARY else None, n_blocks=dp.n_blocks)
+            fill_keys.append(pd)
+        elif w.fill[1] > w.fill[0]:
+            fill_keys.append(dig[blk_np[w.fill[0]]:blk_np[w.fill[1]]])
+        else:                                    # long / wide: the first half of the batch
+            fill_keys.append(dig[: blk_np[b.n // 2]])
+        if w.random_keys is not None:
+            fill_keys.append(torch.from_numpy(w.random_keys).cuda())
+        keys = torch.cat(fill_keys)
+        t_insert = _time(torch, lambda: (K.table_init(cache.slots), K.insert(cache.slots, keys, cache.status)),
+                         reps=3, warm=1)
+        t_init = _time(torch, lambda: K.table_init(cache.slots), reps=3, warm=1)
+        K.insert(cache.slots, keys, cache.status)
+        p0, p1 = w.probe if w.probe[1] > w.probe[0] else (0, b.n)
+        pblk_view = blk[p0:p1 + 1]
+        t_probe = _time(torch, lambda: K.probe(cache.slots, dig, pblk_view, pre[: p1 - p0]))
+        t_fused = _time(torch, lambda: K.chain_hash_probe(mode, db.tokens, db.tok_off, blk, cache.slots, pr, sl, bt,
+                                                          dig, pre))
+        torch.cuda.synchronize()
+        cache.check_status()
+        L = K.probe(cache.slots, dig, pblk_view).cpu().numpy()
+        nb = np.diff(blk_np[p0:p1 + 1])
+        algo_probes = int(np.minimum(L + 1, nb).sum())
+        ops = nominal_chain_ops(b.lengths() // 16, mode, b.boundary_tok // 16)
+        line = {"workload": name, "mode": names[mode], "requests": b.n, "blocks": n_blocks,
+                "table_slots": cap, "table_fits_l2": cap * 32 <= l2,
+                "chain_ms": t_chain, "chain_digests_per_s": n_blocks / (t_chain / 1e3),
+                "chain_tokens_per_s": 16 * n_blocks / (t_chain / 1e3),
+                "chain_frac_int32_peak": ops / (t_chain / 1e3) / peak,
+                "chain_us_per_block_per_chain": 1e3 * t_chain / max(1, int((b.lengths() // 16).max())),
+                "fused_chain_probe_ms": t_fused, "salts_ms": t_salts, "block_offsets_ms": t_blk,
+                "probe_ms": t_probe, "probed_requests": p1 - p0, "algorithmic_probes": algo_probes,
+                "probes_per_s": algo_probes / (t_probe / 1e3), "mean_prefix_blocks": float(L.mean()),
+                "insert_keys": int(keys.shape[0]), "insert_ms": t_insert - t_init,
+                "inserts_per_s": keys.shape[0] / ((t_insert - t_init) / 1e3)}
+        if not args.no_cpu_baseline:
+            line.update(_oracle_rate(w, mode, cores))
+            line["oracle_cores"] = cores
+        print(json.dumps(line), flush=True)
+        del cache, keys, dig
+        torch.cuda.empty_cache()
+    return 0
 
 
 if __name__ == "__main__":

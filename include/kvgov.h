@@ -151,7 +151,10 @@ int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t *d_tok_off
  * (paper section 2.1: the block keys of a request and its longest cached
  * prefix).  Each thread looks up a block's digest as soon as it has computed
  * it, while other warps go on hashing; the table must not change during the
- * call (run inserts after it).  Arguments as for those two calls;
+ * call (run inserts after it).  A batch too small to give each SM
+ * sub-partition two warps (n_req < 2 * 32 * 4 * SMs) runs the lookups as a
+ * second kernel after the chain instead, since a warp alone on its scheduler
+ * would stall on each lookup; the results are the same.  Arguments as for those two calls;
  * d_prefix_blocks [n_req] int32 output, required.  EINVAL: as for
  * kvgov_chain_hash, plus a NULL or misaligned d_slots or a bad capacity.
  */

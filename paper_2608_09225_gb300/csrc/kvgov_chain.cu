@@ -307,7 +307,7 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
             const uint4 q1 = make_uint4(bswap32(h[4]), bswap32(h[5]), bswap32(h[6]), bswap32(h[7]));
             dst[0] = q0;
             dst[1] = q1;
-            if (PROBE && hits == j && lookup(p.slots, p.mask, q0, q1)) hits = j + 1;
+            if (PROBE && hits == j && lookup<false>(p.slots, p.mask, q0, q1)) hits = j + 1;
         }
         __syncthreads();
     }
@@ -366,6 +366,23 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     p.prefix_blocks = d_prefix_blocks;
     const unsigned grid = (unsigned)(((long long)n_req + kR - 1) / kR);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    // A batch too small to give every SM sub-partition two warps leaves each
+    // warp alone on its scheduler, where a fused lookup would stall the chain;
+    // there the lookups run as a second launch (same results).
+    const DeviceInfo dev = device_info();
+    const long long min_fused = 2ll * 32 * 4 * (dev.sms > 0 ? dev.sms : 152);
+    if (probe && n_req < min_fused) {
+        p.mask = 0;
+        p.prefix_blocks = nullptr;
+        switch (mode) {
+        case KVGOV_UNSALTED: chain_kernel<KVGOV_UNSALTED, false><<<grid, kR, 0, s>>>(p); break;
+        case KVGOV_ROOT: chain_kernel<KVGOV_ROOT, false><<<grid, kR, 0, s>>>(p); break;
+        default: chain_kernel<KVGOV_BOUNDARY, false><<<grid, kR, 0, s>>>(p); break;
+        }
+        const int rc = kvgov_host::launch_status();
+        if (rc != KVGOV_OK) return rc;
+        return kvgov_probe(d_slots, capacity, d_digests, d_blk_off, n_req, d_prefix_blocks, d_status, stream);
+    }
     if (probe) {
         switch (mode) {
         case KVGOV_UNSALTED: chain_kernel<KVGOV_UNSALTED, true><<<grid, kR, 0, s>>>(p); break;

@@ -19,7 +19,12 @@ __device__ __forceinline__ unsigned long long probe_window(unsigned long long ma
 }
 
 // Is the key q0 || q1 (bytes 0-15, 16-31, as stored) in the table?  Slots are
-// read through the read-only path.
+// read through the read-only path.  WHOLE_SLOT reads both halves of a slot at
+// once (one memory round trip per slot: the probe kernel, whose warps wait on
+// their lookups); otherwise the second half is read only when the first
+// matches (fewer loads: the fused chain kernel, whose lookups hide behind
+// other warps' hashing).
+template <bool WHOLE_SLOT>
 __device__ __forceinline__ bool lookup(const uint4 *__restrict__ slots, unsigned long long mask, uint4 q0, uint4 q1) {
     const unsigned long long k0 = u64_of(q0.x, q0.y), k1 = u64_of(q0.z, q0.w);
     if ((k0 | k1) == 0ull || u64_of(q1.x, q1.y) == 0ull || u64_of(q1.z, q1.w) == 0ull)
@@ -28,9 +33,11 @@ __device__ __forceinline__ bool lookup(const uint4 *__restrict__ slots, unsigned
     unsigned long long pos = k0 & mask;
     for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
         const uint4 a = __ldg(slots + 2 * pos);
+        uint4 b;
+        if (WHOLE_SLOT) b = __ldg(slots + 2 * pos + 1);
         if ((a.x | a.y | a.z | a.w) == 0u) return false;   // empty slot ends the walk
         if (a.x == q0.x && a.y == q0.y && a.z == q0.z && a.w == q0.w) {
-            const uint4 b = __ldg(slots + 2 * pos + 1);
+            if (!WHOLE_SLOT) b = __ldg(slots + 2 * pos + 1);
             if (b.x == q1.x && b.y == q1.y && b.z == q1.z && b.w == q1.w) return true;
         }
     }

@@ -257,7 +257,7 @@ __global__ void __launch_bounds__(kProbeThreads) probe_kernel(const uint4 *__res
             bool miss = false;
             if (mine) {
                 const uint4 *q = digests + 2 * (base + j);
-                miss = !lookup(slots, mask, __ldg(q), __ldg(q + 1));
+                miss = !lookup<true>(slots, mask, __ldg(q), __ldg(q + 1));
             }
             const unsigned seg_miss = (__ballot_sync(0xffffffffu, miss) >> (seg * G)) & kSegMask;
             if (active) {

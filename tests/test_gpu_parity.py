@@ -338,17 +338,21 @@ def test_insert_uncached_bad_offsets_flagged(kv):
 
 @pytest.mark.parametrize("mode", [0, 1, 2])
 @pytest.mark.parametrize("fill", [0.0, 0.5, 1.0])
-def test_chain_hash_probe_matches_separate_calls(kv, mode, fill):
-    """The fused launch writes the digests of kvgov_chain_hash and the prefix
-    lengths of kvgov_probe; both equal the oracle's."""
-    b = W.ragged(77, RAGGED * 9)
+@pytest.mark.parametrize("n_req", [180, 40960], ids=["two_launches", "fused"])
+def test_chain_hash_probe_matches_separate_calls(kv, mode, fill, n_req):
+    """kvgov_chain_hash_probe writes the digests of kvgov_chain_hash and the
+    prefix lengths of kvgov_probe, both equal to the oracle's, for a batch
+    small enough to take two launches and one that takes the fused kernel."""
+    lengths = (RAGGED * 9 if n_req == 180 else
+               list(np.random.default_rng(n_req + mode).integers(0, 260, n_req)))
+    b = W.ragged(77, lengths)
     salts = oracle.derive_salts(b"fused", *W.principal_ids(8))
     ref = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
     blk_ref = oracle.block_offsets(b.tok_off)
     rng = np.random.default_rng(int(fill * 10) + mode)
     member = rng.random(len(ref)) < fill
     member[blk_ref[5]:blk_ref[9]] = True          # some requests fully cached
-    slots = kv.new_table(1 << 14)
+    slots = kv.new_table(max(1 << 14, 1 << int(4 * member.sum()).bit_length()))
     st = status_tensor()
     if member.any():
         kv.insert(slots, dev(ref[member]), st)
