@@ -334,7 +334,7 @@ def main():
     from paper_2608_09225_gb300 import build as kbuild
     from paper_2608_09225_gb300 import kvgov as K
     from paper_2608_09225_gb300 import workloads as W
-    from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache
+    from paper_2608_09225_gb300.pipeline import DeviceBatch, DevicePipeline, PrefixCache
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -372,25 +372,20 @@ def main():
     if not gate["prefix_all_zero_on_empty_table"] or gate["n_new"] != gate["n_new_expected"]:
         raise SystemExit(f"gate failed: {gate}")
 
-    stream = torch.cuda.current_stream()
+    # ---- the timed steps: DevicePipeline computes each batch's salts and block
+    # offsets on a prep stream beside the previous batch's chain hash
+    pipe = DevicePipeline(cache, W.BOUNDARY, n_req, n_blocks)
     epoch = [1]
     launches = [0]
 
     def step(db, ev=None):
-        if flush.before_step():                   # load factor would pass 0.5: flush the cache
-            K.table_init(cache.slots)
-            launches[0] += 1
-        K.derive_salts(epoch_secret(cache.secret, epoch[0]), cache.ids, cache.id_off, cache.salts, cache.status)
+        cache.set_secret(epoch_secret(w0.secret, epoch[0]))
         epoch[0] += 1
-        K.block_offsets(db.tok_off, bufs["blk_off"], cache.status)
-        if ev is not None:
-            ev[0].record(stream)
-        K.chain_hash_probe(W.BOUNDARY, db.tokens, db.tok_off, bufs["blk_off"], cache.slots, db.principal,
-                           cache.salts, db.boundary_tok, bufs["digests"], bufs["prefix"], status=cache.status)
-        if ev is not None:
-            ev[1].record(stream)
-        K.insert_uncached(cache.slots, bufs["digests"], bufs["blk_off"], bufs["prefix"], cache.status, cache.n_new)
-        launches[0] += 4   # salts, block offsets, chain hash + probe, insert
+        flushed = flush.before_step()              # load factor would pass 0.5: flush the cache
+        before = (lambda: K.table_init(cache.slots, pipe.compute_stream)) if flushed else None
+        prefix, _ = pipe.submit(db, before, ev)
+        launches[0] += 5 + int(flushed)   # salts, block offsets (2), chain hash + probe, insert (+ table init)
+        return prefix
 
     for i in range(args.warmup):
         step(pool[(1 + i) % args.pool])
@@ -405,10 +400,13 @@ def main():
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize()
-        t_start.record(stream)
+        t_start.record(pipe.compute_stream)
+        pipe.prep_stream.wait_event(t_start)
+        h0 = time.perf_counter()
         for i in range(args.steps):
-            step(pool[(1 + args.warmup + i) % args.pool], chain_ev[i])
-        t_stop.record(stream)
+            last_prefix = step(pool[(1 + args.warmup + i) % args.pool], chain_ev[i])
+        host_ms = (time.perf_counter() - h0) * 1e3
+        t_stop.record(pipe.compute_stream)
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
@@ -417,7 +415,7 @@ def main():
     gate["n_new_total_expected"] = flush.expected_new
     gate["flushes_in_timed_steps"] = flush.flushes - flushes_before
     gate["last_step_prefix_expected"] = flush.last_prefix
-    gate["last_step_prefix_ok"] = bool((bufs["prefix"] == flush.last_prefix).all().item())
+    gate["last_step_prefix_ok"] = bool((last_prefix == flush.last_prefix).all().item())
     if gate["n_new_total"] != gate["n_new_total_expected"] or not gate["last_step_prefix_ok"]:
         raise SystemExit(f"gate failed: {gate}")
     kernel_launches = launches[0]
@@ -463,6 +461,9 @@ def main():
                                   "miss and are inserted; the cache is flushed (table re-initialised, inside the "
                                   "timed steps) whenever the next step would take it past load factor 0.5"),
             "tokens_per_s": 16 * value, "chain_digests_per_s": world * n_blocks / (chain_ms / 1e3),
+            "host_enqueue_ms_per_step": host_ms / args.steps,
+            "schedule": "DevicePipeline: salts (new epoch) and block offsets of batch i+1 on a prep stream beside "
+                        "the chain hash of batch i; chain hash + probe, insert on a higher-priority compute stream",
             "e2e": e2e, "gpu_launches": kernel_launches, "clocks": clock, "roofline": roofline,
             "gate": gate}
     if rank == 0 and not args.no_cpu_baseline and world == 1:
@@ -516,8 +517,22 @@ def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots):
     cache.check_status()
     last_ok = bool((out == 4).all()) if flush.last_prefix == 4 else bool((out == 0).all())
     ms = max_over_ranks(a.elapsed_time(b), world, dist, "cuda")
-    return {"value": world * steps * n_blocks / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+    # the host link alone: one plain pinned -> device copy of a step's tokens
+    link = []
+    dst = torch.empty_like(pinned[0][0], device="cuda")
+    for _ in range(5):
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        c0.record()
+        dst.copy_(pinned[0][0], non_blocking=True)
+        c1.record()
+        c1.synchronize()
+        link.append(c0.elapsed_time(c1))
+    link_gbs = pinned[0][0].numel() * 4 / (min(link) / 1e3) / 1e9
+    value = world * steps * n_blocks / (ms / 1e3)
+    copy_bound = world * n_blocks / (h2d / (link_gbs * 1e9))
+    return {"value": value, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps, "last_step_prefix_ok": last_ok,
+            "h2d_link_gbs": link_gbs, "copy_bound_value": copy_bound, "frac_of_copy_bound": value / copy_bound,
             "api": "paper_2608_09225_gb300.pipeline.HostPipeline (copy of step i+1 overlaps serving of step i)"}
 
 

@@ -86,6 +86,10 @@ const char *kvgov_status_string(int status);
  *   d_status  nullable; KVGOV_F_BADINDEX if some len_r < 0 (that request
  *             then counts 0 blocks).
  * n_req = 0 writes d_blk_off[0] = 0.  EINVAL: n_req < 0 or a NULL array.
+ * Two ordinary (non-cooperative) launches on `stream`, so the scan may run
+ * beside other kernels; between them d_blk_off holds per-chunk partial
+ * totals (it is its own scratch space), so nothing may read d_blk_off until
+ * the call's work on `stream` has completed.
  */
 int kvgov_block_offsets(const int64_t *d_tok_off, int32_t n_req, int64_t *d_blk_off,
                         uint32_t *d_status, kvgov_stream_t stream);

@@ -1,5 +1,5 @@
-// kvgov_chain.cu -- blocking (kvgov_block_offsets) and the chained, salted
-// block digests (kvgov_chain_hash).
+// kvgov_chain.cu -- the chained, salted block digests (kvgov_chain_hash,
+// kvgov_chain_hash_probe).
 //
 // Paper: section 2.1 equation (h_0 = H(tokens_0..B-1), h_j = H(h_{j-1},
 // tokens_j)), section 4.1 equation (sigma_p prepended at the root) and
@@ -15,8 +15,6 @@
 // then reads its 16 tokens from shared memory, byte-swaps them into
 // big-endian SHA words and runs the 2 (or 3) compressions of its message in
 // registers.
-#include <cooperative_groups.h>
-
 #include "kvgov_internal.cuh"
 #include "kvgov_lookup.cuh"
 #include "sha256_dev.cuh"
@@ -25,111 +23,19 @@ namespace {
 
 using namespace kvgov_dev;
 
-// ---------------------------------------------------------------------------
-// Block offsets: exclusive scan of floor(len_r / 16) in one cooperative
-// launch.  CTA c owns a contiguous range of requests.  Phase 1: each CTA sums
-// its range and posts the total at the position of its last request (a slot
-// it alone will overwrite later).  Grid sync.  Phase 2: each CTA adds the
-// totals posted by the CTAs before it.  Grid sync (every total has been read).
-// Phase 3: each CTA rescans its range and writes base + running count.
-// ---------------------------------------------------------------------------
-
-constexpr int kScanThreads = 1024;
-
-// Inclusive scan of one value per thread across a 1024-thread CTA; also
-// returns the CTA total through *total.
-__device__ __forceinline__ long long cta_inclusive_scan(long long v, long long *warp_sums, long long *total) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
-        const long long u = __shfl_up_sync(0xffffffffu, v, d);
-        if (lane >= d) v += u;
-    }
-    if (lane == 31) warp_sums[warp] = v;
-    __syncthreads();
-    if (warp == 0) {
-        long long s = warp_sums[lane];
-#pragma unroll
-        for (int d = 1; d < 32; d <<= 1) {
-            const long long u = __shfl_up_sync(0xffffffffu, s, d);
-            if (lane >= d) s += u;
-        }
-        warp_sums[lane] = s;
-    }
-    __syncthreads();
-    if (warp > 0) v += warp_sums[warp - 1];
-    *total = warp_sums[31];
-    __syncthreads();   // warp_sums is reused by the next call
-    return v;
-}
-
-__device__ __forceinline__ long long blocks_of(const int64_t *tok_off, long long r, bool *bad) {
-    const long long len = tok_off[r + 1] - tok_off[r];
-    if (len < 0) { *bad = true; return 0; }
-    return len / KVGOV_BLOCK;
-}
-
-__global__ void __launch_bounds__(kScanThreads) blkoff_kernel(const int64_t *__restrict__ tok_off, int32_t n,
-                                                              int64_t *blk_off, uint32_t *status, long long per_cta) {
-    __shared__ long long warp_sums[32];
-    __shared__ long long s_base;
-    namespace cg = cooperative_groups;
-    cg::grid_group grid = cg::this_grid();
-    const long long lo = (long long)blockIdx.x * per_cta;
-    const long long hi = lo + per_cta < n ? lo + per_cta : (long long)n;
-    bool bad = false;
-
-    // phase 1: this CTA's total, posted at blk_off[hi]
-    long long part = 0;
-    for (long long r = lo + threadIdx.x; r < hi; r += kScanThreads) part += blocks_of(tok_off, r, &bad);
-    long long total;
-    cta_inclusive_scan(part, warp_sums, &total);
-    if (threadIdx.x == 0 && hi > lo) blk_off[hi] = total;
-    if (bad) raise_flag(status, KVGOV_F_BADINDEX);
-    grid.sync();
-
-    // phase 2: base = totals of the CTAs before this one
-    long long v = 0;
-    for (long long c = threadIdx.x; c < blockIdx.x; c += kScanThreads) {
-        const long long clo = c * per_cta, chi = clo + per_cta < n ? clo + per_cta : (long long)n;
-        if (chi > clo) v += blk_off[chi];
-    }
-    long long base;
-    cta_inclusive_scan(v, warp_sums, &base);
-    grid.sync();
-
-    // phase 3: rescan the range and write the final prefix sums
-    if (blockIdx.x == 0 && threadIdx.x == 0) blk_off[0] = 0;
-    if (threadIdx.x == 0) s_base = base;
-    __syncthreads();
-    long long carry = s_base;
-    for (long long r0 = lo; r0 < hi; r0 += kScanThreads) {
-        const long long r = r0 + threadIdx.x;
-        bool ignored = false;
-        const long long cnt = r < hi ? blocks_of(tok_off, r, &ignored) : 0;
-        long long chunk;
-        const long long inc = cta_inclusive_scan(cnt, warp_sums, &chunk);
-        if (r < hi) blk_off[r + 1] = carry + inc;
-        carry += chunk;
-    }
-}
-
 struct DeviceInfo {
-    int sms = 0, coop_blocks_per_sm = 0;
+    int sms = 0;
 };
 
-// SM count and cooperative residency of blkoff_kernel on the current device,
-// looked up once per device.
+// SM count of the current device, looked up once per device.
 DeviceInfo device_info() {
     static DeviceInfo cache[64];
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return DeviceInfo{};
     DeviceInfo &d = cache[dev];
     if (d.sms == 0) {
-        int sms = 0, per = 0;
+        int sms = 0;
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, blkoff_kernel, kScanThreads, 0);
-        d.coop_blocks_per_sm = per;
         d.sms = sms;
     }
     return d;
@@ -316,28 +222,6 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
 }
 
 }  // namespace
-
-extern "C" int kvgov_block_offsets(const int64_t *d_tok_off, int32_t n_req, int64_t *d_blk_off,
-                                   uint32_t *d_status, kvgov_stream_t stream) {
-    if (n_req < 0 || !d_tok_off || !d_blk_off) return KVGOV_EINVAL;
-    const DeviceInfo d = device_info();
-    if (d.sms <= 0 || d.coop_blocks_per_sm <= 0) return KVGOV_ECUDA;
-    long long grid = ((long long)n_req + kScanThreads - 1) / kScanThreads;
-    const long long max_grid = (long long)d.sms * d.coop_blocks_per_sm;
-    if (grid > max_grid) grid = max_grid;
-    if (grid < 1) grid = 1;
-    long long per_cta = ((long long)n_req + grid - 1) / grid;
-    if (per_cta < 1) per_cta = 1;
-    const int64_t *tok_off = d_tok_off;
-    int64_t *blk_off = d_blk_off;
-    uint32_t *status = d_status;
-    int32_t n = n_req;
-    void *args[] = {(void *)&tok_off, (void *)&n, (void *)&blk_off, (void *)&status, (void *)&per_cta};
-    if (cudaLaunchCooperativeKernel((const void *)blkoff_kernel, dim3((unsigned)grid), dim3(kScanThreads), args, 0,
-                                    reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
-        return KVGOV_ECUDA;
-    return kvgov_host::launch_status();
-}
 
 namespace {
 

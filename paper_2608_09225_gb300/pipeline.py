@@ -2,8 +2,11 @@
 
 ``PrefixCache`` owns the device-resident state of one KVGov prefix-cache
 index (the slot table and the per-principal salts) and runs a batch of
-requests through the library's kernels on one CUDA stream.  Nothing here
-computes; every step is a libkvgov entry point (include/kvgov.h).
+requests through the library's kernels on one CUDA stream.
+``DevicePipeline`` and ``HostPipeline`` serve a stream of batches (resident
+on the device, or in pinned host memory) with each batch's salts, block
+offsets and host-to-device copy overlapping the previous batch's kernels.
+Nothing here computes; every step is a libkvgov entry point (include/kvgov.h).
 """
 from __future__ import annotations
 
@@ -126,50 +129,152 @@ class PrefixCache:
         return s
 
 
-class HostPipeline:
-    """Serve batches that live in pinned host memory, overlapping each batch's
-    host-to-device copy with the serving of the previous one.
+class _Pipelined:
+    """Two alternating slots of per-batch device buffers and the stream
+    schedule shared by DevicePipeline and HostPipeline.
 
-    Two device input slots alternate: ``submit`` copies the batch into the next
-    slot on a copy stream, and the compute stream serves it (salts, blocking,
-    chain hash with the fused probe, insert) once that copy has landed, then
-    copies the prefix lengths back into a pinned host buffer.  A slot is reused
-    only after the compute stream has finished with it.
-
-    submit() returns (prefix_host, event): prefix_host is valid once event has
-    completed (event.synchronize()) and is overwritten two submits later.
-    Every step runs on the GPU; nothing here computes.
+    Batch i uses slot i % 2.  Its salts (under the secret current when it is
+    submitted) and block offsets are computed on a prep stream once batch
+    i-1's chain hash has started, so their small CTAs run in the room the
+    chain kernel leaves on the SMs instead of in front of batch i's chain
+    hash.  The compute stream has the higher priority, so the chain and
+    insert CTAs are placed first.  It waits for the prep, runs the chain hash
+    with the fused probe and inserts the uncached blocks.  Every step runs on
+    the GPU; nothing here computes.
     """
 
-    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_tokens: int, device="cuda"):
+    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_blocks: int, device="cuda"):
         self.cache, self.mode = cache, mode
-        dev = torch.device(device)
-        self.copy_stream = torch.cuda.Stream(dev)
-        self.compute_stream = torch.cuda.Stream(dev)
+        self.device = torch.device(device)
+        self.prep_stream = torch.cuda.Stream(self.device)
+        self.compute_stream = torch.cuda.Stream(self.device, priority=-1)
         cache.stream = self.compute_stream
-        max_blocks = max_tokens // K.BLOCK
         self.slots = []
         for _ in range(2):
             self.slots.append({
-                "tokens": torch.empty(max(max_tokens, 4), dtype=torch.int32, device=dev),
-                "tok_off": torch.empty(max_req + 1, dtype=torch.int64, device=dev),
-                "principal": torch.empty(max(max_req, 1), dtype=torch.int32, device=dev),
-                "boundary_tok": torch.empty(max(max_req, 1), dtype=torch.int32, device=dev),
-                "blk_off": torch.empty(max_req + 1, dtype=torch.int64, device=dev),
-                "digests": torch.empty((max(max_blocks, 1), 32), dtype=torch.uint8, device=dev),
-                "prefix": torch.empty(max(max_req, 1), dtype=torch.int32, device=dev),
-                "out": torch.empty(max(max_req, 1), dtype=torch.int32).pin_memory(),
-                "copied": torch.cuda.Event(), "free": torch.cuda.Event(), "used": False,
+                "salts": torch.empty((max(cache.n_principals, 1), 32), dtype=torch.uint8, device=self.device),
+                "blk_off": torch.empty(max_req + 1, dtype=torch.int64, device=self.device),
+                "digests": torch.empty((max(max_blocks, 1), 32), dtype=torch.uint8, device=self.device),
+                "prefix": torch.empty(max(max_req, 1), dtype=torch.int32, device=self.device),
+                "prepared": torch.cuda.Event(), "chain_start": torch.cuda.Event(), "free": torch.cuda.Event(),
+                "used": False,
             })
         self.i = 0
+        self.last_chain_start = None
 
-    def submit(self, tokens, tok_off, principal, boundary_tok, n_blocks: int, before_serve=None):
-        """Queue one batch given as pinned host tensors (int32 tokens, int64
-        offsets, int32 principal rows and boundary offsets).  before_serve, if
-        given, is called with the compute stream current just before serving
-        (for instance to flush the cache)."""
+    def _next_slot(self):
         s = self.slots[self.i % 2]
         self.i += 1
+        return s
+
+    def _prepare(self, s, db: DeviceBatch, after=None):
+        """Salts and block offsets of one batch on the prep stream."""
+        c = self.cache
+        ps = self.prep_stream
+        if after is not None:
+            ps.wait_event(after)
+        if self.last_chain_start is not None:
+            ps.wait_event(self.last_chain_start)    # the slot's previous batch has finished by then
+        elif s["used"]:
+            ps.wait_event(s["free"])
+        if self.mode != K.UNSALTED:
+            K.derive_salts(c.secret, c.ids, c.id_off, s["salts"], c.status, ps)
+        K.block_offsets(db.tok_off, s["blk_off"][:db.n + 1], c.status, ps)
+        s["prepared"].record(ps)
+
+    def _serve(self, s, db: DeviceBatch, before_serve=None, chain_events=None):
+        """Chain hash with the fused probe and the insert, on the compute stream."""
+        c = self.cache
+        cs = self.compute_stream
+        n = db.n
+        with torch.cuda.stream(cs):
+            cs.wait_event(s["prepared"])
+            if before_serve is not None:
+                before_serve()
+            salted = self.mode != K.UNSALTED
+            blk_off = s["blk_off"][:n + 1]
+            if chain_events is not None:
+                chain_events[0].record(cs)
+            # the last command before the chain launch: the prep of the next
+            # batch starts only once the chain kernel is being placed
+            s["chain_start"].record(cs)
+            self.last_chain_start = s["chain_start"]
+            digests, prefix = K.chain_hash_probe(
+                self.mode, db.tokens, db.tok_off, blk_off, c.slots, db.principal if salted else None,
+                s["salts"] if salted else None, db.boundary_tok if self.mode == K.BOUNDARY else None,
+                s["digests"][:db.n_blocks], s["prefix"][:n], n_blocks=db.n_blocks, status=c.status, stream=cs)
+            if chain_events is not None:
+                chain_events[1].record(cs)
+            K.insert_uncached(c.slots, digests, blk_off, prefix, c.status, c.n_new, cs)
+        s["used"] = True
+        return prefix, digests, blk_off
+
+
+class DevicePipeline(_Pipelined):
+    """Serve device-resident batches back to back, each batch's salts and
+    block offsets computed beside the previous batch's chain hash.
+
+    submit() returns (prefix_blocks, event) on the device: prefix_blocks is
+    valid once event has completed and is overwritten two submits later.
+    The batch's tensors are used on the pipeline's streams after the work
+    queued so far on the caller's current stream.
+    """
+
+    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_blocks: int, device="cuda"):
+        super().__init__(cache, mode, max_req, max_blocks, device)
+        self._ready = [torch.cuda.Event(), torch.cuda.Event()]
+
+    def submit(self, db: DeviceBatch, before_serve=None, chain_events=None):
+        """Queue one device-resident batch.  before_serve, if given, is called
+        with the compute stream current just before the chain hash (for
+        instance to flush the cache); chain_events, a pair of CUDA events, is
+        recorded around the chain-hash launch."""
+        ready = self._ready[self.i % 2]
+        ready.record(torch.cuda.current_stream(self.device))
+        for t in (db.tokens, db.tok_off, db.principal, db.boundary_tok):
+            t.record_stream(self.prep_stream)
+            t.record_stream(self.compute_stream)
+        self.compute_stream.wait_event(ready)
+        s = self._next_slot()
+        self._prepare(s, db, after=ready)
+        prefix, _, _ = self._serve(s, db, before_serve, chain_events)
+        s["free"].record(self.compute_stream)
+        return prefix, s["free"]
+
+
+class HostPipeline(_Pipelined):
+    """Serve batches that live in pinned host memory: each batch's
+    host-to-device copy runs on a copy stream while the previous batch is
+    served, its salts and block offsets follow on the prep stream, and the
+    compute stream serves it and copies the prefix lengths back into a pinned
+    host buffer.  A slot is reused only after the compute stream has finished
+    with it.
+
+    submit() returns (prefix_host, event): prefix_host is valid once event has
+    completed (event.synchronize()) and is overwritten two submits later.
+    """
+
+    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_tokens: int, device="cuda"):
+        super().__init__(cache, mode, max_req, max_tokens // K.BLOCK, device)
+        self.copy_stream = torch.cuda.Stream(self.device)
+        for s in self.slots:
+            s.update({
+                "tokens": torch.empty(max(max_tokens, 4), dtype=torch.int32, device=self.device),
+                "tok_off": torch.empty(max_req + 1, dtype=torch.int64, device=self.device),
+                "principal": torch.empty(max(max_req, 1), dtype=torch.int32, device=self.device),
+                "boundary_tok": torch.empty(max(max_req, 1), dtype=torch.int32, device=self.device),
+                "out": torch.empty(max(max_req, 1), dtype=torch.int32).pin_memory(),
+                "copied": torch.cuda.Event(),
+            })
+
+    def submit(self, tokens, tok_off, principal, boundary_tok, n_blocks: int, before_serve=None,
+               chain_events=None):
+        """Queue one batch given as pinned host tensors (int32 tokens, int64
+        offsets, int32 principal rows and boundary offsets).  before_serve, if
+        given, is called with the compute stream current just before the
+        chain hash (for instance to flush the cache); chain_events as in
+        DevicePipeline.submit."""
+        s = self._next_slot()
         n, t = tok_off.numel() - 1, tokens.numel()
         with torch.cuda.stream(self.copy_stream):
             if s["used"]:
@@ -179,15 +284,11 @@ class HostPipeline:
             s["principal"][:n].copy_(principal, non_blocking=True)
             s["boundary_tok"][:n].copy_(boundary_tok, non_blocking=True)
             s["copied"].record(self.copy_stream)
-        s["used"] = True
+        db = DeviceBatch(s["tokens"][:max(t, 4)], s["tok_off"][:n + 1], s["principal"][:n],
+                         s["boundary_tok"][:n], n_blocks)
+        self._prepare(s, db, after=s["copied"])
+        prefix, _, _ = self._serve(s, db, before_serve, chain_events)
         with torch.cuda.stream(self.compute_stream):
-            self.compute_stream.wait_event(s["copied"])
-            if before_serve is not None:
-                before_serve()
-            db = DeviceBatch(s["tokens"][:max(t, 4)], s["tok_off"][:n + 1], s["principal"][:n],
-                             s["boundary_tok"][:n], n_blocks)
-            bufs = {"blk_off": s["blk_off"][:n + 1], "digests": s["digests"][:n_blocks], "prefix": s["prefix"][:n]}
-            prefix, _, _ = self.cache.serve(self.mode, db, bufs)
             s["out"][:n].copy_(prefix, non_blocking=True)
             s["free"].record(self.compute_stream)
         return s["out"][:n], s["free"]

@@ -73,7 +73,8 @@ def test_salts_bad_offsets_flagged(kv):
 
 
 # --------------------------------------------------------- block offsets
-@pytest.mark.parametrize("n", [0, 1, 5, 127, 1024, 1025, 4097, 10000, 131073, 1000003])
+@pytest.mark.parametrize("n", [0, 1, 5, 127, 1024, 1025, 4097, 10000, 131073, 1000003, 1 << 20, (1 << 20) + 1,
+                               3000001])
 def test_block_offsets(kv, n):
     rng = np.random.default_rng(n)
     lens = rng.integers(0, 200, n)
@@ -83,6 +84,29 @@ def test_block_offsets(kv, n):
     torch.cuda.synchronize()
     assert (blk.cpu().numpy() == oracle.block_offsets(tok_off)).all()
     assert int(st.item()) == 0
+
+
+def test_block_offsets_reused_output_and_side_stream(kv):
+    """The output array doubles as the scan's mailboxes: values left in it by
+    an earlier call must not leak into the next one, and the scan must give
+    the same result on a second stream while a chain-hash launch runs."""
+    rng = np.random.default_rng(5)
+    offs = [np.concatenate([[0], np.cumsum(rng.integers(0, 300, 200000))]).astype(np.int64) for _ in range(3)]
+    out = torch.full((200001,), -7, dtype=torch.int64, device="cuda")
+    b = W.make("wide", seed=3, n_req=16384)
+    db_tok, db_off = dev(b.batch.tokens), dev(b.batch.tok_off)
+    blk_b = kv.block_offsets(db_off)
+    side = torch.cuda.Stream()
+    for t in offs:
+        st = status_tensor()
+        kv.chain_hash(0, db_tok, db_off, blk_b, n_blocks=16384 * 8)
+        ev = torch.cuda.Event()
+        ev.record()
+        side.wait_event(ev)
+        kv.block_offsets(dev(t), out, st, side)
+        torch.cuda.synchronize()
+        assert (out.cpu().numpy() == oracle.block_offsets(t)).all()
+        assert int(st.item()) == 0
 
 
 def test_block_offsets_negative_length_flagged(kv):

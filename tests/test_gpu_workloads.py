@@ -7,7 +7,9 @@ import torch
 
 import oracle
 from paper_2608_09225_gb300 import workloads as W
-from paper_2608_09225_gb300.pipeline import DeviceBatch, HostPipeline, PrefixCache, next_pow2
+from paper_2608_09225_gb300 import kvgov as K
+from paper_2608_09225_gb300.pipeline import (DeviceBatch, DevicePipeline, HostPipeline, PrefixCache,
+                                              next_pow2)
 from tests.pins import run_workload_oracle
 
 pytestmark = pytest.mark.gpu
@@ -177,3 +179,76 @@ def test_host_pipeline_matches_device_serving(kv):
         assert (g == w).all()
     assert int(dev_cache.n_new.item()) == int(host_cache.n_new.item())
     assert [int(x.min()) for x in want] == [0, 4, 4, 8, 4, 4]
+
+
+@pytest.mark.parametrize("mode", [W.UNSALTED, W.ROOT, W.BOUNDARY])
+def test_device_pipeline_matches_sequential_serving(kv, mode):
+    """DevicePipeline (salts and block offsets of batch i+1 on a prep stream
+    beside batch i's insert) gives the prefix lengths and the key count of
+    serving the same batches one by one, across secret changes and a flush
+    of the cache between batches."""
+    ws = [W.make("wide", seed=300 + i, n_req=20000) for i in range(3)]
+    for w in ws[1:]:
+        w.batch.tokens.reshape(-1, 128)[:, :64] = ws[0].batch.tokens[:64]
+    w0 = ws[0]
+    dbs = [DeviceBatch.from_host(w.batch.tokens, w.batch.tok_off, w.batch.principal, w.batch.boundary_tok)
+           for w in ws]
+    seq = PrefixCache(1 << 19, w0.secret, w0.ids, w0.id_off)
+    pip = PrefixCache(1 << 19, w0.secret, w0.ids, w0.id_off)
+    pipe = DevicePipeline(pip, mode, w0.batch.n, dbs[0].n_blocks)
+    order = [0, 1, 2, 0, 1, 2, 0]
+    got, want = [], []
+    for i, k in enumerate(order):
+        secret = w0.secret[:24] + (i // 3).to_bytes(8, "little")     # a new epoch every third batch
+        flush = i == 5
+        seq.set_secret(secret)
+        if flush:
+            K.table_init(seq.slots)
+        pre, _, _ = seq.serve(mode, dbs[k])
+        want.append(pre.cpu().numpy())
+        pip.set_secret(secret)
+        before = (lambda: K.table_init(pip.slots, pipe.compute_stream)) if flush else None
+        out, ev = pipe.submit(dbs[k], before)
+        ev.synchronize()
+        got.append(out.cpu().numpy())
+    torch.cuda.synchronize()
+    seq.check_status()
+    pip.check_status()
+    for g, w in zip(got, want):
+        assert (g == w).all()
+    assert int(seq.n_new.item()) == int(pip.n_new.item())
+    assert int(want[0].min()) == 0
+    if mode != W.ROOT:                 # the shared 64-token prefix is unsalted
+        assert int(want[1].min()) == 4
+
+
+def test_device_pipeline_back_to_back_matches_oracle(kv):
+    """Many batches queued without waiting in between: every batch's prefix
+    lengths (copied out on the compute stream right after its submit) match
+    the oracle's arrival-order replay of the same batches."""
+    ws = [W.make("wide", seed=400 + i, n_req=4096) for i in range(4)]
+    for w in ws[1:]:
+        w.batch.tokens.reshape(-1, 128)[:, :64] = ws[0].batch.tokens[:64]
+    w0 = ws[0]
+    dbs = [DeviceBatch.from_host(w.batch.tokens, w.batch.tok_off, w.batch.principal, w.batch.boundary_tok)
+           for w in ws]
+    cache = PrefixCache(1 << 17, w0.secret, w0.ids, w0.id_off)
+    pipe = DevicePipeline(cache, W.BOUNDARY, w0.batch.n, dbs[0].n_blocks)
+    order = [0, 1, 2, 3, 2, 0, 1, 3]
+    copies = []
+    for i, k in enumerate(order):
+        cache.set_secret(w0.secret[:24] + (i % 2).to_bytes(8, "little"))
+        pre, _ = pipe.submit(dbs[k])
+        with torch.cuda.stream(pipe.compute_stream):
+            copies.append(pre.clone())
+    torch.cuda.synchronize()
+    cache.check_status()
+    ks = oracle.KeySet(1)
+    for i, k in enumerate(order):
+        b = ws[k].batch
+        salts = oracle.derive_salts(w0.secret[:24] + (i % 2).to_bytes(8, "little"), w0.ids, w0.id_off)
+        d = oracle.chain_hash(W.BOUNDARY, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+        blk = oracle.block_offsets(b.tok_off)
+        assert (copies[i].cpu().numpy() == ks.prefix_blocks(d, blk)).all(), f"batch {i}"
+        ks.insert(d)
+    assert int(cache.n_new.item()) == ks.n
