@@ -49,6 +49,19 @@ CHAIN_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_chain.cu", "paper_2608_09225
 CHAIN_PROFILE = "profiles/chain_kernel_wide.md"
 
 
+def load_peaks() -> dict:
+    """Measured copy bandwidth of this GPU pool (written beside the repository
+    by the pool's driver); the profiling fallback of 6.8 TB/s without it."""
+    try:
+        with open(os.path.join(HERE, "MEASURED_PEAKS.json")) as f:
+            return json.load(f)
+    except (OSError, ValueError):
+        return {"hbm_gbs": 6800.0, "fallback": True}
+
+
+PEAKS = load_peaks()
+
+
 def chain_source_hash() -> str:
     import hashlib
     h = hashlib.sha256()
@@ -200,6 +213,32 @@ def measure_int_peak(torch, peak_lib_path):
         rates = [cnt * threads * iters * ops_iter / max(hi - lo, 1) for lo, hi, cnt in per_sm.values()]
         out[name] = float(np.median(rates))
     out["n_sm"] = n_sm
+    return out
+
+
+def measure_gather(torch, peak_lib_path, table: "torch.Tensor", n_reads: int = 1 << 25) -> dict:
+    """Random-slot read rate (GB/s of bytes read, best of 5) over `table`,
+    reading whole 32-byte slots and first halves, from libkvgov_peak."""
+    import ctypes
+    L = ctypes.CDLL(peak_lib_path)
+    L.kvgov_peak_gather.argtypes = [ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int, ctypes.c_int64,
+                                    ctypes.c_uint64, ctypes.c_void_p, ctypes.c_void_p]
+    sink = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = {"table_bytes": table.numel() * table.element_size(), "reads": n_reads}
+    for slot_bytes in (32, 16):
+        best = float("inf")
+        for rep in range(6):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            rc = L.kvgov_peak_gather(table.data_ptr(), table.shape[0], slot_bytes, n_reads, 12345 + rep,
+                                     sink.data_ptr(), torch.cuda.current_stream().cuda_stream)
+            b.record()
+            assert rc == 0, rc
+            b.synchronize()
+            if rep:
+                best = min(best, a.elapsed_time(b))
+        out[f"gbs_{slot_bytes}B"] = n_reads * slot_bytes / (best / 1e3) / 1e9
+        out[f"reads_per_s_{slot_bytes}B"] = n_reads / (best / 1e3)
     return out
 
 
@@ -378,21 +417,25 @@ def main():
     epoch = [1]
     launches = [0]
 
-    def step(db, ev=None):
+    def step(db, ev=None, ins_ev=None):
         cache.set_secret(epoch_secret(w0.secret, epoch[0]))
         epoch[0] += 1
         flushed = flush.before_step()              # load factor would pass 0.5: flush the cache
         before = (lambda: K.table_init(cache.slots, pipe.compute_stream)) if flushed else None
-        prefix, _ = pipe.submit(db, before, ev)
+        prefix, _ = pipe.submit(db, before, ev, ins_ev)
         launches[0] += 5 + int(flushed)   # salts, block offsets (2), chain hash + probe, insert (+ table init)
         return prefix
 
     for i in range(args.warmup):
         step(pool[(1 + i) % args.pool])
     torch.cuda.synchronize()
+    n_new_before = int(cache.n_new.item())
 
     chain_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                 for _ in range(args.steps)]
+    insert_every = 4                               # time every 4th insert: two events fewer on the critical path
+    insert_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                 if i % insert_every == 0 else None for i in range(args.steps)]
     t_start, t_stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     launches[0] = 0
     flushes_before = flush.flushes
@@ -404,7 +447,7 @@ def main():
         pipe.prep_stream.wait_event(t_start)
         h0 = time.perf_counter()
         for i in range(args.steps):
-            last_prefix = step(pool[(1 + args.warmup + i) % args.pool], chain_ev[i])
+            last_prefix = step(pool[(1 + args.warmup + i) % args.pool], chain_ev[i], insert_ev[i])
         host_ms = (time.perf_counter() - h0) * 1e3
         t_stop.record(pipe.compute_stream)
         torch.cuda.synchronize()
@@ -421,6 +464,8 @@ def main():
     kernel_launches = launches[0]
     ms = t_start.elapsed_time(t_stop)
     chain_ms = float(np.mean([a.elapsed_time(b) for a, b in chain_ev]))
+    insert_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in insert_ev if e is not None]))
+    inserted_per_step = (gate["n_new_total"] - n_new_before) / args.steps
     ms = max_over_ranks(ms, world, dist, "cuda")
     value = world * args.steps * n_blocks / (ms / 1e3)
 
@@ -447,6 +492,21 @@ def main():
                 "frac_of_sha256_microbench": achieved / (n_sm * micro["sha_alu"] * SM_MAX_MHZ * 1e6 / 1e12),
                 "frac_of_issue_peak": achieved / (n_sm * 128 * SM_MAX_MHZ * 1e6 / 1e12),
                 "traffic_source": traffic_src}
+    # the table kernel of the step (insert of the uncached blocks) against HBM and a random-read ceiling
+    gather = measure_gather(torch, kbuild.PEAK_LIB, cache.slots)
+    ins_bytes = 96 * inserted_per_step + 20 * n_req
+    ins_gbs = ins_bytes / (insert_ms / 1e3) / 1e9
+    table_roofline = {
+        "kernel": "insert_uncached_kernel<8> (kvgov_insert_uncached)", "bound": "hbm", "achieved": ins_gbs,
+        "peak": PEAKS.get("hbm_gbs"), "unit": "GB/s", "frac": ins_gbs / PEAKS["hbm_gbs"] if PEAKS.get("hbm_gbs") else None,
+        "peak_source": "of fallback (6.8 TB/s)" if PEAKS.get("fallback") else "of measured (MEASURED_PEAKS.json hbm_gbs, a copy)",
+        "random_read_ceiling_gbs": gather["gbs_32B"], "frac_of_random_read_ceiling": ins_gbs / gather["gbs_32B"],
+        "kernel_ms": insert_ms, "timed_launches": f"every {insert_every}th step of the timed region",
+        "keys_inserted_per_launch": inserted_per_step,
+        "inserts_per_s": inserted_per_step / (insert_ms / 1e3),
+        "algorithmic_bytes_per_launch": ins_bytes,
+        "bytes_basis": "per new key 32 B read + one 32 B slot read + 32 B written; per request 4 B prefix + 16 B offsets",
+        "random_read_microbench": gather}
     if clock.get("sm_mhz"):
         roofline["frac_at_run_clock"] = achieved / (n_sm * INT32_LANES_PER_SM * clock["sm_mhz"] * 1e6 / 1e12)
 
@@ -465,6 +525,7 @@ def main():
             "schedule": "DevicePipeline: salts (new epoch) and block offsets of batch i+1 on a prep stream beside "
                         "the chain hash of batch i; chain hash + probe, insert on a higher-priority compute stream",
             "e2e": e2e, "gpu_launches": kernel_launches, "clocks": clock, "roofline": roofline,
+            "table_roofline": table_roofline,
             "gate": gate}
     if rank == 0 and not args.no_cpu_baseline and world == 1:
         line["cpu_baseline"] = cpu_baseline(pool_host[0], args.cpu_sample, gate_digests)
@@ -557,19 +618,21 @@ def cpu_baseline(w, sample, gpu_digests):
 
 # --------------------------------------------------------------------------- per-workload rates
 def _time(torch, fn, reps=10, warm=3):
-    """Median CUDA-event time of fn() in ms (fn enqueues on the current stream)."""
+    """Mean CUDA-event time of fn() in ms over `reps` back-to-back calls (fn
+    enqueues on the current stream).  A GPU spin of about 2 ms is queued first,
+    so that every call is already queued when the first one starts: the time
+    is the GPU's, not the host's launch latency."""
     for _ in range(warm):
         fn()
     torch.cuda.synchronize()
-    ts = []
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda._sleep(4_000_000)
+    a.record()
     for _ in range(reps):
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record()
         fn()
-        b.record()
-        torch.cuda.synchronize()
-        ts.append(a.elapsed_time(b))
-    return float(np.median(ts))
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
 
 
 def _oracle_rate(w, mode, cores, budget_s=3.0):
@@ -618,6 +681,10 @@ def run_configs(args):
     cores = len(os.sched_getaffinity(0))
     l2 = torch.cuda.get_device_properties(0).L2_cache_size
     seed = args.seed
+    scratch_table = K.new_table(1 << 25)
+    gather = measure_gather(torch, kbuild.PEAK_LIB, scratch_table)
+    del scratch_table
+    print(json.dumps({"random_read_microbench": gather, "hbm_gbs": PEAKS.get("hbm_gbs")}), flush=True)
     plan = [("tiny", W.make("tiny"), W.ROOT), ("sysprompt", W.make("sysprompt"), W.ROOT)]
     tmpl = W.make("template")
     plan += [("template", tmpl, m) for m in (W.UNSALTED, W.ROOT, W.BOUNDARY)]
@@ -673,6 +740,13 @@ def run_configs(args):
         nb = np.diff(blk_np[p0:p1 + 1])
         algo_probes = int(np.minimum(L + 1, nb).sum())
         ops = nominal_chain_ops(b.lengths() // 16, mode, b.boundary_tok // 16)
+        # algorithmic table bytes, linear probing at load factor a: a hit walks 1/2 (1 + 1/(1-a)) slots,
+        # a miss 1/2 (1 + 1/(1-a)^2); a fill from empty to a averages 1/2 (1 + 1/(1-a)) per insert
+        a = keys.shape[0] / cap
+        hits = int(np.minimum(L, nb).sum())
+        misses = int((L < nb).sum())
+        probe_bytes = hits * (32 + 16 * (1 + 1 / (1 - a))) + misses * (32 + 16 * (1 + 1 / (1 - a) ** 2)) + 4 * (p1 - p0)
+        insert_bytes = keys.shape[0] * (32 + 16 * (1 + 1 / (1 - a)) + 32)
         line = {"workload": name, "mode": names[mode], "requests": b.n, "blocks": n_blocks,
                 "table_slots": cap, "table_fits_l2": cap * 32 <= l2,
                 "chain_ms": t_chain, "chain_digests_per_s": n_blocks / (t_chain / 1e3),
@@ -683,7 +757,12 @@ def run_configs(args):
                 "probe_ms": t_probe, "probed_requests": p1 - p0, "algorithmic_probes": algo_probes,
                 "probes_per_s": algo_probes / (t_probe / 1e3), "mean_prefix_blocks": float(L.mean()),
                 "insert_keys": int(keys.shape[0]), "insert_ms": t_insert - t_init,
-                "inserts_per_s": keys.shape[0] / ((t_insert - t_init) / 1e3)}
+                "inserts_per_s": keys.shape[0] / ((t_insert - t_init) / 1e3), "load_factor": a,
+                "probe_gbs": probe_bytes / (t_probe / 1e3) / 1e9,
+                "probe_frac_hbm": probe_bytes / (t_probe / 1e3) / 1e9 / PEAKS["hbm_gbs"],
+                "probe_frac_random_read": probe_bytes / (t_probe / 1e3) / 1e9 / gather["gbs_32B"],
+                "insert_gbs": insert_bytes / ((t_insert - t_init) / 1e3) / 1e9,
+                "insert_frac_random_read": insert_bytes / ((t_insert - t_init) / 1e3) / 1e9 / gather["gbs_32B"]}
         if not args.no_cpu_baseline:
             line.update(_oracle_rate(w, mode, cores))
             line["oracle_cores"] = cores

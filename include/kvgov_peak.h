@@ -1,7 +1,9 @@
 /*
  * kvgov_peak.h -- C ABI of libkvgov_peak: the integer issue-rate
- * microbenchmark that sets the roofline denominator for the hashing kernels.
- * It is a measurement tool beside libkvgov, not part of the method.
+ * microbenchmark that sets the roofline denominator for the hashing kernels,
+ * and the random-slot read microbenchmark that sets the ceiling for the
+ * table kernels.  They are measurement tools beside libkvgov, not part of
+ * the method.
  *
  * The hashing path of the paper (SHA-256 block keys and HMAC salts, section
  * 4.1; Table 9) is integer work: rotates, three-input booleans and adds.
@@ -30,6 +32,21 @@ typedef struct CUstream_st *kvgov_stream_t;
  */
 int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint32_t *d_sink,
                    unsigned long long *d_clocks, kvgov_stream_t stream);
+
+/*
+ * kvgov_peak_gather -- the bandwidth ceiling of the table kernels: `n_reads`
+ * reads of `slot_bytes` (16: the first half of a slot, as the fused lookup
+ * reads; 32: a whole slot, as the probe and insert read) at pseudo-random
+ * slots of a table of `n_slots` 32-byte slots (slot of read i =
+ * splitmix64(seed + i) mod n_slots).
+ *   d_table  [n_slots][32] bytes, device, 16-byte aligned, only read.
+ *   n_slots  a power of two.
+ *   d_sink   [1] u32, written only in a case that never happens.
+ * Asynchronous on `stream`.  Returns 0, 1 for a bad argument (nothing
+ * launched), 2 for a launch error.  Algorithmic bytes = n_reads x slot_bytes.
+ */
+int kvgov_peak_gather(const void *d_table, uint64_t n_slots, int slot_bytes, int64_t n_reads, uint64_t seed,
+                      uint32_t *d_sink, kvgov_stream_t stream);
 
 /* Thread-operations one thread executes per iteration of `kind` (nominal
  * SHA-256 count of 1384 per compression for kinds 3 and 4), or 0 for a bad

@@ -182,7 +182,7 @@ class _Pipelined:
         K.block_offsets(db.tok_off, s["blk_off"][:db.n + 1], c.status, ps)
         s["prepared"].record(ps)
 
-    def _serve(self, s, db: DeviceBatch, before_serve=None, chain_events=None):
+    def _serve(self, s, db: DeviceBatch, before_serve=None, chain_events=None, insert_events=None):
         """Chain hash with the fused probe and the insert, on the compute stream."""
         c = self.cache
         cs = self.compute_stream
@@ -205,7 +205,11 @@ class _Pipelined:
                 s["digests"][:db.n_blocks], s["prefix"][:n], n_blocks=db.n_blocks, status=c.status, stream=cs)
             if chain_events is not None:
                 chain_events[1].record(cs)
+            if insert_events is not None:
+                insert_events[0].record(cs)
             K.insert_uncached(c.slots, digests, blk_off, prefix, c.status, c.n_new, cs)
+            if insert_events is not None:
+                insert_events[1].record(cs)
         s["used"] = True
         return prefix, digests, blk_off
 
@@ -224,11 +228,11 @@ class DevicePipeline(_Pipelined):
         super().__init__(cache, mode, max_req, max_blocks, device)
         self._ready = [torch.cuda.Event(), torch.cuda.Event()]
 
-    def submit(self, db: DeviceBatch, before_serve=None, chain_events=None):
+    def submit(self, db: DeviceBatch, before_serve=None, chain_events=None, insert_events=None):
         """Queue one device-resident batch.  before_serve, if given, is called
         with the compute stream current just before the chain hash (for
-        instance to flush the cache); chain_events, a pair of CUDA events, is
-        recorded around the chain-hash launch."""
+        instance to flush the cache); chain_events and insert_events, pairs of
+        CUDA events, are recorded around the chain-hash and insert launches."""
         ready = self._ready[self.i % 2]
         ready.record(torch.cuda.current_stream(self.device))
         for t in (db.tokens, db.tok_off, db.principal, db.boundary_tok):
@@ -237,7 +241,7 @@ class DevicePipeline(_Pipelined):
         self.compute_stream.wait_event(ready)
         s = self._next_slot()
         self._prepare(s, db, after=ready)
-        prefix, _, _ = self._serve(s, db, before_serve, chain_events)
+        prefix, _, _ = self._serve(s, db, before_serve, chain_events, insert_events)
         s["free"].record(self.compute_stream)
         return prefix, s["free"]
 

@@ -24,8 +24,8 @@ def libkv():
     return ctypes.CDLL(path)
 
 
-def declared_functions():
-    text = open(HEADER).read()
+def declared_functions(header=HEADER):
+    text = open(header).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
     return sorted(set(re.findall(r"\b(kvgov_\w+)\s*\(", text)))
 
@@ -42,6 +42,32 @@ def test_header_declares_the_boundary():
 def test_library_exports_every_declared_symbol(libkv):
     for name in declared_functions():
         assert hasattr(libkv, name), name
+
+
+def test_peak_library_exports_every_declared_symbol():
+    kbuild.build()
+    lib = ctypes.CDLL(kbuild.PEAK_LIB)
+    names = declared_functions(os.path.join(ROOT, "include", "kvgov_peak.h"))
+    assert {"kvgov_peak_int", "kvgov_peak_gather", "kvgov_peak_ops_per_iter"} <= set(names)
+    for name in names:
+        assert hasattr(lib, name), name
+    assert sorted(os.listdir(os.path.join(ROOT, "include"))) == ["kvgov.h", "kvgov_peak.h"]
+
+
+def test_peak_gather_rejects_bad_arguments():
+    """Argument checks run on the host and launch nothing."""
+    kbuild.build()
+    f = ctypes.CDLL(kbuild.PEAK_LIB).kvgov_peak_gather
+    f.argtypes = [ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int, ctypes.c_int64, ctypes.c_uint64, ctypes.c_void_p,
+                  ctypes.c_void_p]
+    fake, sink = 1 << 20, 1 << 21          # never dereferenced: every call below fails its checks first
+    assert f(None, 1024, 32, 10, 0, sink, None) == 1
+    assert f(fake, 1000, 32, 10, 0, sink, None) == 1          # not a power of two
+    assert f(fake, 1024, 24, 10, 0, sink, None) == 1          # 16 or 32 bytes per read
+    assert f(fake, 1024, 32, -1, 0, sink, None) == 1
+    assert f(fake + 8, 1024, 32, 10, 0, sink, None) == 1      # not 16-byte aligned
+    assert f(fake, 1024, 32, 10, 0, None, None) == 1
+    assert f(fake, 1024, 32, 0, 0, sink, None) == 0           # nothing to read: nothing launched
 
 
 def test_status_strings(libkv):
