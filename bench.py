@@ -734,6 +734,26 @@ def run_configs(args):
         t_probe = _time(torch, lambda: K.probe(cache.slots, dig, pblk_view, pre[: p1 - p0]))
         t_fused = _time(torch, lambda: K.chain_hash_probe(mode, db.tokens, db.tok_off, blk, cache.slots, pr, sl, bt,
                                                           dig, pre))
+        # arrival order: the whole batch served request by request into an empty cache
+        acap = next_pow2(4 * n_blocks)
+        aslots, owner = K.new_table(acap), K.new_owner(acap)
+        slot_of = torch.empty(n_blocks, dtype=torch.int32, device="cuda")
+        pre_a = torch.empty(b.n, dtype=torch.int32, device="cuda")
+        seq = [1]
+
+        def arrival(probe=True):
+            K.table_init(aslots)
+            K.insert_arrival(aslots, owner, dig, blk, seq[0], cache.status, slot_of)
+            if probe:
+                K.probe_arrival(owner, slot_of, blk, seq[0], pre_a, cache.status)
+            seq[0] += n_blocks
+
+        t_arr = _time(torch, arrival, reps=5, warm=1)
+        t_arr_ins = _time(torch, lambda: arrival(False), reps=5, warm=1)
+        t_ainit = _time(torch, lambda: K.table_init(aslots), reps=5, warm=1)
+        arrival()
+        La = pre_a.cpu().numpy()
+        del aslots, owner, slot_of
         torch.cuda.synchronize()
         cache.check_status()
         L = K.probe(cache.slots, dig, pblk_view).cpu().numpy()
@@ -761,6 +781,10 @@ def run_configs(args):
                 "probe_gbs": probe_bytes / (t_probe / 1e3) / 1e9,
                 "probe_frac_hbm": probe_bytes / (t_probe / 1e3) / 1e9 / PEAKS["hbm_gbs"],
                 "probe_frac_random_read": probe_bytes / (t_probe / 1e3) / 1e9 / gather["gbs_32B"],
+                "arrival_insert_ms": t_arr_ins - t_ainit, "arrival_probe_ms": t_arr - t_arr_ins,
+                "arrival_blocks_per_s": n_blocks / ((t_arr - t_ainit) / 1e3),
+                "arrival_mean_prefix_blocks": float(La.mean()),
+                "arrival_hit_fraction": float(La.sum()) / max(1, n_blocks),
                 "insert_gbs": insert_bytes / ((t_insert - t_init) / 1e3) / 1e9,
                 "insert_frac_random_read": insert_bytes / ((t_insert - t_init) / 1e3) / 1e9 / gather["gbs_32B"]}
         if not args.no_cpu_baseline:

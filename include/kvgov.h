@@ -243,6 +243,75 @@ int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_
                           unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * Arrival-order serving of one batch -- paper section 2.1 (a lookup matches
+ * the longest cached prefix of blocks from position 0) and section 4.2
+ * (prefill cost is proportional to the uncached tokens), applied request by
+ * request: the requests of the batch arrive in order; request r's cached
+ * prefix is its longest run of leading blocks that were cached when it
+ * arrived (in the table before the batch, or blocks of a request that
+ * arrived before it), and then all its blocks are cached.  The result equals
+ * serving the requests one at a time with kvgov_probe and kvgov_insert, in
+ * one pass over the batch:
+ *
+ *   kvgov_insert_arrival(...)   every block's key into the table, recording
+ *                               its slot and, per slot, the first arrival;
+ *   kvgov_probe_arrival(...)    the prefix lengths.
+ *
+ * Arrival positions: block j of request r has position
+ * seq_base + blk_off[r] + j, so a batch covers blk_off[n_req] positions from
+ * seq_base.  The owner array d_owner [capacity] u64, beside the table, holds
+ * per slot the smallest position whose block inserted the slot's key through
+ * kvgov_insert_arrival (0 for keys inserted any other way, which count as
+ * cached before every arrival).  Zero it once with kvgov_owner_init when the
+ * table is created; it stays valid across kvgov_table_init as long as
+ * positions only grow: every call's seq_base must be at least the previous
+ * call's seq_base + blk_off[n_req] (on the same owner array).  seq_base lies
+ * in [1, 2^62].  capacity: a power of two in [32, 2^31].
+ */
+
+/*
+ * kvgov_owner_init -- zero d_owner [capacity] u64 (16-byte aligned).
+ * EINVAL: NULL or misaligned pointer, bad capacity.
+ */
+int kvgov_owner_init(uint64_t *d_owner, uint64_t capacity, kvgov_stream_t stream);
+
+/*
+ * kvgov_insert_arrival -- insert every block of the batch (the set semantics
+ * and protocol of kvgov_insert) and settle the owners of the keys it adds.
+ *   d_slots, capacity, d_digests, d_blk_off, n_req  as for kvgov_probe.
+ *   d_owner    [capacity] u64, see above.
+ *   seq_base   arrival position of the batch's first block.
+ *   d_slot_of  [d_blk_off[n_req]] u32 output: the slot holding each block's
+ *              key, or 0xFFFFFFFF if it could not be stored (reserved key,
+ *              full window, timeout -- flagged in *d_status).  This is the
+ *              block's handle in the cache and the input of
+ *              kvgov_probe_arrival.
+ *   d_n_new, d_status  as for kvgov_insert (d_status required); also
+ *              KVGOV_F_BADINDEX if d_blk_off[n_req] < 0.
+ * Two launches on `stream`, one thread per block.  Must not overlap in time
+ * with other calls on the same table or owner array.  n_req = 0 is a no-op.
+ * EINVAL: bad capacity, NULL or misaligned pointer, seq_base out of range.
+ */
+int kvgov_insert_arrival(uint8_t *d_slots, uint64_t *d_owner, uint64_t capacity, const uint8_t *d_digests,
+                         const int64_t *d_blk_off, int32_t n_req, uint64_t seq_base, uint32_t *d_slot_of,
+                         unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream);
+
+/*
+ * kvgov_probe_arrival -- d_prefix_blocks[r] = the smallest j such that block
+ * j of request r was not cached when r arrived (its d_slot_of is 0xFFFFFFFF,
+ * or its slot's owner is >= seq_base + d_blk_off[r]), or n_b(r) if every
+ * block was.  Run after kvgov_insert_arrival of the same batch (same
+ * d_blk_off, n_req and seq_base) and before the next call on the owner array.
+ *   d_owner, capacity  as for kvgov_insert_arrival; d_slot_of its output.
+ *   d_status  nullable; KVGOV_F_BADINDEX for malformed offsets.
+ * n_req = 0 is a no-op.  EINVAL: bad capacity, NULL pointer, seq_base out of
+ * range.
+ */
+int kvgov_probe_arrival(const uint64_t *d_owner, uint64_t capacity, const uint32_t *d_slot_of,
+                        const int64_t *d_blk_off, int32_t n_req, uint64_t seq_base, int32_t *d_prefix_blocks,
+                        uint32_t *d_status, kvgov_stream_t stream);
+
+/*
  * kvgov_set_spin_limit -- bound on how many times an inserting thread
  * re-reads a slot whose key another thread is still writing before it gives
  * up with KVGOV_F_TIMEOUT (about 100 ns per re-read).

@@ -62,6 +62,8 @@ def _configure(L):
     L.oracle_set_insert.restype = _i64
     L.oracle_prefix_blocks.argtypes = [_p, _i64, _p, _p, _i32, _p]
     L.oracle_prefix_blocks.restype = ctypes.c_int
+    L.oracle_arrival_prefix.argtypes = [_p, _i64, _p, _p, _i32, _p, _p]
+    L.oracle_arrival_prefix.restype = ctypes.c_int
     return L
 
 
@@ -218,3 +220,18 @@ class KeySet:
         if rc != 0:
             raise ValueError("oracle_prefix_blocks: malformed block offsets")
         return out
+
+    def arrival_prefix(self, digests: np.ndarray, blk_off: np.ndarray):
+        """Arrival-order serving of a batch against this set (left unchanged):
+        request r's prefix counts the set's keys and every block of requests
+        before r; returns (prefix_blocks, n_new), n_new = keys the batch adds."""
+        digests = _c(digests, np.uint8).reshape(-1, 32)
+        blk_off = _c(blk_off, np.int64)
+        n = len(blk_off) - 1
+        out = np.zeros(n, np.int32)
+        n_new = ctypes.c_int64(0)
+        rc = lib().oracle_arrival_prefix(_ptr(self.keys), self.n, _ptr(digests), _ptr(blk_off), n, _ptr(out),
+                                         ctypes.byref(n_new))
+        if rc != 0:
+            raise ValueError("oracle_arrival_prefix: malformed block offsets or out of memory")
+        return out, n_new.value

@@ -23,6 +23,9 @@
  *                        row 1 (the oracle returns the first k matched
  *                        blocks) and section 5.7 (a divergence at token i
  *                        invalidates blocks floor(i/B) onward).
+ *   arrival-order ...... the same lookup applied request by request, each
+ *   serving              request then caching its blocks (sections 2.1 and
+ *                        4.2): a sequential replay over a chained hash set.
  *
  * Byte conventions (readings where the paper is silent): a token is its
  * int32 value serialised as 4 little-endian bytes; a block is B = 16 tokens
@@ -40,7 +43,9 @@
  * Parity pins (tests/test_oracle_pins.py): SHA-256 against Python hashlib on
  * every message length 0..300 and random messages; HMAC against Python hmac;
  * each chain equation against hashlib compositions; the paper's worked
- * examples of section 4.2 and section 5.7; brute force on tiny inputs.
+ * examples of section 4.2 and section 5.7; brute force on tiny inputs; the
+ * arrival-order replay against a Python-set replay and closed forms
+ * (repeated requests, multi-turn prefix extensions, per-principal salts).
  */
 #include <stddef.h>
 #include <stdint.h>
@@ -393,5 +398,98 @@ int oracle_prefix_blocks(const uint8_t *set_keys, int64_t n_set,
             j++;
         prefix_blocks[r] = (int32_t)j;
     }
+    return 0;
+}
+
+/* --------------------------------------------------------------------- */
+/*
+ * Arrival-order serving of one batch (paper section 2.1: a lookup matches
+ * the longest cached prefix of blocks from position 0; section 4.2: the
+ * uncached blocks are prefilled, after which they are cached), written as its
+ * definition: the requests are taken one at a time, in order.  Request r's
+ * prefix length is its number of leading blocks present in the set as it
+ * stands -- the keys given (cached before the batch) plus every block of
+ * requests 0..r-1 -- and then all of r's storable blocks join the set.
+ *
+ * The set is a chained hash set: bucket heads indexed by bytes 8..15 of the
+ * key, a node array with next links, keys compared whole.
+ */
+typedef struct {
+    int64_t *head;            /* [n_buckets] first node or -1 */
+    int64_t *next;            /* [cap] next node or -1 */
+    const uint8_t **key;      /* [cap] the node's key (points into the inputs) */
+    int64_t n, cap;
+    uint64_t mask;
+} chain_set;
+
+static uint64_t chain_set_bucket(const chain_set *s, const uint8_t *k)
+{
+    uint64_t h = 0;
+    for (int i = 15; i >= 8; i--) h = (h << 8) | k[i];
+    return h & s->mask;
+}
+
+static int chain_set_contains(const chain_set *s, const uint8_t *k)
+{
+    for (int64_t i = s->head[chain_set_bucket(s, k)]; i >= 0; i = s->next[i])
+        if (memcmp(s->key[i], k, 32) == 0) return 1;
+    return 0;
+}
+
+/* Adds k if absent; returns 1 if it was added. */
+static int chain_set_add(chain_set *s, const uint8_t *k)
+{
+    if (chain_set_contains(s, k)) return 0;
+    const uint64_t b = chain_set_bucket(s, k);
+    s->key[s->n] = k;
+    s->next[s->n] = s->head[b];
+    s->head[b] = s->n;
+    s->n++;
+    return 1;
+}
+
+/*
+ * set_keys[0..n_set): the keys cached before the batch.  digests, blk_off,
+ * n_req: the batch (request-major digests, block offsets).  prefix_blocks
+ * [n_req] receives the prefix lengths, *n_new how many keys the batch added
+ * to the set.  Reserved keys (oracle_key_reserved) are never added, as in
+ * oracle_set_insert.  Returns 0, or -1 for malformed offsets or no memory.
+ */
+int oracle_arrival_prefix(const uint8_t *set_keys, int64_t n_set, const uint8_t *digests,
+                          const int64_t *blk_off, int32_t n_req, int32_t *prefix_blocks,
+                          int64_t *n_new)
+{
+    if (n_set < 0 || n_req < 0 || blk_off[0] != 0) return -1;
+    for (int32_t r = 0; r < n_req; r++)
+        if (blk_off[r + 1] < blk_off[r]) return -1;
+    const int64_t cap = n_set + blk_off[n_req] + 1;
+    uint64_t n_buckets = 1;
+    while (n_buckets < (uint64_t)(2 * cap)) n_buckets <<= 1;
+    chain_set s;
+    s.head = malloc(n_buckets * sizeof(int64_t));
+    s.next = malloc((size_t)cap * sizeof(int64_t));
+    s.key = malloc((size_t)cap * sizeof(const uint8_t *));
+    s.n = 0;
+    s.cap = cap;
+    s.mask = n_buckets - 1;
+    if (!s.head || !s.next || !s.key) {
+        free(s.head); free(s.next); free(s.key);
+        return -1;
+    }
+    for (uint64_t b = 0; b < n_buckets; b++) s.head[b] = -1;
+    for (int64_t i = 0; i < n_set; i++) chain_set_add(&s, set_keys + 32 * (size_t)i);
+    const int64_t before = s.n;
+    for (int32_t r = 0; r < n_req; r++) {
+        const uint8_t *req = digests + 32 * (size_t)blk_off[r];
+        const int64_t nb = blk_off[r + 1] - blk_off[r];
+        int64_t j = 0;
+        while (j < nb && chain_set_contains(&s, req + 32 * (size_t)j))
+            j++;
+        prefix_blocks[r] = (int32_t)j;
+        for (int64_t q = 0; q < nb; q++)
+            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);
+    }
+    *n_new = s.n - before;
+    free(s.head); free(s.next); free(s.key);
     return 0;
 }

@@ -29,6 +29,9 @@ namespace kvgov_host {
 inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline bool pow2_capacity(uint64_t cap) { return cap >= KVGOV_MIN_CAPACITY && (cap & (cap - 1)) == 0; }
 
+// The bound on every wait of the insert protocol (kvgov_set_spin_limit).
+uint32_t spin_limit();
+
 inline int launch_status() {
     return cudaGetLastError() == cudaSuccess ? KVGOV_OK : KVGOV_ECUDA;
 }

@@ -59,10 +59,15 @@ def _load():
         L.kvgov_insert.argtypes = [_p, ctypes.c_uint64, _p, ctypes.c_int64, _p, _p, _p]
         L.kvgov_probe.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p]
         L.kvgov_insert_uncached.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p, _p]
+        L.kvgov_owner_init.argtypes = [_p, ctypes.c_uint64, _p]
+        L.kvgov_insert_arrival.argtypes = [_p, _p, ctypes.c_uint64, _p, _p, ctypes.c_int32, ctypes.c_uint64, _p, _p,
+                                           _p, _p]
+        L.kvgov_probe_arrival.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, ctypes.c_uint64, _p, _p, _p]
         L.kvgov_set_spin_limit.argtypes = [ctypes.c_uint32]
         L.kvgov_set_spin_limit.restype = ctypes.c_uint32
         for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
-                   "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe"):
+                   "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
+                   "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival"):
             getattr(L, fn).restype = ctypes.c_int
         _lib = L
         return L
@@ -252,6 +257,55 @@ def insert_uncached(slots: torch.Tensor, digests: torch.Tensor, blk_off: torch.T
                                        _dev(n_new, torch.int64, "n_new", True), _dev(status, torch.int32, "status"),
                                        _stream(stream)),
            "kvgov_insert_uncached")
+
+
+# ---- arrival-order serving (paper sections 2.1 and 4.2, request by request)
+def owner_init(owner: torch.Tensor, stream=None) -> torch.Tensor:
+    """Zero a table's owner array ([capacity] int64 holding u64 arrival positions)."""
+    _check(lib().kvgov_owner_init(_dev(owner, torch.int64, "owner"), owner.numel(), _stream(stream)),
+           "kvgov_owner_init")
+    return owner
+
+
+def new_owner(capacity: int, device="cuda", stream=None) -> torch.Tensor:
+    return owner_init(torch.empty(capacity, dtype=torch.int64, device=device), stream)
+
+
+def insert_arrival(slots: torch.Tensor, owner: torch.Tensor, digests: torch.Tensor, blk_off: torch.Tensor,
+                   seq_base: int, status: torch.Tensor, slot_of: torch.Tensor | None = None,
+                   n_new: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Insert every block of the batch, block j of request r arriving at
+    position seq_base + blk_off[r] + j; returns slot_of ([n_blocks] int32:
+    the slot of each block, -1 if not stored)."""
+    n = blk_off.numel() - 1
+    n_blocks = digests.shape[0] if digests.dim() == 2 else 0
+    if slot_of is None:
+        slot_of = torch.empty(n_blocks, dtype=torch.int32, device=blk_off.device)
+    _check(lib().kvgov_insert_arrival(_dev(slots, torch.uint8, "slots"), _dev(owner, torch.int64, "owner"),
+                                      slots.shape[0],
+                                      _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(blk_off),
+                                      _dev(blk_off, torch.int64, "blk_off"), n, int(seq_base),
+                                      _dev(slot_of, torch.int32, "slot_of") if slot_of.numel() else _dummy(blk_off),
+                                      _dev(n_new, torch.int64, "n_new", True), _dev(status, torch.int32, "status"),
+                                      _stream(stream)),
+           "kvgov_insert_arrival")
+    return slot_of
+
+
+def probe_arrival(owner: torch.Tensor, slot_of: torch.Tensor, blk_off: torch.Tensor, seq_base: int,
+                  prefix_blocks: torch.Tensor | None = None, status: torch.Tensor | None = None,
+                  stream=None) -> torch.Tensor:
+    """prefix_blocks[r] = blocks of request r cached when it arrived (after insert_arrival)."""
+    n = blk_off.numel() - 1
+    if prefix_blocks is None:
+        prefix_blocks = torch.empty(n, dtype=torch.int32, device=blk_off.device)
+    _check(lib().kvgov_probe_arrival(_dev(owner, torch.int64, "owner"), owner.numel(),
+                                     _dev(slot_of, torch.int32, "slot_of") if slot_of.numel() else _dummy(blk_off),
+                                     _dev(blk_off, torch.int64, "blk_off"), n, int(seq_base),
+                                     _dev(prefix_blocks, torch.int32, "prefix_blocks"),
+                                     _dev(status, torch.int32, "status", True), _stream(stream)),
+           "kvgov_probe_arrival")
+    return prefix_blocks
 
 
 def set_spin_limit(limit: int) -> int:

@@ -382,4 +382,108 @@ def pin_template_ordering():
     assert Ls[UNSALTED].mean() > Ls[BOUNDARY].mean()
 
 
+# ------------------------------------------------------ arrival-order serving
+def _reserved_py(k: bytes) -> bool:
+    return not any(k[:16]) or not any(k[16:24]) or not any(k[24:])
+
+
+def _replay_python(S0, digests, off):
+    """Serve the requests one at a time with a Python set: count the leading
+    cached blocks, then cache the request's blocks."""
+    S = {bytes(k) for k in S0}
+    before, out = len(S), []
+    for r in range(len(off) - 1):
+        rows = [digests[i].tobytes() for i in range(int(off[r]), int(off[r + 1]))]
+        L = 0
+        while L < len(rows) and rows[L] in S:
+            L += 1
+        out.append(L)
+        S.update(k for k in rows if not _reserved_py(k))
+    return out, len(S) - before
+
+
+def pin_arrival_brute_force():
+    """Arrival-order serving == a Python-set replay, request by request, on
+    batches whose requests copy leading keys of earlier ones, with keys cached
+    before the batch and the odd reserved key."""
+    rng = np.random.default_rng(19)
+    for trial in range(40):
+        n_req = int(rng.integers(1, 40))
+        pool = rng.integers(0, 256, (16, 32), dtype=np.uint8)
+        pool[:, 0] |= 1
+        pool[15, :16] = 0                                  # reserved: never stored
+        reqs = []
+        for r in range(n_req):
+            nb = int(rng.integers(0, 10))
+            keys = list(rng.integers(0, 16, nb))
+            if reqs and rng.random() < 0.6:               # start with a copy of an earlier request's prefix
+                src = reqs[int(rng.integers(0, len(reqs)))]
+                c = int(rng.integers(0, len(src) + 1))
+                keys = list(src[:c]) + keys
+            reqs.append(keys)
+        off = np.concatenate([[0], np.cumsum([len(k) for k in reqs])]).astype(np.int64)
+        digests = pool[np.array([i for k in reqs for i in k], dtype=np.int64)].reshape(-1, 32)
+        s0 = pool[:15][rng.random(15) < 0.3]
+        ks = oracle.KeySet(1)
+        ks.insert(s0)
+        got, n_new = ks.arrival_prefix(digests, off)
+        want, want_new = _replay_python(s0, digests, off)
+        assert list(got) == want and n_new == want_new, trial
+
+
+def pin_arrival_repeats_and_turns():
+    """Closed forms: a request repeated by its principal hits every block the
+    second time; the turns of one conversation, each an exact prefix extension
+    of the one before (section 6: multi-turn reuse), hit all blocks of the
+    previous turn."""
+    salts = oracle.derive_salts(b"q" * 32, *W.principal_ids(4))
+    rng = np.random.default_rng(20)
+    t = rng.integers(0, W.VOCAB, 100, dtype=np.int32)
+    toks = np.tile(t, 5)
+    off = np.arange(0, 501, 100, dtype=np.int64)
+    d = oracle.chain_hash(ROOT, toks, off, np.full(5, 2, np.int32), salts, np.zeros(5, np.int32))
+    L, n_new = oracle.KeySet(1).arrival_prefix(d, oracle.block_offsets(off))
+    assert list(L) == [0, 6, 6, 6, 6] and n_new == 6
+    conv = rng.integers(0, W.VOCAB, 200, dtype=np.int32)
+    turns = [conv[: 16 * (r + 1) + 5] for r in range(10)]
+    toks = np.concatenate(turns)
+    off = np.concatenate([[0], np.cumsum([len(x) for x in turns])]).astype(np.int64)
+    d = oracle.chain_hash(ROOT, toks, off, np.ones(10, np.int32), salts, np.zeros(10, np.int32))
+    L, n_new = oracle.KeySet(1).arrival_prefix(d, oracle.block_offsets(off))
+    assert list(L) == list(range(10)) and n_new == 10
+
+
+def pin_arrival_per_principal():
+    """Sixteen requests with one prompt, principal r mod 4: salted at the
+    root, a principal's first request misses and its later ones hit every
+    block (section 4.1); unsalted, only request 0 misses; salted at block 2
+    (section 4.2), the first request of principals 1-3 still hits the 2 shared
+    blocks."""
+    salts = oracle.derive_salts(b"r" * 32, *W.principal_ids(4))
+    t = np.random.default_rng(21).integers(0, W.VOCAB, 130, dtype=np.int32)
+    toks = np.tile(t, 16)
+    off = np.arange(0, 16 * 130 + 1, 130, dtype=np.int64)
+    pr = (np.arange(16) % 4).astype(np.int32)
+    b = np.full(16, 32, np.int32)
+    blk = oracle.block_offsets(off)
+    want = {ROOT: [0] * 4 + [8] * 12, UNSALTED: [0] + [8] * 15, BOUNDARY: [0] + [2] * 3 + [8] * 12}
+    for mode, w in want.items():
+        d = oracle.chain_hash(mode, toks, off, pr, salts, b)
+        L, _ = oracle.KeySet(1).arrival_prefix(d, blk)
+        assert list(L) == w, mode
+
+
+def pin_arrival_tiny_closed_form():
+    """Tiny workload served in arrival order into an empty cache: request r of
+    the 32 template requests hits the 8 template blocks once request r-8 (same
+    principal) has been served; the 32 others share nothing."""
+    w = W.make("tiny")
+    salts = oracle.derive_salts(w.secret, w.ids, w.id_off)
+    b = w.batch
+    d = oracle.chain_hash(ROOT, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+    L, n_new = oracle.KeySet(1).arrival_prefix(d, oracle.block_offsets(b.tok_off))
+    assert list(L) == [0] * 8 + [8] * 24 + [0] * 32
+    assert n_new == 64 * 16 - 24 * 8
+
+
 PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

@@ -34,7 +34,7 @@ def test_header_declares_the_boundary():
     names = declared_functions()
     for want in ("kvgov_derive_salts", "kvgov_block_offsets", "kvgov_chain_hash", "kvgov_table_init",
                  "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
-                 "kvgov_status_string",
+                 "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_status_string",
                  "kvgov_set_spin_limit"):
         assert want in names
 
@@ -137,6 +137,25 @@ def test_host_validation_rejects_bad_arguments(libkv):
     bo = libkv.kvgov_block_offsets
     bo.argtypes = [p, ctypes.c_int32, p, p, p]
     assert bo(fake, -2, fake, None, None) == 1
+    oi = libkv.kvgov_owner_init
+    oi.argtypes = [p, ctypes.c_uint64, p]
+    assert oi(None, 64, None) == 1
+    assert oi(odd, 64, None) == 1
+    assert oi(fake, 100, None) == 1
+    assert oi(fake, 1 << 32, None) == 1                                   # slot index must fit in u32
+    ia = libkv.kvgov_insert_arrival
+    ia.argtypes = [p, p, ctypes.c_uint64, p, p, ctypes.c_int32, ctypes.c_uint64, p, p, p, p]
+    assert ia(fake, fake, 64, fake, fake, 3, 0, fake, None, fake, None) == 1            # position 0 is reserved
+    assert ia(fake, fake, 64, fake, fake, 3, (1 << 62) + 1, fake, None, fake, None) == 1   # past 2^62
+    assert ia(fake, fake, 64, fake, fake, 3, 1, fake, None, None, None) == 1            # status is required
+    assert ia(fake, fake, 64, fake, fake, 3, 1, None, None, fake, None) == 1            # no slot_of
+    assert ia(fake, fake, 64, odd, fake, 3, 1, fake, None, fake, None) == 1             # misaligned digests
+    assert ia(fake, fake, 64, None, None, 0, 1, None, None, fake, None) == 0            # empty batch
+    pa = libkv.kvgov_probe_arrival
+    pa.argtypes = [p, ctypes.c_uint64, p, p, ctypes.c_int32, ctypes.c_uint64, p, p, p]
+    assert pa(fake, 64, fake, fake, 3, 0, fake, None, None) == 1
+    assert pa(fake, 64, fake, fake, 3, 1, None, None, None) == 1
+    assert pa(fake, 64, None, None, 0, 1, None, None, None) == 0
 
 
 def test_golden_file_is_what_the_oracle_computes():

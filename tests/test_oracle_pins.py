@@ -59,6 +59,23 @@ MUTATIONS = [
     ("lookup_counts_all_hits",
      "while (j < nb && oracle_set_contains(set_keys, n_set, digests + 32 * (size_t)(blk_off[r] + j)))\n            j++;",
      "for (int64_t q = 0; q < nb; q++) j += oracle_set_contains(set_keys, n_set, digests + 32 * (size_t)(blk_off[r] + q));"),
+    ("arrival_caches_before_lookup",
+     "        while (j < nb && chain_set_contains(&s, req + 32 * (size_t)j))\n            j++;\n"
+     "        prefix_blocks[r] = (int32_t)j;\n"
+     "        for (int64_t q = 0; q < nb; q++)\n"
+     "            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);",
+     "        for (int64_t q = 0; q < nb; q++)\n"
+     "            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);\n"
+     "        while (j < nb && chain_set_contains(&s, req + 32 * (size_t)j))\n            j++;\n"
+     "        prefix_blocks[r] = (int32_t)j;"),
+    ("arrival_initial_set_dropped",
+     "for (int64_t i = 0; i < n_set; i++) chain_set_add(&s, set_keys + 32 * (size_t)i);", ""),
+    ("arrival_counts_all_hits",
+     "        while (j < nb && chain_set_contains(&s, req + 32 * (size_t)j))\n            j++;",
+     "        for (int64_t q = 0; q < nb; q++) j += chain_set_contains(&s, req + 32 * (size_t)q);"),
+    ("arrival_reserved_keys_stored",
+     "            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);",
+     "            chain_set_add(&s, req + 32 * (size_t)q);"),
 ]
 
 
