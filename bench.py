@@ -352,6 +352,7 @@ def main():
     ap.add_argument("--impl", default="kvgov", choices=["kvgov", "reference"])
     ap.add_argument("--pool", type=int, default=16, help="distinct resident batches cycled by the steps")
     ap.add_argument("--e2e-steps", type=int, default=100)
+    ap.add_argument("--arrival-steps", type=int, default=50)
     ap.add_argument("--table-slots", type=int, default=1 << 25, help="cache capacity (power of two)")
     ap.add_argument("--seed", type=int, default=None, help="base seed (default: fresh per run)")
     ap.add_argument("--cpu-sample", type=int, default=16384, help="requests per oracle step")
@@ -469,6 +470,9 @@ def main():
     ms = max_over_ranks(ms, world, dist, "cuda")
     value = world * args.steps * n_blocks / (ms / 1e3)
 
+    # ---- arrival-order serving of the same batches (kvgov_chain_hash_arrival), each into an empty cache
+    arrival = arrival_leg(torch, K, W, pool, n_req, n_blocks, cache, args.arrival_steps, chain_ms)
+
     # ---- end to end through the public API with host buffers
     e2e = e2e_leg(torch, K, W, w0, pool_host[: min(4, args.pool)], args.e2e_steps, world, dist, args.table_slots)
 
@@ -526,7 +530,7 @@ def main():
                         "the chain hash of batch i; chain hash + probe, insert on a higher-priority compute stream",
             "e2e": e2e, "gpu_launches": kernel_launches, "clocks": clock, "roofline": roofline,
             "table_roofline": table_roofline,
-            "gate": gate}
+            "arrival": arrival, "gate": gate}
     if rank == 0 and not args.no_cpu_baseline and world == 1:
         line["cpu_baseline"] = cpu_baseline(pool_host[0], args.cpu_sample, gate_digests)
         if not line["cpu_baseline"]["gate_sample_digests_equal_gpu"]:
@@ -536,6 +540,44 @@ def main():
     if world > 1:
         dist.destroy_process_group()
     return 0
+
+
+def arrival_leg(torch, K, W, pool, n_req, n_blocks, cache, steps, chain_ms):
+    """kvgov_chain_hash_arrival on the pool's batches: each batch is served in
+    arrival order into an empty 2^22-slot cache (re-initialised before the
+    timed call), CUDA events around the call on its stream."""
+    cap = 1 << 22
+    slots, owner = K.new_table(cap), K.new_owner(cap)
+    blk = torch.empty(n_req + 1, dtype=torch.int64, device="cuda")
+    dig = torch.empty((n_blocks, 32), dtype=torch.uint8, device="cuda")
+    slot_of = torch.empty(n_blocks, dtype=torch.int32, device="cuda")
+    pre = torch.empty(n_req, dtype=torch.int32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    n_new = torch.zeros(1, dtype=torch.int64, device="cuda")
+    seq, times, means = 1, [], []
+    for i in range(steps + 3):
+        db = pool[i % len(pool)]
+        K.table_init(slots)
+        K.block_offsets(db.tok_off, blk, status)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        K.chain_hash_arrival(W.BOUNDARY, db.tokens, db.tok_off, blk, slots, owner, seq, status, db.principal,
+                             cache.salts, db.boundary_tok, dig, slot_of, pre, n_new=n_new)
+        b.record()
+        seq += n_blocks
+        if i >= 3:
+            times.append((a, b))
+            if i == 3:
+                means.append(float(pre.float().mean().item()))
+    torch.cuda.synchronize()
+    if int(status.item()) != 0:
+        raise SystemExit(f"arrival leg: device status {int(status.item())}")
+    ms = float(np.mean([x.elapsed_time(y) for x, y in times]))
+    return {"api": "kvgov_chain_hash_arrival (chain hash, arrival-order insert fused into it, owner min, probe)",
+            "ms_per_batch": ms, "blocks_per_s": n_blocks / (ms / 1e3), "steps": steps,
+            "chain_hash_probe_ms": chain_ms, "extra_over_chain_hash_probe_ms": ms - chain_ms,
+            "mean_prefix_blocks": means[0] if means else None,
+            "cache": f"empty {cap}-slot table per batch (re-initialised outside the timed call)"}
 
 
 def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots):
@@ -748,6 +790,13 @@ def run_configs(args):
                 K.probe_arrival(owner, slot_of, blk, seq[0], pre_a, cache.status)
             seq[0] += n_blocks
 
+        def arrival_fused():
+            K.table_init(aslots)
+            K.chain_hash_arrival(mode, db.tokens, db.tok_off, blk, aslots, owner, seq[0], cache.status, pr, sl, bt,
+                                 dig, slot_of, pre_a)
+            seq[0] += n_blocks
+
+        t_arr_fused = _time(torch, arrival_fused, reps=5, warm=1)
         t_arr = _time(torch, arrival, reps=5, warm=1)
         t_arr_ins = _time(torch, lambda: arrival(False), reps=5, warm=1)
         t_ainit = _time(torch, lambda: K.table_init(aslots), reps=5, warm=1)
@@ -782,6 +831,8 @@ def run_configs(args):
                 "probe_frac_hbm": probe_bytes / (t_probe / 1e3) / 1e9 / PEAKS["hbm_gbs"],
                 "probe_frac_random_read": probe_bytes / (t_probe / 1e3) / 1e9 / gather["gbs_32B"],
                 "arrival_insert_ms": t_arr_ins - t_ainit, "arrival_probe_ms": t_arr - t_arr_ins,
+                "chain_arrival_ms": t_arr_fused - t_ainit,
+                "chain_arrival_blocks_per_s": n_blocks / ((t_arr_fused - t_ainit) / 1e3),
                 "arrival_blocks_per_s": n_blocks / ((t_arr - t_ainit) / 1e3),
                 "arrival_mean_prefix_blocks": float(La.mean()),
                 "arrival_hit_fraction": float(La.sum()) / max(1, n_blocks),

@@ -312,6 +312,34 @@ int kvgov_probe_arrival(const uint64_t *d_owner, uint64_t capacity, const uint32
                         uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * kvgov_chain_hash_arrival -- a batch's chain hash and its arrival-order
+ * serving in one call: the digests of kvgov_chain_hash, then the table,
+ * owners, slot handles, prefix lengths and key count of kvgov_insert_arrival
+ * followed by kvgov_probe_arrival, bit for bit.
+ *   mode .. d_digests  as for kvgov_chain_hash.
+ *   d_slots, d_owner, capacity, seq_base, d_slot_of, d_n_new  as for
+ *              kvgov_insert_arrival (d_slot_of [d_blk_off[n_req]]).
+ *   d_prefix_blocks  [n_req] int32 output, as for kvgov_probe_arrival.
+ *   d_status   required: KVGOV_F_BADINDEX as for kvgov_chain_hash, and the
+ *              insert flags.
+ * Batches that give every SM sub-partition at least two warps
+ * (n_req >= 2 x 32 x 4 x SMs) insert each digest from the chain kernel as
+ * soon as it is computed -- the lanes of a warp hold block j of 32
+ * consecutive requests, so a key their prefixes share is inserted once per
+ * warp -- then settle the owners and probe (three launches); smaller batches
+ * run the chain, the insert and the probe as separate launches.  Same
+ * results either way.  Must not overlap in time with other calls on the same
+ * table or owner array.  n_req = 0 is a no-op.  EINVAL: as for
+ * kvgov_chain_hash and kvgov_insert_arrival.
+ */
+int kvgov_chain_hash_arrival(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                             const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                             const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                             uint8_t *d_slots, uint64_t *d_owner, uint64_t capacity, uint64_t seq_base,
+                             uint32_t *d_slot_of, int32_t *d_prefix_blocks, unsigned long long *d_n_new,
+                             uint32_t *d_status, kvgov_stream_t stream);
+
+/*
  * kvgov_set_spin_limit -- bound on how many times an inserting thread
  * re-reads a slot whose key another thread is still writing before it gives
  * up with KVGOV_F_TIMEOUT (about 100 ns per re-read).

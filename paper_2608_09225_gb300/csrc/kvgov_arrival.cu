@@ -40,11 +40,10 @@ namespace {
 
 using namespace kvgov_dev;
 
-constexpr unsigned long long kPending = ~0ull;  // owner of a slot claimed by the running insert
+constexpr unsigned long long kPending = kOwnerPending;
 // Largest first position of a batch: positions stay below kPending for any
 // batch that fits in memory (2^62 blocks).
 constexpr unsigned long long kMaxSeq = 1ull << 62;
-constexpr uint32_t kNoSlot = 0xffffffffu;         // slot_of of a block whose key is not in the table
 constexpr int kThreads = 256;
 constexpr int G = 8;                         // lanes per request
 constexpr int kSegs = 32 / G;
@@ -133,6 +132,28 @@ __global__ void __launch_bounds__(kThreads) owner_min_kernel(const int64_t *__re
     }
 }
 
+// The same min with one thread per request walking its blocks, for batches
+// of many requests: the 32 lanes of a warp hold block j of 32 consecutive
+// requests, so one key shared by their prefixes is settled once per warp.
+__global__ void __launch_bounds__(kThreads) owner_min_req_kernel(const int64_t *__restrict__ blk_off, int32_t n_req,
+                                                                 const uint32_t *__restrict__ slot_of,
+                                                                 unsigned long long *__restrict__ owner,
+                                                                 unsigned long long seq_base) {
+    const long long r = (long long)blockIdx.x * kThreads + threadIdx.x;
+    const int lane = threadIdx.x & 31;
+    long long base, nb;
+    unsigned ignored = 0;                         // the insert has flagged bad ranges
+    request_range(blk_off, n_req, r, base, nb, ignored);
+    const int jmax = __reduce_max_sync(0xffffffffu, (unsigned)nb);
+    for (int j = 0; j < jmax; ++j) {                           // warp-uniform
+        const uint32_t s = j < nb ? __ldg(slot_of + base + j) : kNoSlot;
+        const unsigned same = __match_any_sync(0xffffffffu, s);
+        if (s == kNoSlot || lane != __ffs(same) - 1) continue;   // the lowest lane has the earliest position
+        const unsigned long long p = seq_base + (unsigned long long)(base + j);
+        if (ld_relaxed(owner + s) > p) atomicMin(owner + s, p);
+    }
+}
+
 __global__ void __launch_bounds__(kThreads) probe_arrival_kernel(const unsigned long long *__restrict__ owner,
                                                                  const uint32_t *__restrict__ slot_of,
                                                                  const int64_t *__restrict__ blk_off, int32_t n_req,
@@ -191,6 +212,24 @@ bool arrival_capacity(uint64_t capacity) {
 }
 
 }  // namespace
+
+namespace kvgov_host {
+
+// Owner min of a batch whose keys a fused chain kernel has inserted (one
+// thread per request; see owner_min_req_kernel).
+int arrival_owner_min_by_request(const int64_t *d_blk_off, int32_t n_req, const uint32_t *d_slot_of,
+                                 uint64_t *d_owner, uint64_t seq_base, cudaStream_t stream) {
+    const unsigned grid = (unsigned)(((long long)n_req + kThreads - 1) / kThreads);
+    owner_min_req_kernel<<<grid, kThreads, 0, stream>>>(d_blk_off, n_req, d_slot_of,
+                                                        reinterpret_cast<unsigned long long *>(d_owner), seq_base);
+    return launch_status();
+}
+
+bool arrival_args_ok(uint64_t capacity, uint64_t seq_base) {
+    return arrival_capacity(capacity) && seq_base != 0 && seq_base <= kMaxSeq;
+}
+
+}  // namespace kvgov_host
 
 extern "C" int kvgov_owner_init(uint64_t *d_owner, uint64_t capacity, kvgov_stream_t stream) {
     if (!d_owner || !kvgov_host::aligned16(d_owner) || !arrival_capacity(capacity)) return KVGOV_EINVAL;

@@ -15,6 +15,7 @@
 // then reads its 16 tokens from shared memory, byte-swaps them into
 // big-endian SHA words and runs the 2 (or 3) compressions of its message in
 // registers.
+#include "kvgov_insert.cuh"
 #include "kvgov_internal.cuh"
 #include "kvgov_lookup.cuh"
 #include "sha256_dev.cuh"
@@ -65,11 +66,26 @@ struct ChainParams {
     int32_t n_req;
     int32_t n_principals;
     uint32_t one;   // 1, opaque to the compiler (see AddFma)
-    // fused probe (kvgov_chain_hash_probe) only
+    // fused probe (kvgov_chain_hash_probe) and fused arrival insert
+    // (kvgov_chain_hash_arrival) only
     const uint4 *slots;
     unsigned long long mask;
     int32_t *prefix_blocks;
 };
+
+// The fused arrival insert's own arguments (a separate kernel parameter, so
+// that the other variants keep their parameter block).
+struct ArrivalParams {
+    unsigned long long *owner = nullptr;
+    uint32_t *slot_of = nullptr;
+    unsigned long long *n_new = nullptr;
+    uint32_t spin_limit = 0;
+};
+
+// What the chain kernel does with each digest besides storing it.
+constexpr int kFuseNone = 0;      // nothing (kvgov_chain_hash)
+constexpr int kFuseProbe = 1;     // look it up (kvgov_chain_hash_probe)
+constexpr int kFuseArrival = 2;   // insert it, arrival order (kvgov_chain_hash_arrival)
 
 // Which adder the SHA-256 rounds use.  Measured on GB300: IMAD shares the
 // integer pipe with SHF/LOP3/IADD3 (libkvgov_peak kinds 3-5), so AddFma
@@ -86,20 +102,26 @@ __device__ __forceinline__ void load_salt(const uint8_t *salts, int pi, uint32_t
     sw[4] = bswap32(b.x); sw[5] = bswap32(b.y); sw[6] = bswap32(b.z); sw[7] = bswap32(b.w);
 }
 
-// PROBE: after storing block j's digest, a thread whose blocks 0..j-1 were
-// all found in the table looks block j up too (kvgov_probe's definition),
-// and at the end writes its request's cached-prefix length.  The lookup's
-// memory latency is covered by the other warps' hashing.
-template <int MODE, bool PROBE>
-__global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
+// kFuseProbe: after storing block j's digest, a thread whose blocks 0..j-1
+// were all found in the table looks block j up too (kvgov_probe's
+// definition), and at the end writes its request's cached-prefix length.
+// kFuseArrival: block j's key goes into the table at once (the insert of
+// kvgov_insert_arrival): the lanes of a warp hold block j of 32 consecutive
+// requests, so a key their prefixes share is inserted by its lowest lane
+// only and the others take its slot.  Either way the memory latency is
+// covered by the other warps' hashing.
+template <int MODE, int FUSE>
+__device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalParams &a) {
     __shared__ __align__(16) uint32_t stage[kStages][kR * kSlotWords];
     __shared__ long long s_tok[kR];
     __shared__ int s_nb[kR];
     __shared__ int s_jmax;
+    __shared__ unsigned int s_new, s_flags, s_done;   // kFuseArrival counts
 
     const int tid = threadIdx.x;
     const long long r = (long long)blockIdx.x * kR + tid;
     if (tid == 0) s_jmax = 0;
+    if (FUSE == kFuseArrival && tid == 0) { s_new = 0; s_flags = 0; s_done = 0; }
 
     // Per-request set-up and validation.
     const long long tok_end = p.tok_off[p.n_req];
@@ -164,8 +186,11 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
     uint32_t h[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) h[i] = 0u;
-    int hits = 0;   // PROBE: leading blocks found in the table so far
+    int hits = 0;   // kFuseProbe: leading blocks found in the table so far
+    unsigned my_new = 0, my_flags = 0;   // kFuseArrival
 
+    unsigned long long ak[4] = {0ull, 0ull, 0ull, 0ull};   // kFuseArrival: block j's key
+    bool have = false;                                      // ... to be inserted by this lane
     for (int j = 0; j < jmax; ++j) {
         const int jn = j + kStages - 1;
         if (jn < jmax) issue(jn, jn % kStages);
@@ -213,22 +238,93 @@ __global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
             const uint4 q1 = make_uint4(bswap32(h[4]), bswap32(h[5]), bswap32(h[6]), bswap32(h[7]));
             dst[0] = q0;
             dst[1] = q1;
-            if (PROBE && hits == j && lookup<false>(p.slots, p.mask, q0, q1)) hits = j + 1;
+            if (FUSE == kFuseProbe && hits == j && lookup<false>(p.slots, p.mask, q0, q1)) hits = j + 1;
+            if (FUSE == kFuseArrival) {
+                ak[0] = u64_of(q0.x, q0.y); ak[1] = u64_of(q0.z, q0.w);
+                ak[2] = u64_of(q1.x, q1.y); ak[3] = u64_of(q1.z, q1.w);
+                have = !key_reserved(ak);
+                if (!have) {
+                    my_flags |= KVGOV_F_SENTINEL;
+                    a.slot_of[row + j] = kNoSlot;
+                }
+            }
+        }
+        if (FUSE == kFuseArrival) {                     // every lane of the warp is here
+            const unsigned inserting = __ballot_sync(0xffffffffu, have);
+            if (have) {
+                const unsigned same = __match_any_sync(inserting, ak[0]) & __match_any_sync(inserting, ak[1]) &
+                                      __match_any_sync(inserting, ak[2]) & __match_any_sync(inserting, ak[3]);
+                const int leader = __ffs(same) - 1;
+                unsigned long long pos = 0ull;
+                int res = kDuplicate;
+                if ((tid & 31) == leader) {
+                    res = insert_one(reinterpret_cast<unsigned long long *>(const_cast<uint4 *>(p.slots)), p.mask,
+                                     ak, a.spin_limit, &pos);
+                    count_insert(static_cast<InsertResult>(res), my_new, my_flags);
+                    if (res == kNew) a.owner[pos] = kOwnerPending;
+                }
+                pos = __shfl_sync(inserting, pos, leader);
+                res = __shfl_sync(inserting, res, leader);
+                a.slot_of[row + j] = (res == kNew || res == kDuplicate) ? (uint32_t)pos : kNoSlot;
+            }
+            have = false;
         }
         __syncthreads();
     }
     cp_async_wait<0>();
-    if (PROBE && r < p.n_req) p.prefix_blocks[r] = hits;
+    if (FUSE == kFuseProbe && r < p.n_req) p.prefix_blocks[r] = hits;
+    if (FUSE == kFuseArrival) publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, a.n_new, p.status);
+}
+
+template <int MODE, int FUSE>
+__global__ void __launch_bounds__(kR) chain_kernel(const ChainParams p) {
+    chain_body<MODE, FUSE>(p, ArrivalParams{});
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kR) chain_arrival_kernel(const ChainParams p, const ArrivalParams a) {
+    chain_body<MODE, kFuseArrival>(p, a);
 }
 
 }  // namespace
 
 namespace {
 
+// Launch chain_kernel<mode, FUSE> (chain_arrival_kernel<mode> for kFuseArrival).
+template <int FUSE>
+void launch_chain_kernel(int mode, unsigned grid, cudaStream_t s, const ChainParams &p,
+                         const ArrivalParams &a = ArrivalParams{}) {
+    if constexpr (FUSE == kFuseArrival) {
+        switch (mode) {
+        case KVGOV_UNSALTED: chain_arrival_kernel<KVGOV_UNSALTED><<<grid, kR, 0, s>>>(p, a); break;
+        case KVGOV_ROOT: chain_arrival_kernel<KVGOV_ROOT><<<grid, kR, 0, s>>>(p, a); break;
+        default: chain_arrival_kernel<KVGOV_BOUNDARY><<<grid, kR, 0, s>>>(p, a); break;
+        }
+    } else {
+        switch (mode) {
+        case KVGOV_UNSALTED: chain_kernel<KVGOV_UNSALTED, FUSE><<<grid, kR, 0, s>>>(p); break;
+        case KVGOV_ROOT: chain_kernel<KVGOV_ROOT, FUSE><<<grid, kR, 0, s>>>(p); break;
+        default: chain_kernel<KVGOV_BOUNDARY, FUSE><<<grid, kR, 0, s>>>(p); break;
+        }
+    }
+}
+
+// The table and arrival arguments of the fused variants.
+struct FuseArgs {
+    int fuse = kFuseNone;
+    const uint8_t *slots = nullptr;
+    uint64_t capacity = 0;
+    int32_t *prefix_blocks = nullptr;   // kFuseProbe
+    uint64_t *owner = nullptr;          // kFuseArrival
+    uint64_t seq_base = 0;
+    uint32_t *slot_of = nullptr;
+    unsigned long long *n_new = nullptr;
+};
+
 int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
                  const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
                  const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests, uint32_t *d_status,
-                 const uint8_t *d_slots, uint64_t capacity, int32_t *d_prefix_blocks, kvgov_stream_t stream) {
+                 const FuseArgs &f, kvgov_stream_t stream) {
     using kvgov_host::aligned16;
     if (mode != KVGOV_UNSALTED && mode != KVGOV_ROOT && mode != KVGOV_BOUNDARY) return KVGOV_EINVAL;
     if (n_req < 0) return KVGOV_EINVAL;
@@ -237,50 +333,58 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     if (mode != KVGOV_UNSALTED && (!d_principal || !d_salts || !aligned16(d_salts) || n_principals <= 0))
         return KVGOV_EINVAL;
     if (mode == KVGOV_BOUNDARY && !d_boundary_tok) return KVGOV_EINVAL;
-    const bool probe = d_prefix_blocks != nullptr;
-    if (probe && (!d_slots || !aligned16(d_slots) || !kvgov_host::pow2_capacity(capacity))) return KVGOV_EINVAL;
+    if (f.fuse == kFuseProbe &&
+        (!f.prefix_blocks || !f.slots || !aligned16(f.slots) || !kvgov_host::pow2_capacity(f.capacity)))
+        return KVGOV_EINVAL;
+    if (f.fuse == kFuseArrival &&
+        (!f.prefix_blocks || !f.slots || !aligned16(f.slots) || !f.owner || !f.slot_of || !d_status ||
+         !kvgov_host::arrival_args_ok(f.capacity, f.seq_base)))
+        return KVGOV_EINVAL;
     if (n_req == 0) return KVGOV_OK;
 
     ChainParams p;
     p.tokens = d_tokens; p.tok_off = d_tok_off; p.principal = d_principal; p.salts = d_salts;
     p.boundary_tok = d_boundary_tok; p.blk_off = d_blk_off; p.digests = d_digests; p.status = d_status;
     p.n_req = n_req; p.n_principals = n_principals; p.one = 1u;
-    p.slots = reinterpret_cast<const uint4 *>(d_slots);
-    p.mask = probe ? capacity - 1 : 0;
-    p.prefix_blocks = d_prefix_blocks;
+    p.slots = reinterpret_cast<const uint4 *>(f.slots);
+    p.mask = f.fuse != kFuseNone ? f.capacity - 1 : 0;
+    p.prefix_blocks = f.prefix_blocks;
+    ArrivalParams a;
+    a.owner = reinterpret_cast<unsigned long long *>(f.owner);
+    a.slot_of = f.slot_of;
+    a.n_new = f.n_new;
+    a.spin_limit = kvgov_host::spin_limit();
     const unsigned grid = (unsigned)(((long long)n_req + kR - 1) / kR);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     // A batch too small to give every SM sub-partition two warps leaves each
-    // warp alone on its scheduler, where a fused lookup would stall the chain;
-    // there the lookups run as a second launch (same results).
+    // warp alone on its scheduler, where a fused lookup or insert would stall
+    // the chain; there they run as separate launches (same results).
     const DeviceInfo dev = device_info();
     const long long min_fused = 2ll * 32 * 4 * (dev.sms > 0 ? dev.sms : 152);
-    if (probe && n_req < min_fused) {
-        p.mask = 0;
-        p.prefix_blocks = nullptr;
-        switch (mode) {
-        case KVGOV_UNSALTED: chain_kernel<KVGOV_UNSALTED, false><<<grid, kR, 0, s>>>(p); break;
-        case KVGOV_ROOT: chain_kernel<KVGOV_ROOT, false><<<grid, kR, 0, s>>>(p); break;
-        default: chain_kernel<KVGOV_BOUNDARY, false><<<grid, kR, 0, s>>>(p); break;
-        }
-        const int rc = kvgov_host::launch_status();
+    const bool fused = f.fuse != kFuseNone && n_req >= min_fused;
+    if (!fused) {
+        launch_chain_kernel<kFuseNone>(mode, grid, s, p);
+        int rc = kvgov_host::launch_status();
+        if (rc != KVGOV_OK || f.fuse == kFuseNone) return rc;
+        if (f.fuse == kFuseProbe)
+            return kvgov_probe(f.slots, f.capacity, d_digests, d_blk_off, n_req, f.prefix_blocks, d_status, stream);
+        rc = kvgov_insert_arrival(const_cast<uint8_t *>(f.slots), f.owner, f.capacity, d_digests, d_blk_off, n_req,
+                                  f.seq_base, f.slot_of, f.n_new, d_status, stream);
         if (rc != KVGOV_OK) return rc;
-        return kvgov_probe(d_slots, capacity, d_digests, d_blk_off, n_req, d_prefix_blocks, d_status, stream);
+        return kvgov_probe_arrival(f.owner, f.capacity, f.slot_of, d_blk_off, n_req, f.seq_base, f.prefix_blocks,
+                                   d_status, stream);
     }
-    if (probe) {
-        switch (mode) {
-        case KVGOV_UNSALTED: chain_kernel<KVGOV_UNSALTED, true><<<grid, kR, 0, s>>>(p); break;
-        case KVGOV_ROOT: chain_kernel<KVGOV_ROOT, true><<<grid, kR, 0, s>>>(p); break;
-        default: chain_kernel<KVGOV_BOUNDARY, true><<<grid, kR, 0, s>>>(p); break;
-        }
-    } else {
-        switch (mode) {
-        case KVGOV_UNSALTED: chain_kernel<KVGOV_UNSALTED, false><<<grid, kR, 0, s>>>(p); break;
-        case KVGOV_ROOT: chain_kernel<KVGOV_ROOT, false><<<grid, kR, 0, s>>>(p); break;
-        default: chain_kernel<KVGOV_BOUNDARY, false><<<grid, kR, 0, s>>>(p); break;
-        }
+    if (f.fuse == kFuseProbe) {
+        launch_chain_kernel<kFuseProbe>(mode, grid, s, p);
+        return kvgov_host::launch_status();
     }
-    return kvgov_host::launch_status();
+    launch_chain_kernel<kFuseArrival>(mode, grid, s, p, a);
+    int rc = kvgov_host::launch_status();
+    if (rc != KVGOV_OK) return rc;
+    rc = kvgov_host::arrival_owner_min_by_request(d_blk_off, n_req, f.slot_of, f.owner, f.seq_base, s);
+    if (rc != KVGOV_OK) return rc;
+    return kvgov_probe_arrival(f.owner, f.capacity, f.slot_of, d_blk_off, n_req, f.seq_base, f.prefix_blocks,
+                               d_status, stream);
 }
 
 }  // namespace
@@ -290,7 +394,7 @@ extern "C" int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t
                                 const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
                                 uint32_t *d_status, kvgov_stream_t stream) {
     return launch_chain(mode, d_tokens, d_tok_off, n_req, d_principal, d_salts, n_principals, d_boundary_tok,
-                        d_blk_off, d_digests, d_status, nullptr, 0, nullptr, stream);
+                        d_blk_off, d_digests, d_status, FuseArgs{}, stream);
 }
 
 extern "C" int kvgov_chain_hash_probe(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
@@ -298,7 +402,30 @@ extern "C" int kvgov_chain_hash_probe(int mode, const int32_t *d_tokens, const i
                                       const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
                                       const uint8_t *d_slots, uint64_t capacity, int32_t *d_prefix_blocks,
                                       uint32_t *d_status, kvgov_stream_t stream) {
-    if (!d_prefix_blocks) return KVGOV_EINVAL;
+    FuseArgs f;
+    f.fuse = kFuseProbe;
+    f.slots = d_slots;
+    f.capacity = capacity;
+    f.prefix_blocks = d_prefix_blocks;
     return launch_chain(mode, d_tokens, d_tok_off, n_req, d_principal, d_salts, n_principals, d_boundary_tok,
-                        d_blk_off, d_digests, d_status, d_slots, capacity, d_prefix_blocks, stream);
+                        d_blk_off, d_digests, d_status, f, stream);
+}
+
+extern "C" int kvgov_chain_hash_arrival(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                                        const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                                        const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                                        uint8_t *d_slots, uint64_t *d_owner, uint64_t capacity, uint64_t seq_base,
+                                        uint32_t *d_slot_of, int32_t *d_prefix_blocks, unsigned long long *d_n_new,
+                                        uint32_t *d_status, kvgov_stream_t stream) {
+    FuseArgs f;
+    f.fuse = kFuseArrival;
+    f.slots = d_slots;
+    f.capacity = capacity;
+    f.prefix_blocks = d_prefix_blocks;
+    f.owner = d_owner;
+    f.seq_base = seq_base;
+    f.slot_of = d_slot_of;
+    f.n_new = d_n_new;
+    return launch_chain(mode, d_tokens, d_tok_off, n_req, d_principal, d_salts, n_principals, d_boundary_tok,
+                        d_blk_off, d_digests, d_status, f, stream);
 }

@@ -32,6 +32,11 @@ inline bool pow2_capacity(uint64_t cap) { return cap >= KVGOV_MIN_CAPACITY && (c
 // The bound on every wait of the insert protocol (kvgov_set_spin_limit).
 uint32_t spin_limit();
 
+// Arrival-order serving helpers (kvgov_arrival.cu).
+int arrival_owner_min_by_request(const int64_t *d_blk_off, int32_t n_req, const uint32_t *d_slot_of,
+                                 uint64_t *d_owner, uint64_t seq_base, cudaStream_t stream);
+bool arrival_args_ok(uint64_t capacity, uint64_t seq_base);
+
 inline int launch_status() {
     return cudaGetLastError() == cudaSuccess ? KVGOV_OK : KVGOV_ECUDA;
 }

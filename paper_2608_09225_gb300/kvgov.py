@@ -63,11 +63,13 @@ def _load():
         L.kvgov_insert_arrival.argtypes = [_p, _p, ctypes.c_uint64, _p, _p, ctypes.c_int32, ctypes.c_uint64, _p, _p,
                                            _p, _p]
         L.kvgov_probe_arrival.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, ctypes.c_uint64, _p, _p, _p]
+        L.kvgov_chain_hash_arrival.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p,
+                                               _p, _p, _p, ctypes.c_uint64, ctypes.c_uint64, _p, _p, _p, _p, _p]
         L.kvgov_set_spin_limit.argtypes = [ctypes.c_uint32]
         L.kvgov_set_spin_limit.restype = ctypes.c_uint32
         for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
                    "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
-                   "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival"):
+                   "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival"):
             getattr(L, fn).restype = ctypes.c_int
         _lib = L
         return L
@@ -306,6 +308,45 @@ def probe_arrival(owner: torch.Tensor, slot_of: torch.Tensor, blk_off: torch.Ten
                                      _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_probe_arrival")
     return prefix_blocks
+
+
+def chain_hash_arrival(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, blk_off: torch.Tensor,
+                       slots: torch.Tensor, owner: torch.Tensor, seq_base: int, status: torch.Tensor,
+                       principal: torch.Tensor | None = None, salts: torch.Tensor | None = None,
+                       boundary_tok: torch.Tensor | None = None, digests: torch.Tensor | None = None,
+                       slot_of: torch.Tensor | None = None, prefix_blocks: torch.Tensor | None = None,
+                       n_blocks: int | None = None, n_new: torch.Tensor | None = None, stream=None):
+    """chain_hash, insert_arrival and probe_arrival in one call (the insert
+    fused into the chain kernel for large batches); returns (digests,
+    slot_of, prefix_blocks)."""
+    L = lib()
+    n = tok_off.numel() - 1
+    if digests is None:
+        if n_blocks is None:
+            n_blocks = int(blk_off[-1].item())
+        digests = torch.empty((n_blocks, 32), dtype=torch.uint8, device=tokens.device)
+    if slot_of is None:
+        slot_of = torch.empty(digests.shape[0], dtype=torch.int32, device=tokens.device)
+    if prefix_blocks is None:
+        prefix_blocks = torch.empty(n, dtype=torch.int32, device=tok_off.device)
+    if tokens.numel() == 0:
+        tokens = torch.zeros(4, dtype=torch.int32, device=tok_off.device)
+    n_p = 0 if salts is None else salts.shape[0]
+    _check(L.kvgov_chain_hash_arrival(int(mode), _dev(tokens, torch.int32, "tokens"),
+                                      _dev(tok_off, torch.int64, "tok_off"), n,
+                                      _dev(principal, torch.int32, "principal", True),
+                                      _dev(salts, torch.uint8, "salts", True), n_p,
+                                      _dev(boundary_tok, torch.int32, "boundary_tok", True),
+                                      _dev(blk_off, torch.int64, "blk_off"),
+                                      _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(tokens),
+                                      _dev(slots, torch.uint8, "slots"), _dev(owner, torch.int64, "owner"),
+                                      slots.shape[0], int(seq_base),
+                                      _dev(slot_of, torch.int32, "slot_of") if slot_of.numel() else _dummy(tokens),
+                                      _dev(prefix_blocks, torch.int32, "prefix_blocks") if n else _dummy(tokens),
+                                      _dev(n_new, torch.int64, "n_new", True), _dev(status, torch.int32, "status"),
+                                      _stream(stream)),
+           "kvgov_chain_hash_arrival")
+    return digests, slot_of, prefix_blocks
 
 
 def set_spin_limit(limit: int) -> int:

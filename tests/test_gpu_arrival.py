@@ -213,3 +213,101 @@ def test_arrival_wide_full(kv):
     _, L, n_keys = oracle_arrival(w, W.BOUNDARY)
     assert (pre == L).all() and int(cache.n_new.item()) == n_keys
     assert pre[0] == 0 and (pre[1:] >= 4).all()         # the shared 64-token prefix is unsalted
+
+
+# ------------------------------------------------- chain hash + arrival in one call
+def shared_prefix_batch(seed, n_req):
+    """Requests that start with one of four 200-token prompts (cut at a
+    random length, then their own tokens), a tenth of them an exact repeat
+    of an earlier request by the same principal; principals 0..7; boundary
+    offsets cycling as in workloads.ragged."""
+    rng = np.random.default_rng(seed)
+    prompts = rng.integers(0, W.VOCAB, (4, 200), dtype=np.int32)
+    reqs, principal = [], []
+    for r in range(n_req):
+        if reqs and rng.random() < 0.1:
+            src = int(rng.integers(0, len(reqs)))
+            reqs.append(reqs[src].copy())
+            principal.append(principal[src])
+            continue
+        cut = int(rng.integers(0, 200))
+        own = rng.integers(0, W.VOCAB, int(rng.integers(0, 120)), dtype=np.int32)
+        reqs.append(np.concatenate([prompts[int(rng.integers(0, 4))][:cut], own]).astype(np.int32))
+        principal.append(int(rng.integers(0, 8)))
+    tok_off = np.concatenate([[0], np.cumsum([len(t) for t in reqs])]).astype(np.int64)
+    cyc = np.array([0, 15, 16, 17, 31, 32, 64, 10 ** 6], dtype=np.int32)
+    return W.Batch(tokens=np.concatenate(reqs).astype(np.int32), tok_off=tok_off,
+                   principal=np.array(principal, np.int32), boundary_tok=cyc[np.arange(n_req) % len(cyc)])
+
+
+@pytest.mark.parametrize("mode", [W.UNSALTED, W.ROOT, W.BOUNDARY])
+@pytest.mark.parametrize("n_req", [180, 40960], ids=["separate_launches", "fused"])
+def test_chain_hash_arrival_matches_oracle_and_separate_calls(kv, mode, n_req):
+    """kvgov_chain_hash_arrival gives the oracle's digests and arrival-order
+    prefix lengths, and the table, key count and prefix lengths of the
+    separate calls, for a batch small enough for separate launches and one
+    that takes the fused kernel; keys cached before the batch count."""
+    b = shared_prefix_batch(500 + n_req + mode, n_req)
+    salts = oracle.derive_salts(b"arrival", *W.principal_ids(8))
+    ref = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+    blk_ref = oracle.block_offsets(b.tok_off)
+    early = ref[np.random.default_rng(mode).random(len(ref)) < 0.05]     # cached before the batch
+    ks = oracle.KeySet(1)
+    ks.insert(early)
+    want, n_batch = ks.arrival_prefix(ref, blk_ref)
+    cap = next_pow2(4 * len(ref))
+    toks, tok_off = dev(b.tokens, np.int32), dev(b.tok_off, np.int64)
+    pr, sl, bt = dev(b.principal, np.int32), dev(salts), dev(b.boundary_tok, np.int32)
+    outs = []
+    for fused_call in (True, False):
+        a = Arrival(kv, cap)
+        kv.insert(a.slots, dev(early), a.status, a.n_new)
+        blk = kv.block_offsets(tok_off, status=a.status)
+        if fused_call:
+            d, slot_of, pre = kv.chain_hash_arrival(mode, toks, tok_off, blk, a.slots, a.owner, 7, a.status, pr, sl, bt,
+                                                    n_blocks=len(ref), n_new=a.n_new)
+        else:
+            d = kv.chain_hash(mode, toks, tok_off, blk, pr, sl, bt, n_blocks=len(ref), status=a.status)
+            slot_of = kv.insert_arrival(a.slots, a.owner, d, blk, 7, a.status, n_new=a.n_new)
+            pre = kv.probe_arrival(a.owner, slot_of, blk, 7, status=a.status)
+        torch.cuda.synchronize()
+        assert int(a.status.item()) == 0
+        assert (d.cpu().numpy() == ref).all()
+        so = slot_of.cpu().numpy()
+        assert (a.slots.cpu().numpy()[so] == ref).all()
+        assert (pre.cpu().numpy() == want).all()
+        assert int(a.n_new.item()) == ks.n + n_batch
+        outs.append(table_contents(a.slots))
+    assert outs[0] == outs[1]
+    assert want.max() > 0 and (want == 0).any()
+
+
+@pytest.mark.parametrize("name", ["wide", "probe", "template"])
+def test_chain_hash_arrival_full_workloads(kv, name):
+    """The one-call path at full size: the wide batch (131,072 requests, the
+    fused kernel, 4 shared-prefix keys inserted by every request), the
+    probe-heavy batch into its table of 8.1 M keys (fused), and the 8192
+    template requests (separate launches)."""
+    w = W.make(name, seed=43) if name == "wide" else W.make(name)
+    mode = W.BOUNDARY if name != "probe" else W.ROOT
+    fill = name == "probe"
+    b = w.batch
+    n_blocks = int((b.lengths() // 16).sum())
+    cap = w.capacity if fill else next_pow2(4 * n_blocks)
+    cache = PrefixCache(cap, w.secret, w.ids, w.id_off)
+    db = DeviceBatch.from_host(b.tokens, b.tok_off, b.principal, b.boundary_tok)
+    owner = kv.new_owner(cap)
+    if fill:
+        cache.insert(torch.from_numpy(w.random_keys).cuda())
+    blk = kv.block_offsets(db.tok_off, status=cache.status)
+    d, slot_of, pre = kv.chain_hash_arrival(mode, db.tokens, db.tok_off, blk, cache.slots, owner, 1 << 40,
+                                            cache.status, db.principal, cache.salts, db.boundary_tok,
+                                            n_blocks=n_blocks, n_new=cache.n_new)
+    torch.cuda.synchronize()
+    cache.check_status()
+    dref, L, n_keys = oracle_arrival(w, mode, fill)
+    assert (d.cpu().numpy() == dref).all()
+    assert (pre.cpu().numpy() == L).all()
+    assert int(cache.n_new.item()) == n_keys
+    so = slot_of.cpu().numpy()
+    assert (so >= 0).all() and (cache.slots.cpu().numpy()[so] == dref).all()

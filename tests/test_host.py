@@ -34,7 +34,8 @@ def test_header_declares_the_boundary():
     names = declared_functions()
     for want in ("kvgov_derive_salts", "kvgov_block_offsets", "kvgov_chain_hash", "kvgov_table_init",
                  "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
-                 "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_status_string",
+                 "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
+                 "kvgov_status_string",
                  "kvgov_set_spin_limit"):
         assert want in names
 
@@ -151,6 +152,17 @@ def test_host_validation_rejects_bad_arguments(libkv):
     assert ia(fake, fake, 64, fake, fake, 3, 1, None, None, fake, None) == 1            # no slot_of
     assert ia(fake, fake, 64, odd, fake, 3, 1, fake, None, fake, None) == 1             # misaligned digests
     assert ia(fake, fake, 64, None, None, 0, 1, None, None, fake, None) == 0            # empty batch
+    ca = libkv.kvgov_chain_hash_arrival
+    ca.argtypes = [ctypes.c_int, p, p, ctypes.c_int32, p, p, ctypes.c_int32, p, p, p, p, p, ctypes.c_uint64,
+                   ctypes.c_uint64, p, p, p, p, p]
+    assert ca(0, fake, fake, 4, None, None, 0, None, fake, fake, fake, fake, 64, 1, fake, fake, None, None,
+              None) == 1                                                                 # status is required
+    assert ca(0, fake, fake, 4, None, None, 0, None, fake, fake, fake, None, 64, 1, fake, fake, None, fake,
+              None) == 1                                                                 # no owner array
+    assert ca(0, fake, fake, 4, None, None, 0, None, fake, fake, fake, fake, 64, 0, fake, fake, None, fake,
+              None) == 1                                                                 # position 0
+    assert ca(0, fake, fake, 0, None, None, 0, None, fake, fake, fake, fake, 64, 1, fake, fake, None, fake,
+              None) == 0                                                                 # empty batch
     pa = libkv.kvgov_probe_arrival
     pa.argtypes = [p, ctypes.c_uint64, p, p, ctypes.c_int32, ctypes.c_uint64, p, p, p]
     assert pa(fake, 64, fake, fake, 3, 0, fake, None, None) == 1
