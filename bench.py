@@ -45,7 +45,8 @@ SM_MAX_MHZ = 2070.0            # maximum SM clock of a GB300 (profiling recipe)
 INT32_LANES_PER_SM = 64        # 4 SMSPs x 16 lanes of the integer pipe (LOP3/SHF/IMAD microbench: 64.0/clk/SM)
 CHAIN_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_chain.cu", "paper_2608_09225_gb300/csrc/sha256_dev.cuh",
                  "paper_2608_09225_gb300/csrc/kvgov_internal.cuh", "paper_2608_09225_gb300/csrc/kvgov_lookup.cuh",
-                 "include/kvgov.h"]
+                 "paper_2608_09225_gb300/csrc/kvgov_insert.cuh"]
+CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain kernel's code
 CHAIN_PROFILE = "profiles/chain_kernel_wide.md"
 
 
@@ -63,11 +64,15 @@ PEAKS = load_peaks()
 
 
 def chain_source_hash() -> str:
+    """SHA-256 over the chain kernel's translation unit: its sources, and the
+    constants (#define lines) of the public header it includes."""
     import hashlib
     h = hashlib.sha256()
     for rel in CHAIN_SOURCES:
         with open(os.path.join(HERE, rel), "rb") as f:
             h.update(f.read())
+    with open(os.path.join(HERE, CHAIN_HEADER), "rb") as f:
+        h.update(b"".join(line for line in f.read().splitlines(keepends=True) if line.lstrip().startswith(b"#define")))
     return h.hexdigest()
 
 
@@ -776,6 +781,18 @@ def run_configs(args):
         t_probe = _time(torch, lambda: K.probe(cache.slots, dig, pblk_view, pre[: p1 - p0]))
         t_fused = _time(torch, lambda: K.chain_hash_probe(mode, db.tokens, db.tok_off, blk, cache.slots, pr, sl, bt,
                                                           dig, pre))
+        # divergence boundaries against the workload's registered shared preamble
+        n_pre = {"tiny": 128, "sysprompt": 1024, "template": 96, "long": 64, "wide": 64}.get(name, 0)
+        t0 = int(b.tok_off[0])
+        pre_tok = db.tokens[t0:t0 + n_pre].contiguous() if n_pre else db.tokens[:4].contiguous()
+        pre_off = torch.tensor([0, n_pre], dtype=torch.int64, device="cuda")
+        tid = torch.full((b.n,), 0 if n_pre else K.TEMPLATE_NONE, dtype=torch.int32, device="cuda")
+        bnd = torch.empty(b.n, dtype=torch.int32, device="cuda")
+        t_bnd = _time(torch, lambda: K.divergence_boundary(db.tokens, db.tok_off, tid, pre_tok, pre_off, bnd,
+                                                           cache.status))
+        bnd_np = bnd.cpu().numpy()
+        bnd_bytes = 4 * int(np.minimum(bnd_np + 1, b.lengths()).sum()) if n_pre else 0
+
         # arrival order: the whole batch served request by request into an empty cache
         acap = next_pow2(4 * n_blocks)
         aslots, owner = K.new_table(acap), K.new_owner(acap)
@@ -830,6 +847,9 @@ def run_configs(args):
                 "probe_gbs": probe_bytes / (t_probe / 1e3) / 1e9,
                 "probe_frac_hbm": probe_bytes / (t_probe / 1e3) / 1e9 / PEAKS["hbm_gbs"],
                 "probe_frac_random_read": probe_bytes / (t_probe / 1e3) / 1e9 / gather["gbs_32B"],
+                "boundary_preamble_tokens": n_pre, "boundary_ms": t_bnd,
+                "boundary_mean_tokens": float(bnd_np.mean()) if b.n else 0.0,
+                "boundary_gbs": bnd_bytes / (t_bnd / 1e3) / 1e9,
                 "arrival_insert_ms": t_arr_ins - t_ainit, "arrival_probe_ms": t_arr - t_arr_ins,
                 "chain_arrival_ms": t_arr_fused - t_ainit,
                 "chain_arrival_blocks_per_s": n_blocks / ((t_arr_fused - t_ainit) / 1e3),

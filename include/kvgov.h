@@ -46,6 +46,8 @@ typedef struct CUstream_st *kvgov_stream_t;
 #define KVGOV_MIN_CAPACITY 32      /* smallest table capacity (slots)         */
 #define KVGOV_PROBE_WINDOW 1024    /* a key lives within this many slots of its
                                       home slot (fewer if the table is smaller) */
+#define KVGOV_TEMPLATE_NONE (-1)   /* kvgov_divergence_boundary: no preamble   */
+#define KVGOV_TEMPLATE_ANY (-2)    /* ... the longest match over all preambles */
 
 /* Return codes (host-detected). */
 #define KVGOV_OK 0
@@ -93,6 +95,34 @@ const char *kvgov_status_string(int status);
  */
 int kvgov_block_offsets(const int64_t *d_tok_off, int32_t n_req, int64_t *d_blk_off,
                         uint32_t *d_status, kvgov_stream_t stream);
+
+/*
+ * kvgov_divergence_boundary -- where each request's salt goes in, paper
+ * section 4.2 (salt at the divergence boundary k: the blocks before it hold
+ * the shared preamble, which tells no principal apart) and section 5.7 (a
+ * divergence at token i invalidates every block from floor(i/B) on).
+ * d_boundary_tok[r] = the length of the longest common prefix of request r's
+ * tokens and its registered preamble: the index of the first token where
+ * they differ, or the shorter length if one is a prefix of the other.  It is
+ * the d_boundary_tok input of kvgov_chain_hash in BOUNDARY mode (k = b / 16).
+ *   d_tokens, d_tok_off, n_req  the batch (CSR int32 tokens, int64 offsets).
+ *   d_template_id  [n_req] int32: the preamble of request r, an index into
+ *               the registered preambles, KVGOV_TEMPLATE_NONE (b = 0: salt at
+ *               the root) or KVGOV_TEMPLATE_ANY (the longest match over all
+ *               preambles).
+ *   d_tpl_tokens, d_tpl_off, n_tpl  the registered preambles (CSR int32
+ *               tokens, int64 offsets [n_tpl + 1]); may be NULL if n_tpl = 0.
+ *   d_boundary_tok [n_req] int32 output.
+ *   d_status    nullable; KVGOV_F_BADINDEX for an id outside
+ *               [KVGOV_TEMPLATE_ANY, n_tpl) or malformed offsets (that
+ *               request gets b = 0).
+ * One warp per request.  n_req = 0 is a no-op.  EINVAL: negative counts,
+ * NULL arrays.
+ */
+int kvgov_divergence_boundary(const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                              const int32_t *d_template_id, const int32_t *d_tpl_tokens,
+                              const int64_t *d_tpl_off, int32_t n_tpl, int32_t *d_boundary_tok,
+                              uint32_t *d_status, kvgov_stream_t stream);
 
 /*
  * kvgov_derive_salts -- per-principal salt, paper section 4.1:

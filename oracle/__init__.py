@@ -64,6 +64,8 @@ def _configure(L):
     L.oracle_prefix_blocks.restype = ctypes.c_int
     L.oracle_arrival_prefix.argtypes = [_p, _i64, _p, _p, _i32, _p, _p]
     L.oracle_arrival_prefix.restype = ctypes.c_int
+    L.oracle_divergence_boundary.argtypes = [_p, _p, _i32, _p, _p, _p, _i32, _p]
+    L.oracle_divergence_boundary.restype = ctypes.c_int
     return L
 
 
@@ -177,6 +179,27 @@ def chain_hash(mode: int, tokens: np.ndarray, tok_off: np.ndarray,
     if rc != 0:
         raise ValueError("oracle_chain_hash: invalid argument")
     return out
+
+
+def divergence_boundary(tokens: np.ndarray, tok_off: np.ndarray, template_id: np.ndarray,
+                        tpl_tokens: np.ndarray, tpl_off: np.ndarray):
+    """Boundary token offset per request: the longest common prefix with its
+    registered preamble (ids: index, -1 none, -2 best of all).  Returns
+    (boundary_tok int32 [n], flag) -- flag set if an id was out of range."""
+    tokens = _c(tokens, np.int32)
+    if tokens.size == 0:
+        tokens = np.zeros(1, np.int32)
+    tok_off = _c(tok_off, np.int64)
+    template_id = _c(template_id, np.int32)
+    tpl_tokens = _c(tpl_tokens, np.int32)
+    if tpl_tokens.size == 0:
+        tpl_tokens = np.zeros(1, np.int32)
+    tpl_off = _c(tpl_off, np.int64)
+    n = len(tok_off) - 1
+    out = np.zeros(max(n, 1), np.int32)
+    flag = lib().oracle_divergence_boundary(_ptr(tokens), _ptr(tok_off), n, _ptr(template_id), _ptr(tpl_tokens),
+                                            _ptr(tpl_off), len(tpl_off) - 1, _ptr(out))
+    return out[:n], bool(flag)
 
 
 def key_reserved(key: bytes) -> bool:

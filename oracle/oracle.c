@@ -26,6 +26,8 @@
  *   arrival-order ...... the same lookup applied request by request, each
  *   serving              request then caching its blocks (sections 2.1 and
  *                        4.2): a sequential replay over a chained hash set.
+ *   divergence ......... section 4.2 / 5.7: a request's boundary token is its
+ *   boundary             longest common prefix with its registered preamble.
  *
  * Byte conventions (readings where the paper is silent): a token is its
  * int32 value serialised as 4 little-endian bytes; a block is B = 16 tokens
@@ -492,4 +494,42 @@ int oracle_arrival_prefix(const uint8_t *set_keys, int64_t n_set, const uint8_t 
     *n_new = s.n - before;
     free(s.head); free(s.next); free(s.key);
     return 0;
+}
+
+/* --------------------------------------------------------------------- */
+/*
+ * Divergence boundary (paper section 4.2: the salt goes in at the block
+ * where a request diverges from the shared preamble; section 5.7: a
+ * divergence at token i invalidates blocks floor(i/B) onward).  For request
+ * r, boundary_tok[r] is the number of leading tokens it has in common with
+ * its registered preamble: compare token by token from position 0 and stop
+ * at the first difference or at the end of the shorter sequence.
+ * template_id[r] names the preamble (an index below n_tpl), -1 (none:
+ * boundary 0) or -2 (the longest such prefix over all preambles).  An id out
+ * of range gives boundary 0.  Returns 1 if some id or offset was out of
+ * range, else 0.
+ */
+int oracle_divergence_boundary(const int32_t *tokens, const int64_t *tok_off, int32_t n_req,
+                               const int32_t *template_id, const int32_t *tpl_tokens,
+                               const int64_t *tpl_off, int32_t n_tpl, int32_t *boundary_tok)
+{
+    int flag = 0;
+    for (int32_t r = 0; r < n_req; r++) {
+        const int32_t id = template_id[r];
+        const int64_t len_r = tok_off[r + 1] - tok_off[r];
+        boundary_tok[r] = 0;
+        if (id < -2 || id >= n_tpl || len_r < 0) { flag = 1; continue; }
+        if (id == -1) continue;
+        int64_t best = 0;
+        for (int32_t t = 0; t < n_tpl; t++) {
+            if (id >= 0 && t != id) continue;
+            const int64_t len_t = tpl_off[t + 1] - tpl_off[t];
+            int64_t i = 0;
+            while (i < len_r && i < len_t && tokens[tok_off[r] + i] == tpl_tokens[tpl_off[t] + i])
+                i++;
+            if (i > best) best = i;
+        }
+        boundary_tok[r] = (int32_t)best;
+    }
+    return flag;
 }

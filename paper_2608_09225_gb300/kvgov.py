@@ -22,6 +22,7 @@ MIN_CAPACITY = 32
 
 OK, EINVAL, ECUDA = 0, 1, 2
 F_BADINDEX, F_SENTINEL, F_TABLE_FULL, F_TIMEOUT = 0x10, 0x20, 0x40, 0x80
+TEMPLATE_NONE, TEMPLATE_ANY = -1, -2
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libkvgov.so")
@@ -65,11 +66,13 @@ def _load():
         L.kvgov_probe_arrival.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, ctypes.c_uint64, _p, _p, _p]
         L.kvgov_chain_hash_arrival.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p,
                                                _p, _p, _p, ctypes.c_uint64, ctypes.c_uint64, _p, _p, _p, _p, _p]
+        L.kvgov_divergence_boundary.argtypes = [_p, _p, ctypes.c_int32, _p, _p, _p, ctypes.c_int32, _p, _p, _p]
         L.kvgov_set_spin_limit.argtypes = [ctypes.c_uint32]
         L.kvgov_set_spin_limit.restype = ctypes.c_uint32
         for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
                    "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
-                   "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival"):
+                   "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
+                   "kvgov_divergence_boundary"):
             getattr(L, fn).restype = ctypes.c_int
         _lib = L
         return L
@@ -347,6 +350,31 @@ def chain_hash_arrival(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, b
                                       _stream(stream)),
            "kvgov_chain_hash_arrival")
     return digests, slot_of, prefix_blocks
+
+
+def divergence_boundary(tokens: torch.Tensor, tok_off: torch.Tensor, template_id: torch.Tensor,
+                        tpl_tokens: torch.Tensor | None = None, tpl_off: torch.Tensor | None = None,
+                        boundary_tok: torch.Tensor | None = None, status: torch.Tensor | None = None,
+                        stream=None) -> torch.Tensor:
+    """Boundary token offset of each request: its longest common prefix with
+    its registered preamble (paper sections 4.2 and 5.7); template_id[r] is a
+    preamble index, TEMPLATE_NONE or TEMPLATE_ANY."""
+    n = tok_off.numel() - 1
+    n_tpl = 0 if tpl_off is None else tpl_off.numel() - 1
+    if boundary_tok is None:
+        boundary_tok = torch.empty(max(n, 0), dtype=torch.int32, device=tok_off.device)
+    if tokens.numel() == 0:
+        tokens = torch.zeros(4, dtype=torch.int32, device=tok_off.device)
+    if tpl_tokens is not None and tpl_tokens.numel() == 0:
+        tpl_tokens = torch.zeros(4, dtype=torch.int32, device=tok_off.device)
+    _check(lib().kvgov_divergence_boundary(_dev(tokens, torch.int32, "tokens"), _dev(tok_off, torch.int64, "tok_off"), n,
+                                           _dev(template_id, torch.int32, "template_id") if n else _dummy(tokens),
+                                           _dev(tpl_tokens, torch.int32, "tpl_tokens", True),
+                                           _dev(tpl_off, torch.int64, "tpl_off", True), n_tpl,
+                                           _dev(boundary_tok, torch.int32, "boundary_tok") if n else _dummy(tokens),
+                                           _dev(status, torch.int32, "status", True), _stream(stream)),
+           "kvgov_divergence_boundary")
+    return boundary_tok
 
 
 def set_spin_limit(limit: int) -> int:

@@ -486,4 +486,83 @@ def pin_arrival_tiny_closed_form():
     assert n_new == 64 * 16 - 24 * 8
 
 
+# ------------------------------------------------------ divergence boundary
+def _lcp_python(a, b):
+    n = 0
+    for x, y in zip(a, b):
+        if int(x) != int(y):
+            break
+        n += 1
+    return n
+
+
+def pin_boundary_brute_force():
+    """Boundary detection == a Python zip comparison: the longest common
+    prefix with the named preamble, the longest over all preambles for id -2,
+    0 for id -1 and for ids out of range (flagged)."""
+    rng = np.random.default_rng(22)
+    for trial in range(30):
+        tpls = [rng.integers(0, 5, int(rng.integers(0, 40)), dtype=np.int32) for _ in range(int(rng.integers(0, 4)))]
+        reqs, ids = [], []
+        for r in range(int(rng.integers(1, 30))):
+            base = tpls[int(rng.integers(0, len(tpls)))] if tpls and rng.random() < 0.8 else np.zeros(0, np.int32)
+            cut = int(rng.integers(0, len(base) + 1))
+            tail = rng.integers(0, 5, int(rng.integers(0, 10)), dtype=np.int32)
+            reqs.append(np.concatenate([base[:cut], tail]).astype(np.int32))
+            ids.append(int(rng.integers(-3, len(tpls) + 1)))
+        tok_off = np.concatenate([[0], np.cumsum([len(x) for x in reqs])]).astype(np.int64)
+        tpl_off = np.concatenate([[0], np.cumsum([len(x) for x in tpls])]).astype(np.int64)
+        toks = np.concatenate(reqs + [np.zeros(0, np.int32)]).astype(np.int32)
+        tt = np.concatenate(tpls + [np.zeros(0, np.int32)]).astype(np.int32)
+        got, flag = oracle.divergence_boundary(toks, tok_off, np.array(ids, np.int32), tt, tpl_off)
+        want, bad = [], False
+        for req, i in zip(reqs, ids):
+            if i < -2 or i >= len(tpls):
+                want.append(0)
+                bad = True
+            elif i == -1:
+                want.append(0)
+            elif i == -2:
+                want.append(max([_lcp_python(req, t) for t in tpls], default=0))
+            else:
+                want.append(_lcp_python(req, tpls[i]))
+        assert list(got) == want and flag == bad, trial
+
+
+def pin_boundary_paper_layout():
+    """Section 5.7 again, through boundary detection: a 2119-token request
+    whose preamble is registered and which diverges at token 1990 gets its
+    boundary at block 124; diverging at token 5, at block 0.  Salting there
+    (section 4.2) leaves another principal exactly those leading blocks."""
+    ex = _paper()["divergence_layout"]
+    n = ex["prompt_tokens"]
+    rng = np.random.default_rng(23)
+    pre = rng.integers(0, W.VOCAB, n, dtype=np.int32)
+    salts = oracle.derive_salts(b"z" * 32, *W.principal_ids(2))
+    for i, want in zip(ex["diverge_at_token"], ex["hit_blocks"]):
+        req = pre.copy()
+        req[i] = (req[i] + 1) % W.VOCAB
+        b, _ = oracle.divergence_boundary(req, np.array([0, n], np.int64), np.array([0], np.int32), pre,
+                                          np.array([0, n], np.int64))
+        assert int(b[0]) == i and int(b[0]) // 16 == want
+        assert _prefix(BOUNDARY, req, 0, req, 1, salts, b=int(b[0])) == want
+
+
+def pin_boundary_workload_preambles():
+    """Registering the template's first 96 tokens (up to its first field) gives
+    every template request boundary 96, and the wide batch's shared 64-token
+    prefix gives 64: the boundaries those workloads are built with."""
+    w = W.template(n_req=512)
+    b = w.batch
+    first = b.tokens[int(b.tok_off[0]):int(b.tok_off[0]) + 96]
+    got, flag = oracle.divergence_boundary(b.tokens, b.tok_off, np.zeros(b.n, np.int32), first,
+                                           np.array([0, 96], np.int64))
+    assert not flag and (got == 96).all() and (got == b.boundary_tok).all()
+    w = W.wide(seed=5, n_req=300)
+    b = w.batch
+    got, _ = oracle.divergence_boundary(b.tokens, b.tok_off, np.full(b.n, -2, np.int32), b.tokens[:64],
+                                        np.array([0, 64], np.int64))
+    assert (got == 64).all() and (got == b.boundary_tok).all()
+
+
 PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

@@ -35,7 +35,7 @@ def test_header_declares_the_boundary():
     for want in ("kvgov_derive_salts", "kvgov_block_offsets", "kvgov_chain_hash", "kvgov_table_init",
                  "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
                  "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
-                 "kvgov_status_string",
+                 "kvgov_divergence_boundary", "kvgov_status_string",
                  "kvgov_set_spin_limit"):
         assert want in names
 
@@ -163,6 +163,12 @@ def test_host_validation_rejects_bad_arguments(libkv):
               None) == 1                                                                 # position 0
     assert ca(0, fake, fake, 0, None, None, 0, None, fake, fake, fake, fake, 64, 1, fake, fake, None, fake,
               None) == 0                                                                 # empty batch
+    db = libkv.kvgov_divergence_boundary
+    db.argtypes = [p, p, ctypes.c_int32, p, p, p, ctypes.c_int32, p, p, p]
+    assert db(fake, fake, -1, fake, None, None, 0, fake, None, None) == 1                # negative n_req
+    assert db(fake, fake, 3, None, None, None, 0, fake, None, None) == 1                 # no template ids
+    assert db(fake, fake, 3, fake, None, None, 2, fake, None, None) == 1                 # preambles missing
+    assert db(None, fake, 0, None, None, None, 0, None, None, None) == 0                 # empty batch
     pa = libkv.kvgov_probe_arrival
     pa.argtypes = [p, ctypes.c_uint64, p, p, ctypes.c_int32, ctypes.c_uint64, p, p, p]
     assert pa(fake, 64, fake, fake, 3, 0, fake, None, None) == 1

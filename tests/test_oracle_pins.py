@@ -73,6 +73,12 @@ MUTATIONS = [
     ("arrival_counts_all_hits",
      "        while (j < nb && chain_set_contains(&s, req + 32 * (size_t)j))\n            j++;",
      "        for (int64_t q = 0; q < nb; q++) j += chain_set_contains(&s, req + 32 * (size_t)q);"),
+    ("boundary_off_by_one",
+     "while (i < len_r && i < len_t && tokens[tok_off[r] + i] == tpl_tokens[tpl_off[t] + i])\n                i++;",
+     "while (i < len_r && i < len_t && tokens[tok_off[r] + i] == tpl_tokens[tpl_off[t] + i])\n                i++;\n"
+     "            if (i < len_r && i < len_t) i++;"),
+    ("boundary_any_takes_first", "if (i > best) best = i;", "if (best == 0) best = i;"),
+    ("boundary_none_compares", "        if (id == -1) continue;\n", ""),
     ("arrival_reserved_keys_stored",
      "            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);",
      "            chain_set_add(&s, req + 32 * (size_t)q);"),
