@@ -793,6 +793,13 @@ def run_configs(args):
         bnd_np = bnd.cpu().numpy()
         bnd_bytes = 4 * int(np.minimum(bnd_np + 1, b.lengths()).sum()) if n_pre else 0
 
+        # exact-response keys of the whole prompts (salted when the workload is)
+        rmode = W.UNSALTED if mode == W.UNSALTED else W.ROOT
+        rkeys = torch.empty((b.n, 32), dtype=torch.uint8, device="cuda")
+        t_resp = _time(torch, lambda: K.response_key(rmode, db.tokens, db.tok_off, db.principal, cache.salts, rkeys,
+                                                     cache.status))
+        resp_comp = int((((8 if rmode == W.ROOT else 0) + b.lengths() + 3 + 15) // 16).sum())
+
         # arrival order: the whole batch served request by request into an empty cache
         acap = next_pow2(4 * n_blocks)
         aslots, owner = K.new_table(acap), K.new_owner(acap)
@@ -847,6 +854,10 @@ def run_configs(args):
                 "probe_gbs": probe_bytes / (t_probe / 1e3) / 1e9,
                 "probe_frac_hbm": probe_bytes / (t_probe / 1e3) / 1e9 / PEAKS["hbm_gbs"],
                 "probe_frac_random_read": probe_bytes / (t_probe / 1e3) / 1e9 / gather["gbs_32B"],
+                "response_key_ms": t_resp, "response_keys_per_s": b.n / (t_resp / 1e3),
+                "response_tokens_per_s": float(b.lengths().sum()) / (t_resp / 1e3),
+                "response_compressions": resp_comp,
+                "response_frac_int32_peak": resp_comp * 1384 / (t_resp / 1e3) / peak,
                 "boundary_preamble_tokens": n_pre, "boundary_ms": t_bnd,
                 "boundary_mean_tokens": float(bnd_np.mean()) if b.n else 0.0,
                 "boundary_gbs": bnd_bytes / (t_bnd / 1e3) / 1e9,

@@ -125,6 +125,28 @@ int kvgov_divergence_boundary(const int32_t *d_tokens, const int64_t *d_tok_off,
                               uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * kvgov_response_key -- exact-response cache keys, paper Table 1 (an
+ * exact-response cache keys on byte equality of the whole prompt) and
+ * section 4.1 (sigma_p is prepended to that key):
+ *   ROOT      key_r = SHA-256(sigma_p || bytes(tokens of r))
+ *   UNSALTED  key_r = SHA-256(bytes(tokens of r))
+ * with every token of the request (no block truncation), tokens as int32
+ * little-endian.  The keys go into the same table as block digests
+ * (kvgov_insert; kvgov_probe with one "block" per request gives 1 for a
+ * cached response, 0 otherwise).
+ *   d_tokens, d_tok_off, n_req  the batch (CSR; tokens 16-byte aligned).
+ *   d_principal, d_salts, n_principals  as for kvgov_chain_hash (ROOT only).
+ *   d_keys     [n_req][32] u8 output (16-byte aligned).
+ *   d_status   nullable; KVGOV_F_BADINDEX for a malformed range or principal
+ *              (that request's key is undefined).
+ * One thread per request.  n_req = 0 is a no-op.  EINVAL: mode BOUNDARY or
+ * unknown, NULL or misaligned arrays, ROOT without salts.
+ */
+int kvgov_response_key(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                       const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals, uint8_t *d_keys,
+                       uint32_t *d_status, kvgov_stream_t stream);
+
+/*
  * kvgov_derive_salts -- per-principal salt, paper section 4.1:
  * sigma_p = HMAC_K(secret, principal_id), HMAC per RFC 2104 with SHA-256.
  *

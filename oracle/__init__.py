@@ -66,6 +66,8 @@ def _configure(L):
     L.oracle_arrival_prefix.restype = ctypes.c_int
     L.oracle_divergence_boundary.argtypes = [_p, _p, _i32, _p, _p, _p, _i32, _p]
     L.oracle_divergence_boundary.restype = ctypes.c_int
+    L.oracle_response_key.argtypes = [ctypes.c_int, _p, _p, _i32, _p, _p, _i32, _p]
+    L.oracle_response_key.restype = ctypes.c_int
     return L
 
 
@@ -200,6 +202,25 @@ def divergence_boundary(tokens: np.ndarray, tok_off: np.ndarray, template_id: np
     flag = lib().oracle_divergence_boundary(_ptr(tokens), _ptr(tok_off), n, _ptr(template_id), _ptr(tpl_tokens),
                                             _ptr(tpl_off), len(tpl_off) - 1, _ptr(out))
     return out[:n], bool(flag)
+
+
+def response_key(mode: int, tokens: np.ndarray, tok_off: np.ndarray, principal: np.ndarray,
+                 salts: np.ndarray) -> np.ndarray:
+    """Exact-response cache keys [n, 32]: SHA-256(sigma_p || prompt bytes) for
+    ROOT, SHA-256(prompt bytes) for UNSALTED (paper Table 1, section 4.1)."""
+    tokens = _c(tokens, np.int32)
+    if tokens.size == 0:
+        tokens = np.zeros(1, np.int32)
+    tok_off = _c(tok_off, np.int64)
+    principal = _c(principal, np.int32)
+    salts = _c(salts, np.uint8).reshape(-1, 32)
+    n = len(tok_off) - 1
+    out = np.zeros((max(n, 1), 32), np.uint8)
+    rc = lib().oracle_response_key(int(mode), _ptr(tokens), _ptr(tok_off), n, _ptr(principal), _ptr(salts),
+                                   salts.shape[0], _ptr(out))
+    if rc != 0:
+        raise ValueError("oracle_response_key: bad mode, range or principal")
+    return out[:n]
 
 
 def key_reserved(key: bytes) -> bool:

@@ -28,6 +28,7 @@
  *                        4.2): a sequential replay over a chained hash set.
  *   divergence ......... section 4.2 / 5.7: a request's boundary token is its
  *   boundary             longest common prefix with its registered preamble.
+ *   exact-response key . Table 1 / section 4.1: SHA-256(sigma_p || prompt).
  *
  * Byte conventions (readings where the paper is silent): a token is its
  * int32 value serialised as 4 little-endian bytes; a block is B = 16 tokens
@@ -532,4 +533,41 @@ int oracle_divergence_boundary(const int32_t *tokens, const int64_t *tok_off, in
         boundary_tok[r] = (int32_t)best;
     }
     return flag;
+}
+
+/* --------------------------------------------------------------------- */
+/*
+ * Exact-response cache key (paper Table 1: the key is the whole prompt;
+ * section 4.1: sigma_p is prepended to it): SHA-256 over the byte string
+ * sigma_p || LE32(t_0) || LE32(t_1) || ... with every token of the request,
+ * or over the token bytes alone in mode UNSALTED.  The message is built in
+ * full and hashed with oracle_sha256.  Returns -1 for a bad mode, range or
+ * principal, or no memory; 0 otherwise.
+ */
+int oracle_response_key(int mode, const int32_t *tokens, const int64_t *tok_off, int32_t n_req,
+                        const int32_t *principal, const uint8_t *salts, int32_t n_principals,
+                        uint8_t *keys)
+{
+    if (mode != ORACLE_UNSALTED && mode != ORACLE_ROOT) return -1;
+    for (int32_t r = 0; r < n_req; r++) {
+        const int64_t len = tok_off[r + 1] - tok_off[r];
+        if (len < 0) return -1;
+        const size_t salt_len = mode == ORACLE_ROOT ? 32 : 0;
+        uint8_t *msg = malloc(salt_len + 4 * (size_t)len + 1);
+        if (!msg) return -1;
+        if (mode == ORACLE_ROOT) {
+            if (principal[r] < 0 || principal[r] >= n_principals) { free(msg); return -1; }
+            memcpy(msg, salts + 32 * (size_t)principal[r], 32);
+        }
+        for (int64_t i = 0; i < len; i++) {
+            const uint32_t v = (uint32_t)tokens[tok_off[r] + i];
+            msg[salt_len + 4 * i] = (uint8_t)v;
+            msg[salt_len + 4 * i + 1] = (uint8_t)(v >> 8);
+            msg[salt_len + 4 * i + 2] = (uint8_t)(v >> 16);
+            msg[salt_len + 4 * i + 3] = (uint8_t)(v >> 24);
+        }
+        oracle_sha256(msg, salt_len + 4 * (size_t)len, keys + 32 * (size_t)r);
+        free(msg);
+    }
+    return 0;
 }

@@ -67,12 +67,13 @@ def _load():
         L.kvgov_chain_hash_arrival.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p,
                                                _p, _p, _p, ctypes.c_uint64, ctypes.c_uint64, _p, _p, _p, _p, _p]
         L.kvgov_divergence_boundary.argtypes = [_p, _p, ctypes.c_int32, _p, _p, _p, ctypes.c_int32, _p, _p, _p]
+        L.kvgov_response_key.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p, _p]
         L.kvgov_set_spin_limit.argtypes = [ctypes.c_uint32]
         L.kvgov_set_spin_limit.restype = ctypes.c_uint32
         for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
                    "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
                    "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
-                   "kvgov_divergence_boundary"):
+                   "kvgov_divergence_boundary", "kvgov_response_key"):
             getattr(L, fn).restype = ctypes.c_int
         _lib = L
         return L
@@ -375,6 +376,26 @@ def divergence_boundary(tokens: torch.Tensor, tok_off: torch.Tensor, template_id
                                            _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_divergence_boundary")
     return boundary_tok
+
+
+def response_key(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, principal: torch.Tensor | None = None,
+                 salts: torch.Tensor | None = None, keys: torch.Tensor | None = None,
+                 status: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Exact-response cache key per request: SHA-256(sigma_p || prompt bytes)
+    (ROOT) or SHA-256(prompt bytes) (UNSALTED); returns [n, 32] u8."""
+    n = tok_off.numel() - 1
+    if keys is None:
+        keys = torch.empty((max(n, 0), 32), dtype=torch.uint8, device=tok_off.device)
+    if tokens.numel() == 0:
+        tokens = torch.zeros(4, dtype=torch.int32, device=tok_off.device)
+    n_p = 0 if salts is None else salts.shape[0]
+    _check(lib().kvgov_response_key(int(mode), _dev(tokens, torch.int32, "tokens"), _dev(tok_off, torch.int64, "tok_off"),
+                                    n, _dev(principal, torch.int32, "principal", True),
+                                    _dev(salts, torch.uint8, "salts", True), n_p,
+                                    _dev(keys, torch.uint8, "keys") if n else _dummy(tokens),
+                                    _dev(status, torch.int32, "status", True), _stream(stream)),
+           "kvgov_response_key")
+    return keys
 
 
 def set_spin_limit(limit: int) -> int:

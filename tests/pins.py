@@ -565,4 +565,42 @@ def pin_boundary_workload_preambles():
     assert (got == 64).all() and (got == b.boundary_tok).all()
 
 
+# ------------------------------------------------------ exact-response key
+def pin_response_key_hashlib():
+    """Exact-response keys == hashlib over sigma_p || struct-packed tokens
+    (and over the tokens alone unsalted), for prompts of every length 0..70
+    tokens (all padding edges of a 32-byte salt plus 4-byte tokens) and a
+    2119-token prompt."""
+    salts = oracle.derive_salts(b"resp", *W.principal_ids(3))
+    rng = np.random.default_rng(24)
+    lens = list(range(71)) + [2119]
+    reqs = [rng.integers(0, W.VOCAB, n, dtype=np.int32) for n in lens]
+    tok_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    toks = np.concatenate(reqs).astype(np.int32)
+    pr = (np.arange(len(lens)) % 3).astype(np.int32)
+    root = oracle.response_key(ROOT, toks, tok_off, pr, salts)
+    plain = oracle.response_key(UNSALTED, toks, tok_off, pr, salts)
+    for r, t in enumerate(reqs):
+        assert root[r].tobytes() == H(salts[pr[r]].tobytes() + block_le(t)), r
+        assert plain[r].tobytes() == H(block_le(t)), r
+
+
+def pin_response_key_whole_prompt():
+    """The exact-response key covers every token (a change in a 7-token tail
+    changes it, while the block chain ignores the tail), and it separates
+    principals on identical prompts (section 4.1)."""
+    salts = oracle.derive_salts(b"resp2", *W.principal_ids(2))
+    rng = np.random.default_rng(25)
+    a = rng.integers(0, W.VOCAB, 2119, dtype=np.int32)
+    b = a.copy()
+    b[-1] = (b[-1] + 1) % W.VOCAB
+    toks = np.concatenate([a, b, a]).astype(np.int32)
+    off = np.array([0, 2119, 4238, 6357], np.int64)
+    pr = np.array([0, 0, 1], np.int32)
+    k = oracle.response_key(ROOT, toks, off, pr, salts)
+    assert k[0].tobytes() != k[1].tobytes() and k[0].tobytes() != k[2].tobytes()
+    d = oracle.chain_hash(UNSALTED, toks[:4238], off[:3], pr[:2], salts, np.zeros(2, np.int32))
+    assert (d[:132] == d[132:]).all()                  # the blocks never see the tail
+
+
 PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

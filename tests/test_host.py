@@ -35,7 +35,7 @@ def test_header_declares_the_boundary():
     for want in ("kvgov_derive_salts", "kvgov_block_offsets", "kvgov_chain_hash", "kvgov_table_init",
                  "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
                  "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
-                 "kvgov_divergence_boundary", "kvgov_status_string",
+                 "kvgov_divergence_boundary", "kvgov_response_key", "kvgov_status_string",
                  "kvgov_set_spin_limit"):
         assert want in names
 
@@ -169,6 +169,12 @@ def test_host_validation_rejects_bad_arguments(libkv):
     assert db(fake, fake, 3, None, None, None, 0, fake, None, None) == 1                 # no template ids
     assert db(fake, fake, 3, fake, None, None, 2, fake, None, None) == 1                 # preambles missing
     assert db(None, fake, 0, None, None, None, 0, None, None, None) == 0                 # empty batch
+    rk = libkv.kvgov_response_key
+    rk.argtypes = [ctypes.c_int, p, p, ctypes.c_int32, p, p, ctypes.c_int32, p, p, p]
+    assert rk(2, fake, fake, 3, fake, fake, 1, fake, None, None) == 1                    # BOUNDARY has no meaning
+    assert rk(1, fake, fake, 3, None, fake, 1, fake, None, None) == 1                    # ROOT without principals
+    assert rk(0, odd, fake, 3, None, None, 0, fake, None, None) == 1                     # misaligned tokens
+    assert rk(0, fake, fake, 0, None, None, 0, None, None, None) == 0                    # empty batch
     pa = libkv.kvgov_probe_arrival
     pa.argtypes = [p, ctypes.c_uint64, p, p, ctypes.c_int32, ctypes.c_uint64, p, p, p]
     assert pa(fake, 64, fake, fake, 3, 0, fake, None, None) == 1

@@ -79,6 +79,11 @@ MUTATIONS = [
      "            if (i < len_r && i < len_t) i++;"),
     ("boundary_any_takes_first", "if (i > best) best = i;", "if (best == 0) best = i;"),
     ("boundary_none_compares", "        if (id == -1) continue;\n", ""),
+    ("response_salt_after_prompt", "oracle_sha256(msg, salt_len + 4 * (size_t)len, keys + 32 * (size_t)r);",
+     "oracle_sha256(msg + salt_len, 4 * (size_t)len, keys + 32 * (size_t)r);"),
+    ("response_token_bytes_swapped",
+     "msg[salt_len + 4 * i] = (uint8_t)v;\n            msg[salt_len + 4 * i + 1] = (uint8_t)(v >> 8);",
+     "msg[salt_len + 4 * i + 1] = (uint8_t)v;\n            msg[salt_len + 4 * i] = (uint8_t)(v >> 8);"),
     ("arrival_reserved_keys_stored",
      "            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);",
      "            chain_set_add(&s, req + 32 * (size_t)q);"),
