@@ -875,7 +875,36 @@ def run_configs(args):
         print(json.dumps(line), flush=True)
         del cache, keys, dig
         torch.cuda.empty_cache()
+    print(json.dumps(audit_rates(torch, K, W, seed, cores, args.no_cpu_baseline)), flush=True)
     return 0
+
+
+def audit_rates(torch, K, W, seed, cores, no_cpu):
+    """ORIGAMI allocation (kvgov_origami) on 2^20 problems of the section 5.5
+    setting: 50 tenants with Pareto(1.29) values, K = 10."""
+    import oracle
+    b = W.audit(seed=seed, n_prob=1 << 20)
+    v = torch.from_numpy(b.values).cuda()
+    off = torch.from_numpy(b.off).cuda()
+    bud = torch.from_numpy(b.budget).cuda()
+    p = torch.empty_like(v)
+    lam = torch.empty(b.n, dtype=torch.float32, device="cuda")
+    util = torch.empty(b.n, dtype=torch.float32, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    t = _time(torch, lambda: K.origami(v, off, bud, p, lam, util, st))
+    n_val = int(b.off[-1])
+    bytes_ = 8 * n_val + 8 * (b.n + 1) + 12 * b.n         # values in, p out; offsets, budget, lambda, utility
+    line = {"workload": "audit", "problems": b.n, "tenants_per_problem": 50, "budget": 10.0,
+            "values": "Pareto(1.29), x_m = 1", "origami_ms": t, "problems_per_s": b.n / (t / 1e3),
+            "gbs": bytes_ / (t / 1e3) / 1e9, "frac_hbm": bytes_ / (t / 1e3) / 1e9 / PEAKS["hbm_gbs"],
+            "mean_lambda": float(lam.mean().item()), "status": int(st.item())}
+    if not no_cpu:
+        sample = W.audit(seed=seed, n_prob=1 << 16)
+        t0 = time.perf_counter()
+        oracle.origami(sample.values, sample.off, sample.budget)
+        dt = time.perf_counter() - t0
+        line["oracle_problems_per_s_1_thread"] = sample.n / dt
+    return line
 
 
 if __name__ == "__main__":

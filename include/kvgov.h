@@ -147,6 +147,30 @@ int kvgov_response_key(int mode, const int32_t *d_tokens, const int64_t *d_tok_o
                        uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * kvgov_origami -- ORIGAMI audit allocation for a batch of problems, paper
+ * section 4.3, Theorem (ORIGAMI water-filling solution): for each problem,
+ * tenants with values at risk v_i and an audit budget K, the audit
+ * probabilities minimising the adversary's best payoff max_i v_i (1 - p_i)
+ * subject to sum p_i = K, p_i in [0, 1]:
+ *     p_i = max(0, 1 - lambda / v_i),  lambda the unique level with sum = K.
+ *   d_values   float32, the problems' tenant values back to back (CSR).
+ *   d_off      [n_prob + 1] int64 offsets into d_values.
+ *   d_budget   [n_prob] float32 K.  K is capped at the number of usable
+ *              tenants (all audited, lambda = 0); K = 0 gives p = 0 and
+ *              lambda = the largest value.
+ *   d_p        float32 output beside d_values.
+ *   d_lambda   [n_prob] float32 output (nullable): the water level.
+ *   d_utility  [n_prob] float32 output (nullable): the adversary's best
+ *              payoff max_i v_i (1 - p_i) under the allocation.
+ *   d_status   nullable; KVGOV_F_BADINDEX for a NaN or infinite value, a
+ *              negative or NaN budget (read as 0) or malformed offsets.
+ * Tenants with v_i <= 0 get p_i = 0.  fp32 arithmetic, one warp per problem.
+ * n_prob = 0 is a no-op.  EINVAL: negative n_prob, NULL arrays.
+ */
+int kvgov_origami(const float *d_values, const int64_t *d_off, int32_t n_prob, const float *d_budget, float *d_p,
+                  float *d_lambda, float *d_utility, uint32_t *d_status, kvgov_stream_t stream);
+
+/*
  * kvgov_derive_salts -- per-principal salt, paper section 4.1:
  * sigma_p = HMAC_K(secret, principal_id), HMAC per RFC 2104 with SHA-256.
  *

@@ -68,6 +68,8 @@ def _configure(L):
     L.oracle_divergence_boundary.restype = ctypes.c_int
     L.oracle_response_key.argtypes = [ctypes.c_int, _p, _p, _i32, _p, _p, _i32, _p]
     L.oracle_response_key.restype = ctypes.c_int
+    L.oracle_origami.argtypes = [_p, _p, _i32, _p, _p, _p, _p]
+    L.oracle_origami.restype = ctypes.c_int
     return L
 
 
@@ -221,6 +223,24 @@ def response_key(mode: int, tokens: np.ndarray, tok_off: np.ndarray, principal: 
     if rc != 0:
         raise ValueError("oracle_response_key: bad mode, range or principal")
     return out[:n]
+
+
+def origami(values: np.ndarray, off: np.ndarray, budget: np.ndarray):
+    """ORIGAMI audit probabilities (paper section 4.3): float32 values in CSR
+    by off, float32 budgets.  Returns (p fp64, lambda fp64, utility fp64, flag)."""
+    values = _c(values, np.float32)
+    if values.size == 0:
+        values = np.zeros(1, np.float32)
+    off = _c(off, np.int64)
+    budget = _c(budget, np.float32)
+    n = len(off) - 1
+    p = np.zeros(max(values.size, 1), np.float64)
+    lam = np.zeros(max(n, 1), np.float64)
+    u = np.zeros(max(n, 1), np.float64)
+    rc = lib().oracle_origami(_ptr(values), _ptr(off), n, _ptr(budget), _ptr(p), _ptr(lam), _ptr(u))
+    if rc < 0:
+        raise MemoryError("oracle_origami")
+    return p[: int(off[-1])], lam[:n], u[:n], bool(rc)
 
 
 def key_reserved(key: bytes) -> bool:

@@ -29,6 +29,9 @@
  *   divergence ......... section 4.2 / 5.7: a request's boundary token is its
  *   boundary             longest common prefix with its registered preamble.
  *   exact-response key . Table 1 / section 4.1: SHA-256(sigma_p || prompt).
+ *   ORIGAMI ............ section 4.3, Theorem: the water-filling audit
+ *                        allocation, from its closed form over the sorted
+ *                        values (fp64).
  *
  * Byte conventions (readings where the paper is silent): a token is its
  * int32 value serialised as 4 little-endian bytes; a block is B = 16 tokens
@@ -53,6 +56,7 @@
 #include <stddef.h>
 #include <stdint.h>
 #include <stdlib.h>
+#include <math.h>
 #include <string.h>
 
 /* --------------------------------------------------------------------- */
@@ -570,4 +574,73 @@ int oracle_response_key(int mode, const int32_t *tokens, const int64_t *tok_off,
         free(msg);
     }
     return 0;
+}
+
+/* --------------------------------------------------------------------- */
+/*
+ * ORIGAMI audit allocation (paper section 4.3, Theorem): minimise
+ * max_i v_i (1 - p_i) subject to sum_i p_i = K and p_i in [0, 1]; the
+ * optimum is p_i = max(0, 1 - lambda / v_i) with the water level lambda that
+ * meets the budget.  Written out from that statement, in fp64: take the
+ * tenants with positive value in decreasing order of value; if the top m of
+ * them are the audited ones, sum_{i <= m} (1 - lambda / v_(i)) = K gives
+ * lambda_m = (m - K) / sum_{i <= m} 1 / v_(i); the water level is the
+ * lambda_m that lies in [v_(m+1), v_(m)) (v_(n+1) = 0), i.e. exactly the top
+ * m tenants are above it.  K is capped at the number of positive values
+ * (all audited, lambda = 0); K = 0 gives lambda = the largest value.  Values
+ * <= 0 get p = 0.  utility[q] = max_i v_i (1 - p_i).  Returns 1 if some
+ * value was not a finite number or some budget was negative (read as 0),
+ * -1 for no memory, 0 otherwise.
+ */
+static int cmp_desc(const void *a, const void *b)
+{
+    const double x = *(const double *)a, y = *(const double *)b;
+    return (x < y) - (x > y);
+}
+
+int oracle_origami(const float *values, const int64_t *off, int32_t n_prob, const float *budget,
+                   double *p, double *lambda, double *utility)
+{
+    int flag = 0;
+    for (int32_t q = 0; q < n_prob; q++) {
+        const int64_t b0 = off[q], n = off[q + 1] - off[q];
+        double *pos = malloc((size_t)(n > 0 ? n : 1) * sizeof(double));
+        if (!pos) return -1;
+        int64_t npos = 0;
+        for (int64_t i = 0; i < n; i++) {
+            const double x = values[b0 + i];
+            if (x > 0.0 && x <= 3.0e38) pos[npos++] = x;
+            else if (!(x <= 0.0)) flag = 1;
+        }
+        qsort(pos, (size_t)npos, sizeof(double), cmp_desc);
+        double K = budget[q];
+        if (!(K >= 0.0)) { flag = 1; K = 0.0; }
+        if (K > (double)npos) K = (double)npos;
+        double lam;
+        if (npos == 0 || K <= 0.0) {
+            lam = npos > 0 ? pos[0] : 0.0;
+        } else if (K >= (double)npos) {
+            lam = 0.0;
+        } else {
+            double inv_sum = 0.0;
+            lam = 0.0;
+            for (int64_t m = 1; m <= npos; m++) {
+                inv_sum += 1.0 / pos[m - 1];
+                const double lm = ((double)m - K) / inv_sum;
+                const double below = m < npos ? pos[m] : 0.0;
+                if (lm >= below && lm < pos[m - 1]) { lam = lm; break; }
+            }
+        }
+        double u = -HUGE_VAL;
+        for (int64_t i = 0; i < n; i++) {
+            const double x = values[b0 + i];
+            const double pi = (x > 0.0 && x <= 3.0e38) ? (1.0 - lam / x > 0.0 ? 1.0 - lam / x : 0.0) : 0.0;
+            p[b0 + i] = pi;
+            if (x == x && x * (1.0 - pi) > u) u = x * (1.0 - pi);
+        }
+        lambda[q] = lam;
+        utility[q] = n > 0 ? u : 0.0;
+        free(pos);
+    }
+    return flag;
 }

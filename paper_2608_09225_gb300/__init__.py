@@ -7,4 +7,4 @@ first binding call loads the library and raises if it or a GPU is missing.
 """
 from .kvgov import (BLOCK, BOUNDARY, DIGEST_BYTES, ROOT, UNSALTED, KVGovError, block_offsets,  # noqa: F401
                     chain_hash, chain_hash_arrival, chain_hash_probe, derive_salts, divergence_boundary, insert, insert_arrival, insert_uncached, new_owner,
-                    new_table, owner_init, probe, probe_arrival, response_key, set_spin_limit, status_string, table_init)
+                    new_table, origami, owner_init, probe, probe_arrival, response_key, set_spin_limit, status_string, table_init)

@@ -68,12 +68,13 @@ def _load():
                                                _p, _p, _p, ctypes.c_uint64, ctypes.c_uint64, _p, _p, _p, _p, _p]
         L.kvgov_divergence_boundary.argtypes = [_p, _p, ctypes.c_int32, _p, _p, _p, ctypes.c_int32, _p, _p, _p]
         L.kvgov_response_key.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p, _p]
+        L.kvgov_origami.argtypes = [_p, _p, ctypes.c_int32, _p, _p, _p, _p, _p, _p]
         L.kvgov_set_spin_limit.argtypes = [ctypes.c_uint32]
         L.kvgov_set_spin_limit.restype = ctypes.c_uint32
         for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
                    "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
                    "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
-                   "kvgov_divergence_boundary", "kvgov_response_key"):
+                   "kvgov_divergence_boundary", "kvgov_response_key", "kvgov_origami"):
             getattr(L, fn).restype = ctypes.c_int
         _lib = L
         return L
@@ -396,6 +397,32 @@ def response_key(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, princip
                                     _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_response_key")
     return keys
+
+
+def origami(values: torch.Tensor, off: torch.Tensor, budget: torch.Tensor, p: torch.Tensor | None = None,
+            lam: torch.Tensor | None = None, utility: torch.Tensor | None = None, status: torch.Tensor | None = None,
+            stream=None):
+    """ORIGAMI audit probabilities per problem (paper section 4.3): float32
+    values in CSR by off, float32 budgets; returns (p, lambda, utility)."""
+    n = off.numel() - 1
+    if p is None:
+        p = torch.empty_like(values)
+    if lam is None:
+        lam = torch.empty(max(n, 0), dtype=torch.float32, device=off.device)
+    if utility is None:
+        utility = torch.empty(max(n, 0), dtype=torch.float32, device=off.device)
+    if values.numel() == 0:
+        values = torch.zeros(1, dtype=torch.float32, device=off.device)
+        p_arg = _dummy(off)
+    else:
+        p_arg = _dev(p, torch.float32, "p")
+    _check(lib().kvgov_origami(_dev(values, torch.float32, "values"), _dev(off, torch.int64, "off"), n,
+                               _dev(budget, torch.float32, "budget") if n else _dummy(off), p_arg,
+                               _dev(lam, torch.float32, "lambda") if n else None,
+                               _dev(utility, torch.float32, "utility") if n else None,
+                               _dev(status, torch.int32, "status", True), _stream(stream)),
+           "kvgov_origami")
+    return p, lam, utility
 
 
 def set_spin_limit(limit: int) -> int:

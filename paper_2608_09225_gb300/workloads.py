@@ -245,3 +245,44 @@ def ragged(seed: int, lengths) -> Batch:
     cyc = np.array([0, 15, 16, 17, 31, 32, 64, 10 ** 6], dtype=np.int32)
     boundary = cyc[np.arange(n) % len(cyc)]
     return Batch(tokens=tokens, tok_off=tok_off, principal=principal, boundary_tok=boundary)
+
+
+@dataclass
+class AuditBatch:
+    """ORIGAMI audit problems (paper section 4.3): tenant values at risk in
+    CSR form and one budget per problem."""
+    values: np.ndarray          # float32 [total tenants]
+    off: np.ndarray             # int64 [n_prob + 1]
+    budget: np.ndarray          # float32 [n_prob]
+
+    @property
+    def n(self) -> int:
+        return len(self.off) - 1
+
+
+def audit(seed: int = 2032, n_prob: int = 1 << 20, n_tenants: int = 50, budget: float = 10.0,
+          alpha: float = 1.29) -> AuditBatch:
+    """The adversarial-load setting of section 5.5, batched: n_prob problems
+    of n_tenants tenants whose values are Pareto(alpha) (x_m = 1; alpha = 1.29
+    gives Gini about 0.63), budget K each."""
+    rng = np.random.default_rng(seed)
+    values = (1.0 + rng.pareto(alpha, n_prob * n_tenants)).astype(np.float32)
+    off = np.arange(0, n_prob * n_tenants + 1, n_tenants, dtype=np.int64)
+    return AuditBatch(values=values, off=off, budget=np.full(n_prob, budget, np.float32))
+
+
+def audit_ragged(seed: int, n_prob: int, max_tenants: int = 300) -> AuditBatch:
+    """Audit problems of 0..max_tenants tenants, Pareto or uniform values (a
+    fifth of the problems all-equal), budgets in [0, n + 2] (some above n)."""
+    rng = np.random.default_rng(seed)
+    sizes = rng.integers(0, max_tenants + 1, n_prob)
+    vals = []
+    for n in sizes:
+        if rng.random() < 0.2:
+            vals.append(np.full(n, float(rng.uniform(0.5, 5.0)), np.float32))
+        else:
+            vals.append((1.0 + rng.pareto(float(rng.uniform(0.8, 3.0)), n)).astype(np.float32))
+    off = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int64)
+    budget = (rng.random(n_prob) * (sizes + 2)).astype(np.float32)
+    return AuditBatch(values=np.concatenate(vals + [np.zeros(0, np.float32)]).astype(np.float32), off=off,
+                      budget=budget)

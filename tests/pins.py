@@ -603,4 +603,76 @@ def pin_response_key_whole_prompt():
     assert (d[:132] == d[132:]).all()                  # the blocks never see the tail
 
 
+# ------------------------------------------------------ ORIGAMI (section 4.3)
+def pin_origami_linear_program():
+    """The allocation == scipy's LP solution of the epigraph form the paper's
+    proof uses: minimise t subject to v_i (1 - p_i) <= t, sum p = K,
+    0 <= p <= 1.  t* is the water level and p* the probabilities."""
+    from scipy.optimize import linprog
+    rng = np.random.default_rng(26)
+    for trial in range(25):
+        n = int(rng.integers(2, 12))
+        v = (1.0 + rng.pareto(1.29, n)).astype(np.float32)
+        K = float(np.float32(rng.uniform(0.2, n - 0.2)))
+        c = np.zeros(n + 1)
+        c[-1] = 1.0
+        A = np.zeros((n, n + 1))
+        A[np.arange(n), np.arange(n)] = -v.astype(np.float64)
+        A[:, -1] = -1.0
+        res = linprog(c, A_ub=A, b_ub=-v.astype(np.float64), A_eq=np.concatenate([np.ones(n), [0.0]])[None],
+                      b_eq=[K], bounds=[(0, 1)] * n + [(None, None)], method="highs")
+        assert res.status == 0
+        p, lam, u, flag = oracle.origami(v, np.array([0, n], np.int64), np.array([K], np.float32))
+        assert not flag
+        assert abs(lam[0] - res.x[-1]) <= 1e-7 * max(1.0, res.x[-1]), trial
+        assert np.abs(p - res.x[:n]).max() <= 1e-6, trial
+        assert abs(u[0] - res.fun) <= 1e-7 * max(1.0, res.fun)
+
+
+def pin_origami_bisection():
+    """The paper finds lambda by bisection on sum_i max(0, 1 - lambda/v_i) = K;
+    a plain Python bisection (fp64, 200 halvings) lands on the oracle's level."""
+    rng = np.random.default_rng(27)
+    b = W.audit(seed=27, n_prob=40, n_tenants=50)
+    p, lam, _, _ = oracle.origami(b.values, b.off, b.budget)
+    for q in range(b.n):
+        v = [float(x) for x in b.values[b.off[q]:b.off[q + 1]]]
+        K = float(b.budget[q])
+        lo, hi = 0.0, max(v)
+        for _ in range(200):
+            mid = (lo + hi) / 2
+            if sum(max(0.0, 1.0 - mid / x) for x in v) > K:
+                lo = mid
+            else:
+                hi = mid
+        assert abs((lo + hi) / 2 - lam[q]) <= 1e-12 * lam[q], q
+    del rng
+
+
+def pin_origami_closed_forms():
+    """Equal values: p = K/n, the same as uniform random audit (section 5.4);
+    K >= n: every tenant audited, lambda = 0; K = 0: none, lambda = max v;
+    tenants of value <= 0 get nothing; and on Pareto batches the water-filling
+    properties: sum p = K, 0 <= p <= 1, v (1 - p) = lambda where p > 0,
+    v <= lambda where p = 0, utility = lambda."""
+    v = np.array([3.0] * 10 + [2, 4, 8] + [5, 1] + [-1.0, 0.0, 7.0], np.float32)
+    off = np.array([0, 10, 13, 15, 18], np.int64)
+    K = np.array([5, 3.5, 0, 1], np.float32)
+    p, lam, u, flag = oracle.origami(v, off, K)
+    assert not flag
+    assert np.allclose(p[:10], 0.5) and abs(lam[0] - 1.5) < 1e-12 and abs(u[0] - 1.5) < 1e-12
+    assert np.allclose(p[10:13], 1.0) and lam[1] == 0.0           # K capped at n
+    assert np.allclose(p[13:15], 0.0) and lam[2] == 5.0 and u[2] == 5.0
+    assert list(p[15:18]) == [0.0, 0.0, 1.0] and lam[3] == 0.0     # one usable tenant, K = 1
+    b = W.audit(seed=28, n_prob=200, n_tenants=50)
+    p, lam, u, _ = oracle.origami(b.values, b.off, b.budget)
+    for q in range(b.n):
+        s, e = int(b.off[q]), int(b.off[q + 1])
+        pq, vq = p[s:e], b.values[s:e].astype(np.float64)
+        assert abs(pq.sum() - b.budget[q]) < 1e-9 and (pq >= 0).all() and (pq <= 1).all()
+        act = pq > 0
+        assert np.allclose(vq[act] * (1 - pq[act]), lam[q], rtol=1e-12)
+        assert (vq[~act] <= lam[q] * (1 + 1e-12)).all() and abs(u[q] - lam[q]) <= 1e-12 * lam[q]
+
+
 PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

@@ -1,0 +1,88 @@
+"""ORIGAMI audit allocation on the GPU (kvgov_origami, fp32) against the
+oracle (fp64 closed form).  Marked gpu.
+
+Tolerance, from the arithmetic: the kernel's water level is (m - K) / S with
+S a fp32 sum of m reciprocals (each correctly rounded), so its relative error
+is at most about (m + 3) u, u = 2^-24; p_i = 1 - lambda / v_i adds one more
+rounding, and lambda / v_i <= 1 for every audited tenant.  The tests allow
+8 (n + 4) u: twice that bound with room for the order of the sum."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_09225_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+U = 2.0 ** -24
+
+
+def tol(n):
+    return 8.0 * (n + 4) * U
+
+
+def gpu(kv, b: W.AuditBatch):
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    v = torch.from_numpy(np.ascontiguousarray(b.values)).to(DEV)
+    p, lam, u = kv.origami(v, torch.from_numpy(b.off).to(DEV), torch.from_numpy(b.budget).to(DEV), status=st)
+    torch.cuda.synchronize()
+    return p.cpu().numpy().astype(np.float64), lam.cpu().numpy().astype(np.float64), \
+        u.cpu().numpy().astype(np.float64), int(st.item())
+
+
+def check(b, p, lam, u, p_ref, lam_ref, u_ref):
+    for q in range(b.n):
+        s, e = int(b.off[q]), int(b.off[q + 1])
+        t = tol(e - s)
+        assert np.abs(p[s:e] - p_ref[s:e]).max(initial=0.0) <= t, q
+        assert abs(lam[q] - lam_ref[q]) <= t * max(lam_ref[q], 1e-30), q
+        assert abs(u[q] - u_ref[q]) <= t * max(abs(u_ref[q]), 1e-30), q
+
+
+@pytest.mark.parametrize("seed,n_prob", [(1, 1), (2, 64), (3, 3000)])
+def test_origami_ragged_matches_oracle(kv, seed, n_prob):
+    b = W.audit_ragged(seed, n_prob)
+    p, lam, u, st = gpu(kv, b)
+    p_ref, lam_ref, u_ref, flag = oracle.origami(b.values, b.off, b.budget)
+    assert st == 0 and not flag
+    check(b, p, lam, u, p_ref, lam_ref, u_ref)
+
+
+def test_origami_pareto_batch(kv):
+    """131,072 problems of the section 5.5 setting (50 tenants, Pareto 1.29,
+    K = 10): every probability within tolerance, and each problem's budget
+    spent to within the rounding of its sum."""
+    b = W.audit(seed=5, n_prob=131072)
+    p, lam, u, st = gpu(kv, b)
+    p_ref, lam_ref, u_ref, _ = oracle.origami(b.values, b.off, b.budget)
+    assert st == 0
+    assert np.abs(p - p_ref).max() <= tol(50)
+    assert (np.abs(lam - lam_ref) <= tol(50) * lam_ref).all()
+    sums = np.add.reduceat(p, b.off[:-1])
+    assert np.abs(sums - 10.0).max() <= 50 * tol(50)
+
+
+def test_origami_edge_cases_and_flags(kv):
+    """Empty problems, K above n, K = 0, values <= 0, and flagged inputs: a NaN
+    value, an infinite value, a negative budget."""
+    vals = [np.zeros(0, np.float32), np.array([2, 4, 8], np.float32), np.array([5, 1], np.float32),
+            np.array([-1, 0, 7], np.float32), np.array([3.0] * 10, np.float32)]
+    off = np.concatenate([[0], np.cumsum([len(x) for x in vals])]).astype(np.int64)
+    b = W.AuditBatch(values=np.concatenate(vals), off=off, budget=np.array([1, 3.5, 0, 1, 5], np.float32))
+    p, lam, u, st = gpu(kv, b)
+    p_ref, lam_ref, u_ref, flag = oracle.origami(b.values, b.off, b.budget)
+    assert st == 0 and not flag
+    check(b, p, lam, u, p_ref, lam_ref, u_ref)
+    assert list(p[0:3]) == [1.0, 1.0, 1.0] and lam[1] == 0.0 and lam[2] == 5.0 and list(p[5:8]) == [0, 0, 1]
+    for bad_vals, bad_budget in ((np.array([1, np.nan, 2], np.float32), 1.0),
+                                 (np.array([1, np.inf, 2], np.float32), 1.0),
+                                 (np.array([1, 3, 2], np.float32), -1.0)):
+        b = W.AuditBatch(values=bad_vals, off=np.array([0, 3], np.int64), budget=np.array([bad_budget], np.float32))
+        p, lam, u, st = gpu(kv, b)
+        p_ref, lam_ref, _, flag = oracle.origami(b.values, b.off, b.budget)
+        assert st == kv.F_BADINDEX and flag
+        assert np.abs(p - p_ref).max() <= tol(3) and abs(lam[0] - lam_ref[0]) <= tol(3) * max(lam_ref[0], 1)
+        assert math.isfinite(lam[0])

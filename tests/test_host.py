@@ -35,7 +35,7 @@ def test_header_declares_the_boundary():
     for want in ("kvgov_derive_salts", "kvgov_block_offsets", "kvgov_chain_hash", "kvgov_table_init",
                  "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
                  "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
-                 "kvgov_divergence_boundary", "kvgov_response_key", "kvgov_status_string",
+                 "kvgov_divergence_boundary", "kvgov_response_key", "kvgov_origami", "kvgov_status_string",
                  "kvgov_set_spin_limit"):
         assert want in names
 
@@ -175,6 +175,11 @@ def test_host_validation_rejects_bad_arguments(libkv):
     assert rk(1, fake, fake, 3, None, fake, 1, fake, None, None) == 1                    # ROOT without principals
     assert rk(0, odd, fake, 3, None, None, 0, fake, None, None) == 1                     # misaligned tokens
     assert rk(0, fake, fake, 0, None, None, 0, None, None, None) == 0                    # empty batch
+    og = libkv.kvgov_origami
+    og.argtypes = [p, p, ctypes.c_int32, p, p, p, p, p, p]
+    assert og(fake, fake, -1, fake, fake, None, None, None, None) == 1                   # negative count
+    assert og(fake, fake, 3, None, fake, None, None, None, None) == 1                    # no budgets
+    assert og(None, fake, 0, None, None, None, None, None, None) == 0                    # no problems
     pa = libkv.kvgov_probe_arrival
     pa.argtypes = [p, ctypes.c_uint64, p, p, ctypes.c_int32, ctypes.c_uint64, p, p, p]
     assert pa(fake, 64, fake, fake, 3, 0, fake, None, None) == 1

@@ -84,6 +84,9 @@ MUTATIONS = [
     ("response_token_bytes_swapped",
      "msg[salt_len + 4 * i] = (uint8_t)v;\n            msg[salt_len + 4 * i + 1] = (uint8_t)(v >> 8);",
      "msg[salt_len + 4 * i + 1] = (uint8_t)v;\n            msg[salt_len + 4 * i] = (uint8_t)(v >> 8);"),
+    ("origami_ascending_order", "return (x < y) - (x > y);", "return (x > y) - (x < y);"),
+    ("origami_budget_sign", "const double lm = ((double)m - K) / inv_sum;", "const double lm = ((double)m + K) / inv_sum;"),
+    ("origami_no_clamp", "(1.0 - lam / x > 0.0 ? 1.0 - lam / x : 0.0)", "(1.0 - lam / x)"),
     ("arrival_reserved_keys_stored",
      "            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);",
      "            chain_set_add(&s, req + 32 * (size_t)q);"),
