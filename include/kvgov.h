@@ -388,6 +388,26 @@ int kvgov_probe_arrival(const uint64_t *d_owner, uint64_t capacity, const uint32
                         uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * kvgov_serve_arrival_static -- kvgov_insert_arrival followed by
+ * kvgov_probe_arrival on one batch, allocating nothing: the slot of each
+ * block lives in a device array of 2^21 entries (8 MiB) inside the library
+ * rather than in caller memory.  The paper has no counterpart; it is an
+ * allocation-free form of the same computation (same table, owners, key
+ * count and prefix lengths; the slot handles are not returned).
+ *   Arguments as for kvgov_insert_arrival and kvgov_probe_arrival;
+ *   n_blocks   the batch's block count, d_blk_off[n_req].
+ * EINVAL also when n_blocks exceeds 2^21; if d_blk_off[n_req] itself does, no
+ * block is inserted and every request is flagged KVGOV_F_BADINDEX with
+ * prefix 0.  The array is shared by every call on the device: calls that
+ * overlap in time (other streams, other host threads) race on it and give
+ * wrong results.  Three launches on `stream`.
+ */
+int kvgov_serve_arrival_static(uint8_t *d_slots, uint64_t *d_owner, uint64_t capacity, const uint8_t *d_digests,
+                               const int64_t *d_blk_off, int32_t n_req, int64_t n_blocks, uint64_t seq_base,
+                               int32_t *d_prefix_blocks, unsigned long long *d_n_new, uint32_t *d_status,
+                               kvgov_stream_t stream);
+
+/*
  * kvgov_chain_hash_arrival -- a batch's chain hash and its arrival-order
  * serving in one call: the digests of kvgov_chain_hash, then the table,
  * owners, slot handles, prefix lengths and key count of kvgov_insert_arrival

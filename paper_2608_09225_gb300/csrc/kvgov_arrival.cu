@@ -44,6 +44,7 @@ constexpr unsigned long long kPending = kOwnerPending;
 // Largest first position of a batch: positions stay below kPending for any
 // batch that fits in memory (2^62 blocks).
 constexpr unsigned long long kMaxSeq = 1ull << 62;
+constexpr long long kNoRowCap = 0x7fffffffffffffffll;   // slot_of sized by the caller
 constexpr int kThreads = 256;
 constexpr int G = 8;                         // lanes per request
 constexpr int kSegs = 32 / G;
@@ -70,11 +71,12 @@ __device__ __forceinline__ void request_range(const int64_t *__restrict__ blk_of
     }
 }
 
-// The batch's block count, blk_off[n_req] (0, flagged, if negative).
+// The batch's block count, blk_off[n_req] (0, flagged, if negative or above
+// row_cap, the rows slot_of can hold).
 __device__ __forceinline__ long long batch_rows(const int64_t *__restrict__ blk_off, int32_t n_req, uint32_t *status,
-                                                bool flag) {
+                                                bool flag, long long row_cap) {
     const long long n = blk_off[n_req];
-    if (n < 0) {
+    if (n < 0 || n > row_cap) {
         if (flag && blockIdx.x == 0 && threadIdx.x == 0) raise_flag(status, KVGOV_F_BADINDEX);
         return 0;
     }
@@ -84,11 +86,12 @@ __device__ __forceinline__ long long batch_rows(const int64_t *__restrict__ blk_
 __global__ void __launch_bounds__(kThreads) insert_arrival_kernel(
     unsigned long long *__restrict__ slots, unsigned long long mask, unsigned long long *__restrict__ owner,
     const uint4 *__restrict__ digests, const int64_t *__restrict__ blk_off, int32_t n_req,
-    uint32_t *__restrict__ slot_of, unsigned long long *n_new, uint32_t *status, uint32_t spin_limit) {
+    uint32_t *__restrict__ slot_of, unsigned long long *n_new, uint32_t *status, uint32_t spin_limit,
+    long long row_cap) {
     __shared__ unsigned int s_new, s_flags, s_done;
     if (threadIdx.x == 0) { s_new = 0; s_flags = 0; s_done = 0; }
     __syncthreads();
-    const long long n_rows = batch_rows(blk_off, n_req, status, true);
+    const long long n_rows = batch_rows(blk_off, n_req, status, true, row_cap);
     const long long stride = (long long)gridDim.x * kThreads;
     const int lane = threadIdx.x & 31;
     unsigned my_new = 0, my_flags = 0;
@@ -114,8 +117,8 @@ __global__ void __launch_bounds__(kThreads) insert_arrival_kernel(
 __global__ void __launch_bounds__(kThreads) owner_min_kernel(const int64_t *__restrict__ blk_off, int32_t n_req,
                                                              const uint32_t *__restrict__ slot_of,
                                                              unsigned long long *__restrict__ owner,
-                                                             unsigned long long seq_base) {
-    const long long n_rows = batch_rows(blk_off, n_req, nullptr, false);
+                                                             unsigned long long seq_base, long long row_cap) {
+    const long long n_rows = batch_rows(blk_off, n_req, nullptr, false, row_cap);
     const long long stride = (long long)gridDim.x * kThreads;
     const int lane = threadIdx.x & 31;
     for (long long r0 = (long long)blockIdx.x * kThreads + (threadIdx.x & ~31); r0 < n_rows; r0 += stride) {
@@ -158,15 +161,21 @@ __global__ void __launch_bounds__(kThreads) probe_arrival_kernel(const unsigned 
                                                                  const uint32_t *__restrict__ slot_of,
                                                                  const int64_t *__restrict__ blk_off, int32_t n_req,
                                                                  unsigned long long seq_base,
-                                                                 int32_t *__restrict__ prefix_blocks, uint32_t *status) {
+                                                                 int32_t *__restrict__ prefix_blocks, uint32_t *status,
+                                                                 long long row_cap) {
     const int lane = threadIdx.x & 31, seg = lane / G, sl = lane % G;
     const long long warps_total = (long long)gridDim.x * (kThreads / 32);
+    const bool over = blk_off[n_req] > row_cap;           // the insert stored no slot: every request is bad
     for (long long w = ((long long)blockIdx.x * kThreads + threadIdx.x) / 32; w * kSegs < n_req;
          w += warps_total) {                                   // warp-uniform
         const long long r = w * kSegs + seg;
         long long base, nb;
         unsigned flags = 0;
         request_range(blk_off, n_req, r, base, nb, flags);
+        if (over && r < n_req) {
+            flags |= KVGOV_F_BADINDEX;
+            nb = 0;
+        }
         if (flags && sl == 0) raise_flag(status, flags);
         const unsigned long long first = seq_base + (unsigned long long)base;   // position of r's block 0
         bool active = nb > 0;
@@ -209,6 +218,25 @@ unsigned row_grid() { return (unsigned)(kvgov_host::sm_count() * 8); }
 // Capacities whose slot index fits slot_of's u32 with kNoSlot to spare.
 bool arrival_capacity(uint64_t capacity) {
     return kvgov_host::pow2_capacity(capacity) && capacity <= (1ull << 31);
+}
+
+// Scratch of kvgov_serve_arrival_static: the slot of each block of one batch,
+// 2^21 entries (8 MiB), in a file-scope device array instead of caller
+// memory.  Every call on the device uses it, so calls must not overlap.
+constexpr long long kStaticRows = 1ll << 21;
+static __device__ __align__(256) uint32_t g_static_slot_of[kStaticRows];
+
+// Its device address, looked up once per device.
+uint32_t *static_slot_of() {
+    static uint32_t *addr[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    if (!addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_static_slot_of) != cudaSuccess || !p) return nullptr;
+        addr[dev] = static_cast<uint32_t *>(p);
+    }
+    return addr[dev];
 }
 
 }  // namespace
@@ -256,9 +284,10 @@ extern "C" int kvgov_insert_arrival(uint8_t *d_slots, uint64_t *d_owner, uint64_
     insert_arrival_kernel<<<grid, kThreads, 0, s>>>(reinterpret_cast<unsigned long long *>(d_slots), capacity - 1,
                                                     reinterpret_cast<unsigned long long *>(d_owner),
                                                     reinterpret_cast<const uint4 *>(d_digests), d_blk_off, n_req,
-                                                    d_slot_of, d_n_new, d_status, kvgov_host::spin_limit());
+                                                    d_slot_of, d_n_new, d_status, kvgov_host::spin_limit(),
+                                                    kNoRowCap);
     owner_min_kernel<<<grid, kThreads, 0, s>>>(d_blk_off, n_req, d_slot_of,
-                                               reinterpret_cast<unsigned long long *>(d_owner), seq_base);
+                                               reinterpret_cast<unsigned long long *>(d_owner), seq_base, kNoRowCap);
     return kvgov_host::launch_status();
 }
 
@@ -271,6 +300,34 @@ extern "C" int kvgov_probe_arrival(const uint64_t *d_owner, uint64_t capacity, c
     if (!d_slot_of || !d_blk_off || !d_prefix_blocks) return KVGOV_EINVAL;
     probe_arrival_kernel<<<request_grid(n_req), kThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
         reinterpret_cast<const unsigned long long *>(d_owner), d_slot_of, d_blk_off, n_req, seq_base,
-        d_prefix_blocks, d_status);
+        d_prefix_blocks, d_status, kNoRowCap);
+    return kvgov_host::launch_status();
+}
+
+extern "C" int kvgov_serve_arrival_static(uint8_t *d_slots, uint64_t *d_owner, uint64_t capacity,
+                                          const uint8_t *d_digests, const int64_t *d_blk_off, int32_t n_req,
+                                          int64_t n_blocks, uint64_t seq_base, int32_t *d_prefix_blocks,
+                                          unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream) {
+    using kvgov_host::aligned16;
+    if (!d_slots || !aligned16(d_slots) || !d_owner || !arrival_capacity(capacity) || n_req < 0 || !d_status ||
+        seq_base == 0 || seq_base > kMaxSeq || n_blocks < 0 || n_blocks > kStaticRows)
+        return KVGOV_EINVAL;
+    if (n_req == 0) return KVGOV_OK;
+    if (!d_digests || !aligned16(d_digests) || !d_blk_off || !d_prefix_blocks) return KVGOV_EINVAL;
+    uint32_t *slot_of = static_slot_of();
+    if (!slot_of) return KVGOV_ECUDA;
+    // Nothing in the scratch has to start at zero: the insert writes the entry
+    // of every block that the owner min and the probe read.
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const unsigned grid = row_grid();
+    insert_arrival_kernel<<<grid, kThreads, 0, s>>>(reinterpret_cast<unsigned long long *>(d_slots), capacity - 1,
+                                                    reinterpret_cast<unsigned long long *>(d_owner),
+                                                    reinterpret_cast<const uint4 *>(d_digests), d_blk_off, n_req,
+                                                    slot_of, d_n_new, d_status, kvgov_host::spin_limit(), kStaticRows);
+    owner_min_kernel<<<grid, kThreads, 0, s>>>(d_blk_off, n_req, slot_of,
+                                               reinterpret_cast<unsigned long long *>(d_owner), seq_base, kStaticRows);
+    probe_arrival_kernel<<<request_grid(n_req), kThreads, 0, s>>>(reinterpret_cast<const unsigned long long *>(d_owner),
+                                                                  slot_of, d_blk_off, n_req, seq_base,
+                                                                  d_prefix_blocks, d_status, kStaticRows);
     return kvgov_host::launch_status();
 }

@@ -69,12 +69,15 @@ def _load():
         L.kvgov_divergence_boundary.argtypes = [_p, _p, ctypes.c_int32, _p, _p, _p, ctypes.c_int32, _p, _p, _p]
         L.kvgov_response_key.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p, _p]
         L.kvgov_origami.argtypes = [_p, _p, ctypes.c_int32, _p, _p, _p, _p, _p, _p]
+        L.kvgov_serve_arrival_static.argtypes = [_p, _p, ctypes.c_uint64, _p, _p, ctypes.c_int32, ctypes.c_int64,
+                                                 ctypes.c_uint64, _p, _p, _p, _p]
         L.kvgov_set_spin_limit.argtypes = [ctypes.c_uint32]
         L.kvgov_set_spin_limit.restype = ctypes.c_uint32
         for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
                    "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
                    "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
-                   "kvgov_divergence_boundary", "kvgov_response_key", "kvgov_origami"):
+                   "kvgov_divergence_boundary", "kvgov_response_key", "kvgov_origami",
+                   "kvgov_serve_arrival_static"):
             getattr(L, fn).restype = ctypes.c_int
         _lib = L
         return L
@@ -423,6 +426,26 @@ def origami(values: torch.Tensor, off: torch.Tensor, budget: torch.Tensor, p: to
                                _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_origami")
     return p, lam, utility
+
+
+def serve_arrival_static(slots: torch.Tensor, owner: torch.Tensor, digests: torch.Tensor, blk_off: torch.Tensor,
+                         seq_base: int, status: torch.Tensor, prefix_blocks: torch.Tensor | None = None,
+                         n_new: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """insert_arrival + probe_arrival with the slot handles kept in the
+    library's own device array (at most 2^21 blocks; calls must not overlap)."""
+    n = blk_off.numel() - 1
+    n_blocks = digests.shape[0] if digests.dim() == 2 else 0
+    if prefix_blocks is None:
+        prefix_blocks = torch.empty(max(n, 0), dtype=torch.int32, device=blk_off.device)
+    _check(lib().kvgov_serve_arrival_static(_dev(slots, torch.uint8, "slots"), _dev(owner, torch.int64, "owner"),
+                                            slots.shape[0],
+                                            _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(blk_off),
+                                            _dev(blk_off, torch.int64, "blk_off"), n, n_blocks, int(seq_base),
+                                            _dev(prefix_blocks, torch.int32, "prefix_blocks") if n else _dummy(blk_off),
+                                            _dev(n_new, torch.int64, "n_new", True),
+                                            _dev(status, torch.int32, "status"), _stream(stream)),
+           "kvgov_serve_arrival_static")
+    return prefix_blocks
 
 
 def set_spin_limit(limit: int) -> int:
