@@ -364,6 +364,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--configs", action="store_true",
                     help="instead of the timed serving step: per-kernel rates on every workload, one JSON line each")
+    ap.add_argument("--only", default=None,
+                    help="with --configs: comma-separated workloads to run (tiny, sysprompt, template, probe, long, "
+                         "wide, audit)")
     args = ap.parse_args()
     if args.seed is None:
         args.seed = int.from_bytes(os.urandom(4), "little")
@@ -732,11 +735,22 @@ def run_configs(args):
     gather = measure_gather(torch, kbuild.PEAK_LIB, scratch_table)
     del scratch_table
     print(json.dumps({"random_read_microbench": gather, "hbm_gbs": PEAKS.get("hbm_gbs")}), flush=True)
-    plan = [("tiny", W.make("tiny"), W.ROOT), ("sysprompt", W.make("sysprompt"), W.ROOT)]
-    tmpl = W.make("template")
-    plan += [("template", tmpl, m) for m in (W.UNSALTED, W.ROOT, W.BOUNDARY)]
-    plan += [("probe", W.make("probe"), W.ROOT), ("long", W.make("long", seed=seed), W.BOUNDARY),
-             ("wide", W.make("wide", seed=seed + 1), W.BOUNDARY)]
+    only = set(args.only.split(",")) if args.only else None
+    want = (lambda n: only is None or n in only)
+    plan = []
+    if want("tiny"):
+        plan.append(("tiny", W.make("tiny"), W.ROOT))
+    if want("sysprompt"):
+        plan.append(("sysprompt", W.make("sysprompt"), W.ROOT))
+    if want("template"):
+        tmpl = W.make("template")
+        plan += [("template", tmpl, m) for m in (W.UNSALTED, W.ROOT, W.BOUNDARY)]
+    if want("probe"):
+        plan.append(("probe", W.make("probe"), W.ROOT))
+    if want("long"):
+        plan.append(("long", W.make("long", seed=seed), W.BOUNDARY))
+    if want("wide"):
+        plan.append(("wide", W.make("wide", seed=seed + 1), W.BOUNDARY))
     names = {W.UNSALTED: "UNSALTED", W.ROOT: "ROOT", W.BOUNDARY: "BOUNDARY"}
     for name, w, mode in plan:
         b = w.batch
@@ -875,7 +889,8 @@ def run_configs(args):
         print(json.dumps(line), flush=True)
         del cache, keys, dig
         torch.cuda.empty_cache()
-    print(json.dumps(audit_rates(torch, K, W, seed, cores, args.no_cpu_baseline)), flush=True)
+    if want("audit"):
+        print(json.dumps(audit_rates(torch, K, W, seed, cores, args.no_cpu_baseline)), flush=True)
     return 0
 
 

@@ -43,6 +43,18 @@ __device__ __forceinline__ ulonglong2 ld_relaxed2(const unsigned long long *p) {
 __device__ __forceinline__ void st_relaxed(unsigned long long *p, unsigned long long v) {
     asm volatile("st.relaxed.gpu.global.u64 [%0], %1;\n" ::"l"(p), "l"(v) : "memory");
 }
+// Both words of a 16-byte-aligned pair in one store.  Each word is written
+// once, from zero, so a reader that sees one word and not the other still
+// sees a zero word and waits.
+__device__ __forceinline__ void st_relaxed2(unsigned long long *p, unsigned long long a, unsigned long long b) {
+    asm volatile("st.relaxed.gpu.global.v2.u64 [%0], {%1, %2};\n" ::"l"(p), "l"(a), "l"(b) : "memory");
+}
+
+// Build-time choice: KVGOV_INSERT_ST16 writes a claimed key's second half
+// with one 16-byte store (default) instead of two 8-byte stores.
+#ifndef KVGOV_INSERT_ST16
+#define KVGOV_INSERT_ST16 1
+#endif
 // 128-bit compare-and-swap of the 16-byte-aligned pair p[0..1]: if it holds
 // (c0, c1) it becomes (n0, n1); the previous value is returned in (o0, o1).
 __device__ __forceinline__ void cas128(unsigned long long *p, unsigned long long c0, unsigned long long c1,
@@ -90,8 +102,12 @@ __device__ __forceinline__ InsertResult insert_one(unsigned long long *slots, un
         {
             cas128(slot, 0ull, 0ull, k[0], k[1], o0, o1);
             if ((o0 | o1) == 0ull) {                 // claimed: write the second half
+#if KVGOV_INSERT_ST16
+                st_relaxed2(slot + 2, k[2], k[3]);
+#else
                 st_relaxed(slot + 2, k[2]);
                 st_relaxed(slot + 3, k[3]);
+#endif
                 if (pos_out) *pos_out = pos;
                 return kNew;
             }

@@ -54,6 +54,11 @@ using namespace kvgov_dev;
 #ifndef KVGOV_INSERT_DEDUP
 #define KVGOV_INSERT_DEDUP 0
 #endif
+// KVGOV_INSERT_PACK selects the warp-packed kvgov_insert_uncached kernel
+// (insert_uncached_packed_kernel) over the one with 8 lanes per request.
+#ifndef KVGOV_INSERT_PACK
+#define KVGOV_INSERT_PACK 1
+#endif
 
 constexpr uint32_t kDefaultSpin = 1u << 23;
 std::atomic<uint32_t> g_spin_limit{kDefaultSpin};
@@ -217,6 +222,77 @@ __global__ void __launch_bounds__(kInsertThreads) insert_uncached_kernel(
     publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
 }
 
+// The same insert with the uncached blocks of kPackReq requests packed into
+// the 32 lanes of a warp: lanes 0..kPackReq-1 read their request's range and
+// count of uncached blocks, a warp scan numbers the blocks, and in each round
+// lane l takes block i0 + l, finding its request with a 5-step search over the
+// scan.  No lane idles while blocks remain (with 8 lanes per request, a
+// request with 4 cached and 4 uncached blocks leaves half the lanes idle).
+constexpr int kPackReq = 8;
+
+__global__ void __launch_bounds__(kInsertThreads) insert_uncached_packed_kernel(
+    unsigned long long *__restrict__ slots, unsigned long long mask, const uint4 *__restrict__ digests,
+    const int64_t *__restrict__ blk_off, int32_t n_req, const int32_t *__restrict__ prefix_blocks,
+    unsigned long long *n_new, uint32_t *status, uint32_t spin_limit) {
+    __shared__ unsigned int s_new, s_flags, s_done;
+    if (threadIdx.x == 0) { s_new = 0; s_flags = 0; s_done = 0; }
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    const long long warps_total = (long long)gridDim.x * (kInsertThreads / 32);
+    unsigned my_new = 0, my_flags = 0;
+    for (long long w = ((long long)blockIdx.x * kInsertThreads + threadIdx.x) / 32; w * kPackReq < n_req;
+         w += warps_total) {                                   // warp-uniform
+        const long long r = w * kPackReq + lane;
+        long long first = 0;                                   // row of the request's first uncached block
+        int c = 0;                                             // its uncached blocks
+        if (lane < kPackReq && r < n_req) {
+            const long long base = blk_off[r], nb = blk_off[r + 1] - base;
+            if (nb < 0 || base < 0 || base + nb > blk_off[n_req]) {
+                my_flags |= KVGOV_F_BADINDEX;
+            } else {
+                long long L = prefix_blocks[r];
+                L = L < 0 ? 0 : (L > nb ? nb : L);
+                first = base + L;
+                c = (int)(nb - L);
+            }
+        }
+        int incl = c;                                          // inclusive scan of c over the lanes
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+            const int t = __shfl_up_sync(0xffffffffu, incl, d);
+            if (lane >= d) incl += t;
+        }
+        const int total = __shfl_sync(0xffffffffu, incl, 31);
+        for (int i0 = 0; i0 < total; i0 += 32) {               // warp-uniform
+            const int k = i0 + lane;
+            int lo = 0, hi = 31;                               // the first lane whose scan passes k
+#pragma unroll
+            for (int step = 0; step < 5; ++step) {
+                const int mid = (lo + hi) >> 1;
+                if (__shfl_sync(0xffffffffu, incl, mid) > k) hi = mid;
+                else lo = mid + 1;
+            }
+            const long long f = __shfl_sync(0xffffffffu, first, lo);
+            const int before = __shfl_sync(0xffffffffu, incl - c, lo);
+            bool mine = k < total;
+            unsigned long long key[4] = {0ull, 0ull, 0ull, 0ull};
+            if (mine) {
+                const long long row = f + (k - before);
+                const uint4 a = __ldg(digests + 2 * row), b = __ldg(digests + 2 * row + 1);
+                key[0] = u64_of(a.x, a.y); key[1] = u64_of(a.z, a.w);
+                key[2] = u64_of(b.x, b.y); key[3] = u64_of(b.z, b.w);
+                if (key_reserved(key)) {
+                    my_flags |= KVGOV_F_SENTINEL;
+                    mine = false;
+                }
+            }
+            const unsigned inserting = __ballot_sync(0xffffffffu, mine);
+            if (mine) count_insert(insert_warp_dedup(slots, mask, key, spin_limit, inserting), my_new, my_flags);
+        }
+    }
+    publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
+}
+
 }  // namespace
 
 extern "C" int kvgov_table_init(uint8_t *d_slots, uint64_t capacity, kvgov_stream_t stream) {
@@ -269,12 +345,21 @@ extern "C" int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const 
         return KVGOV_EINVAL;
     if (n_req == 0) return KVGOV_OK;
     if (!d_digests || !aligned16(d_digests) || !d_blk_off || !d_prefix_blocks) return KVGOV_EINVAL;
+#if KVGOV_INSERT_PACK
+    const long long warps = ((long long)n_req + kPackReq - 1) / kPackReq;
+    long long grid = (warps + (kInsertThreads / 32) - 1) / (kInsertThreads / 32);
+    if (grid > 152ll * 64) grid = 152ll * 64;
+    insert_uncached_packed_kernel<<<(unsigned)grid, kInsertThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+        reinterpret_cast<unsigned long long *>(d_slots), capacity - 1, reinterpret_cast<const uint4 *>(d_digests),
+        d_blk_off, n_req, d_prefix_blocks, d_n_new, d_status, g_spin_limit.load());
+#else
     constexpr int G = 8;
     long long grid = ((long long)n_req * G + kInsertThreads - 1) / kInsertThreads;
     if (grid > 152ll * 64) grid = 152ll * 64;
     insert_uncached_kernel<G><<<(unsigned)grid, kInsertThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
         reinterpret_cast<unsigned long long *>(d_slots), capacity - 1, reinterpret_cast<const uint4 *>(d_digests),
         d_blk_off, n_req, d_prefix_blocks, d_n_new, d_status, g_spin_limit.load());
+#endif
     return kvgov_host::launch_status();
 }
 

@@ -11,7 +11,7 @@ KVGOV_CHAIN_R=64|128|256, KVGOV_FMA_ADDS=0|1): kvgov_chain_hash is timed on
 three workload shapes (15 launches each, CUDA events, median) and every
 variant's digests must equal the first variant's, byte for byte.
 
-Insert mode (flags KVGOV_INSERT_LOOK=0|1, KVGOV_INSERT_DEDUP=0|1): 80 serving
+Insert mode (flags KVGOV_INSERT_LOOK, _DEDUP, _PACK, _ST16 = 0|1): 80 serving
 steps of the wide batch (131,072 x 128 tokens, BOUNDARY at token 64) against
 a 2^25-slot table under a new secret epoch per step, flushed before a step
 would take it past load factor 0.5; CUDA events around every kernel.  Reports
@@ -39,7 +39,7 @@ DEFAULT = ["compact128:-DKVGOV_COMPACT_ROUNDS=1 -DKVGOV_CHAIN_R=128",
            "compact256:-DKVGOV_COMPACT_ROUNDS=1 -DKVGOV_CHAIN_R=256",
            "unroll256:-DKVGOV_COMPACT_ROUNDS=0 -DKVGOV_CHAIN_R=256",
            "unroll128_imad:-DKVGOV_COMPACT_ROUNDS=0 -DKVGOV_FMA_ADDS=1"]
-SOURCES = ["kvgov_chain.cu", "kvgov_salts.cu", "kvgov_table.cu"]
+SOURCES = kbuild.LIBS[kbuild.LIB]
 
 
 def build_variant(name: str, flags: list[str]) -> str:
@@ -59,10 +59,12 @@ def build_variant(name: str, flags: list[str]) -> str:
     return lib
 
 
-INSERT_DEFAULT = ["look1_dedup1:-DKVGOV_INSERT_LOOK=1 -DKVGOV_INSERT_DEDUP=1",
-                  "look0_dedup0:-DKVGOV_INSERT_LOOK=0 -DKVGOV_INSERT_DEDUP=0",
-                  "look1_dedup0:-DKVGOV_INSERT_LOOK=1 -DKVGOV_INSERT_DEDUP=0",
-                  "look0_dedup1:-DKVGOV_INSERT_LOOK=0 -DKVGOV_INSERT_DEDUP=1"]
+INSERT_DEFAULT = ["st16_pack1:-DKVGOV_INSERT_ST16=1 -DKVGOV_INSERT_PACK=1",
+                  "st8_pack1:-DKVGOV_INSERT_ST16=0 -DKVGOV_INSERT_PACK=1",
+                  "st16_pack0:-DKVGOV_INSERT_ST16=1 -DKVGOV_INSERT_PACK=0",
+                  "st8_pack0:-DKVGOV_INSERT_ST16=0 -DKVGOV_INSERT_PACK=0",
+                  "st16_pack1_dedup1:-DKVGOV_INSERT_ST16=1 -DKVGOV_INSERT_PACK=1 -DKVGOV_INSERT_DEDUP=1",
+                  "st16_pack1_look0:-DKVGOV_INSERT_ST16=1 -DKVGOV_INSERT_PACK=1 -DKVGOV_INSERT_LOOK=0"]
 
 
 def _bind(L):
