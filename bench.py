@@ -247,6 +247,32 @@ def measure_gather(torch, peak_lib_path, table: "torch.Tensor", n_reads: int = 1
     return out
 
 
+def measure_slot_ops(torch, peak_lib_path, table: "torch.Tensor", n_ops: int) -> dict:
+    """Random-slot claims per second (best of 5) on `table`, zeroed before
+    each run: 128-bit CAS; CAS + 16-byte store; 16-byte read + CAS + store."""
+    import ctypes
+    L = ctypes.CDLL(peak_lib_path)
+    L.kvgov_peak_slot_ops.argtypes = [ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int, ctypes.c_int64,
+                                      ctypes.c_uint64, ctypes.c_void_p, ctypes.c_void_p]
+    sink = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = {"table_bytes": table.numel() * table.element_size(), "ops": n_ops}
+    for kind, name in ((0, "cas"), (1, "cas_store"), (2, "read_cas_store")):
+        best = float("inf")
+        for rep in range(6):
+            table.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            rc = L.kvgov_peak_slot_ops(table.data_ptr(), table.shape[0], kind, n_ops, 777 + rep, sink.data_ptr(),
+                                       torch.cuda.current_stream().cuda_stream)
+            b.record()
+            assert rc == 0, rc
+            b.synchronize()
+            if rep:
+                best = min(best, a.elapsed_time(b))
+        out[f"{name}_per_s"] = n_ops / (best / 1e3)
+    return out
+
+
 # --------------------------------------------------------------------------- reference arm
 def epoch_secret(base: bytes, step: int) -> bytes:
     """The server secret of step `step` (an input of the step, not a hash)."""
@@ -506,6 +532,7 @@ def main():
                 "traffic_source": traffic_src}
     # the table kernel of the step (insert of the uncached blocks) against HBM and a random-read ceiling
     gather = measure_gather(torch, kbuild.PEAK_LIB, cache.slots)
+    claims = measure_slot_ops(torch, kbuild.PEAK_LIB, cache.slots, int(inserted_per_step))
     ins_bytes = 96 * inserted_per_step + 20 * n_req
     ins_gbs = ins_bytes / (insert_ms / 1e3) / 1e9
     table_roofline = {
@@ -518,7 +545,10 @@ def main():
         "inserts_per_s": inserted_per_step / (insert_ms / 1e3),
         "algorithmic_bytes_per_launch": ins_bytes,
         "bytes_basis": "per new key 32 B read + one 32 B slot read + 32 B written; per request 4 B prefix + 16 B offsets",
-        "random_read_microbench": gather}
+        "random_read_microbench": gather,
+        "claim_ceiling_per_s": claims["read_cas_store_per_s"],
+        "frac_of_claim_ceiling": (inserted_per_step / (insert_ms / 1e3)) / claims["read_cas_store_per_s"],
+        "slot_op_microbench": claims}
     if clock.get("sm_mhz"):
         roofline["frac_at_run_clock"] = achieved / (n_sm * INT32_LANES_PER_SM * clock["sm_mhz"] * 1e6 / 1e12)
 

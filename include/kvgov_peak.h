@@ -48,6 +48,20 @@ int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint32_t *d_sin
 int kvgov_peak_gather(const void *d_table, uint64_t n_slots, int slot_bytes, int64_t n_reads, uint64_t seed,
                       uint32_t *d_sink, kvgov_stream_t stream);
 
+/*
+ * kvgov_peak_slot_ops -- the write side of that ceiling: `n_ops` operations
+ * on pseudo-random 32-byte slots (slot of op i = splitmix64(seed + i) mod
+ * n_slots) of a table that must be zero: kind 0 a 128-bit compare-and-swap
+ * of the slot's first 16 bytes from zero; kind 1 that CAS and a 16-byte
+ * store of the second half (an insert's claim of a new key); kind 2 a
+ * 16-byte read of the first half before them (the insert's look first).
+ *   d_table  [n_slots][32] bytes, device, 16-byte aligned, zeroed; modified.
+ * Asynchronous on `stream`.  Returns 0, 1 for a bad argument (nothing
+ * launched), 2 for a launch error.
+ */
+int kvgov_peak_slot_ops(void *d_table, uint64_t n_slots, int kind, int64_t n_ops, uint64_t seed, uint32_t *d_sink,
+                        kvgov_stream_t stream);
+
 /* Thread-operations one thread executes per iteration of `kind` (nominal
  * SHA-256 count of 1384 per compression for kinds 3 and 4), or 0 for a bad
  * kind. */
