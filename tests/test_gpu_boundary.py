@@ -44,9 +44,13 @@ def random_case(seed, n_req, n_tpl, max_tpl=3000, max_tail=2000):
     return toks, tok_off, np.array(ids, np.int32), tt, tpl_off
 
 
-@pytest.mark.parametrize("n_req,n_tpl", [(1, 1), (50, 0), (700, 3), (5000, 8)])
+@pytest.mark.parametrize("n_req,n_tpl", [(1, 1), (50, 0), (700, 3), (5000, 8), (40000, 4)])
 def test_boundary_matches_oracle(kv, n_req, n_tpl):
-    toks, tok_off, ids, tt, tpl_off = random_case(n_req * 7 + n_tpl, n_req, n_tpl)
+    """Random batches with every id kind; 40,000 requests take the
+    four-requests-per-warp layout."""
+    big = n_req >= 32 * 1024
+    toks, tok_off, ids, tt, tpl_off = random_case(n_req * 7 + n_tpl, n_req, n_tpl, max_tpl=300 if big else 3000,
+                                                  max_tail=100 if big else 2000)
     got, st = gpu_boundary(kv, toks, tok_off, ids, tt, tpl_off)
     want, flag = oracle.divergence_boundary(toks, tok_off, ids, tt, tpl_off)
     assert st == 0 and not flag
