@@ -119,8 +119,9 @@ __device__ __forceinline__ float rcp_approx(float x) {
 }
 
 // One problem solved by one thread, its values x[0..n) in shared memory.
-// Each value is replaced by its reciprocal (0 for a tenant that is not
-// usable) and then by p_i: the steps compare lambda * (1 / v_i) with 1 and
+// Each value is replaced by its reciprocal (+infinity for a tenant that is
+// not usable, which then never counts as above the level and gets p = 0)
+// and then by p_i: the steps compare lambda * (1 / v_i) with 1 and
 // sum reciprocals, with no division per tenant, and
 // p_i = 1 - lambda * (1 / v_i).  The adversary's payoff is lambda whenever a
 // tenant is usable (min(v_i, lambda) over the usable ones, the others at most
@@ -129,7 +130,7 @@ __device__ __forceinline__ void solve_thread(float *x, const float *__restrict__
                                              float *__restrict__ lambda_out, float *__restrict__ utility_out,
                                              uint32_t *status) {
     int npos = 0, nbad = 0;
-    float vmax = 0.0f;
+    float vmax = 0.0f, sum_all = 0.0f;       // the first Newton step's sum: every usable tenant
 #pragma unroll 4
     for (int i = 0; i < n; ++i) {
         const float xi = x[i];
@@ -137,7 +138,9 @@ __device__ __forceinline__ void solve_thread(float *x, const float *__restrict__
         npos += use;
         nbad += !use && !(xi <= 0.0f);
         vmax = use ? fmaxf(vmax, xi) : vmax;
-        x[i] = use ? rcp_approx(xi) : 0.0f;
+        const float r = use ? rcp_approx(xi) : __int_as_float(0x7f800000);   // +infinity: never above the level
+        sum_all += use ? r : 0.0f;
+        x[i] = r;
     }
     float K = K_in;
     const bool bad = nbad > 0 || !(K >= 0.0f);
@@ -149,15 +152,15 @@ __device__ __forceinline__ void solve_thread(float *x, const float *__restrict__
     } else if (K >= (float)npos) {
         lam = 0.0f;
     } else {
-        lam = 0.0f;
-        int prev_m = -1;
-        for (int step = 0; step <= npos + 1; ++step) {
+        lam = ((float)npos - K) / sum_all;            // the first step, from lambda = 0
+        int prev_m = npos;
+        for (int step = 0; step <= npos; ++step) {
             float sum = 0.0f;
             int m = 0;
 #pragma unroll 4
             for (int i = 0; i < n; ++i) {
                 const float r = x[i];
-                const bool on = r > 0.0f && lam * r < 1.0f;
+                const bool on = lam * r < 1.0f;               // false for r = +inf (inf or NaN product)
                 sum += on ? r : 0.0f;
                 m += on;
             }
@@ -168,10 +171,7 @@ __device__ __forceinline__ void solve_thread(float *x, const float *__restrict__
         }
     }
 #pragma unroll 4
-    for (int i = 0; i < n; ++i) {
-        const float r = x[i];
-        x[i] = r > 0.0f ? fmaxf(0.0f, 1.0f - lam * r) : 0.0f;
-    }
+    for (int i = 0; i < n; ++i) x[i] = fmaxf(0.0f, 1.0f - lam * x[i]);   // 0 for r = +inf (-inf or NaN)
     float u = lam;
     if (npos == 0) {                      // no usable tenant: the largest value (read again), or 0 if none
         u = n > 0 ? -3.0e38f : 0.0f;
