@@ -342,7 +342,7 @@ int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_
  * table is created; it stays valid across kvgov_table_init as long as
  * positions only grow: every call's seq_base must be at least the previous
  * call's seq_base + blk_off[n_req] (on the same owner array).  seq_base lies
- * in [1, 2^62].  capacity: a power of two in [32, 2^31].
+ * in [1, 2^62].  capacity: a power of two in [32, 2^30].
  */
 
 /*

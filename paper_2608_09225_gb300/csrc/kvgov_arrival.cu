@@ -19,15 +19,19 @@
 // in an earlier request has a smaller position than every block of r.
 //
 //   insert_arrival_kernel  one thread per block: inserts its key (the insert
-//                          protocol of kvgov_table.cu), records the slot that
-//                          holds it in slot_of, and marks the slots it claims
-//                          (keys new to the table) kPending.
-//   owner_min_kernel       after every claim, one thread per block: an atomic
-//                          min of its slot's owner with its position.  It
-//                          moves only kPending slots (any other owner belongs
-//                          to an earlier batch or to no arrival, so it is
-//                          smaller), which end at the first block that holds
-//                          their key.
+//                          protocol of kvgov_table.cu) and records the slot
+//                          that holds it in slot_of.  A block whose insert
+//                          claims a slot (a key new to the table) writes its own
+//                          position as the owner -- no other thread writes that
+//                          owner in this launch -- and marks its slot_of entry
+//                          settled.
+//   owner_min_kernel       after every claim, one thread per block: for each
+//                          block not marked, an atomic min of its slot's owner
+//                          with its position, which can only lower an owner
+//                          set in this batch (any other owner belongs to an
+//                          earlier batch or to no arrival, so it is smaller);
+//                          owners end at the first block that holds their key.
+//                          The marks are cleared.
 //   probe_arrival_kernel   after every min: block j of request r was cached
 //                          when r arrived iff its slot's owner is below the
 //                          position of r's first block.  The prefix ends at the
@@ -40,9 +44,8 @@ namespace {
 
 using namespace kvgov_dev;
 
-constexpr unsigned long long kPending = kOwnerPending;
-// Largest first position of a batch: positions stay below kPending for any
-// batch that fits in memory (2^62 blocks).
+// Largest first position of a batch (positions stay below 2^63 for any batch
+// that fits in memory).
 constexpr unsigned long long kMaxSeq = 1ull << 62;
 constexpr long long kNoRowCap = 0x7fffffffffffffffll;   // slot_of sized by the caller
 constexpr int kThreads = 256;
@@ -87,7 +90,7 @@ __global__ void __launch_bounds__(kThreads) insert_arrival_kernel(
     unsigned long long *__restrict__ slots, unsigned long long mask, unsigned long long *__restrict__ owner,
     const uint4 *__restrict__ digests, const int64_t *__restrict__ blk_off, int32_t n_req,
     uint32_t *__restrict__ slot_of, unsigned long long *n_new, uint32_t *status, uint32_t spin_limit,
-    long long row_cap) {
+    long long row_cap, unsigned long long seq_base) {
     __shared__ unsigned int s_new, s_flags, s_done;
     if (threadIdx.x == 0) { s_new = 0; s_flags = 0; s_done = 0; }
     __syncthreads();
@@ -108,14 +111,14 @@ __global__ void __launch_bounds__(kThreads) insert_arrival_kernel(
         unsigned long long pos = 0;
         const InsertResult res = insert_one(slots, mask, k, spin_limit, &pos);
         count_insert(res, my_new, my_flags);
-        if (res == kNew) owner[pos] = kPending;
-        slot_of[row] = (res == kNew || res == kDuplicate) ? (uint32_t)pos : kNoSlot;
+        if (res == kNew) owner[pos] = seq_base + (unsigned long long)row;   // settled: the first writer's position
+        slot_of[row] = res == kNew ? ((uint32_t)pos | kSettled) : (res == kDuplicate ? (uint32_t)pos : kNoSlot);
     }
     publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
 }
 
 __global__ void __launch_bounds__(kThreads) owner_min_kernel(const int64_t *__restrict__ blk_off, int32_t n_req,
-                                                             const uint32_t *__restrict__ slot_of,
+                                                             uint32_t *__restrict__ slot_of,
                                                              unsigned long long *__restrict__ owner,
                                                              unsigned long long seq_base, long long row_cap) {
     const long long n_rows = batch_rows(blk_off, n_req, nullptr, false, row_cap);
@@ -123,7 +126,11 @@ __global__ void __launch_bounds__(kThreads) owner_min_kernel(const int64_t *__re
     const int lane = threadIdx.x & 31;
     for (long long r0 = (long long)blockIdx.x * kThreads + (threadIdx.x & ~31); r0 < n_rows; r0 += stride) {
         const long long row = r0 + lane;                       // warp-uniform trip count
-        const uint32_t s = row < n_rows ? __ldg(slot_of + row) : kNoSlot;
+        uint32_t s = row < n_rows ? slot_of[row] : kNoSlot;
+        if (s != kNoSlot && (s & kSettled)) {                  // settled by the insert: clear the mark
+            slot_of[row] = s & ~kSettled;
+            s = kNoSlot;
+        }
         // Shared prefixes put one key in many rows: within a warp only the
         // lowest row of each slot takes part (rows ascend with the lane), and
         // it skips the atomic when the owner already holds an earlier
@@ -136,24 +143,47 @@ __global__ void __launch_bounds__(kThreads) owner_min_kernel(const int64_t *__re
 }
 
 // The same min with one thread per request walking its blocks, for batches
-// of many requests: the 32 lanes of a warp hold block j of 32 consecutive
-// requests, so one key shared by their prefixes is settled once per warp.
+// of many requests (after the fused chain insert): the 32 lanes of a warp
+// hold block j of 32 consecutive requests, so one key shared by their
+// prefixes is settled once per warp.  Eight blocks at a time: their slot
+// handles, then the owners of the slots this lane settles, then the atomics,
+// so that each group of eight costs two memory round trips rather than
+// sixteen.
 __global__ void __launch_bounds__(kThreads) owner_min_req_kernel(const int64_t *__restrict__ blk_off, int32_t n_req,
-                                                                 const uint32_t *__restrict__ slot_of,
+                                                                 uint32_t *__restrict__ slot_of,
                                                                  unsigned long long *__restrict__ owner,
                                                                  unsigned long long seq_base) {
+    constexpr int kGroup = 8;
     const long long r = (long long)blockIdx.x * kThreads + threadIdx.x;
     const int lane = threadIdx.x & 31;
     long long base, nb;
     unsigned ignored = 0;                         // the insert has flagged bad ranges
     request_range(blk_off, n_req, r, base, nb, ignored);
     const int jmax = __reduce_max_sync(0xffffffffu, (unsigned)nb);
-    for (int j = 0; j < jmax; ++j) {                           // warp-uniform
-        const uint32_t s = j < nb ? __ldg(slot_of + base + j) : kNoSlot;
-        const unsigned same = __match_any_sync(0xffffffffu, s);
-        if (s == kNoSlot || lane != __ffs(same) - 1) continue;   // the lowest lane has the earliest position
-        const unsigned long long p = seq_base + (unsigned long long)(base + j);
-        if (ld_relaxed(owner + s) > p) atomicMin(owner + s, p);
+    for (int j0 = 0; j0 < jmax; j0 += kGroup) {                // warp-uniform
+        uint32_t s[kGroup];
+#pragma unroll
+        for (int u = 0; u < kGroup; ++u) {
+            s[u] = j0 + u < nb ? slot_of[base + j0 + u] : kNoSlot;
+            if (s[u] != kNoSlot && (s[u] & kSettled)) {        // settled by the insert: clear the mark
+                slot_of[base + j0 + u] = s[u] & ~kSettled;
+                s[u] = kNoSlot;
+            }
+        }
+        bool lead[kGroup];
+#pragma unroll
+        for (int u = 0; u < kGroup; ++u) {
+            const unsigned same = __match_any_sync(0xffffffffu, s[u]);
+            lead[u] = s[u] != kNoSlot && lane == __ffs(same) - 1;   // the lowest lane: the earliest position
+        }
+        unsigned long long cur[kGroup];
+#pragma unroll
+        for (int u = 0; u < kGroup; ++u) cur[u] = lead[u] ? ld_relaxed(owner + s[u]) : 0ull;
+#pragma unroll
+        for (int u = 0; u < kGroup; ++u) {
+            const unsigned long long p = seq_base + (unsigned long long)(base + j0 + u);
+            if (lead[u] && cur[u] > p) atomicMin(owner + s[u], p);
+        }
     }
 }
 
@@ -215,9 +245,9 @@ unsigned request_grid(int32_t n_req) {
 // resident CTAs per SM strides over the blocks.
 unsigned row_grid() { return (unsigned)(kvgov_host::sm_count() * 8); }
 
-// Capacities whose slot index fits slot_of's u32 with kNoSlot to spare.
+// Capacities whose slot index fits slot_of's u32 below the kSettled mark.
 bool arrival_capacity(uint64_t capacity) {
-    return kvgov_host::pow2_capacity(capacity) && capacity <= (1ull << 31);
+    return kvgov_host::pow2_capacity(capacity) && capacity <= (1ull << 30);
 }
 
 // Scratch of kvgov_serve_arrival_static: the slot of each block of one batch,
@@ -245,7 +275,7 @@ namespace kvgov_host {
 
 // Owner min of a batch whose keys a fused chain kernel has inserted (one
 // thread per request; see owner_min_req_kernel).
-int arrival_owner_min_by_request(const int64_t *d_blk_off, int32_t n_req, const uint32_t *d_slot_of,
+int arrival_owner_min_by_request(const int64_t *d_blk_off, int32_t n_req, uint32_t *d_slot_of,
                                  uint64_t *d_owner, uint64_t seq_base, cudaStream_t stream) {
     const unsigned grid = (unsigned)(((long long)n_req + kThreads - 1) / kThreads);
     owner_min_req_kernel<<<grid, kThreads, 0, stream>>>(d_blk_off, n_req, d_slot_of,
@@ -285,7 +315,7 @@ extern "C" int kvgov_insert_arrival(uint8_t *d_slots, uint64_t *d_owner, uint64_
                                                     reinterpret_cast<unsigned long long *>(d_owner),
                                                     reinterpret_cast<const uint4 *>(d_digests), d_blk_off, n_req,
                                                     d_slot_of, d_n_new, d_status, kvgov_host::spin_limit(),
-                                                    kNoRowCap);
+                                                    kNoRowCap, seq_base);
     owner_min_kernel<<<grid, kThreads, 0, s>>>(d_blk_off, n_req, d_slot_of,
                                                reinterpret_cast<unsigned long long *>(d_owner), seq_base, kNoRowCap);
     return kvgov_host::launch_status();
@@ -323,7 +353,8 @@ extern "C" int kvgov_serve_arrival_static(uint8_t *d_slots, uint64_t *d_owner, u
     insert_arrival_kernel<<<grid, kThreads, 0, s>>>(reinterpret_cast<unsigned long long *>(d_slots), capacity - 1,
                                                     reinterpret_cast<unsigned long long *>(d_owner),
                                                     reinterpret_cast<const uint4 *>(d_digests), d_blk_off, n_req,
-                                                    slot_of, d_n_new, d_status, kvgov_host::spin_limit(), kStaticRows);
+                                                    slot_of, d_n_new, d_status, kvgov_host::spin_limit(), kStaticRows,
+                                                    seq_base);
     owner_min_kernel<<<grid, kThreads, 0, s>>>(d_blk_off, n_req, slot_of,
                                                reinterpret_cast<unsigned long long *>(d_owner), seq_base, kStaticRows);
     probe_arrival_kernel<<<request_grid(n_req), kThreads, 0, s>>>(reinterpret_cast<const unsigned long long *>(d_owner),

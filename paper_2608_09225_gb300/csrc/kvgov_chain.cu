@@ -79,6 +79,7 @@ struct ArrivalParams {
     unsigned long long *owner = nullptr;
     uint32_t *slot_of = nullptr;
     unsigned long long *n_new = nullptr;
+    unsigned long long seq_base = 0;
     uint32_t spin_limit = 0;
 };
 
@@ -257,15 +258,19 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
                 const int leader = __ffs(same) - 1;
                 unsigned long long pos = 0ull;
                 int res = kDuplicate;
-                if ((tid & 31) == leader) {
+                const bool lead = (tid & 31) == leader;
+                if (lead) {
                     res = insert_one(reinterpret_cast<unsigned long long *>(const_cast<uint4 *>(p.slots)), p.mask,
                                      ak, a.spin_limit, &pos);
                     count_insert(static_cast<InsertResult>(res), my_new, my_flags);
-                    if (res == kNew) a.owner[pos] = kOwnerPending;
+                    if (res == kNew) a.owner[pos] = a.seq_base + (unsigned long long)(row + j);
                 }
                 pos = __shfl_sync(inserting, pos, leader);
                 res = __shfl_sync(inserting, res, leader);
-                a.slot_of[row + j] = (res == kNew || res == kDuplicate) ? (uint32_t)pos : kNoSlot;
+                // settled (no owner min needed): the block that claimed the slot,
+                // and every block behind an earlier lane with the same key
+                const uint32_t mark = (res == kNew || !lead) ? kSettled : 0u;
+                a.slot_of[row + j] = (res == kNew || res == kDuplicate) ? ((uint32_t)pos | mark) : kNoSlot;
             }
             have = false;
         }
@@ -353,6 +358,7 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     a.owner = reinterpret_cast<unsigned long long *>(f.owner);
     a.slot_of = f.slot_of;
     a.n_new = f.n_new;
+    a.seq_base = f.seq_base;
     a.spin_limit = kvgov_host::spin_limit();
     const unsigned grid = (unsigned)(((long long)n_req + kR - 1) / kR);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

@@ -72,11 +72,11 @@ __device__ __forceinline__ void cas128(unsigned long long *p, unsigned long long
 
 enum InsertResult { kNew = 0, kDuplicate = 1, kFull = 2, kTimeout = 3 };
 
-// Arrival-order serving (kvgov_arrival.cu): the owner of a slot claimed by
-// the running insert, and the slot_of entry of a block whose key is not in
-// the table.
-constexpr unsigned long long kOwnerPending = ~0ull;
+// Arrival-order serving (kvgov_arrival.cu): the slot_of entry of a block
+// whose key is not in the table, and the mark the insert sets on a block
+// whose owner it has already settled (the owner min clears it).
 constexpr uint32_t kNoSlot = 0xffffffffu;
+constexpr uint32_t kSettled = 0x80000000u;
 
 // Insert the key k (w0..w3) with the protocol described in kvgov_table.cu.
 // On kNew and kDuplicate, *pos receives the slot that holds the key.

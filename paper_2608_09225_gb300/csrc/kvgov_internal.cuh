@@ -33,7 +33,7 @@ inline bool pow2_capacity(uint64_t cap) { return cap >= KVGOV_MIN_CAPACITY && (c
 uint32_t spin_limit();
 
 // Arrival-order serving helpers (kvgov_arrival.cu).
-int arrival_owner_min_by_request(const int64_t *d_blk_off, int32_t n_req, const uint32_t *d_slot_of,
+int arrival_owner_min_by_request(const int64_t *d_blk_off, int32_t n_req, uint32_t *d_slot_of,
                                  uint64_t *d_owner, uint64_t seq_base, cudaStream_t stream);
 bool arrival_args_ok(uint64_t capacity, uint64_t seq_base);
 
