@@ -239,7 +239,7 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             const uint4 q1 = make_uint4(bswap32(h[4]), bswap32(h[5]), bswap32(h[6]), bswap32(h[7]));
             dst[0] = q0;
             dst[1] = q1;
-            if (FUSE == kFuseProbe && hits == j && lookup<false>(p.slots, p.mask, q0, q1)) hits = j + 1;
+            if (FUSE == kFuseProbe && hits == j && lookup(p.slots, p.mask, q0, q1)) hits = j + 1;
             if (FUSE == kFuseArrival) {
                 ak[0] = u64_of(q0.x, q0.y); ak[1] = u64_of(q0.z, q0.w);
                 ak[2] = u64_of(q1.x, q1.y); ak[3] = u64_of(q1.z, q1.w);

@@ -1,6 +1,6 @@
 // kvgov_lookup.cuh -- read-only lookup of a 32-byte key in the prefix-cache
 // table (slot encoding and probe window as described in kvgov_table.cu and
-// include/kvgov.h), shared by the probe kernel and the fused chain + probe
+// include/kvgov.h), shared by the probe kernels and the fused chain + probe
 // kernel.  The table must not change while a lookup runs.
 #pragma once
 #include <cstdint>
@@ -19,12 +19,9 @@ __device__ __forceinline__ unsigned long long probe_window(unsigned long long ma
 }
 
 // Is the key q0 || q1 (bytes 0-15, 16-31, as stored) in the table?  Slots are
-// read through the read-only path.  WHOLE_SLOT reads both halves of a slot at
-// once (one memory round trip per slot: the probe kernel, whose warps wait on
-// their lookups); otherwise the second half is read only when the first
-// matches (fewer loads: the fused chain kernel, whose lookups hide behind
-// other warps' hashing).
-template <bool WHOLE_SLOT>
+// read through the read-only path, the second half of a slot only when the
+// first matches (fewer loads: the fused chain kernel, whose lookups hide
+// behind other warps' hashing).
 __device__ __forceinline__ bool lookup(const uint4 *__restrict__ slots, unsigned long long mask, uint4 q0, uint4 q1) {
     const unsigned long long k0 = u64_of(q0.x, q0.y), k1 = u64_of(q0.z, q0.w);
     if ((k0 | k1) == 0ull || u64_of(q1.x, q1.y) == 0ull || u64_of(q1.z, q1.w) == 0ull)
@@ -33,15 +30,41 @@ __device__ __forceinline__ bool lookup(const uint4 *__restrict__ slots, unsigned
     unsigned long long pos = k0 & mask;
     for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
         const uint4 a = __ldg(slots + 2 * pos);
-        uint4 b;
-        if (WHOLE_SLOT) b = __ldg(slots + 2 * pos + 1);
         if ((a.x | a.y | a.z | a.w) == 0u) return false;   // empty slot ends the walk
         if (a.x == q0.x && a.y == q0.y && a.z == q0.z && a.w == q0.w) {
-            if (!WHOLE_SLOT) b = __ldg(slots + 2 * pos + 1);
+            const uint4 b = __ldg(slots + 2 * pos + 1);
             if (b.x == q1.x && b.y == q1.y && b.z == q1.z && b.w == q1.w) return true;
         }
     }
     return false;
+}
+
+// The home slot of the key q0 || q1.
+__device__ __forceinline__ unsigned long long home_slot(uint4 q0, unsigned long long mask) {
+    return u64_of(q0.x, q0.y) & mask;
+}
+
+// lookup() whose first slot, the key's home slot (both halves a, b), the
+// caller has read already: the probe kernels issue the home-slot loads of
+// several keys together and finish each walk after.  Same result as
+// lookup().
+__device__ __forceinline__ bool lookup_from_home(const uint4 *__restrict__ slots, unsigned long long mask, uint4 q0,
+                                                 uint4 q1, uint4 a, uint4 b) {
+    if ((u64_of(q0.x, q0.y) | u64_of(q0.z, q0.w)) == 0ull || u64_of(q1.x, q1.y) == 0ull ||
+        u64_of(q1.z, q1.w) == 0ull)
+        return false;                               // reserved keys are never stored
+    const unsigned long long window = probe_window(mask);
+    unsigned long long pos = home_slot(q0, mask);
+    for (unsigned long long n = 1;; ++n) {
+        if ((a.x | a.y | a.z | a.w) == 0u) return false;   // empty slot ends the walk
+        if (a.x == q0.x && a.y == q0.y && a.z == q0.z && a.w == q0.w && b.x == q1.x && b.y == q1.y &&
+            b.z == q1.z && b.w == q1.w)
+            return true;
+        if (n == window) return false;
+        pos = (pos + 1) & mask;
+        a = __ldg(slots + 2 * pos);
+        b = __ldg(slots + 2 * pos + 1);
+    }
 }
 
 }  // namespace kvgov_dev

@@ -33,12 +33,16 @@
 // Insert of a probed batch (kvgov_insert_uncached): only the blocks at and
 // after each request's first miss, with the same per-key protocol.
 //
-// Probe: G lanes of a warp serve one request.  The lanes look up the next G
-// consecutive blocks in parallel; a ballot over the window's misses gives the
-// first miss (the prefix length) and ends the request, else the window moves
-// on.  A request of n_b blocks takes ceil((L+1)/G) rounds of two dependent
-// memory accesses (digest, slot); lookups past the first miss inside the last
-// window are wasted, which costs bandwidth but not latency.
+// Probe: a request's prefix length is its first block not found.  G lanes
+// of a warp serve one request and look up a window of its next blocks in
+// parallel; a ballot over the window's misses gives the first miss, else the
+// window moves on (probe_seg_kernel).  The layout depends on the batch size:
+// batches of many requests take 4 lanes per request and a first window of
+// one block (most requests of a batch of fresh prompts miss there), then 4;
+// mid-size batches 16 lanes, windows of 16 then 32; few requests a warp each,
+// windows of 32, 64, then 128 blocks, so that a long cached prefix takes few
+// rounds.  Lookups past the first miss inside a window are wasted: they cost
+// bandwidth but not latency.
 #include <atomic>
 
 #include "kvgov_internal.cuh"
@@ -122,49 +126,118 @@ __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long lo
 
 // ---------------------------------------------------------------------------
 constexpr int kProbeThreads = 256;
+// Probe layouts, by batch size (build options, measured side by side by
+// variants.py --probe): probe_seg_kernel<G, kPer> with first window F for
+//   n_req >= KVGOV_PROBE_MANY_MIN                  (MANY_G, MANY_PER, MANY_FIRST)
+//   KVGOV_PROBE_MID_MIN <= n_req < ..._MANY_MIN     (MID_G, MID_PER, MID_FIRST)
+//   n_req < KVGOV_PROBE_MID_MIN                     (FEW_G, FEW_PER, FEW_FIRST)
+#ifndef KVGOV_PROBE_MANY_MIN
+#define KVGOV_PROBE_MANY_MIN 32768
+#endif
+#ifndef KVGOV_PROBE_MID_MIN
+#define KVGOV_PROBE_MID_MIN 2048
+#endif
+#ifndef KVGOV_PROBE_MANY_G
+#define KVGOV_PROBE_MANY_G 4
+#endif
+#ifndef KVGOV_PROBE_MANY_PER
+#define KVGOV_PROBE_MANY_PER 1
+#endif
+#ifndef KVGOV_PROBE_MANY_FIRST
+#define KVGOV_PROBE_MANY_FIRST 1
+#endif
+#ifndef KVGOV_PROBE_MID_G
+#define KVGOV_PROBE_MID_G 16
+#endif
+#ifndef KVGOV_PROBE_MID_PER
+#define KVGOV_PROBE_MID_PER 2
+#endif
+#ifndef KVGOV_PROBE_MID_FIRST
+#define KVGOV_PROBE_MID_FIRST 16
+#endif
+#ifndef KVGOV_PROBE_FEW_G
+#define KVGOV_PROBE_FEW_G 32
+#endif
+#ifndef KVGOV_PROBE_FEW_PER
+#define KVGOV_PROBE_FEW_PER 4
+#endif
+#ifndef KVGOV_PROBE_FEW_FIRST
+#define KVGOV_PROBE_FEW_FIRST 32
+#endif
 
-template <int G>
-__global__ void __launch_bounds__(kProbeThreads) probe_kernel(const uint4 *__restrict__ slots, unsigned long long mask,
-                                                              const uint4 *__restrict__ digests,
-                                                              const int64_t *__restrict__ blk_off, int32_t n_req,
-                                                              int32_t *__restrict__ prefix_blocks, uint32_t *status) {
+// Request r's block range; a malformed one is flagged and counts as empty.
+__device__ __forceinline__ void probe_range(const int64_t *__restrict__ blk_off, int32_t n_req, long long r,
+                                            long long &base, long long &nb, uint32_t *status) {
+    base = blk_off[r];
+    nb = blk_off[r + 1] - base;
+    if (nb < 0 || base < 0 || base + nb > blk_off[n_req]) {
+        raise_flag(status, KVGOV_F_BADINDEX);
+        nb = 0;
+    }
+}
+
+// G lanes per request (32 / G requests per warp).  A request's first round
+// looks up its first `first` blocks; later rounds G, 2G, 4G ... blocks up to
+// G * kPer (kPer lookups per lane, their home slots read together so that
+// their memory accesses overlap).  A small first window wastes few lookups
+// on a request that misses early; the growing windows take a long cached
+// prefix in few rounds.
+template <int G, int kPer>
+__global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *__restrict__ slots,
+                                                                  unsigned long long mask,
+                                                                  const uint4 *__restrict__ digests,
+                                                                  const int64_t *__restrict__ blk_off,
+                                                                  int32_t n_req, int32_t *__restrict__ prefix_blocks,
+                                                                  uint32_t *status, int first) {
     constexpr int kSegs = 32 / G;
     constexpr unsigned kSegMask = G == 32 ? 0xffffffffu : ((1u << G) - 1u);
     const int lane = threadIdx.x & 31, seg = lane / G, sl = lane % G;
     const long long warps_total = (long long)gridDim.x * (kProbeThreads / 32);
     for (long long wg = ((long long)blockIdx.x * kProbeThreads + threadIdx.x) / 32; wg * kSegs < n_req;
-         wg += warps_total) {
+         wg += warps_total) {                                  // warp-uniform
         const long long r = wg * kSegs + seg;
         long long base = 0, nb = 0;
-        bool active = false;
-        if (r < n_req) {
-            base = blk_off[r];
-            nb = blk_off[r + 1] - base;
-            if (nb < 0 || base < 0 || base + nb > blk_off[n_req]) {
-                if (sl == 0) raise_flag(status, KVGOV_F_BADINDEX);
-                nb = 0;
-            }
-            active = nb > 0;
-        }
+        if (r < n_req) probe_range(blk_off, n_req, r, base, nb, sl == 0 ? status : nullptr);
         long long L = 0;
-        const int win = G;
+        int w = first;
+        bool active = nb > 0;
         while (__any_sync(0xffffffffu, active)) {
-            const long long j = L + sl;
-            const bool mine = active && sl < win && j < nb;
-            bool miss = false;
-            if (mine) {
-                const uint4 *q = digests + 2 * (base + j);
-                miss = !lookup<true>(slots, mask, __ldg(q), __ldg(q + 1));
+            uint4 q0[kPer], q1[kPer], a[kPer], b[kPer];
+#pragma unroll
+            for (int u = 0; u < kPer; ++u) {
+                const int o = sl + G * u;
+                if (active && o < w && L + o < nb) {
+                    q0[u] = __ldg(digests + 2 * (base + L + o));
+                    q1[u] = __ldg(digests + 2 * (base + L + o) + 1);
+                }
             }
-            const unsigned seg_miss = (__ballot_sync(0xffffffffu, miss) >> (seg * G)) & kSegMask;
+#pragma unroll
+            for (int u = 0; u < kPer; ++u) {
+                const int o = sl + G * u;
+                if (active && o < w && L + o < nb) {
+                    const unsigned long long h = home_slot(q0[u], mask);
+                    a[u] = __ldg(slots + 2 * h);
+                    b[u] = __ldg(slots + 2 * h + 1);
+                }
+            }
+            int miss_at = -1;                                  // the window's first miss (per segment)
+#pragma unroll
+            for (int u = 0; u < kPer; ++u) {
+                const int o = sl + G * u;
+                const bool miss = active && o < w && L + o < nb && !lookup_from_home(slots, mask, q0[u], q1[u],
+                                                                                     a[u], b[u]);
+                const unsigned m = (__ballot_sync(0xffffffffu, miss) >> (seg * G)) & kSegMask;
+                if (m && miss_at < 0) miss_at = G * u + __ffs((int)m) - 1;
+            }
             if (active) {
-                if (seg_miss) {
-                    L += __ffs((int)seg_miss) - 1;
+                if (miss_at >= 0) {
+                    L += miss_at;
                     active = false;
                 } else {
-                    L += (nb - L < win) ? (nb - L) : win;
+                    L += (nb - L < w) ? (nb - L) : w;
                     if (L >= nb) active = false;
                 }
+                w = w < G ? G : (2 * w < G * kPer ? 2 * w : G * kPer);
             }
         }
         if (r < n_req && sl == 0) prefix_blocks[r] = (int32_t)L;
@@ -293,6 +366,15 @@ __global__ void __launch_bounds__(kInsertThreads) insert_uncached_packed_kernel(
     publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
 }
 
+// G lanes per request: 32 / G requests per warp, at most 64 CTAs per SM.
+unsigned probe_grid(int32_t n_req, int G) {
+    const long long per_warp = 32 / G;
+    const long long warps = ((long long)n_req + per_warp - 1) / per_warp;
+    long long grid = (warps + (kProbeThreads / 32) - 1) / (kProbeThreads / 32);
+    const long long cap = (long long)kvgov_host::sm_count() * 64;
+    return (unsigned)(grid < cap ? grid : cap);
+}
+
 }  // namespace
 
 extern "C" int kvgov_table_init(uint8_t *d_slots, uint64_t capacity, kvgov_stream_t stream) {
@@ -327,13 +409,20 @@ extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint
     if (!d_slots || !aligned16(d_slots) || !kvgov_host::pow2_capacity(capacity) || n_req < 0) return KVGOV_EINVAL;
     if (n_req == 0) return KVGOV_OK;
     if (!d_digests || !aligned16(d_digests) || !d_blk_off || !d_prefix_blocks) return KVGOV_EINVAL;
-    constexpr int G = 8;
-    const long long warps = ((long long)n_req + (32 / G) - 1) / (32 / G);
-    long long grid = (warps + (kProbeThreads / 32) - 1) / (kProbeThreads / 32);
-    if (grid > 152ll * 64) grid = 152ll * 64;
-    probe_kernel<G><<<(unsigned)grid, kProbeThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-        reinterpret_cast<const uint4 *>(d_slots), capacity - 1, reinterpret_cast<const uint4 *>(d_digests), d_blk_off,
-        n_req, d_prefix_blocks, d_status);
+    const uint4 *slots = reinterpret_cast<const uint4 *>(d_slots), *dig = reinterpret_cast<const uint4 *>(d_digests);
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (n_req >= KVGOV_PROBE_MANY_MIN)
+        probe_seg_kernel<KVGOV_PROBE_MANY_G, KVGOV_PROBE_MANY_PER>
+            <<<probe_grid(n_req, KVGOV_PROBE_MANY_G), kProbeThreads, 0, s>>>(
+                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, KVGOV_PROBE_MANY_FIRST);
+    else if (n_req >= KVGOV_PROBE_MID_MIN)
+        probe_seg_kernel<KVGOV_PROBE_MID_G, KVGOV_PROBE_MID_PER>
+            <<<probe_grid(n_req, KVGOV_PROBE_MID_G), kProbeThreads, 0, s>>>(
+                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, KVGOV_PROBE_MID_FIRST);
+    else
+        probe_seg_kernel<KVGOV_PROBE_FEW_G, KVGOV_PROBE_FEW_PER>
+            <<<probe_grid(n_req, KVGOV_PROBE_FEW_G), kProbeThreads, 0, s>>>(
+                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, KVGOV_PROBE_FEW_FIRST);
     return kvgov_host::launch_status();
 }
 

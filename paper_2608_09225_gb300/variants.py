@@ -2,6 +2,7 @@
 
     python -m paper_2608_09225_gb300.variants [name:flags ...]
     python -m paper_2608_09225_gb300.variants --insert [name:flags ...]
+    python -m paper_2608_09225_gb300.variants --probe [name:flags ...]
 
 Each variant is the library compiled with extra nvcc -D flags into
 _build/variants/<name>/libkvgov.so.
@@ -18,6 +19,13 @@ would take it past load factor 0.5; CUDA events around every kernel.  Reports
 the median steady-state insert, the insert of the first step after a flush
 (where every request's shared-prefix blocks are new, a hot key), probe and
 step times; the number of keys inserted must equal the closed form.
+
+Probe mode (flags KVGOV_PROBE_{MANY,MID,FEW}_{G,PER,FIRST}, _MANY_MIN,
+_MID_MIN): kvgov_probe on every workload's probed requests against its table
+as bench.py --configs fills it, plus two mid-size batches (all 8192 template
+requests, the first 16,384 probe-heavy requests); mean of 20 back-to-back
+launches queued behind a GPU spin.  Every variant's prefix lengths must
+equal the first variant's.
 
 Prints one JSON line per variant.  Needs a GPU.
 """
@@ -147,10 +155,103 @@ def insert_mode(specs):
     return 0
 
 
+PROBE_DEFAULT = [
+    "default:",
+    "many_8x1_first8:-DKVGOV_PROBE_MANY_G=8 -DKVGOV_PROBE_MANY_FIRST=8",
+    "many_8x1_first1:-DKVGOV_PROBE_MANY_G=8",
+    "many_2x1_first1:-DKVGOV_PROBE_MANY_G=2",
+    "many_4x1_first2:-DKVGOV_PROBE_MANY_FIRST=2",
+    "many_4x1_first4:-DKVGOV_PROBE_MANY_FIRST=4",
+    "mid_4x1_first1:-DKVGOV_PROBE_MID_G=4 -DKVGOV_PROBE_MID_PER=1 -DKVGOV_PROBE_MID_FIRST=1",
+    "mid_4x2_first1:-DKVGOV_PROBE_MID_G=4 -DKVGOV_PROBE_MID_PER=2 -DKVGOV_PROBE_MID_FIRST=1",
+    "mid_4x1_first4:-DKVGOV_PROBE_MID_G=4 -DKVGOV_PROBE_MID_PER=1 -DKVGOV_PROBE_MID_FIRST=4",
+    "mid_8x2_first1:-DKVGOV_PROBE_MID_G=8 -DKVGOV_PROBE_MID_PER=2 -DKVGOV_PROBE_MID_FIRST=1",
+    "mid_16x2_first1:-DKVGOV_PROBE_MID_FIRST=1",
+    "mid_8x1_first8:-DKVGOV_PROBE_MID_G=8 -DKVGOV_PROBE_MID_PER=1 -DKVGOV_PROBE_MID_FIRST=8",
+    "few_warp32_first1:-DKVGOV_PROBE_FEW_FIRST=1",
+]
+
+
+def probe_cases(torch, seed=2030):
+    """Each workload's digests, table and probed range, made with the default
+    library (the fill of bench.py --configs)."""
+    from . import kvgov as K
+    from .pipeline import DeviceBatch, PrefixCache, next_pow2
+    tmpl = W.make("template")
+    cases = []
+    for name, mode, w in (("tiny", W.ROOT, W.make("tiny")), ("sysprompt", W.ROOT, W.make("sysprompt")),
+                          ("template_unsalted", W.UNSALTED, tmpl), ("template_root", W.ROOT, tmpl),
+                          ("probe", W.ROOT, W.make("probe")), ("long", W.BOUNDARY, W.make("long", seed=seed)),
+                          ("wide", W.BOUNDARY, W.make("wide", seed=seed + 1))):
+        b = w.batch
+        cap = w.capacity or next_pow2(4 * int((b.lengths() // 16).sum()))
+        cache = PrefixCache(cap, w.secret, w.ids, w.id_off)
+        db = DeviceBatch.from_host(b.tokens, b.tok_off, b.principal, b.boundary_tok)
+        blk, dig = cache.hash(mode, db)
+        blk_np = blk.cpu().numpy()
+        keys = []
+        if w.fill_from == "prior":
+            pdb = DeviceBatch.from_host(w.prior.tokens, w.prior.tok_off, w.prior.principal, w.prior.boundary_tok)
+            keys.append(cache.hash(mode, pdb)[1])
+        elif w.fill[1] > w.fill[0]:
+            keys.append(dig[blk_np[w.fill[0]]:blk_np[w.fill[1]]])
+        else:
+            keys.append(dig[: blk_np[b.n // 2]])
+        if w.random_keys is not None:
+            keys.append(torch.from_numpy(w.random_keys).cuda())
+        K.insert(cache.slots, torch.cat(keys), cache.status)
+        torch.cuda.synchronize()
+        cache.check_status()
+        p0, p1 = w.probe if w.probe[1] > w.probe[0] else (0, b.n)
+        cases.append(dict(name=name, slots=cache.slots, cap=cap, dig=dig, blk=blk[p0:p1 + 1], n=p1 - p0))
+        if name in ("template_root", "probe"):      # mid-size batches: every template request, 16,384 probes
+            q1 = b.n if name == "template_root" else 16384
+            cases.append(dict(name=name + f"_{q1}", slots=cache.slots, cap=cap, dig=dig, blk=blk[:q1 + 1], n=q1))
+    return cases
+
+
+def probe_mode(specs):
+    import torch
+    cases = probe_cases(torch)
+    stream = torch.cuda.current_stream().cuda_stream
+    ref = {}
+    for spec in specs:
+        name, _, flags = spec.partition(":")
+        L = _bind(ctypes.CDLL(build_variant(name, flags.split())))
+        res, same = {}, True
+        for c in cases:
+            pre = torch.full((c["n"],), -1, dtype=torch.int32, device="cuda")
+            st = torch.zeros(1, dtype=torch.int32, device="cuda")
+
+            def run():
+                assert L.kvgov_probe(c["slots"].data_ptr(), c["cap"], c["dig"].data_ptr(), c["blk"].data_ptr(),
+                                     c["n"], pre.data_ptr(), st.data_ptr(), stream) == 0
+
+            for _ in range(3):
+                run()
+            torch.cuda.synchronize()
+            a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda._sleep(4_000_000)
+            a.record()
+            for _ in range(20):
+                run()
+            e.record()
+            torch.cuda.synchronize()
+            res[c["name"]] = round(a.elapsed_time(e) / 20 * 1e3, 2)
+            got = pre.cpu().numpy()
+            same = same and int(st.item()) == 0 and (c["name"] not in ref or (got == ref[c["name"]]).all())
+            ref.setdefault(c["name"], got)
+        print(json.dumps({"variant": name, "flags": flags, "probe_us": res, "same_prefix_as_first": bool(same)}),
+              flush=True)
+    return 0
+
+
 def main(argv):
     import torch
     if argv and argv[0] == "--insert":
         return insert_mode(argv[1:] or INSERT_DEFAULT)
+    if argv and argv[0] == "--probe":
+        return probe_mode(argv[1:] or PROBE_DEFAULT)
     specs = argv or DEFAULT
     p = ctypes.c_void_p
     cases = []

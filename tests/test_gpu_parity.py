@@ -324,6 +324,76 @@ def test_probe_matches_oracle(kv, cap_log2):
     assert (pre.cpu().numpy() == ks.prefix_blocks(digests, off)).all()
 
 
+@pytest.mark.parametrize("n_req,max_nb,p_member", [(700, 400, 0.995), (3000, 70, 0.6), (40000, 40, 0.9),
+                                                    (40000, 3, 0.5), (70000, 300, 0.999)],
+                         ids=["warp_long", "warp_short", "queue", "queue_tiny_requests", "queue_long"])
+def test_probe_layouts_match_oracle(kv, n_req, max_nb, p_member):
+    """Both probe layouts (a warp per request below 32,768 requests, 32
+    requests per warp with a queue above), with requests of 0, 1 and 2
+    blocks, prefixes that span several rounds (up to 400 blocks), and
+    prefixes that end exactly at a round's edge."""
+    rng = np.random.default_rng(n_req + max_nb)
+    pool = keys_np(6000, n_req % 997 + 3)
+    nb = rng.integers(0, max_nb + 1, n_req)
+    nb[:8] = [0, 1, 2, 1, 0, max_nb, 33, 129][:8] if max_nb >= 129 else [0, 1, 2, 1, 0, max_nb, 0, 1]
+    off = np.concatenate([[0], np.cumsum(nb)]).astype(np.int64)
+    digests = pool[rng.integers(0, len(pool), int(off[-1]))]
+    member = rng.random(len(pool)) < p_member
+    # request 6 misses exactly at block 32 (the end of a warp's first round),
+    # request 7 at block 128, when they are that long
+    for r, j in ((6, 32), (7, 128)):
+        if nb[r] > j:
+            digests[off[r]:off[r] + j] = pool[np.nonzero(member)[0][:j]]
+            digests[off[r] + j] = pool[np.nonzero(~member)[0][0]]
+    slots = kv.new_table(1 << 14)
+    st = status_tensor()
+    kv.insert(slots, dev(pool[member]), st)
+    pre = kv.probe(slots, dev(digests), dev(off), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    ks = oracle.KeySet(1)
+    ks.insert(pool[member])
+    want = ks.prefix_blocks(digests, off)
+    got = pre.cpu().numpy()
+    assert (got == want).all(), f"{int((got != want).sum())} of {n_req} prefix lengths differ"
+    if max_nb >= 129:
+        assert want[6] == 32 and want[7] == 128
+    assert want.max() > (100 if max_nb >= 300 else 0)
+
+
+@pytest.mark.parametrize("n_req", [500, 40000], ids=["warp", "queue"])
+def test_probe_bad_range_in_a_batch(kv, n_req):
+    """A malformed range (its end before its start) in the middle of a batch
+    is flagged and gets prefix 0; every other request, including the next one
+    whose range now starts earlier, gets the oracle's prefix for its range."""
+    rng = np.random.default_rng(n_req)
+    pool = keys_np(2000, 41)
+    nb = rng.integers(1, 12, n_req)
+    off = np.concatenate([[0], np.cumsum(nb)]).astype(np.int64)
+    digests = pool[rng.integers(0, len(pool), int(off[-1]))]
+    member = rng.random(len(pool)) < 0.8
+    k = n_req // 2
+    off_bad = off.copy()
+    off_bad[k + 1] = off[k] - 1                 # request k: -1 blocks; request k+1 starts one block early
+    slots = kv.new_table(1 << 13)
+    st = status_tensor()
+    kv.insert(slots, dev(pool[member]), st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    pre = kv.probe(slots, dev(digests), dev(off_bad), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & kv.F_BADINDEX
+    # the same requests laid out back to back for the oracle, the bad one empty
+    ranges = [(int(off_bad[r]), max(0, int(off_bad[r + 1] - off_bad[r]))) for r in range(n_req)]
+    ranges[k] = (0, 0)
+    flat = np.concatenate([digests[b:b + n] for b, n in ranges])
+    off2 = np.concatenate([[0], np.cumsum([n for _, n in ranges])]).astype(np.int64)
+    ks = oracle.KeySet(1)
+    ks.insert(pool[member])
+    want = ks.prefix_blocks(flat, off2)
+    assert (pre.cpu().numpy() == want).all()
+
+
 @pytest.mark.parametrize("cap_log2", [6, 12, 16])
 def test_insert_uncached_after_probe_matches_insert_all(kv, cap_log2):
     """Probe, then insert each request's suffix from its prefix length: the
