@@ -67,4 +67,35 @@ __device__ __forceinline__ bool lookup_from_home(const uint4 *__restrict__ slots
     }
 }
 
+// lookup() whose first two slots, the key's home slot (a, b) and the next
+// one (c, d), the caller has read already (four independent loads, one
+// memory round trip); the walk goes on two slots per round trip.  A walk
+// of up to two slots -- most hits and, at load factor 0.5, half the misses
+// -- then costs one round trip.  Same result as lookup().
+__device__ __forceinline__ bool lookup_from_pair(const uint4 *__restrict__ slots, unsigned long long mask, uint4 q0,
+                                                 uint4 q1, uint4 a, uint4 b, uint4 c, uint4 d) {
+    if ((u64_of(q0.x, q0.y) | u64_of(q0.z, q0.w)) == 0ull || u64_of(q1.x, q1.y) == 0ull ||
+        u64_of(q1.z, q1.w) == 0ull)
+        return false;                               // reserved keys are never stored
+    const unsigned long long window = probe_window(mask);   // even: capacity is a power of two >= 32
+    unsigned long long pos = home_slot(q0, mask);
+    for (unsigned long long n = 2;; n += 2) {
+        if ((a.x | a.y | a.z | a.w) == 0u) return false;   // empty slot ends the walk
+        if (a.x == q0.x && a.y == q0.y && a.z == q0.z && a.w == q0.w && b.x == q1.x && b.y == q1.y &&
+            b.z == q1.z && b.w == q1.w)
+            return true;
+        if ((c.x | c.y | c.z | c.w) == 0u) return false;
+        if (c.x == q0.x && c.y == q0.y && c.z == q0.z && c.w == q0.w && d.x == q1.x && d.y == q1.y &&
+            d.z == q1.z && d.w == q1.w)
+            return true;
+        if (n == window) return false;
+        pos = (pos + 2) & mask;
+        const unsigned long long nxt = (pos + 1) & mask;
+        a = __ldg(slots + 2 * pos);
+        b = __ldg(slots + 2 * pos + 1);
+        c = __ldg(slots + 2 * nxt);
+        d = __ldg(slots + 2 * nxt + 1);
+    }
+}
+
 }  // namespace kvgov_dev

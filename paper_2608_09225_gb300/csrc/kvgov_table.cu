@@ -127,10 +127,12 @@ __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long lo
 // ---------------------------------------------------------------------------
 constexpr int kProbeThreads = 256;
 // Probe layouts, by batch size (build options, measured side by side by
-// variants.py --probe): probe_seg_kernel<G, kPer> with first window F for
-//   n_req >= KVGOV_PROBE_MANY_MIN                  (MANY_G, MANY_PER, MANY_FIRST)
-//   KVGOV_PROBE_MID_MIN <= n_req < ..._MANY_MIN     (MID_G, MID_PER, MID_FIRST)
-//   n_req < KVGOV_PROBE_MID_MIN                     (FEW_G, FEW_PER, FEW_FIRST)
+// variants.py --probe): probe_seg_kernel<G, kPer, PAIR> with first window F
+//   n_req >= KVGOV_PROBE_MANY_MIN                  (MANY_G, _PER, _PAIR, _FIRST)
+//   KVGOV_PROBE_MID_MIN <= n_req < ..._MANY_MIN     (MID_G, _PER, _PAIR, _FIRST)
+//   n_req < KVGOV_PROBE_MID_MIN                     (FEW_G, _PER, _PAIR, _FIRST)
+// PAIR reads a key's home slot and the next one together (a walk of two
+// slots in one memory round trip) rather than the home slot alone.
 #ifndef KVGOV_PROBE_MANY_MIN
 #define KVGOV_PROBE_MANY_MIN 32768
 #endif
@@ -142,6 +144,15 @@ constexpr int kProbeThreads = 256;
 #endif
 #ifndef KVGOV_PROBE_MANY_PER
 #define KVGOV_PROBE_MANY_PER 1
+#endif
+#ifndef KVGOV_PROBE_MANY_PAIR
+#define KVGOV_PROBE_MANY_PAIR 0
+#endif
+#ifndef KVGOV_PROBE_MID_PAIR
+#define KVGOV_PROBE_MID_PAIR 1
+#endif
+#ifndef KVGOV_PROBE_FEW_PAIR
+#define KVGOV_PROBE_FEW_PAIR 1
 #endif
 #ifndef KVGOV_PROBE_MANY_FIRST
 #define KVGOV_PROBE_MANY_FIRST 1
@@ -182,7 +193,7 @@ __device__ __forceinline__ void probe_range(const int64_t *__restrict__ blk_off,
 // their memory accesses overlap).  A small first window wastes few lookups
 // on a request that misses early; the growing windows take a long cached
 // prefix in few rounds.
-template <int G, int kPer>
+template <int G, int kPer, bool PAIR>
 __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *__restrict__ slots,
                                                                   unsigned long long mask,
                                                                   const uint4 *__restrict__ digests,
@@ -202,7 +213,7 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
         int w = first;
         bool active = nb > 0;
         while (__any_sync(0xffffffffu, active)) {
-            uint4 q0[kPer], q1[kPer], a[kPer], b[kPer];
+            uint4 q0[kPer], q1[kPer], a[kPer], b[kPer], c[kPer], d[kPer];
 #pragma unroll
             for (int u = 0; u < kPer; ++u) {
                 const int o = sl + G * u;
@@ -218,14 +229,20 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
                     const unsigned long long h = home_slot(q0[u], mask);
                     a[u] = __ldg(slots + 2 * h);
                     b[u] = __ldg(slots + 2 * h + 1);
+                    if (PAIR) {
+                        const unsigned long long h1 = (h + 1) & mask;
+                        c[u] = __ldg(slots + 2 * h1);
+                        d[u] = __ldg(slots + 2 * h1 + 1);
+                    }
                 }
             }
             int miss_at = -1;                                  // the window's first miss (per segment)
 #pragma unroll
             for (int u = 0; u < kPer; ++u) {
                 const int o = sl + G * u;
-                const bool miss = active && o < w && L + o < nb && !lookup_from_home(slots, mask, q0[u], q1[u],
-                                                                                     a[u], b[u]);
+                const bool miss = active && o < w && L + o < nb &&
+                                  !(PAIR ? lookup_from_pair(slots, mask, q0[u], q1[u], a[u], b[u], c[u], d[u])
+                                         : lookup_from_home(slots, mask, q0[u], q1[u], a[u], b[u]));
                 const unsigned m = (__ballot_sync(0xffffffffu, miss) >> (seg * G)) & kSegMask;
                 if (m && miss_at < 0) miss_at = G * u + __ffs((int)m) - 1;
             }
@@ -412,15 +429,15 @@ extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint
     const uint4 *slots = reinterpret_cast<const uint4 *>(d_slots), *dig = reinterpret_cast<const uint4 *>(d_digests);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     if (n_req >= KVGOV_PROBE_MANY_MIN)
-        probe_seg_kernel<KVGOV_PROBE_MANY_G, KVGOV_PROBE_MANY_PER>
+        probe_seg_kernel<KVGOV_PROBE_MANY_G, KVGOV_PROBE_MANY_PER, (KVGOV_PROBE_MANY_PAIR != 0)>
             <<<probe_grid(n_req, KVGOV_PROBE_MANY_G), kProbeThreads, 0, s>>>(
                 slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, KVGOV_PROBE_MANY_FIRST);
     else if (n_req >= KVGOV_PROBE_MID_MIN)
-        probe_seg_kernel<KVGOV_PROBE_MID_G, KVGOV_PROBE_MID_PER>
+        probe_seg_kernel<KVGOV_PROBE_MID_G, KVGOV_PROBE_MID_PER, (KVGOV_PROBE_MID_PAIR != 0)>
             <<<probe_grid(n_req, KVGOV_PROBE_MID_G), kProbeThreads, 0, s>>>(
                 slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, KVGOV_PROBE_MID_FIRST);
     else
-        probe_seg_kernel<KVGOV_PROBE_FEW_G, KVGOV_PROBE_FEW_PER>
+        probe_seg_kernel<KVGOV_PROBE_FEW_G, KVGOV_PROBE_FEW_PER, (KVGOV_PROBE_FEW_PAIR != 0)>
             <<<probe_grid(n_req, KVGOV_PROBE_FEW_G), kProbeThreads, 0, s>>>(
                 slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, KVGOV_PROBE_FEW_FIRST);
     return kvgov_host::launch_status();

@@ -20,8 +20,8 @@ the median steady-state insert, the insert of the first step after a flush
 (where every request's shared-prefix blocks are new, a hot key), probe and
 step times; the number of keys inserted must equal the closed form.
 
-Probe mode (flags KVGOV_PROBE_{MANY,MID,FEW}_{G,PER,FIRST}, _MANY_MIN,
-_MID_MIN): kvgov_probe on every workload's probed requests against its table
+Probe mode (flags KVGOV_PROBE_{MANY,MID,FEW}_{G,PER,PAIR,FIRST},
+_MANY_MIN, _MID_MIN): kvgov_probe on every workload's probed requests against its table
 as bench.py --configs fills it, plus two mid-size batches (all 8192 template
 requests, the first 16,384 probe-heavy requests); mean of 20 back-to-back
 launches queued behind a GPU spin.  Every variant's prefix lengths must
@@ -157,18 +157,11 @@ def insert_mode(specs):
 
 PROBE_DEFAULT = [
     "default:",
-    "many_8x1_first8:-DKVGOV_PROBE_MANY_G=8 -DKVGOV_PROBE_MANY_FIRST=8",
-    "many_8x1_first1:-DKVGOV_PROBE_MANY_G=8",
-    "many_2x1_first1:-DKVGOV_PROBE_MANY_G=2",
-    "many_4x1_first2:-DKVGOV_PROBE_MANY_FIRST=2",
-    "many_4x1_first4:-DKVGOV_PROBE_MANY_FIRST=4",
-    "mid_4x1_first1:-DKVGOV_PROBE_MID_G=4 -DKVGOV_PROBE_MID_PER=1 -DKVGOV_PROBE_MID_FIRST=1",
-    "mid_4x2_first1:-DKVGOV_PROBE_MID_G=4 -DKVGOV_PROBE_MID_PER=2 -DKVGOV_PROBE_MID_FIRST=1",
-    "mid_4x1_first4:-DKVGOV_PROBE_MID_G=4 -DKVGOV_PROBE_MID_PER=1 -DKVGOV_PROBE_MID_FIRST=4",
-    "mid_8x2_first1:-DKVGOV_PROBE_MID_G=8 -DKVGOV_PROBE_MID_PER=2 -DKVGOV_PROBE_MID_FIRST=1",
-    "mid_16x2_first1:-DKVGOV_PROBE_MID_FIRST=1",
+    "all_single:-DKVGOV_PROBE_MID_PAIR=0 -DKVGOV_PROBE_FEW_PAIR=0",
+    "all_pair:-DKVGOV_PROBE_MANY_PAIR=1",
+    "mid_single:-DKVGOV_PROBE_MID_PAIR=0",
     "mid_8x1_first8:-DKVGOV_PROBE_MID_G=8 -DKVGOV_PROBE_MID_PER=1 -DKVGOV_PROBE_MID_FIRST=8",
-    "few_warp32_first1:-DKVGOV_PROBE_FEW_FIRST=1",
+    "many_8x1_first8:-DKVGOV_PROBE_MANY_G=8 -DKVGOV_PROBE_MANY_FIRST=8",
 ]
 
 
