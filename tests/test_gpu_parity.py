@@ -324,14 +324,14 @@ def test_probe_matches_oracle(kv, cap_log2):
     assert (pre.cpu().numpy() == ks.prefix_blocks(digests, off)).all()
 
 
-@pytest.mark.parametrize("n_req,max_nb,p_member", [(700, 400, 0.995), (3000, 70, 0.6), (40000, 40, 0.9),
-                                                    (40000, 3, 0.5), (70000, 300, 0.999)],
-                         ids=["warp_long", "warp_short", "queue", "queue_tiny_requests", "queue_long"])
+@pytest.mark.parametrize("n_req,max_nb,p_member", [(700, 400, 0.995), (3000, 70, 0.6), (20000, 150, 0.99),
+                                                    (40000, 40, 0.9), (40000, 3, 0.5), (70000, 300, 0.999)],
+                         ids=["few_long", "mid_short", "mid_long", "many", "many_tiny_requests", "many_long"])
 def test_probe_layouts_match_oracle(kv, n_req, max_nb, p_member):
-    """Both probe layouts (a warp per request below 32,768 requests, 32
-    requests per warp with a queue above), with requests of 0, 1 and 2
+    """Every probe layout (a warp per request below 2048 requests, 16 lanes
+    per request up to 32,768, 4 lanes above), with requests of 0, 1 and 2
     blocks, prefixes that span several rounds (up to 400 blocks), and
-    prefixes that end exactly at a round's edge."""
+    prefixes that end exactly at a window's edge."""
     rng = np.random.default_rng(n_req + max_nb)
     pool = keys_np(6000, n_req % 997 + 3)
     nb = rng.integers(0, max_nb + 1, n_req)
@@ -339,7 +339,7 @@ def test_probe_layouts_match_oracle(kv, n_req, max_nb, p_member):
     off = np.concatenate([[0], np.cumsum(nb)]).astype(np.int64)
     digests = pool[rng.integers(0, len(pool), int(off[-1]))]
     member = rng.random(len(pool)) < p_member
-    # request 6 misses exactly at block 32 (the end of a warp's first round),
+    # request 6 misses exactly at block 32 (the end of a warp's first window),
     # request 7 at block 128, when they are that long
     for r, j in ((6, 32), (7, 128)):
         if nb[r] > j:
@@ -361,7 +361,7 @@ def test_probe_layouts_match_oracle(kv, n_req, max_nb, p_member):
     assert want.max() > (100 if max_nb >= 300 else 0)
 
 
-@pytest.mark.parametrize("n_req", [500, 40000], ids=["warp", "queue"])
+@pytest.mark.parametrize("n_req", [500, 5000, 40000], ids=["few", "mid", "many"])
 def test_probe_bad_range_in_a_batch(kv, n_req):
     """A malformed range (its end before its start) in the middle of a batch
     is flagged and gets prefix 0; every other request, including the next one

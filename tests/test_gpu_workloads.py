@@ -147,8 +147,9 @@ def test_full_wide_serving_steps(kv):
 
 def test_host_pipeline_matches_device_serving(kv):
     """Batches served from pinned host memory through HostPipeline (copies
-    overlapping the previous batch's serving) give the prefix lengths of the
-    same batches served from device memory, and the same cache contents."""
+    overlapping the previous batch's serving; each batch's result read only
+    after the next batch is queued) give the prefix lengths of the same
+    batches served from device memory, and the same cache contents."""
     ws = [W.make("wide", seed=200 + i, n_req=8192) for i in range(4)]
     for w in ws[1:]:
         w.batch.tokens.reshape(-1, 128)[:, :64] = ws[0].batch.tokens[:64]
@@ -158,7 +159,7 @@ def test_host_pipeline_matches_device_serving(kv):
     n_tok = int(w0.batch.tok_off[-1])
     pipe = HostPipeline(host_cache, W.BOUNDARY, w0.batch.n, n_tok)
     order = [0, 1, 2, 0, 3, 1]
-    got, want = [], []
+    got, want, pending = [], [], None
     for i, k in enumerate(order):
         b = ws[k].batch
         secret = w0.secret[:24] + (0 if i < 4 else 1).to_bytes(8, "little")   # a new epoch from batch 4 on
@@ -170,8 +171,12 @@ def test_host_pipeline_matches_device_serving(kv):
         host = [torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
                 for a in (b.tokens, b.tok_off, b.principal, b.boundary_tok)]
         out, ev = pipe.submit(*host, b.n * 8)
-        ev.synchronize()
-        got.append(out.numpy().copy())
+        if pending is not None:                  # the previous batch's result, read while this one runs
+            pending[1].synchronize()
+            got.append(pending[0].numpy().copy())
+        pending = (out, ev)
+    pending[1].synchronize()
+    got.append(pending[0].numpy().copy())
     torch.cuda.synchronize()
     dev_cache.check_status()
     host_cache.check_status()
@@ -222,10 +227,12 @@ def test_device_pipeline_matches_sequential_serving(kv, mode):
         assert int(want[1].min()) == 4
 
 
-def test_device_pipeline_back_to_back_matches_oracle(kv):
-    """Many batches queued without waiting in between: every batch's prefix
-    lengths (copied out on the compute stream right after its submit) match
-    the oracle's arrival-order replay of the same batches."""
+@pytest.mark.parametrize("flush_at", [None, 5])
+def test_device_pipeline_back_to_back_matches_oracle(kv, flush_at):
+    """Many batches queued without waiting in between (and a cache flush
+    queued in the middle): every batch's prefix lengths, copied out on the
+    compute stream right after its submit, match the oracle's replay of the
+    same batches in order."""
     ws = [W.make("wide", seed=400 + i, n_req=4096) for i in range(4)]
     for w in ws[1:]:
         w.batch.tokens.reshape(-1, 128)[:, :64] = ws[0].batch.tokens[:64]
@@ -238,17 +245,20 @@ def test_device_pipeline_back_to_back_matches_oracle(kv):
     copies = []
     for i, k in enumerate(order):
         cache.set_secret(w0.secret[:24] + (i % 2).to_bytes(8, "little"))
-        pre, _ = pipe.submit(dbs[k])
+        before = (lambda: K.table_init(cache.slots, pipe.compute_stream)) if i == flush_at else None
+        pre, _ = pipe.submit(dbs[k], before)
         with torch.cuda.stream(pipe.compute_stream):
             copies.append(pre.clone())
     torch.cuda.synchronize()
     cache.check_status()
-    ks = oracle.KeySet(1)
+    ks, before_flush = oracle.KeySet(1), 0
     for i, k in enumerate(order):
+        if i == flush_at:
+            ks, before_flush = oracle.KeySet(1), ks.n
         b = ws[k].batch
         salts = oracle.derive_salts(w0.secret[:24] + (i % 2).to_bytes(8, "little"), w0.ids, w0.id_off)
         d = oracle.chain_hash(W.BOUNDARY, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
         blk = oracle.block_offsets(b.tok_off)
         assert (copies[i].cpu().numpy() == ks.prefix_blocks(d, blk)).all(), f"batch {i}"
         ks.insert(d)
-    assert int(cache.n_new.item()) == ks.n
+    assert int(cache.n_new.item()) == before_flush + ks.n
