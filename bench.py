@@ -4,8 +4,10 @@
 One step = one serving batch through the whole hot path, every step a
 libkvgov kernel: per-principal salts (HMAC-SHA-256, 4096 principals) ->
 blocking (block offsets) -> BOUNDARY-salted chain hash (salt at token 64,
-block 4) with the probe of the resident prefix-cache table fused into the
-same launch -> insert of each request's uncached blocks.  Workload: 131,072 requests x 128 tokens (8 blocks
+block 4) -> probe of the resident prefix-cache table -> insert of each
+request's uncached blocks.  DevicePipeline runs each batch's insert inside
+the next batch's chain-hash launch (the last one after the timed loop,
+still inside the timed region).  Workload: 131,072 requests x 128 tokens (8 blocks
 each; the largest batch), a 64-token prefix shared by all requests, 4096
 principals.
 
@@ -297,6 +299,12 @@ class FlushPolicy:
         self.capacity, self.new_per_step = capacity, new_per_step
         self.in_table, self.expected_new, self.flushes, self.last_prefix = 0, 0, 0, 0
         self.fresh = True
+        self.seen = []
+
+    def mean_load_factor(self) -> float:
+        """Mean load factor the steps so far probed against (the table before
+        each step's insert)."""
+        return float(np.mean(self.seen)) / self.capacity if self.seen else 0.0
 
     def before_step(self) -> bool:
         flushed = False
@@ -304,6 +312,7 @@ class FlushPolicy:
             self.in_table, self.fresh, flushed = 0, True, True
             self.flushes += 1
         add = self.new_per_step + (4 if self.fresh else 0)
+        self.seen.append(self.in_table)
         self.last_prefix = 0 if self.fresh else 4
         self.in_table += add
         self.expected_new += add
@@ -388,6 +397,10 @@ def main():
     ap.add_argument("--seed", type=int, default=None, help="base seed (default: fresh per run)")
     ap.add_argument("--cpu-sample", type=int, default=16384, help="requests per oracle step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--schedule", default="insert_in_chain", choices=["insert_in_chain", "inline"],
+                    help="insert_in_chain: each batch's insert runs inside the next batch's chain launch and the "
+                         "batch is probed after its chain hash; inline: chain hash with the fused probe, then the "
+                         "insert")
     ap.add_argument("--configs", action="store_true",
                     help="instead of the timed serving step: per-kernel rates on every workload, one JSON line each")
     ap.add_argument("--only", default=None,
@@ -448,17 +461,21 @@ def main():
 
     # ---- the timed steps: DevicePipeline computes each batch's salts and block
     # offsets on a prep stream beside the previous batch's chain hash
-    pipe = DevicePipeline(cache, W.BOUNDARY, n_req, n_blocks)
+    in_chain = args.schedule == "insert_in_chain"
+    pipe = DevicePipeline(cache, W.BOUNDARY, n_req, n_blocks, insert_in_chain=in_chain)
     epoch = [1]
     launches = [0]
 
-    def step(db, ev=None, ins_ev=None):
+    def step(db, ev=None, tab_ev=None):
         cache.set_secret(epoch_secret(w0.secret, epoch[0]))
         epoch[0] += 1
         flushed = flush.before_step()              # load factor would pass 0.5: flush the cache
         before = (lambda: K.table_init(cache.slots, pipe.compute_stream)) if flushed else None
-        prefix, _ = pipe.submit(db, before, ev, ins_ev)
-        launches[0] += 5 + int(flushed)   # salts, block offsets (2), chain hash + probe, insert (+ table init)
+        pending = pipe.pending is not None
+        prefix, _ = pipe.submit(db, before, ev, tab_ev)
+        # salts, block offsets (2), the chain hash (with the previous batch's insert, or with the probe fused
+        # in), the probe (or the insert); a flush adds the table init and, in_chain, the pending insert
+        launches[0] += 5 + (int(flushed) * (1 + int(pending)) if in_chain else int(flushed))
         return prefix
 
     for i in range(args.warmup):
@@ -468,9 +485,9 @@ def main():
 
     chain_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                 for _ in range(args.steps)]
-    insert_every = 4                               # time every 4th insert: two events fewer on the critical path
-    insert_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                 if i % insert_every == 0 else None for i in range(args.steps)]
+    table_every = 4                                # time every 4th table kernel: two events fewer on the critical path
+    table_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                if i % table_every == 0 else None for i in range(args.steps)]
     t_start, t_stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     launches[0] = 0
     flushes_before = flush.flushes
@@ -482,7 +499,10 @@ def main():
         pipe.prep_stream.wait_event(t_start)
         h0 = time.perf_counter()
         for i in range(args.steps):
-            last_prefix = step(pool[(1 + args.warmup + i) % args.pool], chain_ev[i], insert_ev[i])
+            last_prefix = step(pool[(1 + args.warmup + i) % args.pool], chain_ev[i], table_ev[i])
+        if in_chain:
+            pipe.drain()                           # the last batch's insert
+            launches[0] += 1
         host_ms = (time.perf_counter() - h0) * 1e3
         t_stop.record(pipe.compute_stream)
         torch.cuda.synchronize()
@@ -499,7 +519,7 @@ def main():
     kernel_launches = launches[0]
     ms = t_start.elapsed_time(t_stop)
     chain_ms = float(np.mean([a.elapsed_time(b) for a, b in chain_ev]))
-    insert_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in insert_ev if e is not None]))
+    table_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in table_ev if e is not None]))
     inserted_per_step = (gate["n_new_total"] - n_new_before) / args.steps
     ms = max_over_ranks(ms, world, dist, "cuda")
     value = world * args.steps * n_blocks / (ms / 1e3)
@@ -521,8 +541,12 @@ def main():
     traffic, traffic_src = profiled_traffic()
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s (int32)",
                 "frac": achieved / peak_tops, "traffic": traffic,
-                "kernel": "chain_kernel<BOUNDARY, probe> (kvgov_chain_hash_probe)", "ops_per_launch": ops,
-                "kernel_ms": chain_ms, "ops_counted": "SHA-256 ops of the chain only; the fused lookups are extra",
+                "kernel": ("chain_prev_kernel<BOUNDARY> (kvgov_chain_hash_insert_prev: the chain hash with the "
+                           "previous batch's insert)" if in_chain else
+                           "chain_kernel<BOUNDARY, probe> (kvgov_chain_hash_probe)"), "ops_per_launch": ops,
+                "kernel_ms": chain_ms,
+                "ops_counted": "SHA-256 ops of the chain only; the fused " +
+                               ("inserts of the previous batch" if in_chain else "lookups") + " are extra",
                 "algorithmic_bytes_per_launch": 96 * n_blocks,
                 "peak_basis": f"{n_sm} SMs x 4 SMSPs x 16 int32 lanes x {SM_MAX_MHZ:.0f} MHz; every SHF, LOP3, "
                               f"IADD3 and IMAD of SHA-256 issues to that one 16-lane pipe per SMSP",
@@ -533,22 +557,50 @@ def main():
     # the table kernel of the step (insert of the uncached blocks) against HBM and a random-read ceiling
     gather = measure_gather(torch, kbuild.PEAK_LIB, cache.slots)
     claims = measure_slot_ops(torch, kbuild.PEAK_LIB, cache.slots, int(inserted_per_step))
-    ins_bytes = 96 * inserted_per_step + 20 * n_req
-    ins_gbs = ins_bytes / (insert_ms / 1e3) / 1e9
-    table_roofline = {
-        "kernel": "insert_uncached_kernel<8> (kvgov_insert_uncached)", "bound": "hbm", "achieved": ins_gbs,
-        "peak": PEAKS.get("hbm_gbs"), "unit": "GB/s", "frac": ins_gbs / PEAKS["hbm_gbs"] if PEAKS.get("hbm_gbs") else None,
-        "peak_source": "of fallback (6.8 TB/s)" if PEAKS.get("fallback") else "of measured (MEASURED_PEAKS.json hbm_gbs, a copy)",
-        "random_read_ceiling_gbs": gather["gbs_32B"], "frac_of_random_read_ceiling": ins_gbs / gather["gbs_32B"],
-        "kernel_ms": insert_ms, "timed_launches": f"every {insert_every}th step of the timed region",
-        "keys_inserted_per_launch": inserted_per_step,
-        "inserts_per_s": inserted_per_step / (insert_ms / 1e3),
-        "algorithmic_bytes_per_launch": ins_bytes,
-        "bytes_basis": "per new key 32 B read + one 32 B slot read + 32 B written; per request 4 B prefix + 16 B offsets",
-        "random_read_microbench": gather,
-        "claim_ceiling_per_s": claims["read_cas_store_per_s"],
-        "frac_of_claim_ceiling": (inserted_per_step / (insert_ms / 1e3)) / claims["read_cas_store_per_s"],
-        "slot_op_microbench": claims}
+    if in_chain:
+        # the probe: every request looks up its 4 shared-prefix blocks (hits) and block 4 (a miss); a hit
+        # walks (1 + 1/(1-a))/2 slots and a miss (1 + 1/(1-a)^2)/2 at the table's mean load factor a
+        lf = flush.mean_load_factor()
+        walk = 4 * (1 + 1 / (1 - lf)) / 2 + (1 + 1 / (1 - lf) ** 2) / 2
+        lookups = 5 * n_req
+        tab_bytes = lookups * 32 + walk * n_req * 32 + 20 * n_req
+        tab_gbs = tab_bytes / (table_ms / 1e3) / 1e9
+        table_roofline = {
+            "kernel": "probe_seg_kernel<4, 1> (kvgov_probe)", "bound": "hbm", "achieved": tab_gbs,
+            "peak": PEAKS.get("hbm_gbs"), "unit": "GB/s",
+            "frac": tab_gbs / PEAKS["hbm_gbs"] if PEAKS.get("hbm_gbs") else None,
+            "peak_source": "of fallback (6.8 TB/s)" if PEAKS.get("fallback") else
+                           "of measured (MEASURED_PEAKS.json hbm_gbs, a copy)",
+            "random_read_ceiling_gbs": gather["gbs_32B"], "frac_of_random_read_ceiling": tab_gbs / gather["gbs_32B"],
+            "kernel_ms": table_ms, "timed_launches": f"every {table_every}th step of the timed region",
+            "lookups_per_launch": lookups, "lookups_per_s": lookups / (table_ms / 1e3),
+            "mean_load_factor": lf, "algorithmic_bytes_per_launch": tab_bytes,
+            "bytes_basis": "per lookup its 32 B digest and 32 B per slot walked at the mean load factor; per "
+                           "request 16 B offsets + 4 B prefix",
+            "random_read_microbench": gather,
+            "insert": {"where": "inside the next batch's chain launch (kvgov_chain_hash_insert_prev)",
+                       "keys_inserted_per_step": inserted_per_step,
+                       "claim_ceiling_per_s": claims["read_cas_store_per_s"], "slot_op_microbench": claims}}
+    else:
+        ins_bytes = 96 * inserted_per_step + 20 * n_req
+        ins_gbs = ins_bytes / (table_ms / 1e3) / 1e9
+        table_roofline = {
+            "kernel": "insert_uncached_packed_kernel (kvgov_insert_uncached)", "bound": "hbm", "achieved": ins_gbs,
+            "peak": PEAKS.get("hbm_gbs"), "unit": "GB/s",
+            "frac": ins_gbs / PEAKS["hbm_gbs"] if PEAKS.get("hbm_gbs") else None,
+            "peak_source": "of fallback (6.8 TB/s)" if PEAKS.get("fallback") else
+                           "of measured (MEASURED_PEAKS.json hbm_gbs, a copy)",
+            "random_read_ceiling_gbs": gather["gbs_32B"], "frac_of_random_read_ceiling": ins_gbs / gather["gbs_32B"],
+            "kernel_ms": table_ms, "timed_launches": f"every {table_every}th step of the timed region",
+            "keys_inserted_per_launch": inserted_per_step,
+            "inserts_per_s": inserted_per_step / (table_ms / 1e3),
+            "algorithmic_bytes_per_launch": ins_bytes,
+            "bytes_basis": "per new key 32 B read + one 32 B slot read + 32 B written; per request 4 B prefix + "
+                           "16 B offsets",
+            "random_read_microbench": gather,
+            "claim_ceiling_per_s": claims["read_cas_store_per_s"],
+            "frac_of_claim_ceiling": (inserted_per_step / (table_ms / 1e3)) / claims["read_cas_store_per_s"],
+            "slot_op_microbench": claims}
     if clock.get("sm_mhz"):
         roofline["frac_at_run_clock"] = achieved / (n_sm * INT32_LANES_PER_SM * clock["sm_mhz"] * 1e6 / 1e12)
 
@@ -564,8 +616,13 @@ def main():
                                   "timed steps) whenever the next step would take it past load factor 0.5"),
             "tokens_per_s": 16 * value, "chain_digests_per_s": world * n_blocks / (chain_ms / 1e3),
             "host_enqueue_ms_per_step": host_ms / args.steps,
-            "schedule": "DevicePipeline: salts (new epoch) and block offsets of batch i+1 on a prep stream beside "
-                        "the chain hash of batch i; chain hash + probe, insert on a higher-priority compute stream",
+            "schedule": ("DevicePipeline (insert in chain): salts (new epoch) and block offsets of batch i+1 on a "
+                         "prep stream beside the chain hash of batch i; on a higher-priority compute stream the "
+                         "chain hash of batch i with batch i-1's insert in the same launch, then the probe of batch "
+                         "i" if in_chain else
+                         "DevicePipeline (inline): salts (new epoch) and block offsets of batch i+1 on a prep stream "
+                         "beside the chain hash of batch i; chain hash with the fused probe, then the insert, on a "
+                         "higher-priority compute stream"),
             "e2e": e2e, "gpu_launches": kernel_launches, "clocks": clock, "roofline": roofline,
             "table_roofline": table_roofline,
             "arrival": arrival, "gate": gate}
@@ -653,6 +710,7 @@ def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots):
     a.record(pipe.copy_stream)
     for i in range(steps):
         out, ev = one(warm + i)
+    pipe.drain()                                   # the last batch's insert
     b.record(pipe.compute_stream)
     torch.cuda.synchronize()
     cache.check_status()
@@ -674,7 +732,8 @@ def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots):
     return {"value": value, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps, "last_step_prefix_ok": last_ok,
             "h2d_link_gbs": link_gbs, "copy_bound_value": copy_bound, "frac_of_copy_bound": value / copy_bound,
-            "api": "paper_2608_09225_gb300.pipeline.HostPipeline (copy of step i+1 overlaps serving of step i)"}
+            "api": "paper_2608_09225_gb300.pipeline.HostPipeline (copy of step i+1 overlaps serving of step i; "
+                   "each step's insert inside the next step's chain launch)"}
 
 
 def cpu_baseline(w, sample, gpu_digests):

@@ -319,6 +319,37 @@ int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_
                           unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * kvgov_chain_hash_insert_prev -- kvgov_chain_hash of one batch and, in the
+ * same launch, kvgov_insert_uncached of the previous batch (paper section
+ * 2.1: a served request's uncached blocks are computed and cached).  In a
+ * stream of batches, batch i+1's chain hash does not read the table, so
+ * batch i's insert can run inside it: each thread inserts uncached blocks of
+ * the previous batch between its own compressions, and the memory latency of
+ * the inserts is covered by the other warps' hashing.  The digests equal
+ * kvgov_chain_hash's; the table, *d_n_new and the insert flags equal
+ * kvgov_insert_uncached's on the previous batch.
+ *   mode .. d_digests  as for kvgov_chain_hash (this batch).
+ *   d_slots, capacity  the table (as for kvgov_insert).
+ *   d_prev_digests, d_prev_blk_off, prev_n_req, d_prev_prefix_blocks
+ *              the previous batch, as for kvgov_insert_uncached; its arrays
+ *              must not overlap this batch's d_digests.  prev_n_req = 0:
+ *              kvgov_chain_hash alone.
+ *   d_n_new, d_status  as for kvgov_insert_uncached (d_status required).
+ * The table must not be read or written by other calls while this one runs
+ * (probe this batch after it).  A batch too small to give every SM
+ * sub-partition two warps (n_req < 2 * 32 * 4 * SMs) runs the chain hash and
+ * the insert as two launches instead; the results are the same.  EINVAL: as
+ * for kvgov_chain_hash and kvgov_insert_uncached, prev_n_req < 0.
+ */
+int kvgov_chain_hash_insert_prev(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                                 const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                                 const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                                 uint8_t *d_slots, uint64_t capacity, const uint8_t *d_prev_digests,
+                                 const int64_t *d_prev_blk_off, int32_t prev_n_req,
+                                 const int32_t *d_prev_prefix_blocks, unsigned long long *d_n_new,
+                                 uint32_t *d_status, kvgov_stream_t stream);
+
+/*
  * Arrival-order serving of one batch -- paper section 2.1 (a lookup matches
  * the longest cached prefix of blocks from position 0) and section 4.2
  * (prefill cost is proportional to the uncached tokens), applied request by

@@ -1,5 +1,6 @@
 // kvgov_chain.cu -- the chained, salted block digests (kvgov_chain_hash,
-// kvgov_chain_hash_probe).
+// kvgov_chain_hash_probe, kvgov_chain_hash_arrival,
+// kvgov_chain_hash_insert_prev).
 //
 // Paper: section 2.1 equation (h_0 = H(tokens_0..B-1), h_j = H(h_{j-1},
 // tokens_j)), section 4.1 equation (sigma_p prepended at the root) and
@@ -83,10 +84,23 @@ struct ArrivalParams {
     uint32_t spin_limit = 0;
 };
 
+// The previous batch whose uncached blocks kFuseInsertPrev inserts.
+struct PrevParams {
+    unsigned long long *slots = nullptr;
+    unsigned long long mask = 0;
+    const uint4 *digests = nullptr;
+    const int64_t *blk_off = nullptr;
+    const int32_t *prefix_blocks = nullptr;
+    int32_t n_req = 0;
+    unsigned long long *n_new = nullptr;
+    uint32_t spin_limit = 0;
+};
+
 // What the chain kernel does with each digest besides storing it.
 constexpr int kFuseNone = 0;      // nothing (kvgov_chain_hash)
 constexpr int kFuseProbe = 1;     // look it up (kvgov_chain_hash_probe)
 constexpr int kFuseArrival = 2;   // insert it, arrival order (kvgov_chain_hash_arrival)
+constexpr int kFuseInsertPrev = 3;   // insert the previous batch's uncached blocks (kvgov_chain_hash_insert_prev)
 
 // Which adder the SHA-256 rounds use.  Measured on GB300: IMAD shares the
 // integer pipe with SHF/LOP3/IADD3 (libkvgov_peak kinds 3-5), so AddFma
@@ -111,8 +125,13 @@ __device__ __forceinline__ void load_salt(const uint8_t *salts, int pi, uint32_t
 // requests, so a key their prefixes share is inserted by its lowest lane
 // only and the others take its slot.  Either way the memory latency is
 // covered by the other warps' hashing.
+// kFuseInsertPrev: thread t inserts the uncached blocks of the previous
+// batch's requests t, t + T, ... (T threads in the grid), one block per
+// iteration of its own chain and the rest after it (the insert of
+// kvgov_insert_uncached).
 template <int MODE, int FUSE>
-__device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalParams &a) {
+__device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalParams &a,
+                                           const PrevParams &q = PrevParams{}) {
     __shared__ __align__(16) uint32_t stage[kStages][kR * kSlotWords];
     __shared__ long long s_tok[kR];
     __shared__ int s_nb[kR];
@@ -122,7 +141,7 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
     const int tid = threadIdx.x;
     const long long r = (long long)blockIdx.x * kR + tid;
     if (tid == 0) s_jmax = 0;
-    if (FUSE == kFuseArrival && tid == 0) { s_new = 0; s_flags = 0; s_done = 0; }
+    if ((FUSE == kFuseArrival || FUSE == kFuseInsertPrev) && tid == 0) { s_new = 0; s_flags = 0; s_done = 0; }
 
     // Per-request set-up and validation.
     const long long tok_end = p.tok_off[p.n_req];
@@ -192,6 +211,45 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
 
     unsigned long long ak[4] = {0ull, 0ull, 0ull, 0ull};   // kFuseArrival: block j's key
     bool have = false;                                      // ... to be inserted by this lane
+
+    // kFuseInsertPrev: the previous batch's request pq this thread inserts,
+    // its next uncached row and how many of its uncached blocks remain.
+    const long long pstride = (long long)gridDim.x * kR;
+    long long pq = r, prow = 0;
+    long long pleft = 0;
+    auto prev_next = [&]() {                     // from pq on: the first request with uncached blocks
+        for (; pq < q.n_req; pq += pstride) {
+            const long long base = q.blk_off[pq], pnb = q.blk_off[pq + 1] - base;
+            if (pnb < 0 || base < 0 || base + pnb > q.blk_off[q.n_req]) {
+                my_flags |= KVGOV_F_BADINDEX;
+                continue;
+            }
+            long long L = q.prefix_blocks[pq];
+            L = L < 0 ? 0 : (L > pnb ? pnb : L);
+            if (pnb > L) {
+                prow = base + L;
+                pleft = pnb - L;
+                return;
+            }
+        }
+        pleft = 0;
+    };
+    auto prev_insert_one = [&]() {               // insert row prow of the previous batch
+        const uint4 x = __ldg(q.digests + 2 * prow), y = __ldg(q.digests + 2 * prow + 1);
+        const unsigned long long key[4] = {u64_of(x.x, x.y), u64_of(x.z, x.w), u64_of(y.x, y.y), u64_of(y.z, y.w)};
+        if (key_reserved(key)) {
+            my_flags |= KVGOV_F_SENTINEL;
+        } else {
+            unsigned long long pos = 0;
+            count_insert(insert_one(q.slots, q.mask, key, q.spin_limit, &pos), my_new, my_flags);
+        }
+        ++prow;
+        if (--pleft == 0) {
+            pq += pstride;
+            prev_next();
+        }
+    };
+    if (FUSE == kFuseInsertPrev) prev_next();
     for (int j = 0; j < jmax; ++j) {
         const int jn = j + kStages - 1;
         if (jn < jmax) issue(jn, jn % kStages);
@@ -274,11 +332,16 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             }
             have = false;
         }
+        if (FUSE == kFuseInsertPrev && pleft > 0) prev_insert_one();
         __syncthreads();
     }
     cp_async_wait<0>();
     if (FUSE == kFuseProbe && r < p.n_req) p.prefix_blocks[r] = hits;
-    if (FUSE == kFuseArrival) publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, a.n_new, p.status);
+    if (FUSE == kFuseInsertPrev)
+        while (pleft > 0) prev_insert_one();
+    if (FUSE == kFuseArrival || FUSE == kFuseInsertPrev)
+        publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, FUSE == kFuseArrival ? a.n_new : q.n_new,
+                       p.status);
 }
 
 template <int MODE, int FUSE>
@@ -291,15 +354,27 @@ __global__ void __launch_bounds__(kR) chain_arrival_kernel(const ChainParams p, 
     chain_body<MODE, kFuseArrival>(p, a);
 }
 
+template <int MODE>
+__global__ void __launch_bounds__(kR) chain_prev_kernel(const ChainParams p, const PrevParams q) {
+    chain_body<MODE, kFuseInsertPrev>(p, ArrivalParams{}, q);
+}
+
 }  // namespace
 
 namespace {
 
-// Launch chain_kernel<mode, FUSE> (chain_arrival_kernel<mode> for kFuseArrival).
+// Launch chain_kernel<mode, FUSE> (chain_arrival_kernel<mode> for kFuseArrival,
+// chain_prev_kernel<mode> for kFuseInsertPrev).
 template <int FUSE>
 void launch_chain_kernel(int mode, unsigned grid, cudaStream_t s, const ChainParams &p,
-                         const ArrivalParams &a = ArrivalParams{}) {
-    if constexpr (FUSE == kFuseArrival) {
+                         const ArrivalParams &a = ArrivalParams{}, const PrevParams &q = PrevParams{}) {
+    if constexpr (FUSE == kFuseInsertPrev) {
+        switch (mode) {
+        case KVGOV_UNSALTED: chain_prev_kernel<KVGOV_UNSALTED><<<grid, kR, 0, s>>>(p, q); break;
+        case KVGOV_ROOT: chain_prev_kernel<KVGOV_ROOT><<<grid, kR, 0, s>>>(p, q); break;
+        default: chain_prev_kernel<KVGOV_BOUNDARY><<<grid, kR, 0, s>>>(p, q); break;
+        }
+    } else if constexpr (FUSE == kFuseArrival) {
         switch (mode) {
         case KVGOV_UNSALTED: chain_arrival_kernel<KVGOV_UNSALTED><<<grid, kR, 0, s>>>(p, a); break;
         case KVGOV_ROOT: chain_arrival_kernel<KVGOV_ROOT><<<grid, kR, 0, s>>>(p, a); break;
@@ -324,6 +399,10 @@ struct FuseArgs {
     uint64_t seq_base = 0;
     uint32_t *slot_of = nullptr;
     unsigned long long *n_new = nullptr;
+    const uint8_t *prev_digests = nullptr;     // kFuseInsertPrev
+    const int64_t *prev_blk_off = nullptr;
+    int32_t prev_n_req = 0;
+    const int32_t *prev_prefix_blocks = nullptr;
 };
 
 int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
@@ -345,7 +424,18 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
         (!f.prefix_blocks || !f.slots || !aligned16(f.slots) || !f.owner || !f.slot_of || !d_status ||
          !kvgov_host::arrival_args_ok(f.capacity, f.seq_base)))
         return KVGOV_EINVAL;
-    if (n_req == 0) return KVGOV_OK;
+    if (f.fuse == kFuseInsertPrev &&
+        (!f.slots || !aligned16(f.slots) || !kvgov_host::pow2_capacity(f.capacity) || !d_status ||
+         f.prev_n_req < 0 ||
+         (f.prev_n_req > 0 && (!f.prev_digests || !aligned16(f.prev_digests) || !f.prev_blk_off ||
+                               !f.prev_prefix_blocks))))
+        return KVGOV_EINVAL;
+    // the previous batch's insert alone when this batch is empty
+    auto insert_prev = [&]() {
+        return kvgov_insert_uncached(const_cast<uint8_t *>(f.slots), f.capacity, f.prev_digests, f.prev_blk_off,
+                                     f.prev_n_req, f.prev_prefix_blocks, f.n_new, d_status, stream);
+    };
+    if (n_req == 0) return (f.fuse == kFuseInsertPrev && f.prev_n_req > 0) ? insert_prev() : KVGOV_OK;
 
     ChainParams p;
     p.tokens = d_tokens; p.tok_off = d_tok_off; p.principal = d_principal; p.salts = d_salts;
@@ -360,6 +450,15 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     a.n_new = f.n_new;
     a.seq_base = f.seq_base;
     a.spin_limit = kvgov_host::spin_limit();
+    PrevParams q;
+    q.slots = reinterpret_cast<unsigned long long *>(const_cast<uint8_t *>(f.slots));
+    q.mask = p.mask;
+    q.digests = reinterpret_cast<const uint4 *>(f.prev_digests);
+    q.blk_off = f.prev_blk_off;
+    q.prefix_blocks = f.prev_prefix_blocks;
+    q.n_req = f.prev_n_req;
+    q.n_new = f.n_new;
+    q.spin_limit = a.spin_limit;
     const unsigned grid = (unsigned)(((long long)n_req + kR - 1) / kR);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     // A batch too small to give every SM sub-partition two warps leaves each
@@ -367,11 +466,13 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     // the chain; there they run as separate launches (same results).
     const DeviceInfo dev = device_info();
     const long long min_fused = 2ll * 32 * 4 * (dev.sms > 0 ? dev.sms : 152);
-    const bool fused = f.fuse != kFuseNone && n_req >= min_fused;
+    const bool none = f.fuse == kFuseNone || (f.fuse == kFuseInsertPrev && f.prev_n_req == 0);
+    const bool fused = !none && n_req >= min_fused;
     if (!fused) {
         launch_chain_kernel<kFuseNone>(mode, grid, s, p);
         int rc = kvgov_host::launch_status();
-        if (rc != KVGOV_OK || f.fuse == kFuseNone) return rc;
+        if (rc != KVGOV_OK || none) return rc;
+        if (f.fuse == kFuseInsertPrev) return insert_prev();
         if (f.fuse == kFuseProbe)
             return kvgov_probe(f.slots, f.capacity, d_digests, d_blk_off, n_req, f.prefix_blocks, d_status, stream);
         rc = kvgov_insert_arrival(const_cast<uint8_t *>(f.slots), f.owner, f.capacity, d_digests, d_blk_off, n_req,
@@ -382,6 +483,10 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     }
     if (f.fuse == kFuseProbe) {
         launch_chain_kernel<kFuseProbe>(mode, grid, s, p);
+        return kvgov_host::launch_status();
+    }
+    if (f.fuse == kFuseInsertPrev) {
+        launch_chain_kernel<kFuseInsertPrev>(mode, grid, s, p, a, q);
         return kvgov_host::launch_status();
     }
     launch_chain_kernel<kFuseArrival>(mode, grid, s, p, a);
@@ -432,6 +537,26 @@ extern "C" int kvgov_chain_hash_arrival(int mode, const int32_t *d_tokens, const
     f.seq_base = seq_base;
     f.slot_of = d_slot_of;
     f.n_new = d_n_new;
+    return launch_chain(mode, d_tokens, d_tok_off, n_req, d_principal, d_salts, n_principals, d_boundary_tok,
+                        d_blk_off, d_digests, d_status, f, stream);
+}
+
+extern "C" int kvgov_chain_hash_insert_prev(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                                            const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                                            const int32_t *d_boundary_tok, const int64_t *d_blk_off,
+                                            uint8_t *d_digests, uint8_t *d_slots, uint64_t capacity,
+                                            const uint8_t *d_prev_digests, const int64_t *d_prev_blk_off,
+                                            int32_t prev_n_req, const int32_t *d_prev_prefix_blocks,
+                                            unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream) {
+    FuseArgs f;
+    f.fuse = kFuseInsertPrev;
+    f.slots = d_slots;
+    f.capacity = capacity;
+    f.n_new = d_n_new;
+    f.prev_digests = d_prev_digests;
+    f.prev_blk_off = d_prev_blk_off;
+    f.prev_n_req = prev_n_req;
+    f.prev_prefix_blocks = d_prev_prefix_blocks;
     return launch_chain(mode, d_tokens, d_tok_off, n_req, d_principal, d_salts, n_principals, d_boundary_tok,
                         d_blk_off, d_digests, d_status, f, stream);
 }

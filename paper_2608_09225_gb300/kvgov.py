@@ -56,6 +56,9 @@ def _load():
                                        _p, _p]
         L.kvgov_chain_hash_probe.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p,
                                              _p, _p, ctypes.c_uint64, _p, _p, _p]
+        L.kvgov_chain_hash_insert_prev.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32,
+                                                   _p, _p, _p, _p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p,
+                                                   _p, _p]
         L.kvgov_table_init.argtypes = [_p, ctypes.c_uint64, _p]
         L.kvgov_insert.argtypes = [_p, ctypes.c_uint64, _p, ctypes.c_int64, _p, _p, _p]
         L.kvgov_probe.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p]
@@ -206,6 +209,40 @@ def chain_hash_probe(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, blk
                                     _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_chain_hash_probe")
     return digests, prefix_blocks
+
+
+def chain_hash_insert_prev(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, blk_off: torch.Tensor,
+                           slots: torch.Tensor, prev_digests: torch.Tensor, prev_blk_off: torch.Tensor,
+                           prev_prefix_blocks: torch.Tensor, status: torch.Tensor,
+                           principal: torch.Tensor | None = None, salts: torch.Tensor | None = None,
+                           boundary_tok: torch.Tensor | None = None, digests: torch.Tensor | None = None,
+                           n_blocks: int | None = None, n_new: torch.Tensor | None = None,
+                           stream=None) -> torch.Tensor:
+    """chain_hash of this batch and insert_uncached of the previous batch
+    (prev_digests, prev_blk_off, prev_prefix_blocks) in one launch; returns
+    this batch's digests."""
+    L = lib()
+    n = tok_off.numel() - 1
+    pn = prev_blk_off.numel() - 1
+    if digests is None:
+        if n_blocks is None:
+            n_blocks = int(blk_off[-1].item())
+        digests = torch.empty((n_blocks, 32), dtype=torch.uint8, device=tokens.device)
+    if tokens.numel() == 0:
+        tokens = torch.zeros(4, dtype=torch.int32, device=tok_off.device)
+    n_p = 0 if salts is None else salts.shape[0]
+    _check(L.kvgov_chain_hash_insert_prev(
+        int(mode), _dev(tokens, torch.int32, "tokens"), _dev(tok_off, torch.int64, "tok_off"), n,
+        _dev(principal, torch.int32, "principal", True), _dev(salts, torch.uint8, "salts", True), n_p,
+        _dev(boundary_tok, torch.int32, "boundary_tok", True), _dev(blk_off, torch.int64, "blk_off"),
+        _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(tokens),
+        _dev(slots, torch.uint8, "slots"), slots.shape[0],
+        _dev(prev_digests, torch.uint8, "prev_digests") if prev_digests.numel() else _dummy(tokens),
+        _dev(prev_blk_off, torch.int64, "prev_blk_off"), pn,
+        _dev(prev_prefix_blocks, torch.int32, "prev_prefix_blocks") if pn else _dummy(tokens),
+        _dev(n_new, torch.int64, "n_new", True), _dev(status, torch.int32, "status"), _stream(stream)),
+        "kvgov_chain_hash_insert_prev")
+    return digests
 
 
 def _dummy(like: torch.Tensor):

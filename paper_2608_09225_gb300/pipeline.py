@@ -130,40 +130,55 @@ class PrefixCache:
 
 
 class _Pipelined:
-    """Two alternating slots of per-batch device buffers and the stream
-    schedule shared by DevicePipeline and HostPipeline.
+    """Per-batch device buffers in rotating slots and the stream schedule
+    shared by DevicePipeline and HostPipeline.
 
-    Batch i uses slot i % 2.  Its salts (under the secret current when it is
-    submitted) and block offsets are computed on a prep stream once batch
-    i-1's chain hash has started, so their small CTAs run in the room the
-    chain kernel leaves on the SMs instead of in front of batch i's chain
-    hash.  The compute stream has the higher priority, so the chain and
-    insert CTAs are placed first.  It waits for the prep, runs the chain hash
-    with the fused probe and inserts the uncached blocks.  Every step runs on
-    the GPU; nothing here computes.
+    Batch i's salts (under the secret current when it is submitted) and block
+    offsets are computed on a prep stream once batch i-1's chain hash has
+    started, so their small CTAs run in the room the chain kernel leaves on
+    the SMs instead of in front of batch i's chain hash.  The compute stream
+    (higher priority, so its CTAs are placed first) then serves the batch:
+
+    insert_in_chain=True (default): batch i's chain hash runs in one launch
+    with the insert of batch i-1's uncached blocks
+    (kvgov_chain_hash_insert_prev), then batch i is probed against the table
+    as batch i-1 left it.  Batch i's own insert is left pending for the next
+    batch's chain launch (or drain()); three slots rotate, since batch i's
+    buffers are read by batch i+1's chain launch while batch i+2 is prepared.
+
+    insert_in_chain=False: the chain hash with the probe fused in, then the
+    insert of the uncached blocks; two slots.
+
+    Either way every probe sees the table exactly as the previous batch's
+    insert left it, and every step runs on the GPU; nothing here computes.
+    A cache flush (before_serve) first runs a pending insert, so that the
+    flush follows it.
     """
 
-    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_blocks: int, device="cuda"):
+    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_blocks: int, device="cuda",
+                 insert_in_chain: bool = True):
         self.cache, self.mode = cache, mode
         self.device = torch.device(device)
+        self.insert_in_chain = insert_in_chain
         self.prep_stream = torch.cuda.Stream(self.device)
         self.compute_stream = torch.cuda.Stream(self.device, priority=-1)
         cache.stream = self.compute_stream
         self.slots = []
-        for _ in range(2):
+        for _ in range(3 if insert_in_chain else 2):
             self.slots.append({
                 "salts": torch.empty((max(cache.n_principals, 1), 32), dtype=torch.uint8, device=self.device),
                 "blk_off": torch.empty(max_req + 1, dtype=torch.int64, device=self.device),
                 "digests": torch.empty((max(max_blocks, 1), 32), dtype=torch.uint8, device=self.device),
                 "prefix": torch.empty(max(max_req, 1), dtype=torch.int32, device=self.device),
-                "prepared": torch.cuda.Event(), "chain_start": torch.cuda.Event(), "free": torch.cuda.Event(),
-                "used": False,
+                "prepared": torch.cuda.Event(), "chain_start": torch.cuda.Event(), "probed": torch.cuda.Event(),
+                "free": torch.cuda.Event(), "used": False, "n": 0, "n_blocks": 0,
             })
         self.i = 0
         self.last_chain_start = None
+        self.pending = None          # the slot whose batch's insert has not run yet
 
     def _next_slot(self):
-        s = self.slots[self.i % 2]
+        s = self.slots[self.i % len(self.slots)]
         self.i += 1
         return s
 
@@ -174,66 +189,119 @@ class _Pipelined:
         if after is not None:
             ps.wait_event(after)
         if self.last_chain_start is not None:
-            ps.wait_event(self.last_chain_start)    # the slot's previous batch has finished by then
-        elif s["used"]:
-            ps.wait_event(s["free"])
+            ps.wait_event(self.last_chain_start)    # start beside the previous batch's chain hash
+        if s["used"]:
+            ps.wait_event(s["free"])                # the slot's previous batch has been inserted
         if self.mode != K.UNSALTED:
             K.derive_salts(c.secret, c.ids, c.id_off, s["salts"], c.status, ps)
         K.block_offsets(db.tok_off, s["blk_off"][:db.n + 1], c.status, ps)
         s["prepared"].record(ps)
 
-    def _serve(self, s, db: DeviceBatch, before_serve=None, chain_events=None, insert_events=None):
-        """Chain hash with the fused probe and the insert, on the compute stream."""
+    def _views(self, s):
+        return s["blk_off"][:s["n"] + 1], s["digests"][:s["n_blocks"]], s["prefix"][:s["n"]]
+
+    def _insert_pending(self):
+        """The pending batch's insert as its own launch (compute stream)."""
+        q = self.pending
+        if q is None:
+            return
+        c = self.cache
+        blk, dig, pre = self._views(q)
+        K.insert_uncached(c.slots, dig, blk, pre, c.status, c.n_new, self.compute_stream)
+        q["free"].record(self.compute_stream)
+        self.pending = None
+
+    def drain(self):
+        """Run the pending insert, if any; returns an event recorded after it
+        on the compute stream."""
+        with torch.cuda.stream(self.compute_stream):
+            self._insert_pending()
+        ev = torch.cuda.Event()
+        ev.record(self.compute_stream)
+        return ev
+
+    def _serve(self, s, db: DeviceBatch, before_serve=None, chain_events=None, table_events=None):
+        """Serve one batch on the compute stream (see the class docstring).
+        chain_events are recorded around the chain-hash launch, table_events
+        around the batch's table kernel on the critical path: its probe, or
+        its insert when the insert does not run in the next chain launch."""
         c = self.cache
         cs = self.compute_stream
         n = db.n
+        s["n"], s["n_blocks"] = n, db.n_blocks
+        blk_off, digests, prefix = self._views(s)
+        salted = self.mode != K.UNSALTED
+        kw = dict(principal=db.principal if salted else None, salts=s["salts"] if salted else None,
+                  boundary_tok=db.boundary_tok if self.mode == K.BOUNDARY else None, digests=digests,
+                  stream=cs)
         with torch.cuda.stream(cs):
             cs.wait_event(s["prepared"])
             if before_serve is not None:
+                self._insert_pending()
                 before_serve()
-            salted = self.mode != K.UNSALTED
-            blk_off = s["blk_off"][:n + 1]
             if chain_events is not None:
                 chain_events[0].record(cs)
             # the last command before the chain launch: the prep of the next
             # batch starts only once the chain kernel is being placed
             s["chain_start"].record(cs)
             self.last_chain_start = s["chain_start"]
-            digests, prefix = K.chain_hash_probe(
-                self.mode, db.tokens, db.tok_off, blk_off, c.slots, db.principal if salted else None,
-                s["salts"] if salted else None, db.boundary_tok if self.mode == K.BOUNDARY else None,
-                s["digests"][:db.n_blocks], s["prefix"][:n], n_blocks=db.n_blocks, status=c.status, stream=cs)
+            q = self.pending
+            if not self.insert_in_chain:
+                K.chain_hash_probe(self.mode, db.tokens, db.tok_off, blk_off, c.slots, prefix_blocks=prefix,
+                                   n_blocks=db.n_blocks, status=c.status, **kw)
+            elif q is not None:
+                qb, qd, qp = self._views(q)
+                K.chain_hash_insert_prev(self.mode, db.tokens, db.tok_off, blk_off, c.slots, qd, qb, qp, c.status,
+                                         n_new=c.n_new, **kw)
+            else:
+                K.chain_hash(self.mode, db.tokens, db.tok_off, blk_off, status=c.status, **kw)
             if chain_events is not None:
                 chain_events[1].record(cs)
-            if insert_events is not None:
-                insert_events[0].record(cs)
-            K.insert_uncached(c.slots, digests, blk_off, prefix, c.status, c.n_new, cs)
-            if insert_events is not None:
-                insert_events[1].record(cs)
+            if q is not None:
+                q["free"].record(cs)
+                self.pending = None
+            if table_events is not None:
+                table_events[0].record(cs)
+            if self.insert_in_chain:
+                K.probe(c.slots, digests, blk_off, prefix, c.status, cs)
+            else:
+                K.insert_uncached(c.slots, digests, blk_off, prefix, c.status, c.n_new, cs)
+            if table_events is not None:
+                table_events[1].record(cs)
+            s["probed"].record(cs)
+            if self.insert_in_chain:
+                self.pending = s
+            else:
+                s["free"].record(cs)
         s["used"] = True
         return prefix, digests, blk_off
 
 
 class DevicePipeline(_Pipelined):
     """Serve device-resident batches back to back, each batch's salts and
-    block offsets computed beside the previous batch's chain hash.
+    block offsets computed beside the previous batch's chain hash and (by
+    default) its insert run inside the next batch's chain launch.
 
     submit() returns (prefix_blocks, event) on the device: prefix_blocks is
-    valid once event has completed and is overwritten two submits later.
-    The batch's tensors are used on the pipeline's streams after the work
-    queued so far on the caller's current stream.
+    valid once event has completed and is overwritten by a later submit (the
+    second or third after it).  The batch's uncached blocks are in the table
+    once the next submit's chain launch or drain() has run.  The batch's
+    tensors are used on the pipeline's streams after the work queued so far
+    on the caller's current stream.
     """
 
-    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_blocks: int, device="cuda"):
-        super().__init__(cache, mode, max_req, max_blocks, device)
-        self._ready = [torch.cuda.Event(), torch.cuda.Event()]
+    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_blocks: int, device="cuda",
+                 insert_in_chain: bool = True):
+        super().__init__(cache, mode, max_req, max_blocks, device, insert_in_chain)
+        self._ready = [torch.cuda.Event() for _ in self.slots]
 
-    def submit(self, db: DeviceBatch, before_serve=None, chain_events=None, insert_events=None):
+    def submit(self, db: DeviceBatch, before_serve=None, chain_events=None, table_events=None):
         """Queue one device-resident batch.  before_serve, if given, is called
-        with the compute stream current just before the chain hash (for
-        instance to flush the cache); chain_events and insert_events, pairs of
-        CUDA events, are recorded around the chain-hash and insert launches."""
-        ready = self._ready[self.i % 2]
+        with the compute stream current just before the chain hash, after any
+        pending insert (for instance to flush the cache); chain_events and
+        table_events, pairs of CUDA events, are recorded around the
+        chain-hash launch and the batch's probe (or insert)."""
+        ready = self._ready[self.i % len(self.slots)]
         ready.record(torch.cuda.current_stream(self.device))
         for t in (db.tokens, db.tok_off, db.principal, db.boundary_tok):
             t.record_stream(self.prep_stream)
@@ -241,25 +309,26 @@ class DevicePipeline(_Pipelined):
         self.compute_stream.wait_event(ready)
         s = self._next_slot()
         self._prepare(s, db, after=ready)
-        prefix, _, _ = self._serve(s, db, before_serve, chain_events, insert_events)
-        s["free"].record(self.compute_stream)
-        return prefix, s["free"]
+        prefix, _, _ = self._serve(s, db, before_serve, chain_events, table_events)
+        return prefix, s["probed"]
 
 
 class HostPipeline(_Pipelined):
     """Serve batches that live in pinned host memory: each batch's
     host-to-device copy runs on a copy stream while the previous batch is
-    served, its salts and block offsets follow on the prep stream, and the
-    compute stream serves it and copies the prefix lengths back into a pinned
-    host buffer.  A slot is reused only after the compute stream has finished
-    with it.
+    served, its salts and block offsets follow on the prep stream, the
+    compute stream serves it as in DevicePipeline and copies its prefix
+    lengths back into a pinned host buffer.  A slot's buffers are reused
+    only after its batch has been inserted.
 
     submit() returns (prefix_host, event): prefix_host is valid once event has
-    completed (event.synchronize()) and is overwritten two submits later.
+    completed (event.synchronize()) and is overwritten by a later submit (the
+    second or third after it).
     """
 
-    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_tokens: int, device="cuda"):
-        super().__init__(cache, mode, max_req, max_tokens // K.BLOCK, device)
+    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_tokens: int, device="cuda",
+                 insert_in_chain: bool = True):
+        super().__init__(cache, mode, max_req, max_tokens // K.BLOCK, device, insert_in_chain)
         self.copy_stream = torch.cuda.Stream(self.device)
         for s in self.slots:
             s.update({
@@ -268,7 +337,7 @@ class HostPipeline(_Pipelined):
                 "principal": torch.empty(max(max_req, 1), dtype=torch.int32, device=self.device),
                 "boundary_tok": torch.empty(max(max_req, 1), dtype=torch.int32, device=self.device),
                 "out": torch.empty(max(max_req, 1), dtype=torch.int32).pin_memory(),
-                "copied": torch.cuda.Event(),
+                "copied": torch.cuda.Event(), "out_done": torch.cuda.Event(),
             })
 
     def submit(self, tokens, tok_off, principal, boundary_tok, n_blocks: int, before_serve=None,
@@ -276,13 +345,14 @@ class HostPipeline(_Pipelined):
         """Queue one batch given as pinned host tensors (int32 tokens, int64
         offsets, int32 principal rows and boundary offsets).  before_serve, if
         given, is called with the compute stream current just before the
-        chain hash (for instance to flush the cache); chain_events as in
-        DevicePipeline.submit."""
+        chain hash, after any pending insert (for instance to flush the
+        cache); chain_events as in DevicePipeline.submit."""
         s = self._next_slot()
         n, t = tok_off.numel() - 1, tokens.numel()
         with torch.cuda.stream(self.copy_stream):
             if s["used"]:
                 self.copy_stream.wait_event(s["free"])
+                self.copy_stream.wait_event(s["out_done"])
             s["tokens"][:t].copy_(tokens, non_blocking=True)
             s["tok_off"][:n + 1].copy_(tok_off, non_blocking=True)
             s["principal"][:n].copy_(principal, non_blocking=True)
@@ -294,5 +364,5 @@ class HostPipeline(_Pipelined):
         prefix, _, _ = self._serve(s, db, before_serve, chain_events)
         with torch.cuda.stream(self.compute_stream):
             s["out"][:n].copy_(prefix, non_blocking=True)
-            s["free"].record(self.compute_stream)
-        return s["out"][:n], s["free"]
+            s["out_done"].record(self.compute_stream)
+        return s["out"][:n], s["out_done"]

@@ -464,6 +464,80 @@ def test_chain_hash_probe_matches_separate_calls(kv, mode, fill, n_req):
     assert (pre.cpu().numpy() == pref).all() and (pre_sep.cpu().numpy() == pref).all()
 
 
+@pytest.mark.parametrize("mode", [0, 1, 2])
+@pytest.mark.parametrize("n_req,prev_n", [(180, 150), (40960, 40960), (40960, 90000), (40960, 0), (0, 300)],
+                         ids=["two_launches", "fused", "fused_more_prev", "no_prev", "empty_batch"])
+def test_chain_hash_insert_prev_matches_separate_calls(kv, mode, n_req, prev_n):
+    """kvgov_chain_hash_insert_prev writes kvgov_chain_hash's digests and
+    leaves the table, key count and flags of kvgov_insert_uncached on the
+    previous batch: on a batch small enough to take two launches, on fused
+    batches (the previous one with more requests than the grid has threads,
+    or none), and with an empty batch.  The previous batch holds a reserved
+    key, a request whose prefix covers it whole, and out-of-range prefixes."""
+    rng = np.random.default_rng(n_req + prev_n + mode)
+    lengths = list(rng.integers(0, 200, n_req)) if n_req else []
+    b = W.ragged(19 + mode, lengths) if n_req else None
+    salts = oracle.derive_salts(b"prev", *W.principal_ids(8))
+    # the previous batch: random keys, a third of them present already
+    pnb = rng.integers(0, 12, prev_n)
+    if prev_n:
+        pnb[0] = max(int(pnb[0]), 1)
+    poff = np.concatenate([[0], np.cumsum(pnb)]).astype(np.int64)
+    pdig = keys_np(int(poff[-1]), 5 + mode) if prev_n else np.zeros((0, 32), np.uint8)
+    ppre = rng.integers(-2, 14, prev_n).astype(np.int32)      # < 0 reads as 0, > n_b as n_b
+    if prev_n:
+        pdig[0] = 0                                           # a reserved (all-zero) key, uncached
+        ppre[0] = 0
+    present = pdig[rng.random(len(pdig)) < 0.3] if prev_n else pdig
+    cap = 1 << 20
+    def fresh_table():
+        slots = kv.new_table(cap)
+        st = status_tensor()
+        if len(present):
+            kv.insert(slots, dev(present[present.any(axis=1)]), st)
+        return slots
+    slots_a, slots_b = fresh_table(), fresh_table()
+    st_a, st_b = status_tensor(), status_tensor()
+    n_a = torch.zeros(1, dtype=torch.int64, device=DEV)
+    n_b = torch.zeros(1, dtype=torch.int64, device=DEV)
+    d_pdig, d_poff, d_ppre = dev(pdig), dev(poff), dev(ppre)
+    if n_req:
+        toks, tok_off = dev(b.tokens, np.int32), dev(b.tok_off, np.int64)
+        pr, bt = dev(b.principal, np.int32), dev(b.boundary_tok, np.int32)
+    else:
+        toks, tok_off = torch.zeros(4, dtype=torch.int32, device=DEV), torch.zeros(1, dtype=torch.int64, device=DEV)
+        # no requests; the salted modes still take non-NULL principal and boundary arrays
+        pr, bt = torch.zeros(1, dtype=torch.int32, device=DEV), torch.zeros(1, dtype=torch.int32, device=DEV)
+    blk = kv.block_offsets(tok_off, status=st_a)
+    nbk = int(blk[-1].item())
+    d_salts = dev(salts) if mode else None
+    pr_, bt_ = (pr if mode else None), (bt if mode == 2 else None)
+    d_a = kv.chain_hash_insert_prev(mode, toks, tok_off, blk, slots_a, d_pdig, d_poff, d_ppre, st_a,
+                                    principal=pr_, salts=d_salts, boundary_tok=bt_, n_blocks=nbk, n_new=n_a)
+    d_b = kv.chain_hash(mode, toks, tok_off, blk, pr_, d_salts, bt_, n_blocks=nbk, status=st_b)
+    kv.insert_uncached(slots_b, d_pdig, d_poff, d_ppre, st_b, n_b)
+    torch.cuda.synchronize()
+    assert int(st_a.item()) == int(st_b.item())
+    if prev_n:
+        assert int(st_a.item()) & kv.F_SENTINEL
+    assert (d_a.cpu().numpy() == d_b.cpu().numpy()).all()
+    assert int(n_a.item()) == int(n_b.item())
+    assert table_contents(slots_a) == table_contents(slots_b)
+    if n_req:
+        ref = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+        assert (d_a.cpu().numpy() == ref).all()
+    # the oracle's set: the keys present before plus every uncached key of the previous batch
+    ks = oracle.KeySet(1)
+    ks.insert(present[present.any(axis=1)])
+    before = ks.n
+    rows = [np.arange(poff[r] + min(max(int(ppre[r]), 0), pnb[r]), poff[r + 1]) for r in range(prev_n)]
+    rows = np.concatenate(rows + [np.zeros(0, np.int64)]).astype(np.int64)
+    new_keys = pdig[rows]
+    ks.insert(new_keys[new_keys.any(axis=1)])
+    assert int(n_a.item()) == ks.n - before
+    assert table_contents(slots_a) == {r.tobytes() for r in ks.contents()}
+
+
 def test_probe_empty_and_bad_offsets(kv):
     slots = kv.new_table(64)
     st = status_tensor()

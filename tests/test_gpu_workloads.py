@@ -145,7 +145,8 @@ def test_full_wide_serving_steps(kv):
     assert seen == [0, 4, 8]
 
 
-def test_host_pipeline_matches_device_serving(kv):
+@pytest.mark.parametrize("in_chain", [True, False], ids=["insert_in_chain", "inline"])
+def test_host_pipeline_matches_device_serving(kv, in_chain):
     """Batches served from pinned host memory through HostPipeline (copies
     overlapping the previous batch's serving; each batch's result read only
     after the next batch is queued) give the prefix lengths of the same
@@ -157,7 +158,7 @@ def test_host_pipeline_matches_device_serving(kv):
     dev_cache = PrefixCache(1 << 18, w0.secret, w0.ids, w0.id_off)
     host_cache = PrefixCache(1 << 18, w0.secret, w0.ids, w0.id_off)
     n_tok = int(w0.batch.tok_off[-1])
-    pipe = HostPipeline(host_cache, W.BOUNDARY, w0.batch.n, n_tok)
+    pipe = HostPipeline(host_cache, W.BOUNDARY, w0.batch.n, n_tok, insert_in_chain=in_chain)
     order = [0, 1, 2, 0, 3, 1]
     got, want, pending = [], [], None
     for i, k in enumerate(order):
@@ -177,6 +178,7 @@ def test_host_pipeline_matches_device_serving(kv):
         pending = (out, ev)
     pending[1].synchronize()
     got.append(pending[0].numpy().copy())
+    pipe.drain()
     torch.cuda.synchronize()
     dev_cache.check_status()
     host_cache.check_status()
@@ -186,12 +188,14 @@ def test_host_pipeline_matches_device_serving(kv):
     assert [int(x.min()) for x in want] == [0, 4, 4, 8, 4, 4]
 
 
+@pytest.mark.parametrize("in_chain", [True, False], ids=["insert_in_chain", "inline"])
 @pytest.mark.parametrize("mode", [W.UNSALTED, W.ROOT, W.BOUNDARY])
-def test_device_pipeline_matches_sequential_serving(kv, mode):
+def test_device_pipeline_matches_sequential_serving(kv, mode, in_chain):
     """DevicePipeline (salts and block offsets of batch i+1 on a prep stream
-    beside batch i's insert) gives the prefix lengths and the key count of
-    serving the same batches one by one, across secret changes and a flush
-    of the cache between batches."""
+    beside batch i's chain hash; batch i's insert inside batch i+1's chain
+    launch, or inline) gives the prefix lengths and the key count of serving
+    the same batches one by one, across secret changes and a flush of the
+    cache between batches."""
     ws = [W.make("wide", seed=300 + i, n_req=20000) for i in range(3)]
     for w in ws[1:]:
         w.batch.tokens.reshape(-1, 128)[:, :64] = ws[0].batch.tokens[:64]
@@ -200,7 +204,7 @@ def test_device_pipeline_matches_sequential_serving(kv, mode):
            for w in ws]
     seq = PrefixCache(1 << 19, w0.secret, w0.ids, w0.id_off)
     pip = PrefixCache(1 << 19, w0.secret, w0.ids, w0.id_off)
-    pipe = DevicePipeline(pip, mode, w0.batch.n, dbs[0].n_blocks)
+    pipe = DevicePipeline(pip, mode, w0.batch.n, dbs[0].n_blocks, insert_in_chain=in_chain)
     order = [0, 1, 2, 0, 1, 2, 0]
     got, want = [], []
     for i, k in enumerate(order):
@@ -216,6 +220,7 @@ def test_device_pipeline_matches_sequential_serving(kv, mode):
         out, ev = pipe.submit(dbs[k], before)
         ev.synchronize()
         got.append(out.cpu().numpy())
+    pipe.drain()
     torch.cuda.synchronize()
     seq.check_status()
     pip.check_status()
@@ -227,8 +232,9 @@ def test_device_pipeline_matches_sequential_serving(kv, mode):
         assert int(want[1].min()) == 4
 
 
+@pytest.mark.parametrize("in_chain", [True, False], ids=["insert_in_chain", "inline"])
 @pytest.mark.parametrize("flush_at", [None, 5])
-def test_device_pipeline_back_to_back_matches_oracle(kv, flush_at):
+def test_device_pipeline_back_to_back_matches_oracle(kv, flush_at, in_chain):
     """Many batches queued without waiting in between (and a cache flush
     queued in the middle): every batch's prefix lengths, copied out on the
     compute stream right after its submit, match the oracle's replay of the
@@ -240,7 +246,7 @@ def test_device_pipeline_back_to_back_matches_oracle(kv, flush_at):
     dbs = [DeviceBatch.from_host(w.batch.tokens, w.batch.tok_off, w.batch.principal, w.batch.boundary_tok)
            for w in ws]
     cache = PrefixCache(1 << 17, w0.secret, w0.ids, w0.id_off)
-    pipe = DevicePipeline(cache, W.BOUNDARY, w0.batch.n, dbs[0].n_blocks)
+    pipe = DevicePipeline(cache, W.BOUNDARY, w0.batch.n, dbs[0].n_blocks, insert_in_chain=in_chain)
     order = [0, 1, 2, 3, 2, 0, 1, 3]
     copies = []
     for i, k in enumerate(order):
@@ -249,6 +255,7 @@ def test_device_pipeline_back_to_back_matches_oracle(kv, flush_at):
         pre, _ = pipe.submit(dbs[k], before)
         with torch.cuda.stream(pipe.compute_stream):
             copies.append(pre.clone())
+    pipe.drain()
     torch.cuda.synchronize()
     cache.check_status()
     ks, before_flush = oracle.KeySet(1), 0
