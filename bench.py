@@ -398,9 +398,9 @@ def main():
     ap.add_argument("--cpu-sample", type=int, default=16384, help="requests per oracle step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--schedule", default="insert_in_chain", choices=["insert_in_chain", "inline"],
-                    help="insert_in_chain: each batch's insert runs inside the next batch's chain launch and the "
-                         "batch is probed after its chain hash; inline: chain hash with the fused probe, then the "
-                         "insert")
+                    help="insert_in_chain: each batch's insert runs inside the next batch's chain-hash launch, and "
+                         "each batch is probed after its chain hash; inline: chain hash with the fused probe, then "
+                         "the insert")
     ap.add_argument("--configs", action="store_true",
                     help="instead of the timed serving step: per-kernel rates on every workload, one JSON line each")
     ap.add_argument("--only", default=None,
@@ -465,6 +465,7 @@ def main():
     pipe = DevicePipeline(cache, W.BOUNDARY, n_req, n_blocks, insert_in_chain=in_chain)
     epoch = [1]
     launches = [0]
+    table_timed = []
 
     def step(db, ev=None, tab_ev=None):
         cache.set_secret(epoch_secret(w0.secret, epoch[0]))
@@ -472,15 +473,25 @@ def main():
         flushed = flush.before_step()              # load factor would pass 0.5: flush the cache
         before = (lambda: K.table_init(cache.slots, pipe.compute_stream)) if flushed else None
         pending = pipe.pending is not None
+        if in_chain and (flushed or not pending):
+            tab_ev = None                          # this step runs no probe of its own (chain hash + fused probe)
+        if tab_ev is not None:
+            table_timed.append(tab_ev)
         prefix, _ = pipe.submit(db, before, ev, tab_ev)
-        # salts, block offsets (2), the chain hash (with the previous batch's insert, or with the probe fused
-        # in), the probe (or the insert); a flush adds the table init and, in_chain, the pending insert
-        launches[0] += 5 + (int(flushed) * (1 + int(pending)) if in_chain else int(flushed))
+        if in_chain:
+            # salts, block offsets (2), then the chain hash with the previous batch's insert and the probe or,
+            # after a flush (which runs the pending insert and the table init first), the chain hash with
+            # the probe fused in
+            launches[0] += 3 + (2 + int(pending) if flushed else (2 if pending else 1))
+        else:
+            # salts, block offsets (2), chain hash with the fused probe, insert (+ table init)
+            launches[0] += 5 + int(flushed)
         return prefix
 
     for i in range(args.warmup):
         step(pool[(1 + i) % args.pool])
     torch.cuda.synchronize()
+    table_timed.clear()
     n_new_before = int(cache.n_new.item())
 
     chain_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -519,7 +530,7 @@ def main():
     kernel_launches = launches[0]
     ms = t_start.elapsed_time(t_stop)
     chain_ms = float(np.mean([a.elapsed_time(b) for a, b in chain_ev]))
-    table_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in table_ev if e is not None]))
+    table_ms = float(np.mean([a.elapsed_time(b) for a, b in table_timed]))
     inserted_per_step = (gate["n_new_total"] - n_new_before) / args.steps
     ms = max_over_ranks(ms, world, dist, "cuda")
     value = world * args.steps * n_blocks / (ms / 1e3)
@@ -528,7 +539,7 @@ def main():
     arrival = arrival_leg(torch, K, W, pool, n_req, n_blocks, cache, args.arrival_steps, chain_ms)
 
     # ---- end to end through the public API with host buffers
-    e2e = e2e_leg(torch, K, W, w0, pool_host[: min(4, args.pool)], args.e2e_steps, world, dist, args.table_slots)
+    e2e = e2e_leg(torch, K, W, w0, pool_host[: min(4, args.pool)], args.e2e_steps, world, dist, args.table_slots, in_chain)
 
     # ---- roofline of the chain kernel (integer-pipe bound)
     micro = measure_int_peak(torch, kbuild.PEAK_LIB)
@@ -675,7 +686,7 @@ def arrival_leg(torch, K, W, pool, n_req, n_blocks, cache, steps, chain_ms):
             "cache": f"empty {cap}-slot table per batch (re-initialised outside the timed call)"}
 
 
-def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots):
+def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots, in_chain=True):
     """Same step with host buffers, through the public HostPipeline: each
     step's inputs are copied from pinned host memory (a copy stream, which
     overlaps the previous step's serving) and its prefix lengths are copied
@@ -690,7 +701,7 @@ def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots):
     n_tok = int(hosts[0].batch.tok_off[-1])
     n_blocks = int((hosts[0].batch.lengths() // 16).sum())
     cache = PrefixCache(table_slots, w0.secret, w0.ids, w0.id_off)
-    pipe = HostPipeline(cache, W.BOUNDARY, n_req, n_tok)
+    pipe = HostPipeline(cache, W.BOUNDARY, n_req, n_tok, insert_in_chain=in_chain)
     flush = FlushPolicy(table_slots, 4 * n_req)
     h2d = sum(t.numel() * t.element_size() for t in pinned[0])
     d2h = n_req * 4

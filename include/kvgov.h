@@ -319,35 +319,39 @@ int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_
                           unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream);
 
 /*
- * kvgov_chain_hash_insert_prev -- kvgov_chain_hash of one batch and, in the
- * same launch, kvgov_insert_uncached of the previous batch (paper section
- * 2.1: a served request's uncached blocks are computed and cached).  In a
- * stream of batches, batch i+1's chain hash does not read the table, so
- * batch i's insert can run inside it: each thread inserts uncached blocks of
- * the previous batch between its own compressions, and the memory latency of
- * the inserts is covered by the other warps' hashing.  The digests equal
- * kvgov_chain_hash's; the table, *d_n_new and the insert flags equal
- * kvgov_insert_uncached's on the previous batch.
+ * kvgov_chain_hash_insert_prev -- kvgov_chain_hash of one batch with, in the
+ * same launch, kvgov_insert_uncached of the previous batch, and (if
+ * d_prefix_blocks is given) kvgov_probe of this batch after that insert
+ * (paper section 2.1: a served request's uncached blocks are computed and
+ * cached; the next lookups see them).  In a stream of batches, batch i+1's
+ * chain hash does not touch the table, so batch i's insert can run inside
+ * it: each thread inserts uncached blocks of the previous batch between its
+ * own compressions, and the inserts' memory latency is covered by the other
+ * warps' hashing.  Results: the digests of kvgov_chain_hash; the table,
+ * *d_n_new and the insert flags of kvgov_insert_uncached on the previous
+ * batch; the prefix lengths of kvgov_probe of this batch on the table after
+ * that insert (a second launch).
  *   mode .. d_digests  as for kvgov_chain_hash (this batch).
  *   d_slots, capacity  the table (as for kvgov_insert).
  *   d_prev_digests, d_prev_blk_off, prev_n_req, d_prev_prefix_blocks
  *              the previous batch, as for kvgov_insert_uncached; its arrays
- *              must not overlap this batch's d_digests.  prev_n_req = 0:
- *              kvgov_chain_hash alone.
+ *              must not overlap this batch's d_digests.  prev_n_req = 0: no
+ *              insert.
+ *   d_prefix_blocks  [n_req] int32 output, or NULL for no probe.
  *   d_n_new, d_status  as for kvgov_insert_uncached (d_status required).
- * The table must not be read or written by other calls while this one runs
- * (probe this batch after it).  A batch too small to give every SM
- * sub-partition two warps (n_req < 2 * 32 * 4 * SMs) runs the chain hash and
- * the insert as two launches instead; the results are the same.  EINVAL: as
- * for kvgov_chain_hash and kvgov_insert_uncached, prev_n_req < 0.
+ * The table must not be read or written by other calls while this one runs.
+ * A batch too small to give every SM sub-partition two warps (n_req < 2 * 32
+ * * 4 * SMs) runs the chain hash and the insert as separate launches
+ * instead; the results are the same.  EINVAL: as for kvgov_chain_hash and
+ * kvgov_insert_uncached, prev_n_req < 0.
  */
 int kvgov_chain_hash_insert_prev(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
                                  const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
                                  const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
                                  uint8_t *d_slots, uint64_t capacity, const uint8_t *d_prev_digests,
                                  const int64_t *d_prev_blk_off, int32_t prev_n_req,
-                                 const int32_t *d_prev_prefix_blocks, unsigned long long *d_n_new,
-                                 uint32_t *d_status, kvgov_stream_t stream);
+                                 const int32_t *d_prev_prefix_blocks, int32_t *d_prefix_blocks,
+                                 unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream);
 
 /*
  * Arrival-order serving of one batch -- paper section 2.1 (a lookup matches

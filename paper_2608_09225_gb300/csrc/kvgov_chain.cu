@@ -217,6 +217,7 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
     const long long pstride = (long long)gridDim.x * kR;
     long long pq = r, prow = 0;
     long long pleft = 0;
+    uint2 wl = make_uint2(0u, 0u);               // first digest word of row prow + 1
     auto prev_next = [&]() {                     // from pq on: the first request with uncached blocks
         for (; pq < q.n_req; pq += pstride) {
             const long long base = q.blk_off[pq], pnb = q.blk_off[pq + 1] - base;
@@ -229,12 +230,20 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             if (pnb > L) {
                 prow = base + L;
                 pleft = pnb - L;
+                if (pleft > 1) wl = __ldg(reinterpret_cast<const uint2 *>(q.digests + 2 * (prow + 1)));
                 return;
             }
         }
         pleft = 0;
     };
+    // Each call prefetches the home slot of the next key into L2 (from the
+    // digest word the previous call loaded) and loads the word of the key
+    // after it, so that no insert but a request's first waits on DRAM and no
+    // load is waited for.
     auto prev_insert_one = [&]() {               // insert row prow of the previous batch
+        if (pleft > 1) prefetch_l2(q.slots + 4 * (u64_of(wl.x, wl.y) & q.mask));
+        uint2 wn = make_uint2(0u, 0u);
+        if (pleft > 2) wn = __ldg(reinterpret_cast<const uint2 *>(q.digests + 2 * (prow + 2)));
         const uint4 x = __ldg(q.digests + 2 * prow), y = __ldg(q.digests + 2 * prow + 1);
         const unsigned long long key[4] = {u64_of(x.x, x.y), u64_of(x.z, x.w), u64_of(y.x, y.y), u64_of(y.z, y.w)};
         if (key_reserved(key)) {
@@ -243,6 +252,7 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             unsigned long long pos = 0;
             count_insert(insert_one(q.slots, q.mask, key, q.spin_limit, &pos), my_new, my_flags);
         }
+        wl = wn;
         ++prow;
         if (--pleft == 0) {
             pq += pstride;
@@ -354,8 +364,10 @@ __global__ void __launch_bounds__(kR) chain_arrival_kernel(const ChainParams p, 
     chain_body<MODE, kFuseArrival>(p, a);
 }
 
+// At most 64 registers, so that 8 CTAs fit an SM: the batch's CTAs leave
+// room beside them for the next batch's salts and block offsets.
 template <int MODE>
-__global__ void __launch_bounds__(kR) chain_prev_kernel(const ChainParams p, const PrevParams q) {
+__global__ void __launch_bounds__(kR, 8) chain_prev_kernel(const ChainParams p, const PrevParams q) {
     chain_body<MODE, kFuseInsertPrev>(p, ArrivalParams{}, q);
 }
 
@@ -403,6 +415,7 @@ struct FuseArgs {
     const int64_t *prev_blk_off = nullptr;
     int32_t prev_n_req = 0;
     const int32_t *prev_prefix_blocks = nullptr;
+    int32_t *probe_prefix_blocks = nullptr;     // kFuseInsertPrev: probe this batch after the insert
 };
 
 int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
@@ -466,13 +479,27 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     // the chain; there they run as separate launches (same results).
     const DeviceInfo dev = device_info();
     const long long min_fused = 2ll * 32 * 4 * (dev.sms > 0 ? dev.sms : 152);
-    const bool none = f.fuse == kFuseNone || (f.fuse == kFuseInsertPrev && f.prev_n_req == 0);
+    if (f.fuse == kFuseInsertPrev) {
+        int rc;
+        if (f.prev_n_req > 0 && n_req >= min_fused) {
+            launch_chain_kernel<kFuseInsertPrev>(mode, grid, s, p, a, q);
+            rc = kvgov_host::launch_status();
+        } else {                                   // a small batch (or no insert): separate launches
+            launch_chain_kernel<kFuseNone>(mode, grid, s, p);
+            rc = kvgov_host::launch_status();
+            if (rc == KVGOV_OK && f.prev_n_req > 0) rc = insert_prev();
+        }
+        if (rc == KVGOV_OK && f.probe_prefix_blocks)
+            rc = kvgov_probe(f.slots, f.capacity, d_digests, d_blk_off, n_req, f.probe_prefix_blocks, d_status,
+                             stream);
+        return rc;
+    }
+    const bool none = f.fuse == kFuseNone;
     const bool fused = !none && n_req >= min_fused;
     if (!fused) {
         launch_chain_kernel<kFuseNone>(mode, grid, s, p);
         int rc = kvgov_host::launch_status();
         if (rc != KVGOV_OK || none) return rc;
-        if (f.fuse == kFuseInsertPrev) return insert_prev();
         if (f.fuse == kFuseProbe)
             return kvgov_probe(f.slots, f.capacity, d_digests, d_blk_off, n_req, f.prefix_blocks, d_status, stream);
         rc = kvgov_insert_arrival(const_cast<uint8_t *>(f.slots), f.owner, f.capacity, d_digests, d_blk_off, n_req,
@@ -483,10 +510,6 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     }
     if (f.fuse == kFuseProbe) {
         launch_chain_kernel<kFuseProbe>(mode, grid, s, p);
-        return kvgov_host::launch_status();
-    }
-    if (f.fuse == kFuseInsertPrev) {
-        launch_chain_kernel<kFuseInsertPrev>(mode, grid, s, p, a, q);
         return kvgov_host::launch_status();
     }
     launch_chain_kernel<kFuseArrival>(mode, grid, s, p, a);
@@ -547,9 +570,11 @@ extern "C" int kvgov_chain_hash_insert_prev(int mode, const int32_t *d_tokens, c
                                             uint8_t *d_digests, uint8_t *d_slots, uint64_t capacity,
                                             const uint8_t *d_prev_digests, const int64_t *d_prev_blk_off,
                                             int32_t prev_n_req, const int32_t *d_prev_prefix_blocks,
-                                            unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream) {
+                                            int32_t *d_prefix_blocks, unsigned long long *d_n_new,
+                                            uint32_t *d_status, kvgov_stream_t stream) {
     FuseArgs f;
     f.fuse = kFuseInsertPrev;
+    f.probe_prefix_blocks = d_prefix_blocks;
     f.slots = d_slots;
     f.capacity = capacity;
     f.n_new = d_n_new;

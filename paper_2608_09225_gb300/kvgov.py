@@ -58,7 +58,7 @@ def _load():
                                              _p, _p, ctypes.c_uint64, _p, _p, _p]
         L.kvgov_chain_hash_insert_prev.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32,
                                                    _p, _p, _p, _p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p,
-                                                   _p, _p]
+                                                   _p, _p, _p]
         L.kvgov_table_init.argtypes = [_p, ctypes.c_uint64, _p]
         L.kvgov_insert.argtypes = [_p, ctypes.c_uint64, _p, ctypes.c_int64, _p, _p, _p]
         L.kvgov_probe.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p]
@@ -217,10 +217,11 @@ def chain_hash_insert_prev(mode: int, tokens: torch.Tensor, tok_off: torch.Tenso
                            principal: torch.Tensor | None = None, salts: torch.Tensor | None = None,
                            boundary_tok: torch.Tensor | None = None, digests: torch.Tensor | None = None,
                            n_blocks: int | None = None, n_new: torch.Tensor | None = None,
-                           stream=None) -> torch.Tensor:
-    """chain_hash of this batch and insert_uncached of the previous batch
-    (prev_digests, prev_blk_off, prev_prefix_blocks) in one launch; returns
-    this batch's digests."""
+                           prefix_blocks: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """chain_hash of this batch with insert_uncached of the previous batch
+    (prev_digests, prev_blk_off, prev_prefix_blocks) and, if prefix_blocks
+    is given, the probe of this batch after that insert; returns this
+    batch's digests."""
     L = lib()
     n = tok_off.numel() - 1
     pn = prev_blk_off.numel() - 1
@@ -240,6 +241,8 @@ def chain_hash_insert_prev(mode: int, tokens: torch.Tensor, tok_off: torch.Tenso
         _dev(prev_digests, torch.uint8, "prev_digests") if prev_digests.numel() else _dummy(tokens),
         _dev(prev_blk_off, torch.int64, "prev_blk_off"), pn,
         _dev(prev_prefix_blocks, torch.int32, "prev_prefix_blocks") if pn else _dummy(tokens),
+        (_dev(prefix_blocks, torch.int32, "prefix_blocks") if n else _dummy(tokens))
+        if prefix_blocks is not None else None,
         _dev(n_new, torch.int64, "n_new", True), _dev(status, torch.int32, "status"), _stream(stream)),
         "kvgov_chain_hash_insert_prev")
     return digests

@@ -223,8 +223,9 @@ class _Pipelined:
     def _serve(self, s, db: DeviceBatch, before_serve=None, chain_events=None, table_events=None):
         """Serve one batch on the compute stream (see the class docstring).
         chain_events are recorded around the chain-hash launch, table_events
-        around the batch's table kernel on the critical path: its probe, or
-        its insert when the insert does not run in the next chain launch."""
+        around the batch's table kernel after it: the probe (when the chain
+        launch carried the previous batch's insert) or the insert
+        (insert_in_chain=False)."""
         c = self.cache
         cs = self.compute_stream
         n = db.n
@@ -245,29 +246,31 @@ class _Pipelined:
             # batch starts only once the chain kernel is being placed
             s["chain_start"].record(cs)
             self.last_chain_start = s["chain_start"]
-            q = self.pending
-            if not self.insert_in_chain:
-                K.chain_hash_probe(self.mode, db.tokens, db.tok_off, blk_off, c.slots, prefix_blocks=prefix,
-                                   n_blocks=db.n_blocks, status=c.status, **kw)
-            elif q is not None:
+            q = self.pending if self.insert_in_chain else None
+            if q is not None:
                 qb, qd, qp = self._views(q)
                 K.chain_hash_insert_prev(self.mode, db.tokens, db.tok_off, blk_off, c.slots, qd, qb, qp, c.status,
                                          n_new=c.n_new, **kw)
             else:
-                K.chain_hash(self.mode, db.tokens, db.tok_off, blk_off, status=c.status, **kw)
+                K.chain_hash_probe(self.mode, db.tokens, db.tok_off, blk_off, c.slots, prefix_blocks=prefix,
+                                   n_blocks=db.n_blocks, status=c.status, **kw)
             if chain_events is not None:
                 chain_events[1].record(cs)
             if q is not None:
+                if table_events is not None:
+                    table_events[0].record(cs)
+                K.probe(c.slots, digests, blk_off, prefix, c.status, cs)
+                if table_events is not None:
+                    table_events[1].record(cs)
+            if q is not None:
                 q["free"].record(cs)
                 self.pending = None
-            if table_events is not None:
-                table_events[0].record(cs)
-            if self.insert_in_chain:
-                K.probe(c.slots, digests, blk_off, prefix, c.status, cs)
-            else:
+            if not self.insert_in_chain:
+                if table_events is not None:
+                    table_events[0].record(cs)
                 K.insert_uncached(c.slots, digests, blk_off, prefix, c.status, c.n_new, cs)
-            if table_events is not None:
-                table_events[1].record(cs)
+                if table_events is not None:
+                    table_events[1].record(cs)
             s["probed"].record(cs)
             if self.insert_in_chain:
                 self.pending = s
@@ -300,7 +303,8 @@ class DevicePipeline(_Pipelined):
         with the compute stream current just before the chain hash, after any
         pending insert (for instance to flush the cache); chain_events and
         table_events, pairs of CUDA events, are recorded around the
-        chain-hash launch and the batch's probe (or insert)."""
+        chain-hash launch and the table kernel after it (the probe, or the
+        insert)."""
         ready = self._ready[self.i % len(self.slots)]
         ready.record(torch.cuda.current_stream(self.device))
         for t in (db.tokens, db.tok_off, db.principal, db.boundary_tok):

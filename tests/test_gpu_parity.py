@@ -538,6 +538,64 @@ def test_chain_hash_insert_prev_matches_separate_calls(kv, mode, n_req, prev_n):
     assert table_contents(slots_a) == {r.tobytes() for r in ks.contents()}
 
 
+@pytest.mark.parametrize("mode", [0, 1, 2])
+@pytest.mark.parametrize("n_req", [180, 40960], ids=["separate_launches", "fused"])
+def test_chain_hash_insert_prev_with_probe(kv, mode, n_req):
+    """With a prefix output, kvgov_chain_hash_insert_prev gives this batch's
+    digests, the previous batch's insert, and this batch's prefix lengths
+    against the table after that insert -- the results of kvgov_chain_hash,
+    kvgov_insert_uncached and kvgov_probe in sequence.  The previous batch
+    shares keys with this one, so the probe must see the insert."""
+    rng = np.random.default_rng(7 * n_req + mode)
+    lengths = list(rng.integers(0, 300, n_req))
+    b = W.ragged(23 + mode, lengths)
+    salts = oracle.derive_salts(b"probe-after-insert", *W.principal_ids(8))
+    ref = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+    blk_ref = oracle.block_offsets(b.tok_off)
+    # the previous batch: this batch's digests of every third request (so its insert makes them hit), plus
+    # random keys; its prefix lengths cut some requests short
+    prev_req = np.arange(0, n_req, 3)
+    prev_rows = [ref[blk_ref[r]:blk_ref[r + 1]] for r in prev_req]
+    pnb = np.array([len(x) for x in prev_rows], np.int64)
+    poff = np.concatenate([[0], np.cumsum(pnb)]).astype(np.int64)
+    pdig = np.concatenate(prev_rows + [np.zeros((0, 32), np.uint8)])
+    ppre = np.where(rng.random(len(prev_req)) < 0.2, rng.integers(0, 5, len(prev_req)), 0).astype(np.int32)
+    present = ref[rng.random(len(ref)) < 0.05]                 # a few keys cached before
+    cap = 1 << 21
+    slots_a, slots_b = kv.new_table(cap), kv.new_table(cap)
+    st_a, st_b = status_tensor(), status_tensor()
+    for sl in (slots_a, slots_b):
+        kv.insert(sl, dev(present), st_b)
+    n_a = torch.zeros(1, dtype=torch.int64, device=DEV)
+    n_b = torch.zeros(1, dtype=torch.int64, device=DEV)
+    toks, tok_off = dev(b.tokens, np.int32), dev(b.tok_off, np.int64)
+    pr, bt = dev(b.principal, np.int32), dev(b.boundary_tok, np.int32)
+    d_salts = dev(salts) if mode else None
+    pr_, bt_ = (pr if mode else None), (bt if mode == 2 else None)
+    blk = kv.block_offsets(tok_off, status=st_a)
+    d_pdig, d_poff, d_ppre = dev(pdig), dev(poff), dev(ppre)
+    pre_a = torch.full((n_req,), -5, dtype=torch.int32, device=DEV)
+    d_a = kv.chain_hash_insert_prev(mode, toks, tok_off, blk, slots_a, d_pdig, d_poff, d_ppre, st_a,
+                                    principal=pr_, salts=d_salts, boundary_tok=bt_, n_blocks=len(ref), n_new=n_a,
+                                    prefix_blocks=pre_a)
+    d_b = kv.chain_hash(mode, toks, tok_off, blk, pr_, d_salts, bt_, n_blocks=len(ref), status=st_b)
+    kv.insert_uncached(slots_b, d_pdig, d_poff, d_ppre, st_b, n_b)
+    pre_b = kv.probe(slots_b, d_b, blk, status=st_b)
+    torch.cuda.synchronize()
+    assert int(st_a.item()) == 0 and int(st_b.item()) == 0
+    assert (d_a.cpu().numpy() == ref).all() and (d_b.cpu().numpy() == ref).all()
+    assert int(n_a.item()) == int(n_b.item())
+    assert table_contents(slots_a) == table_contents(slots_b)
+    ks = oracle.KeySet(1)
+    ks.insert(present)
+    rows = np.concatenate([np.arange(poff[i] + ppre[i], poff[i + 1]) for i in range(len(prev_req))] +
+                          [np.zeros(0, np.int64)]).astype(np.int64)
+    ks.insert(pdig[rows])
+    want = ks.prefix_blocks(ref, blk_ref)
+    assert (pre_a.cpu().numpy() == want).all() and (pre_b.cpu().numpy() == want).all()
+    assert (want[prev_req][ppre == 0] == (np.diff(blk_ref)[prev_req][ppre == 0])).all()   # inserted: all hit
+
+
 def test_probe_empty_and_bad_offsets(kv):
     slots = kv.new_table(64)
     st = status_tensor()
