@@ -118,29 +118,33 @@ __device__ __forceinline__ float rcp_approx(float x) {
     return r;
 }
 
-// One problem solved by one thread, its values x[0..n) in shared memory.
-// Each value is replaced by its reciprocal (+infinity for a tenant that is
-// not usable, which then never counts as above the level and gets p = 0)
-// and then by p_i: the steps compare lambda * (1 / v_i) with 1 and
-// sum reciprocals, with no division per tenant, and
-// p_i = 1 - lambda * (1 / v_i).  The adversary's payoff is lambda whenever a
-// tenant is usable (min(v_i, lambda) over the usable ones, the others at most
-// 0), else the largest value.
-__device__ __forceinline__ void solve_thread(float *x, const float *__restrict__ vg, int n, float K_in, long long q,
-                                             float *__restrict__ lambda_out, float *__restrict__ utility_out,
-                                             uint32_t *status) {
+// One problem solved by one thread, its n <= kMax values x[0..n) staged in
+// shared memory and held in registers for the solve: one pass over shared
+// memory in and one out, every Newton step on registers (from shared memory
+// the steps' re-reads made the kernel bound by its load pipe).  Each value
+// is replaced by its reciprocal (+infinity for a tenant that is not usable,
+// which then never counts as above the level and gets p = 0): the steps
+// compare lambda * (1 / v_i) with 1 and sum reciprocals, with no division
+// per tenant, and p_i = 1 - lambda * (1 / v_i).  The kMax - n padding slots
+// hold 0 -- not usable, not flagged, adding exactly 0 to every sum.  The
+// adversary's payoff is lambda whenever a tenant is usable (min(v_i, lambda)
+// over the usable ones, the others at most 0), else the largest value.
+template <int kMax>
+__device__ __forceinline__ void solve_thread_reg(float *x, const float *__restrict__ vg, int n, float K_in,
+                                                 long long q, float *__restrict__ lambda_out,
+                                                 float *__restrict__ utility_out, uint32_t *status) {
+    float r[kMax];
     int npos = 0, nbad = 0;
-    float vmax = 0.0f, sum_all = 0.0f;       // the first Newton step's sum: every usable tenant
-#pragma unroll 4
-    for (int i = 0; i < n; ++i) {
-        const float xi = x[i];
+    float vmax = 0.0f, sum_all = 0.0f;
+#pragma unroll
+    for (int i = 0; i < kMax; ++i) {
+        const float xi = i < n ? x[i] : 0.0f;
         const bool use = usable(xi);
         npos += use;
         nbad += !use && !(xi <= 0.0f);
         vmax = use ? fmaxf(vmax, xi) : vmax;
-        const float r = use ? rcp_approx(xi) : __int_as_float(0x7f800000);   // +infinity: never above the level
-        sum_all += use ? r : 0.0f;
-        x[i] = r;
+        r[i] = use ? rcp_approx(xi) : __int_as_float(0x7f800000);
+        sum_all += use ? r[i] : 0.0f;
     }
     float K = K_in;
     const bool bad = nbad > 0 || !(K >= 0.0f);
@@ -152,16 +156,15 @@ __device__ __forceinline__ void solve_thread(float *x, const float *__restrict__
     } else if (K >= (float)npos) {
         lam = 0.0f;
     } else {
-        lam = ((float)npos - K) / sum_all;            // the first step, from lambda = 0
+        lam = ((float)npos - K) / sum_all;
         int prev_m = npos;
         for (int step = 0; step <= npos; ++step) {
             float sum = 0.0f;
             int m = 0;
-#pragma unroll 4
-            for (int i = 0; i < n; ++i) {
-                const float r = x[i];
-                const bool on = lam * r < 1.0f;               // false for r = +inf (inf or NaN product)
-                sum += on ? r : 0.0f;
+#pragma unroll
+            for (int i = 0; i < kMax; ++i) {
+                const bool on = lam * r[i] < 1.0f;
+                sum += on ? r[i] : 0.0f;
                 m += on;
             }
             const float next = ((float)m - K) / sum;
@@ -170,10 +173,11 @@ __device__ __forceinline__ void solve_thread(float *x, const float *__restrict__
             prev_m = m;
         }
     }
-#pragma unroll 4
-    for (int i = 0; i < n; ++i) x[i] = fmaxf(0.0f, 1.0f - lam * x[i]);   // 0 for r = +inf (-inf or NaN)
+#pragma unroll
+    for (int i = 0; i < kMax; ++i)
+        if (i < n) x[i] = fmaxf(0.0f, 1.0f - lam * r[i]);
     float u = lam;
-    if (npos == 0) {                      // no usable tenant: the largest value (read again), or 0 if none
+    if (npos == 0) {
         u = n > 0 ? -3.0e38f : 0.0f;
         for (int i = 0; i < n; ++i) {
             const float xi = vg[i];
@@ -217,9 +221,13 @@ __global__ void __launch_bounds__(kCta) origami_kernel(const float *__restrict__
         const int span = (int)(base1 - base0);
         for (int i = threadIdx.x; i < span; i += kCta) sv[i] = values[base0 + i];
         __syncthreads();
-        if (q < q1)
-            solve_thread(sv + (my0 - base0), values + my0, (int)(my1 - my0), budget[q], q, lambda_out, utility_out,
-                         status);
+        if (q < q1) {
+            float *x = sv + (my0 - base0);
+            const int n = (int)(my1 - my0);
+            if (n <= 16) solve_thread_reg<16>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
+            else if (n <= 32) solve_thread_reg<32>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
+            else solve_thread_reg<kSmallN>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
+        }
         __syncthreads();
         for (int i = threadIdx.x; i < span; i += kCta) p[base0 + i] = sv[i];
     } else {
