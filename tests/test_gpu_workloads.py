@@ -145,6 +145,46 @@ def test_full_wide_serving_steps(kv):
     assert seen == [0, 4, 8]
 
 
+def test_full_wide_device_pipeline_matches_oracle(kv):
+    """The bench's timed path at full size: DevicePipeline in its default
+    schedule (each batch's insert inside the next batch's chain launch,
+    chain_prev_kernel at 131,072 requests) over batches A, B, A, B under one
+    secret, then A under a new secret epoch.  Every batch's prefix lengths,
+    copied on the compute stream right after its submit, and the final key
+    count equal the oracle's replay."""
+    wa, wb = W.make("wide", seed=111), W.make("wide", seed=112)
+    wb.secret, wb.ids, wb.id_off = wa.secret, wa.ids, wa.id_off
+    wb.batch.tokens.reshape(-1, 128)[:, :64] = wa.batch.tokens[:64]
+    n_blocks = wa.batch.n * 8
+    cache = PrefixCache(next_pow2(4 * 5 * n_blocks), wa.secret, wa.ids, wa.id_off)
+    pipe = DevicePipeline(cache, W.BOUNDARY, wa.batch.n, n_blocks)
+    dbs = [DeviceBatch.from_host(w.batch.tokens, w.batch.tok_off, w.batch.principal, w.batch.boundary_tok)
+           for w in (wa, wb)]
+    plan = [(0, 0), (1, 0), (0, 0), (1, 0), (0, 1)]            # (batch, secret epoch)
+    copies = []
+    for k, e in plan:
+        cache.set_secret(wa.secret[:24] + e.to_bytes(8, "little"))
+        pre, _ = pipe.submit(dbs[k])
+        with torch.cuda.stream(pipe.compute_stream):
+            copies.append(pre.clone())
+    pipe.drain()
+    torch.cuda.synchronize()
+    cache.check_status()
+    ks = oracle.KeySet(1)
+    mins = []
+    for i, (k, e) in enumerate(plan):
+        b = (wa, wb)[k].batch
+        salts = oracle.derive_salts(wa.secret[:24] + e.to_bytes(8, "little"), wa.ids, wa.id_off)
+        dref = oracle.chain_hash(W.BOUNDARY, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+        bref = oracle.block_offsets(b.tok_off)
+        pref = ks.prefix_blocks(dref, bref)
+        assert (copies[i].cpu().numpy() == pref).all(), f"batch {i}"
+        ks.insert(dref)
+        mins.append(int(pref.min()))
+    assert int(cache.n_new.item()) == ks.n
+    assert mins == [0, 4, 8, 8, 4]
+
+
 @pytest.mark.parametrize("in_chain", [True, False], ids=["insert_in_chain", "inline"])
 def test_host_pipeline_matches_device_serving(kv, in_chain):
     """Batches served from pinned host memory through HostPipeline (copies
