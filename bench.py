@@ -471,13 +471,12 @@ def main():
         cache.set_secret(epoch_secret(w0.secret, epoch[0]))
         epoch[0] += 1
         flushed = flush.before_step()              # load factor would pass 0.5: flush the cache
-        before = (lambda: K.table_init(cache.slots, pipe.compute_stream)) if flushed else None
-        pending = pipe.pending is not None
+        pending = pipe.pending
         if in_chain and (flushed or not pending):
             tab_ev = None                          # this step runs no probe of its own (chain hash + fused probe)
         if tab_ev is not None:
             table_timed.append(tab_ev)
-        prefix, _ = pipe.submit(db, before, ev, tab_ev)
+        prefix, _ = pipe.submit(db, flushed, ev, tab_ev)
         if in_chain:
             # salts, block offsets (2), then the chain hash with the previous batch's insert and the probe or,
             # after a flush (which runs the pending insert and the table init first), the chain hash with
@@ -500,6 +499,12 @@ def main():
     table_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                 if i % table_every == 0 else None for i in range(args.steps)]
     t_start, t_stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # create every timing event now (a CUDA event is created on its first record, which costs the host far
+    # more than a step's launches): inside the timed loop they are only recorded
+    for pair in chain_ev + [e for e in table_ev if e is not None] + [(t_start, t_stop)]:
+        for e in pair:
+            e.record(pipe.compute_stream)
+    torch.cuda.synchronize()
     launches[0] = 0
     flushes_before = flush.flushes
     with ClockSampler(local) as clk:
@@ -627,7 +632,8 @@ def main():
                                   "timed steps) whenever the next step would take it past load factor 0.5"),
             "tokens_per_s": 16 * value, "chain_digests_per_s": world * n_blocks / (chain_ms / 1e3),
             "host_enqueue_ms_per_step": host_ms / args.steps,
-            "schedule": ("DevicePipeline (insert in chain): salts (new epoch) and block offsets of batch i+1 on a "
+            "schedule": ("DevicePipeline over the library's serving engine (kvgov_pipeline_submit, one call per "
+                         "step), insert in chain: salts (new epoch) and block offsets of batch i+1 on a "
                          "prep stream beside the chain hash of batch i; on a higher-priority compute stream the "
                          "chain hash of batch i with batch i-1's insert in the same launch, then the probe of batch "
                          "i" if in_chain else
@@ -661,11 +667,16 @@ def arrival_leg(torch, K, W, pool, n_req, n_blocks, cache, steps, chain_ms):
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
     n_new = torch.zeros(1, dtype=torch.int64, device="cuda")
     seq, times, means = 1, [], []
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps + 3)]
+    for pair in evs:                               # created here, only recorded in the loop
+        for e in pair:
+            e.record()
+    torch.cuda.synchronize()
     for i in range(steps + 3):
         db = pool[i % len(pool)]
         K.table_init(slots)
         K.block_offsets(db.tok_off, blk, status)
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a, b = evs[i]
         a.record()
         K.chain_hash_arrival(W.BOUNDARY, db.tokens, db.tok_off, blk, slots, owner, seq, status, db.principal,
                              cache.salts, db.boundary_tok, dig, slot_of, pre, n_new=n_new)
@@ -708,10 +719,9 @@ def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots, in_chain=Tr
 
     def one(i):
         cache.set_secret(epoch_secret(w0.secret, i))
-        before = (lambda: K.table_init(cache.slots, pipe.compute_stream)) if flush.before_step() else None
-        return pipe.submit(*pinned[i % len(pinned)], n_blocks, before)
+        return pipe.submit(*pinned[i % len(pinned)], n_blocks, flush.before_step())
 
-    warm = 3
+    warm = len(pinned) + 1                         # every pinned input set is copied once before timing
     for i in range(warm):
         one(i)
     torch.cuda.synchronize()
@@ -719,9 +729,11 @@ def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots, in_chain=Tr
     if world > 1:
         dist.barrier()
     a.record(pipe.copy_stream)
+    h0 = time.perf_counter()
     for i in range(steps):
         out, ev = one(warm + i)
     pipe.drain()                                   # the last batch's insert
+    host_ms = (time.perf_counter() - h0) * 1e3
     b.record(pipe.compute_stream)
     torch.cuda.synchronize()
     cache.check_status()
@@ -742,6 +754,7 @@ def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots, in_chain=Tr
     copy_bound = world * n_blocks / (h2d / (link_gbs * 1e9))
     return {"value": value, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps, "last_step_prefix_ok": last_ok,
+            "host_enqueue_ms_per_step": host_ms / steps, "ms_per_step": ms / steps,
             "h2d_link_gbs": link_gbs, "copy_bound_value": copy_bound, "frac_of_copy_bound": value / copy_bound,
             "api": "paper_2608_09225_gb300.pipeline.HostPipeline (copy of step i+1 overlaps serving of step i; "
                    "each step's insert inside the next step's chain launch)"}

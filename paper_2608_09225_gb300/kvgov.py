@@ -32,6 +32,21 @@ _lib = None
 _p = ctypes.c_void_p
 
 
+MAX_SLOTS = 3
+_S3 = _p * MAX_SLOTS
+
+
+class PipelineDesc(ctypes.Structure):
+    """kvgov_pipeline_desc (include/kvgov_pipeline.h)."""
+    _fields_ = [("mode", ctypes.c_int), ("insert_in_chain", ctypes.c_int), ("n_slots", ctypes.c_int),
+                ("max_req", ctypes.c_int32), ("max_blocks", ctypes.c_int64),
+                ("d_slots", _p), ("capacity", ctypes.c_uint64), ("d_status", _p), ("d_n_new", _p),
+                ("d_ids", _p), ("d_id_off", _p), ("n_principals", ctypes.c_int32),
+                ("d_salts", _S3), ("d_blk_off", _S3), ("d_digests", _S3), ("d_prefix", _S3),
+                ("prepared", _S3), ("chain_start", _S3), ("probed", _S3), ("free_ev", _S3),
+                ("prep_stream", _p), ("compute_stream", _p)]
+
+
 class KVGovError(RuntimeError):
     def __init__(self, status: int, where: str):
         self.status = status
@@ -76,11 +91,20 @@ def _load():
                                                  ctypes.c_uint64, _p, _p, _p, _p]
         L.kvgov_set_spin_limit.argtypes = [ctypes.c_uint32]
         L.kvgov_set_spin_limit.restype = ctypes.c_uint32
+        L.kvgov_pipeline_create.argtypes = [ctypes.POINTER(PipelineDesc), ctypes.POINTER(_p)]
+        L.kvgov_pipeline_submit.argtypes = [_p, ctypes.c_char_p, ctypes.c_size_t, _p, _p, ctypes.c_int32, _p, _p,
+                                            ctypes.c_int64, _p, ctypes.c_int, _p, _p, _p, _p,
+                                            ctypes.POINTER(ctypes.c_int32)]
+        L.kvgov_pipeline_drain.argtypes = [_p]
+        L.kvgov_pipeline_pending.argtypes = [_p]
+        L.kvgov_pipeline_destroy.argtypes = [_p]
+        L.kvgov_pipeline_destroy.restype = None
         for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
                    "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
                    "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
                    "kvgov_divergence_boundary", "kvgov_response_key", "kvgov_origami",
-                   "kvgov_serve_arrival_static"):
+                   "kvgov_serve_arrival_static", "kvgov_pipeline_create", "kvgov_pipeline_submit",
+                   "kvgov_pipeline_drain", "kvgov_pipeline_pending"):
             getattr(L, fn).restype = ctypes.c_int
         _lib = L
         return L
@@ -490,3 +514,42 @@ def serve_arrival_static(slots: torch.Tensor, owner: torch.Tensor, digests: torc
 
 def set_spin_limit(limit: int) -> int:
     return int(lib().kvgov_set_spin_limit(int(limit)))
+
+
+# ---- the serving engine (include/kvgov_pipeline.h)
+def event_handle(ev: torch.cuda.Event, stream) -> int:
+    """The cudaEvent_t of a torch event, created (by one record on stream) if it has none yet."""
+    if ev.cuda_event == 0:
+        ev.record(stream)
+    return ev.cuda_event
+
+
+class Engine:
+    """A kvgov_pipeline engine over caller-owned buffers, events and streams
+    (kept alive by the caller).  submit() is one foreign call per batch."""
+
+    def __init__(self, desc: PipelineDesc):
+        self._desc = desc
+        self._h = _p()
+        _check(lib().kvgov_pipeline_create(ctypes.byref(desc), ctypes.byref(self._h)), "kvgov_pipeline_create")
+        self._slot = ctypes.c_int32(0)
+
+    def submit(self, secret: bytes, tokens: int, tok_off: int, n_req: int, principal: int | None,
+               boundary_tok: int | None, n_blocks: int, after: int | None, flush: bool,
+               chain_ev=(None, None), table_ev=(None, None)) -> int:
+        _check(lib().kvgov_pipeline_submit(self._h, secret, len(secret), tokens, tok_off, n_req, principal,
+                                           boundary_tok, n_blocks, after, int(bool(flush)), chain_ev[0],
+                                           chain_ev[1], table_ev[0], table_ev[1], ctypes.byref(self._slot)),
+               "kvgov_pipeline_submit")
+        return self._slot.value
+
+    def drain(self):
+        _check(lib().kvgov_pipeline_drain(self._h), "kvgov_pipeline_drain")
+
+    def pending(self) -> bool:
+        return bool(lib().kvgov_pipeline_pending(self._h))
+
+    def __del__(self):
+        if getattr(self, "_h", None) and _lib is not None:
+            _lib.kvgov_pipeline_destroy(self._h)
+            self._h = None

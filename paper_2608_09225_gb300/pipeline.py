@@ -4,9 +4,10 @@
 index (the slot table and the per-principal salts) and runs a batch of
 requests through the library's kernels on one CUDA stream.
 ``DevicePipeline`` and ``HostPipeline`` serve a stream of batches (resident
-on the device, or in pinned host memory) with each batch's salts, block
-offsets and host-to-device copy overlapping the previous batch's kernels.
-Nothing here computes; every step is a libkvgov entry point (include/kvgov.h).
+on the device, or in pinned host memory) through the library's serving
+engine (include/kvgov_pipeline.h), with each batch's salts, block offsets and
+host-to-device copy overlapping the previous batch's kernels.  Nothing here
+computes; every step is a libkvgov entry point (include/kvgov.h).
 """
 from __future__ import annotations
 
@@ -130,29 +131,24 @@ class PrefixCache:
 
 
 class _Pipelined:
-    """Per-batch device buffers in rotating slots and the stream schedule
-    shared by DevicePipeline and HostPipeline.
-
-    Batch i's salts (under the secret current when it is submitted) and block
-    offsets are computed on a prep stream once batch i-1's chain hash has
-    started, so their small CTAs run in the room the chain kernel leaves on
-    the SMs instead of in front of batch i's chain hash.  The compute stream
-    (higher priority, so its CTAs are placed first) then serves the batch:
+    """Buffers, events and streams of one serving engine (kvgov_pipeline.h),
+    shared by DevicePipeline and HostPipeline.  The stream schedule itself
+    -- batch i's salts and block offsets on a prep stream beside batch i-1's
+    chain launch; on the compute stream (higher priority) the chain hash,
+    the probe and the insert; slots reused only once free -- is the
+    library's: one foreign call per batch (kvgov_pipeline_submit).
 
     insert_in_chain=True (default): batch i's chain hash runs in one launch
     with the insert of batch i-1's uncached blocks
     (kvgov_chain_hash_insert_prev), then batch i is probed against the table
-    as batch i-1 left it.  Batch i's own insert is left pending for the next
-    batch's chain launch (or drain()); three slots rotate, since batch i's
-    buffers are read by batch i+1's chain launch while batch i+2 is prepared.
-
+    as batch i-1 left it; batch i's own insert waits for the next batch's
+    chain launch (or drain()), and three slots rotate.
     insert_in_chain=False: the chain hash with the probe fused in, then the
-    insert of the uncached blocks; two slots.
+    insert; two slots.
 
     Either way every probe sees the table exactly as the previous batch's
-    insert left it, and every step runs on the GPU; nothing here computes.
-    A cache flush (before_serve) first runs a pending insert, so that the
-    flush follows it.
+    insert left it.  A flush (submit(..., flush=True)) first runs a pending
+    insert, then empties the table.  Nothing here computes.
     """
 
     def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_blocks: int, device="cuda",
@@ -163,127 +159,62 @@ class _Pipelined:
         self.prep_stream = torch.cuda.Stream(self.device)
         self.compute_stream = torch.cuda.Stream(self.device, priority=-1)
         cache.stream = self.compute_stream
+        n_slots = 3 if insert_in_chain else 2
         self.slots = []
-        for _ in range(3 if insert_in_chain else 2):
+        for _ in range(n_slots):
             self.slots.append({
                 "salts": torch.empty((max(cache.n_principals, 1), 32), dtype=torch.uint8, device=self.device),
                 "blk_off": torch.empty(max_req + 1, dtype=torch.int64, device=self.device),
                 "digests": torch.empty((max(max_blocks, 1), 32), dtype=torch.uint8, device=self.device),
                 "prefix": torch.empty(max(max_req, 1), dtype=torch.int32, device=self.device),
                 "prepared": torch.cuda.Event(), "chain_start": torch.cuda.Event(), "probed": torch.cuda.Event(),
-                "free": torch.cuda.Event(), "used": False, "n": 0, "n_blocks": 0,
+                "free": torch.cuda.Event(),
             })
-        self.i = 0
-        self.last_chain_start = None
-        self.pending = None          # the slot whose batch's insert has not run yet
+        d = K.PipelineDesc()
+        d.mode, d.insert_in_chain, d.n_slots = int(mode), int(insert_in_chain), n_slots
+        d.max_req, d.max_blocks = int(max_req), int(max_blocks)
+        d.d_slots, d.capacity = cache.slots.data_ptr(), cache.capacity
+        d.d_status, d.d_n_new = cache.status.data_ptr(), cache.n_new.data_ptr()
+        d.d_ids, d.d_id_off, d.n_principals = cache.ids.data_ptr(), cache.id_off.data_ptr(), cache.n_principals
+        cs = self.compute_stream
+        for i, sl in enumerate(self.slots):
+            d.d_salts[i], d.d_blk_off[i] = sl["salts"].data_ptr(), sl["blk_off"].data_ptr()
+            d.d_digests[i], d.d_prefix[i] = sl["digests"].data_ptr(), sl["prefix"].data_ptr()
+            d.prepared[i] = K.event_handle(sl["prepared"], cs)
+            d.chain_start[i] = K.event_handle(sl["chain_start"], cs)
+            d.probed[i] = K.event_handle(sl["probed"], cs)
+            d.free_ev[i] = K.event_handle(sl["free"], cs)
+        d.prep_stream, d.compute_stream = self.prep_stream.cuda_stream, cs.cuda_stream
+        self.engine = K.Engine(d)
+        self._after = [torch.cuda.Event() for _ in self.slots]
+        self._i = 0
 
-    def _next_slot(self):
-        s = self.slots[self.i % len(self.slots)]
-        self.i += 1
-        return s
-
-    def _prepare(self, s, db: DeviceBatch, after=None):
-        """Salts and block offsets of one batch on the prep stream."""
-        c = self.cache
-        ps = self.prep_stream
-        if after is not None:
-            ps.wait_event(after)
-        if self.last_chain_start is not None:
-            ps.wait_event(self.last_chain_start)    # start beside the previous batch's chain hash
-        if s["used"]:
-            ps.wait_event(s["free"])                # the slot's previous batch has been inserted
-        if self.mode != K.UNSALTED:
-            K.derive_salts(c.secret, c.ids, c.id_off, s["salts"], c.status, ps)
-        K.block_offsets(db.tok_off, s["blk_off"][:db.n + 1], c.status, ps)
-        s["prepared"].record(ps)
-
-    def _views(self, s):
-        return s["blk_off"][:s["n"] + 1], s["digests"][:s["n_blocks"]], s["prefix"][:s["n"]]
-
-    def _insert_pending(self):
-        """The pending batch's insert as its own launch (compute stream)."""
-        q = self.pending
-        if q is None:
-            return
-        c = self.cache
-        blk, dig, pre = self._views(q)
-        K.insert_uncached(c.slots, dig, blk, pre, c.status, c.n_new, self.compute_stream)
-        q["free"].record(self.compute_stream)
-        self.pending = None
+    @property
+    def pending(self) -> bool:
+        return self.engine.pending()
 
     def drain(self):
         """Run the pending insert, if any; returns an event recorded after it
         on the compute stream."""
-        with torch.cuda.stream(self.compute_stream):
-            self._insert_pending()
+        self.engine.drain()
         ev = torch.cuda.Event()
         ev.record(self.compute_stream)
         return ev
 
-    def _serve(self, s, db: DeviceBatch, before_serve=None, chain_events=None, table_events=None):
-        """Serve one batch on the compute stream (see the class docstring).
-        chain_events are recorded around the chain-hash launch, table_events
-        around the batch's table kernel after it: the probe (when the chain
-        launch carried the previous batch's insert) or the insert
-        (insert_in_chain=False)."""
-        c = self.cache
+    def _submit(self, db: DeviceBatch, after: torch.cuda.Event, flush: bool, chain_events, table_events) -> int:
         cs = self.compute_stream
-        n = db.n
-        s["n"], s["n_blocks"] = n, db.n_blocks
-        blk_off, digests, prefix = self._views(s)
+        ce = tuple(K.event_handle(e, cs) for e in chain_events) if chain_events is not None else (None, None)
+        te = tuple(K.event_handle(e, cs) for e in table_events) if table_events is not None else (None, None)
         salted = self.mode != K.UNSALTED
-        kw = dict(principal=db.principal if salted else None, salts=s["salts"] if salted else None,
-                  boundary_tok=db.boundary_tok if self.mode == K.BOUNDARY else None, digests=digests,
-                  stream=cs)
-        with torch.cuda.stream(cs):
-            cs.wait_event(s["prepared"])
-            if before_serve is not None:
-                self._insert_pending()
-                before_serve()
-            if chain_events is not None:
-                chain_events[0].record(cs)
-            # the last command before the chain launch: the prep of the next
-            # batch starts only once the chain kernel is being placed
-            s["chain_start"].record(cs)
-            self.last_chain_start = s["chain_start"]
-            q = self.pending if self.insert_in_chain else None
-            if q is not None:
-                qb, qd, qp = self._views(q)
-                K.chain_hash_insert_prev(self.mode, db.tokens, db.tok_off, blk_off, c.slots, qd, qb, qp, c.status,
-                                         n_new=c.n_new, **kw)
-            else:
-                K.chain_hash_probe(self.mode, db.tokens, db.tok_off, blk_off, c.slots, prefix_blocks=prefix,
-                                   n_blocks=db.n_blocks, status=c.status, **kw)
-            if chain_events is not None:
-                chain_events[1].record(cs)
-            if q is not None:
-                if table_events is not None:
-                    table_events[0].record(cs)
-                K.probe(c.slots, digests, blk_off, prefix, c.status, cs)
-                if table_events is not None:
-                    table_events[1].record(cs)
-            if q is not None:
-                q["free"].record(cs)
-                self.pending = None
-            if not self.insert_in_chain:
-                if table_events is not None:
-                    table_events[0].record(cs)
-                K.insert_uncached(c.slots, digests, blk_off, prefix, c.status, c.n_new, cs)
-                if table_events is not None:
-                    table_events[1].record(cs)
-            s["probed"].record(cs)
-            if self.insert_in_chain:
-                self.pending = s
-            else:
-                s["free"].record(cs)
-        s["used"] = True
-        return prefix, digests, blk_off
+        return self.engine.submit(self.cache.secret, db.tokens.data_ptr(), db.tok_off.data_ptr(), db.n,
+                                  db.principal.data_ptr() if salted else None,
+                                  db.boundary_tok.data_ptr() if self.mode == K.BOUNDARY else None,
+                                  db.n_blocks, K.event_handle(after, cs), flush, ce, te)
 
 
 class DevicePipeline(_Pipelined):
-    """Serve device-resident batches back to back, each batch's salts and
-    block offsets computed beside the previous batch's chain hash and (by
-    default) its insert run inside the next batch's chain launch.
+    """Serve device-resident batches back to back through the library's
+    serving engine (see _Pipelined).
 
     submit() returns (prefix_blocks, event) on the device: prefix_blocks is
     valid once event has completed and is overwritten by a later submit (the
@@ -293,37 +224,29 @@ class DevicePipeline(_Pipelined):
     on the caller's current stream.
     """
 
-    def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_blocks: int, device="cuda",
-                 insert_in_chain: bool = True):
-        super().__init__(cache, mode, max_req, max_blocks, device, insert_in_chain)
-        self._ready = [torch.cuda.Event() for _ in self.slots]
-
-    def submit(self, db: DeviceBatch, before_serve=None, chain_events=None, table_events=None):
-        """Queue one device-resident batch.  before_serve, if given, is called
-        with the compute stream current just before the chain hash, after any
-        pending insert (for instance to flush the cache); chain_events and
-        table_events, pairs of CUDA events, are recorded around the
-        chain-hash launch and the table kernel after it (the probe, or the
-        insert)."""
-        ready = self._ready[self.i % len(self.slots)]
-        ready.record(torch.cuda.current_stream(self.device))
+    def submit(self, db: DeviceBatch, flush: bool = False, chain_events=None, table_events=None):
+        """Queue one device-resident batch.  flush empties the cache before
+        it (after any pending insert).  chain_events and table_events, pairs
+        of CUDA events, are recorded around the chain-hash launch and the
+        table kernel after it (the probe, or the insert)."""
+        after = self._after[self._i % len(self._after)]
+        self._i += 1
+        after.record(torch.cuda.current_stream(self.device))
         for t in (db.tokens, db.tok_off, db.principal, db.boundary_tok):
             t.record_stream(self.prep_stream)
             t.record_stream(self.compute_stream)
-        self.compute_stream.wait_event(ready)
-        s = self._next_slot()
-        self._prepare(s, db, after=ready)
-        prefix, _, _ = self._serve(s, db, before_serve, chain_events, table_events)
-        return prefix, s["probed"]
+        slot = self._submit(db, after, flush, chain_events, table_events)
+        sl = self.slots[slot]
+        return sl["prefix"][:db.n], sl["probed"]
 
 
 class HostPipeline(_Pipelined):
     """Serve batches that live in pinned host memory: each batch's
     host-to-device copy runs on a copy stream while the previous batch is
-    served, its salts and block offsets follow on the prep stream, the
-    compute stream serves it as in DevicePipeline and copies its prefix
-    lengths back into a pinned host buffer.  A slot's buffers are reused
-    only after its batch has been inserted.
+    served, then the library's serving engine serves it (see _Pipelined) and
+    an output stream copies its prefix lengths back into a pinned host buffer
+    once its probe is done.  A slot's buffers are reused only after its
+    batch has been inserted and its output copied.
 
     submit() returns (prefix_host, event): prefix_host is valid once event has
     completed (event.synchronize()) and is overwritten by a later submit (the
@@ -334,6 +257,7 @@ class HostPipeline(_Pipelined):
                  insert_in_chain: bool = True):
         super().__init__(cache, mode, max_req, max_tokens // K.BLOCK, device, insert_in_chain)
         self.copy_stream = torch.cuda.Stream(self.device)
+        self.out_stream = torch.cuda.Stream(self.device)
         for s in self.slots:
             s.update({
                 "tokens": torch.empty(max(max_tokens, 4), dtype=torch.int32, device=self.device),
@@ -341,17 +265,16 @@ class HostPipeline(_Pipelined):
                 "principal": torch.empty(max(max_req, 1), dtype=torch.int32, device=self.device),
                 "boundary_tok": torch.empty(max(max_req, 1), dtype=torch.int32, device=self.device),
                 "out": torch.empty(max(max_req, 1), dtype=torch.int32).pin_memory(),
-                "copied": torch.cuda.Event(), "out_done": torch.cuda.Event(),
+                "copied": torch.cuda.Event(), "out_done": torch.cuda.Event(), "used": False,
             })
 
-    def submit(self, tokens, tok_off, principal, boundary_tok, n_blocks: int, before_serve=None,
+    def submit(self, tokens, tok_off, principal, boundary_tok, n_blocks: int, flush: bool = False,
                chain_events=None):
         """Queue one batch given as pinned host tensors (int32 tokens, int64
-        offsets, int32 principal rows and boundary offsets).  before_serve, if
-        given, is called with the compute stream current just before the
-        chain hash, after any pending insert (for instance to flush the
-        cache); chain_events as in DevicePipeline.submit."""
-        s = self._next_slot()
+        offsets, int32 principal rows and boundary offsets).  flush empties
+        the cache before it (after any pending insert); chain_events as in
+        DevicePipeline.submit."""
+        s = self.slots[self._i % len(self.slots)]   # the slot the engine gives this batch
         n, t = tok_off.numel() - 1, tokens.numel()
         with torch.cuda.stream(self.copy_stream):
             if s["used"]:
@@ -364,9 +287,12 @@ class HostPipeline(_Pipelined):
             s["copied"].record(self.copy_stream)
         db = DeviceBatch(s["tokens"][:max(t, 4)], s["tok_off"][:n + 1], s["principal"][:n],
                          s["boundary_tok"][:n], n_blocks)
-        self._prepare(s, db, after=s["copied"])
-        prefix, _, _ = self._serve(s, db, before_serve, chain_events)
-        with torch.cuda.stream(self.compute_stream):
-            s["out"][:n].copy_(prefix, non_blocking=True)
-            s["out_done"].record(self.compute_stream)
+        self._i += 1
+        slot = self._submit(db, s["copied"], flush, chain_events, None)
+        assert self.slots[slot] is s
+        with torch.cuda.stream(self.out_stream):
+            self.out_stream.wait_event(s["probed"])
+            s["out"][:n].copy_(s["prefix"][:n], non_blocking=True)
+            s["out_done"].record(self.out_stream)
+        s["used"] = True
         return s["out"][:n], s["out_done"]

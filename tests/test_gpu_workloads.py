@@ -256,8 +256,7 @@ def test_device_pipeline_matches_sequential_serving(kv, mode, in_chain):
         pre, _, _ = seq.serve(mode, dbs[k])
         want.append(pre.cpu().numpy())
         pip.set_secret(secret)
-        before = (lambda: K.table_init(pip.slots, pipe.compute_stream)) if flush else None
-        out, ev = pipe.submit(dbs[k], before)
+        out, ev = pipe.submit(dbs[k], flush)
         ev.synchronize()
         got.append(out.cpu().numpy())
     pipe.drain()
@@ -291,8 +290,7 @@ def test_device_pipeline_back_to_back_matches_oracle(kv, flush_at, in_chain):
     copies = []
     for i, k in enumerate(order):
         cache.set_secret(w0.secret[:24] + (i % 2).to_bytes(8, "little"))
-        before = (lambda: K.table_init(cache.slots, pipe.compute_stream)) if i == flush_at else None
-        pre, _ = pipe.submit(dbs[k], before)
+        pre, _ = pipe.submit(dbs[k], i == flush_at)
         with torch.cuda.stream(pipe.compute_stream):
             copies.append(pre.clone())
     pipe.drain()

@@ -52,7 +52,81 @@ def test_peak_library_exports_every_declared_symbol():
     assert {"kvgov_peak_int", "kvgov_peak_gather", "kvgov_peak_ops_per_iter"} <= set(names)
     for name in names:
         assert hasattr(lib, name), name
-    assert sorted(os.listdir(os.path.join(ROOT, "include"))) == ["kvgov.h", "kvgov_peak.h"]
+    assert sorted(os.listdir(os.path.join(ROOT, "include"))) == ["kvgov.h", "kvgov_peak.h", "kvgov_pipeline.h"]
+
+
+def test_library_exports_the_serving_engine(libkv):
+    names = declared_functions(os.path.join(ROOT, "include", "kvgov_pipeline.h"))
+    assert {"kvgov_pipeline_create", "kvgov_pipeline_submit", "kvgov_pipeline_drain", "kvgov_pipeline_pending",
+            "kvgov_pipeline_destroy"} <= set(names)
+    for name in names:
+        assert hasattr(libkv, name), name
+
+
+def _engine_desc(insert_in_chain=1):
+    """A description whose pointers are never dereferenced on the host (the
+    checks below run before any CUDA call)."""
+    from paper_2608_09225_gb300.kvgov import PipelineDesc
+    d = PipelineDesc()
+    d.mode, d.insert_in_chain, d.n_slots = 2, insert_in_chain, 3 if insert_in_chain else 2
+    d.max_req, d.max_blocks = 100, 800
+    d.d_slots, d.capacity, d.d_status, d.d_n_new = 0x10000, 1 << 10, 0x20000, 0x30000
+    d.d_ids, d.d_id_off, d.n_principals = 0x40000, 0x50000, 4
+    for i in range(d.n_slots):
+        d.d_salts[i], d.d_blk_off[i], d.d_digests[i], d.d_prefix[i] = (0x100000 * (i + 1) + 0x1000 * k
+                                                                       for k in range(4))
+        d.prepared[i], d.chain_start[i], d.probed[i], d.free_ev[i] = (0x9000000 + 0x100 * i + k for k in range(4))
+    d.prep_stream, d.compute_stream = 0x7000, 0x7100
+    return d
+
+
+def test_serving_engine_checks_its_arguments(libkv):
+    """kvgov_pipeline_create refuses bad descriptions and kvgov_pipeline_submit
+    bad batches with KVGOV_EINVAL, on the host, before anything is queued."""
+    from paper_2608_09225_gb300.kvgov import PipelineDesc
+    P = ctypes.c_void_p
+    libkv.kvgov_pipeline_create.argtypes = [ctypes.POINTER(PipelineDesc), ctypes.POINTER(P)]
+    libkv.kvgov_pipeline_submit.argtypes = [P, ctypes.c_char_p, ctypes.c_size_t, P, P, ctypes.c_int32, P, P,
+                                            ctypes.c_int64, P, ctypes.c_int, P, P, P, P,
+                                            ctypes.POINTER(ctypes.c_int32)]
+    libkv.kvgov_pipeline_destroy.argtypes = [P]
+    libkv.kvgov_pipeline_destroy.restype = None
+    libkv.kvgov_pipeline_drain.argtypes = [P]
+    libkv.kvgov_pipeline_pending.argtypes = [P]
+    h = P()
+    bad = []
+    d = _engine_desc(); d.n_slots = 2; bad.append(d)                 # insert in chain needs 3 slots
+    d = _engine_desc(0); d.n_slots = 3; bad.append(d)                # inline takes 2
+    d = _engine_desc(); d.mode = 7; bad.append(d)
+    d = _engine_desc(); d.capacity = 1000; bad.append(d)             # not a power of two
+    d = _engine_desc(); d.d_digests[2] = 0x100008; bad.append(d)     # misaligned
+    d = _engine_desc(); d.probed[1] = 0; bad.append(d)               # missing event
+    d = _engine_desc(); d.d_ids = 0; bad.append(d)                   # salted mode without ids
+    d = _engine_desc(); d.max_req = -1; bad.append(d)
+    for d in bad:
+        assert libkv.kvgov_pipeline_create(ctypes.byref(d), ctypes.byref(h)) == 1
+    d = _engine_desc()
+    assert libkv.kvgov_pipeline_create(ctypes.byref(d), ctypes.byref(h)) == 0 and h.value
+    slot = ctypes.c_int32(-1)
+    sec = b"s" * 32
+    args = dict(tokens=0x800000, tok_off=0x810000, n_req=10, principal=0x820000, boundary=0x830000, n_blocks=80)
+
+    def submit(**kw):
+        a = dict(args, **kw)
+        return libkv.kvgov_pipeline_submit(h, kw.get("secret", sec), kw.get("secret_len", len(sec)), a["tokens"],
+                                           a["tok_off"], a["n_req"], a["principal"], a["boundary"], a["n_blocks"],
+                                           None, 0, kw.get("ev0"), None, None, None, ctypes.byref(slot))
+    assert submit(n_req=101) == 1                                     # above max_req
+    assert submit(n_blocks=801) == 1                                  # above max_blocks
+    assert submit(principal=None) == 1                                # salted mode
+    assert submit(boundary=None) == 1                                 # BOUNDARY mode
+    assert submit(tok_off=None) == 1
+    assert submit(secret_len=2000) == 1                               # longer than KVGOV_MAX_SECRET
+    assert submit(ev0=0x1234) == 1                                    # an unpaired timing event
+    assert slot.value == -1 and libkv.kvgov_pipeline_pending(h) == 0
+    assert libkv.kvgov_pipeline_drain(h) == 0                         # nothing pending: nothing queued
+    libkv.kvgov_pipeline_destroy(h)
+    libkv.kvgov_pipeline_destroy(None)
 
 
 def test_peak_gather_rejects_bad_arguments():
