@@ -226,6 +226,7 @@ __global__ void __launch_bounds__(kCta) origami_kernel(const float *__restrict__
             const int n = (int)(my1 - my0);
             if (n <= 16) solve_thread_reg<16>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
             else if (n <= 32) solve_thread_reg<32>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
+            else if (n <= 56) solve_thread_reg<56>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
             else solve_thread_reg<kSmallN>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
         }
         __syncthreads();

@@ -51,6 +51,20 @@ def test_origami_ragged_matches_oracle(kv, seed, n_prob):
     check(b, p, lam, u, p_ref, lam_ref, u_ref)
 
 
+@pytest.mark.parametrize("seed", [11, 12])
+def test_origami_thread_tiers_match_oracle(kv, seed):
+    """Problems of 0 to 64 tenants, so that every CTA takes the thread-per-
+    problem path and every register size (16, 32, 56, 64 slots) is used, with
+    all-equal and Pareto values and budgets above n."""
+    b = W.audit_ragged(seed, 4096, max_tenants=64)
+    sizes = np.diff(b.off)
+    assert sizes.max() <= 64 and ((sizes > 56) & (sizes <= 64)).any() and ((sizes > 32) & (sizes <= 56)).any()
+    p, lam, u, st = gpu(kv, b)
+    p_ref, lam_ref, u_ref, flag = oracle.origami(b.values, b.off, b.budget)
+    assert st == 0 and not flag
+    check(b, p, lam, u, p_ref, lam_ref, u_ref)
+
+
 def test_origami_pareto_batch(kv):
     """131,072 problems of the section 5.5 setting (50 tenants, Pareto 1.29,
     K = 10): every probability within tolerance, and each problem's budget
