@@ -217,7 +217,8 @@ int kvgov_derive_salts(const uint8_t *secret, size_t secret_len, const uint8_t *
  *   d_status        nullable; KVGOV_F_BADINDEX for a principal outside
  *                   [0, n_principals), a negative b_r, or a malformed token
  *                   offset (that request's digests are not written).
- * n_req = 0 is a no-op.  EINVAL: bad mode, misaligned or NULL array.
+ * n_req = 0 is a no-op (d_principal, d_salts and d_boundary_tok may then be
+ * NULL).  EINVAL: bad mode, misaligned or NULL array.
  */
 int kvgov_chain_hash(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
                      const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,

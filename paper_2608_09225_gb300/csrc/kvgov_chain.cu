@@ -427,9 +427,11 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     if (n_req < 0) return KVGOV_EINVAL;
     if (!d_tokens || !aligned16(d_tokens) || !d_tok_off || !d_blk_off || !d_digests || !aligned16(d_digests))
         return KVGOV_EINVAL;
-    if (mode != KVGOV_UNSALTED && (!d_principal || !d_salts || !aligned16(d_salts) || n_principals <= 0))
+    // the per-request arrays are needed only when there are requests
+    if (mode != KVGOV_UNSALTED && n_req > 0 &&
+        (!d_principal || !d_salts || !aligned16(d_salts) || n_principals <= 0))
         return KVGOV_EINVAL;
-    if (mode == KVGOV_BOUNDARY && !d_boundary_tok) return KVGOV_EINVAL;
+    if (mode == KVGOV_BOUNDARY && n_req > 0 && !d_boundary_tok) return KVGOV_EINVAL;
     if (f.fuse == kFuseProbe &&
         (!f.prefix_blocks || !f.slots || !aligned16(f.slots) || !kvgov_host::pow2_capacity(f.capacity)))
         return KVGOV_EINVAL;

@@ -186,6 +186,47 @@ def test_full_wide_device_pipeline_matches_oracle(kv):
 
 
 @pytest.mark.parametrize("in_chain", [True, False], ids=["insert_in_chain", "inline"])
+def test_device_pipeline_empty_and_tiny_batches(kv, in_chain):
+    """Batches of no requests, of one request shorter than a block, and
+    ordinary batches, mixed in one stream through the serving engine: the
+    empty ones give empty results and leave the cache alone, the others match
+    the oracle's replay."""
+    w = W.make("tiny")
+    b = w.batch
+    full = DeviceBatch.from_host(b.tokens, b.tok_off, b.principal, b.boundary_tok)
+    empty = DeviceBatch.from_host(np.zeros(4, np.int32), np.zeros(1, np.int64), np.zeros(0, np.int32),
+                                  np.zeros(0, np.int32))
+    short_toks = b.tokens[:7].copy()
+    short = DeviceBatch.from_host(short_toks, np.array([0, 7], np.int64), b.principal[:1], b.boundary_tok[:1])
+    cache = PrefixCache(1 << 12, w.secret, w.ids, w.id_off)
+    pipe = DevicePipeline(cache, W.ROOT, b.n, full.n_blocks, insert_in_chain=in_chain)
+    order = [empty, full, empty, short, full, empty]
+    copies = []
+    for db in order:
+        pre, _ = pipe.submit(db)
+        with torch.cuda.stream(pipe.compute_stream):
+            copies.append(pre.clone())
+    pipe.drain()
+    torch.cuda.synchronize()
+    cache.check_status()
+    salts = oracle.derive_salts(w.secret, w.ids, w.id_off)
+    ks = oracle.KeySet(1)
+    for db, got in zip(order, copies):
+        got = got.cpu().numpy()
+        if db is empty:
+            assert got.shape == (0,)
+            continue
+        if db is short:
+            assert list(got) == [0]
+            continue
+        d = oracle.chain_hash(W.ROOT, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+        blk = oracle.block_offsets(b.tok_off)
+        assert (got == ks.prefix_blocks(d, blk)).all()
+        ks.insert(d)
+    assert int(cache.n_new.item()) == ks.n
+
+
+@pytest.mark.parametrize("in_chain", [True, False], ids=["insert_in_chain", "inline"])
 def test_host_pipeline_matches_device_serving(kv, in_chain):
     """Batches served from pinned host memory through HostPipeline (copies
     overlapping the previous batch's serving; each batch's result read only
