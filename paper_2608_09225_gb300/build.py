@@ -21,7 +21,7 @@ PEAK_LIB = os.path.join(HERE, "libkvgov_peak.so")
 BUILD_DIR = os.path.join(HERE, "_build")
 
 # library -> its translation units
-LIBS = {LIB: ["kvgov_chain.cu", "kvgov_blkoff.cu", "kvgov_salts.cu", "kvgov_table.cu", "kvgov_arrival.cu", "kvgov_boundary.cu", "kvgov_response.cu", "kvgov_origami.cu", "kvgov_pipeline.cu"], PEAK_LIB: ["int_peak.cu", "gather_peak.cu"]}
+LIBS = {LIB: ["kvgov_chain.cu", "kvgov_chain_split.cu", "kvgov_blkoff.cu", "kvgov_salts.cu", "kvgov_table.cu", "kvgov_arrival.cu", "kvgov_boundary.cu", "kvgov_response.cu", "kvgov_origami.cu", "kvgov_pipeline.cu"], PEAK_LIB: ["int_peak.cu", "gather_peak.cu"]}
 SOURCES = [s for srcs in LIBS.values() for s in srcs]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE]

@@ -401,6 +401,17 @@ void launch_chain_kernel(int mode, unsigned grid, cudaStream_t s, const ChainPar
     }
 }
 
+// The chain hash alone: kvgov_chain_split.cu's kernel for a batch too small
+// to fill the GPU (each chain's rounds and schedule on two warps), the
+// chain kernel above otherwise.
+int launch_plain(int mode, unsigned grid, cudaStream_t s, const ChainParams &p) {
+    if (p.n_req <= kvgov_host::chain_split_max_req())
+        return kvgov_host::launch_chain_split(mode, p.tokens, p.tok_off, p.n_req, p.principal, p.salts,
+                                              p.n_principals, p.boundary_tok, p.blk_off, p.digests, p.status, s);
+    launch_chain_kernel<kFuseNone>(mode, grid, s, p);
+    return kvgov_host::launch_status();
+}
+
 // The table and arrival arguments of the fused variants.
 struct FuseArgs {
     int fuse = kFuseNone;
@@ -487,8 +498,7 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
             launch_chain_kernel<kFuseInsertPrev>(mode, grid, s, p, a, q);
             rc = kvgov_host::launch_status();
         } else {                                   // a small batch (or no insert): separate launches
-            launch_chain_kernel<kFuseNone>(mode, grid, s, p);
-            rc = kvgov_host::launch_status();
+            rc = launch_plain(mode, grid, s, p);
             if (rc == KVGOV_OK && f.prev_n_req > 0) rc = insert_prev();
         }
         if (rc == KVGOV_OK && f.probe_prefix_blocks)
@@ -499,8 +509,7 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     const bool none = f.fuse == kFuseNone;
     const bool fused = !none && n_req >= min_fused;
     if (!fused) {
-        launch_chain_kernel<kFuseNone>(mode, grid, s, p);
-        int rc = kvgov_host::launch_status();
+        int rc = launch_plain(mode, grid, s, p);
         if (rc != KVGOV_OK || none) return rc;
         if (f.fuse == kFuseProbe)
             return kvgov_probe(f.slots, f.capacity, d_digests, d_blk_off, n_req, f.prefix_blocks, d_status, stream);

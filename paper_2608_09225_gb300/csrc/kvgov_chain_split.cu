@@ -1,0 +1,353 @@
+// kvgov_chain_split.cu -- the chain hash of a batch too small to fill the
+// GPU (the chain launch of kvgov_chain_hash and of its fused variants when
+// the batch has at most kvgov_host::chain_split_max_req() requests).
+//
+// Paper: section 2.1 equation (h_0 = H(tokens_0..B-1), h_j = H(h_{j-1},
+// tokens_j)), section 4.1 equation (sigma_p prepended at the root) and
+// section 4.2 equation (sigma_p prepended at the divergence block k); the
+// digests are the ones kvgov_chain.cu computes.
+//
+// Why a second kernel.  A chain is sequential in its blocks, so parallelism
+// comes only from the batch.  A batch of a few thousand requests gives each
+// SM sub-partition one warp (or none); a warp alone on its sub-partition
+// issues one integer instruction every two cycles (the integer pipe is 16
+// lanes wide), so its time per block is its instruction count, about 2900
+// per block for the two compressions with their message schedules.
+// Here the work of 32 chains is split over two warps on two
+// sub-partitions:
+//   * the round warp runs only the 64 rounds of each compression (about 14
+//     integer instructions a round) with K_t + W_t read from shared memory;
+//   * the schedule warp stages the tokens (cp.async, two blocks ahead),
+//     builds each compression's message (tokens, salt, the previous digest
+//     or padding), expands its schedule into K_t + W_t in shared memory, and
+//     stores the digests.
+// The round warp's work per block drops to about 1800 integer instructions;
+// the schedule warp's (about 1300) runs beside it.
+//
+// Hand-off per block j, on named barriers of 64 threads (one warp arrives,
+// the other waits):
+//   H       round -> schedule: h_j is in shared memory;
+//   A..D    schedule -> round: K_t + W_t of block j's first compression,
+//           t in [16q, 16q + 16) for chunk q (that message holds h_{j-1},
+//           so its schedule starts only after H);
+//   E0, E1  schedule -> round: the whole second compression of block j
+//           (E_{j mod 2}); its message has no digest in it, so the schedule
+//           warp builds it one block ahead into the other buffer.
+// Both warps of a pair run the same number of blocks (the pair's longest
+// chain) and execute each barrier once per block, so every wait is matched
+// by exactly one arrival; a buffer is rewritten only after the wait that
+// proves the round warp is done with it.
+#include "kvgov_internal.cuh"
+#include "sha256_dev.cuh"
+
+namespace {
+
+using namespace kvgov_dev;
+
+constexpr int kPairs = 2;                   // round/schedule warp pairs per CTA
+constexpr int kThreads = 64 * kPairs;
+constexpr int kChainsPerCta = 32 * kPairs;
+constexpr int kTokStages = 3;               // token buffers: blocks j, j + 1 and j + 2 in flight
+constexpr int kChunks = 5;                  // 16-byte chunks that cover one 64-byte block
+
+// Shared memory of one pair.  K_t + W_t is stored as uint4 [t / 4][lane], so
+// that the round warp reads four rounds' values with one 16-byte load.
+struct PairSmem {
+    uint4 kw1[16][32];              // first compression of the current block
+    uint4 kw2[2][16][32];           // second compression, by block parity
+    uint4 h[2][32];                 // the round warp's state after the block
+    uint4 tok[kTokStages][32][kChunks];
+};
+constexpr size_t kSmemBytes = sizeof(PairSmem) * kPairs;
+
+struct SplitParams {
+    const int32_t *tokens;
+    const int64_t *tok_off;
+    const int32_t *principal;
+    const uint8_t *salts;
+    const int32_t *boundary_tok;
+    const int64_t *blk_off;
+    uint8_t *digests;
+    uint32_t *status;
+    int32_t n_req;
+    int32_t n_principals;
+};
+
+// Named barriers of the pair's 64 threads.  Each is executed by a whole warp
+// at once (the lanes are reconverged first: some code before them is
+// per-lane).
+__device__ __forceinline__ void bar_sync(int id) {
+    __syncwarp();
+    asm volatile("bar.sync %0, 64;\n" ::"r"(id) : "memory");
+}
+__device__ __forceinline__ void bar_arrive(int id) {
+    __syncwarp();
+    asm volatile("bar.arrive %0, 64;\n" ::"r"(id) : "memory");
+}
+
+// What block j's message is, per section 2.1 / 4.1 / 4.2.
+constexpr int kSteadyH = 0;      // H(h_{j-1} || T_j)
+constexpr int kSteadySalt = 1;   // H(sigma_p || T_0)
+constexpr int kFirst = 2;        // H(T_0), unsalted root
+constexpr int kBoundary = 3;     // H(sigma_p || h_{k-1} || T_k), k >= 1
+
+template <int MODE>
+__device__ __forceinline__ int block_kind(int j, int k) {
+    if (MODE == KVGOV_UNSALTED) return j == 0 ? kFirst : kSteadyH;
+    if (MODE == KVGOV_ROOT) return j == 0 ? kSteadySalt : kSteadyH;
+    if (j == 0) return k == 0 ? kSteadySalt : kFirst;
+    return j == k ? kBoundary : kSteadyH;
+}
+
+// 16 rounds with K_t + W_t given (FIPS 180-4 section 6.2.2 step 3).  After
+// 16 rounds the eight working variables are back in their original roles.
+__device__ __forceinline__ void rounds16(uint32_t v[8], const uint32_t kw[16]) {
+#pragma unroll
+    for (int t = 0; t < 16; ++t) {
+        uint32_t &a = v[(8 - t % 8) % 8], &b = v[(9 - t % 8) % 8], &c = v[(10 - t % 8) % 8], &d = v[(11 - t % 8) % 8];
+        uint32_t &e = v[(12 - t % 8) % 8], &f = v[(13 - t % 8) % 8], &g = v[(14 - t % 8) % 8], &h = v[(15 - t % 8) % 8];
+        const uint32_t t1 = h + kw[t] + ch(e, f, g) + bsig1(e);
+        const uint32_t t2 = bsig0(a) + maj(a, b, c);
+        d += t1;
+        h = t1 + t2;
+    }
+}
+
+// One compression of the round warp: state s, K_t + W_t from kw.  bar0 >= 0:
+// wait on barrier bar0 + q before chunk q (the schedule warp is still
+// producing it); bar0 < 0: the whole schedule is already there.
+__device__ __forceinline__ void compress_kw(uint32_t s[8], const uint4 (*kw)[32], int lane, int bar0) {
+    uint32_t v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = s[i];
+#pragma unroll 1
+    for (int q = 0; q < 4; ++q) {
+        if (bar0 >= 0) bar_sync(bar0 + q);
+        uint32_t k[16];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const uint4 x = kw[4 * q + i][lane];
+            k[4 * i] = x.x; k[4 * i + 1] = x.y; k[4 * i + 2] = x.z; k[4 * i + 3] = x.w;
+        }
+        rounds16(v, k);
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s[i] += v[i];
+}
+
+// The schedule warp's half of a compression: expand the message w[0..15]
+// (FIPS 180-4 section 6.2.2 step 1) into K_t + W_t, t = 0..63, stored to kw.
+// bar0 >= 0: arrive on barrier bar0 + q after chunk q; bar_end >= 0: arrive
+// on it after the last chunk.
+__device__ __forceinline__ void schedule_kw(uint32_t w[16], uint4 (*kw)[32], int lane, int bar0, int bar_end) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        kw[i][lane] = make_uint4(w[4 * i] + sha_k(4 * i), w[4 * i + 1] + sha_k(4 * i + 1),
+                                 w[4 * i + 2] + sha_k(4 * i + 2), w[4 * i + 3] + sha_k(4 * i + 3));
+    if (bar0 >= 0) bar_arrive(bar0);
+#pragma unroll 1
+    for (int q = 1; q < 4; ++q) {
+#pragma unroll
+        for (int t = 0; t < 16; ++t)
+            w[t] = w[t] + w[(t + 9) & 15] + ssig0(w[(t + 1) & 15]) + ssig1(w[(t + 14) & 15]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            kw[4 * q + i][lane] = make_uint4(w[4 * i] + c_sha_k[16 * q + 4 * i], w[4 * i + 1] + c_sha_k[16 * q + 4 * i + 1],
+                                             w[4 * i + 2] + c_sha_k[16 * q + 4 * i + 2],
+                                             w[4 * i + 3] + c_sha_k[16 * q + 4 * i + 3]);
+        if (bar0 >= 0) bar_arrive(bar0 + q);
+    }
+    if (bar_end >= 0) bar_arrive(bar_end);
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, 1) chain_split_kernel(const SplitParams p) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int pair = warp >> 1;
+    const bool round_warp = (warp & 1) == 0;
+    PairSmem &sm = reinterpret_cast<PairSmem *>(smem_raw)[pair];
+    const int bar_h = 1 + 7 * pair, bar_a = bar_h + 1, bar_e = bar_h + 5;   // A..D = bar_a + 0..3, E0/E1 = bar_e + 0/1
+
+    // Per-chain set-up (both warps of the pair hold the same chain in the same lane).
+    const long long r = (long long)blockIdx.x * kChainsPerCta + pair * 32 + lane;
+    const long long tok_end = p.tok_off[p.n_req];
+    long long t0 = 0, row = 0;
+    int nb = 0, k = -1, pi = 0;
+    if (r < p.n_req) {
+        t0 = p.tok_off[r];
+        const long long t1 = p.tok_off[r + 1];
+        const long long nbl = (t1 - t0) / KVGOV_BLOCK;
+        bool ok = t0 >= 0 && t1 >= t0 && t1 <= tok_end && nbl < (1ll << 31);
+        row = p.blk_off[r];
+        ok = ok && row >= 0 && p.blk_off[r + 1] - row == nbl && row + nbl <= p.blk_off[p.n_req];
+        if (MODE != KVGOV_UNSALTED) {
+            pi = p.principal[r];
+            ok = ok && pi >= 0 && pi < p.n_principals;
+        }
+        if (MODE == KVGOV_ROOT) k = 0;
+        if (MODE == KVGOV_BOUNDARY) {
+            const int b = p.boundary_tok[r];
+            ok = ok && b >= 0;
+            k = b / KVGOV_BLOCK;
+        }
+        if (ok) nb = (int)nbl;
+        else if (!round_warp) raise_flag(p.status, KVGOV_F_BADINDEX);
+    }
+    const int jmax = (int)__reduce_max_sync(0xffffffffu, (unsigned)nb);   // the same in both warps
+
+    if (round_warp) {
+        for (int j = 0; j < jmax; ++j) {
+            uint32_t s[8];
+            sha_iv(s);
+            compress_kw(s, sm.kw1, lane, bar_a);
+            bar_sync(bar_e + (j & 1));
+            compress_kw(s, sm.kw2[j & 1], lane, -1);
+            if (MODE == KVGOV_BOUNDARY && j > 0 && j == k && j < nb) {   // the boundary block's padding block
+                uint32_t w[16];
+                pad_block(w, 0, 128u * 8u);
+                sha_compress_t<true, false>(s, w, AddAlu{});
+            }
+            sm.h[0][lane] = make_uint4(s[0], s[1], s[2], s[3]);
+            sm.h[1][lane] = make_uint4(s[4], s[5], s[6], s[7]);
+            bar_arrive(bar_h);
+        }
+        return;
+    }
+
+    // Schedule warp.
+    uint32_t sw[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) sw[i] = 0u;
+    if (MODE != KVGOV_UNSALTED && nb > 0) {
+        const uint4 *sp = reinterpret_cast<const uint4 *>(p.salts + 32ll * pi);
+        const uint4 a = __ldg(sp), b = __ldg(sp + 1);
+        sw[0] = bswap32(a.x); sw[1] = bswap32(a.y); sw[2] = bswap32(a.z); sw[3] = bswap32(a.w);
+        sw[4] = bswap32(b.x); sw[5] = bswap32(b.y); sw[6] = bswap32(b.z); sw[7] = bswap32(b.w);
+    }
+    const char *tok_bytes = reinterpret_cast<const char *>(p.tokens);
+    const long long end_bytes = tok_end * 4;
+    auto stage = [&](int jj) {   // block jj of this lane's chain -> tok[jj % 3]; one commit group per call
+        if (jj < nb) {
+            const long long sb = (t0 + (long long)KVGOV_BLOCK * jj) * 4;
+            const long long a0 = sb & ~15ll;
+            const int n = a0 == sb ? 4 : 5;
+            for (int c = 0; c < n; ++c) {
+                const long long ca = a0 + 16ll * c;
+                const long long avail = end_bytes - ca;
+                cp_async16(&sm.tok[jj % kTokStages][lane][c], tok_bytes + ca, avail >= 16 ? 16 : (int)avail);
+            }
+        }
+        cp_async_commit();
+    };
+    const int sh = (int)(t0 & 3);   // word offset of every block inside its first chunk
+    auto read_tokens = [&](int jj, uint32_t tw[16]) {
+        const uint32_t *src = reinterpret_cast<const uint32_t *>(&sm.tok[jj % kTokStages][lane][0]) + sh;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) tw[i] = bswap32(src[i]);
+    };
+    // Second compression of block jj: the message words after the first 64 bytes.
+    auto second_message = [&](int jj, const uint32_t tw[16], uint32_t w[16]) {
+        const int kind = block_kind<MODE>(jj, k);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            uint32_t pad = 0u;   // SHA-256 padding (FIPS 180-4 section 5.1.1)
+            if (kind == kFirst) pad = i == 0 ? 0x80000000u : (i == 15 ? 64u * 8u : 0u);
+            else pad = i == 8 ? 0x80000000u : (i == 15 ? 96u * 8u : 0u);
+            w[i] = kind == kBoundary ? tw[i] : (kind != kFirst && i < 8 ? tw[8 + i] : pad);
+        }
+    };
+    auto store_digest = [&](int jj, const uint32_t hw[8]) {
+        uint4 *dst = reinterpret_cast<uint4 *>(p.digests + (row + jj) * 32);
+        dst[0] = make_uint4(bswap32(hw[0]), bswap32(hw[1]), bswap32(hw[2]), bswap32(hw[3]));
+        dst[1] = make_uint4(bswap32(hw[4]), bswap32(hw[5]), bswap32(hw[6]), bswap32(hw[7]));
+    };
+    auto read_state = [&](uint32_t hw[8]) {
+        const uint4 x = sm.h[0][lane], y = sm.h[1][lane];
+        hw[0] = x.x; hw[1] = x.y; hw[2] = x.z; hw[3] = x.w;
+        hw[4] = y.x; hw[5] = y.y; hw[6] = y.z; hw[7] = y.w;
+    };
+
+    stage(0);
+    stage(1);
+    uint32_t hw[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) hw[i] = 0u;
+    for (int j = 0; j < jmax; ++j) {
+        stage(j + 2);                      // its buffer last held block j - 1, read for the last time before
+        if (j > 0) {
+            bar_sync(bar_h);
+            read_state(hw);                // h_{j-1}
+        }
+        cp_async_wait<1>();                // blocks j and j + 1 have landed
+        uint32_t tw[16], w[16];
+        read_tokens(j, tw);
+        const int kind = block_kind<MODE>(j, k);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {      // first 64 bytes of the message
+            w[i] = kind == kFirst ? tw[i] : (kind == kSteadyH ? hw[i] : sw[i]);
+            w[8 + i] = kind == kFirst ? tw[8 + i] : (kind == kBoundary ? hw[i] : tw[i]);
+        }
+        schedule_kw(w, sm.kw1, lane, bar_a, -1);
+        if (j > 0 && j - 1 < nb) store_digest(j - 1, hw);
+        if (j == 0) {
+            second_message(0, tw, w);
+            schedule_kw(w, sm.kw2[0], lane, -1, bar_e);
+        }
+        if (j + 1 < jmax) {
+            read_tokens(j + 1, tw);
+            second_message(j + 1, tw, w);
+            schedule_kw(w, sm.kw2[(j + 1) & 1], lane, -1, bar_e + ((j + 1) & 1));
+        }
+    }
+    if (jmax > 0) {
+        bar_sync(bar_h);
+        read_state(hw);
+        if (jmax - 1 < nb) store_digest(jmax - 1, hw);
+    }
+    cp_async_wait<0>();
+}
+
+template <int MODE>
+int launch_mode(unsigned grid, const SplitParams &p, cudaStream_t s) {
+    static bool attr_set[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return KVGOV_ECUDA;
+    if (dev < 0 || dev >= 64 || !attr_set[dev]) {
+        if (cudaFuncSetAttribute(chain_split_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kSmemBytes) != cudaSuccess)
+            return KVGOV_ECUDA;
+        if (dev >= 0 && dev < 64) attr_set[dev] = true;
+    }
+    chain_split_kernel<MODE><<<grid, kThreads, kSmemBytes, s>>>(p);
+    return kvgov_host::launch_status();
+}
+
+}  // namespace
+
+namespace kvgov_host {
+
+#ifndef KVGOV_SPLIT_CTAS_PER_SM
+#define KVGOV_SPLIT_CTAS_PER_SM 1
+#endif
+
+long long chain_split_max_req() { return (long long)KVGOV_SPLIT_CTAS_PER_SM * sm_count() * kChainsPerCta; }
+
+int launch_chain_split(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                       const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                       const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                       uint32_t *d_status, cudaStream_t stream) {
+    if (n_req <= 0) return KVGOV_OK;
+    SplitParams p;
+    p.tokens = d_tokens; p.tok_off = d_tok_off; p.principal = d_principal; p.salts = d_salts;
+    p.boundary_tok = d_boundary_tok; p.blk_off = d_blk_off; p.digests = d_digests; p.status = d_status;
+    p.n_req = n_req; p.n_principals = n_principals;
+    const unsigned grid = (unsigned)(((long long)n_req + kChainsPerCta - 1) / kChainsPerCta);
+    switch (mode) {
+    case KVGOV_UNSALTED: return launch_mode<KVGOV_UNSALTED>(grid, p, stream);
+    case KVGOV_ROOT: return launch_mode<KVGOV_ROOT>(grid, p, stream);
+    default: return launch_mode<KVGOV_BOUNDARY>(grid, p, stream);
+    }
+}
+
+}  // namespace kvgov_host

@@ -43,6 +43,14 @@ int arrival_owner_min_by_request(const int64_t *d_blk_off, int32_t n_req, uint32
                                  uint64_t *d_owner, uint64_t seq_base, cudaStream_t stream);
 bool arrival_args_ok(uint64_t capacity, uint64_t seq_base);
 
+// The chain hash of a small batch (kvgov_chain_split.cu): the largest batch
+// it takes, and its launch (arguments already checked by the caller).
+long long chain_split_max_req();
+int launch_chain_split(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                       const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                       const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                       uint32_t *d_status, cudaStream_t stream);
+
 inline int launch_status() {
     return cudaGetLastError() == cudaSuccess ? KVGOV_OK : KVGOV_ECUDA;
 }

@@ -121,9 +121,16 @@ def test_block_offsets_negative_length_flagged(kv):
 RAGGED = [0, 15, 16, 17, 31, 32, 33, 2119, 64, 100, 7, 48, 3, 19, 257, 1, 128, 129, 130, 131]
 
 
+def split_limit():
+    """Largest batch the chain hash runs on its small-batch kernel (one
+    round warp and one schedule warp per 32 chains, 64 chains per SM)."""
+    return 64 * torch.cuda.get_device_properties(0).multi_processor_count
+
+
 @pytest.mark.parametrize("mode", [0, 1, 2])
-@pytest.mark.parametrize("lengths", [RAGGED, RAGGED * 17, [3, 16], [1, 16 * 9 + 2], [5] * 300],
-                         ids=["ragged", "ragged_many_ctas", "tail_at_array_end", "tail2", "all_short"])
+@pytest.mark.parametrize("lengths", [RAGGED, RAGGED * 17, [3, 16], [1, 16 * 9 + 2], [5] * 300, RAGGED * 600],
+                         ids=["ragged", "ragged_many_ctas", "tail_at_array_end", "tail2", "all_short",
+                              "ragged_above_split_limit"])
 def test_chain_matches_oracle(kv, mode, lengths):
     b = W.ragged(31 + len(lengths), lengths)
     salts = oracle.derive_salts(b"salt key", *W.principal_ids(8))
@@ -138,14 +145,35 @@ def test_chain_matches_oracle(kv, mode, lengths):
 
 
 @pytest.mark.parametrize("boundary", [0, 15, 16, 17, 100, 16 * 20, 16 * 39, 16 * 40, 16 * 41, 10 ** 9])
-def test_chain_boundary_positions(kv, boundary):
+@pytest.mark.parametrize("n_req", [150, 12000], ids=["split_kernel", "chain_kernel"])
+def test_chain_boundary_positions(kv, boundary, n_req):
     """k = 0, interior, last block (k = n_b - 1), past the end."""
-    b = W.ragged(5, [16 * 40] * 150)
+    b = W.ragged(5, [16 * 40] * n_req)
     b.boundary_tok[:] = boundary
     salts = oracle.derive_salts(b"B", *W.principal_ids(8))
     _, d = gpu_chain(kv, 2, b, salts)
     ref = oracle.chain_hash(2, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
     assert (d == ref).all()
+
+
+@pytest.mark.parametrize("delta", [-1, 0, 1])
+def test_chain_at_the_split_limit(kv, delta):
+    """Batches at the small-batch kernel's limit and one past it, every mode,
+    ragged lengths (empty, sub-block, unaligned starts, a long chain) and a
+    boundary per request anywhere from block 0 to past the end."""
+    n = split_limit() + delta
+    lengths = (RAGGED * (n // len(RAGGED) + 1))[:n]
+    b = W.ragged(77 + delta, lengths)
+    rng = np.random.default_rng(5 + delta)
+    b.boundary_tok[:] = rng.integers(0, 2200, n)
+    salts = oracle.derive_salts(b"limit", *W.principal_ids(8))
+    for mode in (0, 1, 2):
+        st = status_tensor()
+        _, d = gpu_chain(kv, mode, b, salts, st)
+        assert int(st.item()) == 0
+        ref = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+        bad = np.nonzero((d != ref).any(axis=1))[0]
+        assert len(bad) == 0, f"mode {mode}: {len(bad)} digests differ, first rows {bad[:5]}"
 
 
 def test_chain_against_golden_file(kv):
