@@ -16,6 +16,11 @@
 //      the ALU pipe
 //   4  the same with every add issued as IMAD on the FMA pipe
 //   5  IMAD  x_s = x_s * one + x_{s+1}   (one = 1 at run time)
+//   6  SHA-256 rounds only (64 a iteration, K_t + W_t from registers, as the
+//      small-batch chain kernel's round warp runs them): sha_rounds16_t1t2
+//   7  the same with sha_rounds16_short
+// Kinds 6 and 7 count 14 nominal ops a round; launched with one warp per SM
+// sub-partition they give a lone warp's round rate.
 // Each update reads two other streams' latest values, so no chain of updates
 // collapses into fewer instructions (a three-input boolean of three fixed
 // inputs would fold into one LOP3; these never have three fixed inputs).
@@ -45,7 +50,23 @@ __global__ void peak_kernel(int iters, uint32_t seed, uint32_t one, uint32_t *si
     __syncthreads();
     if (threadIdx.x == 0) t_start = clock64();
     __syncthreads();
-    if (KIND == 3 || KIND == 4) {
+    if (KIND == 6 || KIND == 7) {
+        uint32_t v[8], kw[16];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = x[i];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) kw[i] = x[i & 7] * (2u * i + 1u);
+        for (int it = 0; it < iters; ++it) {
+#pragma unroll 1
+            for (int q = 0; q < 4; ++q) {
+                if (KIND == 6) kvgov_dev::sha_rounds16_t1t2(v, kw);
+                else kvgov_dev::sha_rounds16_short(v, kw);
+            }
+            kw[it & 15] ^= v[0];   // a new schedule word each iteration (one op per 64 rounds)
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) x[i] = v[i];
+    } else if (KIND == 3 || KIND == 4) {
         uint32_t st[kShaChains][8], w[kShaChains][16];
 #pragma unroll
         for (int c = 0; c < kShaChains; ++c) {
@@ -103,13 +124,14 @@ extern "C" int kvgov_peak_ops_per_iter(int kind) {
     case 2: return 4 * kStreams;
     case 3: case 4: return kShaChains * 1384;
     case 5: return 4 * kStreams;
+    case 6: case 7: return 64 * 14;
     default: return 0;
     }
 }
 
 extern "C" int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint32_t *d_sink,
                               unsigned long long *d_clocks, kvgov_stream_t stream) {
-    if (kind < 0 || kind > 5 || iters <= 0 || blocks <= 0 || threads <= 0 || threads > 1024 || !d_sink ||
+    if (kind < 0 || kind > 7 || iters <= 0 || blocks <= 0 || threads <= 0 || threads > 1024 || !d_sink ||
         !d_clocks)
         return 1;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
@@ -119,7 +141,9 @@ extern "C" int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint
     case 2: peak_kernel<2><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
     case 3: peak_kernel<3><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
     case 4: peak_kernel<4><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
-    default: peak_kernel<5><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 5: peak_kernel<5><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 6: peak_kernel<6><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    default: peak_kernel<7><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
     }
     return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }

@@ -26,13 +26,16 @@
 //
 // Hand-off per block j, on named barriers of 64 threads (one warp arrives,
 // the other waits):
+//   E0, E1  schedule -> round (E_{j mod 2}, waited on at the start of block
+//           j): K_t + W_t of block j's whole second compression, whose
+//           message holds no digest, and of the first 16 rounds of its first
+//           compression with every word that is h_{j-1} left out -- the round
+//           warp adds h_{j-1} itself, so block j starts without waiting for
+//           the schedule warp.  Built one block ahead into the other buffer.
 //   H       round -> schedule: h_j is in shared memory;
-//   A..D    schedule -> round: K_t + W_t of block j's first compression,
-//           t in [16q, 16q + 16) for chunk q (that message holds h_{j-1},
-//           so its schedule starts only after H);
-//   E0, E1  schedule -> round: the whole second compression of block j
-//           (E_{j mod 2}); its message has no digest in it, so the schedule
-//           warp builds it one block ahead into the other buffer.
+//   B..D    schedule -> round: K_t + W_t of block j's first compression for
+//           t in [16q, 16q + 16), chunk q = 1..3 (from h_{j-1} on, so the
+//           schedule warp starts them after H).
 // Both warps of a pair run the same number of blocks (the pair's longest
 // chain) and execute each barrier once per block, so every wait is matched
 // by exactly one arrival; a buffer is rewritten only after the wait that
@@ -53,7 +56,8 @@ constexpr int kChunks = 5;                  // 16-byte chunks that cover one 64-
 // Shared memory of one pair.  K_t + W_t is stored as uint4 [t / 4][lane], so
 // that the round warp reads four rounds' values with one 16-byte load.
 struct PairSmem {
-    uint4 kw1[16][32];              // first compression of the current block
+    uint4 kw1[12][32];              // first compression of the current block, t = 16..63
+    uint4 pm[2][4][32];             // its t = 0..15 without h_{j-1}, by block parity
     uint4 kw2[2][16][32];           // second compression, by block parity
     uint4 h[2][32];                 // the round warp's state after the block
     uint4 tok[kTokStages][32][kChunks];
@@ -71,6 +75,9 @@ struct SplitParams {
     uint32_t *status;
     int32_t n_req;
     int32_t n_principals;
+    // K_t + W_t of the padding block that ends a 128-byte message (the
+    // boundary block's third compression), the same for every chain
+    uint32_t pad128_kw[64];
 };
 
 // Named barriers of the pair's 64 threads.  Each is executed by a whole warp
@@ -99,52 +106,40 @@ __device__ __forceinline__ int block_kind(int j, int k) {
     return j == k ? kBoundary : kSteadyH;
 }
 
-// 16 rounds with K_t + W_t given (FIPS 180-4 section 6.2.2 step 3).  After
-// 16 rounds the eight working variables are back in their original roles.
+// The round warp's 16 rounds (sha256_dev.cuh): the grouping of the sums is a
+// compile-time choice, measured on a lone warp (libkvgov_peak kinds 6, 7).
+#ifndef KVGOV_SPLIT_SHORT_ROUNDS
+#define KVGOV_SPLIT_SHORT_ROUNDS 0
+#endif
 __device__ __forceinline__ void rounds16(uint32_t v[8], const uint32_t kw[16]) {
+#if KVGOV_SPLIT_SHORT_ROUNDS
+    sha_rounds16_short(v, kw);
+#else
+    sha_rounds16_t1t2(v, kw);
+#endif
+}
+
+__device__ __forceinline__ void load16(const uint4 (*kw)[32], int lane, uint32_t k[16]) {
 #pragma unroll
-    for (int t = 0; t < 16; ++t) {
-        uint32_t &a = v[(8 - t % 8) % 8], &b = v[(9 - t % 8) % 8], &c = v[(10 - t % 8) % 8], &d = v[(11 - t % 8) % 8];
-        uint32_t &e = v[(12 - t % 8) % 8], &f = v[(13 - t % 8) % 8], &g = v[(14 - t % 8) % 8], &h = v[(15 - t % 8) % 8];
-        const uint32_t t1 = h + kw[t] + ch(e, f, g) + bsig1(e);
-        const uint32_t t2 = bsig0(a) + maj(a, b, c);
-        d += t1;
-        h = t1 + t2;
+    for (int i = 0; i < 4; ++i) {
+        const uint4 x = kw[i][lane];
+        k[4 * i] = x.x; k[4 * i + 1] = x.y; k[4 * i + 2] = x.z; k[4 * i + 3] = x.w;
     }
 }
 
-// One compression of the round warp: state s, K_t + W_t from kw.  bar0 >= 0:
-// wait on barrier bar0 + q before chunk q (the schedule warp is still
-// producing it); bar0 < 0: the whole schedule is already there.
-__device__ __forceinline__ void compress_kw(uint32_t s[8], const uint4 (*kw)[32], int lane, int bar0) {
-    uint32_t v[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) v[i] = s[i];
-#pragma unroll 1
-    for (int q = 0; q < 4; ++q) {
-        if (bar0 >= 0) bar_sync(bar0 + q);
-        uint32_t k[16];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const uint4 x = kw[4 * q + i][lane];
-            k[4 * i] = x.x; k[4 * i + 1] = x.y; k[4 * i + 2] = x.z; k[4 * i + 3] = x.w;
-        }
-        rounds16(v, k);
-    }
-#pragma unroll
-    for (int i = 0; i < 8; ++i) s[i] += v[i];
-}
-
-// The schedule warp's half of a compression: expand the message w[0..15]
-// (FIPS 180-4 section 6.2.2 step 1) into K_t + W_t, t = 0..63, stored to kw.
-// bar0 >= 0: arrive on barrier bar0 + q after chunk q; bar_end >= 0: arrive
-// on it after the last chunk.
-__device__ __forceinline__ void schedule_kw(uint32_t w[16], uint4 (*kw)[32], int lane, int bar0, int bar_end) {
+// K_t + W_t, t = 0..15, of a message w into kw[0..3].
+__device__ __forceinline__ void store_kw16(const uint32_t w[16], uint4 (*kw)[32], int lane) {
 #pragma unroll
     for (int i = 0; i < 4; ++i)
         kw[i][lane] = make_uint4(w[4 * i] + sha_k(4 * i), w[4 * i + 1] + sha_k(4 * i + 1),
                                  w[4 * i + 2] + sha_k(4 * i + 2), w[4 * i + 3] + sha_k(4 * i + 3));
-    if (bar0 >= 0) bar_arrive(bar0);
+}
+
+// The schedule warp's half of a compression: expand the message w[0..15]
+// (FIPS 180-4 section 6.2.2 step 1) into K_t + W_t for t = 16..63, chunk q
+// = t / 16 stored to kw[4 (q - 1) ..]; bar0 >= 0: arrive on barrier
+// bar0 + q - 1 after chunk q.  w is overwritten.
+__device__ __forceinline__ void schedule_kw48(uint32_t w[16], uint4 (*kw)[32], int lane, int bar0) {
 #pragma unroll 1
     for (int q = 1; q < 4; ++q) {
 #pragma unroll
@@ -152,12 +147,11 @@ __device__ __forceinline__ void schedule_kw(uint32_t w[16], uint4 (*kw)[32], int
             w[t] = w[t] + w[(t + 9) & 15] + ssig0(w[(t + 1) & 15]) + ssig1(w[(t + 14) & 15]);
 #pragma unroll
         for (int i = 0; i < 4; ++i)
-            kw[4 * q + i][lane] = make_uint4(w[4 * i] + c_sha_k[16 * q + 4 * i], w[4 * i + 1] + c_sha_k[16 * q + 4 * i + 1],
-                                             w[4 * i + 2] + c_sha_k[16 * q + 4 * i + 2],
-                                             w[4 * i + 3] + c_sha_k[16 * q + 4 * i + 3]);
-        if (bar0 >= 0) bar_arrive(bar0 + q);
+            kw[4 * (q - 1) + i][lane] =
+                make_uint4(w[4 * i] + c_sha_k[16 * q + 4 * i], w[4 * i + 1] + c_sha_k[16 * q + 4 * i + 1],
+                           w[4 * i + 2] + c_sha_k[16 * q + 4 * i + 2], w[4 * i + 3] + c_sha_k[16 * q + 4 * i + 3]);
+        if (bar0 >= 0) bar_arrive(bar0 + q - 1);
     }
-    if (bar_end >= 0) bar_arrive(bar_end);
 }
 
 template <int MODE>
@@ -167,7 +161,7 @@ __global__ void __launch_bounds__(kThreads, 1) chain_split_kernel(const SplitPar
     const int pair = warp >> 1;
     const bool round_warp = (warp & 1) == 0;
     PairSmem &sm = reinterpret_cast<PairSmem *>(smem_raw)[pair];
-    const int bar_h = 1 + 7 * pair, bar_a = bar_h + 1, bar_e = bar_h + 5;   // A..D = bar_a + 0..3, E0/E1 = bar_e + 0/1
+    const int bar_h = 1 + 6 * pair, bar_b = bar_h + 1, bar_e = bar_h + 4;   // B..D = bar_b + 0..2, E0/E1 = bar_e + 0/1
 
     // Per-chain set-up (both warps of the pair hold the same chain in the same lane).
     const long long r = (long long)blockIdx.x * kChainsPerCta + pair * 32 + lane;
@@ -197,20 +191,68 @@ __global__ void __launch_bounds__(kThreads, 1) chain_split_kernel(const SplitPar
     const int jmax = (int)__reduce_max_sync(0xffffffffu, (unsigned)nb);   // the same in both warps
 
     if (round_warp) {
+        uint32_t hp[8];   // h_{j-1}
+#pragma unroll
+        for (int i = 0; i < 8; ++i) hp[i] = 0u;
         for (int j = 0; j < jmax; ++j) {
-            uint32_t s[8];
-            sha_iv(s);
-            compress_kw(s, sm.kw1, lane, bar_a);
             bar_sync(bar_e + (j & 1));
-            compress_kw(s, sm.kw2[j & 1], lane, -1);
-            if (MODE == KVGOV_BOUNDARY && j > 0 && j == k && j < nb) {   // the boundary block's padding block
-                uint32_t w[16];
-                pad_block(w, 0, 128u * 8u);
-                sha_compress_t<true, false>(s, w, AddAlu{});
+            uint32_t s[8], v[8], kw[16];
+            load16(sm.pm[j & 1], lane, kw);
+            const int kind = block_kind<MODE>(j, k);
+            if (kind == kSteadyH) {            // h_{j-1} is message words 0..7
+#pragma unroll
+                for (int i = 0; i < 8; ++i) kw[i] += hp[i];
+            } else if (kind == kBoundary) {    // words 8..15, after the salt
+#pragma unroll
+                for (int i = 0; i < 8; ++i) kw[8 + i] += hp[i];
+            }
+            sha_iv(s);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[i] = s[i];
+            rounds16(v, kw);
+#pragma unroll 1
+            for (int q = 1; q < 4; ++q) {
+                bar_sync(bar_b + q - 1);
+                load16(sm.kw1 + 4 * (q - 1), lane, kw);
+                rounds16(v, kw);
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) { s[i] += v[i]; v[i] = s[i]; }
+            // second compression: the whole schedule is there since E, so each
+            // chunk's values are loaded while the previous chunk's rounds run
+            // (two register sets, no copies)
+            const uint4 (*k2)[32] = sm.kw2[j & 1];
+            uint32_t kb[16];
+            load16(k2, lane, kw);
+#pragma unroll 1
+            for (int q = 0; q < 4; q += 2) {
+                load16(k2 + 4 * (q + 1), lane, kb);
+                rounds16(v, kw);
+                if (q + 2 < 4) load16(k2 + 4 * (q + 2), lane, kw);
+                rounds16(v, kb);
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) s[i] += v[i];
+            // the boundary block's padding block: K_t + W_t from the launch parameters
+            if (MODE == KVGOV_BOUNDARY && __any_sync(0xffffffffu, j > 0 && j == k && j < nb)) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) v[i] = s[i];
+#pragma unroll 1
+                for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) kw[i] = p.pad128_kw[16 * q + i];
+                    rounds16(v, kw);
+                }
+                if (j > 0 && j == k && j < nb) {
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) s[i] += v[i];
+                }
             }
             sm.h[0][lane] = make_uint4(s[0], s[1], s[2], s[3]);
             sm.h[1][lane] = make_uint4(s[4], s[5], s[6], s[7]);
             bar_arrive(bar_h);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) hp[i] = s[i];
         }
         return;
     }
@@ -246,6 +288,15 @@ __global__ void __launch_bounds__(kThreads, 1) chain_split_kernel(const SplitPar
 #pragma unroll
         for (int i = 0; i < 16; ++i) tw[i] = bswap32(src[i]);
     };
+    // First 64 bytes of block jj's message with the words that are h_{jj-1} set to 0.
+    auto first_premessage = [&](int jj, const uint32_t tw[16], uint32_t w[16]) {
+        const int kind = block_kind<MODE>(jj, k);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            w[i] = kind == kFirst ? tw[i] : (kind == kSteadyH ? 0u : sw[i]);
+            w[8 + i] = kind == kFirst ? tw[8 + i] : (kind == kBoundary ? 0u : tw[i]);
+        }
+    };
     // Second compression of block jj: the message words after the first 64 bytes.
     auto second_message = [&](int jj, const uint32_t tw[16], uint32_t w[16]) {
         const int kind = block_kind<MODE>(jj, k);
@@ -267,6 +318,17 @@ __global__ void __launch_bounds__(kThreads, 1) chain_split_kernel(const SplitPar
         hw[0] = x.x; hw[1] = x.y; hw[2] = x.z; hw[3] = x.w;
         hw[4] = y.x; hw[5] = y.y; hw[6] = y.z; hw[7] = y.w;
     };
+    // Block jj's second compression and its first compression's pre-message
+    // into buffer jj mod 2, then E_{jj mod 2} (tw: block jj's tokens).
+    auto ahead = [&](int jj, const uint32_t tw[16]) {
+        uint32_t w[16];
+        second_message(jj, tw, w);
+        store_kw16(w, sm.kw2[jj & 1], lane);
+        schedule_kw48(w, sm.kw2[jj & 1] + 4, lane, -1);
+        first_premessage(jj, tw, w);
+        store_kw16(w, sm.pm[jj & 1], lane);
+        bar_arrive(bar_e + (jj & 1));
+    };
 
     stage(0);
     stage(1);
@@ -282,22 +344,18 @@ __global__ void __launch_bounds__(kThreads, 1) chain_split_kernel(const SplitPar
         cp_async_wait<1>();                // blocks j and j + 1 have landed
         uint32_t tw[16], w[16];
         read_tokens(j, tw);
+        if (j == 0) ahead(0, tw);
         const int kind = block_kind<MODE>(j, k);
 #pragma unroll
         for (int i = 0; i < 8; ++i) {      // first 64 bytes of the message
             w[i] = kind == kFirst ? tw[i] : (kind == kSteadyH ? hw[i] : sw[i]);
             w[8 + i] = kind == kFirst ? tw[8 + i] : (kind == kBoundary ? hw[i] : tw[i]);
         }
-        schedule_kw(w, sm.kw1, lane, bar_a, -1);
+        schedule_kw48(w, sm.kw1, lane, bar_b);
         if (j > 0 && j - 1 < nb) store_digest(j - 1, hw);
-        if (j == 0) {
-            second_message(0, tw, w);
-            schedule_kw(w, sm.kw2[0], lane, -1, bar_e);
-        }
         if (j + 1 < jmax) {
             read_tokens(j + 1, tw);
-            second_message(j + 1, tw, w);
-            schedule_kw(w, sm.kw2[(j + 1) & 1], lane, -1, bar_e + ((j + 1) & 1));
+            ahead(j + 1, tw);
         }
     }
     if (jmax > 0) {
@@ -328,10 +386,30 @@ int launch_mode(unsigned grid, const SplitParams &p, cudaStream_t s) {
 namespace kvgov_host {
 
 #ifndef KVGOV_SPLIT_CTAS_PER_SM
-#define KVGOV_SPLIT_CTAS_PER_SM 1
+#define KVGOV_SPLIT_CTAS_PER_SM 3   // measured: ahead of chain_kernel up to 3 CTAs (192 chains) per SM
 #endif
 
 long long chain_split_max_req() { return (long long)KVGOV_SPLIT_CTAS_PER_SM * sm_count() * kChainsPerCta; }
+
+namespace {
+
+// FIPS 180-4 section 6.2.2 step 1 on the host: K_t + W_t of the padding
+// block (0x80, zeros, the 64-bit bit length) of a message of `bytes` bytes
+// that fills whole 64-byte blocks.
+void padding_schedule(uint32_t bytes, uint32_t kw[64]) {
+    auto rotr = [](uint32_t x, int n) { return (x >> n) | (x << (32 - n)); };
+    uint32_t w[64] = {};
+    w[0] = 0x80000000u;
+    w[15] = bytes * 8u;
+    for (int t = 16; t < 64; ++t) {
+        const uint32_t s0 = rotr(w[t - 15], 7) ^ rotr(w[t - 15], 18) ^ (w[t - 15] >> 3);
+        const uint32_t s1 = rotr(w[t - 2], 17) ^ rotr(w[t - 2], 19) ^ (w[t - 2] >> 10);
+        w[t] = w[t - 16] + s0 + w[t - 7] + s1;
+    }
+    for (int t = 0; t < 64; ++t) kw[t] = kvgov_dev::kShaKHost[t] + w[t];
+}
+
+}  // namespace
 
 int launch_chain_split(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
                        const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
@@ -342,6 +420,7 @@ int launch_chain_split(int mode, const int32_t *d_tokens, const int64_t *d_tok_o
     p.tokens = d_tokens; p.tok_off = d_tok_off; p.principal = d_principal; p.salts = d_salts;
     p.boundary_tok = d_boundary_tok; p.blk_off = d_blk_off; p.digests = d_digests; p.status = d_status;
     p.n_req = n_req; p.n_principals = n_principals;
+    padding_schedule(128, p.pad128_kw);
     const unsigned grid = (unsigned)(((long long)n_req + kChainsPerCta - 1) / kChainsPerCta);
     switch (mode) {
     case KVGOV_UNSALTED: return launch_mode<KVGOV_UNSALTED>(grid, p, stream);

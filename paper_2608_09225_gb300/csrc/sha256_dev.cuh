@@ -143,16 +143,20 @@ __device__ __forceinline__ void sha_compress(uint32_t s[8], uint32_t w[16], Add 
     sha_compress_t<false, false>(s, w, add);
 }
 
-// FIPS 180-4 K_t in constant memory, for the compact compression below.
-static __constant__ uint32_t c_sha_k[64] = {
-    0x428a2f98u, 0x71374491u, 0xb5c0fbcfu, 0xe9b5dba5u, 0x3956c25bu, 0x59f111f1u, 0x923f82a4u, 0xab1c5ed5u,
-    0xd807aa98u, 0x12835b01u, 0x243185beu, 0x550c7dc3u, 0x72be5d74u, 0x80deb1feu, 0x9bdc06a7u, 0xc19bf174u,
-    0xe49b69c1u, 0xefbe4786u, 0x0fc19dc6u, 0x240ca1ccu, 0x2de92c6fu, 0x4a7484aau, 0x5cb0a9dcu, 0x76f988dau,
-    0x983e5152u, 0xa831c66du, 0xb00327c8u, 0xbf597fc7u, 0xc6e00bf3u, 0xd5a79147u, 0x06ca6351u, 0x14292967u,
-    0x27b70a85u, 0x2e1b2138u, 0x4d2c6dfcu, 0x53380d13u, 0x650a7354u, 0x766a0abbu, 0x81c2c92eu, 0x92722c85u,
-    0xa2bfe8a1u, 0xa81a664bu, 0xc24b8b70u, 0xc76c51a3u, 0xd192e819u, 0xd6990624u, 0xf40e3585u, 0x106aa070u,
-    0x19a4c116u, 0x1e376c08u, 0x2748774cu, 0x34b0bcb5u, 0x391c0cb3u, 0x4ed8aa4au, 0x5b9cca4fu, 0x682e6ff3u,
-    0x748f82eeu, 0x78a5636fu, 0x84c87814u, 0x8cc70208u, 0x90befffau, 0xa4506cebu, 0xbef9a3f7u, 0xc67178f2u};
+// FIPS 180-4 section 4.2.2 K_t: in constant memory for the compact
+// compression below, and as a host-side array for schedules the host
+// computes ahead (a fixed padding block's).
+#define KVGOV_SHA256_K \
+    0x428a2f98u, 0x71374491u, 0xb5c0fbcfu, 0xe9b5dba5u, 0x3956c25bu, 0x59f111f1u, 0x923f82a4u, 0xab1c5ed5u, \
+    0xd807aa98u, 0x12835b01u, 0x243185beu, 0x550c7dc3u, 0x72be5d74u, 0x80deb1feu, 0x9bdc06a7u, 0xc19bf174u, \
+    0xe49b69c1u, 0xefbe4786u, 0x0fc19dc6u, 0x240ca1ccu, 0x2de92c6fu, 0x4a7484aau, 0x5cb0a9dcu, 0x76f988dau, \
+    0x983e5152u, 0xa831c66du, 0xb00327c8u, 0xbf597fc7u, 0xc6e00bf3u, 0xd5a79147u, 0x06ca6351u, 0x14292967u, \
+    0x27b70a85u, 0x2e1b2138u, 0x4d2c6dfcu, 0x53380d13u, 0x650a7354u, 0x766a0abbu, 0x81c2c92eu, 0x92722c85u, \
+    0xa2bfe8a1u, 0xa81a664bu, 0xc24b8b70u, 0xc76c51a3u, 0xd192e819u, 0xd6990624u, 0xf40e3585u, 0x106aa070u, \
+    0x19a4c116u, 0x1e376c08u, 0x2748774cu, 0x34b0bcb5u, 0x391c0cb3u, 0x4ed8aa4au, 0x5b9cca4fu, 0x682e6ff3u, \
+    0x748f82eeu, 0x78a5636fu, 0x84c87814u, 0x8cc70208u, 0x90befffau, 0xa4506cebu, 0xbef9a3f7u, 0xc67178f2u
+static __constant__ uint32_t c_sha_k[64] = {KVGOV_SHA256_K};
+constexpr uint32_t kShaKHost[64] = {KVGOV_SHA256_K};
 
 // The same compression with a small instruction footprint: rounds 0-15 are
 // unrolled, rounds 16-63 run as three passes of one unrolled 16-round body
@@ -189,6 +193,39 @@ __device__ __forceinline__ void sha_compress_small(uint32_t s[8], uint32_t w[16]
     }
 #pragma unroll
     for (int i = 0; i < 8; ++i) s[i] = add(s[i], v[i]);
+}
+
+// 16 rounds (FIPS 180-4 section 6.2.2 step 3) with K_t + W_t given, for
+// kernels whose message schedule is computed elsewhere.  v holds a..h in
+// rotating roles; after 16 rounds every variable is back in its original
+// slot.  Two groupings of the same sums:
+//   sha_rounds16_t1t2: T1 = h + KW + Ch + Sigma1, T2 = Sigma0 + Maj,
+//                      e' = d + T1, a' = T1 + T2;
+//   sha_rounds16_short: x = h + KW + Ch, e' = d + x + Sigma1 (one three-input
+//                      add after Sigma1), a' = x + Sigma1 + Sigma0 + Maj;
+// the second puts one add fewer between e and the next e.
+__device__ __forceinline__ void sha_rounds16_t1t2(uint32_t v[8], const uint32_t kw[16]) {
+#pragma unroll
+    for (int t = 0; t < 16; ++t) {
+        uint32_t &a = v[(8 - t % 8) % 8], &b = v[(9 - t % 8) % 8], &c = v[(10 - t % 8) % 8], &d = v[(11 - t % 8) % 8];
+        uint32_t &e = v[(12 - t % 8) % 8], &f = v[(13 - t % 8) % 8], &g = v[(14 - t % 8) % 8], &h = v[(15 - t % 8) % 8];
+        const uint32_t t1 = h + kw[t] + ch(e, f, g) + bsig1(e);
+        const uint32_t t2 = bsig0(a) + maj(a, b, c);
+        d += t1;
+        h = t1 + t2;
+    }
+}
+__device__ __forceinline__ void sha_rounds16_short(uint32_t v[8], const uint32_t kw[16]) {
+#pragma unroll
+    for (int t = 0; t < 16; ++t) {
+        uint32_t &a = v[(8 - t % 8) % 8], &b = v[(9 - t % 8) % 8], &c = v[(10 - t % 8) % 8], &d = v[(11 - t % 8) % 8];
+        uint32_t &e = v[(12 - t % 8) % 8], &f = v[(13 - t % 8) % 8], &g = v[(14 - t % 8) % 8], &h = v[(15 - t % 8) % 8];
+        const uint32_t x = h + kw[t] + ch(e, f, g);
+        const uint32_t s1 = bsig1(e);
+        const uint32_t y = x + s1 + bsig0(a);
+        d = d + x + s1;
+        h = y + maj(a, b, c);
+    }
 }
 
 // Compression of a data block inside the fixed-length messages below:

@@ -27,6 +27,13 @@ requests, the first 16,384 probe-heavy requests); mean of 20 back-to-back
 launches queued behind a GPU spin.  Every variant's prefix lengths must
 equal the first variant's.
 
+Split mode (flag KVGOV_SPLIT_CTAS_PER_SM = 0..3: the largest batch the
+small-batch chain kernel takes, in CTAs of 64 chains per SM; 0 never uses it):
+kvgov_chain_hash in ROOT mode on batches of 512-token requests from a quarter
+to four times the SM count x 64 requests (mean of 10 back-to-back launches
+queued behind a GPU spin); every variant's digests must equal the first
+variant's.
+
 Prints one JSON line per variant.  Needs a GPU.
 """
 from __future__ import annotations
@@ -239,8 +246,58 @@ def probe_mode(specs):
     return 0
 
 
+SPLIT_DEFAULT = ["split0:-DKVGOV_SPLIT_CTAS_PER_SM=0", "split1:-DKVGOV_SPLIT_CTAS_PER_SM=1",
+                 "split2:-DKVGOV_SPLIT_CTAS_PER_SM=2", "split3:-DKVGOV_SPLIT_CTAS_PER_SM=3"]
+
+
+def split_mode(specs):
+    import torch
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    sizes = [sms * 64 * f // 4 for f in (1, 2, 4, 6, 8, 12, 16)]
+    b = W.ragged(11, [512] * sizes[-1])
+    salts = torch.from_numpy(np.random.default_rng(3).integers(0, 256, (8, 32), dtype=np.uint8)).cuda()
+    toks = torch.from_numpy(b.tokens).cuda()
+    tok_off = torch.from_numpy(b.tok_off).cuda()
+    pr = torch.from_numpy(b.principal).cuda()
+    stream = torch.cuda.current_stream().cuda_stream
+    ref = {}
+    for spec in specs:
+        name, _, flags = spec.partition(":")
+        L = _bind(ctypes.CDLL(build_variant(name, flags.split())))
+        res, same = {}, True
+        for n in sizes:
+            blk = torch.empty(n + 1, dtype=torch.int64, device="cuda")
+            assert L.kvgov_block_offsets(tok_off.data_ptr(), n, blk.data_ptr(), None, stream) == 0
+            dig = torch.empty((n * 32, 32), dtype=torch.uint8, device="cuda")
+            st = torch.zeros(1, dtype=torch.int32, device="cuda")
+
+            def run():
+                assert L.kvgov_chain_hash(1, toks.data_ptr(), tok_off.data_ptr(), n, pr.data_ptr(), salts.data_ptr(),
+                                          8, None, blk.data_ptr(), dig.data_ptr(), st.data_ptr(), stream) == 0
+
+            for _ in range(3):
+                run()
+            torch.cuda.synchronize()
+            a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda._sleep(4_000_000)
+            a.record()
+            for _ in range(10):
+                run()
+            e.record()
+            torch.cuda.synchronize()
+            res[str(n)] = round(a.elapsed_time(e) / 10 * 1e3, 1)
+            got = dig.cpu().numpy()
+            same = same and int(st.item()) == 0 and (n not in ref or (got == ref[n]).all())
+            ref.setdefault(n, got)
+        print(json.dumps({"variant": name, "flags": flags, "chain_us_by_requests": res,
+                          "same_digests_as_first": bool(same)}), flush=True)
+    return 0
+
+
 def main(argv):
     import torch
+    if argv and argv[0] == "--split":
+        return split_mode(argv[1:] or SPLIT_DEFAULT)
     if argv and argv[0] == "--insert":
         return insert_mode(argv[1:] or INSERT_DEFAULT)
     if argv and argv[0] == "--probe":
