@@ -223,6 +223,27 @@ def measure_int_peak(torch, peak_lib_path):
     return out
 
 
+def measure_lone_warp_round(torch, peak_lib_path) -> float:
+    """SM clock cycles of one SHA-256 round for a warp alone on its SM
+    sub-partition (libkvgov_peak kind 6: rounds only, K_t + W_t in
+    registers, one CTA of four warps per SM): the latency floor of the
+    small-batch chain kernel, whose round warp runs alone."""
+    import ctypes
+    L = ctypes.CDLL(peak_lib_path)
+    L.kvgov_peak_int.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                 ctypes.c_void_p, ctypes.c_void_p]
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    iters = 400
+    sink = torch.zeros(1, dtype=torch.int32, device="cuda")
+    clocks = torch.zeros(n_sm * 3, dtype=torch.int64, device="cuda")
+    for _ in range(2):
+        assert L.kvgov_peak_int(6, iters, n_sm, 128, sink.data_ptr(), clocks.data_ptr(),
+                                torch.cuda.current_stream().cuda_stream) == 0
+    torch.cuda.synchronize()
+    c = clocks.view(n_sm, 3).cpu().numpy()
+    return float(np.median(c[:, 2] - c[:, 1])) / (iters * 64)
+
+
 def measure_gather(torch, peak_lib_path, table: "torch.Tensor", n_reads: int = 1 << 25) -> dict:
     """Random-slot read rate (GB/s of bytes read, best of 5) over `table`,
     reading whole 32-byte slots and first halves, from libkvgov_peak."""
@@ -847,7 +868,9 @@ def run_configs(args):
     scratch_table = K.new_table(1 << 25)
     gather = measure_gather(torch, kbuild.PEAK_LIB, scratch_table)
     del scratch_table
-    print(json.dumps({"random_read_microbench": gather, "hbm_gbs": PEAKS.get("hbm_gbs")}), flush=True)
+    round_cycles = measure_lone_warp_round(torch, kbuild.PEAK_LIB)
+    print(json.dumps({"random_read_microbench": gather, "hbm_gbs": PEAKS.get("hbm_gbs"),
+                      "lone_warp_cycles_per_round": round_cycles}), flush=True)
     only = set(args.only.split(",")) if args.only else None
     want = (lambda n: only is None or n in only)
     plan = []
@@ -967,12 +990,22 @@ def run_configs(args):
         misses = int((L < nb).sum())
         probe_bytes = hits * (32 + 16 * (1 + 1 / (1 - a))) + misses * (32 + 16 * (1 + 1 / (1 - a) ** 2)) + 4 * (p1 - p0)
         insert_bytes = keys.shape[0] * (32 + 16 * (1 + 1 / (1 - a)) + 32)
+        # a batch that leaves every round warp alone on its sub-partition (at most 64 chains
+        # per SM) is bound by the latency of its longest chain: 2 compressions per block,
+        # one more for a boundary block, 64 rounds each at the lone-warp round time
+        nb_all = b.lengths() // 16
+        k_all = b.boundary_tok // 16
+        comp = 2 * nb_all + ((k_all >= 1) & (k_all < nb_all) if mode == W.BOUNDARY else 0)
+        lat_ms = (float(comp.max()) * 64 * round_cycles / (SM_MAX_MHZ * 1e3)
+                  if 0 < b.n <= 64 * n_sm else None)
         line = {"workload": name, "mode": names[mode], "requests": b.n, "blocks": n_blocks,
                 "table_slots": cap, "table_fits_l2": cap * 32 <= l2,
                 "chain_ms": t_chain, "chain_digests_per_s": n_blocks / (t_chain / 1e3),
                 "chain_tokens_per_s": 16 * n_blocks / (t_chain / 1e3),
                 "chain_frac_int32_peak": ops / (t_chain / 1e3) / peak,
                 "chain_us_per_block_per_chain": 1e3 * t_chain / max(1, int((b.lengths() // 16).max())),
+                "chain_latency_bound_ms": lat_ms,
+                "chain_frac_latency_bound": (lat_ms / t_chain) if lat_ms else None,
                 "fused_chain_probe_ms": t_fused, "salts_ms": t_salts, "block_offsets_ms": t_blk,
                 "probe_ms": t_probe, "probed_requests": p1 - p0, "algorithmic_probes": algo_probes,
                 "probes_per_s": algo_probes / (t_probe / 1e3), "mean_prefix_blocks": float(L.mean()),
