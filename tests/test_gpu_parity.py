@@ -460,11 +460,15 @@ def test_insert_uncached_bad_offsets_flagged(kv):
 
 @pytest.mark.parametrize("mode", [0, 1, 2])
 @pytest.mark.parametrize("fill", [0.0, 0.5, 1.0])
-@pytest.mark.parametrize("n_req", [180, 40960], ids=["two_launches", "fused"])
+@pytest.mark.parametrize("n_req", [180, 20000, 34000, 40960],
+                         ids=["split_then_probe", "split_3_ctas_per_sm_then_probe", "chain_then_probe", "fused"])
 def test_chain_hash_probe_matches_separate_calls(kv, mode, fill, n_req):
     """kvgov_chain_hash_probe writes the digests of kvgov_chain_hash and the
-    prefix lengths of kvgov_probe, both equal to the oracle's, for a batch
-    small enough to take two launches and one that takes the fused kernel."""
+    prefix lengths of kvgov_probe, both equal to the oracle's, on each of its
+    routes: the small-batch chain kernel then the probe kernel (up to 192
+    requests per SM), the chain kernel then the probe kernel (up to two warps
+    per SM sub-partition), and the chain kernel probing each digest as it
+    computes it."""
     lengths = (RAGGED * 9 if n_req == 180 else
                list(np.random.default_rng(n_req + mode).integers(0, 260, n_req)))
     b = W.ragged(77, lengths)
