@@ -41,6 +41,7 @@
 // by exactly one arrival; a buffer is rewritten only after the wait that
 // proves the round warp is done with it.
 #include "kvgov_internal.cuh"
+#include "kvgov_split.cuh"
 #include "sha256_dev.cuh"
 
 namespace {
@@ -80,18 +81,6 @@ struct SplitParams {
     uint32_t pad128_kw[64];
 };
 
-// Named barriers of the pair's 64 threads.  Each is executed by a whole warp
-// at once (the lanes are reconverged first: some code before them is
-// per-lane).
-__device__ __forceinline__ void bar_sync(int id) {
-    __syncwarp();
-    asm volatile("bar.sync %0, 64;\n" ::"r"(id) : "memory");
-}
-__device__ __forceinline__ void bar_arrive(int id) {
-    __syncwarp();
-    asm volatile("bar.arrive %0, 64;\n" ::"r"(id) : "memory");
-}
-
 // What block j's message is, per section 2.1 / 4.1 / 4.2.
 constexpr int kSteadyH = 0;      // H(h_{j-1} || T_j)
 constexpr int kSteadySalt = 1;   // H(sigma_p || T_0)
@@ -117,41 +106,6 @@ __device__ __forceinline__ void rounds16(uint32_t v[8], const uint32_t kw[16]) {
 #else
     sha_rounds16_t1t2(v, kw);
 #endif
-}
-
-__device__ __forceinline__ void load16(const uint4 (*kw)[32], int lane, uint32_t k[16]) {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const uint4 x = kw[i][lane];
-        k[4 * i] = x.x; k[4 * i + 1] = x.y; k[4 * i + 2] = x.z; k[4 * i + 3] = x.w;
-    }
-}
-
-// K_t + W_t, t = 0..15, of a message w into kw[0..3].
-__device__ __forceinline__ void store_kw16(const uint32_t w[16], uint4 (*kw)[32], int lane) {
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-        kw[i][lane] = make_uint4(w[4 * i] + sha_k(4 * i), w[4 * i + 1] + sha_k(4 * i + 1),
-                                 w[4 * i + 2] + sha_k(4 * i + 2), w[4 * i + 3] + sha_k(4 * i + 3));
-}
-
-// The schedule warp's half of a compression: expand the message w[0..15]
-// (FIPS 180-4 section 6.2.2 step 1) into K_t + W_t for t = 16..63, chunk q
-// = t / 16 stored to kw[4 (q - 1) ..]; bar0 >= 0: arrive on barrier
-// bar0 + q - 1 after chunk q.  w is overwritten.
-__device__ __forceinline__ void schedule_kw48(uint32_t w[16], uint4 (*kw)[32], int lane, int bar0) {
-#pragma unroll 1
-    for (int q = 1; q < 4; ++q) {
-#pragma unroll
-        for (int t = 0; t < 16; ++t)
-            w[t] = w[t] + w[(t + 9) & 15] + ssig0(w[(t + 1) & 15]) + ssig1(w[(t + 14) & 15]);
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-            kw[4 * (q - 1) + i][lane] =
-                make_uint4(w[4 * i] + c_sha_k[16 * q + 4 * i], w[4 * i + 1] + c_sha_k[16 * q + 4 * i + 1],
-                           w[4 * i + 2] + c_sha_k[16 * q + 4 * i + 2], w[4 * i + 3] + c_sha_k[16 * q + 4 * i + 3]);
-        if (bar0 >= 0) bar_arrive(bar0 + q - 1);
-    }
 }
 
 template <int MODE>

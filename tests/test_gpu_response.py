@@ -40,6 +40,25 @@ def test_response_key_every_length(kv, mode):
     assert (got == oracle.response_key(mode, toks, tok_off, pr, salts)).all()
 
 
+@pytest.mark.parametrize("mode", [W.UNSALTED, W.ROOT])
+@pytest.mark.parametrize("delta", [0, 1])
+def test_response_key_at_the_split_limit(kv, mode, delta):
+    """Batches at the small-batch kernel's limit (192 requests per SM, two
+    warps per 32 requests) and one past it (one thread per request): lengths
+    0..600 tokens, every start offset, empty prompts included."""
+    n = 192 * torch.cuda.get_device_properties(0).multi_processor_count + delta
+    rng = np.random.default_rng(40 + delta + 2 * mode)
+    lens = rng.integers(0, 601, n)
+    lens[:50] = 0
+    tok_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    toks = rng.integers(0, W.VOCAB, int(tok_off[-1]), dtype=np.int32)
+    salts = oracle.derive_salts(b"limit", *W.principal_ids(16))
+    pr = rng.integers(0, 16, n).astype(np.int32)
+    got, st = gpu_keys(kv, mode, toks, tok_off, pr, salts)
+    assert st == 0
+    assert (got == oracle.response_key(mode, toks, tok_off, pr, salts)).all()
+
+
 @pytest.mark.parametrize("name", ["sysprompt", "wide", "long"])
 def test_response_key_workloads(kv, name):
     w = W.make(name, seed=71) if name in ("wide", "long") else W.make(name)

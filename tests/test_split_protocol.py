@@ -1,5 +1,6 @@
-"""The named-barrier hand-off of the small-batch chain kernel
-(csrc/kvgov_chain_split.cu), checked on the CPU over random interleavings.
+"""The named-barrier hand-offs of the small-batch kernels (the chain hash in
+csrc/kvgov_chain_split.cu, the exact-response keys in csrc/kvgov_response.cu),
+checked on the CPU over random interleavings.
 
 Per 32 chains a round warp and a schedule warp meet on barriers of 64
 threads: a barrier completes when both warps have reached it (bar.arrive or
@@ -108,6 +109,59 @@ def run(jmax, rng, warps=(round_warp, schedule_warp)):
             step(w)
     if any(count.values()):
         raise ProtocolError(f"a barrier phase left open: {count}")
+
+
+# The exact-response key kernel's two warps (csrc/kvgov_response.cu,
+# response_split_kernel): message m's K_t + W_t go through a ring of two
+# buffers; the schedule warp waits for a buffer to be emptied before reusing
+# it (EMPTY), the round warp for it to be filled (FULL).  Barrier ids relative
+# to the pair's base: FULL0/1 = 0/1, EMPTY0/1 = 2/3.
+FULL, EMPTY = 0, 2
+
+
+def response_round_warp(mmax):
+    for m in range(mmax):
+        yield ("sync", FULL + (m & 1))
+        for q in range(4):
+            yield ("read", ("kw", m & 1, q), m)
+        if m + 2 < mmax:                                # the schedule warp reuses the buffer
+            yield ("arrive", EMPTY + (m & 1))
+
+
+def response_schedule_warp(mmax):
+    for m in range(mmax):
+        if m >= 2:
+            yield ("sync", EMPTY + (m & 1))
+        for q in range(4):
+            yield ("write", ("kw", m & 1, q), m)
+        yield ("arrive", FULL + (m & 1))
+
+
+@pytest.mark.parametrize("mmax", [0, 1, 2, 3, 4, 7])
+def test_response_ring_is_deadlock_and_race_free(mmax):
+    rng = random.Random(100 + mmax)
+    warps = (response_round_warp, response_schedule_warp)
+    for _ in range(1500):
+        run(mmax, rng, warps)
+
+
+def test_model_catches_a_ring_without_the_empty_wait():
+    """A planted mistake: the schedule warp refills a buffer without waiting
+    for the round warp to empty it."""
+    def sw(mmax):
+        for op in response_schedule_warp(mmax):
+            if op[0] != "sync":
+                yield op
+
+    def rw(mmax):
+        for op in response_round_warp(mmax):
+            if op[0] != "arrive":
+                yield op
+
+    sw.__name__, rw.__name__ = "response_schedule_warp", "response_round_warp"
+    with pytest.raises(ProtocolError):
+        for seed in range(200):
+            run(5, random.Random(seed), (rw, sw))
 
 
 @pytest.mark.parametrize("jmax", [0, 1, 2, 3, 5, 8])
