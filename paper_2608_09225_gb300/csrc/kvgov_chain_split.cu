@@ -9,12 +9,15 @@
 //
 // Why a second kernel.  A chain is sequential in its blocks, so parallelism
 // comes only from the batch.  A batch of a few thousand requests gives each
-// SM sub-partition one warp (or none); a warp alone on its sub-partition
-// issues one integer instruction every two cycles (the integer pipe is 16
-// lanes wide), so its time per block is its instruction count, about 2900
-// per block for the two compressions with their message schedules.
-// Here the work of 32 chains is split over two warps on two
-// sub-partitions:
+// SM sub-partition one warp (or none), and a warp alone there runs at the
+// pace of its own instruction stream: at best one integer instruction every
+// two cycles (the integer pipe is 16 lanes wide), in practice slower, since
+// each instruction waits on the one it depends on (measured: a lone warp
+// takes 35 cycles per SHA-256 round with K_t + W_t in registers, two warps
+// sharing a sub-partition 27 each).  Its time per block then grows with the
+// instructions on its path, about 2900 for the two compressions with their
+// message schedules.  Here the work of 32 chains is split over two warps on
+// two sub-partitions:
 //   * the round warp runs only the 64 rounds of each compression (about 14
 //     integer instructions a round) with K_t + W_t read from shared memory;
 //   * the schedule warp stages the tokens (cp.async, two blocks ahead),
