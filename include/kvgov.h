@@ -431,12 +431,20 @@ int kvgov_probe_arrival(const uint64_t *d_owner, uint64_t capacity, const uint32
  * allocation-free form of the same computation (same table, owners, key
  * count and prefix lengths; the slot handles are not returned).
  *   Arguments as for kvgov_insert_arrival and kvgov_probe_arrival;
- *   n_blocks   the batch's block count, d_blk_off[n_req].
- * EINVAL also when n_blocks exceeds 2^21; if d_blk_off[n_req] itself does, no
- * block is inserted and every request is flagged KVGOV_F_BADINDEX with
+ *   n_blocks   the batch's block count, d_blk_off[n_req]; d_digests must
+ *              hold at least n_blocks rows.  Every kernel of the call bounds
+ *              the rows it reads by n_blocks.
+ * EINVAL also when n_blocks exceeds 2^21.  If d_blk_off[n_req] differs from
+ * n_blocks by being larger, no block is inserted, no digest row past
+ * n_blocks is read, and every request is flagged KVGOV_F_BADINDEX with
  * prefix 0.  The array is shared by every call on the device: calls that
  * overlap in time (other streams, other host threads) race on it and give
- * wrong results.  Three launches on `stream`.
+ * wrong results.  Its device address is looked up (cudaGetSymbolAddress) on
+ * the first call made with each device current and kept for the process, so
+ * that first call should come before any stream capture, and the library
+ * does not survive a cudaDeviceReset of that device.  Three launches on
+ * `stream`, four for batches of 4096 requests or more (their first 32
+ * requests' blocks are inserted first, as in kvgov_insert_arrival).
  */
 int kvgov_serve_arrival_static(uint8_t *d_slots, uint64_t *d_owner, uint64_t capacity, const uint8_t *d_digests,
                                const int64_t *d_blk_off, int32_t n_req, int64_t n_blocks, uint64_t seq_base,

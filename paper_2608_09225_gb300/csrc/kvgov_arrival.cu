@@ -37,6 +37,8 @@
 //                          position of r's first block.  The prefix ends at the
 //                          first block that was not (or whose key could not be
 //                          stored).
+#include <atomic>
+
 #include "kvgov_insert.cuh"
 #include "kvgov_internal.cuh"
 
@@ -265,17 +267,23 @@ bool arrival_capacity(uint64_t capacity) {
 constexpr long long kStaticRows = 1ll << 21;
 static __device__ __align__(256) uint32_t g_static_slot_of[kStaticRows];
 
-// Its device address, looked up once per device.
+// Its device address on the current device, looked up with
+// cudaGetSymbolAddress on the first call made with that device current and
+// kept for the life of the process.  Host threads that make their first calls
+// at the same time may each look it up; they store the same address.
 uint32_t *static_slot_of() {
-    static uint32_t *addr[64] = {};
+    constexpr int kMaxDevices = 64;
+    static std::atomic<uint32_t *> addr[kMaxDevices] = {};
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-    if (!addr[dev]) {
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    uint32_t *a = addr[dev].load(std::memory_order_acquire);
+    if (!a) {
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_static_slot_of) != cudaSuccess || !p) return nullptr;
-        addr[dev] = static_cast<uint32_t *>(p);
+        a = static_cast<uint32_t *>(p);
+        addr[dev].store(a, std::memory_order_release);
     }
-    return addr[dev];
+    return a;
 }
 
 }  // namespace
@@ -383,20 +391,25 @@ extern "C" int kvgov_serve_arrival_static(uint8_t *d_slots, uint64_t *d_owner, u
     uint32_t *slot_of = static_slot_of();
     if (!slot_of) return KVGOV_ECUDA;
     // Nothing in the scratch has to start at zero: the insert writes the entry
-    // of every block that the owner min and the probe read.
+    // of every block that the owner min and the probe read.  Every kernel
+    // takes n_blocks (<= kStaticRows) as its row bound, so a batch whose
+    // d_blk_off[n_req] exceeds it reads no digest row past n_blocks and
+    // touches no scratch entry past it: nothing is inserted and the probe
+    // flags every request.
+    const long long row_cap = (long long)n_blocks;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     const unsigned grid = row_grid();
     insert_first_requests(d_slots, capacity, d_owner, d_digests, d_blk_off, n_req, slot_of, d_n_new, d_status,
-                          kStaticRows, seq_base, s);
+                          row_cap, seq_base, s);
     insert_arrival_kernel<<<grid, kThreads, 0, s>>>(reinterpret_cast<unsigned long long *>(d_slots), capacity - 1,
                                                     reinterpret_cast<unsigned long long *>(d_owner),
                                                     reinterpret_cast<const uint4 *>(d_digests), d_blk_off, n_req,
-                                                    slot_of, d_n_new, d_status, kvgov_host::spin_limit(), kStaticRows,
+                                                    slot_of, d_n_new, d_status, kvgov_host::spin_limit(), row_cap,
                                                     seq_base, 0);
     owner_min_kernel<<<grid, kThreads, 0, s>>>(d_blk_off, n_req, slot_of,
-                                               reinterpret_cast<unsigned long long *>(d_owner), seq_base, kStaticRows);
+                                               reinterpret_cast<unsigned long long *>(d_owner), seq_base, row_cap);
     probe_arrival_kernel<<<request_grid(n_req), kThreads, 0, s>>>(reinterpret_cast<const unsigned long long *>(d_owner),
                                                                   slot_of, d_blk_off, n_req, seq_base,
-                                                                  d_prefix_blocks, d_status, kStaticRows);
+                                                                  d_prefix_blocks, d_status, row_cap);
     return kvgov_host::launch_status();
 }

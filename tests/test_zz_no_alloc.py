@@ -1,7 +1,9 @@
 """kvgov_serve_arrival_static (slot handles in the library's static device
 array) against kvgov_insert_arrival + kvgov_probe_arrival (caller scratch):
 the same prefix lengths, key counts and table contents on two consecutive
-calls on one table; oversized batches are refused.  Marked gpu."""
+calls on one table; oversized batches are refused, and a batch whose offsets
+run past the block count it is given is flagged without a read past that
+count.  Marked gpu."""
 import numpy as np
 import pytest
 import torch
@@ -55,3 +57,24 @@ def test_static_scratch_refuses_oversized_batches(kv):
         kv.serve_arrival_static(slots, owner, d, blk, 1, st)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
+
+
+@pytest.mark.parametrize("total", [96, (1 << 21) + 1])
+def test_static_scratch_bounds_rows_by_n_blocks(kv, total):
+    """d_blk_off[n_req] above the n_blocks argument (the digest buffer still
+    holds d_blk_off[n_req] rows, so every read stays inside it either way):
+    nothing is inserted, every request is flagged KVGOV_F_BADINDEX with
+    prefix 0, and the table and owners are unchanged."""
+    digests = torch.full((total, 32), 7, dtype=torch.uint8, device="cuda")
+    digests[:, 0] = torch.arange(total, device="cuda").to(torch.uint8) | 1
+    blk = torch.tensor([0, 40, total], dtype=torch.int64, device="cuda")
+    slots, owner = kv.new_table(256), kv.new_owner(256)
+    slots_before, owner_before = slots.clone(), owner.clone()
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    n_new = torch.zeros(1, dtype=torch.int64, device="cuda")
+    pre = kv.serve_arrival_static(slots, owner, digests[:64], blk, 1, st, n_new=n_new)
+    torch.cuda.synchronize()
+    assert int(st.item()) == kv.F_BADINDEX
+    assert (pre.cpu().numpy() == 0).all()
+    assert int(n_new.item()) == 0
+    assert torch.equal(slots, slots_before) and torch.equal(owner, owner_before)
