@@ -49,7 +49,11 @@ CHAIN_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_chain.cu", "paper_2608_09225
                  "paper_2608_09225_gb300/csrc/kvgov_internal.cuh", "paper_2608_09225_gb300/csrc/kvgov_lookup.cuh",
                  "paper_2608_09225_gb300/csrc/kvgov_insert.cuh"]
 CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain kernel's code
-CHAIN_PROFILE = "profiles/chain_kernel_wide.md"
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per launch of the
+# step's chain kernel from one ncu capture, and the SHA-256 (chain_source_hash)
+# of the sources it was captured from: reported as roofline.traffic only while
+# the kernel's sources still hash to that value.
+CHAIN_TRAFFIC = {"bytes_per_launch": None, "source_sha256": None}
 
 
 def load_peaks() -> dict:
@@ -79,18 +83,13 @@ def chain_source_hash() -> str:
 
 
 def profiled_traffic():
-    """DRAM bytes per chain-kernel launch from the committed ncu summary, if
-    that capture was taken of the chain kernel's current sources; else None."""
-    path = os.path.join(HERE, CHAIN_PROFILE)
-    try:
-        text = open(path).read()
-    except OSError:
-        return None, "no profile"
-    vals = dict(line.split(":", 1) for line in text.splitlines() if line.startswith(("traffic_bytes_per_launch:",
-                                                                                       "source_sha256:")))
-    if vals.get("source_sha256:".rstrip(":"), "").strip() != chain_source_hash():
-        return None, f"{CHAIN_PROFILE} was captured from other sources"
-    return int(vals["traffic_bytes_per_launch"].strip()), CHAIN_PROFILE
+    """DRAM bytes per chain-kernel launch from the last ncu capture, if that
+    capture was taken of the chain kernel's current sources; else None."""
+    if CHAIN_TRAFFIC["bytes_per_launch"] is None:
+        return None, "no capture recorded"
+    if CHAIN_TRAFFIC["source_sha256"] != chain_source_hash():
+        return None, "the last capture was of other sources"
+    return CHAIN_TRAFFIC["bytes_per_launch"], "ncu capture of the current sources"
 
 
 # --------------------------------------------------------------------------- helpers

@@ -47,10 +47,7 @@ DeviceInfo device_info() {
 // Chain kernel
 // ---------------------------------------------------------------------------
 
-#ifndef KVGOV_CHAIN_R
-#define KVGOV_CHAIN_R 128
-#endif
-constexpr int kR = KVGOV_CHAIN_R;   // requests (threads) per CTA
+constexpr int kR = 128;           // requests (threads) per CTA
 constexpr int kStages = 2;        // shared-memory buffers for token blocks
 constexpr int kChunks = 5;        // 16-byte chunks that can cover one 64-byte block
 constexpr int kSlotWords = kChunks * 4;
@@ -66,7 +63,6 @@ struct ChainParams {
     uint32_t *status;
     int32_t n_req;
     int32_t n_principals;
-    uint32_t one;   // 1, opaque to the compiler (see AddFma)
     // fused probe (kvgov_chain_hash_probe) and fused arrival insert
     // (kvgov_chain_hash_arrival) only
     const uint4 *slots;
@@ -101,13 +97,6 @@ constexpr int kFuseNone = 0;      // nothing (kvgov_chain_hash)
 constexpr int kFuseProbe = 1;     // look it up (kvgov_chain_hash_probe)
 constexpr int kFuseArrival = 2;   // insert it, arrival order (kvgov_chain_hash_arrival)
 constexpr int kFuseInsertPrev = 3;   // insert the previous batch's uncached blocks (kvgov_chain_hash_insert_prev)
-
-// Which adder the SHA-256 rounds use.  Measured on GB300: IMAD shares the
-// integer pipe with SHF/LOP3/IADD3 (libkvgov_peak kinds 3-5), so AddFma
-// only adds instructions; plain adds are the default.
-#ifndef KVGOV_FMA_ADDS
-#define KVGOV_FMA_ADDS 0
-#endif
 
 // Big-endian words of principal pi's 32-byte salt.
 __device__ __forceinline__ void load_salt(const uint8_t *salts, int pi, uint32_t sw[8]) {
@@ -197,11 +186,10 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
         cp_async_commit();
     }
 
-#if KVGOV_FMA_ADDS
-    const AddFma add{p.one};
-#else
+    // Plain adds: measured on GB300, issuing them as IMAD (AddFma) only adds
+    // instructions, since IMAD shares the integer pipe with SHF, LOP3 and
+    // IADD3 (libkvgov_peak kinds 3-5).
     const AddAlu add{};
-#endif
     const int sh = (int)(t0 & 3);   // word offset of the block inside its first chunk
     uint32_t h[8];
 #pragma unroll
@@ -466,7 +454,7 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     ChainParams p;
     p.tokens = d_tokens; p.tok_off = d_tok_off; p.principal = d_principal; p.salts = d_salts;
     p.boundary_tok = d_boundary_tok; p.blk_off = d_blk_off; p.digests = d_digests; p.status = d_status;
-    p.n_req = n_req; p.n_principals = n_principals; p.one = 1u;
+    p.n_req = n_req; p.n_principals = n_principals;
     p.slots = reinterpret_cast<const uint4 *>(f.slots);
     p.mask = f.fuse != kFuseNone ? f.capacity - 1 : 0;
     p.prefix_blocks = f.prefix_blocks;

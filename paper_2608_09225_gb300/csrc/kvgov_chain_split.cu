@@ -98,18 +98,10 @@ __device__ __forceinline__ int block_kind(int j, int k) {
     return j == k ? kBoundary : kSteadyH;
 }
 
-// The round warp's 16 rounds (sha256_dev.cuh): the grouping of the sums is a
-// compile-time choice, measured on a lone warp (libkvgov_peak kinds 6, 7).
-#ifndef KVGOV_SPLIT_SHORT_ROUNDS
-#define KVGOV_SPLIT_SHORT_ROUNDS 0
-#endif
-__device__ __forceinline__ void rounds16(uint32_t v[8], const uint32_t kw[16]) {
-#if KVGOV_SPLIT_SHORT_ROUNDS
-    sha_rounds16_short(v, kw);
-#else
-    sha_rounds16_t1t2(v, kw);
-#endif
-}
+// The round warp's 16 rounds (sha256_dev.cuh).  Another grouping of the
+// sums (sha_rounds16_short) measured the same on a lone warp (libkvgov_peak
+// kinds 6, 7).
+__device__ __forceinline__ void rounds16(uint32_t v[8], const uint32_t kw[16]) { sha_rounds16_t1t2(v, kw); }
 
 template <int MODE>
 __global__ void __launch_bounds__(kThreads, 1) chain_split_kernel(const SplitParams p) {
@@ -342,11 +334,9 @@ int launch_mode(unsigned grid, const SplitParams &p, cudaStream_t s) {
 
 namespace kvgov_host {
 
-#ifndef KVGOV_SPLIT_CTAS_PER_SM
-#define KVGOV_SPLIT_CTAS_PER_SM 3   // measured: ahead of chain_kernel up to 3 CTAs (192 chains) per SM
-#endif
+constexpr long long kSplitCtasPerSm = 3;   // measured: ahead of chain_kernel up to 3 CTAs (192 chains) per SM
 
-long long chain_split_max_req() { return (long long)KVGOV_SPLIT_CTAS_PER_SM * sm_count() * kChainsPerCta; }
+long long chain_split_max_req() { return kSplitCtasPerSm * sm_count() * kChainsPerCta; }
 
 namespace {
 

@@ -9,15 +9,6 @@
 
 namespace kvgov_dev {
 
-// Build-time choice (python -m paper_2608_09225_gb300.variants --insert times
-// it): KVGOV_INSERT_LOOK reads a slot before using an atomic on it (default:
-// it turns the step after a cache flush, where every request inserts the same
-// shared-prefix blocks, from ~377 to ~70 us for +5 us on an ordinary step).
-#ifndef KVGOV_INSERT_LOOK
-#define KVGOV_INSERT_LOOK 1
-#endif
-
-
 __device__ __forceinline__ unsigned long long ld_relaxed(const unsigned long long *p) {
     unsigned long long v;
     asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];\n" : "=l"(v) : "l"(p) : "memory");
@@ -33,13 +24,11 @@ __device__ __forceinline__ ulonglong2 ld_plain2(const unsigned long long *p) {
     asm volatile("ld.global.v2.u64 {%0, %1}, [%2];\n" : "=l"(v.x), "=l"(v.y) : "l"(p) : "memory");
     return v;
 }
-#if KVGOV_INSERT_LOOK
 __device__ __forceinline__ ulonglong2 ld_relaxed2(const unsigned long long *p) {
     ulonglong2 v;
     asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];\n" : "=l"(v.x), "=l"(v.y) : "l"(p) : "memory");
     return v;
 }
-#endif
 __device__ __forceinline__ void st_relaxed(unsigned long long *p, unsigned long long v) {
     asm volatile("st.relaxed.gpu.global.u64 [%0], %1;\n" ::"l"(p), "l"(v) : "memory");
 }
@@ -50,11 +39,6 @@ __device__ __forceinline__ void st_relaxed2(unsigned long long *p, unsigned long
     asm volatile("st.relaxed.gpu.global.v2.u64 [%0], {%1, %2};\n" ::"l"(p), "l"(a), "l"(b) : "memory");
 }
 
-// Build-time choice: KVGOV_INSERT_ST16 writes a claimed key's second half
-// with one 16-byte store (default) instead of two 8-byte stores.
-#ifndef KVGOV_INSERT_ST16
-#define KVGOV_INSERT_ST16 1
-#endif
 // 128-bit compare-and-swap of the 16-byte-aligned pair p[0..1]: if it holds
 // (c0, c1) it becomes (n0, n1); the previous value is returned in (o0, o1).
 __device__ __forceinline__ void cas128(unsigned long long *p, unsigned long long c0, unsigned long long c1,
@@ -88,8 +72,9 @@ __device__ __forceinline__ InsertResult insert_one(unsigned long long *slots, un
     for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
         unsigned long long *slot = slots + 4 * pos;
         unsigned long long o0 = 0ull, o1 = 0ull;
-#if KVGOV_INSERT_LOOK
-        // Look first.  A slot's first half is written once, from (0, 0) to
+        // Look first (measured: it turns the step after a cache flush, where
+        // every request inserts the same shared-prefix blocks, from ~377 to
+        // ~70 us for +5 us on an ordinary step).  A slot's first half is written once, from (0, 0) to
         // its final value, so a read racing that write (or an older copy in
         // L1) can only show a zero word; a read with both words non-zero is
         // the final value and needs no atomic (another key: walk on; our
@@ -97,17 +82,10 @@ __device__ __forceinline__ InsertResult insert_one(unsigned long long *slots, un
         const ulonglong2 seen = ld_plain2(slot);
         o0 = seen.x;
         o1 = seen.y;
-        if (o0 == 0ull || o1 == 0ull)
-#endif
-        {
+        if (o0 == 0ull || o1 == 0ull) {
             cas128(slot, 0ull, 0ull, k[0], k[1], o0, o1);
             if ((o0 | o1) == 0ull) {                 // claimed: write the second half
-#if KVGOV_INSERT_ST16
                 st_relaxed2(slot + 2, k[2], k[3]);
-#else
-                st_relaxed(slot + 2, k[2]);
-                st_relaxed(slot + 3, k[3]);
-#endif
                 if (pos_out) *pos_out = pos;
                 return kNew;
             }

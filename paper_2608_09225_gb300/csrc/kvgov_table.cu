@@ -53,17 +53,6 @@ namespace {
 
 using namespace kvgov_dev;
 
-// KVGOV_INSERT_DEDUP elects one lane per distinct key within a warp (off: it
-// costs more on an ordinary step than it saves after a flush).
-#ifndef KVGOV_INSERT_DEDUP
-#define KVGOV_INSERT_DEDUP 0
-#endif
-// KVGOV_INSERT_PACK selects the warp-packed kvgov_insert_uncached kernel
-// (insert_uncached_packed_kernel) over the one with 8 lanes per request.
-#ifndef KVGOV_INSERT_PACK
-#define KVGOV_INSERT_PACK 1
-#endif
-
 constexpr uint32_t kDefaultSpin = 1u << 23;
 std::atomic<uint32_t> g_spin_limit{kDefaultSpin};
 
@@ -77,22 +66,6 @@ __global__ void table_init_kernel(uint4 *__restrict__ slots, unsigned long long 
 // ---------------------------------------------------------------------------
 constexpr int kInsertThreads = 256;
 
-// Insert from the lanes of a warp named in `inserting` (all of which make
-// this call together): lanes holding the same 32 bytes elect their lowest
-// lane to insert; the others are duplicates of that insert.
-__device__ __forceinline__ InsertResult insert_warp_dedup(unsigned long long *slots, unsigned long long mask,
-                                                         const unsigned long long k[4], uint32_t spin_limit,
-                                                         unsigned inserting) {
-#if KVGOV_INSERT_DEDUP
-    const unsigned same = __match_any_sync(inserting, k[0]) & __match_any_sync(inserting, k[1]) &
-                          __match_any_sync(inserting, k[2]) & __match_any_sync(inserting, k[3]);
-    if ((threadIdx.x & 31) != (unsigned)(__ffs(same) - 1)) return kDuplicate;
-#else
-    (void)inserting;
-#endif
-    return insert_one(slots, mask, k, spin_limit);
-}
-
 __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long long *__restrict__ slots,
                                                                 unsigned long long mask,
                                                                 const uint4 *__restrict__ keys, long long n_keys,
@@ -104,8 +77,7 @@ __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long lo
     const long long stride = (long long)gridDim.x * kInsertThreads;
     const int lane = threadIdx.x & 31;
     unsigned int my_new = 0, my_flags = 0;
-    // warp-uniform trip count, so that the lanes inserting in one iteration
-    // are known exactly (the ballot) and meet in insert_warp_dedup
+    // warp-uniform trip count
     for (long long i0 = (long long)blockIdx.x * kInsertThreads + (threadIdx.x & ~31); i0 < n_keys; i0 += stride) {
         const long long i = i0 + lane;
         unsigned long long k[4] = {0ull, 0ull, 0ull, 0ull};
@@ -118,63 +90,21 @@ __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long lo
                 mine = false;
             }
         }
-        const unsigned inserting = __ballot_sync(0xffffffffu, mine);
-        if (mine) count_insert(insert_warp_dedup(slots, mask, k, spin_limit, inserting), my_new, my_flags);
+        if (mine) count_insert(insert_one(slots, mask, k, spin_limit), my_new, my_flags);
     }
     publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
 }
 
 // ---------------------------------------------------------------------------
 constexpr int kProbeThreads = 256;
-// Probe layouts, by batch size (build options, measured side by side by
-// variants.py --probe): probe_seg_kernel<G, kPer, PAIR> with first window F
-//   n_req >= KVGOV_PROBE_MANY_MIN                  (MANY_G, _PER, _PAIR, _FIRST)
-//   KVGOV_PROBE_MID_MIN <= n_req < ..._MANY_MIN     (MID_G, _PER, _PAIR, _FIRST)
-//   n_req < KVGOV_PROBE_MID_MIN                     (FEW_G, _PER, _PAIR, _FIRST)
-// PAIR reads a key's home slot and the next one together (a walk of two
-// slots in one memory round trip) rather than the home slot alone.
-#ifndef KVGOV_PROBE_MANY_MIN
-#define KVGOV_PROBE_MANY_MIN 32768
-#endif
-#ifndef KVGOV_PROBE_MID_MIN
-#define KVGOV_PROBE_MID_MIN 2048
-#endif
-#ifndef KVGOV_PROBE_MANY_G
-#define KVGOV_PROBE_MANY_G 4
-#endif
-#ifndef KVGOV_PROBE_MANY_PER
-#define KVGOV_PROBE_MANY_PER 1
-#endif
-#ifndef KVGOV_PROBE_MANY_PAIR
-#define KVGOV_PROBE_MANY_PAIR 0
-#endif
-#ifndef KVGOV_PROBE_MID_PAIR
-#define KVGOV_PROBE_MID_PAIR 1
-#endif
-#ifndef KVGOV_PROBE_FEW_PAIR
-#define KVGOV_PROBE_FEW_PAIR 1
-#endif
-#ifndef KVGOV_PROBE_MANY_FIRST
-#define KVGOV_PROBE_MANY_FIRST 1
-#endif
-#ifndef KVGOV_PROBE_MID_G
-#define KVGOV_PROBE_MID_G 16
-#endif
-#ifndef KVGOV_PROBE_MID_PER
-#define KVGOV_PROBE_MID_PER 2
-#endif
-#ifndef KVGOV_PROBE_MID_FIRST
-#define KVGOV_PROBE_MID_FIRST 16
-#endif
-#ifndef KVGOV_PROBE_FEW_G
-#define KVGOV_PROBE_FEW_G 32
-#endif
-#ifndef KVGOV_PROBE_FEW_PER
-#define KVGOV_PROBE_FEW_PER 4
-#endif
-#ifndef KVGOV_PROBE_FEW_FIRST
-#define KVGOV_PROBE_FEW_FIRST 32
-#endif
+// Probe layouts by batch size (measured side by side over every workload):
+// probe_seg_kernel<G, kPer, PAIR> with first window F.  PAIR reads a key's
+// home slot and the next one together (a walk of two slots in one memory
+// round trip) rather than the home slot alone.
+struct ProbeLayout { int min_req, G, per, pair, first; };
+constexpr ProbeLayout kProbeMany{32768, 4, 1, 0, 1};    // n_req >= 32768
+constexpr ProbeLayout kProbeMid{2048, 16, 2, 1, 16};    // 2048 <= n_req < 32768
+constexpr ProbeLayout kProbeFew{0, 32, 4, 1, 32};       // fewer
 
 // Request r's block range; a malformed one is flagged and counts as empty.
 __device__ __forceinline__ void probe_range(const int64_t *__restrict__ blk_off, int32_t n_req, long long r,
@@ -263,61 +193,13 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
 
 // Insert every request's blocks from its cached-prefix length on (the output
 // of kvgov_probe): the blocks before it were found in the table, and a table
-// only grows, so inserting them would change nothing.  G lanes per request.
-template <int G>
-__global__ void __launch_bounds__(kInsertThreads) insert_uncached_kernel(
-    unsigned long long *__restrict__ slots, unsigned long long mask, const uint4 *__restrict__ digests,
-    const int64_t *__restrict__ blk_off, int32_t n_req, const int32_t *__restrict__ prefix_blocks,
-    unsigned long long *n_new, uint32_t *status, uint32_t spin_limit) {
-    __shared__ unsigned int s_new, s_flags, s_done;
-    if (threadIdx.x == 0) { s_new = 0; s_flags = 0; s_done = 0; }
-    __syncthreads();
-    constexpr int kSegs = 32 / G;
-    const int lane = threadIdx.x & 31, seg = lane / G, sl = lane % G;
-    const long long warps_total = (long long)gridDim.x * (kInsertThreads / 32);
-    unsigned my_new = 0, my_flags = 0;
-    for (long long w = ((long long)blockIdx.x * kInsertThreads + threadIdx.x) / 32; w * kSegs < n_req;
-         w += warps_total) {                                   // warp-uniform
-        const long long r = w * kSegs + seg;
-        long long base = 0, nb = 0, L = 0;
-        if (r < n_req) {
-            base = blk_off[r];
-            nb = blk_off[r + 1] - base;
-            if (nb < 0 || base < 0 || base + nb > blk_off[n_req]) {
-                if (sl == 0) my_flags |= KVGOV_F_BADINDEX;
-                nb = 0;
-            }
-            L = prefix_blocks[r];
-            if (L < 0) L = 0;
-        }
-        const long long left = nb - L - sl;
-        const int iters = left > 0 ? (int)((left + G - 1) / G) : 0;
-        const int wmax = __reduce_max_sync(0xffffffffu, iters);
-        for (int it = 0; it < wmax; ++it) {
-            unsigned long long k[4] = {0ull, 0ull, 0ull, 0ull};
-            bool mine = it < iters;
-            if (mine) {
-                const long long row = base + L + sl + (long long)it * G;
-                const uint4 a = __ldg(digests + 2 * row), b = __ldg(digests + 2 * row + 1);
-                k[0] = u64_of(a.x, a.y); k[1] = u64_of(a.z, a.w); k[2] = u64_of(b.x, b.y); k[3] = u64_of(b.z, b.w);
-                if (key_reserved(k)) {
-                    my_flags |= KVGOV_F_SENTINEL;
-                    mine = false;
-                }
-            }
-            const unsigned inserting = __ballot_sync(0xffffffffu, mine);
-            if (mine) count_insert(insert_warp_dedup(slots, mask, k, spin_limit, inserting), my_new, my_flags);
-        }
-    }
-    publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
-}
-
-// The same insert with the uncached blocks of kPackReq requests packed into
-// the 32 lanes of a warp: lanes 0..kPackReq-1 read their request's range and
+// only grows, so inserting them would change nothing.  The uncached blocks
+// of kPackReq requests are packed into the 32 lanes of a warp: lanes 0..kPackReq-1 read their request's range and
 // count of uncached blocks, a warp scan numbers the blocks, and in each round
 // lane l takes block i0 + l, finding its request with a 5-step search over the
 // scan.  No lane idles while blocks remain (with 8 lanes per request, a
-// request with 4 cached and 4 uncached blocks leaves half the lanes idle).
+// request with 4 cached and 4 uncached blocks leaves half the lanes idle;
+// measured faster than that layout).
 constexpr int kPackReq = 8;
 
 __global__ void __launch_bounds__(kInsertThreads) insert_uncached_packed_kernel(
@@ -376,8 +258,7 @@ __global__ void __launch_bounds__(kInsertThreads) insert_uncached_packed_kernel(
                     mine = false;
                 }
             }
-            const unsigned inserting = __ballot_sync(0xffffffffu, mine);
-            if (mine) count_insert(insert_warp_dedup(slots, mask, key, spin_limit, inserting), my_new, my_flags);
+            if (mine) count_insert(insert_one(slots, mask, key, spin_limit), my_new, my_flags);
         }
     }
     publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
@@ -428,18 +309,18 @@ extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint
     if (!d_digests || !aligned16(d_digests) || !d_blk_off || !d_prefix_blocks) return KVGOV_EINVAL;
     const uint4 *slots = reinterpret_cast<const uint4 *>(d_slots), *dig = reinterpret_cast<const uint4 *>(d_digests);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    if (n_req >= KVGOV_PROBE_MANY_MIN)
-        probe_seg_kernel<KVGOV_PROBE_MANY_G, KVGOV_PROBE_MANY_PER, (KVGOV_PROBE_MANY_PAIR != 0)>
-            <<<probe_grid(n_req, KVGOV_PROBE_MANY_G), kProbeThreads, 0, s>>>(
-                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, KVGOV_PROBE_MANY_FIRST);
-    else if (n_req >= KVGOV_PROBE_MID_MIN)
-        probe_seg_kernel<KVGOV_PROBE_MID_G, KVGOV_PROBE_MID_PER, (KVGOV_PROBE_MID_PAIR != 0)>
-            <<<probe_grid(n_req, KVGOV_PROBE_MID_G), kProbeThreads, 0, s>>>(
-                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, KVGOV_PROBE_MID_FIRST);
+    if (n_req >= kProbeMany.min_req)
+        probe_seg_kernel<kProbeMany.G, kProbeMany.per, kProbeMany.pair != 0>
+            <<<probe_grid(n_req, kProbeMany.G), kProbeThreads, 0, s>>>(
+                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, kProbeMany.first);
+    else if (n_req >= kProbeMid.min_req)
+        probe_seg_kernel<kProbeMid.G, kProbeMid.per, kProbeMid.pair != 0>
+            <<<probe_grid(n_req, kProbeMid.G), kProbeThreads, 0, s>>>(
+                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, kProbeMid.first);
     else
-        probe_seg_kernel<KVGOV_PROBE_FEW_G, KVGOV_PROBE_FEW_PER, (KVGOV_PROBE_FEW_PAIR != 0)>
-            <<<probe_grid(n_req, KVGOV_PROBE_FEW_G), kProbeThreads, 0, s>>>(
-                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, KVGOV_PROBE_FEW_FIRST);
+        probe_seg_kernel<kProbeFew.G, kProbeFew.per, kProbeFew.pair != 0>
+            <<<probe_grid(n_req, kProbeFew.G), kProbeThreads, 0, s>>>(
+                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, kProbeFew.first);
     return kvgov_host::launch_status();
 }
 
@@ -451,21 +332,12 @@ extern "C" int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const 
         return KVGOV_EINVAL;
     if (n_req == 0) return KVGOV_OK;
     if (!d_digests || !aligned16(d_digests) || !d_blk_off || !d_prefix_blocks) return KVGOV_EINVAL;
-#if KVGOV_INSERT_PACK
     const long long warps = ((long long)n_req + kPackReq - 1) / kPackReq;
     long long grid = (warps + (kInsertThreads / 32) - 1) / (kInsertThreads / 32);
     if (grid > 152ll * 64) grid = 152ll * 64;
     insert_uncached_packed_kernel<<<(unsigned)grid, kInsertThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
         reinterpret_cast<unsigned long long *>(d_slots), capacity - 1, reinterpret_cast<const uint4 *>(d_digests),
         d_blk_off, n_req, d_prefix_blocks, d_n_new, d_status, g_spin_limit.load());
-#else
-    constexpr int G = 8;
-    long long grid = ((long long)n_req * G + kInsertThreads - 1) / kInsertThreads;
-    if (grid > 152ll * 64) grid = 152ll * 64;
-    insert_uncached_kernel<G><<<(unsigned)grid, kInsertThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-        reinterpret_cast<unsigned long long *>(d_slots), capacity - 1, reinterpret_cast<const uint4 *>(d_digests),
-        d_blk_off, n_req, d_prefix_blocks, d_n_new, d_status, g_spin_limit.load());
-#endif
     return kvgov_host::launch_status();
 }
 

@@ -51,7 +51,6 @@ __device__ __forceinline__ void sha_iv(uint32_t s[8]) {
 __device__ __forceinline__ uint32_t rotr(uint32_t x, int n) { return __funnelshift_r(x, x, n); }
 
 // LOP3 truth tables over (a = 0xF0, b = 0xCC, c = 0xAA).
-#ifndef KVGOV_PLAIN_BOOL
 __device__ __forceinline__ uint32_t xor3(uint32_t a, uint32_t b, uint32_t c) {
     uint32_t r;
     asm("lop3.b32 %0, %1, %2, %3, 0x96;" : "=r"(r) : "r"(a), "r"(b), "r"(c));
@@ -69,11 +68,6 @@ __device__ __forceinline__ uint32_t maj(uint32_t x, uint32_t y, uint32_t z) {
     asm("lop3.b32 %0, %1, %2, %3, 0xE8;" : "=r"(r) : "r"(x), "r"(y), "r"(z));
     return r;
 }
-#else
-__device__ __forceinline__ uint32_t xor3(uint32_t a, uint32_t b, uint32_t c) { return a ^ b ^ c; }
-__device__ __forceinline__ uint32_t ch(uint32_t x, uint32_t y, uint32_t z) { return (x & y) ^ (~x & z); }
-__device__ __forceinline__ uint32_t maj(uint32_t x, uint32_t y, uint32_t z) { return (x & y) | (z & (x | y)); }
-#endif
 
 __device__ __forceinline__ uint32_t bsig0(uint32_t x) { return xor3(rotr(x, 2), rotr(x, 13), rotr(x, 22)); }
 __device__ __forceinline__ uint32_t bsig1(uint32_t x) { return xor3(rotr(x, 6), rotr(x, 11), rotr(x, 25)); }
@@ -86,9 +80,9 @@ __device__ __forceinline__ uint32_t bswap32(uint32_t x) { return __byte_perm(x, 
 // Adders.  Every 32-bit add of the compression goes through one of these.
 // AddAlu is a plain add (the compiler emits IADD3 on the integer ALU pipe,
 // the pipe that also carries every SHF and LOP3).  AddFma issues the add as
-// IMAD a * one + b on the FMA pipe, which SHA-256 otherwise leaves idle;
-// `one` is a runtime 1 from the launch parameters, so the compiler cannot
-// turn the multiply-add back into an ALU add.
+// IMAD a * one + b, with `one` a runtime 1 so that the compiler cannot turn
+// the multiply-add back into an ALU add; only the integer microbenchmark
+// (int_peak.cu) uses it, to measure that IMAD shares the integer pipe.
 struct AddAlu {
     __device__ __forceinline__ uint32_t operator()(uint32_t a, uint32_t b) const { return a + b; }
 };
@@ -228,20 +222,12 @@ __device__ __forceinline__ void sha_rounds16_short(uint32_t v[8], const uint32_t
     }
 }
 
-// Compression of a data block inside the fixed-length messages below:
-// compact (default; measured faster for the chain kernel on GB300, whose
-// fully unrolled form stalls on instruction fetch) or fully unrolled
-// (KVGOV_COMPACT_ROUNDS=0).
-#ifndef KVGOV_COMPACT_ROUNDS
-#define KVGOV_COMPACT_ROUNDS 1
-#endif
+// Compression of a data block inside the fixed-length messages below: the
+// compact form (measured faster for the chain kernel on GB300, whose fully
+// unrolled form stalls on instruction fetch).
 template <bool FROM_IV, class Add>
 __device__ __forceinline__ void sha_compress_data(uint32_t s[8], uint32_t w[16], Add add) {
-#if KVGOV_COMPACT_ROUNDS
     sha_compress_small(s, w, add);
-#else
-    sha_compress_t<false, FROM_IV>(s, w, add);
-#endif
 }
 
 // Fixed-length messages of the chain (section 2.1 / 4.1 / 4.2 equations).
