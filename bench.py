@@ -457,7 +457,7 @@ def main():
     share_prefix(pool_host)
     w0 = pool_host[0]
     n_req = w0.batch.n
-    n_blocks = int((w0.batch.lengths() // 16).sum())
+    n_blocks, w0_blk = K.count_blocks(w0.batch.tok_off)
     new_per_step = 4 * n_req                       # the salted blocks 4..7 of every request
     pool = [DeviceBatch.from_host(w.batch.tokens, w.batch.tok_off, w.batch.principal, w.batch.boundary_tok)
             for w in pool_host]
@@ -568,8 +568,7 @@ def main():
 
     # ---- roofline of the chain kernel (integer-pipe bound)
     micro = measure_int_peak(torch, kbuild.PEAK_LIB)
-    nb = (w0.batch.lengths() // 16)
-    ops = nominal_chain_ops(nb, 2, w0.batch.boundary_tok // 16)
+    ops = nominal_chain_ops(np.diff(w0_blk), 2, w0.batch.boundary_tok // K.BLOCK)
     achieved = ops / (chain_ms / 1e3) / 1e12
     clock = clk.summary()
     n_sm = micro["n_sm"]
@@ -730,7 +729,7 @@ def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots, in_chain=Tr
                             for a in (b.tokens, b.tok_off, b.principal, b.boundary_tok)))
     n_req = hosts[0].batch.n
     n_tok = int(hosts[0].batch.tok_off[-1])
-    n_blocks = int((hosts[0].batch.lengths() // 16).sum())
+    n_blocks, _ = K.count_blocks(hosts[0].batch.tok_off)
     cache = PrefixCache(table_slots, w0.secret, w0.ids, w0.id_off)
     pipe = HostPipeline(cache, W.BOUNDARY, n_req, n_tok, insert_in_chain=in_chain)
     flush = FlushPolicy(table_slots, 4 * n_req)
@@ -889,7 +888,8 @@ def run_configs(args):
     names = {W.UNSALTED: "UNSALTED", W.ROOT: "ROOT", W.BOUNDARY: "BOUNDARY"}
     for name, w, mode in plan:
         b = w.batch
-        cap = w.capacity or next_pow2(4 * int((b.lengths() // 16).sum()))
+        nb_all = np.diff(K.count_blocks(b.tok_off)[1])     # blocks per request
+        cap = w.capacity or next_pow2(4 * int(nb_all.sum()))
         cache = PrefixCache(cap, w.secret, w.ids, w.id_off)
         db = DeviceBatch.from_host(b.tokens, b.tok_off, b.principal, b.boundary_tok)
         n_blocks = db.n_blocks
@@ -981,7 +981,7 @@ def run_configs(args):
         L = K.probe(cache.slots, dig, pblk_view).cpu().numpy()
         nb = np.diff(blk_np[p0:p1 + 1])
         algo_probes = int(np.minimum(L + 1, nb).sum())
-        ops = nominal_chain_ops(b.lengths() // 16, mode, b.boundary_tok // 16)
+        ops = nominal_chain_ops(nb_all, mode, b.boundary_tok // K.BLOCK)
         # algorithmic table bytes, linear probing at load factor a: a hit walks 1/2 (1 + 1/(1-a)) slots,
         # a miss 1/2 (1 + 1/(1-a)^2); a fill from empty to a averages 1/2 (1 + 1/(1-a)) per insert
         a = keys.shape[0] / cap
@@ -992,8 +992,7 @@ def run_configs(args):
         # a batch that leaves every round warp alone on its sub-partition (at most 64 chains
         # per SM) is bound by the latency of its longest chain: 2 compressions per block,
         # one more for a boundary block, 64 rounds each at the lone-warp round time
-        nb_all = b.lengths() // 16
-        k_all = b.boundary_tok // 16
+        k_all = b.boundary_tok // K.BLOCK
         comp = 2 * nb_all + ((k_all >= 1) & (k_all < nb_all) if mode == W.BOUNDARY else 0)
         lat_ms = (float(comp.max()) * 64 * round_cycles / (SM_MAX_MHZ * 1e3)
                   if 0 < b.n <= 64 * n_sm else None)
@@ -1002,7 +1001,7 @@ def run_configs(args):
                 "chain_ms": t_chain, "chain_digests_per_s": n_blocks / (t_chain / 1e3),
                 "chain_tokens_per_s": 16 * n_blocks / (t_chain / 1e3),
                 "chain_frac_int32_peak": ops / (t_chain / 1e3) / peak,
-                "chain_us_per_block_per_chain": 1e3 * t_chain / max(1, int((b.lengths() // 16).max())),
+                "chain_us_per_block_per_chain": 1e3 * t_chain / max(1, int(nb_all.max())),
                 "chain_latency_bound_ms": lat_ms,
                 "chain_frac_latency_bound": (lat_ms / t_chain) if lat_ms else None,
                 "fused_chain_probe_ms": t_fused, "salts_ms": t_salts, "block_offsets_ms": t_blk,

@@ -97,6 +97,21 @@ int kvgov_block_offsets(const int64_t *d_tok_off, int32_t n_req, int64_t *d_blk_
                         uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * kvgov_count_blocks -- the blocking of kvgov_block_offsets computed on the
+ * host, for sizing buffers before any launch: *n_blocks = the sum over
+ * requests of floor(len_r / 16) (paper section 2.1), a negative len_r
+ * counting 0, so it equals the d_blk_off[n_req] that kvgov_block_offsets
+ * writes for the same offsets.
+ *   h_tok_off [n_req + 1] int64 HOST token offsets (CSR).
+ *   h_blk_off [n_req + 1] int64 HOST output, nullable: the same exclusive
+ *             prefix sum kvgov_block_offsets writes.
+ *   n_blocks  HOST output, required.
+ * Runs on the calling thread; touches no device.  EINVAL: n_req < 0, a NULL
+ * h_tok_off or n_blocks.
+ */
+int kvgov_count_blocks(const int64_t *h_tok_off, int32_t n_req, int64_t *h_blk_off, int64_t *n_blocks);
+
+/*
  * kvgov_divergence_boundary -- where each request's salt goes in, paper
  * section 4.2 (salt at the divergence boundary k: the blocks before it hold
  * the shared preamble, which tells no principal apart) and section 5.7 (a

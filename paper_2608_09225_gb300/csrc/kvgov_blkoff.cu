@@ -160,3 +160,18 @@ extern "C" int kvgov_block_offsets(const int64_t *d_tok_off, int32_t n_req, int6
     blkoff_scan_kernel<<<grid, kScanThreads, 0, s>>>(d_tok_off, n_req, d_blk_off, per);
     return kvgov_host::launch_status();
 }
+
+extern "C" int kvgov_count_blocks(const int64_t *h_tok_off, int32_t n_req, int64_t *h_blk_off, int64_t *n_blocks) {
+    if (n_req < 0 || !h_tok_off || !n_blocks) return KVGOV_EINVAL;
+    // floor(len_r / 16) per request, a negative length counting 0, as
+    // blocks_of does on the device
+    long long total = 0;
+    if (h_blk_off) h_blk_off[0] = 0;
+    for (int32_t r = 0; r < n_req; ++r) {
+        const long long len = h_tok_off[r + 1] - h_tok_off[r];
+        total += len < 0 ? 0 : len / KVGOV_BLOCK;
+        if (h_blk_off) h_blk_off[r + 1] = total;
+    }
+    *n_blocks = total;
+    return KVGOV_OK;
+}

@@ -66,6 +66,7 @@ def _load():
         L.kvgov_status_string.argtypes = [ctypes.c_int]
         L.kvgov_status_string.restype = ctypes.c_char_p
         L.kvgov_block_offsets.argtypes = [_p, ctypes.c_int32, _p, _p, _p]
+        L.kvgov_count_blocks.argtypes = [_p, ctypes.c_int32, _p, _p]
         L.kvgov_derive_salts.argtypes = [_p, ctypes.c_size_t, _p, _p, ctypes.c_int32, _p, _p, _p]
         L.kvgov_chain_hash.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p, _p,
                                        _p, _p]
@@ -99,7 +100,7 @@ def _load():
         L.kvgov_pipeline_pending.argtypes = [_p]
         L.kvgov_pipeline_destroy.argtypes = [_p]
         L.kvgov_pipeline_destroy.restype = None
-        for fn in ("kvgov_block_offsets", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
+        for fn in ("kvgov_block_offsets", "kvgov_count_blocks", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
                    "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
                    "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
                    "kvgov_divergence_boundary", "kvgov_response_key", "kvgov_origami",
@@ -154,6 +155,21 @@ def block_offsets(tok_off: torch.Tensor, blk_off: torch.Tensor | None = None,
                                  _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_block_offsets")
     return blk_off
+
+
+def count_blocks(tok_off) -> tuple[int, "np.ndarray"]:
+    """kvgov_count_blocks on host offsets (numpy or a CPU tensor): the batch's
+    block count and its block offsets, as kvgov_block_offsets computes them."""
+    import numpy as np
+    off = np.ascontiguousarray(tok_off.cpu().numpy() if isinstance(tok_off, torch.Tensor) else tok_off,
+                               dtype=np.int64)
+    n = off.size - 1
+    blk = np.empty(max(n, 0) + 1, dtype=np.int64)
+    total = ctypes.c_int64(0)
+    if n < 0:
+        raise ValueError("tok_off needs at least one entry")
+    _check(lib().kvgov_count_blocks(off.ctypes.data, n, blk.ctypes.data, ctypes.byref(total)), "kvgov_count_blocks")
+    return int(total.value), blk
 
 
 def derive_salts(secret: bytes, ids: torch.Tensor, id_off: torch.Tensor, salts: torch.Tensor | None = None,

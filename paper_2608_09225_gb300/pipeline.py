@@ -39,7 +39,7 @@ class DeviceBatch:
     @staticmethod
     def from_host(tokens, tok_off, principal, boundary_tok, device="cuda", non_blocking=False) -> "DeviceBatch":
         tok_off_np = np.asarray(tok_off, dtype=np.int64)
-        n_blocks = int((np.diff(tok_off_np) // K.BLOCK).sum())
+        n_blocks, _ = K.count_blocks(tok_off_np)
 
         def put(a, dt):
             t = a if isinstance(a, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(a, dtype=dt))
@@ -255,7 +255,8 @@ class HostPipeline(_Pipelined):
 
     def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_tokens: int, device="cuda",
                  insert_in_chain: bool = True):
-        super().__init__(cache, mode, max_req, max_tokens // K.BLOCK, device, insert_in_chain)
+        max_blocks, _ = K.count_blocks([0, max_tokens])        # no batch of max_tokens tokens has more
+        super().__init__(cache, mode, max_req, max_blocks, device, insert_in_chain)
         self.copy_stream = torch.cuda.Stream(self.device)
         self.out_stream = torch.cuda.Stream(self.device)
         for s in self.slots:

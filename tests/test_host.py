@@ -324,3 +324,32 @@ def test_oracle_key_reserved_rule():
     assert oracle.key_reserved(one + one + one + bytes(8))
     assert not oracle.key_reserved(bytes(8) + one + one + one)
     assert not oracle.key_reserved(b"\xff" * 8 + one + one + one)
+
+
+def test_count_blocks_on_the_host(libkv):
+    """kvgov_count_blocks (host code, no device) against the oracle's
+    blocking: the same block offsets on ragged lengths (tails of 0..15 tokens,
+    empty requests, the workloads' shapes), a negative length counting 0 as
+    on the device, and its argument checks."""
+    p = ctypes.c_void_p
+    cb = libkv.kvgov_count_blocks
+    cb.argtypes = [p, ctypes.c_int32, p, p]
+    rng = np.random.default_rng(41)
+    for lens in (np.array([0, 1, 15, 16, 17, 31, 32, 2119, 128, 0], np.int64), rng.integers(0, 5000, 777),
+                 np.full(64, 256), np.zeros(0, np.int64)):
+        tok_off = np.zeros(len(lens) + 1, np.int64)
+        tok_off[1:] = np.cumsum(lens)
+        blk = np.empty(len(lens) + 1, np.int64)
+        total = ctypes.c_int64(-1)
+        assert cb(tok_off.ctypes.data, len(lens), blk.ctypes.data, ctypes.byref(total)) == 0
+        want = oracle.block_offsets(tok_off)
+        assert (blk == want).all() and total.value == int(want[-1])
+        assert cb(tok_off.ctypes.data, len(lens), None, ctypes.byref(total)) == 0 and total.value == int(want[-1])
+    bad = np.array([0, 40, 20, 60], np.int64)                 # request 1 has length -20
+    blk = np.empty(4, np.int64)
+    total = ctypes.c_int64(-1)
+    assert cb(bad.ctypes.data, 3, blk.ctypes.data, ctypes.byref(total)) == 0
+    assert list(blk) == [0, 2, 2, 4] and total.value == 4
+    assert cb(None, 3, None, ctypes.byref(total)) == 1
+    assert cb(bad.ctypes.data, -1, None, ctypes.byref(total)) == 1
+    assert cb(bad.ctypes.data, 3, None, None) == 1
