@@ -19,7 +19,7 @@ import threading
 import numpy as np
 
 UNSALTED, ROOT, BOUNDARY = 0, 1, 2
-FLAG_RESERVED = 1
+FLAG_ZERO_KEY = 1
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "oracle.c")
@@ -56,8 +56,8 @@ def _configure(L):
     L.oracle_block_offsets.restype = ctypes.c_int
     L.oracle_chain_hash.argtypes = [ctypes.c_int, _p, _p, _i32, _p, _p, _i32, _p, _p]
     L.oracle_chain_hash.restype = ctypes.c_int
-    L.oracle_key_reserved.argtypes = [_p]
-    L.oracle_key_reserved.restype = ctypes.c_int
+    L.oracle_key_is_zero.argtypes = [_p]
+    L.oracle_key_is_zero.restype = ctypes.c_int
     L.oracle_set_insert.argtypes = [_p, _p, _i64, _p, _i64, _p]
     L.oracle_set_insert.restype = _i64
     L.oracle_prefix_blocks.argtypes = [_p, _i64, _p, _p, _i32, _p]
@@ -243,9 +243,10 @@ def origami(values: np.ndarray, off: np.ndarray, budget: np.ndarray):
     return p[: int(off[-1])], lam[:n], u[:n], bool(rc)
 
 
-def key_reserved(key: bytes) -> bool:
+def key_is_zero(key: bytes) -> bool:
+    """The one key the set refuses: all 32 bytes zero."""
     k = np.frombuffer(bytes(key), dtype=np.uint8)
-    return bool(lib().oracle_key_reserved(_ptr(k)))
+    return bool(lib().oracle_key_is_zero(_ptr(k)))
 
 
 class KeySet:
@@ -256,7 +257,8 @@ class KeySet:
         self.n = 0
 
     def insert(self, keys: np.ndarray):
-        """Returns (n_new, reserved_flag)."""
+        """Returns (n_new, zero_key_flag): the keys the set gained, and whether
+        an all-zero key was given (and skipped)."""
         keys = _c(keys, np.uint8).reshape(-1, 32)
         if self.n + keys.shape[0] > self.keys.shape[0]:
             grown = np.zeros((self.n + keys.shape[0], 32), np.uint8)
@@ -269,7 +271,7 @@ class KeySet:
         if rc < 0:
             raise ValueError("KeySet capacity exceeded")
         self.n = n_set.value
-        return n_new.value, bool(rc & FLAG_RESERVED)
+        return n_new.value, bool(rc & FLAG_ZERO_KEY)
 
     def contents(self) -> np.ndarray:
         return self.keys[: self.n]

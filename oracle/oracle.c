@@ -41,10 +41,10 @@
  *
  * The cache index is modelled as a mathematical set of 32-byte keys, kept as
  * a sorted array searched with bsearch; it has nothing in common with the
- * GPU's open-addressing table except the keys it holds.  Keys whose bytes
- * 0..15, 16..23 or 24..31 are all zero are reserved by the GPU table
- * encoding (empty slot, key still being written); the set refuses them the
- * same way.
+ * GPU's open-addressing table except the keys it holds.  Every 32-byte key
+ * but one can be a member: the all-zero key is refused, as the library's
+ * boundary refuses it (it is the value of an empty slot).  A SHA-256 digest
+ * equals it with probability 2^-256.
  *
  * Parity pins (tests/test_oracle_pins.py): SHA-256 against Python hashlib on
  * every message length 0..300 and random messages; HMAC against Python hmac;
@@ -331,23 +331,16 @@ int oracle_chain_hash(int mode, const int32_t *tokens, const int64_t *tok_off,
 /* The cache index as a set; paper section 2.1 / Table 1 row 1 lookup     */
 /* --------------------------------------------------------------------- */
 
-#define ORACLE_FLAG_RESERVED 1u
+#define ORACLE_FLAG_ZERO_KEY 1u
 
 static int key_cmp(const void *a, const void *b) { return memcmp(a, b, 32); }
 
-/* Keys the GPU table cannot store (see header): bytes 0..15 all zero (an
- * empty slot), or bytes 16..23 or 24..31 all zero (a key still being
- * written). */
-int oracle_key_reserved(const uint8_t *key)
+/* The one key the set refuses (see header): all 32 bytes zero. */
+int oracle_key_is_zero(const uint8_t *key)
 {
-    int lo = 1, mid = 1, hi = 1;
-    for (int i = 0; i < 16; i++)
-        if (key[i] != 0) lo = 0;
-    for (int i = 16; i < 24; i++)
-        if (key[i] != 0) mid = 0;
-    for (int i = 24; i < 32; i++)
-        if (key[i] != 0) hi = 0;
-    return lo || mid || hi;
+    for (int i = 0; i < 32; i++)
+        if (key[i] != 0) return 0;
+    return 1;
 }
 
 int oracle_set_contains(const uint8_t *set_keys, int64_t n_set, const uint8_t *key)
@@ -357,12 +350,12 @@ int oracle_set_contains(const uint8_t *set_keys, int64_t n_set, const uint8_t *k
 
 /*
  * Add keys to the set held sorted and duplicate-free in set_keys[0..*n_set)
- * (room for set_cap keys): append the storable keys, sort, drop repeats.
- * Duplicates, within the batch or with the set, are therefore no-ops, and
- * the result does not depend on the order of keys.  *n_new receives how many
- * keys the set gained.  Returns ORACLE_FLAG_RESERVED if any key was reserved
- * (it is skipped), 0 otherwise, or -1 if set_cap is too small for the
- * appended keys.
+ * (room for set_cap keys): append every key but the all-zero one, sort,
+ * drop repeats.  Duplicates, within the batch or with the set, are therefore
+ * no-ops, and the result does not depend on the order of keys.  *n_new
+ * receives how many keys the set gained.  Returns ORACLE_FLAG_ZERO_KEY if an
+ * all-zero key was given (it is skipped), 0 otherwise, or -1 if set_cap is
+ * too small for the appended keys.
  */
 int64_t oracle_set_insert(uint8_t *set_keys, int64_t *n_set, int64_t set_cap,
                           const uint8_t *keys, int64_t n_keys, int64_t *n_new)
@@ -370,7 +363,7 @@ int64_t oracle_set_insert(uint8_t *set_keys, int64_t *n_set, int64_t set_cap,
     int64_t flags = 0, n = *n_set;
     for (int64_t i = 0; i < n_keys; i++) {
         const uint8_t *key = keys + 32 * (size_t)i;
-        if (oracle_key_reserved(key)) { flags |= ORACLE_FLAG_RESERVED; continue; }
+        if (oracle_key_is_zero(key)) { flags |= ORACLE_FLAG_ZERO_KEY; continue; }
         if (n >= set_cap) return -1;
         memcpy(set_keys + 32 * (size_t)n, key, 32);
         n++;
@@ -416,7 +409,8 @@ int oracle_prefix_blocks(const uint8_t *set_keys, int64_t n_set,
  * definition: the requests are taken one at a time, in order.  Request r's
  * prefix length is its number of leading blocks present in the set as it
  * stands -- the keys given (cached before the batch) plus every block of
- * requests 0..r-1 -- and then all of r's storable blocks join the set.
+ * requests 0..r-1 -- and then all of r's blocks join the set (the all-zero
+ * key excepted).
  *
  * The set is a chained hash set: bucket heads indexed by bytes 8..15 of the
  * key, a node array with next links, keys compared whole.
@@ -459,8 +453,7 @@ static int chain_set_add(chain_set *s, const uint8_t *k)
  * set_keys[0..n_set): the keys cached before the batch.  digests, blk_off,
  * n_req: the batch (request-major digests, block offsets).  prefix_blocks
  * [n_req] receives the prefix lengths, *n_new how many keys the batch added
- * to the set.  Reserved keys (oracle_key_reserved) are never added, as in
- * oracle_set_insert.  Returns 0, or -1 for malformed offsets or no memory.
+ * to the set.  The all-zero key is never added, as in oracle_set_insert.  Returns 0, or -1 for malformed offsets or no memory.
  */
 int oracle_arrival_prefix(const uint8_t *set_keys, int64_t n_set, const uint8_t *digests,
                           const int64_t *blk_off, int32_t n_req, int32_t *prefix_blocks,
@@ -494,7 +487,7 @@ int oracle_arrival_prefix(const uint8_t *set_keys, int64_t n_set, const uint8_t 
             j++;
         prefix_blocks[r] = (int32_t)j;
         for (int64_t q = 0; q < nb; q++)
-            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);
+            if (!oracle_key_is_zero(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);
     }
     *n_new = s.n - before;
     free(s.head); free(s.next); free(s.key);

@@ -193,10 +193,6 @@ def probe(seed: int = 2029, n_req: int = 65536, n_prior: int = 8192, capacity: i
     if n_random is None:
         n_random = capacity // 2 - n_prior * 32
     keys = rng.integers(0, 256, size=(max(n_random, 0), 32), dtype=np.uint8)
-    # keys with bytes 0-15, 16-23 or 24-31 all zero are not storable
-    bad = (np.all(keys[:, :16] == 0, axis=1) | np.all(keys[:, 16:24] == 0, axis=1)
-           | np.all(keys[:, 24:] == 0, axis=1))
-    keys[bad] |= 1
     ids, id_off = principal_ids(1024)
     w = Workload("probe", seed, secret, ids, id_off, _regular(toks, principal),
                  modes=(ROOT,), capacity=capacity, fill=(0, n_prior), fill_from="prior",

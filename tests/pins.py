@@ -278,7 +278,9 @@ def pin_prefix_brute_force():
         nb = rng.integers(0, 12, 30)
         off = np.concatenate([[0], np.cumsum(nb)]).astype(np.int64)
         pool = rng.integers(0, 256, (8, 32), dtype=np.uint8)
-        pool[:, 0] |= 1                                   # no reserved keys
+        pool[:, 31] |= 1                                  # no all-zero key
+        pool[0, :16] = 0                                  # zero first half: an ordinary key
+        pool[1, 16:24] = 0                                # a zero 8-byte word: an ordinary key
         digests = pool[rng.integers(0, 8, int(off[-1]))]
         member = rng.random(8) < 0.6
         ks = oracle.KeySet(1)
@@ -293,8 +295,11 @@ def pin_prefix_brute_force():
 
 
 def pin_set_semantics():
-    """Set insert: duplicates are no-ops in any order; reserved keys (bytes
-    0-15, 16-23 or 24-31 all zero) are refused and flagged."""
+    """Set insert (section 2.1: the cache index holds the keys of cached
+    blocks): duplicates are no-ops in any order; every key but the all-zero
+    one becomes a member -- keys with a zero half or zero 8-byte words
+    included -- and the all-zero key is refused and flagged.  Contents and
+    lookups are checked against a Python set."""
     rng = np.random.default_rng(18)
     keys = rng.integers(0, 256, (50, 32), dtype=np.uint8)
     keys[:, 0] |= 1
@@ -304,21 +309,26 @@ def pin_set_semantics():
     assert n_new == 50 and not flag
     n_new, flag = ks.insert(keys[:20])
     assert n_new == 0 and not flag
-    bad = np.full((4, 32), 7, np.uint8)
-    bad[0, :] = 0               # all zero
-    bad[1, :16] = 0             # first half zero
-    bad[2, 16:24] = 0           # third word zero
-    bad[3, 24:] = 0             # fourth word zero
-    n_new, flag = ks.insert(bad)
-    assert n_new == 0 and flag and ks.n == 50
-    ok = np.full((3, 32), 7, np.uint8)
-    ok[0, :8] = 0               # a zero first word alone is storable
-    ok[1, 8:16] = 0
-    ok[2, :8] = 255
-    n_new, flag = ks.insert(ok)
-    assert n_new == 3 and not flag and ks.n == 53
+    odd = np.full((8, 32), 7, np.uint8)
+    odd[0, :16] = 0             # first half zero
+    odd[1, 16:24] = 0           # third word zero
+    odd[2, 24:] = 0             # fourth word zero
+    odd[3, 16:] = 0             # second half zero
+    odd[4, :8] = 0              # first word zero
+    odd[5, :24] = 0             # only the last word non-zero
+    odd[6, 1:] = 0              # one non-zero byte, first
+    odd[7, :31] = 0             # one non-zero byte, last
+    n_new, flag = ks.insert(np.concatenate([odd, odd[::-1]]))
+    assert n_new == 8 and not flag and ks.n == 58
+    n_new, flag = ks.insert(np.zeros((2, 32), np.uint8))
+    assert n_new == 0 and flag and ks.n == 58
+    S = {k.tobytes() for k in np.concatenate([keys, odd])}
+    assert {k.tobytes() for k in ks.contents()} == S
+    probe = np.concatenate([odd, np.zeros((1, 32), np.uint8), keys[:3]])
+    assert list(ks.prefix_blocks(probe, np.array([0, 8, 12, 12], np.int64))) == [8, 0, 0]
+    assert list(ks.prefix_blocks(probe[9:], np.array([0, 3], np.int64))) == [3]
     ks2 = oracle.KeySet(1)
-    ks2.insert(np.concatenate([ok, batch])[rng.permutation(len(batch) + 3)])
+    ks2.insert(np.concatenate([odd, batch])[rng.permutation(len(batch) + 8)])
     assert (ks2.contents() == ks.contents()).all()
 
 
@@ -383,8 +393,8 @@ def pin_template_ordering():
 
 
 # ------------------------------------------------------ arrival-order serving
-def _reserved_py(k: bytes) -> bool:
-    return not any(k[:16]) or not any(k[16:24]) or not any(k[24:])
+def _zero_py(k: bytes) -> bool:
+    return not any(k)
 
 
 def _replay_python(S0, digests, off):
@@ -398,20 +408,23 @@ def _replay_python(S0, digests, off):
         while L < len(rows) and rows[L] in S:
             L += 1
         out.append(L)
-        S.update(k for k in rows if not _reserved_py(k))
+        S.update(k for k in rows if not _zero_py(k))
     return out, len(S) - before
 
 
 def pin_arrival_brute_force():
     """Arrival-order serving == a Python-set replay, request by request, on
     batches whose requests copy leading keys of earlier ones, with keys cached
-    before the batch and the odd reserved key."""
+    before the batch, keys with a zero half or word (ordinary members) and
+    the odd all-zero key (never cached)."""
     rng = np.random.default_rng(19)
     for trial in range(40):
         n_req = int(rng.integers(1, 40))
         pool = rng.integers(0, 256, (16, 32), dtype=np.uint8)
         pool[:, 0] |= 1
-        pool[15, :16] = 0                                  # reserved: never stored
+        pool[13, :16] = 0                                  # zero first half: an ordinary key
+        pool[14, 24:] = 0                                  # zero last word: an ordinary key
+        pool[15] = 0                                       # the all-zero key: never cached
         reqs = []
         for r in range(n_req):
             nb = int(rng.integers(0, 10))

@@ -305,7 +305,7 @@ def test_workload_structure():
         assert (pt[r, :c] == prt[src[r], :c]).all()
         assert pw.batch.principal[r] == pw.prior.principal[src[r]]
     keys = pw.random_keys
-    assert not any(oracle.key_reserved(k.tobytes()) for k in keys)
+    assert not any(oracle.key_is_zero(k.tobytes()) for k in keys)
     lw = W.make("long", n_req=4)
     assert lw.batch.tokens.shape[0] == 4 * 32768 and (lw.batch.boundary_tok == 64).all()
 
@@ -316,14 +316,13 @@ def test_full_size_shapes():
     assert W.make("sysprompt").batch.lengths()[0] == 2119
 
 
-def test_oracle_key_reserved_rule():
+def test_oracle_zero_key_rule():
+    """Only the all-zero key is refused by the oracle's set."""
     one = b"\x01" * 8
-    assert oracle.key_reserved(bytes(32))
-    assert oracle.key_reserved(bytes(16) + one + one)
-    assert oracle.key_reserved(one + one + bytes(8) + one)
-    assert oracle.key_reserved(one + one + one + bytes(8))
-    assert not oracle.key_reserved(bytes(8) + one + one + one)
-    assert not oracle.key_reserved(b"\xff" * 8 + one + one + one)
+    assert oracle.key_is_zero(bytes(32))
+    for k in (bytes(16) + one + one, one + one + bytes(8) + one, one + one + one + bytes(8), bytes(31) + b"\x01",
+              b"\x01" + bytes(31), bytes(8) + one + one + one):
+        assert not oracle.key_is_zero(k)
 
 
 def test_count_blocks_on_the_host(libkv):

@@ -63,9 +63,9 @@ MUTATIONS = [
      "        while (j < nb && chain_set_contains(&s, req + 32 * (size_t)j))\n            j++;\n"
      "        prefix_blocks[r] = (int32_t)j;\n"
      "        for (int64_t q = 0; q < nb; q++)\n"
-     "            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);",
+     "            if (!oracle_key_is_zero(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);",
      "        for (int64_t q = 0; q < nb; q++)\n"
-     "            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);\n"
+     "            if (!oracle_key_is_zero(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);\n"
      "        while (j < nb && chain_set_contains(&s, req + 32 * (size_t)j))\n            j++;\n"
      "        prefix_blocks[r] = (int32_t)j;"),
     ("arrival_initial_set_dropped",
@@ -87,9 +87,17 @@ MUTATIONS = [
     ("origami_ascending_order", "return (x < y) - (x > y);", "return (x > y) - (x < y);"),
     ("origami_budget_sign", "const double lm = ((double)m - K) / inv_sum;", "const double lm = ((double)m + K) / inv_sum;"),
     ("origami_no_clamp", "(1.0 - lam / x > 0.0 ? 1.0 - lam / x : 0.0)", "(1.0 - lam / x)"),
-    ("arrival_reserved_keys_stored",
-     "            if (!oracle_key_reserved(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);",
+    ("arrival_zero_key_stored",
+     "            if (!oracle_key_is_zero(req + 32 * (size_t)q)) chain_set_add(&s, req + 32 * (size_t)q);",
      "            chain_set_add(&s, req + 32 * (size_t)q);"),
+    ("set_zero_key_stored", "        if (oracle_key_is_zero(key)) { flags |= ORACLE_FLAG_ZERO_KEY; continue; }", ""),
+    ("set_refuses_zero_first_half",
+     "    for (int i = 0; i < 32; i++)\n        if (key[i] != 0) return 0;",
+     "    for (int i = 0; i < 16; i++)\n        if (key[i] != 0) return 0;"),
+    ("set_refuses_zero_last_word",
+     "    for (int i = 0; i < 32; i++)\n        if (key[i] != 0) return 0;\n    return 1;",
+     "    { int z = 1; for (int i = 24; i < 32; i++) if (key[i] != 0) z = 0; if (z) return 1; }\n"
+     "    for (int i = 0; i < 32; i++)\n        if (key[i] != 0) return 0;\n    return 1;"),
 ]
 
 
