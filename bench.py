@@ -44,16 +44,25 @@ WORKLOAD = {"workload": "wide: 131072 requests x 128 tokens, BOUNDARY salt at to
             "requests": 131072, "tokens_per_request": 128, "block": 16, "blocks_per_step": 131072 * 8,
             "principals": 4096, "mode": "BOUNDARY (k=4)"}
 SM_MAX_MHZ = 2070.0            # maximum SM clock of a GB300 (profiling recipe)
+DRIFT_LIMIT = 0.05             # the two halves of the timed steps must agree to within 5 %
 INT32_LANES_PER_SM = 64        # 4 SMSPs x 16 lanes of the integer pipe (LOP3/SHF/IMAD microbench: 64.0/clk/SM)
 CHAIN_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_chain.cu", "paper_2608_09225_gb300/csrc/sha256_dev.cuh",
                  "paper_2608_09225_gb300/csrc/kvgov_internal.cuh", "paper_2608_09225_gb300/csrc/kvgov_lookup.cuh",
-                 "paper_2608_09225_gb300/csrc/kvgov_insert.cuh"]
+                 "paper_2608_09225_gb300/csrc/kvgov_insert.cuh", "paper_2608_09225_gb300/csrc/kvgov_stash.cuh"]
 CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain kernel's code
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per launch of the
 # step's chain kernel from one ncu capture, and the SHA-256 (chain_source_hash)
 # of the sources it was captured from: reported as roofline.traffic only while
 # the kernel's sources still hash to that value.
 CHAIN_TRAFFIC = {"bytes_per_launch": None, "source_sha256": None}
+
+
+# DRAM bytes per launch of the probe on the probe-heavy workload from one ncu
+# capture, with the SHA-256 of the table kernels' sources it was taken from.
+TABLE_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_table.cu", "paper_2608_09225_gb300/csrc/kvgov_lookup.cuh",
+                 "paper_2608_09225_gb300/csrc/kvgov_stash.cuh", "paper_2608_09225_gb300/csrc/kvgov_internal.cuh",
+                 "paper_2608_09225_gb300/csrc/kvgov_insert.cuh"]
+TABLE_TRAFFIC = {"probe_seg_kernel<4, 1>": {"bytes_per_launch": None, "source_sha256": None}}
 
 
 def load_peaks() -> dict:
@@ -69,17 +78,33 @@ def load_peaks() -> dict:
 PEAKS = load_peaks()
 
 
-def chain_source_hash() -> str:
-    """SHA-256 over the chain kernel's translation unit: its sources, and the
-    constants (#define lines) of the public header it includes."""
+def sources_hash(sources) -> str:
+    """SHA-256 over a kernel's translation-unit sources and the constants
+    (#define lines) of the public header they include."""
     import hashlib
     h = hashlib.sha256()
-    for rel in CHAIN_SOURCES:
+    for rel in sources:
         with open(os.path.join(HERE, rel), "rb") as f:
             h.update(f.read())
     with open(os.path.join(HERE, CHAIN_HEADER), "rb") as f:
         h.update(b"".join(line for line in f.read().splitlines(keepends=True) if line.lstrip().startswith(b"#define")))
     return h.hexdigest()
+
+
+def table_traffic(kernel: str):
+    """DRAM bytes per launch of a table kernel from its last ncu capture, if
+    that capture was taken of the current sources; else None."""
+    rec = TABLE_TRAFFIC.get(kernel, {})
+    if rec.get("bytes_per_launch") is None:
+        return None, "no capture recorded"
+    if rec.get("source_sha256") != sources_hash(TABLE_SOURCES):
+        return None, "the last capture was of other sources"
+    return rec["bytes_per_launch"], "ncu capture of the current sources"
+
+
+def chain_source_hash() -> str:
+    """sources_hash of the chain kernel's translation unit."""
+    return sources_hash(CHAIN_SOURCES)
 
 
 def profiled_traffic():
@@ -201,7 +226,9 @@ def measure_int_peak(torch, peak_lib_path):
     out = {}
     for kind, name, threads, blocks_per_sm, iters in ((0, "lop3", 256, 8, 4000), (1, "shf", 256, 8, 4000),
                                                       (2, "iadd3", 256, 8, 4000), (3, "sha_alu", 256, 4, 200),
-                                                      (4, "sha_fma", 256, 4, 200), (5, "imad", 256, 8, 4000)):
+                                                      (4, "sha_fma", 256, 4, 200), (5, "imad", 256, 8, 4000),
+                                                      (8, "lop3+iadd3", 256, 8, 4000), (9, "lop3+imad", 256, 8, 4000),
+                                                      (10, "shf+iadd3", 256, 8, 4000)):
         blocks = n_sm * blocks_per_sm
         sink = torch.zeros(1, dtype=torch.int32, device="cuda")
         clocks = torch.zeros(blocks * 3, dtype=torch.int64, device="cuda")
@@ -243,6 +270,12 @@ def measure_lone_warp_round(torch, peak_lib_path) -> float:
     return float(np.median(c[:, 2] - c[:, 1])) / (iters * 64)
 
 
+def main_slots(table) -> int:
+    """The main slots of a table tensor (a power of two; the side store's
+    slots follow them)."""
+    return 1 << (table.shape[0].bit_length() - 1)
+
+
 def measure_gather(torch, peak_lib_path, table: "torch.Tensor", n_reads: int = 1 << 25) -> dict:
     """Random-slot read rate (GB/s of bytes read, best of 5) over `table`,
     reading whole 32-byte slots and first halves, from libkvgov_peak."""
@@ -257,7 +290,7 @@ def measure_gather(torch, peak_lib_path, table: "torch.Tensor", n_reads: int = 1
         for rep in range(6):
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record()
-            rc = L.kvgov_peak_gather(table.data_ptr(), table.shape[0], slot_bytes, n_reads, 12345 + rep,
+            rc = L.kvgov_peak_gather(table.data_ptr(), main_slots(table), slot_bytes, n_reads, 12345 + rep,
                                      sink.data_ptr(), torch.cuda.current_stream().cuda_stream)
             b.record()
             assert rc == 0, rc
@@ -284,7 +317,7 @@ def measure_slot_ops(torch, peak_lib_path, table: "torch.Tensor", n_ops: int) ->
             table.zero_()
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record()
-            rc = L.kvgov_peak_slot_ops(table.data_ptr(), table.shape[0], kind, n_ops, 777 + rep, sink.data_ptr(),
+            rc = L.kvgov_peak_slot_ops(table.data_ptr(), main_slots(table), kind, n_ops, 777 + rep, sink.data_ptr(),
                                        torch.cuda.current_stream().cuda_stream)
             b.record()
             assert rc == 0, rc
@@ -519,9 +552,10 @@ def main():
     table_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                 if i % table_every == 0 else None for i in range(args.steps)]
     t_start, t_stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_mid = torch.cuda.Event(enable_timing=True)   # between the two halves of the timed steps (drift gate)
     # create every timing event now (a CUDA event is created on its first record, which costs the host far
     # more than a step's launches): inside the timed loop they are only recorded
-    for pair in chain_ev + [e for e in table_ev if e is not None] + [(t_start, t_stop)]:
+    for pair in chain_ev + [e for e in table_ev if e is not None] + [(t_start, t_stop), (t_mid,)]:
         for e in pair:
             e.record(pipe.compute_stream)
     torch.cuda.synchronize()
@@ -534,7 +568,10 @@ def main():
         t_start.record(pipe.compute_stream)
         pipe.prep_stream.wait_event(t_start)
         h0 = time.perf_counter()
+        half = args.steps // 2
         for i in range(args.steps):
+            if i == half:
+                t_mid.record(pipe.compute_stream)
             last_prefix = step(pool[(1 + args.warmup + i) % args.pool], chain_ev[i], table_ev[i])
         if in_chain:
             pipe.drain()                           # the last batch's insert
@@ -554,6 +591,16 @@ def main():
         raise SystemExit(f"gate failed: {gate}")
     kernel_launches = launches[0]
     ms = t_start.elapsed_time(t_stop)
+    # gate: two independent halves of the timed steps must agree (the paper's section 5.7 gates ask two
+    # independent blocks of a measurement to agree)
+    if half > 0:
+        ms_a, ms_b = t_start.elapsed_time(t_mid) / half, t_mid.elapsed_time(t_stop) / (args.steps - half)
+        drift = abs(ms_a - ms_b) / ((ms_a + ms_b) / 2)
+        gate["drift"] = {"ms_per_step_first_half": ms_a, "ms_per_step_second_half": ms_b, "drift": drift,
+                         "limit": DRIFT_LIMIT}
+        if drift > DRIFT_LIMIT:
+            raise SystemExit(f"gate failed: the two halves of the timed steps differ by {100 * drift:.2f} % "
+                             f"(limit {100 * DRIFT_LIMIT:.0f} %): {gate['drift']}")
     chain_ms = float(np.mean([a.elapsed_time(b) for a, b in chain_ev]))
     table_ms = float(np.mean([a.elapsed_time(b) for a, b in table_timed]))
     inserted_per_step = (gate["n_new_total"] - n_new_before) / args.steps
@@ -600,13 +647,21 @@ def main():
         lookups = 5 * n_req
         tab_bytes = lookups * 32 + walk * n_req * 32 + 20 * n_req
         tab_gbs = tab_bytes / (table_ms / 1e3) / 1e9
+        # 4 of a request's 5 lookups are the shared prefix's 4 keys, the same slots for every request, which
+        # L2 serves; only block 4's lookup walks slots that come from DRAM
+        dram_fed = n_req * 32 * (1 + (1 + 1 / (1 - lf) ** 2) / 2)
         table_roofline = {
             "kernel": "probe_seg_kernel<4, 1> (kvgov_probe)", "bound": "hbm", "achieved": tab_gbs,
             "peak": PEAKS.get("hbm_gbs"), "unit": "GB/s",
             "frac": tab_gbs / PEAKS["hbm_gbs"] if PEAKS.get("hbm_gbs") else None,
             "peak_source": "of fallback (6.8 TB/s)" if PEAKS.get("fallback") else
                            "of measured (MEASURED_PEAKS.json hbm_gbs, a copy)",
-            "random_read_ceiling_gbs": gather["gbs_32B"], "frac_of_random_read_ceiling": tab_gbs / gather["gbs_32B"],
+            "l2_resident_share": 1 - dram_fed / tab_bytes,
+            "note": "L2-fed for the most part: the 4 shared-prefix lookups of every request hit the same 4 slots; "
+                    "the DRAM-bound table case is table_roofline_cfg4",
+            "dram_fed_bytes_per_launch": dram_fed,
+            "random_read_ceiling_gbs": gather["gbs_32B"],
+            "frac_of_random_read_ceiling_dram_fed": dram_fed / (table_ms / 1e3) / 1e9 / gather["gbs_32B"],
             "kernel_ms": table_ms, "timed_launches": f"every {table_every}th step of the timed region",
             "lookups_per_launch": lookups, "lookups_per_s": lookups / (table_ms / 1e3),
             "mean_load_factor": lf, "algorithmic_bytes_per_launch": tab_bytes,
@@ -639,6 +694,19 @@ def main():
     if clock.get("sm_mhz"):
         roofline["frac_at_run_clock"] = achieved / (n_sm * INT32_LANES_PER_SM * clock["sm_mhz"] * 1e6 / 1e12)
 
+    # ---- the probe-heavy workload: the table kernels on a 512 MiB table (larger than L2)
+    table_cfg4 = probe_heavy_leg(torch, K, W, kbuild)
+
+    # gate: no kernel may run above its own ceiling (the paper's section 5.7 gate rejects a result that
+    # implies more than 100 % of the GPU's peak)
+    fracs = {"roofline.frac": roofline["frac"], "table_roofline.frac": table_roofline["frac"],
+             "table_roofline_cfg4.probe.frac": table_cfg4["probe"]["frac"],
+             "table_roofline_cfg4.insert.frac": table_cfg4["insert"]["frac"]}
+    gate["frac_ok"] = all(f is not None and f <= 1.0 for f in fracs.values())
+    gate["fracs"] = fracs
+    if not gate["frac_ok"]:
+        raise SystemExit(f"gate failed: a kernel measured above its ceiling: {fracs}")
+
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "u32", "data": "synthetic",
@@ -660,7 +728,7 @@ def main():
                          "beside the chain hash of batch i; chain hash with the fused probe, then the insert, on a "
                          "higher-priority compute stream"),
             "e2e": e2e, "gpu_launches": kernel_launches, "clocks": clock, "roofline": roofline,
-            "table_roofline": table_roofline,
+            "table_roofline": table_roofline, "table_roofline_cfg4": table_cfg4,
             "arrival": arrival, "gate": gate}
     if rank == 0 and not args.no_cpu_baseline and world == 1:
         line["cpu_baseline"] = cpu_baseline(pool_host[0], args.cpu_sample, gate_digests)
@@ -671,6 +739,94 @@ def main():
     if world > 1:
         dist.destroy_process_group()
     return 0
+
+
+def probe_heavy_leg(torch, K, W, kbuild, reps: int = 10) -> dict:
+    """The table kernels where the table is larger than L2: the probe-heavy
+    workload (65,536 requests x 512 tokens, ROOT, 1024 principals; 30 % reuse
+    the first 0-31 blocks of one of 8192 prior requests) probed against a
+    2^24-slot (512 MiB) table at load factor 0.5 (the prior requests' chains
+    and 8,126,464 random keys), and that table's fill from empty.  Each probe
+    is timed alone with CUDA events after a 256 MiB write that flushes L2;
+    each fill is a table initialisation then the insert, timed around the
+    insert.  Both against the random-read ceiling measured on the same table."""
+    from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache
+    w = W.make("probe")
+    b, p = w.batch, w.prior
+    cache = PrefixCache(w.capacity, w.secret, w.ids, w.id_off)
+    db = DeviceBatch.from_host(b.tokens, b.tok_off, b.principal, b.boundary_tok)
+    dp = DeviceBatch.from_host(p.tokens, p.tok_off, p.principal, p.boundary_tok)
+    blk, pblk = K.block_offsets(db.tok_off), K.block_offsets(dp.tok_off)
+    dig = K.chain_hash(W.ROOT, db.tokens, db.tok_off, blk, db.principal, cache.salts, n_blocks=db.n_blocks)
+    pdig = K.chain_hash(W.ROOT, dp.tokens, dp.tok_off, pblk, dp.principal, cache.salts, n_blocks=dp.n_blocks)
+    keys = torch.cat([pdig, torch.from_numpy(w.random_keys).cuda()])
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    pre = torch.empty(b.n, dtype=torch.int32, device="cuda")
+    n_new = torch.zeros(1, dtype=torch.int64, device="cuda")
+    ins_ms, probe_ms = [], []
+    for i in range(3 + reps):
+        K.table_init(cache.slots)
+        n_new.zero_()
+        a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        K.insert(cache.slots, keys, cache.status, n_new)
+        e.record()
+        for _ in range(2):                         # two probes per fill, each after an L2 flush
+            flush.zero_()
+            pa, pe = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            pa.record()
+            K.probe(cache.slots, dig, blk, pre, cache.status)
+            pe.record()
+            torch.cuda.synchronize()
+            if i >= 3:
+                probe_ms.append(pa.elapsed_time(pe))
+        if i >= 3:
+            ins_ms.append(a.elapsed_time(e))
+    cache.check_status()
+    n_keys, stored = keys.shape[0], int(n_new.item())
+    L = pre.cpu().numpy().astype(np.int64)
+    nb = np.diff(K.count_blocks(b.tok_off)[1])
+    if stored != n_keys:
+        raise SystemExit(f"probe-heavy leg: {stored} of {n_keys} keys stored")
+    reuse, cut = w.info["reuse"], w.info["cut"]
+    if not (L == np.where(reuse, cut, 0)).all():          # closed form: a reused request hits its cut, else 0
+        raise SystemExit("probe-heavy leg: prefix lengths differ from the closed form")
+    gather = measure_gather(torch, kbuild.PEAK_LIB, cache.slots)
+    ceiling = gather["gbs_32B"]
+    cap = K.capacity_of(cache.slots)
+    alpha = n_keys / cap
+    hit_walk, miss_walk = (1 + 1 / (1 - alpha)) / 2, (1 + 1 / (1 - alpha) ** 2) / 2
+    hits = int(np.minimum(L, nb).sum())
+    misses = int((L < nb).sum())
+    probe_bytes = hits * 32 * (1 + hit_walk) + misses * 32 * (1 + miss_walk) + 20 * b.n
+    t_probe = float(np.mean(probe_ms))
+    probe_gbs = probe_bytes / (t_probe / 1e3) / 1e9
+    fill_walk = np.mean([(1 + 1 / (1 - a) ** 2) / 2 for a in np.linspace(0, alpha, 64, endpoint=False)])
+    ins_bytes = n_keys * (32 + 32 * fill_walk + 32)
+    t_ins = float(np.mean(ins_ms))
+    ins_gbs = ins_bytes / (t_ins / 1e3) / 1e9
+    traffic, traffic_src = table_traffic("probe_seg_kernel<4, 1>")
+    return {"workload": "probe-heavy: 65536 requests x 512 tokens, ROOT, 1024 principals, table 2^24 slots "
+                        "(512 MiB) at load factor 0.5", "table_bytes": cap * 32, "load_factor": alpha,
+            "random_read_ceiling_gbs": ceiling, "random_read_microbench": gather,
+            "probe": {"kernel": "probe_seg_kernel<4, 1> (kvgov_probe)", "bound": "hbm (random 32-byte reads)",
+                      "kernel_ms": t_probe, "timed_launches": len(probe_ms), "l2": "flushed before each launch",
+                      "algorithmic_probes": hits + misses, "probes_per_s": (hits + misses) / (t_probe / 1e3),
+                      "algorithmic_bytes_per_launch": probe_bytes, "achieved": probe_gbs, "unit": "GB/s",
+                      "peak": ceiling, "frac": probe_gbs / ceiling,
+                      "peak_source": "random 32-byte-read microbenchmark on this table (libkvgov_peak)",
+                      "frac_of_hbm_copy_peak": probe_gbs / PEAKS["hbm_gbs"],
+                      "traffic": traffic, "traffic_source": traffic_src,
+                      "bytes_basis": "per lookup up to the first miss: its 32 B digest and 32 B per slot walked "
+                                     "(linear probing at the load factor: (1 + 1/(1-a))/2 for a hit, "
+                                     "(1 + 1/(1-a)^2)/2 for a miss); per request 16 B offsets + 4 B prefix"},
+            "insert": {"kernel": "insert_kernel (kvgov_insert)", "bound": "hbm (random 32-byte slots)",
+                       "kernel_ms": t_ins, "timed_launches": len(ins_ms), "keys": n_keys,
+                       "inserts_per_s": n_keys / (t_ins / 1e3), "algorithmic_bytes_per_launch": ins_bytes,
+                       "achieved": ins_gbs, "unit": "GB/s", "peak": ceiling, "frac": ins_gbs / ceiling,
+                       "peak_source": "random 32-byte-read microbenchmark on this table (libkvgov_peak)",
+                       "bytes_basis": "per key its 32 B, 32 B per slot walked while the table fills from empty "
+                                      "to the load factor, and the 32 B slot written"}}
 
 
 def arrival_leg(torch, K, W, pool, n_req, n_blocks, cache, steps, chain_ms):
@@ -792,9 +948,17 @@ def cpu_baseline(w, sample, gpu_digests):
         blocks += cpu_oracle_step(w, sample, cores, epoch_secret(w.secret, 1 + reps))[0]
         reps += 1
     dt = time.perf_counter() - t0
+    one_reps, one_blocks, t1 = 0, 0, time.perf_counter()   # the same step on one thread
+    one_sample = max(1, sample // 8)
+    while one_reps < 1 or time.perf_counter() - t1 < 4.0:
+        one_blocks += cpu_oracle_step(w, one_sample, 1, epoch_secret(w.secret, 100 + one_reps))[0]
+        one_reps += 1
+    dt1 = time.perf_counter() - t1
     return {"value": blocks / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": f"{reps} steps over the first {sample} requests of one batch (salts for 4096 principals, "
                       f"chain on {cores} threads, probe, insert of the uncached blocks); {dt:.1f} s",
+            "value_1_thread": one_blocks / dt1,
+            "sample_1_thread": f"{one_reps} steps over the first {one_sample} requests, one thread; {dt1:.1f} s",
             "gate_sample_digests_equal_gpu": same}
 
 

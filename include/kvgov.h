@@ -11,8 +11,8 @@
  *  - Return value: KVGOV_OK, or a host-detected error (KVGOV_EINVAL for a bad
  *    argument, KVGOV_ECUDA when a launch fails).  On a host-detected error
  *    nothing is enqueued.
- *  - Errors that only the device can see (a bad per-request index, a
- *    reserved key, a full table, a wait that ran out) are OR-ed as
+ *  - Errors that only the device can see (a bad per-request index, the
+ *    all-zero key, a full table, a wait that ran out) are OR-ed as
  *    KVGOV_F_* bits into the u32 at d_status.  The caller zeroes it before
  *    the call and reads it after synchronising.  Where d_status may be NULL
  *    the flags are dropped.
@@ -46,6 +46,9 @@ typedef struct CUstream_st *kvgov_stream_t;
 #define KVGOV_MIN_CAPACITY 32      /* smallest table capacity (slots)         */
 #define KVGOV_PROBE_WINDOW 1024    /* a key lives within this many slots of its
                                       home slot (fewer if the table is smaller) */
+#define KVGOV_STASH_SLOTS 64       /* slots after the `capacity` main ones: the
+                                      table's side store (see the table section) */
+#define KVGOV_STASH_KEYS 56        /* keys the side store holds               */
 #define KVGOV_TEMPLATE_NONE (-1)   /* kvgov_divergence_boundary: no preamble   */
 #define KVGOV_TEMPLATE_ANY (-2)    /* ... the longest match over all preambles */
 
@@ -58,12 +61,12 @@ typedef struct CUstream_st *kvgov_stream_t;
 #define KVGOV_F_BADINDEX 0x10u     /* a principal index, boundary offset or
                                       offset array entry was out of range; the
                                       affected request produced no output     */
-#define KVGOV_F_SENTINEL 0x20u     /* a reserved key (bytes 0-15, 16-23 or
-                                      24-31 all zero) was given to an insert; it
-                                      is skipped (these values mark empty slots
-                                      and keys still being written)           */
+#define KVGOV_F_SENTINEL 0x20u     /* the all-zero key (the value of an empty
+                                      slot) was given to an insert; it is
+                                      skipped                                  */
 #define KVGOV_F_TABLE_FULL 0x40u   /* an insert found no free slot in a key's
-                                      probe window; the key is not stored     */
+                                      probe window, or the side store was
+                                      full; the key is not stored             */
 #define KVGOV_F_TIMEOUT 0x80u      /* an insert gave up waiting for another
                                       thread to finish writing a slot's key   */
 
@@ -262,22 +265,33 @@ int kvgov_chain_hash_probe(int mode, const int32_t *d_tokens, const int64_t *d_t
 
 /*
  * The prefix-cache index (paper section 2.1 and Table 1, row 1: a block
- * prefix cache keyed by chained block hashes).  The caller owns a table of
- * `capacity` 32-byte slots (capacity a power of two >= KVGOV_MIN_CAPACITY,
- * d_slots 16-byte aligned).  A slot is empty when its first 16 bytes are
+ * prefix cache keyed by chained block hashes): the set of 32-byte keys of
+ * cached blocks.  Every key but the all-zero one (KVGOV_F_SENTINEL) can be
+ * stored.  The caller owns the table's memory: capacity + KVGOV_STASH_SLOTS
+ * slots of 32 bytes (capacity a power of two >= KVGOV_MIN_CAPACITY, d_slots
+ * 16-byte aligned), and passes `capacity`.
+ *
+ * Main slots 0 .. capacity-1: a slot is empty when its first 16 bytes are
  * zero; a key's home slot is its first 8 bytes read as a little-endian u64,
  * modulo capacity, with linear probing inside a window of
  * min(capacity, KVGOV_PROBE_WINDOW) slots: an insert that finds no free slot
  * in its window reports KVGOV_F_TABLE_FULL (at load factor 0.5 a walk longer
  * than a few dozen slots practically never happens), and lookups stop at the
- * end of the window.  Keys are stored verbatim and claimed
- * with a 128-bit compare-and-swap of their first 16 bytes, so keys whose
- * bytes 0-15, 16-23 or 24-31 are all zero cannot be stored
- * (KVGOV_F_SENTINEL); for SHA-256 digests that happens with probability
- * about 2^-63.
+ * end of the window.  Keys are stored verbatim, claimed with a 128-bit
+ * compare-and-swap of their first 16 bytes, the second half written after.
+ *
+ * Side store, slots capacity .. capacity+63: the keys a main slot cannot
+ * hold -- those whose bytes 0-15 are all zero (they would read as empty) or
+ * whose bytes 16-23 or 24-31 are all zero (they would read as still being
+ * written) -- up to KVGOV_STASH_KEYS of them (KVGOV_F_TABLE_FULL past that).
+ * For SHA-256 digests that is a key with probability about 2^-63.  Its
+ * layout: bytes 0-3 of slot `capacity` count the entries handed out, the
+ * u32 at byte 32 + 4e of that slot onwards is entry e's state (1 = live),
+ * and entry e's key is slot capacity + 8 + e.
  */
 
-/* kvgov_table_init -- mark every slot empty.  EINVAL: bad capacity/pointer. */
+/* kvgov_table_init -- mark every slot empty, main slots and side store
+ * (capacity + KVGOV_STASH_SLOTS slots).  EINVAL: bad capacity/pointer. */
 int kvgov_table_init(uint8_t *d_slots, uint64_t capacity, kvgov_stream_t stream);
 
 /*
@@ -386,8 +400,10 @@ int kvgov_chain_hash_insert_prev(int mode, const int32_t *d_tokens, const int64_
  *
  * Arrival positions: block j of request r has position
  * seq_base + blk_off[r] + j, so a batch covers blk_off[n_req] positions from
- * seq_base.  The owner array d_owner [capacity] u64, beside the table, holds
- * per slot the smallest position whose block inserted the slot's key through
+ * seq_base.  The owner array d_owner [capacity + KVGOV_STASH_SLOTS] u64,
+ * beside the table, holds per slot (a main slot, or a side-store entry at its
+ * handle capacity + 8 + e) the smallest position whose block inserted the
+ * slot's key through
  * kvgov_insert_arrival (0 for keys inserted any other way, which count as
  * cached before every arrival).  Zero it once with kvgov_owner_init when the
  * table is created; it stays valid across kvgov_table_init as long as
@@ -397,7 +413,8 @@ int kvgov_chain_hash_insert_prev(int mode, const int32_t *d_tokens, const int64_
  */
 
 /*
- * kvgov_owner_init -- zero d_owner [capacity] u64 (16-byte aligned).
+ * kvgov_owner_init -- zero d_owner [capacity + KVGOV_STASH_SLOTS] u64
+ * (16-byte aligned).
  * EINVAL: NULL or misaligned pointer, bad capacity.
  */
 int kvgov_owner_init(uint64_t *d_owner, uint64_t capacity, kvgov_stream_t stream);
@@ -406,11 +423,13 @@ int kvgov_owner_init(uint64_t *d_owner, uint64_t capacity, kvgov_stream_t stream
  * kvgov_insert_arrival -- insert every block of the batch (the set semantics
  * and protocol of kvgov_insert) and settle the owners of the keys it adds.
  *   d_slots, capacity, d_digests, d_blk_off, n_req  as for kvgov_probe.
- *   d_owner    [capacity] u64, see above.
+ *   d_owner    [capacity + KVGOV_STASH_SLOTS] u64, see above.
  *   seq_base   arrival position of the batch's first block.
- *   d_slot_of  [d_blk_off[n_req]] u32 output: the slot holding each block's
- *              key, or 0xFFFFFFFF if it could not be stored (reserved key,
- *              full window, timeout -- flagged in *d_status).  This is the
+ *   d_slot_of  [d_blk_off[n_req]] u32 output: the handle of each block's
+ *              key (its main slot, or capacity + 8 + its side-store entry),
+ *              or 0xFFFFFFFF if it could not be stored (the all-zero key, a
+ *              full window or side store, a timeout -- flagged in
+ *              *d_status).  This is the
  *              block's handle in the cache and the input of
  *              kvgov_probe_arrival.
  *   d_n_new, d_status  as for kvgov_insert (d_status required); also

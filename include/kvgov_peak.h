@@ -26,7 +26,9 @@ typedef struct CUstream_st *kvgov_stream_t;
  *   0 LOP3, 1 SHF (funnel shift), 2 IADD3, 3 SHA-256 compression (FIPS 180-4)
  *   with ALU adds, 4 the same with every add as IMAD (FMA pipe), 5 IMAD,
  *   6 SHA-256 rounds alone with K_t + W_t in registers (T1/T2 grouping),
- *   7 the same rounds with the shorter e-to-e grouping.
+ *   7 the same rounds with the shorter e-to-e grouping, and two-kind mixes
+ *   (half the streams each, interleaved) that show whether two kinds share
+ *   a pipe: 8 LOP3 + IADD3, 9 LOP3 + IMAD, 10 SHF + IADD3.
  * d_clocks [blocks][3] u64 receives, per CTA, its SM id and its clock64()
  * at start and end.  d_sink [1] u32 is written only in a case that never
  * happens (keeps results live).  Asynchronous on `stream`.

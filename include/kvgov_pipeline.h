@@ -61,7 +61,7 @@ typedef struct kvgov_pipeline_desc {
     int32_t max_req;              /* capacity of each slot: requests ...                 */
     int64_t max_blocks;           /* ... and blocks                                      */
     /* the cache */
-    uint8_t *d_slots;             /* [capacity][32] table                                */
+    uint8_t *d_slots;             /* [capacity + KVGOV_STASH_SLOTS][32] table             */
     uint64_t capacity;
     uint32_t *d_status;           /* flags (required)                                    */
     unsigned long long *d_n_new;  /* keys inserted (nullable)                            */

@@ -19,6 +19,11 @@
 //   6  SHA-256 rounds only (64 a iteration, K_t + W_t from registers, as the
 //      small-batch chain kernel's round warp runs them): sha_rounds16_t1t2
 //   7  the same with sha_rounds16_short
+//   8  LOP3 on streams 0-3 and IADD3 on streams 4-7, interleaved
+//   9  LOP3 on streams 0-3 and IMAD on streams 4-7
+//  10  SHF on streams 0-3 and IADD3 on streams 4-7
+// Kinds 8-10 show whether two kinds of instruction share one pipe: if they
+// do, the mix runs at the slower kind's rate; if not, it can run above it.
 // Kinds 6 and 7 count 14 nominal ops a round; launched with one warp per SM
 // sub-partition they give a lone warp's round rate.
 // Each update reads two other streams' latest values, so no chain of updates
@@ -91,11 +96,14 @@ __global__ void peak_kernel(int iters, uint32_t seed, uint32_t one, uint32_t *si
 #pragma unroll
                 for (int s = 0; s < kStreams; ++s) {
                     const uint32_t a = x[(s + 1) % kStreams], b = x[(s + 2) % kStreams];
-                    if (KIND == 0)
+                    // the kind of instruction for this stream
+                    const int op = KIND <= 2 || KIND == 5 ? KIND
+                                 : (s < kStreams / 2 ? (KIND == 10 ? 1 : 0) : (KIND == 9 ? 5 : 2));
+                    if (op == 0)
                         asm("lop3.b32 %0, %0, %1, %2, 0x96;" : "+r"(x[s]) : "r"(a), "r"(b));
-                    else if (KIND == 1)
+                    else if (op == 1)
                         x[s] = __funnelshift_r(x[s], a, (s * 5 + rep * 3 + 1) & 31);
-                    else if (KIND == 2)
+                    else if (op == 2)
                         x[s] = x[s] + a + b;
                     else
                         asm("mad.lo.u32 %0, %0, %1, %2;" : "+r"(x[s]) : "r"(one), "r"(a));
@@ -125,13 +133,14 @@ extern "C" int kvgov_peak_ops_per_iter(int kind) {
     case 3: case 4: return kShaChains * 1384;
     case 5: return 4 * kStreams;
     case 6: case 7: return 64 * 14;
+    case 8: case 9: case 10: return 4 * kStreams;
     default: return 0;
     }
 }
 
 extern "C" int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint32_t *d_sink,
                               unsigned long long *d_clocks, kvgov_stream_t stream) {
-    if (kind < 0 || kind > 7 || iters <= 0 || blocks <= 0 || threads <= 0 || threads > 1024 || !d_sink ||
+    if (kind < 0 || kind > 10 || iters <= 0 || blocks <= 0 || threads <= 0 || threads > 1024 || !d_sink ||
         !d_clocks)
         return 1;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
@@ -143,7 +152,10 @@ extern "C" int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint
     case 4: peak_kernel<4><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
     case 5: peak_kernel<5><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
     case 6: peak_kernel<6><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
-    default: peak_kernel<7><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 7: peak_kernel<7><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 8: peak_kernel<8><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 9: peak_kernel<9><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    default: peak_kernel<10><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
     }
     return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }

@@ -37,6 +37,10 @@
 //                          position of r's first block.  The prefix ends at the
 //                          first block that was not (or whose key could not be
 //                          stored).
+//
+// A key held in the table's side store (kvgov_stash.cuh) has the handle
+// capacity + 8 + its entry, so the owner array has capacity +
+// KVGOV_STASH_SLOTS entries.
 #include <atomic>
 
 #include "kvgov_insert.cuh"
@@ -111,7 +115,7 @@ __global__ void __launch_bounds__(kThreads) insert_arrival_kernel(
         if (row >= n_rows) continue;
         const uint4 a = __ldg(digests + 2 * row), b = __ldg(digests + 2 * row + 1);
         const unsigned long long k[4] = {u64_of(a.x, a.y), u64_of(a.z, a.w), u64_of(b.x, b.y), u64_of(b.z, b.w)};
-        if (key_reserved(k)) {
+        if (key_is_zero(k)) {
             if (handles) {
                 my_flags |= KVGOV_F_SENTINEL;
                 slot_of[row] = kNoSlot;
@@ -333,7 +337,7 @@ static void insert_first_requests(uint8_t *d_slots, uint64_t capacity, uint64_t 
 
 extern "C" int kvgov_owner_init(uint64_t *d_owner, uint64_t capacity, kvgov_stream_t stream) {
     if (!d_owner || !kvgov_host::aligned16(d_owner) || !arrival_capacity(capacity)) return KVGOV_EINVAL;
-    const unsigned long long n_vec = capacity / 2;          // capacity >= 32: a whole number of uint4
+    const unsigned long long n_vec = (capacity + KVGOV_STASH_SLOTS) / 2;   // main slots and side store: whole uint4s
     const unsigned long long want = (n_vec + 255) / 256;
     const unsigned long long cap = (unsigned long long)kvgov_host::sm_count() * 16;
     const unsigned grid = (unsigned)(want < cap ? want : cap);

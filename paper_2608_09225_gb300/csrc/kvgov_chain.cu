@@ -234,7 +234,7 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
         if (pleft > 2) wn = __ldg(reinterpret_cast<const uint2 *>(q.digests + 2 * (prow + 2)));
         const uint4 x = __ldg(q.digests + 2 * prow), y = __ldg(q.digests + 2 * prow + 1);
         const unsigned long long key[4] = {u64_of(x.x, x.y), u64_of(x.z, x.w), u64_of(y.x, y.y), u64_of(y.z, y.w)};
-        if (key_reserved(key)) {
+        if (key_is_zero(key)) {
             my_flags |= KVGOV_F_SENTINEL;
         } else {
             unsigned long long pos = 0;
@@ -299,7 +299,7 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             if (FUSE == kFuseArrival) {
                 ak[0] = u64_of(q0.x, q0.y); ak[1] = u64_of(q0.z, q0.w);
                 ak[2] = u64_of(q1.x, q1.y); ak[3] = u64_of(q1.z, q1.w);
-                have = !key_reserved(ak);
+                have = !key_is_zero(ak);
                 if (!have) {
                     my_flags |= KVGOV_F_SENTINEL;
                     a.slot_of[row + j] = kNoSlot;

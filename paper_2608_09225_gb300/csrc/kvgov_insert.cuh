@@ -6,6 +6,7 @@
 #include <cstdint>
 
 #include "kvgov_lookup.cuh"
+#include "kvgov_stash.cuh"
 
 namespace kvgov_dev {
 
@@ -23,14 +24,6 @@ __device__ __forceinline__ ulonglong2 ld_plain2(const unsigned long long *p) {
     ulonglong2 v;
     asm volatile("ld.global.v2.u64 {%0, %1}, [%2];\n" : "=l"(v.x), "=l"(v.y) : "l"(p) : "memory");
     return v;
-}
-__device__ __forceinline__ ulonglong2 ld_relaxed2(const unsigned long long *p) {
-    ulonglong2 v;
-    asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];\n" : "=l"(v.x), "=l"(v.y) : "l"(p) : "memory");
-    return v;
-}
-__device__ __forceinline__ void st_relaxed(unsigned long long *p, unsigned long long v) {
-    asm volatile("st.relaxed.gpu.global.u64 [%0], %1;\n" ::"l"(p), "l"(v) : "memory");
 }
 // Both words of a 16-byte-aligned pair in one store.  Each word is written
 // once, from zero, so a reader that sees one word and not the other still
@@ -62,11 +55,18 @@ enum InsertResult { kNew = 0, kDuplicate = 1, kFull = 2, kTimeout = 3 };
 constexpr uint32_t kNoSlot = 0xffffffffu;
 constexpr uint32_t kSettled = 0x80000000u;
 
-// Insert the key k (w0..w3) with the protocol described in kvgov_table.cu.
-// On kNew and kDuplicate, *pos receives the slot that holds the key.
+// Insert the non-zero key k (w0..w3) with the protocol described in
+// kvgov_table.cu; keys the main slots cannot hold go to the side store
+// (kvgov_stash.cuh).  On kNew and kDuplicate, *pos receives the key's handle:
+// the slot that holds it, or capacity + 8 + its side-store entry.
 __device__ __forceinline__ InsertResult insert_one(unsigned long long *slots, unsigned long long mask,
                                                    const unsigned long long k[4], uint32_t spin_limit,
                                                    unsigned long long *pos_out = nullptr) {
+    if (key_in_stash(k[0], k[1], k[2], k[3])) {
+        const StashResult r = stash_insert(slots, mask, k[0], k[1], k[2], k[3], spin_limit);
+        if (pos_out && (r.res == kNew || r.res == kDuplicate)) *pos_out = r.pos;
+        return static_cast<InsertResult>(r.res);
+    }
     const unsigned long long window = probe_window(mask);
     unsigned long long pos = k[0] & mask;
     for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
@@ -107,10 +107,6 @@ __device__ __forceinline__ InsertResult insert_one(unsigned long long *slots, un
         }
     }
     return kFull;
-}
-
-__device__ __forceinline__ bool key_reserved(const unsigned long long k[4]) {
-    return (k[0] | k[1]) == 0ull || k[2] == 0ull || k[3] == 0ull;
 }
 
 // Insert counts: warp reduction, shared-memory accumulation, and the CTA's

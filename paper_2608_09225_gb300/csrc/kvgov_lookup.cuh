@@ -6,6 +6,7 @@
 #include <cstdint>
 
 #include "../../include/kvgov.h"
+#include "kvgov_stash.cuh"
 
 namespace kvgov_dev {
 
@@ -24,8 +25,8 @@ __device__ __forceinline__ unsigned long long probe_window(unsigned long long ma
 // behind other warps' hashing).
 __device__ __forceinline__ bool lookup(const uint4 *__restrict__ slots, unsigned long long mask, uint4 q0, uint4 q1) {
     const unsigned long long k0 = u64_of(q0.x, q0.y), k1 = u64_of(q0.z, q0.w);
-    if ((k0 | k1) == 0ull || u64_of(q1.x, q1.y) == 0ull || u64_of(q1.z, q1.w) == 0ull)
-        return false;                               // reserved keys are never stored
+    if (key_in_stash(k0, k1, u64_of(q1.x, q1.y), u64_of(q1.z, q1.w)))
+        return stash_lookup(slots, mask, q0, q1);    // not in the main slots
     const unsigned long long window = probe_window(mask);
     unsigned long long pos = k0 & mask;
     for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
@@ -50,9 +51,8 @@ __device__ __forceinline__ unsigned long long home_slot(uint4 q0, unsigned long 
 // lookup().
 __device__ __forceinline__ bool lookup_from_home(const uint4 *__restrict__ slots, unsigned long long mask, uint4 q0,
                                                  uint4 q1, uint4 a, uint4 b) {
-    if ((u64_of(q0.x, q0.y) | u64_of(q0.z, q0.w)) == 0ull || u64_of(q1.x, q1.y) == 0ull ||
-        u64_of(q1.z, q1.w) == 0ull)
-        return false;                               // reserved keys are never stored
+    if (key_in_stash(u64_of(q0.x, q0.y), u64_of(q0.z, q0.w), u64_of(q1.x, q1.y), u64_of(q1.z, q1.w)))
+        return stash_lookup(slots, mask, q0, q1);    // not in the main slots
     const unsigned long long window = probe_window(mask);
     unsigned long long pos = home_slot(q0, mask);
     for (unsigned long long n = 1;; ++n) {
@@ -74,9 +74,8 @@ __device__ __forceinline__ bool lookup_from_home(const uint4 *__restrict__ slots
 // -- then costs one round trip.  Same result as lookup().
 __device__ __forceinline__ bool lookup_from_pair(const uint4 *__restrict__ slots, unsigned long long mask, uint4 q0,
                                                  uint4 q1, uint4 a, uint4 b, uint4 c, uint4 d) {
-    if ((u64_of(q0.x, q0.y) | u64_of(q0.z, q0.w)) == 0ull || u64_of(q1.x, q1.y) == 0ull ||
-        u64_of(q1.z, q1.w) == 0ull)
-        return false;                               // reserved keys are never stored
+    if (key_in_stash(u64_of(q0.x, q0.y), u64_of(q0.z, q0.w), u64_of(q1.x, q1.y), u64_of(q1.z, q1.w)))
+        return stash_lookup(slots, mask, q0, q1);    // not in the main slots
     const unsigned long long window = probe_window(mask);   // even: capacity is a power of two >= 32
     unsigned long long pos = home_slot(q0, mask);
     for (unsigned long long n = 2;; n += 2) {

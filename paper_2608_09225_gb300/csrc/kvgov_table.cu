@@ -14,8 +14,10 @@
 // of min(capacity, KVGOV_PROBE_WINDOW) slots: an insert that finds no free
 // slot in its key's window fails (table full), so a lookup can stop at the
 // end of the window too.  Every walk is bounded, even in a full table.  Keys with
-// (w0, w1) == 0, w2 == 0 or w3 == 0 are refused (reserved): the first marks
-// empty slots, the other two mark a key still being written.
+// (w0, w1) == 0, w2 == 0 or w3 == 0 cannot live in a main slot (the first
+// pattern marks empty slots, the other two a key still being written): they
+// go to the table's side store after the main slots (kvgov_stash.cuh), so
+// every key but the all-zero one is stored.
 //
 // Insert protocol (one key per thread, no fences): walk the slots.  A plain
 // read whose two first-half words are both non-zero is final (the half is
@@ -85,7 +87,7 @@ __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long lo
         if (mine) {
             const uint4 a = __ldg(keys + 2 * i), b = __ldg(keys + 2 * i + 1);
             k[0] = u64_of(a.x, a.y); k[1] = u64_of(a.z, a.w); k[2] = u64_of(b.x, b.y); k[3] = u64_of(b.z, b.w);
-            if (key_reserved(k)) {
+            if (key_is_zero(k)) {
                 my_flags |= KVGOV_F_SENTINEL;
                 mine = false;
             }
@@ -253,7 +255,7 @@ __global__ void __launch_bounds__(kInsertThreads) insert_uncached_packed_kernel(
                 const uint4 a = __ldg(digests + 2 * row), b = __ldg(digests + 2 * row + 1);
                 key[0] = u64_of(a.x, a.y); key[1] = u64_of(a.z, a.w);
                 key[2] = u64_of(b.x, b.y); key[3] = u64_of(b.z, b.w);
-                if (key_reserved(key)) {
+                if (key_is_zero(key)) {
                     my_flags |= KVGOV_F_SENTINEL;
                     mine = false;
                 }
@@ -277,7 +279,7 @@ unsigned probe_grid(int32_t n_req, int G) {
 
 extern "C" int kvgov_table_init(uint8_t *d_slots, uint64_t capacity, kvgov_stream_t stream) {
     if (!d_slots || !kvgov_host::aligned16(d_slots) || !kvgov_host::pow2_capacity(capacity)) return KVGOV_EINVAL;
-    const unsigned long long n_vec = capacity * 2ull;
+    const unsigned long long n_vec = (capacity + KVGOV_STASH_SLOTS) * 2ull;   // main slots and side store
     unsigned long long grid = (n_vec + 255) / 256;
     if (grid > 152ull * 64) grid = 152ull * 64;
     table_init_kernel<<<(unsigned)grid, 256, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
@@ -355,8 +357,8 @@ extern "C" const char *kvgov_status_string(int status) {
     case KVGOV_EINVAL: return "KVGOV_EINVAL: invalid argument";
     case KVGOV_ECUDA: return "KVGOV_ECUDA: kernel launch failed";
     case (int)KVGOV_F_BADINDEX: return "KVGOV_F_BADINDEX: index or offset out of range";
-    case (int)KVGOV_F_SENTINEL: return "KVGOV_F_SENTINEL: reserved key (bytes 0-15, 16-23 or 24-31 all zero)";
-    case (int)KVGOV_F_TABLE_FULL: return "KVGOV_F_TABLE_FULL: no free slot";
+    case (int)KVGOV_F_SENTINEL: return "KVGOV_F_SENTINEL: the all-zero key (an empty slot's value) was not stored";
+    case (int)KVGOV_F_TABLE_FULL: return "KVGOV_F_TABLE_FULL: no free slot in a key's window or the side store";
     case (int)KVGOV_F_TIMEOUT: return "KVGOV_F_TIMEOUT: gave up waiting for a slot's key to be written";
     default: return "KVGOV: unknown status";
     }

@@ -19,6 +19,8 @@ BLOCK = 16
 DIGEST_BYTES = 32
 MAX_SECRET = 1024
 MIN_CAPACITY = 32
+STASH_SLOTS = 64          # slots after the capacity main ones: the table's side store
+STASH_KEYS = 56
 
 OK, EINVAL, ECUDA = 0, 1, 2
 F_BADINDEX, F_SENTINEL, F_TABLE_FULL, F_TIMEOUT = 0x10, 0x20, 0x40, 0x80
@@ -143,6 +145,15 @@ def _stream(stream=None):
     return s.cuda_stream
 
 
+def capacity_of(slots: torch.Tensor) -> int:
+    """The capacity of a table tensor: its rows minus the side store's."""
+    return slots.shape[0] - STASH_SLOTS
+
+
+def _owner_capacity(owner: torch.Tensor) -> int:
+    return owner.numel() - STASH_SLOTS
+
+
 def block_offsets(tok_off: torch.Tensor, blk_off: torch.Tensor | None = None,
                   status: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """blk_off[r+1] - blk_off[r] = floor(len_r / 16) (paper section 2.1)."""
@@ -244,7 +255,7 @@ def chain_hash_probe(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, blk
                                     _dev(boundary_tok, torch.int32, "boundary_tok", True),
                                     _dev(blk_off, torch.int64, "blk_off"),
                                     _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(tokens),
-                                    _dev(slots, torch.uint8, "slots"), slots.shape[0],
+                                    _dev(slots, torch.uint8, "slots"), capacity_of(slots),
                                     _dev(prefix_blocks, torch.int32, "prefix_blocks") if n else _dummy(tokens),
                                     _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_chain_hash_probe")
@@ -277,7 +288,7 @@ def chain_hash_insert_prev(mode: int, tokens: torch.Tensor, tok_off: torch.Tenso
         _dev(principal, torch.int32, "principal", True), _dev(salts, torch.uint8, "salts", True), n_p,
         _dev(boundary_tok, torch.int32, "boundary_tok", True), _dev(blk_off, torch.int64, "blk_off"),
         _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(tokens),
-        _dev(slots, torch.uint8, "slots"), slots.shape[0],
+        _dev(slots, torch.uint8, "slots"), capacity_of(slots),
         _dev(prev_digests, torch.uint8, "prev_digests") if prev_digests.numel() else _dummy(tokens),
         _dev(prev_blk_off, torch.int64, "prev_blk_off"), pn,
         _dev(prev_prefix_blocks, torch.int32, "prev_prefix_blocks") if pn else _dummy(tokens),
@@ -299,21 +310,22 @@ _dummy_buf = None
 
 
 def table_init(slots: torch.Tensor, stream=None) -> torch.Tensor:
-    """Mark every slot of a [capacity, 32] u8 table empty."""
-    _check(lib().kvgov_table_init(_dev(slots, torch.uint8, "slots"), slots.shape[0], _stream(stream)),
+    """Mark every slot of a [capacity + STASH_SLOTS, 32] u8 table empty."""
+    _check(lib().kvgov_table_init(_dev(slots, torch.uint8, "slots"), capacity_of(slots), _stream(stream)),
            "kvgov_table_init")
     return slots
 
 
 def new_table(capacity: int, device="cuda", stream=None) -> torch.Tensor:
-    slots = torch.empty((capacity, 32), dtype=torch.uint8, device=device)
+    """An empty table of `capacity` main slots and the side store."""
+    slots = torch.empty((capacity + STASH_SLOTS, 32), dtype=torch.uint8, device=device)
     return table_init(slots, stream)
 
 
 def insert(slots: torch.Tensor, keys: torch.Tensor, status: torch.Tensor, n_new: torch.Tensor | None = None,
            stream=None):
     """Set-insert [n, 32] u8 keys; adds the number stored to n_new (int64[1])."""
-    _check(lib().kvgov_insert(_dev(slots, torch.uint8, "slots"), slots.shape[0],
+    _check(lib().kvgov_insert(_dev(slots, torch.uint8, "slots"), capacity_of(slots),
                               _dev(keys, torch.uint8, "keys"), keys.shape[0] if keys.dim() == 2 else 0,
                               _dev(n_new, torch.int64, "n_new", True), _dev(status, torch.int32, "status"),
                               _stream(stream)),
@@ -327,7 +339,7 @@ def probe(slots: torch.Tensor, digests: torch.Tensor, blk_off: torch.Tensor,
     n = blk_off.numel() - 1
     if prefix_blocks is None:
         prefix_blocks = torch.empty(n, dtype=torch.int32, device=blk_off.device)
-    _check(lib().kvgov_probe(_dev(slots, torch.uint8, "slots"), slots.shape[0],
+    _check(lib().kvgov_probe(_dev(slots, torch.uint8, "slots"), capacity_of(slots),
                              _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(blk_off),
                              _dev(blk_off, torch.int64, "blk_off"), n,
                              _dev(prefix_blocks, torch.int32, "prefix_blocks"),
@@ -340,7 +352,7 @@ def insert_uncached(slots: torch.Tensor, digests: torch.Tensor, blk_off: torch.T
                     status: torch.Tensor, n_new: torch.Tensor | None = None, stream=None):
     """Insert each request's blocks from prefix_blocks[r] on (after probe)."""
     n = blk_off.numel() - 1
-    _check(lib().kvgov_insert_uncached(_dev(slots, torch.uint8, "slots"), slots.shape[0],
+    _check(lib().kvgov_insert_uncached(_dev(slots, torch.uint8, "slots"), capacity_of(slots),
                                        _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(blk_off),
                                        _dev(blk_off, torch.int64, "blk_off"), n,
                                        _dev(prefix_blocks, torch.int32, "prefix_blocks"),
@@ -351,14 +363,15 @@ def insert_uncached(slots: torch.Tensor, digests: torch.Tensor, blk_off: torch.T
 
 # ---- arrival-order serving (paper sections 2.1 and 4.2, request by request)
 def owner_init(owner: torch.Tensor, stream=None) -> torch.Tensor:
-    """Zero a table's owner array ([capacity] int64 holding u64 arrival positions)."""
-    _check(lib().kvgov_owner_init(_dev(owner, torch.int64, "owner"), owner.numel(), _stream(stream)),
+    """Zero a table's owner array ([capacity + STASH_SLOTS] int64 holding u64
+    arrival positions)."""
+    _check(lib().kvgov_owner_init(_dev(owner, torch.int64, "owner"), _owner_capacity(owner), _stream(stream)),
            "kvgov_owner_init")
     return owner
 
 
 def new_owner(capacity: int, device="cuda", stream=None) -> torch.Tensor:
-    return owner_init(torch.empty(capacity, dtype=torch.int64, device=device), stream)
+    return owner_init(torch.empty(capacity + STASH_SLOTS, dtype=torch.int64, device=device), stream)
 
 
 def insert_arrival(slots: torch.Tensor, owner: torch.Tensor, digests: torch.Tensor, blk_off: torch.Tensor,
@@ -372,7 +385,7 @@ def insert_arrival(slots: torch.Tensor, owner: torch.Tensor, digests: torch.Tens
     if slot_of is None:
         slot_of = torch.empty(n_blocks, dtype=torch.int32, device=blk_off.device)
     _check(lib().kvgov_insert_arrival(_dev(slots, torch.uint8, "slots"), _dev(owner, torch.int64, "owner"),
-                                      slots.shape[0],
+                                      capacity_of(slots),
                                       _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(blk_off),
                                       _dev(blk_off, torch.int64, "blk_off"), n, int(seq_base),
                                       _dev(slot_of, torch.int32, "slot_of") if slot_of.numel() else _dummy(blk_off),
@@ -389,7 +402,7 @@ def probe_arrival(owner: torch.Tensor, slot_of: torch.Tensor, blk_off: torch.Ten
     n = blk_off.numel() - 1
     if prefix_blocks is None:
         prefix_blocks = torch.empty(n, dtype=torch.int32, device=blk_off.device)
-    _check(lib().kvgov_probe_arrival(_dev(owner, torch.int64, "owner"), owner.numel(),
+    _check(lib().kvgov_probe_arrival(_dev(owner, torch.int64, "owner"), _owner_capacity(owner),
                                      _dev(slot_of, torch.int32, "slot_of") if slot_of.numel() else _dummy(blk_off),
                                      _dev(blk_off, torch.int64, "blk_off"), n, int(seq_base),
                                      _dev(prefix_blocks, torch.int32, "prefix_blocks"),
@@ -428,7 +441,7 @@ def chain_hash_arrival(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, b
                                       _dev(blk_off, torch.int64, "blk_off"),
                                       _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(tokens),
                                       _dev(slots, torch.uint8, "slots"), _dev(owner, torch.int64, "owner"),
-                                      slots.shape[0], int(seq_base),
+                                      capacity_of(slots), int(seq_base),
                                       _dev(slot_of, torch.int32, "slot_of") if slot_of.numel() else _dummy(tokens),
                                       _dev(prefix_blocks, torch.int32, "prefix_blocks") if n else _dummy(tokens),
                                       _dev(n_new, torch.int64, "n_new", True), _dev(status, torch.int32, "status"),
@@ -518,7 +531,7 @@ def serve_arrival_static(slots: torch.Tensor, owner: torch.Tensor, digests: torc
     if prefix_blocks is None:
         prefix_blocks = torch.empty(max(n, 0), dtype=torch.int32, device=blk_off.device)
     _check(lib().kvgov_serve_arrival_static(_dev(slots, torch.uint8, "slots"), _dev(owner, torch.int64, "owner"),
-                                            slots.shape[0],
+                                            capacity_of(slots),
                                             _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(blk_off),
                                             _dev(blk_off, torch.int64, "blk_off"), n, n_blocks, int(seq_base),
                                             _dev(prefix_blocks, torch.int32, "prefix_blocks") if n else _dummy(blk_off),

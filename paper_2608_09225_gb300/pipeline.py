@@ -52,7 +52,8 @@ class DeviceBatch:
 class PrefixCache:
     """A GPU-resident block prefix-cache index with per-principal salts.
 
-    capacity   table slots (power of two, >= 32), 32 bytes each.
+    capacity   main table slots (power of two, >= 32), 32 bytes each; the
+               table also holds the side store's K.STASH_SLOTS slots.
     secret     the server secret K (HMAC key of section 4.1).
     ids/id_off principal-id bytes in CSR form (host numpy or device tensors).
     """
@@ -66,7 +67,7 @@ class PrefixCache:
         self.id_off = torch.as_tensor(np.asarray(id_off, dtype=np.int64)).to(self.device)
         self.n_principals = self.id_off.numel() - 1
         self.salts = torch.empty((self.n_principals, 32), dtype=torch.uint8, device=self.device)
-        self.slots = torch.empty((self.capacity, 32), dtype=torch.uint8, device=self.device)
+        self.slots = torch.empty((self.capacity + K.STASH_SLOTS, 32), dtype=torch.uint8, device=self.device)
         self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
         self.n_new = torch.zeros(1, dtype=torch.int64, device=self.device)
         K.table_init(self.slots, self.stream)

@@ -9,6 +9,7 @@ import torch
 import oracle
 from paper_2608_09225_gb300 import workloads as W
 from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache, next_pow2
+from tests.table_layout import table_keys
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
@@ -23,9 +24,6 @@ def status_tensor():
     return torch.zeros(1, dtype=torch.int32, device=DEV)
 
 
-def table_contents(slots):
-    s = slots.cpu().numpy()
-    return {r.tobytes() for r in s[s[:, :16].any(axis=1)]}
 
 
 class Arrival:
@@ -48,12 +46,18 @@ class Arrival:
         return pre.cpu().numpy(), slot_of.cpu().numpy()
 
 
-def sequences(seed, n_req, pool_n=64, max_blocks=12):
+def sequences(seed, n_req, pool_n=64, max_blocks=12, side=0, zero=False):
     """Requests as key sequences that often start with a copy of an earlier
-    request's leading keys (the structure of shared prefixes)."""
+    request's leading keys (the structure of shared prefixes).  `side` pool
+    keys take the patterns a main slot cannot hold (zero first half, zero
+    third or fourth 8-byte word); `zero` makes the last pool key all-zero."""
     rng = np.random.default_rng(seed)
     pool = rng.integers(0, 256, (pool_n, 32), dtype=np.uint8)
     pool[:, 0] |= 1
+    for i in range(side):
+        pool[i, (slice(0, 16), slice(16, 24), slice(24, 32))[i % 3]] = 0
+    if zero:
+        pool[-1] = 0
     reqs = []
     for _ in range(n_req):
         keys = list(rng.integers(0, pool_n, int(rng.integers(0, max_blocks))))
@@ -77,7 +81,7 @@ def test_arrival_matches_replay(kv, n_req, cap_log2):
     assert int(a.n_new.item()) == n_new
     s = a.slots.cpu().numpy()
     assert (s[slot_of] == d).all()                     # each block's handle holds its key
-    assert table_contents(a.slots) == {r.tobytes() for r in d}
+    assert table_keys(a.slots) == {r.tobytes() for r in d}
 
 
 def test_arrival_batches_in_sequence_and_plain_inserts(kv):
@@ -106,19 +110,32 @@ def test_arrival_batches_in_sequence_and_plain_inserts(kv):
     assert pre2[-1] == 50 and pre2[0] == 3
 
 
-def test_arrival_reserved_full_and_empty(kv):
-    """Reserved keys are flagged, get no slot and end the prefix; a full
-    table flags and ends the prefix at the block it could not store; empty
-    batches and empty requests are no-ops."""
-    pool, d, off = sequences(11, 50, pool_n=20)
-    d = d.copy()
-    d[5, :16] = 0
-    a = Arrival(kv, 1 << 10)
-    pre, slot_of = a.serve(d, off)
-    assert int(a.status.item()) == kv.F_SENTINEL
-    assert slot_of[5] == NO_SLOT
-    want, n_new = oracle.KeySet(1).arrival_prefix(d, off)
-    assert (pre == want).all() and int(a.n_new.item()) == n_new
+def test_arrival_side_store_keys_and_the_zero_key(kv):
+    """Keys a main slot cannot hold (zero first half or a zero 8-byte word in
+    the second half), shared by many requests' prefixes, are served like any
+    other key: their handles point into the side store and hold them, and
+    prefix lengths and key counts match the oracle's replay.  The all-zero
+    key is flagged, gets no handle and ends its request's prefix."""
+    for seed, n_req in ((11, 50), (12, 3000)):
+        pool, d, off = sequences(seed, n_req, pool_n=20, side=6, zero=True)
+        a = Arrival(kv, 1 << 12)
+        pre, slot_of = a.serve(d, off)
+        want, n_new = oracle.KeySet(1).arrival_prefix(d, off)
+        zero_rows = ~d.any(axis=1)
+        assert zero_rows.any() and int(a.status.item()) == kv.F_SENTINEL
+        assert (slot_of[zero_rows] == NO_SLOT).all()
+        assert (pre == want).all() and int(a.n_new.item()) == n_new
+        s = a.slots.cpu().numpy()
+        ok = ~zero_rows
+        assert (s[slot_of[ok]] == d[ok]).all()                   # each handle holds its block's key
+        side_rows = ok & (~d[:, :16].any(axis=1) | ~d[:, 16:24].any(axis=1) | ~d[:, 24:].any(axis=1))
+        assert side_rows.any() and (slot_of[side_rows] >= (1 << 12)).all()
+        assert table_keys(a.slots) == {r.tobytes() for r in d[ok]}
+
+
+def test_arrival_full_and_empty(kv):
+    """A full table flags and ends the prefix at the block it could not
+    store; empty batches and empty requests are no-ops."""
     # a 32-slot table and 64 distinct keys
     k = np.random.default_rng(12).integers(1, 256, (64, 32), dtype=np.uint8)
     b = Arrival(kv, 32)
@@ -277,7 +294,7 @@ def test_chain_hash_arrival_matches_oracle_and_separate_calls(kv, mode, n_req):
         assert (a.slots.cpu().numpy()[so] == ref).all()
         assert (pre.cpu().numpy() == want).all()
         assert int(a.n_new.item()) == ks.n + n_batch
-        outs.append(table_contents(a.slots))
+        outs.append(table_keys(a.slots))
     assert outs[0] == outs[1]
     assert want.max() > 0 and (want == 0).any()
 

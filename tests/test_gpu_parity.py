@@ -10,6 +10,7 @@ import torch
 
 import oracle
 from paper_2608_09225_gb300 import workloads as W
+from tests.table_layout import table_keys
 
 pytestmark = pytest.mark.gpu
 GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
@@ -219,10 +220,6 @@ def keys_np(n, seed):
     return k
 
 
-def table_contents(slots):
-    s = slots.cpu().numpy()
-    full = s[s[:, :16].any(axis=1)]          # first 16 bytes zero = empty slot
-    return {r.tobytes() for r in full}
 
 
 def test_insert_set_semantics(kv):
@@ -234,7 +231,7 @@ def test_insert_set_semantics(kv):
     kv.insert(slots, dev(k[:777]), st, n_new)
     torch.cuda.synchronize()
     assert int(st.item()) == 0 and int(n_new.item()) == 5000
-    assert table_contents(slots) == {r.tobytes() for r in k}
+    assert table_keys(slots) == {r.tobytes() for r in k}
 
 
 def test_insert_heavy_in_batch_duplicates(kv):
@@ -248,29 +245,103 @@ def test_insert_heavy_in_batch_duplicates(kv):
     kv.insert(slots, dev(batch), st, n_new)
     torch.cuda.synchronize()
     assert int(st.item()) == 0 and int(n_new.item()) == 65
-    assert table_contents(slots) == {r.tobytes() for r in k}
+    assert table_keys(slots) == {r.tobytes() for r in k}
 
 
-def test_insert_reserved_keys(kv):
-    k = keys_np(12, 4)
-    k[3, :] = 0                 # all zero
-    k[5, :16] = 0               # first half zero
-    k[7, 16:24] = 0             # third word zero
-    k[9, 24:] = 0               # fourth word zero
-    k[10, :8] = 0               # first word zero alone: storable
-    k[11, :8] = 255             # first word all ones: storable
+def side_store_keys(n, seed):
+    """n distinct keys that a main slot cannot hold, cycling through the
+    patterns: first half zero, third or fourth 8-byte word zero, second half
+    zero, all but the last two bytes zero."""
+    k = keys_np(n, seed)
+    for i in range(n):
+        kind = i % 5
+        if kind == 0:
+            k[i, :16] = 0
+        elif kind == 1:
+            k[i, 16:24] = 0
+        elif kind == 2:
+            k[i, 24:] = 0
+        elif kind == 3:
+            k[i, 16:] = 0
+        else:
+            k[i, :30] = 0
+            k[i, 30] = seed & 0xff
+            k[i, 31] = 1 + i // 5
+    return k
+
+
+def test_insert_side_store_keys(kv):
+    """Keys with a zero first half or a zero 8-byte word in the second half
+    -- which a main slot cannot hold -- are stored (in the side store) and
+    found, like any other key; only the all-zero key is refused.  Checked
+    against the oracle's set: contents, key count, each key's lookup, and a
+    request of them all hitting to its end."""
+    k = np.concatenate([keys_np(12, 4), side_store_keys(10, 40)])
+    k[3, :] = 0                 # all zero: refused
+    k[10, :8] = 0               # first word zero alone: a main slot holds it
+    k[11, :8] = 255
     slots = kv.new_table(64)
     st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
     kv.insert(slots, dev(k), st, n_new)
+    kv.insert(slots, dev(k[::-1].copy()), st, n_new)          # every key again: duplicates
     torch.cuda.synchronize()
     assert int(st.item()) == kv.F_SENTINEL
     ks = oracle.KeySet(1)
     n_ref, flagged = ks.insert(k)
-    assert flagged and int(n_new.item()) == n_ref == 8
-    assert table_contents(slots) == {r.tobytes() for r in ks.contents()}
-    pre = kv.probe(slots, dev(k), dev(np.arange(13, dtype=np.int64)))
+    assert flagged and int(n_new.item()) == n_ref == 21
+    assert table_keys(slots) == {r.tobytes() for r in ks.contents()}
+    pre = kv.probe(slots, dev(k), dev(np.arange(23, dtype=np.int64)))
+    whole = kv.probe(slots, dev(np.delete(k, 3, axis=0)), dev(np.array([0, 21], np.int64)))
+    absent = kv.probe(slots, dev(side_store_keys(10, 41)), dev(np.arange(11, dtype=np.int64)))
     torch.cuda.synchronize()
-    assert list(pre.cpu().numpy()) == [0 if oracle.key_reserved(r.tobytes()) else 1 for r in k]
+    member = {r.tobytes() for r in ks.contents()}
+    assert list(pre.cpu().numpy()) == [int(r.tobytes() in member) for r in k]
+    assert int(whole.item()) == 21
+    assert (absent.cpu().numpy() == 0).all()
+
+
+def test_side_store_concurrent_duplicates(kv):
+    """Ten side-store keys, each inserted 4000 times from every part of one
+    shuffled batch (with 3000 ordinary keys around them) and then once more:
+    each is stored once, the count matches the oracle, every key is found."""
+    side = side_store_keys(10, 42)
+    plain = keys_np(3000, 43)
+    batch = np.concatenate([np.repeat(side, 4000, axis=0), plain])
+    batch = batch[np.random.default_rng(44).permutation(len(batch))]
+    slots = kv.new_table(1 << 14)
+    st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
+    kv.insert(slots, dev(batch), st, n_new)
+    kv.insert(slots, dev(side), st, n_new)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0 and int(n_new.item()) == 3010
+    assert table_keys(slots) == {r.tobytes() for r in np.concatenate([side, plain])}
+    pre = kv.probe(slots, dev(np.concatenate([side, plain[:6]])), dev(np.array([0, 16], np.int64)))
+    torch.cuda.synchronize()
+    assert int(pre.item()) == 16
+
+
+def test_side_store_full(kv):
+    """More distinct side-store keys than it holds: KVGOV_STASH_KEYS are
+    stored, the rest flagged KVGOV_F_TABLE_FULL; every stored key is found
+    and a key inserted again is a duplicate, not a new entry."""
+    k = side_store_keys(70, 45)
+    slots = kv.new_table(32)
+    st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
+    kv.insert(slots, dev(k), st, n_new)
+    torch.cuda.synchronize()
+    assert int(st.item()) == kv.F_TABLE_FULL
+    stored = table_keys(slots)
+    assert int(n_new.item()) == len(stored) == kv.STASH_KEYS and stored <= {r.tobytes() for r in k}
+    st2 = status_tensor()
+    kept = np.array([np.frombuffer(x, np.uint8) for x in sorted(stored)])
+    kv.insert(slots, dev(kept), st2, n_new)
+    pre = kv.probe(slots, dev(k), dev(np.arange(71, dtype=np.int64)))
+    torch.cuda.synchronize()
+    assert int(st2.item()) == 0 and int(n_new.item()) == kv.STASH_KEYS
+    assert list(pre.cpu().numpy()) == [int(r.tobytes() in stored) for r in k]
+    kv.table_init(slots)
+    torch.cuda.synchronize()
+    assert table_keys(slots) == set()
 
 
 def test_table_full(kv):
@@ -280,7 +351,7 @@ def test_table_full(kv):
     kv.insert(slots, dev(k), st, n_new)
     torch.cuda.synchronize()
     assert int(st.item()) & kv.F_TABLE_FULL
-    assert int(n_new.item()) == 32 and len(table_contents(slots)) == 32
+    assert int(n_new.item()) == 32 and len(table_keys(slots)) == 32
 
 
 def test_full_table_inserts_and_lookups_stay_bounded(kv):
@@ -293,7 +364,7 @@ def test_full_table_inserts_and_lookups_stay_bounded(kv):
     kv.insert(slots, dev(k), st, n_new)
     torch.cuda.synchronize()
     assert int(st.item()) & kv.F_TABLE_FULL
-    stored = table_contents(slots)
+    stored = table_keys(slots)
     # with the probe window a nearly full table may refuse a key before the
     # last slot is taken; every refusal is flagged and every store counted
     assert int(n_new.item()) == len(stored) and len(stored) > 0.9 * cap
@@ -446,7 +517,7 @@ def test_insert_uncached_after_probe_matches_insert_all(kv, cap_log2):
     assert (pre.cpu().numpy() == ks.prefix_blocks(digests, off)).all()
     n_ref, _ = ks.insert(digests)
     assert int(n_new.item()) == n_ref
-    assert table_contents(slots) == {r.tobytes() for r in ks.contents()}
+    assert table_keys(slots) == {r.tobytes() for r in ks.contents()}
 
 
 def test_insert_uncached_bad_offsets_flagged(kv):
@@ -504,8 +575,9 @@ def test_chain_hash_insert_prev_matches_separate_calls(kv, mode, n_req, prev_n):
     leaves the table, key count and flags of kvgov_insert_uncached on the
     previous batch: on a batch small enough to take two launches, on fused
     batches (the previous one with more requests than the grid has threads,
-    or none), and with an empty batch.  The previous batch holds a reserved
-    key, a request whose prefix covers it whole, and out-of-range prefixes."""
+    or none), and with an empty batch.  The previous batch holds the all-zero
+    key, keys that live in the side store, a request whose prefix covers it
+    whole, and out-of-range prefixes."""
     rng = np.random.default_rng(n_req + prev_n + mode)
     lengths = list(rng.integers(0, 200, n_req)) if n_req else []
     b = W.ragged(19 + mode, lengths) if n_req else None
@@ -518,8 +590,10 @@ def test_chain_hash_insert_prev_matches_separate_calls(kv, mode, n_req, prev_n):
     pdig = keys_np(int(poff[-1]), 5 + mode) if prev_n else np.zeros((0, 32), np.uint8)
     ppre = rng.integers(-2, 14, prev_n).astype(np.int32)      # < 0 reads as 0, > n_b as n_b
     if prev_n:
-        pdig[0] = 0                                           # a reserved (all-zero) key, uncached
+        pdig[0] = 0                                           # the all-zero key, uncached
         ppre[0] = 0
+        for i in range(1, min(len(pdig), 13), 4):             # keys that live in the side store
+            pdig[i, (slice(0, 16), slice(16, 24), slice(24, 32))[(i // 4) % 3]] = 0
     present = pdig[rng.random(len(pdig)) < 0.3] if prev_n else pdig
     cap = 1 << 20
     def fresh_table():
@@ -554,7 +628,7 @@ def test_chain_hash_insert_prev_matches_separate_calls(kv, mode, n_req, prev_n):
         assert int(st_a.item()) & kv.F_SENTINEL
     assert (d_a.cpu().numpy() == d_b.cpu().numpy()).all()
     assert int(n_a.item()) == int(n_b.item())
-    assert table_contents(slots_a) == table_contents(slots_b)
+    assert table_keys(slots_a) == table_keys(slots_b)
     if n_req:
         ref = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
         assert (d_a.cpu().numpy() == ref).all()
@@ -567,7 +641,7 @@ def test_chain_hash_insert_prev_matches_separate_calls(kv, mode, n_req, prev_n):
     new_keys = pdig[rows]
     ks.insert(new_keys[new_keys.any(axis=1)])
     assert int(n_a.item()) == ks.n - before
-    assert table_contents(slots_a) == {r.tobytes() for r in ks.contents()}
+    assert table_keys(slots_a) == {r.tobytes() for r in ks.contents()}
 
 
 @pytest.mark.parametrize("mode", [0, 1, 2])
@@ -617,7 +691,7 @@ def test_chain_hash_insert_prev_with_probe(kv, mode, n_req):
     assert int(st_a.item()) == 0 and int(st_b.item()) == 0
     assert (d_a.cpu().numpy() == ref).all() and (d_b.cpu().numpy() == ref).all()
     assert int(n_a.item()) == int(n_b.item())
-    assert table_contents(slots_a) == table_contents(slots_b)
+    assert table_keys(slots_a) == table_keys(slots_b)
     ks = oracle.KeySet(1)
     ks.insert(present)
     rows = np.concatenate([np.arange(poff[i] + ppre[i], poff[i + 1]) for i in range(len(prev_req))] +

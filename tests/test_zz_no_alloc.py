@@ -10,13 +10,11 @@ import torch
 
 from paper_2608_09225_gb300 import workloads as W
 from paper_2608_09225_gb300.pipeline import DeviceBatch, PrefixCache, next_pow2
+from tests.table_layout import table_keys
 
 pytestmark = pytest.mark.gpu
 
 
-def table_contents(slots):
-    s = slots.cpu().numpy()
-    return {r.tobytes() for r in s[s[:, :16].any(axis=1)]}
 
 
 def test_static_scratch_matches_caller_scratch(kv):
@@ -42,7 +40,7 @@ def test_static_scratch_matches_caller_scratch(kv):
         assert (got.cpu().numpy() == want.cpu().numpy()).all()
         assert int(st_new.item()) == int(ref_new.item())
         seq += d.shape[0]
-    assert table_contents(st_slots) == table_contents(ref_slots)
+    assert table_keys(st_slots) == table_keys(ref_slots)
     assert (st_owner.cpu().numpy()[st_slots.cpu().numpy()[:, :16].any(axis=1)] > 0).all()
     last = got.cpu().numpy()
     assert last[0] >= 4 and (last >= 4).all()                        # batch 2 reuses batch 1's shared prefix
@@ -78,3 +76,35 @@ def test_static_scratch_bounds_rows_by_n_blocks(kv, total):
     assert (pre.cpu().numpy() == 0).all()
     assert int(n_new.item()) == 0
     assert torch.equal(slots, slots_before) and torch.equal(owner, owner_before)
+
+
+def test_static_scratch_with_side_store_keys(kv):
+    """Keys that live in the table's side store (zero first half, zero third
+    or fourth 8-byte word), shared across requests, and one all-zero key:
+    the same prefix lengths, key count, flags and table as the caller-scratch
+    calls, on two consecutive calls."""
+    rng = np.random.default_rng(77)
+    pool = rng.integers(1, 256, (24, 32), dtype=np.uint8)
+    for i in range(6):
+        pool[i, (slice(0, 16), slice(16, 24), slice(24, 32))[i % 3]] = 0
+    pool[23] = 0
+    cap = 1 << 10
+    ref_slots, ref_owner = kv.new_table(cap), kv.new_owner(cap)
+    st_slots, st_owner = kv.new_table(cap), kv.new_owner(cap)
+    ref_st, st_st = (torch.zeros(1, dtype=torch.int32, device="cuda") for _ in range(2))
+    ref_new, st_new = (torch.zeros(1, dtype=torch.int64, device="cuda") for _ in range(2))
+    seq = 1
+    for call in range(2):
+        lens = rng.integers(0, 9, 400)
+        off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+        d = torch.from_numpy(pool[rng.integers(0, 24, int(off[-1]))]).cuda()
+        blk = torch.from_numpy(off).cuda()
+        slot_of = kv.insert_arrival(ref_slots, ref_owner, d, blk, seq, ref_st, n_new=ref_new)
+        want = kv.probe_arrival(ref_owner, slot_of, blk, seq, status=ref_st)
+        got = kv.serve_arrival_static(st_slots, st_owner, d, blk, seq, st_st, n_new=st_new)
+        torch.cuda.synchronize()
+        assert int(ref_st.item()) == int(st_st.item()) == kv.F_SENTINEL
+        assert (got.cpu().numpy() == want.cpu().numpy()).all()
+        assert int(st_new.item()) == int(ref_new.item()) == 23
+        seq += int(off[-1])
+    assert table_keys(st_slots) == table_keys(ref_slots) == {r.tobytes() for r in pool[:23]}
