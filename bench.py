@@ -459,6 +459,10 @@ def main():
     ap.add_argument("--only", default=None,
                     help="with --configs: comma-separated workloads to run (tiny, sysprompt, template, probe, long, "
                          "wide, audit)")
+    ap.add_argument("--microbench", action="store_true",
+                    help="instead of the timed serving step: the integer issue-rate microbenchmark alone, one JSON line")
+    ap.add_argument("--probe-heavy", action="store_true",
+                    help="instead of the timed serving step: the probe-heavy table leg alone, one JSON line")
     args = ap.parse_args()
     if args.seed is None:
         args.seed = int.from_bytes(os.urandom(4), "little")
@@ -467,6 +471,8 @@ def main():
         return reference_arm(args)
     if args.configs:
         return run_configs(args)
+    if args.microbench or args.probe_heavy:
+        return run_single_leg(args)
 
     import torch
     import torch.distributed as dist
@@ -960,6 +966,25 @@ def cpu_baseline(w, sample, gpu_digests):
             "value_1_thread": one_blocks / dt1,
             "sample_1_thread": f"{one_reps} steps over the first {one_sample} requests, one thread; {dt1:.1f} s",
             "gate_sample_digests_equal_gpu": same}
+
+
+def run_single_leg(args):
+    """One measurement leg of the default run on its own (for a short run or
+    an ncu capture of that leg's kernels)."""
+    import torch
+
+    from paper_2608_09225_gb300 import build as kbuild
+    from paper_2608_09225_gb300 import kvgov as K
+    from paper_2608_09225_gb300 import workloads as W
+    kbuild.build()
+    K.lib()
+    if args.microbench:
+        out = {"int_ops_per_clk_per_sm_measured": measure_int_peak(torch, kbuild.PEAK_LIB),
+               "lone_warp_cycles_per_round": measure_lone_warp_round(torch, kbuild.PEAK_LIB)}
+    else:
+        out = {"table_roofline_cfg4": probe_heavy_leg(torch, K, W, kbuild)}
+    print(json.dumps(out), flush=True)
+    return 0
 
 
 # --------------------------------------------------------------------------- per-workload rates
