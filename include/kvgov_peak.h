@@ -28,7 +28,10 @@ typedef struct CUstream_st *kvgov_stream_t;
  *   6 SHA-256 rounds alone with K_t + W_t in registers (T1/T2 grouping),
  *   7 the same rounds with the shorter e-to-e grouping, and two-kind mixes
  *   (half the streams each, interleaved) that show whether two kinds share
- *   a pipe: 8 LOP3 + IADD3, 9 LOP3 + IMAD, 10 SHF + IADD3.
+ *   a pipe: 8 LOP3 + IADD3, 9 LOP3 + IMAD, 10 SHF + IADD3; 11 the chain
+ *   kernel's steady block (a 96-byte message, two compact compressions,
+ *   2 x 1384 nominal ops) with every add on the ALU, 12 the same with the
+ *   adds off the rounds' dependency chain on the FMA pipe.
  * d_clocks [blocks][3] u64 receives, per CTA, its SM id and its clock64()
  * at start and end.  d_sink [1] u32 is written only in a case that never
  * happens (keeps results live).  Asynchronous on `stream`.

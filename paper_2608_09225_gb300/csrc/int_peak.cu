@@ -22,6 +22,11 @@
 //   8  LOP3 on streams 0-3 and IADD3 on streams 4-7, interleaved
 //   9  LOP3 on streams 0-3 and IMAD on streams 4-7
 //  10  SHF on streams 0-3 and IADD3 on streams 4-7
+//  11  the chain kernel's steady block: H(P || T), a 96-byte message = two
+//      compact compressions (2 x 1384 nominal ops) on each of 2 independent
+//      chains, every add on the ALU (sha_compress_small)
+//  12  the same with the adds off the rounds' dependency chain on the FMA
+//      pipe (sha_compress_small_split)
 // Kinds 8-10 show whether two kinds of instruction share one pipe: if they
 // do, the mix runs at the slower kind's rate; if not, it can run above it.
 // Kinds 6 and 7 count 14 nominal ops a round; launched with one warp per SM
@@ -71,6 +76,37 @@ __global__ void peak_kernel(int iters, uint32_t seed, uint32_t one, uint32_t *si
         }
 #pragma unroll
         for (int i = 0; i < 8; ++i) x[i] = v[i];
+    } else if (KIND == 11 || KIND == 12) {
+        uint32_t st[kShaChains][8];
+#pragma unroll
+        for (int c = 0; c < kShaChains; ++c) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) st[c][i] = x[i] + c;
+        }
+        for (int it = 0; it < iters; ++it) {
+#pragma unroll
+            for (int c = 0; c < kShaChains; ++c) {
+                // H(st || T) with T = 16 words derived from st: two compressions from the IV
+                uint32_t s[8], w[16];
+                kvgov_dev::sha_iv(s);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) { w[i] = st[c][i]; w[8 + i] = st[c][i] ^ (uint32_t)(it + i); }
+                if (KIND == 11) kvgov_dev::sha_compress_small(s, w, kvgov_dev::AddAlu{});
+                else kvgov_dev::sha_compress_small_split(s, w, kvgov_dev::AddFma{one});
+#pragma unroll
+                for (int i = 0; i < 8; ++i) w[i] = st[c][i] + (uint32_t)i;
+                w[8] = 0x80000000u;
+#pragma unroll
+                for (int i = 9; i < 15; ++i) w[i] = 0u;
+                w[15] = 96u * 8u;
+                if (KIND == 11) kvgov_dev::sha_compress_small(s, w, kvgov_dev::AddAlu{});
+                else kvgov_dev::sha_compress_small_split(s, w, kvgov_dev::AddFma{one});
+#pragma unroll
+                for (int i = 0; i < 8; ++i) st[c][i] = s[i];
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) x[i] = st[0][i] ^ st[1][i];
     } else if (KIND == 3 || KIND == 4) {
         uint32_t st[kShaChains][8], w[kShaChains][16];
 #pragma unroll
@@ -134,13 +170,14 @@ extern "C" int kvgov_peak_ops_per_iter(int kind) {
     case 5: return 4 * kStreams;
     case 6: case 7: return 64 * 14;
     case 8: case 9: case 10: return 4 * kStreams;
+    case 11: case 12: return kShaChains * 2 * 1384;
     default: return 0;
     }
 }
 
 extern "C" int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint32_t *d_sink,
                               unsigned long long *d_clocks, kvgov_stream_t stream) {
-    if (kind < 0 || kind > 10 || iters <= 0 || blocks <= 0 || threads <= 0 || threads > 1024 || !d_sink ||
+    if (kind < 0 || kind > 12 || iters <= 0 || blocks <= 0 || threads <= 0 || threads > 1024 || !d_sink ||
         !d_clocks)
         return 1;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
@@ -155,7 +192,9 @@ extern "C" int kvgov_peak_int(int kind, int iters, int blocks, int threads, uint
     case 7: peak_kernel<7><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
     case 8: peak_kernel<8><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
     case 9: peak_kernel<9><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
-    default: peak_kernel<10><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 10: peak_kernel<10><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    case 11: peak_kernel<11><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
+    default: peak_kernel<12><<<blocks, threads, 0, s>>>(iters, 1u, 1u, d_sink, d_clocks); break;
     }
     return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }

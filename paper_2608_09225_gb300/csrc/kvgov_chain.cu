@@ -205,7 +205,6 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
     const long long pstride = (long long)gridDim.x * kR;
     long long pq = r, prow = 0;
     long long pleft = 0;
-    uint2 wl = make_uint2(0u, 0u);               // first digest word of row prow + 1
     auto prev_next = [&]() {                     // from pq on: the first request with uncached blocks
         for (; pq < q.n_req; pq += pstride) {
             const long long base = q.blk_off[pq], pnb = q.blk_off[pq + 1] - base;
@@ -218,20 +217,12 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             if (pnb > L) {
                 prow = base + L;
                 pleft = pnb - L;
-                if (pleft > 1) wl = __ldg(reinterpret_cast<const uint2 *>(q.digests + 2 * (prow + 1)));
                 return;
             }
         }
         pleft = 0;
     };
-    // Each call prefetches the home slot of the next key into L2 (from the
-    // digest word the previous call loaded) and loads the word of the key
-    // after it, so that no insert but a request's first waits on DRAM and no
-    // load is waited for.
     auto prev_insert_one = [&]() {               // insert row prow of the previous batch
-        if (pleft > 1) prefetch_l2(q.slots + 4 * (u64_of(wl.x, wl.y) & q.mask));
-        uint2 wn = make_uint2(0u, 0u);
-        if (pleft > 2) wn = __ldg(reinterpret_cast<const uint2 *>(q.digests + 2 * (prow + 2)));
         const uint4 x = __ldg(q.digests + 2 * prow), y = __ldg(q.digests + 2 * prow + 1);
         const unsigned long long key[4] = {u64_of(x.x, x.y), u64_of(x.z, x.w), u64_of(y.x, y.y), u64_of(y.z, y.w)};
         if (key_is_zero(key)) {
@@ -240,7 +231,6 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             unsigned long long pos = 0;
             count_insert(insert_one(q.slots, q.mask, key, q.spin_limit, &pos), my_new, my_flags);
         }
-        wl = wn;
         ++prow;
         if (--pleft == 0) {
             pq += pstride;

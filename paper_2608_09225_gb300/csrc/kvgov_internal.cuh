@@ -20,11 +20,6 @@ __device__ __forceinline__ void cp_async16(void *smem_dst, const void *gmem_src,
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 
-// Bring the line holding p into L2 without waiting for it (no register is
-// written, so the thread does not stall).
-__device__ __forceinline__ void prefetch_l2(const void *p) {
-    asm volatile("prefetch.global.L2 [%0];\n" ::"l"(p));
-}
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
 

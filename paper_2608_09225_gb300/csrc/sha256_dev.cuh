@@ -189,6 +189,48 @@ __device__ __forceinline__ void sha_compress_small(uint32_t s[8], uint32_t w[16]
     for (int i = 0; i < 8; ++i) s[i] = add(s[i], v[i]);
 }
 
+// sha_compress_small with the adds that are off the rounds' dependency chain
+// issued on the FMA pipe (`side`, an IMAD with a run-time 1), which SHA-256
+// otherwise leaves idle, so that the integer ALU pipe -- which alone runs the
+// funnel shifts and three-input booleans -- carries fewer instructions:
+//   hk = h + K_t + W_t and dk = d + hk, both known rounds ahead (h and d are
+//   the e and a of three rounds before); then e' = dk + Ch + Sigma1 and
+//   a' = (hk + Ch + Sigma1) + Sigma0 + Maj on the ALU;
+//   in the schedule, W_t + W_{t-7} (known seven rounds ahead) on the FMA
+//   pipe, then + sigma0 + sigma1 on the ALU; the final state adds too.
+// The same sums in another grouping: the same digest.
+__device__ __forceinline__ void sha_compress_small_split(uint32_t s[8], uint32_t w[16], AddFma side) {
+    uint32_t v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = s[i];
+#pragma unroll
+    for (int t = 0; t < 16; ++t) {
+        uint32_t &a = v[(8 - t % 8) % 8], &b = v[(9 - t % 8) % 8], &c = v[(10 - t % 8) % 8], &d = v[(11 - t % 8) % 8];
+        uint32_t &e = v[(12 - t % 8) % 8], &f = v[(13 - t % 8) % 8], &g = v[(14 - t % 8) % 8], &h = v[(15 - t % 8) % 8];
+        const uint32_t hk = side(h, side(w[t], sha_k(t)));
+        const uint32_t dk = side(d, hk);
+        const uint32_t cs = ch(e, f, g), s1 = bsig1(e);
+        d = dk + cs + s1;
+        h = (hk + cs + s1) + bsig0(a) + maj(a, b, c);
+    }
+#pragma unroll 1
+    for (int base = 16; base < 64; base += 16) {
+#pragma unroll
+        for (int t = 0; t < 16; ++t) {
+            w[t] = side(w[t], w[(t + 9) & 15]) + ssig0(w[(t + 1) & 15]) + ssig1(w[(t + 14) & 15]);
+            uint32_t &a = v[(8 - t % 8) % 8], &b = v[(9 - t % 8) % 8], &c = v[(10 - t % 8) % 8], &d = v[(11 - t % 8) % 8];
+            uint32_t &e = v[(12 - t % 8) % 8], &f = v[(13 - t % 8) % 8], &g = v[(14 - t % 8) % 8], &h = v[(15 - t % 8) % 8];
+            const uint32_t hk = side(h, side(w[t], c_sha_k[base + t]));
+            const uint32_t dk = side(d, hk);
+            const uint32_t cs = ch(e, f, g), s1 = bsig1(e);
+            d = dk + cs + s1;
+            h = (hk + cs + s1) + bsig0(a) + maj(a, b, c);
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s[i] = side(s[i], v[i]);
+}
+
 // 16 rounds (FIPS 180-4 section 6.2.2 step 3) with K_t + W_t given, for
 // kernels whose message schedule is computed elsewhere.  v holds a..h in
 // rotating roles; after 16 rounds every variable is back in its original
