@@ -15,23 +15,24 @@
 //   slot 0 (bytes 0-3)  count: entry indices handed out so far (saturates at
 //                       KVGOV_STASH_KEYS; zeroed by kvgov_table_init)
 //   bytes 32-255        state of entry e (u32 at byte 32 + 4e): 0 = being
-//                       decided, kLive = holds a key, kDropped = a duplicate
-//                       that lost to an earlier entry
+//                       written, kStashLive = holds its key
 //   slots 8 .. 63       entry e's key in slot 8 + e; its handle (the slot
 //                       index the arrival-order owner array uses) is
 //                       capacity + 8 + e
 //
-// Insert: look through the entries already handed out; if the key is live
-// in one, it is a duplicate.  Otherwise take the next index with a
-// compare-and-swap on the count (never past the last entry), look through
-// the entries handed out in between, and either drop the new entry (the key
-// went live in an earlier one) or write the key and publish the entry live
-// with a release store.  A thread only ever waits for entries with smaller
-// indices, each of which was handed to a thread that is running, so every
-// wait ends; each wait is bounded all the same (spin_limit re-reads, then
-// KVGOV_F_TIMEOUT).  Two inserts of one key therefore leave one live entry,
-// in any interleaving.  Lookups run while the table does not change and
-// scan the live entries.
+// Insert: look through the entries handed out so far, waiting for each to
+// be published; if the key is live in one, it is a duplicate.  Otherwise
+// take the next entry with a compare-and-swap of the count from the value
+// the scan covered to one more: it succeeds only if no entry was handed out
+// since, so the thread has seen every entry below its own; if another
+// thread took one meanwhile, scan the new entries and try again.  The
+// winner writes the key and publishes the entry live with a release store,
+// with no wait in between, so a thread that waits for an entry waits a few
+// instructions of another thread's (each wait is bounded all the same:
+// spin_limit re-reads, then KVGOV_F_TIMEOUT).  Every entry handed out holds
+// a distinct key, and two inserts of one key leave it in one entry, in any
+// interleaving.  Lookups run while the table does not change and scan the
+// live entries.
 #pragma once
 #include <cstdint>
 
@@ -41,7 +42,6 @@ namespace kvgov_dev {
 
 constexpr int kStashHeaderSlots = 8;
 constexpr uint32_t kStashLive = 1u;
-constexpr uint32_t kStashDropped = 2u;
 static_assert(kStashHeaderSlots + KVGOV_STASH_KEYS == KVGOV_STASH_SLOTS, "side store layout");
 static_assert(32 + 4 * KVGOV_STASH_KEYS <= 32 * kStashHeaderSlots, "entry states fit the header");
 
@@ -86,12 +86,11 @@ static __device__ __noinline__ StashResult stash_insert(unsigned long long *slot
     uint32_t *state = count + 8;
     unsigned long long *keys = base + 4 * kStashHeaderSlots;
     const unsigned long long first = mask + 1 + kStashHeaderSlots;    // handle of entry 0
-    // Wait (bounded) until entry e is decided; 0 on timeout.
-    auto decided = [&](int e) -> uint32_t {
+    // Wait (bounded) until entry e is published; false on timeout.
+    auto published = [&](int e) -> bool {
         for (uint32_t spins = 0;; ++spins) {
-            const uint32_t s = stash_ld_acquire(state + e);
-            if (s != 0u) return s;
-            if (spins >= spin_limit) return 0u;
+            if (stash_ld_acquire(state + e) == kStashLive) return true;
+            if (spins >= spin_limit) return false;
             __nanosleep(100);
         }
     };
@@ -100,48 +99,26 @@ static __device__ __noinline__ StashResult stash_insert(unsigned long long *slot
         return stash_ld_relaxed(w) == k0 && stash_ld_relaxed(w + 1) == k1 && stash_ld_relaxed(w + 2) == k2 &&
                stash_ld_relaxed(w + 3) == k3;
     };
-    // Is the key live in one of the entries [lo, hi)?  -1: no; -2: timeout.
-    auto find = [&](int lo, int hi) -> int {
-        for (int e = lo; e < hi; ++e) {
-            const uint32_t s = decided(e);
-            if (s == 0u) return -2;
-            if (s == kStashLive && holds(e)) return e;
+    uint32_t seen = 0;                                       // entries [0, seen) hold other keys
+    // at most KVGOV_STASH_KEYS entries are ever handed out, and each failed
+    // compare-and-swap below means one was: the loop ends
+    for (;;) {
+        uint32_t cur = stash_ld_acquire(count);
+        if (cur > (uint32_t)KVGOV_STASH_KEYS) cur = KVGOV_STASH_KEYS;
+        for (; seen < cur; ++seen) {
+            if (!published((int)seen)) return {3, 0ull};
+            if (holds((int)seen)) return {1, first + seen};
         }
-        return -1;
-    };
-    const uint32_t seen = stash_ld_acquire(count);
-    const int n = seen < (uint32_t)KVGOV_STASH_KEYS ? (int)seen : KVGOV_STASH_KEYS;
-    int e = find(0, n);
-    if (e == -2) return {3, 0ull};
-    if (e >= 0) return {1, first + (unsigned long long)e};
-    uint32_t cur = seen;
-    while (cur < (uint32_t)KVGOV_STASH_KEYS) {               // at most KVGOV_STASH_KEYS successes ever
-        const uint32_t prev = atomicCAS(count, cur, cur + 1u);
-        if (prev == cur) break;
-        cur = prev;
+        if (cur >= (uint32_t)KVGOV_STASH_KEYS) return {2, 0ull};
+        if (atomicCAS(count, cur, cur + 1u) != cur) continue;   // another entry was handed out: scan it
+        unsigned long long *w = keys + 4 * cur;
+        w[0] = k0;
+        w[1] = k1;
+        w[2] = k2;
+        w[3] = k3;
+        stash_st_release(state + cur, kStashLive);          // the key's words are visible before the state
+        return {0, first + cur};
     }
-    if (cur >= (uint32_t)KVGOV_STASH_KEYS) {                 // full: the key may still have gone in
-        e = find(n, KVGOV_STASH_KEYS);
-        if (e == -2) return {3, 0ull};
-        return e >= 0 ? StashResult{1, first + (unsigned long long)e} : StashResult{2, 0ull};
-    }
-    const int mine = (int)cur;
-    e = find(n, mine);
-    if (e == -2) {
-        stash_st_release(state + mine, kStashDropped);
-        return {3, 0ull};
-    }
-    if (e >= 0) {
-        stash_st_release(state + mine, kStashDropped);
-        return {1, first + (unsigned long long)e};
-    }
-    unsigned long long *w = keys + 4 * mine;
-    w[0] = k0;
-    w[1] = k1;
-    w[2] = k2;
-    w[3] = k3;
-    stash_st_release(state + mine, kStashLive);             // the key's words are visible before the state
-    return {0, first + (unsigned long long)mine};
 }
 
 // Is the key (q0, q1: bytes 0-15, 16-31) live in the side store?  For
