@@ -55,7 +55,8 @@ CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain k
 # step's chain kernel from one ncu capture, and the SHA-256 (chain_source_hash)
 # of the sources it was captured from: reported as roofline.traffic only while
 # the kernel's sources still hash to that value.
-CHAIN_TRAFFIC = {"bytes_per_launch": None, "source_sha256": None}
+CHAIN_TRAFFIC = {"bytes_per_launch": 180052992,
+                 "source_sha256": "0ac246e51adf4874a4d8d7397d19b87432078edfbd38d70fadbfeca2e862d11c"}
 
 
 # DRAM bytes per launch of the probe on the probe-heavy workload from one ncu
@@ -63,7 +64,8 @@ CHAIN_TRAFFIC = {"bytes_per_launch": None, "source_sha256": None}
 TABLE_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_table.cu", "paper_2608_09225_gb300/csrc/kvgov_lookup.cuh",
                  "paper_2608_09225_gb300/csrc/kvgov_stash.cuh", "paper_2608_09225_gb300/csrc/kvgov_internal.cuh",
                  "paper_2608_09225_gb300/csrc/kvgov_insert.cuh"]
-TABLE_TRAFFIC = {"probe_seg_kernel<4, 1>": {"bytes_per_launch": None, "source_sha256": None}}
+TABLE_TRAFFIC = {"probe_seg_kernel<4, 1>": {
+    "bytes_per_launch": 54599808, "source_sha256": "60ab2ce224af39ba7f38a440e5940ba07f987f25082cc616b924bc42d89ac955"}}
 
 
 def load_peaks() -> dict:
