@@ -39,12 +39,13 @@
 // of a warp serve one request and look up a window of its next blocks in
 // parallel; a ballot over the window's misses gives the first miss, else the
 // window moves on (probe_seg_kernel).  The layout depends on the batch size:
-// batches of many requests take 4 lanes per request and a first window of
-// one block (most requests of a batch of fresh prompts miss there), then 4;
-// mid-size batches 16 lanes, windows of 16 then 32; few requests a warp each,
-// windows of 32, 64, then 128 blocks, so that a long cached prefix takes few
-// rounds.  Lookups past the first miss inside a window are wasted: they cost
-// bandwidth but not latency.
+// batches of many requests share each warp's lanes among 8 requests, one
+// lane each for block 0 (most requests of a batch of fresh prompts miss
+// there), then the lanes of the requests that ended go to those still going
+// (probe_share_kernel); mid-size batches 16 lanes per request, windows of 16
+// then 32; few requests a warp each, windows of 32, 64, then 128 blocks, so
+// that a long cached prefix takes few rounds.  Lookups past the first miss
+// inside a window are wasted: they cost bandwidth but not latency.
 #include <atomic>
 
 #include "kvgov_internal.cuh"
@@ -104,7 +105,8 @@ constexpr int kProbeThreads = 256;
 // home slot and the next one together (a walk of two slots in one memory
 // round trip) rather than the home slot alone.
 struct ProbeLayout { int min_req, G, per, pair, first; };
-constexpr ProbeLayout kProbeMany{32768, 4, 1, 0, 1};    // n_req >= 32768
+constexpr int32_t kProbeShareMin = 32768;               // n_req >= 32768: probe_share_kernel
+constexpr int kProbeShareR = 8;                          // ... with 8 requests per warp
 constexpr ProbeLayout kProbeMid{2048, 16, 2, 1, 16};    // 2048 <= n_req < 32768
 constexpr ProbeLayout kProbeFew{0, 32, 4, 1, 32};       // fewer
 
@@ -190,6 +192,67 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
             }
         }
         if (r < n_req && sl == 0) prefix_blocks[r] = (int32_t)L;
+    }
+}
+
+// Large batches: R requests per warp, and in each round the warp's 32 lanes
+// are shared out among the requests still active -- 32 / k consecutive lanes
+// each when k are active -- every lane looking up one block (its home slot
+// and the next, read together).  The first round gives each request one lane
+// (block 0: most requests of a batch of fresh prompts miss there); then a
+// request that goes on gets the lanes of those that ended, so a long cached
+// prefix takes few rounds however short its warp-mates' are.  Request state
+// (row base, block count, prefix so far) stays in lanes 0..R-1 and is
+// shuffled to the lanes that serve it.
+template <int R>
+__global__ void __launch_bounds__(kProbeThreads) probe_share_kernel(const uint4 *__restrict__ slots,
+                                                                    unsigned long long mask,
+                                                                    const uint4 *__restrict__ digests,
+                                                                    const int64_t *__restrict__ blk_off,
+                                                                    int32_t n_req, int32_t *__restrict__ prefix_blocks,
+                                                                    uint32_t *status) {
+    constexpr unsigned kReqMask = (1u << R) - 1u;
+    const int lane = threadIdx.x & 31;
+    const long long warps_total = (long long)gridDim.x * (kProbeThreads / 32);
+    for (long long wg = ((long long)blockIdx.x * kProbeThreads + threadIdx.x) / 32; wg * R < n_req;
+         wg += warps_total) {                                  // warp-uniform
+        const long long r = wg * R + lane;                     // lanes 0..R-1: request r
+        long long base = 0, nb = 0, L = 0;
+        if (lane < R && r < n_req) probe_range(blk_off, n_req, r, base, nb, status);
+        unsigned act = __ballot_sync(0xffffffffu, lane < R && nb > 0) & kReqMask;
+        bool first = true;
+        while (act) {                                          // warp-uniform
+            const int k = __popc(act);
+            const int lp = first ? 1 : 32 / k;                 // lanes per active request this round
+            const int rho = lane / lp, o = lane % lp;          // the active request this lane serves, its block
+            const int s = rho < k ? __fns(act, 0, rho + 1) : 0;
+            const long long sb = __shfl_sync(0xffffffffu, base, s);
+            const long long snb = __shfl_sync(0xffffffffu, nb, s);
+            const long long sL = __shfl_sync(0xffffffffu, L, s);
+            bool miss = false;
+            if (rho < k && sL + o < snb) {
+                const uint4 q0 = __ldg(digests + 2 * (sb + sL + o)), q1 = __ldg(digests + 2 * (sb + sL + o) + 1);
+                const unsigned long long h = home_slot(q0, mask), h1 = (h + 1) & mask;
+                const uint4 a = __ldg(slots + 2 * h), b = __ldg(slots + 2 * h + 1);
+                const uint4 c = __ldg(slots + 2 * h1), d = __ldg(slots + 2 * h1 + 1);
+                miss = !lookup_from_pair(slots, mask, q0, q1, a, b, c, d);
+            }
+            const unsigned mb = __ballot_sync(0xffffffffu, miss);
+            if (lane < R && ((act >> lane) & 1u)) {
+                const int my = __popc(act & ((1u << lane) - 1u));       // this request's rank among the active
+                const unsigned seg = (mb >> (my * lp)) & (lp == 32 ? 0xffffffffu : ((1u << lp) - 1u));
+                if (seg) {
+                    L += __ffs((int)seg) - 1;
+                    act &= ~(1u << lane);
+                } else {
+                    L += (nb - L < lp) ? (nb - L) : lp;
+                    if (L >= nb) act &= ~(1u << lane);
+                }
+            }
+            act = __ballot_sync(0xffffffffu, lane < R && ((act >> lane) & 1u)) & kReqMask;
+            first = false;
+        }
+        if (lane < R && r < n_req) prefix_blocks[r] = (int32_t)L;
     }
 }
 
@@ -311,10 +374,9 @@ extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint
     if (!d_digests || !aligned16(d_digests) || !d_blk_off || !d_prefix_blocks) return KVGOV_EINVAL;
     const uint4 *slots = reinterpret_cast<const uint4 *>(d_slots), *dig = reinterpret_cast<const uint4 *>(d_digests);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    if (n_req >= kProbeMany.min_req)
-        probe_seg_kernel<kProbeMany.G, kProbeMany.per, kProbeMany.pair != 0>
-            <<<probe_grid(n_req, kProbeMany.G), kProbeThreads, 0, s>>>(
-                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, kProbeMany.first);
+    if (n_req >= kProbeShareMin)
+        probe_share_kernel<kProbeShareR><<<probe_grid(n_req, 32 / kProbeShareR), kProbeThreads, 0, s>>>(
+            slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status);
     else if (n_req >= kProbeMid.min_req)
         probe_seg_kernel<kProbeMid.G, kProbeMid.per, kProbeMid.pair != 0>
             <<<probe_grid(n_req, kProbeMid.G), kProbeThreads, 0, s>>>(
