@@ -126,7 +126,9 @@ __device__ __forceinline__ float rcp_approx(float x) {
 // which then never counts as above the level and gets p = 0): the steps
 // compare lambda * (1 / v_i) with 1 and sum reciprocals, with no division
 // per tenant, and p_i = 1 - lambda * (1 / v_i).  The kMax - n padding slots
-// hold 0 -- not usable, not flagged, adding exactly 0 to every sum.  The
+// hold 0 -- not usable, not flagged, adding exactly 0 to every sum.  Register
+// tiers of 16, 32, 50 (the paper's 50-tenant problems, section 5.5) and 64
+// slots.  The
 // adversary's payoff is lambda whenever a tenant is usable (min(v_i, lambda)
 // over the usable ones, the others at most 0), else the largest value.
 template <int kMax>
@@ -158,12 +160,17 @@ __device__ __forceinline__ void solve_thread_reg(float *x, const float *__restri
     } else {
         lam = ((float)npos - K) / sum_all;
         int prev_m = npos;
+        // a tenant is above the level when 1 / v_i is below 1 / lambda: one
+        // compare per tenant against a threshold taken once per step (a tenant
+        // on the level adds nothing either way: the budget curve is continuous
+        // there)
         for (int step = 0; step <= npos; ++step) {
+            const float t = rcp_approx(lam);
             float sum = 0.0f;
             int m = 0;
 #pragma unroll
             for (int i = 0; i < kMax; ++i) {
-                const bool on = lam * r[i] < 1.0f;
+                const bool on = r[i] < t;
                 sum += on ? r[i] : 0.0f;
                 m += on;
             }
@@ -226,7 +233,7 @@ __global__ void __launch_bounds__(kCta) origami_kernel(const float *__restrict__
             const int n = (int)(my1 - my0);
             if (n <= 16) solve_thread_reg<16>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
             else if (n <= 32) solve_thread_reg<32>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
-            else if (n <= 56) solve_thread_reg<56>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
+            else if (n <= 50) solve_thread_reg<50>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
             else solve_thread_reg<kSmallN>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
         }
         __syncthreads();
