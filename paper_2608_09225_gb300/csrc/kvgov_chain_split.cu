@@ -79,9 +79,6 @@ struct SplitParams {
     uint32_t *status;
     int32_t n_req;
     int32_t n_principals;
-    // K_t + W_t of the padding block that ends a 128-byte message (the
-    // boundary block's third compression), the same for every chain
-    uint32_t pad128_kw[64];
 };
 
 // What block j's message is, per section 2.1 / 4.1 / 4.2.
@@ -98,10 +95,54 @@ __device__ __forceinline__ int block_kind(int j, int k) {
     return j == k ? kBoundary : kSteadyH;
 }
 
+// K_t + W_t of the padding block that ends a 128-byte message (the boundary
+// block's third compression): FIPS 180-4 section 5.1.1 padding (0x80, zeros,
+// the 64-bit bit length 1024) and section 6.2.2 step 1, evaluated by the
+// compiler.
+struct PadSchedule {
+    uint32_t kw[64];
+};
+constexpr uint32_t rotr_c(uint32_t x, int n) { return (x >> n) | (x << (32 - n)); }
+constexpr PadSchedule pad_schedule(uint32_t bytes) {
+    PadSchedule r{};
+    uint32_t w[64] = {};
+    w[0] = 0x80000000u;
+    w[15] = bytes * 8u;
+    for (int t = 16; t < 64; ++t) {
+        const uint32_t s0 = rotr_c(w[t - 15], 7) ^ rotr_c(w[t - 15], 18) ^ (w[t - 15] >> 3);
+        const uint32_t s1 = rotr_c(w[t - 2], 17) ^ rotr_c(w[t - 2], 19) ^ (w[t - 2] >> 10);
+        w[t] = w[t - 16] + s0 + w[t - 7] + s1;
+    }
+    for (int t = 0; t < 64; ++t) r.kw[t] = kShaKHost[t] + w[t];
+    return r;
+}
+__constant__ PadSchedule c_pad128 = pad_schedule(128);
+
 // The round warp's 16 rounds (sha256_dev.cuh).  Another grouping of the
 // sums (sha_rounds16_short) measured the same on a lone warp (libkvgov_peak
 // kinds 6, 7).
 __device__ __forceinline__ void rounds16(uint32_t v[8], const uint32_t kw[16]) { sha_rounds16_t1t2(v, kw); }
+
+// The boundary block's third compression, the constant padding block, out
+// of the round warp's loop: a chain runs it once, and kept inline its code
+// sat inside the loop every other block runs.
+struct State8 {
+    uint32_t w[8];
+};
+static __device__ __noinline__ State8 padding_compression(State8 s) {
+    uint32_t v[8], kw[16];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = s.w[i];
+#pragma unroll 1
+    for (int q = 0; q < 4; ++q) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) kw[i] = c_pad128.kw[16 * q + i];
+        rounds16(v, kw);
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s.w[i] += v[i];
+    return s;
+}
 
 template <int MODE>
 __global__ void __launch_bounds__(kThreads, 1) chain_split_kernel(const SplitParams p) {
@@ -182,19 +223,15 @@ __global__ void __launch_bounds__(kThreads, 1) chain_split_kernel(const SplitPar
             }
 #pragma unroll
             for (int i = 0; i < 8; ++i) s[i] += v[i];
-            // the boundary block's padding block: K_t + W_t from the launch parameters
+            // the boundary block's padding block
             if (MODE == KVGOV_BOUNDARY && __any_sync(0xffffffffu, j > 0 && j == k && j < nb)) {
+                State8 st;
 #pragma unroll
-                for (int i = 0; i < 8; ++i) v[i] = s[i];
-#pragma unroll 1
-                for (int q = 0; q < 4; ++q) {
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) kw[i] = p.pad128_kw[16 * q + i];
-                    rounds16(v, kw);
-                }
+                for (int i = 0; i < 8; ++i) st.w[i] = s[i];
+                st = padding_compression(st);
                 if (j > 0 && j == k && j < nb) {
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) s[i] += v[i];
+                    for (int i = 0; i < 8; ++i) s[i] = st.w[i];
                 }
             }
             sm.h[0][lane] = make_uint4(s[0], s[1], s[2], s[3]);
@@ -340,22 +377,6 @@ long long chain_split_max_req() { return kSplitCtasPerSm * sm_count() * kChainsP
 
 namespace {
 
-// FIPS 180-4 section 6.2.2 step 1 on the host: K_t + W_t of the padding
-// block (0x80, zeros, the 64-bit bit length) of a message of `bytes` bytes
-// that fills whole 64-byte blocks.
-void padding_schedule(uint32_t bytes, uint32_t kw[64]) {
-    auto rotr = [](uint32_t x, int n) { return (x >> n) | (x << (32 - n)); };
-    uint32_t w[64] = {};
-    w[0] = 0x80000000u;
-    w[15] = bytes * 8u;
-    for (int t = 16; t < 64; ++t) {
-        const uint32_t s0 = rotr(w[t - 15], 7) ^ rotr(w[t - 15], 18) ^ (w[t - 15] >> 3);
-        const uint32_t s1 = rotr(w[t - 2], 17) ^ rotr(w[t - 2], 19) ^ (w[t - 2] >> 10);
-        w[t] = w[t - 16] + s0 + w[t - 7] + s1;
-    }
-    for (int t = 0; t < 64; ++t) kw[t] = kvgov_dev::kShaKHost[t] + w[t];
-}
-
 }  // namespace
 
 int launch_chain_split(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
@@ -367,7 +388,6 @@ int launch_chain_split(int mode, const int32_t *d_tokens, const int64_t *d_tok_o
     p.tokens = d_tokens; p.tok_off = d_tok_off; p.principal = d_principal; p.salts = d_salts;
     p.boundary_tok = d_boundary_tok; p.blk_off = d_blk_off; p.digests = d_digests; p.status = d_status;
     p.n_req = n_req; p.n_principals = n_principals;
-    padding_schedule(128, p.pad128_kw);
     const unsigned grid = (unsigned)(((long long)n_req + kChainsPerCta - 1) / kChainsPerCta);
     switch (mode) {
     case KVGOV_UNSALTED: return launch_mode<KVGOV_UNSALTED>(grid, p, stream);
