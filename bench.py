@@ -1210,6 +1210,14 @@ def run_configs(args):
         misses = int((L < nb).sum())
         probe_bytes = hits * (32 + 16 * (1 + 1 / (1 - a))) + misses * (32 + 16 * (1 + 1 / (1 - a) ** 2)) + 4 * (p1 - p0)
         insert_bytes = keys.shape[0] * (32 + 16 * (1 + 1 / (1 - a)) + 32)
+        # floors: random slot bytes at the random-read ceiling, streamed bytes (digests, keys, results) at
+        # the copy bandwidth
+        probe_random = hits * 16 * (1 + 1 / (1 - a)) + misses * 16 * (1 + 1 / (1 - a) ** 2)
+        probe_floor = 1e3 * (probe_random / (gather["gbs_32B"] * 1e9) +
+                             (probe_bytes - probe_random) / (PEAKS["hbm_gbs"] * 1e9))
+        insert_random = keys.shape[0] * (16 * (1 + 1 / (1 - a)) + 32)
+        insert_floor = 1e3 * (insert_random / (gather["gbs_32B"] * 1e9) +
+                              (insert_bytes - insert_random) / (PEAKS["hbm_gbs"] * 1e9))
         # a batch that leaves every round warp alone on its sub-partition (at most 64 chains
         # per SM) is bound by the latency of its longest chain: 2 compressions per block,
         # one more for a boundary block, 64 rounds each at the lone-warp round time
@@ -1232,11 +1240,11 @@ def run_configs(args):
                 "inserts_per_s": keys.shape[0] / ((t_insert - t_init) / 1e3), "load_factor": a,
                 "probe_gbs": probe_bytes / (t_probe / 1e3) / 1e9,
                 "probe_frac_hbm": probe_bytes / (t_probe / 1e3) / 1e9 / PEAKS["hbm_gbs"],
-                "probe_frac_random_read": probe_bytes / (t_probe / 1e3) / 1e9 / gather["gbs_32B"],
+                "probe_floor_ms": probe_floor, "probe_frac_floor": probe_floor / t_probe,
                 "response_key_ms": t_resp, "response_keys_per_s": b.n / (t_resp / 1e3),
                 "response_tokens_per_s": float(b.lengths().sum()) / (t_resp / 1e3),
                 "response_compressions": resp_comp,
-                "response_frac_int32_peak": resp_comp * 1384 / (t_resp / 1e3) / peak,
+                "response_frac_sha256_ceiling": resp_comp * 1384 / (t_resp / 1e3) / peak,
                 "boundary_preamble_tokens": n_pre, "boundary_ms": t_bnd,
                 "boundary_mean_tokens": float(bnd_np.mean()) if b.n else 0.0,
                 "boundary_gbs": bnd_bytes / (t_bnd / 1e3) / 1e9,
@@ -1247,7 +1255,7 @@ def run_configs(args):
                 "arrival_mean_prefix_blocks": float(La.mean()),
                 "arrival_hit_fraction": float(La.sum()) / max(1, n_blocks),
                 "insert_gbs": insert_bytes / ((t_insert - t_init) / 1e3) / 1e9,
-                "insert_frac_random_read": insert_bytes / ((t_insert - t_init) / 1e3) / 1e9 / gather["gbs_32B"]}
+                "insert_floor_ms": insert_floor, "insert_frac_floor": insert_floor / (t_insert - t_init)}
         if not args.no_cpu_baseline:
             line.update(_oracle_rate(w, mode, cores))
             line["oracle_cores"] = cores
