@@ -39,7 +39,7 @@
 // of a warp serve one request and look up a window of its next blocks in
 // parallel; a ballot over the window's misses gives the first miss, else the
 // window moves on (probe_seg_kernel).  The layout depends on the batch size:
-// batches of many requests share each warp's lanes among 8 requests, one
+// batches of many requests share each warp's lanes among 16 requests, one
 // lane each for block 0 (most requests of a batch of fresh prompts miss
 // there), then the lanes of the requests that ended go to those still going
 // (probe_share_kernel); mid-size batches 16 lanes per request, windows of 16
@@ -106,7 +106,8 @@ constexpr int kProbeThreads = 256;
 // round trip) rather than the home slot alone.
 struct ProbeLayout { int min_req, G, per, pair, first; };
 constexpr int32_t kProbeShareMin = 32768;               // n_req >= 32768: probe_share_kernel
-constexpr int kProbeShareR = 8;                          // ... with 8 requests per warp
+constexpr int kProbeShareR = 16;                         // ... with 16 requests per warp
+constexpr bool kProbeSharePair = true;                   // ... reading the home slot and the next together
 constexpr ProbeLayout kProbeMid{2048, 16, 2, 1, 16};    // 2048 <= n_req < 32768
 constexpr ProbeLayout kProbeFew{0, 32, 4, 1, 32};       // fewer
 
@@ -204,7 +205,7 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
 // prefix takes few rounds however short its warp-mates' are.  Request state
 // (row base, block count, prefix so far) stays in lanes 0..R-1 and is
 // shuffled to the lanes that serve it.
-template <int R>
+template <int R, bool PAIR>
 __global__ void __launch_bounds__(kProbeThreads) probe_share_kernel(const uint4 *__restrict__ slots,
                                                                     unsigned long long mask,
                                                                     const uint4 *__restrict__ digests,
@@ -232,10 +233,15 @@ __global__ void __launch_bounds__(kProbeThreads) probe_share_kernel(const uint4 
             bool miss = false;
             if (rho < k && sL + o < snb) {
                 const uint4 q0 = __ldg(digests + 2 * (sb + sL + o)), q1 = __ldg(digests + 2 * (sb + sL + o) + 1);
-                const unsigned long long h = home_slot(q0, mask), h1 = (h + 1) & mask;
+                const unsigned long long h = home_slot(q0, mask);
                 const uint4 a = __ldg(slots + 2 * h), b = __ldg(slots + 2 * h + 1);
-                const uint4 c = __ldg(slots + 2 * h1), d = __ldg(slots + 2 * h1 + 1);
-                miss = !lookup_from_pair(slots, mask, q0, q1, a, b, c, d);
+                if (PAIR) {
+                    const unsigned long long h1 = (h + 1) & mask;
+                    const uint4 c = __ldg(slots + 2 * h1), d = __ldg(slots + 2 * h1 + 1);
+                    miss = !lookup_from_pair(slots, mask, q0, q1, a, b, c, d);
+                } else {
+                    miss = !lookup_from_home(slots, mask, q0, q1, a, b);
+                }
             }
             const unsigned mb = __ballot_sync(0xffffffffu, miss);
             if (lane < R && ((act >> lane) & 1u)) {
@@ -375,7 +381,7 @@ extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint
     const uint4 *slots = reinterpret_cast<const uint4 *>(d_slots), *dig = reinterpret_cast<const uint4 *>(d_digests);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     if (n_req >= kProbeShareMin)
-        probe_share_kernel<kProbeShareR><<<probe_grid(n_req, 32 / kProbeShareR), kProbeThreads, 0, s>>>(
+        probe_share_kernel<kProbeShareR, kProbeSharePair><<<probe_grid(n_req, 32 / kProbeShareR), kProbeThreads, 0, s>>>(
             slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status);
     else if (n_req >= kProbeMid.min_req)
         probe_seg_kernel<kProbeMid.G, kProbeMid.per, kProbeMid.pair != 0>
