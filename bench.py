@@ -67,7 +67,7 @@ TABLE_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_table.cu", "paper_2608_09225
                  "paper_2608_09225_gb300/csrc/kvgov_stash.cuh", "paper_2608_09225_gb300/csrc/kvgov_internal.cuh",
                  "paper_2608_09225_gb300/csrc/kvgov_insert.cuh"]
 TABLE_TRAFFIC = {"probe_share_kernel<16, true>": {
-    "bytes_per_launch": 54599808, "source_sha256": "60ab2ce224af39ba7f38a440e5940ba07f987f25082cc616b924bc42d89ac955"}}
+    "bytes_per_launch": 70829952, "source_sha256": "a783b5d825a97b2b42927d934ff1e644cb3aa3f343ee86860371c75c0a660472"}}
 
 
 def load_peaks() -> dict:
