@@ -45,7 +45,11 @@
 // (probe_share_kernel); mid-size batches 16 lanes per request, windows of 16
 // then 32; few requests a warp each, windows of 32, 64, then 128 blocks, so
 // that a long cached prefix takes few rounds.  Lookups past the first miss
-// inside a window are wasted: they cost bandwidth but not latency.
+// inside a window are wasted: they cost bandwidth but not latency.  In every
+// layout each lookup first reads its key's home slot and the next one
+// together; the walks that go on past them are finished by the whole warp
+// at once (warp_finish_walks), and a walk past a miss already found for its
+// request is dropped.
 #include <atomic>
 
 #include "kvgov_internal.cuh"
@@ -101,15 +105,21 @@ __global__ void __launch_bounds__(kInsertThreads) insert_kernel(unsigned long lo
 // ---------------------------------------------------------------------------
 constexpr int kProbeThreads = 256;
 // Probe layouts by batch size (measured side by side over every workload):
-// probe_seg_kernel<G, kPer, PAIR> with first window F.  PAIR reads a key's
+// probe_seg_kernel<G, kPer, PAIR, COOP> with first window F.  PAIR reads a key's
 // home slot and the next one together (a walk of two slots in one memory
 // round trip) rather than the home slot alone.
-struct ProbeLayout { int min_req, G, per, pair, first; };
+// COOP finishes the walks that go past their first slots with the whole
+// warp (warp_finish_walks) rather than each lane on its own: it pays where
+// the table is loaded and many lanes look up at once (mid-size batches:
+// 8.5 -> 6.5 us on 4096 requests at load factor 0.5), not with one request
+// a warp, whose four lookups a lane would finish one after another (a
+// 2048-block prefix: 45 -> 57 us).
+struct ProbeLayout { int min_req, G, per, pair, first, coop; };
 constexpr int32_t kProbeShareMin = 32768;               // n_req >= 32768: probe_share_kernel
 constexpr int kProbeShareR = 16;                         // ... with 16 requests per warp
 constexpr bool kProbeSharePair = true;                   // ... reading the home slot and the next together
-constexpr ProbeLayout kProbeMid{2048, 16, 2, 1, 16};    // 2048 <= n_req < 32768
-constexpr ProbeLayout kProbeFew{0, 32, 4, 1, 32};       // fewer
+constexpr ProbeLayout kProbeMid{2048, 16, 2, 1, 16, 1};    // 2048 <= n_req < 32768
+constexpr ProbeLayout kProbeFew{0, 32, 4, 1, 32, 0};     // fewer
 
 // Request r's block range; a malformed one is flagged and counts as empty.
 __device__ __forceinline__ void probe_range(const int64_t *__restrict__ blk_off, int32_t n_req, long long r,
@@ -128,7 +138,7 @@ __device__ __forceinline__ void probe_range(const int64_t *__restrict__ blk_off,
 // their memory accesses overlap).  A small first window wastes few lookups
 // on a request that misses early; the growing windows take a long cached
 // prefix in few rounds.
-template <int G, int kPer, bool PAIR>
+template <int G, int kPer, bool PAIR, bool COOP>
 __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *__restrict__ slots,
                                                                   unsigned long long mask,
                                                                   const uint4 *__restrict__ digests,
@@ -152,6 +162,7 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
 #pragma unroll
             for (int u = 0; u < kPer; ++u) {
                 const int o = sl + G * u;
+                q0[u] = q1[u] = make_uint4(0u, 0u, 0u, 0u);
                 if (active && o < w && L + o < nb) {
                     q0[u] = __ldg(digests + 2 * (base + L + o));
                     q1[u] = __ldg(digests + 2 * (base + L + o) + 1);
@@ -164,6 +175,8 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
                     const unsigned long long h = home_slot(q0[u], mask);
                     a[u] = __ldg(slots + 2 * h);
                     b[u] = __ldg(slots + 2 * h + 1);
+                    c[u] = a[u];
+                    d[u] = b[u];
                     if (PAIR) {
                         const unsigned long long h1 = (h + 1) & mask;
                         c[u] = __ldg(slots + 2 * h1);
@@ -175,10 +188,17 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
 #pragma unroll
             for (int u = 0; u < kPer; ++u) {
                 const int o = sl + G * u;
-                const bool miss = active && o < w && L + o < nb &&
-                                  !(PAIR ? lookup_from_pair(slots, mask, q0[u], q1[u], a[u], b[u], c[u], d[u])
-                                         : lookup_from_home(slots, mask, q0[u], q1[u], a[u], b[u]));
-                const unsigned m = (__ballot_sync(0xffffffffu, miss) >> (seg * G)) & kSegMask;
+                const bool valid = active && o < w && L + o < nb;
+                int st = valid ? walk_start<PAIR ? 2 : 1>(slots, mask, q0[u], q1[u], a[u], b[u], c[u], d[u]) : 1;
+                if (COOP) {
+                    // a walk past a miss already found for its request decides nothing: drop it
+                    const unsigned m0 = (__ballot_sync(0xffffffffu, st == 0) >> (seg * G)) & kSegMask;
+                    if (st < 0 && (miss_at >= 0 || (m0 & ((1u << sl) - 1u)))) st = 0;
+                    st = warp_finish_walks<PAIR ? 2 : 1>(slots, mask, q0[u], q1[u], st);
+                } else if (st < 0) {
+                    st = walk_on<PAIR ? 2 : 1>(slots, mask, q0[u], q1[u]);
+                }
+                const unsigned m = (__ballot_sync(0xffffffffu, valid && st == 0) >> (seg * G)) & kSegMask;
                 if (m && miss_at < 0) miss_at = G * u + __ffs((int)m) - 1;
             }
             if (active) {
@@ -230,19 +250,29 @@ __global__ void __launch_bounds__(kProbeThreads) probe_share_kernel(const uint4 
             const long long sb = __shfl_sync(0xffffffffu, base, s);
             const long long snb = __shfl_sync(0xffffffffu, nb, s);
             const long long sL = __shfl_sync(0xffffffffu, L, s);
-            bool miss = false;
-            if (rho < k && sL + o < snb) {
-                const uint4 q0 = __ldg(digests + 2 * (sb + sL + o)), q1 = __ldg(digests + 2 * (sb + sL + o) + 1);
+            const bool valid = rho < k && sL + o < snb;
+            uint4 q0 = make_uint4(0u, 0u, 0u, 0u), q1 = q0;
+            int st = 1;                                        // walk state (walk_start); no lookup: not a miss
+            if (valid) {
+                q0 = __ldg(digests + 2 * (sb + sL + o));
+                q1 = __ldg(digests + 2 * (sb + sL + o) + 1);
                 const unsigned long long h = home_slot(q0, mask);
                 const uint4 a = __ldg(slots + 2 * h), b = __ldg(slots + 2 * h + 1);
+                uint4 c = a, d = b;
                 if (PAIR) {
                     const unsigned long long h1 = (h + 1) & mask;
-                    const uint4 c = __ldg(slots + 2 * h1), d = __ldg(slots + 2 * h1 + 1);
-                    miss = !lookup_from_pair(slots, mask, q0, q1, a, b, c, d);
-                } else {
-                    miss = !lookup_from_home(slots, mask, q0, q1, a, b);
+                    c = __ldg(slots + 2 * h1);
+                    d = __ldg(slots + 2 * h1 + 1);
                 }
+                st = walk_start<PAIR ? 2 : 1>(slots, mask, q0, q1, a, b, c, d);
             }
+            {   // a walk past a miss already found for its request decides nothing: drop it
+                const unsigned m0 = __ballot_sync(0xffffffffu, st == 0);
+                const unsigned grp = lp == 32 ? 0xffffffffu : ((1u << lp) - 1u) << (rho * lp);
+                if (st < 0 && (m0 & grp & ((1u << lane) - 1u))) st = 0;
+            }
+            st = warp_finish_walks<PAIR ? 2 : 1>(slots, mask, q0, q1, st);
+            const bool miss = valid && st == 0;
             const unsigned mb = __ballot_sync(0xffffffffu, miss);
             if (lane < R && ((act >> lane) & 1u)) {
                 const int my = __popc(act & ((1u << lane) - 1u));       // this request's rank among the active
@@ -384,11 +414,11 @@ extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint
         probe_share_kernel<kProbeShareR, kProbeSharePair><<<probe_grid(n_req, 32 / kProbeShareR), kProbeThreads, 0, s>>>(
             slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status);
     else if (n_req >= kProbeMid.min_req)
-        probe_seg_kernel<kProbeMid.G, kProbeMid.per, kProbeMid.pair != 0>
+        probe_seg_kernel<kProbeMid.G, kProbeMid.per, kProbeMid.pair != 0, kProbeMid.coop != 0>
             <<<probe_grid(n_req, kProbeMid.G), kProbeThreads, 0, s>>>(
                 slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, kProbeMid.first);
     else
-        probe_seg_kernel<kProbeFew.G, kProbeFew.per, kProbeFew.pair != 0>
+        probe_seg_kernel<kProbeFew.G, kProbeFew.per, kProbeFew.pair != 0, kProbeFew.coop != 0>
             <<<probe_grid(n_req, kProbeFew.G), kProbeThreads, 0, s>>>(
                 slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, kProbeFew.first);
     return kvgov_host::launch_status();

@@ -461,6 +461,46 @@ def test_probe_layouts_match_oracle(kv, n_req, max_nb, p_member):
 
 
 @pytest.mark.parametrize("n_req", [500, 5000, 40000], ids=["few", "mid", "many"])
+@pytest.mark.parametrize("cap_log2,n_keys,clustered", [(12, 3686, 0), (12, 2400, 400), (5, 28, 0), (16, 49152, 0)],
+                         ids=["load_0.9", "clustered_run", "window_is_table", "load_0.75"])
+def test_probe_long_walks_match_oracle(kv, cap_log2, n_keys, clustered, n_req):
+    """Every probe layout, where a warp's walks that go past their first two
+    slots are finished together, on tables with long walks: load factor 0.9; `clustered` keys (and 32 absent ones) homed within
+    16 slots, so that walks run for hundreds of slots (the longest run of
+    filled slots is 809, under the 1024-slot window, so every insert fits);
+    a 32-slot table whose window is the whole table.  Requests of 1-3 blocks
+    drawn 80 % from the stored keys and 20 % from absent ones."""
+    cap = 1 << cap_log2
+    pool = keys_np(n_keys + n_keys // 2 + 64, 500 + cap_log2 + clustered)
+    if clustered:
+        idx = np.r_[0:clustered, n_keys:n_keys + 32]
+        h = pool[idx, :8].copy().view(np.uint64)[:, 0]
+        h = (h & ~np.uint64(cap - 1)) | (np.uint64(cap // 4) + (h & np.uint64(15)))
+        pool[idx, :8] = h.reshape(-1, 1).view(np.uint8)
+    present, absent = pool[:n_keys], pool[n_keys:]
+    rng = np.random.default_rng(cap_log2 + clustered + n_req)
+    nb = rng.integers(1, 4, n_req)
+    off = np.concatenate([[0], np.cumsum(nb)]).astype(np.int64)
+    n = int(off[-1])
+    digests = np.where((rng.random(n) < 0.8)[:, None], present[rng.integers(0, n_keys, n)],
+                       absent[rng.integers(0, len(absent), n)])
+    if clustered:                                        # some requests walk the long run
+        digests[off[1:100]] = absent[rng.integers(0, 32, 99)]
+    slots = kv.new_table(cap)
+    st = status_tensor()
+    kv.insert(slots, dev(present), st)
+    pre = kv.probe(slots, dev(digests), dev(off), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    ks = oracle.KeySet(1)
+    ks.insert(present)
+    want = ks.prefix_blocks(digests, off)
+    got = pre.cpu().numpy()
+    assert (got == want).all(), f"{int((got != want).sum())} of {n_req} prefix lengths differ"
+    assert 0 < (want == 0).sum() < n_req and (want == 3).any()
+
+
+@pytest.mark.parametrize("n_req", [500, 5000, 40000], ids=["few", "mid", "many"])
 def test_probe_bad_range_in_a_batch(kv, n_req):
     """A malformed range (its end before its start) in the middle of a batch
     is flagged and gets prefix 0; every other request, including the next one
