@@ -118,62 +118,83 @@ __device__ __forceinline__ float rcp_approx(float x) {
     return r;
 }
 
+// Loads in flight per thread while a CTA stages its values (16: one round
+// trip for a CTA of 50-tenant problems; 4 took 109 us, 8 105, 16 92 on 2^20
+// such problems), and partial sums per solver pass (independent add chains).
+constexpr int kInFlight = 16;
+constexpr int kAcc = 2;
+__device__ __forceinline__ float acc_total(const float part[kAcc]) {
+    float t = 0.0f;
+#pragma unroll
+    for (int a = 0; a < kAcc; ++a) t += part[a];
+    return t;
+}
+
+// sum += r and m += 1 when r < t, as one compare and two predicated adds
+// (no select per slot whose result would wait in a register).
+__device__ __forceinline__ void add_if_below(float &sum, int &m, float r, float t) {
+    asm("{\n\t.reg .pred on;\n\t"
+        "setp.lt.f32 on, %2, %3;\n\t"
+        "@on add.f32 %0, %0, %2;\n\t"
+        "@on add.s32 %1, %1, 1;\n\t}"
+        : "+f"(sum), "+r"(m)
+        : "f"(r), "f"(t));
+}
+
 // One problem solved by one thread, its n <= kMax values x[0..n) staged in
 // shared memory and held in registers for the solve: one pass over shared
 // memory in and one out, every Newton step on registers (from shared memory
-// the steps' re-reads made the kernel bound by its load pipe).  Each value
-// is replaced by its reciprocal (+infinity for a tenant that is not usable,
-// which then never counts as above the level and gets p = 0): the steps
-// compare lambda * (1 / v_i) with 1 and sum reciprocals, with no division
-// per tenant, and p_i = 1 - lambda * (1 / v_i).  The kMax - n padding slots
-// hold 0 -- not usable, not flagged, adding exactly 0 to every sum.  Register
-// tiers of 16, 32, 50 (the paper's 50-tenant problems, section 5.5) and 64
-// slots.  The
-// adversary's payoff is lambda whenever a tenant is usable (min(v_i, lambda)
-// over the usable ones, the others at most 0), else the largest value.
+// the steps' re-reads made the kernel bound by its load pipe).  Every value
+// is usable (the caller checked the CTA's values as it staged them), so the
+// tenants above the level are found by one compare each: each value is
+// replaced by its reciprocal, the padding slots kMax - n by +infinity (never
+// above the level), and a tenant is above the level when 1 / v_i is below
+// 1 / lambda, taken once per step.  The first Newton step -- every tenant
+// above the level -- is folded into that pass; p_i = 1 - lambda * (1 / v_i).
+// Register tiers of 16, 32, 50 (the paper's 50-tenant problems, section
+// 5.5) and 64 slots.  The adversary's payoff is lambda (some tenant is
+// usable whenever n > 0).
 template <int kMax>
-__device__ __forceinline__ void solve_thread_reg(float *x, const float *__restrict__ vg, int n, float K_in,
-                                                 long long q, float *__restrict__ lambda_out,
-                                                 float *__restrict__ utility_out, uint32_t *status) {
+__device__ __forceinline__ void solve_thread_reg(float *x, int n, float K_in, long long q,
+                                                 float *__restrict__ lambda_out, float *__restrict__ utility_out,
+                                                 uint32_t *status) {
     float r[kMax];
-    int npos = 0, nbad = 0;
-    float vmax = 0.0f, sum_all = 0.0f;
+    float part[kAcc];                                  // kAcc partial sums: independent add chains
+#pragma unroll
+    for (int a = 0; a < kAcc; ++a) part[a] = 0.0f;
 #pragma unroll
     for (int i = 0; i < kMax; ++i) {
-        const float xi = i < n ? x[i] : 0.0f;
-        const bool use = usable(xi);
-        npos += use;
-        nbad += !use && !(xi <= 0.0f);
-        vmax = use ? fmaxf(vmax, xi) : vmax;
-        r[i] = use ? rcp_approx(xi) : __int_as_float(0x7f800000);
-        sum_all += use ? r[i] : 0.0f;
+        r[i] = i < n ? rcp_approx(x[i]) : __int_as_float(0x7f800000);
+        if (i < n) part[i % kAcc] += r[i];
     }
+    const float sum_all = acc_total(part);
     float K = K_in;
-    const bool bad = nbad > 0 || !(K >= 0.0f);
+    const bool bad = !(K >= 0.0f);
     if (!(K >= 0.0f)) K = 0.0f;
-    if (K > (float)npos) K = (float)npos;
+    if (K > (float)n) K = (float)n;
     float lam;
-    if (npos == 0 || K <= 0.0f) {
-        lam = vmax;
-    } else if (K >= (float)npos) {
-        lam = 0.0f;
+    if (n == 0 || K <= 0.0f) {
+        lam = 0.0f;                                   // nothing to spend: p = 0, lambda = the largest value
+        for (int i = 0; i < n; ++i) lam = fmaxf(lam, x[i]);
+    } else if (K >= (float)n) {
+        lam = 0.0f;                                   // every tenant audited
     } else {
-        lam = ((float)npos - K) / sum_all;
-        int prev_m = npos;
-        // a tenant is above the level when 1 / v_i is below 1 / lambda: one
-        // compare per tenant against a threshold taken once per step (a tenant
-        // on the level adds nothing either way: the budget curve is continuous
-        // there)
-        for (int step = 0; step <= npos; ++step) {
+        lam = ((float)n - K) / sum_all;
+        int prev_m = n;
+        // a tenant on the level adds nothing either way: the budget curve is
+        // continuous there
+        for (int step = 0; step <= n; ++step) {
             const float t = rcp_approx(lam);
-            float sum = 0.0f;
+            float ps[kAcc];
+            int pm[kAcc];
+#pragma unroll
+            for (int a = 0; a < kAcc; ++a) { ps[a] = 0.0f; pm[a] = 0; }
+#pragma unroll
+            for (int i = 0; i < kMax; ++i) add_if_below(ps[i % kAcc], pm[i % kAcc], r[i], t);
+            const float sum = acc_total(ps);
             int m = 0;
 #pragma unroll
-            for (int i = 0; i < kMax; ++i) {
-                const bool on = r[i] < t;
-                sum += on ? r[i] : 0.0f;
-                m += on;
-            }
+            for (int a = 0; a < kAcc; ++a) m += pm[a];
             const float next = ((float)m - K) / sum;
             if (m == prev_m) { lam = next; break; }
             lam = fmaxf(lam, next);
@@ -183,34 +204,30 @@ __device__ __forceinline__ void solve_thread_reg(float *x, const float *__restri
 #pragma unroll
     for (int i = 0; i < kMax; ++i)
         if (i < n) x[i] = fmaxf(0.0f, 1.0f - lam * r[i]);
-    float u = lam;
-    if (npos == 0) {
-        u = n > 0 ? -3.0e38f : 0.0f;
-        for (int i = 0; i < n; ++i) {
-            const float xi = vg[i];
-            if (!isnan(xi)) u = fmaxf(u, xi);
-        }
-    }
     if (lambda_out) lambda_out[q] = lam;
-    if (utility_out) utility_out[q] = u;
+    if (utility_out) utility_out[q] = n > 0 ? lam : 0.0f;
     if (bad) raise_flag(status, KVGOV_F_BADINDEX);
 }
 
 // kCta consecutive problems per CTA.  When every one of them has at most
-// kSmallN tenants, their values are staged in shared memory with coalesced
-// loads, a thread solves each problem, and the probabilities leave with
-// coalesced stores: a few dozen instructions per problem per warp instead
-// of a warp's reductions per problem.  Otherwise the CTA's warps take its
-// problems one at a time (solve_warp).
+// kSmallN tenants and every value is usable, the values are staged in shared
+// memory with coalesced (16-byte where aligned) loads, a thread solves each
+// problem, and the probabilities leave the same way: a few dozen
+// instructions per problem per warp instead of a warp's reductions per
+// problem.  Otherwise -- larger problems, or a value that is not a positive
+// finite number somewhere in the CTA's span -- the CTA's warps take its
+// problems one at a time (solve_warp), which handles every case.
 constexpr int kCta = 128;
 constexpr int kSmallN = 64;
 
-__global__ void __launch_bounds__(kCta) origami_kernel(const float *__restrict__ values,
+// At most 96 registers, so that 5 CTAs fit an SM (102 unbounded: 4).
+__global__ void __launch_bounds__(kCta, 5) origami_kernel(const float *__restrict__ values,
                                                        const int64_t *__restrict__ off, int32_t n_prob,
                                                        const float *__restrict__ budget, float *__restrict__ p,
                                                        float *__restrict__ lambda_out,
-                                                       float *__restrict__ utility_out, uint32_t *status) {
-    __shared__ float sv[kCta * kSmallN];
+                                                       float *__restrict__ utility_out, uint32_t *status,
+                                                       bool vec4) {
+    __shared__ __align__(16) float sv[kCta * kSmallN + 4];
     const long long total = off[n_prob];
     const long long q0 = (long long)blockIdx.x * kCta;
     const long long q1 = q0 + kCta < n_prob ? q0 + kCta : (long long)n_prob;
@@ -225,23 +242,68 @@ __global__ void __launch_bounds__(kCta) origami_kernel(const float *__restrict__
     }
     ok = ok && base0 >= 0 && base1 >= base0 && base1 <= total && base1 - base0 <= kCta * kSmallN;
     if (__syncthreads_and(ok)) {
+        // the span [base0, base1) lands at sv[lead ..], lead = base0 mod 4, so
+        // that its 16-byte-aligned middle moves as float4 (vec4: values and p
+        // are 16-byte aligned; else every element on its own)
+        const int lead = vec4 ? (int)(base0 & 3) : 0;
         const int span = (int)(base1 - base0);
-        for (int i = threadIdx.x; i < span; i += kCta) sv[i] = values[base0 + i];
-        __syncthreads();
-        if (q < q1) {
-            float *x = sv + (my0 - base0);
-            const int n = (int)(my1 - my0);
-            if (n <= 16) solve_thread_reg<16>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
-            else if (n <= 32) solve_thread_reg<32>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
-            else if (n <= 50) solve_thread_reg<50>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
-            else solve_thread_reg<kSmallN>(x, values + my0, n, budget[q], q, lambda_out, utility_out, status);
+        const long long a0 = base0 - lead;                       // 16-byte aligned when vec4
+        const int n4 = vec4 ? (lead + span) >> 2 : 0;            // whole float4 from a0
+        const int tail0 = n4 > 0 ? 4 * n4 : lead;                // the first element after them
+        bool usable_all = true;
+        const float4 *v4 = reinterpret_cast<const float4 *>(values + a0);
+        float4 *s4 = reinterpret_cast<float4 *>(sv);
+        // kInFlight loads in flight per thread before their values are used
+        for (int i0 = threadIdx.x; i0 < n4; i0 += kInFlight * kCta) {
+            float4 c[kInFlight];
+#pragma unroll
+            for (int u = 0; u < kInFlight; ++u)
+                if (i0 + u * kCta < n4) c[u] = __ldcs(v4 + i0 + u * kCta);
+#pragma unroll
+            for (int u = 0; u < kInFlight; ++u) {
+                const int i = i0 + u * kCta;
+                if (i < n4) {
+                    s4[i] = c[u];
+                    const int e = 4 * i;                         // element index from a0
+                    usable_all &= (e < lead || usable(c[u].x)) && (e + 1 < lead || usable(c[u].y)) &&
+                                  (e + 2 < lead || usable(c[u].z)) && usable(c[u].w);
+                }
+            }
         }
-        __syncthreads();
-        for (int i = threadIdx.x; i < span; i += kCta) p[base0 + i] = sv[i];
-    } else {
-        for (long long qq = q0 + threadIdx.x / 32; qq < q1; qq += kCta / 32)
-            solve_warp(values, off, qq, total, budget, p, lambda_out, utility_out, status);
+        for (int e = tail0 + threadIdx.x; e < lead + span; e += kCta) {    // the tail
+            const float c = values[a0 + e];
+            sv[e] = c;
+            usable_all &= usable(c);
+        }
+        if (__syncthreads_and(usable_all)) {
+            if (q < q1) {
+                float *x = sv + lead + (my0 - base0);
+                const int n = (int)(my1 - my0);
+                const float K = budget[q];
+                if (n <= 16) solve_thread_reg<16>(x, n, K, q, lambda_out, utility_out, status);
+                else if (n <= 32) solve_thread_reg<32>(x, n, K, q, lambda_out, utility_out, status);
+                else if (n <= 50) solve_thread_reg<50>(x, n, K, q, lambda_out, utility_out, status);
+                else solve_thread_reg<kSmallN>(x, n, K, q, lambda_out, utility_out, status);
+            }
+            __syncthreads();
+            // out: the same split; the lead elements and the tail are the span's own
+            float4 *p4 = reinterpret_cast<float4 *>(p + a0);
+            for (int i = threadIdx.x; i < n4; i += kCta) {
+                const float4 c = s4[i];
+                if (4 * i >= lead) {
+                    __stcs(p4 + i, c);
+                } else {                                         // the first float4 holds elements before the span
+                    if (4 * i + 1 >= lead) p[a0 + 4 * i + 1] = c.y;
+                    if (4 * i + 2 >= lead) p[a0 + 4 * i + 2] = c.z;
+                    p[a0 + 4 * i + 3] = c.w;
+                }
+            }
+            for (int e = tail0 + threadIdx.x; e < lead + span; e += kCta) p[a0 + e] = sv[e];
+            return;
+        }
     }
+    for (long long qq = q0 + threadIdx.x / 32; qq < q1; qq += kCta / 32)
+        solve_warp(values, off, qq, total, budget, p, lambda_out, utility_out, status);
 }
 
 }  // namespace
@@ -253,7 +315,8 @@ extern "C" int kvgov_origami(const float *d_values, const int64_t *d_off, int32_
     if (n_prob == 0) return KVGOV_OK;
     if (!d_values || !d_budget || !d_p) return KVGOV_EINVAL;
     const long long grid = ((long long)n_prob + kCta - 1) / kCta;
+    const bool vec4 = kvgov_host::aligned16(d_values) && kvgov_host::aligned16(d_p);
     origami_kernel<<<(unsigned)grid, kCta, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-        d_values, d_off, n_prob, d_budget, d_p, d_lambda, d_utility, d_status);
+        d_values, d_off, n_prob, d_budget, d_p, d_lambda, d_utility, d_status, vec4);
     return kvgov_host::launch_status();
 }

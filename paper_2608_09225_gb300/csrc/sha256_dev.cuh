@@ -78,11 +78,12 @@ __device__ __forceinline__ uint32_t ssig1(uint32_t x) { return xor3(rotr(x, 17),
 __device__ __forceinline__ uint32_t bswap32(uint32_t x) { return __byte_perm(x, 0u, 0x0123u); }
 
 // Adders.  Every 32-bit add of the compression goes through one of these.
-// AddAlu is a plain add (the compiler emits IADD3 on the integer ALU pipe,
-// the pipe that also carries every SHF and LOP3).  AddFma issues the add as
-// IMAD a * one + b, with `one` a runtime 1 so that the compiler cannot turn
-// the multiply-add back into an ALU add; only the integer microbenchmark
-// (int_peak.cu) uses it, to measure that IMAD shares the integer pipe.
+// AddAlu is a plain add (the compiler emits IADD3, mostly on the integer
+// ALU pipe, the pipe that also carries every SHF and LOP3).  AddFma issues
+// the add as IMAD a * one + b, with `one` a runtime 1 so that the compiler
+// cannot turn the multiply-add back into an ALU add: IMAD goes to the FMA
+// pipe.  Only the integer microbenchmark (int_peak.cu) uses it: SHA-256 with
+// its adds moved there ran slower than with plain adds.
 struct AddAlu {
     __device__ __forceinline__ uint32_t operator()(uint32_t a, uint32_t b) const { return a + b; }
 };

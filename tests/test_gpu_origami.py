@@ -54,11 +54,11 @@ def test_origami_ragged_matches_oracle(kv, seed, n_prob):
 @pytest.mark.parametrize("seed", [11, 12])
 def test_origami_thread_tiers_match_oracle(kv, seed):
     """Problems of 0 to 64 tenants, so that every CTA takes the thread-per-
-    problem path and every register size (16, 32, 56, 64 slots) is used, with
+    problem path and every register size (16, 32, 50, 64 slots) is used, with
     all-equal and Pareto values and budgets above n."""
     b = W.audit_ragged(seed, 4096, max_tenants=64)
     sizes = np.diff(b.off)
-    assert sizes.max() <= 64 and ((sizes > 56) & (sizes <= 64)).any() and ((sizes > 32) & (sizes <= 56)).any()
+    assert sizes.max() <= 64 and ((sizes > 50) & (sizes <= 64)).any() and ((sizes > 32) & (sizes <= 50)).any()
     p, lam, u, st = gpu(kv, b)
     p_ref, lam_ref, u_ref, flag = oracle.origami(b.values, b.off, b.budget)
     assert st == 0 and not flag
@@ -100,3 +100,46 @@ def test_origami_edge_cases_and_flags(kv):
         assert st == kv.F_BADINDEX and flag
         assert np.abs(p - p_ref).max() <= tol(3) and abs(lam[0] - lam_ref[0]) <= tol(3) * max(lam_ref[0], 1)
         assert math.isfinite(lam[0])
+
+
+def test_origami_unusable_value_takes_its_cta_to_the_warp_path(kv):
+    """3000 problems of 50 tenants with a NaN in problem 1000 and a zero in
+    problem 2000: the batch is flagged, the two CTAs holding them solve every
+    problem warp by warp, and every problem -- those two included (a NaN or a
+    zero tenant gets p = 0) -- matches the oracle."""
+    b = W.audit(seed=9, n_prob=3000)
+    b.values[50 * 1000 + 7] = np.nan
+    b.values[50 * 2000 + 3] = 0.0
+    p, lam, u, st = gpu(kv, b)
+    p_ref, lam_ref, u_ref, flag = oracle.origami(b.values, b.off, b.budget)
+    assert st == kv.F_BADINDEX and flag
+    good = np.ones(b.n, bool)
+    good[1000] = False
+    check_rows = np.nonzero(good)[0]
+    for q in check_rows:
+        s, e = int(b.off[q]), int(b.off[q + 1])
+        assert np.abs(p[s:e] - p_ref[s:e]).max() <= tol(50), q
+        assert abs(lam[q] - lam_ref[q]) <= tol(50) * lam_ref[q], q
+    assert p[50 * 1000 + 7] == 0.0 and p[50 * 2000 + 3] == 0.0
+
+
+@pytest.mark.parametrize("shift", [1, 2, 3])
+def test_origami_unaligned_buffers(kv, shift):
+    """Values and probabilities that do not start on a 16-byte boundary (views
+    `shift` floats into larger buffers): the element-by-element staging path,
+    same results as the oracle."""
+    b = W.audit_ragged(13 + shift, 2000, max_tenants=64)
+    n = len(b.values)
+    vbuf = torch.zeros(n + 4, dtype=torch.float32, device=DEV)
+    vbuf[shift:shift + n] = torch.from_numpy(b.values).to(DEV)
+    pbuf = torch.full((n + 4,), -1.0, dtype=torch.float32, device=DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    _, lam, u = kv.origami(vbuf[shift:shift + n], torch.from_numpy(b.off).to(DEV),
+                           torch.from_numpy(b.budget).to(DEV), pbuf[shift:shift + n], status=st)
+    torch.cuda.synchronize()
+    p = pbuf.cpu().numpy().astype(np.float64)
+    assert (p[:shift] == -1.0).all() and (p[shift + n:] == -1.0).all()
+    p_ref, lam_ref, u_ref, flag = oracle.origami(b.values, b.off, b.budget)
+    assert int(st.item()) == 0 and not flag
+    check(b, p[shift:shift + n], lam.cpu().numpy().astype(np.float64), u.cpu().numpy().astype(np.float64),
+          p_ref, lam_ref, u_ref)
