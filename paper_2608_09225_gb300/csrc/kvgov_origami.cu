@@ -16,6 +16,7 @@
 // every other step, so there are at most (number of tenants + 1) steps.  The
 // paper finds lambda by bisection; this reaches the same level without an
 // iteration count that sets the precision.
+#include <atomic>
 #include <cmath>
 
 #include "kvgov_internal.cuh"
@@ -41,17 +42,14 @@ __device__ __forceinline__ int warp_isum(int v) { return __reduce_add_sync(0xfff
 // audit (no payoff to protect), NaN or infinity is flagged and gets none.
 __device__ __forceinline__ bool usable(float v) { return v > 0.0f && v <= 3.0e38f; }
 
-// One problem solved by the 32 lanes of a warp (any number of tenants).
-__device__ __forceinline__ void solve_warp(const float *__restrict__ values, const int64_t *__restrict__ off,
-                                           long long q, long long total, const float *__restrict__ budget,
-                                           float *__restrict__ p, float *__restrict__ lambda_out,
-                                           float *__restrict__ utility_out, uint32_t *status) {
+// One problem solved by the 32 lanes of a warp (any number of tenants): its
+// n values v[0..n) and budget K_in; p_i goes to pout[i], which may be v
+// itself (each lane reads a value before it writes that place).  `bad`
+// flags the problem as malformed already.
+__device__ __forceinline__ void solve_warp_core(const float *v, float *pout, long long n, float K_in, bool bad,
+                                                long long q, float *__restrict__ lambda_out,
+                                                float *__restrict__ utility_out, uint32_t *status) {
     const int lane = threadIdx.x & 31;
-    const long long b0 = off[q], b1 = off[q + 1];
-    bool bad = b0 < 0 || b1 < b0 || b1 > total;
-    const long long n = bad ? 0 : b1 - b0;
-    const float *v = values + (bad ? 0 : b0);
-
     // usable tenants, largest value, values that are not numbers
     int my_pos = 0, my_bad = 0;
     float my_max = 0.0f;
@@ -62,7 +60,7 @@ __device__ __forceinline__ void solve_warp(const float *__restrict__ values, con
     }
     const int npos = warp_isum(my_pos);
     const float vmax = warp_max(my_max);
-    float K = budget[q];
+    float K = K_in;
     if (warp_isum(my_bad) > 0 || !(K >= 0.0f)) bad = true;
     if (!(K >= 0.0f)) K = 0.0f;
     if (K > (float)npos) K = (float)npos;
@@ -98,7 +96,7 @@ __device__ __forceinline__ void solve_warp(const float *__restrict__ values, con
     for (long long i = lane; i < n; i += 32) {
         const float x = v[i];
         const float pi = usable(x) ? fmaxf(0.0f, 1.0f - lam / x) : 0.0f;
-        p[b0 + i] = pi;
+        pout[i] = pi;
         if (!isnan(x)) my_u = fmaxf(my_u, usable(x) ? fminf(x, lam) : x);
     }
     const float u = warp_max(my_u);
@@ -107,6 +105,18 @@ __device__ __forceinline__ void solve_warp(const float *__restrict__ values, con
         if (utility_out) utility_out[q] = n > 0 ? u : 0.0f;
         if (bad) raise_flag(status, KVGOV_F_BADINDEX);
     }
+}
+
+// Problem q, its values and probabilities in global memory.
+__device__ __forceinline__ void solve_warp(const float *__restrict__ values, const int64_t *__restrict__ off,
+                                           long long q, long long total, const float *__restrict__ budget,
+                                           float *__restrict__ p, float *__restrict__ lambda_out,
+                                           float *__restrict__ utility_out, uint32_t *status) {
+    const long long b0 = off[q], b1 = off[q + 1];
+    const bool bad = b0 < 0 || b1 < b0 || b1 > total;
+    const long long n = bad ? 0 : b1 - b0;
+    const long long at = bad ? 0 : b0;
+    solve_warp_core(values + at, p + at, n, budget[q], bad, q, lambda_out, utility_out, status);
 }
 
 // Reciprocal with the SFU's one-instruction approximation (relative error
@@ -154,20 +164,28 @@ __device__ __forceinline__ void add_if_below(float &sum, int &m, float r, float 
 // Register tiers of 16, 32, 50 (the paper's 50-tenant problems, section
 // 5.5) and 64 slots.  The adversary's payoff is lambda (some tenant is
 // usable whenever n > 0).
-template <int kMax>
-__device__ __forceinline__ void solve_thread_reg(float *x, int n, float K_in, long long q,
+// CHECK: the values were not checked; the solver returns false, writing
+// nothing, when one is not usable (r = 1 / v not positive and finite: v <= 0,
+// NaN, infinite, or above 2^126, whose reciprocal is not a normal number;
+// the warp solver takes those).
+template <int kMax, bool CHECK = false>
+__device__ __forceinline__ bool solve_thread_reg(float *x, int n, float K_in, long long q,
                                                  float *__restrict__ lambda_out, float *__restrict__ utility_out,
                                                  uint32_t *status) {
     float r[kMax];
     float part[kAcc];                                  // kAcc partial sums: independent add chains
+    float rmin = __int_as_float(0x7f800000);
 #pragma unroll
     for (int a = 0; a < kAcc; ++a) part[a] = 0.0f;
 #pragma unroll
     for (int i = 0; i < kMax; ++i) {
         r[i] = i < n ? rcp_approx(x[i]) : __int_as_float(0x7f800000);
         if (i < n) part[i % kAcc] += r[i];
+        if (CHECK) rmin = fminf(rmin, r[i]);
     }
     const float sum_all = acc_total(part);
+    // a NaN or +infinity reciprocal makes the sum NaN or infinite
+    if (CHECK && !(rmin > 0.0f && sum_all <= 3.0e38f)) return false;
     float K = K_in;
     const bool bad = !(K >= 0.0f);
     if (!(K >= 0.0f)) K = 0.0f;
@@ -207,6 +225,7 @@ __device__ __forceinline__ void solve_thread_reg(float *x, int n, float K_in, lo
     if (lambda_out) lambda_out[q] = lam;
     if (utility_out) utility_out[q] = n > 0 ? lam : 0.0f;
     if (bad) raise_flag(status, KVGOV_F_BADINDEX);
+    return true;
 }
 
 // kCta consecutive problems per CTA.  When every one of them has at most
@@ -306,6 +325,260 @@ __global__ void __launch_bounds__(kCta, 5) origami_kernel(const float *__restric
         solve_warp(values, off, qq, total, budget, p, lambda_out, utility_out, status);
 }
 
+// ---------------------------------------------------------------------------
+// Streaming layout, for values and p on 16-byte boundaries: a persistent CTA
+// per resident slot walks the batch's tiles (kCta problems each) with two
+// shared-memory buffers.  The copy engine brings tile t + G into one buffer
+// -- one bulk copy of the tile's span, rounded out to 16-byte bounds,
+// completing on the buffer's mbarrier -- while the CTA solves tile t in the
+// other, in place, and the probabilities leave by one bulk store, so that
+// no warp waits for a global load or store of values and the copies of some
+// tiles overlap the solves of others (origami_kernel above, 5 CTAs per SM,
+// each staging, solving and storing in turn, left its SMs idle while the
+// resident CTAs staged).  A thread solves its problem in registers
+// (solve_thread_reg, values checked as it goes); a problem it cannot take
+// (a value that is not usable, more than kSmallN tenants, malformed offsets)
+// goes on a list that the CTA's warps solve after, in place in the buffer;
+// a tile whose span does not fit a buffer is solved warp by warp from
+// global memory.
+
+constexpr int kBuf = kCta * kSmallN + 8;          // floats per buffer: a tile's span rounded out to 16 bytes
+constexpr uint32_t kBulkWaitLimit = 1u << 24;     // polls of a buffer's mbarrier before KVGOV_F_TIMEOUT
+constexpr size_t kStreamSmem = 2 * kBuf * sizeof(float);
+
+__device__ __forceinline__ uint32_t smem_u32(const void *ptr) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(ptr));
+}
+__device__ __forceinline__ void mbar_init(unsigned long long *bar) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(bar)) : "memory");
+}
+// one arrival (the issuing thread's) and the bytes the bulk copy will deliver
+__device__ __forceinline__ void mbar_arrive_tx(unsigned long long *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_done(unsigned long long *bar, uint32_t parity) {
+    uint32_t done;
+    asm volatile("{\n\t.reg .pred p;\n\t"
+                 "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+                 "selp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(done)
+                 : "r"(smem_u32(bar)), "r"(parity)
+                 : "memory");
+    return done != 0;
+}
+// Wait for the phase of the given parity to complete, at most kBulkWaitLimit
+// polls; false if it did not.
+__device__ bool mbar_wait(unsigned long long *bar, uint32_t parity) {
+    for (uint32_t i = 0; i < kBulkWaitLimit; ++i) {
+        if (mbar_done(bar, parity)) return true;
+        if (i >= 32) __nanosleep(64);
+    }
+    return false;
+}
+__device__ __forceinline__ void bulk_load(float *dst, const float *src, uint32_t bytes, unsigned long long *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_store(float *dst, const float *src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(smem_u32(src)),
+                 "r"(bytes)
+                 : "memory");
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// the issuing thread's bulk stores have read their shared-memory source
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// ... and are complete
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// this thread's shared-memory writes, ordered before the bulk copies that follow
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__device__ __forceinline__ long long round_down4(long long e) { return e & ~3ll; }
+__device__ __forceinline__ long long round_up4(long long e) { return (e + 3) & ~3ll; }
+
+__global__ void __launch_bounds__(kCta, 3) origami_stream_kernel(const float *__restrict__ values,
+                                                              const int64_t *__restrict__ off, int32_t n_prob,
+                                                              const float *__restrict__ budget,
+                                                              float *__restrict__ p, float *__restrict__ lambda_out,
+                                                              float *__restrict__ utility_out, uint32_t *status) {
+    extern __shared__ __align__(16) float dyn[];
+    __shared__ unsigned long long s_bar[2];
+    __shared__ long long s_b0[2], s_b1[2];        // the span of the tile in each buffer
+    __shared__ int s_fits[2];                     // ... and whether it fits the buffer
+    __shared__ int s_def[kCta], s_ndef;           // problems left to the warps
+
+    const int tid = threadIdx.x;
+    const long long total = off[n_prob];
+    const long long n_tiles = ((long long)n_prob + kCta - 1) / kCta;
+    const long long G = gridDim.x;
+    const long long t_first = blockIdx.x;
+    if (t_first >= n_tiles) return;
+
+    // Thread 0: the copy of tile t (span [b0, b1), offsets already read)
+    // into buffer b.  Elements from round_down4(b0) land at the buffer's
+    // start; at the array's end the last < 4 values come by plain loads.
+    auto issue = [&](long long t, int b, long long b0, long long b1) {
+        const bool fits = b0 >= 0 && b1 >= b0 && b1 <= total && b1 - b0 <= (long long)kCta * kSmallN;
+        float *buf = dyn + b * kBuf;
+        uint32_t bytes = 0;
+        long long a0 = 0, a1 = 0;
+        if (fits) {
+            a0 = round_down4(b0);
+            a1 = round_up4(b1) <= total ? round_up4(b1) : round_down4(b1);
+            if (a1 > a0) bytes = (uint32_t)(4 * (a1 - a0));
+        }
+        s_b0[b] = b0;
+        s_b1[b] = b1;
+        s_fits[b] = fits;
+        mbar_arrive_tx(&s_bar[b], bytes);
+        if (bytes) bulk_load(buf, values + a0, bytes, &s_bar[b]);
+        if (fits)
+            for (long long e = a1 > b0 ? a1 : b0; e < b1; ++e) buf[e - a0] = values[e];
+    };
+
+    // tile t's problem for this thread, read one tile ahead
+    auto read_mine = [&](long long t, long long &m0, long long &m1, float &K) {
+        const long long q = t * kCta + tid;
+        m0 = m1 = 0;
+        K = 0.0f;
+        if (t < n_tiles && q < n_prob) {
+            m0 = off[q];
+            m1 = off[q + 1];
+            K = budget[q];
+        }
+    };
+    // thread 0: tile t's span, read one tile ahead of its copy
+    auto read_span = [&](long long t, long long &b0, long long &b1) {
+        b0 = b1 = 0;
+        if (t < n_tiles) {
+            const long long q0 = t * kCta, q1 = q0 + kCta < n_prob ? q0 + kCta : (long long)n_prob;
+            b0 = off[q0];
+            b1 = off[q1];
+        }
+    };
+
+    long long nb0 = 0, nb1 = 0;                   // thread 0: the span of the tile to issue next
+    if (tid == 0) {
+        mbar_init(&s_bar[0]);
+        mbar_init(&s_bar[1]);
+        s_ndef = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");   // before the copies use them
+        long long b0, b1;
+        read_span(t_first, b0, b1);
+        issue(t_first, 0, b0, b1);
+        read_span(t_first + G, nb0, nb1);
+    }
+    long long m0, m1;
+    float K;
+    read_mine(t_first, m0, m1, K);
+    __syncthreads();
+
+    uint32_t parity[2] = {0u, 0u};
+    bool aborted = false;
+    int b = 0;
+    for (long long t = t_first; t < n_tiles; t += G, b ^= 1) {
+        // the next tile into the other buffer, once its last store has read it
+        if (tid == 0 && t + G < n_tiles) {
+            bulk_wait_read();
+            issue(t + G, b ^ 1, nb0, nb1);
+            read_span(t + 2 * G, nb0, nb1);
+        }
+        const bool arrived = mbar_wait(&s_bar[b], parity[b]);
+        if (__syncthreads_or(!arrived)) {         // the copy never completed: stop (the tile's data is not there)
+            if (tid == 0) raise_flag(status, KVGOV_F_TIMEOUT);
+            aborted = true;
+            break;
+        }
+        parity[b] ^= 1u;
+        const long long b0 = s_b0[b], b1 = s_b1[b];
+        const bool fits = s_fits[b] != 0;
+        const long long q = t * kCta + tid;
+        const long long q1 = t * kCta + kCta < n_prob ? t * kCta + kCta : (long long)n_prob;
+        long long nm0, nm1;                       // this thread's problem of the next tile
+        float nK;
+        read_mine(t + G, nm0, nm1, nK);
+        float *buf = dyn + b * kBuf;
+        const long long a0 = round_down4(b0);
+        if (fits) {
+            if (q < q1) {
+                const bool ok = m0 >= b0 && m1 >= m0 && m1 <= b1 && m1 - m0 <= kSmallN;
+                const int n = ok ? (int)(m1 - m0) : 0;
+                float *x = buf + (m0 - a0);
+                bool done = false;
+                if (ok) {
+                    if (n <= 16) done = solve_thread_reg<16, true>(x, n, K, q, lambda_out, utility_out, status);
+                    else if (n <= 32) done = solve_thread_reg<32, true>(x, n, K, q, lambda_out, utility_out, status);
+                    else if (n <= 50) done = solve_thread_reg<50, true>(x, n, K, q, lambda_out, utility_out, status);
+                    else done = solve_thread_reg<kSmallN, true>(x, n, K, q, lambda_out, utility_out, status);
+                }
+                if (!done) s_def[atomicAdd(&s_ndef, 1)] = tid;
+            }
+            fence_async_smem();
+            __syncthreads();
+            const int ndef = s_ndef;
+            if (ndef > 0) {                       // the warps take the problems left to them, in place
+                for (int k = tid / 32; k < ndef; k += kCta / 32) {
+                    const int d = s_def[k];
+                    const long long dq = t * kCta + d;
+                    const long long d0 = off[dq], d1 = off[dq + 1];
+                    const bool inside = d0 >= b0 && d1 >= d0 && d1 <= b1;
+                    if (inside)
+                        solve_warp_core(buf + (d0 - a0), buf + (d0 - a0), d1 - d0, budget[dq], false, dq, lambda_out,
+                                        utility_out, status);
+                    else
+                        solve_warp(values, off, dq, total, budget, p, lambda_out, utility_out, status);
+                }
+                fence_async_smem();
+                __syncthreads();
+                if (tid == 0) s_ndef = 0;
+            }
+            if (tid == 0) {                       // [b0, b1) out: its 16-byte-aligned middle in one bulk store
+                const long long c0 = round_up4(b0) < b1 ? round_up4(b0) : b1;
+                const long long c1 = round_down4(b1) > c0 ? round_down4(b1) : c0;
+                for (long long e = b0; e < c0; ++e) p[e] = buf[e - a0];
+                for (long long e = c1; e < b1; ++e) p[e] = buf[e - a0];
+                if (c1 > c0) bulk_store(p + c0, buf + (c0 - a0), (uint32_t)(4 * (c1 - c0)));
+            }
+        } else {
+            for (long long qq = t * kCta + tid / 32; qq < q1; qq += kCta / 32)
+                solve_warp(values, off, qq, total, budget, p, lambda_out, utility_out, status);
+        }
+        __syncthreads();                          // buffer b's next copy may go once its store has read it
+        m0 = nm0;
+        m1 = nm1;
+        K = nK;
+    }
+    if (tid == 0) {
+        bulk_wait_all();
+        if (aborted)                              // copies that may still be under way into either buffer
+            for (int k = 0; k < 2; ++k) mbar_wait(&s_bar[k], parity[k]);
+    }
+}
+
+// CTAs of origami_stream_kernel resident at once on the current device
+// (its shared memory set up), looked up once per device; 0 if it cannot run.
+int stream_ctas() {
+    static std::atomic<int> cache[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    int v = cache[dev].load(std::memory_order_relaxed);
+    if (v == 0) {
+        int per_sm = 0, sms = 0;
+        if (cudaFuncSetAttribute(origami_stream_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kStreamSmem) != cudaSuccess ||
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, origami_stream_kernel, kCta, kStreamSmem) !=
+                cudaSuccess ||
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+            cudaGetLastError();
+            return 0;
+        }
+        v = per_sm > 0 ? per_sm * sms : -1;
+        cache[dev].store(v, std::memory_order_relaxed);
+    }
+    return v > 0 ? v : 0;
+}
+
 }  // namespace
 
 extern "C" int kvgov_origami(const float *d_values, const int64_t *d_off, int32_t n_prob, const float *d_budget,
@@ -316,7 +589,14 @@ extern "C" int kvgov_origami(const float *d_values, const int64_t *d_off, int32_
     if (!d_values || !d_budget || !d_p) return KVGOV_EINVAL;
     const long long grid = ((long long)n_prob + kCta - 1) / kCta;
     const bool vec4 = kvgov_host::aligned16(d_values) && kvgov_host::aligned16(d_p);
-    origami_kernel<<<(unsigned)grid, kCta, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-        d_values, d_off, n_prob, d_budget, d_p, d_lambda, d_utility, d_status, vec4);
+    const int resident = vec4 ? stream_ctas() : 0;
+    if (resident > 0) {
+        const long long g = grid < resident ? grid : resident;
+        origami_stream_kernel<<<(unsigned)g, kCta, kStreamSmem, reinterpret_cast<cudaStream_t>(stream)>>>(
+            d_values, d_off, n_prob, d_budget, d_p, d_lambda, d_utility, d_status);
+    } else {
+        origami_kernel<<<(unsigned)grid, kCta, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+            d_values, d_off, n_prob, d_budget, d_p, d_lambda, d_utility, d_status, vec4);
+    }
     return kvgov_host::launch_status();
 }
