@@ -57,8 +57,8 @@ CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain k
 # step's chain kernel from one ncu capture, and the SHA-256 (chain_source_hash)
 # of the sources it was captured from: reported as roofline.traffic only while
 # the kernel's sources still hash to that value.
-CHAIN_TRAFFIC = {"bytes_per_launch": 180052992,
-                 "source_sha256": "0ac246e51adf4874a4d8d7397d19b87432078edfbd38d70fadbfeca2e862d11c"}
+CHAIN_TRAFFIC = {"bytes_per_launch": 179202176,
+                 "source_sha256": "c381000fdcff49648dcde1a6b7f284c9e18ba37224732e2f548562a3d19b61fe"}
 
 
 # DRAM bytes per launch of the probe on the probe-heavy workload from one ncu
@@ -67,7 +67,7 @@ TABLE_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_table.cu", "paper_2608_09225
                  "paper_2608_09225_gb300/csrc/kvgov_stash.cuh", "paper_2608_09225_gb300/csrc/kvgov_internal.cuh",
                  "paper_2608_09225_gb300/csrc/kvgov_insert.cuh"]
 TABLE_TRAFFIC = {"probe_share_kernel<16, true>": {
-    "bytes_per_launch": 70829952, "source_sha256": "a783b5d825a97b2b42927d934ff1e644cb3aa3f343ee86860371c75c0a660472"}}
+    "bytes_per_launch": 74625536, "source_sha256": "bf0b4ece69c570d320a286d9ead7225b89e2d3d5c627f682edbce8f44016b5fe"}}
 
 
 def load_peaks() -> dict:

@@ -326,25 +326,27 @@ __global__ void __launch_bounds__(kCta, 5) origami_kernel(const float *__restric
 }
 
 // ---------------------------------------------------------------------------
-// Streaming layout, for values and p on 16-byte boundaries: a persistent CTA
-// per resident slot walks the batch's tiles (kCta problems each) with two
-// shared-memory buffers.  The copy engine brings tile t + G into one buffer
-// -- one bulk copy of the tile's span, rounded out to 16-byte bounds,
-// completing on the buffer's mbarrier -- while the CTA solves tile t in the
-// other, in place, and the probabilities leave by one bulk store, so that
-// no warp waits for a global load or store of values and the copies of some
-// tiles overlap the solves of others (origami_kernel above, 5 CTAs per SM,
-// each staging, solving and storing in turn, left its SMs idle while the
-// resident CTAs staged).  A thread solves its problem in registers
-// (solve_thread_reg, values checked as it goes); a problem it cannot take
-// (a value that is not usable, more than kSmallN tenants, malformed offsets)
-// goes on a list that the CTA's warps solve after, in place in the buffer;
-// a tile whose span does not fit a buffer is solved warp by warp from
-// global memory.
+// Streaming layout, for values and p on 16-byte boundaries: every warp of a
+// persistent grid (3 CTAs of 4 warps per SM) walks the batch's warp tiles
+// (32 problems each) on its own, with two shared-memory buffers.  The copy
+// engine brings the warp's tile t + W into one buffer -- one bulk copy of
+// the tile's span, rounded out to 16-byte bounds, completing on the
+// buffer's mbarrier -- while the warp solves tile t in the other, in place,
+// and the probabilities leave by one bulk store.  No warp waits for a global
+// load or store of values, nor for another warp (a CTA-wide barrier per
+// tile left warps waiting for the CTA's slowest Newton solve: 1.46 barrier
+// stalls per issue), and the copies of some tiles overlap the solves of
+// others.  A lane solves its problem in registers (solve_thread_reg, values
+// checked as it goes); a problem it cannot take (a value that is not usable,
+// more than kSmallN tenants, malformed offsets) is solved after by the whole
+// warp, in place in the buffer; a tile whose span does not fit a buffer is
+// solved warp-wide from global memory.
 
-constexpr int kBuf = kCta * kSmallN + 8;          // floats per buffer: a tile's span rounded out to 16 bytes
+constexpr int kTile = 32;                         // problems per warp tile
+constexpr int kBuf = kTile * kSmallN + 8;         // floats per buffer: a tile's span rounded out to 16 bytes
+constexpr int kStreamWarps = kCta / 32;
 constexpr uint32_t kBulkWaitLimit = 1u << 24;     // polls of a buffer's mbarrier before KVGOV_F_TIMEOUT
-constexpr size_t kStreamSmem = 2 * kBuf * sizeof(float);
+constexpr size_t kStreamSmem = 2 * kStreamWarps * kBuf * sizeof(float);
 
 __device__ __forceinline__ uint32_t smem_u32(const void *ptr) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(ptr));
@@ -403,24 +405,24 @@ __global__ void __launch_bounds__(kCta, 3) origami_stream_kernel(const float *__
                                                               float *__restrict__ p, float *__restrict__ lambda_out,
                                                               float *__restrict__ utility_out, uint32_t *status) {
     extern __shared__ __align__(16) float dyn[];
-    __shared__ unsigned long long s_bar[2];
-    __shared__ long long s_b0[2], s_b1[2];        // the span of the tile in each buffer
-    __shared__ int s_fits[2];                     // ... and whether it fits the buffer
-    __shared__ int s_def[kCta], s_ndef;           // problems left to the warps
+    __shared__ unsigned long long s_bar[kStreamWarps][2];
+    __shared__ long long s_b0[kStreamWarps][2], s_b1[kStreamWarps][2];   // the span of the tile in each buffer
+    __shared__ int s_fits[kStreamWarps][2];                              // ... and whether it fits the buffer
 
-    const int tid = threadIdx.x;
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     const long long total = off[n_prob];
-    const long long n_tiles = ((long long)n_prob + kCta - 1) / kCta;
-    const long long G = gridDim.x;
-    const long long t_first = blockIdx.x;
-    if (t_first >= n_tiles) return;
+    const long long n_tiles = ((long long)n_prob + kTile - 1) / kTile;
+    const long long W = (long long)gridDim.x * kStreamWarps;            // warps in the grid
+    const long long t_first = (long long)blockIdx.x * kStreamWarps + w;
+    if (t_first >= n_tiles) return;               // this warp has no tile (no CTA-wide barrier follows)
+    float *const bufs = dyn + w * 2 * kBuf;
 
-    // Thread 0: the copy of tile t (span [b0, b1), offsets already read)
-    // into buffer b.  Elements from round_down4(b0) land at the buffer's
-    // start; at the array's end the last < 4 values come by plain loads.
-    auto issue = [&](long long t, int b, long long b0, long long b1) {
-        const bool fits = b0 >= 0 && b1 >= b0 && b1 <= total && b1 - b0 <= (long long)kCta * kSmallN;
-        float *buf = dyn + b * kBuf;
+    // Lane 0: the copy of tile t (span [b0, b1)) into buffer b.  Elements
+    // from round_down4(b0) land at the buffer's start; at the array's end the
+    // last < 4 values come by plain loads.
+    auto issue = [&](int b, long long b0, long long b1) {
+        const bool fits = b0 >= 0 && b1 >= b0 && b1 <= total && b1 - b0 <= (long long)kTile * kSmallN;
+        float *buf = bufs + b * kBuf;
         uint32_t bytes = 0;
         long long a0 = 0, a1 = 0;
         if (fits) {
@@ -428,18 +430,26 @@ __global__ void __launch_bounds__(kCta, 3) origami_stream_kernel(const float *__
             a1 = round_up4(b1) <= total ? round_up4(b1) : round_down4(b1);
             if (a1 > a0) bytes = (uint32_t)(4 * (a1 - a0));
         }
-        s_b0[b] = b0;
-        s_b1[b] = b1;
-        s_fits[b] = fits;
-        mbar_arrive_tx(&s_bar[b], bytes);
-        if (bytes) bulk_load(buf, values + a0, bytes, &s_bar[b]);
+        s_b0[w][b] = b0;
+        s_b1[w][b] = b1;
+        s_fits[w][b] = fits;
+        mbar_arrive_tx(&s_bar[w][b], bytes);
+        if (bytes) bulk_load(buf, values + a0, bytes, &s_bar[w][b]);
         if (fits)
             for (long long e = a1 > b0 ? a1 : b0; e < b1; ++e) buf[e - a0] = values[e];
     };
-
-    // tile t's problem for this thread, read one tile ahead
+    // lane 0: tile t's span, read one tile ahead of its copy
+    auto read_span = [&](long long t, long long &b0, long long &b1) {
+        b0 = b1 = 0;
+        if (t < n_tiles) {
+            const long long q0 = t * kTile, q1 = q0 + kTile < n_prob ? q0 + kTile : (long long)n_prob;
+            b0 = off[q0];
+            b1 = off[q1];
+        }
+    };
+    // tile t's problem for this lane, read one tile ahead
     auto read_mine = [&](long long t, long long &m0, long long &m1, float &K) {
-        const long long q = t * kCta + tid;
+        const long long q = t * kTile + lane;
         m0 = m1 = 0;
         K = 0.0f;
         if (t < n_tiles && q < n_prob) {
@@ -448,59 +458,50 @@ __global__ void __launch_bounds__(kCta, 3) origami_stream_kernel(const float *__
             K = budget[q];
         }
     };
-    // thread 0: tile t's span, read one tile ahead of its copy
-    auto read_span = [&](long long t, long long &b0, long long &b1) {
-        b0 = b1 = 0;
-        if (t < n_tiles) {
-            const long long q0 = t * kCta, q1 = q0 + kCta < n_prob ? q0 + kCta : (long long)n_prob;
-            b0 = off[q0];
-            b1 = off[q1];
-        }
-    };
 
-    long long nb0 = 0, nb1 = 0;                   // thread 0: the span of the tile to issue next
-    if (tid == 0) {
-        mbar_init(&s_bar[0]);
-        mbar_init(&s_bar[1]);
-        s_ndef = 0;
+    long long nb0 = 0, nb1 = 0;                   // lane 0: the span of the tile to issue next
+    if (lane == 0) {
+        mbar_init(&s_bar[w][0]);
+        mbar_init(&s_bar[w][1]);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");   // before the copies use them
         long long b0, b1;
         read_span(t_first, b0, b1);
-        issue(t_first, 0, b0, b1);
-        read_span(t_first + G, nb0, nb1);
+        issue(0, b0, b1);
+        read_span(t_first + W, nb0, nb1);
     }
     long long m0, m1;
     float K;
     read_mine(t_first, m0, m1, K);
-    __syncthreads();
+    __syncwarp();
 
     uint32_t parity[2] = {0u, 0u};
     bool aborted = false;
     int b = 0;
-    for (long long t = t_first; t < n_tiles; t += G, b ^= 1) {
+    for (long long t = t_first; t < n_tiles; t += W, b ^= 1) {
         // the next tile into the other buffer, once its last store has read it
-        if (tid == 0 && t + G < n_tiles) {
+        if (lane == 0 && t + W < n_tiles) {
             bulk_wait_read();
-            issue(t + G, b ^ 1, nb0, nb1);
-            read_span(t + 2 * G, nb0, nb1);
+            issue(b ^ 1, nb0, nb1);
+            read_span(t + 2 * W, nb0, nb1);
         }
-        const bool arrived = mbar_wait(&s_bar[b], parity[b]);
-        if (__syncthreads_or(!arrived)) {         // the copy never completed: stop (the tile's data is not there)
-            if (tid == 0) raise_flag(status, KVGOV_F_TIMEOUT);
+        const bool arrived = mbar_wait(&s_bar[w][b], parity[b]);
+        if (__any_sync(0xffffffffu, !arrived)) {  // the copy never completed: stop (the tile's data is not there)
+            if (lane == 0) raise_flag(status, KVGOV_F_TIMEOUT);
             aborted = true;
             break;
         }
         parity[b] ^= 1u;
-        const long long b0 = s_b0[b], b1 = s_b1[b];
-        const bool fits = s_fits[b] != 0;
-        const long long q = t * kCta + tid;
-        const long long q1 = t * kCta + kCta < n_prob ? t * kCta + kCta : (long long)n_prob;
-        long long nm0, nm1;                       // this thread's problem of the next tile
+        const long long b0 = s_b0[w][b], b1 = s_b1[w][b];
+        const bool fits = s_fits[w][b] != 0;
+        const long long q = t * kTile + lane;
+        const long long q1 = t * kTile + kTile < n_prob ? t * kTile + kTile : (long long)n_prob;
+        long long nm0, nm1;                       // this lane's problem of the next tile
         float nK;
-        read_mine(t + G, nm0, nm1, nK);
-        float *buf = dyn + b * kBuf;
+        read_mine(t + W, nm0, nm1, nK);
+        float *buf = bufs + b * kBuf;
         const long long a0 = round_down4(b0);
         if (fits) {
+            bool left = false;                    // this lane's problem is left to the warp
             if (q < q1) {
                 const bool ok = m0 >= b0 && m1 >= m0 && m1 <= b1 && m1 - m0 <= kSmallN;
                 const int n = ok ? (int)(m1 - m0) : 0;
@@ -512,28 +513,22 @@ __global__ void __launch_bounds__(kCta, 3) origami_stream_kernel(const float *__
                     else if (n <= 50) done = solve_thread_reg<50, true>(x, n, K, q, lambda_out, utility_out, status);
                     else done = solve_thread_reg<kSmallN, true>(x, n, K, q, lambda_out, utility_out, status);
                 }
-                if (!done) s_def[atomicAdd(&s_ndef, 1)] = tid;
+                left = !done;
+            }
+            __syncwarp();
+            for (unsigned pend = __ballot_sync(0xffffffffu, left); pend; pend &= pend - 1) {
+                const long long dq = t * kTile + (__ffs((int)pend) - 1);
+                const long long d0 = off[dq], d1 = off[dq + 1];
+                if (d0 >= b0 && d1 >= d0 && d1 <= b1)
+                    solve_warp_core(buf + (d0 - a0), buf + (d0 - a0), d1 - d0, budget[dq], false, dq, lambda_out,
+                                    utility_out, status);
+                else
+                    solve_warp(values, off, dq, total, budget, p, lambda_out, utility_out, status);
+                __syncwarp();
             }
             fence_async_smem();
-            __syncthreads();
-            const int ndef = s_ndef;
-            if (ndef > 0) {                       // the warps take the problems left to them, in place
-                for (int k = tid / 32; k < ndef; k += kCta / 32) {
-                    const int d = s_def[k];
-                    const long long dq = t * kCta + d;
-                    const long long d0 = off[dq], d1 = off[dq + 1];
-                    const bool inside = d0 >= b0 && d1 >= d0 && d1 <= b1;
-                    if (inside)
-                        solve_warp_core(buf + (d0 - a0), buf + (d0 - a0), d1 - d0, budget[dq], false, dq, lambda_out,
-                                        utility_out, status);
-                    else
-                        solve_warp(values, off, dq, total, budget, p, lambda_out, utility_out, status);
-                }
-                fence_async_smem();
-                __syncthreads();
-                if (tid == 0) s_ndef = 0;
-            }
-            if (tid == 0) {                       // [b0, b1) out: its 16-byte-aligned middle in one bulk store
+            __syncwarp();
+            if (lane == 0) {                      // [b0, b1) out: its 16-byte-aligned middle in one bulk store
                 const long long c0 = round_up4(b0) < b1 ? round_up4(b0) : b1;
                 const long long c1 = round_down4(b1) > c0 ? round_down4(b1) : c0;
                 for (long long e = b0; e < c0; ++e) p[e] = buf[e - a0];
@@ -541,18 +536,18 @@ __global__ void __launch_bounds__(kCta, 3) origami_stream_kernel(const float *__
                 if (c1 > c0) bulk_store(p + c0, buf + (c0 - a0), (uint32_t)(4 * (c1 - c0)));
             }
         } else {
-            for (long long qq = t * kCta + tid / 32; qq < q1; qq += kCta / 32)
+            for (long long qq = t * kTile; qq < q1; ++qq)
                 solve_warp(values, off, qq, total, budget, p, lambda_out, utility_out, status);
         }
-        __syncthreads();                          // buffer b's next copy may go once its store has read it
+        __syncwarp();                             // buffer b's next copy may go once its store has read it
         m0 = nm0;
         m1 = nm1;
         K = nK;
     }
-    if (tid == 0) {
+    if (lane == 0) {
         bulk_wait_all();
         if (aborted)                              // copies that may still be under way into either buffer
-            for (int k = 0; k < 2; ++k) mbar_wait(&s_bar[k], parity[k]);
+            for (int k = 0; k < 2; ++k) mbar_wait(&s_bar[w][k], parity[k]);
     }
 }
 
@@ -591,7 +586,8 @@ extern "C" int kvgov_origami(const float *d_values, const int64_t *d_off, int32_
     const bool vec4 = kvgov_host::aligned16(d_values) && kvgov_host::aligned16(d_p);
     const int resident = vec4 ? stream_ctas() : 0;
     if (resident > 0) {
-        const long long g = grid < resident ? grid : resident;
+        const long long ctas = ((long long)n_prob + kTile * kStreamWarps - 1) / (kTile * kStreamWarps);
+        const long long g = ctas < resident ? ctas : resident;
         origami_stream_kernel<<<(unsigned)g, kCta, kStreamSmem, reinterpret_cast<cudaStream_t>(stream)>>>(
             d_values, d_off, n_prob, d_budget, d_p, d_lambda, d_utility, d_status);
     } else {
