@@ -323,19 +323,29 @@ __global__ void __launch_bounds__(kThreads, 1) chain_split_kernel(const SplitPar
     for (int i = 0; i < 8; ++i) hw[i] = 0u;
     for (int j = 0; j < jmax; ++j) {
         stage(j + 2);                      // its buffer last held block j - 1, read for the last time before
-        if (j > 0) {
-            bar_sync(bar_h);
-            read_state(hw);                // h_{j-1}
-        }
         cp_async_wait<1>();                // blocks j and j + 1 have landed
         uint32_t tw[16], w[16];
         read_tokens(j, tw);
         if (j == 0) ahead(0, tw);
         const int kind = block_kind<MODE>(j, k);
+        // the first 64 bytes of the message: every word but h_{j-1}'s before
+        // the wait for it, so that the schedule's chunk 1, which the round
+        // warp waits for after its first 16 rounds, starts right after H
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {      // first 64 bytes of the message
-            w[i] = kind == kFirst ? tw[i] : (kind == kSteadyH ? hw[i] : sw[i]);
-            w[8 + i] = kind == kFirst ? tw[8 + i] : (kind == kBoundary ? hw[i] : tw[i]);
+        for (int i = 0; i < 8; ++i) {
+            w[i] = kind == kFirst ? tw[i] : sw[i];
+            w[8 + i] = kind == kFirst ? tw[8 + i] : tw[i];
+        }
+        if (j > 0) {
+            bar_sync(bar_h);
+            read_state(hw);                // h_{j-1}
+        }
+        if (kind == kSteadyH) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) w[i] = hw[i];
+        } else if (kind == kBoundary) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) w[8 + i] = hw[i];
         }
         schedule_kw48(w, sm.kw1, lane, bar_b);
         if (j > 0 && j - 1 < nb) store_digest(j - 1, hw);
