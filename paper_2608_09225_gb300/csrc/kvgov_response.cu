@@ -52,8 +52,6 @@ struct ResponseParams {
 template <bool SALTED>
 __global__ void __launch_bounds__(kR) response_key_kernel(const ResponseParams p) {
     __shared__ __align__(16) uint32_t stage[kStages][kR * kSlotWords];
-    __shared__ long long s_tok[kR];
-    __shared__ int s_nbt[kR];
     __shared__ int s_mmax;
 
     constexpr int S = SALTED ? 8 : 0;        // salt words ahead of the prompt
@@ -81,8 +79,6 @@ __global__ void __launch_bounds__(kR) response_key_kernel(const ResponseParams p
             len = 0;
         }
     }
-    s_tok[tid] = nbt > 0 ? t0 : 0;
-    s_nbt[tid] = nbt;
     __syncthreads();
     if (nmsg > 0) atomicMax(&s_mmax, nmsg);
     __syncthreads();
@@ -90,17 +86,18 @@ __global__ void __launch_bounds__(kR) response_key_kernel(const ResponseParams p
 
     const char *tok_bytes = reinterpret_cast<const char *>(p.tokens);
     const long long end_bytes = tok_end * 4;
-    auto issue = [&](int jj, int buf) {
-        for (int idx = tid; idx < kR * kChunks; idx += kR) {
-            const int q = idx / kChunks, c = idx - q * kChunks;
-            if (jj >= s_nbt[q]) continue;
-            const long long sb = (s_tok[q] + (long long)KVGOV_BLOCK * jj) * 4;
+    auto issue = [&](int jj, int buf) {        // this thread's request's token block jj (as the chain kernel)
+        if (jj < nbt) {
+            const long long sb = (t0 + (long long)KVGOV_BLOCK * jj) * 4;
             const long long a0 = sb & ~15ll;
-            if (c == kChunks - 1 && a0 == sb) continue;   // aligned block: four chunks
-            const long long ca = a0 + 16ll * c;
-            const long long avail = end_bytes - ca;
-            if (avail <= 0) continue;                      // a partial last block at the end of the array
-            cp_async16(&stage[buf][q * kSlotWords + c * 4], tok_bytes + ca, avail >= 16 ? 16 : (int)avail);
+#pragma unroll
+            for (int c = 0; c < kChunks; ++c) {
+                if (c == kChunks - 1 && a0 == sb) break;      // aligned block: four chunks
+                const long long ca = a0 + 16ll * c;
+                const long long avail = end_bytes - ca;
+                if (avail <= 0) break;                         // a partial last block at the end of the array
+                cp_async16(&stage[buf][tid * kSlotWords + c * 4], tok_bytes + ca, avail >= 16 ? 16 : (int)avail);
+            }
         }
     };
 #pragma unroll
