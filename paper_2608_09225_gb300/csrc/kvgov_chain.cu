@@ -132,8 +132,13 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
 
     const int tid = threadIdx.x;
     const long long r = (long long)blockIdx.x * kR + tid;
-    if (tid == 0) s_jmax = 0;
-    if ((FUSE == kFuseArrival || FUSE == kFuseInsertPrev) && tid == 0) { s_new = 0; s_flags = 0; s_done = 0; }
+    // The variants that insert keep the CTA in step, block by block: without
+    // that barrier the serving step's chain launch took 498 us against 190
+    // (a mean over steps that include cache flushes, where every request
+    // inserts the same shared-prefix keys) and the arrival-order call 234
+    // against 212 us.  The others need none (next comment).
+    constexpr bool kLockstep = FUSE == kFuseArrival || FUSE == kFuseInsertPrev;
+    if (kLockstep && tid == 0) { s_new = 0; s_flags = 0; s_done = 0; s_jmax = 0; }
 
     // Per-request set-up and validation.
     const long long tok_end = p.tok_off[p.n_req];
@@ -159,12 +164,22 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
         if (ok) nb = (int)nbl;
         else raise_flag(p.status, KVGOV_F_BADINDEX);
     }
-    __syncthreads();
-    if (nb > 0) atomicMax(&s_jmax, nb);
-    __syncthreads();
-    const int jmax = s_jmax;
+    // Each thread stages and reads only its own request's blocks, so the
+    // warps of a CTA need no barrier between blocks: a warp held up by a
+    // fused lookup holds back no other (the probe-heavy batch's chain with
+    // the fused probe: 397 -> 380 us), and the lanes of a warp walk the
+    // warp's longest chain.  With kLockstep the CTA walks its longest.
+    int jmax;
+    if (kLockstep) {
+        __syncthreads();
+        if (nb > 0) atomicMax(&s_jmax, nb);
+        __syncthreads();
+        jmax = s_jmax;
+    } else {
+        jmax = (int)__reduce_max_sync(0xffffffffu, (unsigned)nb);
+    }
 
-    // Stage block jj of every request of the CTA into buffer buf.
+    // Stage this thread's request's block jj into buffer buf.
     const char *tok_bytes = reinterpret_cast<const char *>(p.tokens);
     const long long end_bytes = tok_end * 4;
     auto issue = [&](int jj, int buf) {
@@ -243,8 +258,8 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
         const int jn = j + kStages - 1;
         if (jn < jmax) issue(jn, jn % kStages);
         cp_async_commit();
-        cp_async_wait<kStages - 1>();
-        __syncthreads();
+        cp_async_wait<kStages - 1>();      // this thread's copies of block j have landed
+        if (kLockstep) __syncthreads();
 
         if (j < nb) {
             const uint32_t *src = &stage[j % kStages][tid * kSlotWords + sh];
@@ -322,7 +337,7 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             have = false;
         }
         if (FUSE == kFuseInsertPrev && pleft > 0) prev_insert_one();
-        __syncthreads();
+        if (kLockstep) __syncthreads();
     }
     cp_async_wait<0>();
     if (FUSE == kFuseProbe && r < p.n_req) p.prefix_blocks[r] = hits;
