@@ -7,8 +7,9 @@
 // included (no block truncation), with the FIPS 180-4 padding after it.
 //
 // Layout as in the chain kernel: one thread per request, kR requests per
-// CTA walking their 64-byte token blocks in lockstep, each block staged into
-// shared memory with 16-byte cp.async copies, double-buffered.  The message
+// CTA, each thread staging its own request's 64-byte token blocks into
+// shared memory with 16-byte cp.async copies, double-buffered, with no
+// barrier between blocks (a warp walks its longest message).  The message
 // stream is the salt's 8 words (salted) followed by the big-endian token
 // words, so with a salt a message block is the last 8 words of token block
 // m-1 (kept in registers) and the first 8 of token block m.  Words past the
@@ -52,12 +53,10 @@ struct ResponseParams {
 template <bool SALTED>
 __global__ void __launch_bounds__(kR) response_key_kernel(const ResponseParams p) {
     __shared__ __align__(16) uint32_t stage[kStages][kR * kSlotWords];
-    __shared__ int s_mmax;
 
     constexpr int S = SALTED ? 8 : 0;        // salt words ahead of the prompt
     const int tid = threadIdx.x;
     const long long r = (long long)blockIdx.x * kR + tid;
-    if (tid == 0) s_mmax = 0;
 
     const long long tok_end = p.tok_off[p.n_req];
     long long t0 = 0, len = 0;
@@ -79,10 +78,9 @@ __global__ void __launch_bounds__(kR) response_key_kernel(const ResponseParams p
             len = 0;
         }
     }
-    __syncthreads();
-    if (nmsg > 0) atomicMax(&s_mmax, nmsg);
-    __syncthreads();
-    const int mmax = s_mmax;
+    // Each thread stages and reads only its own request's blocks: no barrier
+    // between message blocks, and a warp walks its own longest message.
+    const int mmax = (int)__reduce_max_sync(0xffffffffu, (unsigned)nmsg);
 
     const char *tok_bytes = reinterpret_cast<const char *>(p.tokens);
     const long long end_bytes = tok_end * 4;
@@ -127,8 +125,7 @@ __global__ void __launch_bounds__(kR) response_key_kernel(const ResponseParams p
         const int jn = m + kStages - 1;
         if (jn < mmax) issue(jn, jn % kStages);
         cp_async_commit();
-        cp_async_wait<kStages - 1>();
-        __syncthreads();
+        cp_async_wait<kStages - 1>();      // this thread's copies of block m have landed
 
         if (m < nmsg) {
             const uint32_t *src = &stage[m % kStages][tid * kSlotWords + sh];
@@ -136,11 +133,16 @@ __global__ void __launch_bounds__(kR) response_key_kernel(const ResponseParams p
 #pragma unroll
             for (int i = 0; i < 16; ++i) tw[i] = bswap32(src[i]);   // stale past the prompt: masked below
             uint32_t w[16];
+            if (16ll * m + 15 < end_word) {                         // every word is the prompt's
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-                const uint32_t v = SALTED ? (i < 8 ? carry[i] : tw[i - 8]) : tw[i];
-                const long long k = 16ll * m + i;                   // stream word index
-                w[i] = k < end_word ? v : (k == end_word ? 0x80000000u : 0u);
+                for (int i = 0; i < 16; ++i) w[i] = SALTED ? (i < 8 ? carry[i] : tw[i - 8]) : tw[i];
+            } else {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const uint32_t v = SALTED ? (i < 8 ? carry[i] : tw[i - 8]) : tw[i];
+                    const long long k = 16ll * m + i;               // stream word index
+                    w[i] = k < end_word ? v : (k == end_word ? 0x80000000u : 0u);
+                }
             }
             if (SALTED) {
 #pragma unroll
@@ -152,7 +154,6 @@ __global__ void __launch_bounds__(kR) response_key_kernel(const ResponseParams p
             }
             sha_compress_small(st, w, add);
         }
-        __syncthreads();
     }
     cp_async_wait<0>();
     if (r < p.n_req) {
