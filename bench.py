@@ -57,8 +57,8 @@ CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain k
 # step's chain kernel from one ncu capture, and the SHA-256 (chain_source_hash)
 # of the sources it was captured from: reported as roofline.traffic only while
 # the kernel's sources still hash to that value.
-CHAIN_TRAFFIC = {"bytes_per_launch": 180470144,
-                 "source_sha256": "8c3842890bd13bafb6239bd74b61d41a0a600f4204d03a65ec2d86667e25989f"}
+CHAIN_TRAFFIC = {"bytes_per_launch": 180044672,
+                 "source_sha256": "899d28ea3ded72913a3263f9e4f86bf540b315b9abdf5d15eda6e46cfe6b9557"}
 
 
 # DRAM bytes per launch of the probe on the probe-heavy workload from one ncu
