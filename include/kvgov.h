@@ -68,7 +68,9 @@ typedef struct CUstream_st *kvgov_stream_t;
                                       probe window, or the side store was
                                       full; the key is not stored             */
 #define KVGOV_F_TIMEOUT 0x80u      /* an insert gave up waiting for another
-                                      thread to finish writing a slot's key   */
+                                      thread to finish writing a slot's key,
+                                      or a bulk copy of kvgov_origami did not
+                                      complete within its bounded wait        */
 
 /* Salt placement (paper section 2.1 equation, section 4.1, section 4.2). */
 #define KVGOV_UNSALTED 0           /* h_0 = H(T_0), h_j = H(h_{j-1} || T_j)   */
@@ -182,8 +184,16 @@ int kvgov_response_key(int mode, const int32_t *d_tokens, const int64_t *d_tok_o
  *              payoff max_i v_i (1 - p_i) under the allocation.
  *   d_status   nullable; KVGOV_F_BADINDEX for a NaN or infinite value, a
  *              negative or NaN budget (read as 0) or malformed offsets.
- * Tenants with v_i <= 0 get p_i = 0.  fp32 arithmetic, one warp per problem.
+ * Tenants with v_i <= 0 get p_i = 0.  fp32 arithmetic.  A problem of at
+ * most 64 tenants with every value positive and finite (and at most 2^126)
+ * is solved by one thread in registers, any other by a warp.  With d_values
+ * and d_p on 16-byte boundaries the values stream through shared memory by
+ * bulk copies (a persistent grid, each warp on its own tiles of 32
+ * problems); otherwise each CTA of 128 problems stages its values with
+ * plain loads.  The results are the same either way.
  * n_prob = 0 is a no-op.  EINVAL: negative n_prob, NULL arrays.
+ * KVGOV_F_TIMEOUT: a bulk copy did not complete within its bounded wait
+ * (the results are then incomplete).
  */
 int kvgov_origami(const float *d_values, const int64_t *d_off, int32_t n_prob, const float *d_budget, float *d_p,
                   float *d_lambda, float *d_utility, uint32_t *d_status, kvgov_stream_t stream);
