@@ -428,9 +428,10 @@ def test_probe_matches_oracle(kv, cap_log2):
                          ids=["few_long", "mid_short", "mid_long", "many", "many_tiny_requests", "many_long"])
 def test_probe_layouts_match_oracle(kv, n_req, max_nb, p_member):
     """Every probe layout (a warp per request below 2048 requests, 16 lanes
-    per request up to 32,768, 4 lanes above), with requests of 0, 1 and 2
-    blocks, prefixes that span several rounds (up to 400 blocks), and
-    prefixes that end exactly at a window's edge."""
+    per request up to 32,768, above that 16 requests per warp sharing its
+    lanes), with requests of 0, 1 and 2 blocks, prefixes that span several
+    rounds (up to 400 blocks), and prefixes that end exactly at a window's
+    edge."""
     rng = np.random.default_rng(n_req + max_nb)
     pool = keys_np(6000, n_req % 997 + 3)
     nb = rng.integers(0, max_nb + 1, n_req)
