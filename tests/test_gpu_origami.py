@@ -143,3 +143,36 @@ def test_origami_unaligned_buffers(kv, shift):
     assert int(st.item()) == 0 and not flag
     check(b, p[shift:shift + n], lam.cpu().numpy().astype(np.float64), u.cpu().numpy().astype(np.float64),
           p_ref, lam_ref, u_ref)
+
+
+def test_origami_large_problems_inside_small_tiles(kv):
+    """Tiles of 32 problems whose values fit a warp's buffer but one of which
+    has more than 64 tenants (the warp solves it in place), and problems with
+    a value above 2^126 (its reciprocal is not a normal number: the warp
+    solver takes it too); every problem against the oracle."""
+    rng = np.random.default_rng(31)
+    n_prob = 32 * 200
+    sizes = np.full(n_prob, 20, np.int64)
+    sizes[7::32] = rng.integers(65, 400, n_prob // 32)
+    vals = (1.0 + rng.pareto(1.29, int(sizes.sum()))).astype(np.float32)
+    off = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int64)
+    for q in range(3, n_prob, 97):
+        vals[off[q] + 1] = np.float32(2.0 ** 127)
+    b = W.AuditBatch(values=vals, off=off, budget=np.full(n_prob, 5.0, np.float32))
+    p, lam, u, st = gpu(kv, b)
+    p_ref, lam_ref, u_ref, flag = oracle.origami(b.values, b.off, b.budget)
+    assert st == 0 and not flag
+    check(b, p, lam, u, p_ref, lam_ref, u_ref)
+
+
+def test_origami_full_size_batch(kv):
+    """The bench's batch: 2^20 problems of the section 5.5 setting (50
+    tenants, Pareto 1.29, K = 10), every probability and level against the
+    oracle."""
+    b = W.audit(seed=2030, n_prob=1 << 20)
+    p, lam, u, st = gpu(kv, b)
+    p_ref, lam_ref, u_ref, _ = oracle.origami(b.values, b.off, b.budget)
+    assert st == 0
+    assert np.abs(p - p_ref).max() <= tol(50)
+    assert (np.abs(lam - lam_ref) <= tol(50) * lam_ref).all()
+    assert (np.abs(u - u_ref) <= tol(50) * np.abs(u_ref)).all()
