@@ -652,12 +652,13 @@ def main():
     traffic, traffic_src = profiled_traffic()
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s (int32)",
                 "frac": achieved / peak_tops, "traffic": traffic,
-                "kernel": ("chain_prev_kernel<BOUNDARY> (kvgov_chain_hash_insert_prev: the chain hash with the "
-                           "previous batch's insert)" if in_chain else
+                "kernel": ("chain_prev_kernel<BOUNDARY, insert + lookups> (kvgov_chain_hash_insert_prev: the chain "
+                           "hash with the previous batch's insert and this batch's lookups)" if in_chain else
                            "chain_kernel<BOUNDARY, probe> (kvgov_chain_hash_probe)"), "ops_per_launch": ops,
                 "kernel_ms": chain_ms,
                 "ops_counted": "SHA-256 ops of the chain only; the fused " +
-                               ("inserts of the previous batch" if in_chain else "lookups") + " are extra",
+                               ("inserts of the previous batch and lookups of this one" if in_chain else "lookups") +
+                               " are extra",
                 "algorithmic_bytes_per_launch": 96 * n_blocks,
                 "peak_basis": f"{n_sm} SMs x {sha_rate:.2f} nominal SHA-256 ops per SM per clock x {SM_MAX_MHZ:.0f} MHz:"
                               " the rate of the chain kernel's own steady-block code (a 96-byte message: two "
@@ -676,33 +677,34 @@ def main():
     gather = measure_gather(torch, kbuild.PEAK_LIB, cache.slots)
     claims = measure_slot_ops(torch, kbuild.PEAK_LIB, cache.slots, int(inserted_per_step))
     if in_chain:
-        # the probe: every request looks up its 4 shared-prefix blocks (hits) and block 4 (a miss); a hit
-        # walks (1 + 1/(1-a))/2 slots and a miss (1 + 1/(1-a)^2)/2 at the table's mean load factor a
+        # the probe resumes each request's walk where the chain launch's own lookups stopped: they found the 4
+        # shared-prefix blocks (L2 hits, as they were hashed), so the probe looks up block 4, a miss walking
+        # (1 + 1/(1-a)^2)/2 slots at the table's mean load factor a
         lf = flush.mean_load_factor()
-        walk = 4 * (1 + 1 / (1 - lf)) / 2 + (1 + 1 / (1 - lf) ** 2) / 2
-        lookups = 5 * n_req
-        tab_bytes = lookups * 32 + walk * n_req * 32 + 20 * n_req
+        miss_walk = (1 + 1 / (1 - lf) ** 2) / 2
+        lookups = n_req
+        tab_bytes = n_req * (32 + miss_walk * 32) + 24 * n_req
         tab_gbs = tab_bytes / (table_ms / 1e3) / 1e9
-        # 4 of a request's 5 lookups are the shared prefix's 4 keys, the same slots for every request, which
-        # L2 serves; only block 4's lookup walks slots that come from DRAM
-        dram_fed = n_req * 32 * (1 + (1 + 1 / (1 - lf) ** 2) / 2)
+        slot_bytes = n_req * 32 * miss_walk
         table_roofline = {
-            "kernel": "probe_share_kernel<16, true> (kvgov_probe)", "bound": "hbm", "achieved": tab_gbs,
+            "kernel": "probe_share_kernel<16, true> (kvgov_probe_resume: the step's probe, each walk resumed where "
+                      "the chain launch's lookups stopped)", "bound": "hbm", "achieved": tab_gbs,
             "peak": PEAKS.get("hbm_gbs"), "unit": "GB/s",
             "frac": tab_gbs / PEAKS["hbm_gbs"] if PEAKS.get("hbm_gbs") else None,
             "peak_source": "of fallback (6.8 TB/s)" if PEAKS.get("fallback") else
                            "of measured (MEASURED_PEAKS.json hbm_gbs, a copy)",
-            "l2_resident_share": 1 - dram_fed / tab_bytes,
-            "note": "L2-fed for the most part: the 4 shared-prefix lookups of every request hit the same 4 slots; "
-                    "the DRAM-bound table case is table_roofline_cfg4",
-            "dram_fed_bytes_per_launch": dram_fed,
+            "note": "one dependent lookup per request after reading its offsets and lower bound: latency, not "
+                    "bandwidth; the DRAM-bound table case is table_roofline_cfg4",
+            "slot_bytes_per_launch": slot_bytes,
             "random_read_ceiling_gbs": gather["gbs_32B"],
-            "frac_of_random_read_ceiling_dram_fed": dram_fed / (table_ms / 1e3) / 1e9 / gather["gbs_32B"],
+            "frac_of_random_read_ceiling_slots": slot_bytes / (table_ms / 1e3) / 1e9 / gather["gbs_32B"],
             "kernel_ms": table_ms, "timed_launches": f"every {table_every}th step of the timed region",
             "lookups_per_launch": lookups, "lookups_per_s": lookups / (table_ms / 1e3),
+            "lookups_in_chain_launch_per_step": 5 * n_req,
             "mean_load_factor": lf, "algorithmic_bytes_per_launch": tab_bytes,
-            "bytes_basis": "per lookup its 32 B digest and 32 B per slot walked at the mean load factor; per "
-                           "request 16 B offsets + 4 B prefix",
+            "bytes_basis": "per request its block-4 digest (32 B), 32 B per slot its miss walks at the mean load "
+                           "factor, 16 B offsets, 4 B lower bound in and 4 B prefix out (counted as if the chain "
+                           "launch's lookups missed nothing: a lookup racing the insert of its own key adds work)",
             "random_read_microbench": gather,
             "insert": {"where": "inside the next batch's chain launch (kvgov_chain_hash_insert_prev)",
                        "keys_inserted_per_step": inserted_per_step,

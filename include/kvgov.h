@@ -340,6 +340,24 @@ int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_dige
                 uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * kvgov_probe_resume -- kvgov_probe when a lower bound of every prefix is
+ * known: request r's walk starts at block d_prefix_blocks[r] (clamped to
+ * [0, n_b(r)]) instead of block 0, and the blocks before it are taken as
+ * cached.  Same definition and output as kvgov_probe (paper section 2.1)
+ * as long as each input entry is at most the request's prefix length on the
+ * table as it is now; a larger entry is not checked and is returned as if
+ * its blocks were cached.  The serving step uses it after a chain launch
+ * whose own lookups ran while the table was still growing
+ * (kvgov_chain_hash_insert_prev).
+ *   d_prefix_blocks [n_req] int32: in, the lower bounds (< 0 reads as 0);
+ *                   out, the prefix lengths.
+ *   other arguments, flags and EINVAL as for kvgov_probe.
+ */
+int kvgov_probe_resume(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,
+                       const int64_t *d_blk_off, int32_t n_req, int32_t *d_prefix_blocks, uint32_t *d_status,
+                       kvgov_stream_t stream);
+
+/*
  * kvgov_insert_uncached -- insert a probed batch: for every request r, its
  * blocks j >= d_prefix_blocks[r] (the output of kvgov_probe on the same
  * table, digests and offsets).  The blocks before that were found in the
@@ -370,7 +388,11 @@ int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_
  * warps' hashing.  Results: the digests of kvgov_chain_hash; the table,
  * *d_n_new and the insert flags of kvgov_insert_uncached on the previous
  * batch; the prefix lengths of kvgov_probe of this batch on the table after
- * that insert (a second launch).
+ * that insert.  With d_prefix_blocks the chain launch also looks each block
+ * up as it is computed, while the insert runs: such a lookup can miss a key
+ * still being inserted but never finds an absent one, so it leaves a lower
+ * bound of each prefix, and a second launch resumes every request's walk
+ * from there to the exact prefix length.
  *   mode .. d_digests  as for kvgov_chain_hash (this batch).
  *   d_slots, capacity  the table (as for kvgov_insert).
  *   d_prev_digests, d_prev_blk_off, prev_n_req, d_prev_prefix_blocks

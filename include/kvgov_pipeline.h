@@ -26,8 +26,11 @@
  *                   chain_start[s] as the last command before the chain
  *                   launch, so that batch i+1's prep runs beside it; then
  *     insert_in_chain = 1: kvgov_chain_hash_insert_prev (batch i's chain
- *                   hash carrying the insert of the pending batch i-1), then
- *                   kvgov_probe of batch i; batch i's insert is left pending
+ *                   hash carrying the insert of the pending batch i-1, its
+ *                   own lookups of batch i leaving in d_prefix[s] a lower
+ *                   bound of each prefix), then the probe of batch i resuming
+ *                   each walk from there (the prefix lengths of kvgov_probe
+ *                   on the table after the insert); batch i's insert is left pending
  *                   for the next submit (or kvgov_pipeline_drain); slot s-1
  *                   is free once the chain launch is done.  With no pending
  *                   batch: kvgov_chain_hash_probe.

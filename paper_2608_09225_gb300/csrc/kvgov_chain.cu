@@ -102,6 +102,7 @@ constexpr int kFuseNone = 0;      // nothing (kvgov_chain_hash)
 constexpr int kFuseProbe = 1;     // look it up (kvgov_chain_hash_probe)
 constexpr int kFuseArrival = 2;   // insert it, arrival order (kvgov_chain_hash_arrival)
 constexpr int kFuseInsertPrev = 3;   // insert the previous batch's uncached blocks (kvgov_chain_hash_insert_prev)
+constexpr int kFuseInsertPrevProbe = 4;   // both: the insert, and a lookup giving a lower bound of the prefix
 
 // Big-endian words of principal pi's 32-byte salt.
 __device__ __forceinline__ void load_salt(const uint8_t *salts, int pi, uint32_t sw[8]) {
@@ -123,6 +124,14 @@ __device__ __forceinline__ void load_salt(const uint8_t *salts, int pi, uint32_t
 // batch's requests t, t + T, ... (T threads in the grid), one block per
 // iteration of its own chain and the rest after it (the insert of
 // kvgov_insert_uncached).
+// kFuseInsertPrevProbe: the insert of kFuseInsertPrev and the lookups of
+// kFuseProbe in one launch.  A lookup that runs while the insert fills the
+// table can miss a key that is being inserted (it reads an empty slot or a
+// claimed slot whose second half is not yet written) but never finds one
+// that is absent, since a slot, once claimed, never changes its key.  So
+// the prefix it leaves is a lower bound of the prefix on the table after the
+// insert, and a probe that resumes each walk where it stopped
+// (kvgov_host::probe_resume) makes it exact.
 template <int MODE, int FUSE>
 __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalParams &a,
                                            const PrevParams &q = PrevParams{}) {
@@ -137,7 +146,9 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
     // (a mean over steps that include cache flushes, where every request
     // inserts the same shared-prefix keys) and the arrival-order call 234
     // against 212 us.  The others need none (next comment).
-    constexpr bool kLockstep = FUSE == kFuseArrival || FUSE == kFuseInsertPrev;
+    constexpr bool kIns = FUSE == kFuseInsertPrev || FUSE == kFuseInsertPrevProbe;   // the previous batch's insert
+    constexpr bool kLook = FUSE == kFuseProbe || FUSE == kFuseInsertPrevProbe;        // lookups of this batch
+    constexpr bool kLockstep = FUSE == kFuseArrival || kIns;
     if (kLockstep && tid == 0) { s_new = 0; s_flags = 0; s_done = 0; s_jmax = 0; }
 
     // Per-request set-up and validation.
@@ -253,7 +264,7 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             prev_next();
         }
     };
-    if (FUSE == kFuseInsertPrev) prev_next();
+    if (kIns) prev_next();
     for (int j = 0; j < jmax; ++j) {
         const int jn = j + kStages - 1;
         if (jn < jmax) issue(jn, jn % kStages);
@@ -301,7 +312,7 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             const uint4 q1 = make_uint4(bswap32(h[4]), bswap32(h[5]), bswap32(h[6]), bswap32(h[7]));
             dst[0] = q0;
             dst[1] = q1;
-            if (FUSE == kFuseProbe && hits == j && lookup(p.slots, p.mask, q0, q1)) hits = j + 1;
+            if (kLook && hits == j && lookup(p.slots, p.mask, q0, q1)) hits = j + 1;
             if (FUSE == kFuseArrival) {
                 ak[0] = u64_of(q0.x, q0.y); ak[1] = u64_of(q0.z, q0.w);
                 ak[2] = u64_of(q1.x, q1.y); ak[3] = u64_of(q1.z, q1.w);
@@ -336,14 +347,14 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             }
             have = false;
         }
-        if (FUSE == kFuseInsertPrev && pleft > 0) prev_insert_one();
+        if (kIns && pleft > 0) prev_insert_one();
         if (kLockstep) __syncthreads();
     }
     cp_async_wait<0>();
-    if (FUSE == kFuseProbe && r < p.n_req) p.prefix_blocks[r] = hits;
-    if (FUSE == kFuseInsertPrev)
+    if (kLook && r < p.n_req) p.prefix_blocks[r] = hits;
+    if (kIns)
         while (pleft > 0) prev_insert_one();
-    if (FUSE == kFuseArrival || FUSE == kFuseInsertPrev)
+    if (FUSE == kFuseArrival || kIns)
         publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, FUSE == kFuseArrival ? a.n_new : q.n_new,
                        p.status);
 }
@@ -360,9 +371,10 @@ __global__ void __launch_bounds__(kR) chain_arrival_kernel(const ChainParams p, 
 
 // At most 64 registers, so that 8 CTAs fit an SM: the batch's CTAs leave
 // room beside them for the next batch's salts and block offsets.
-template <int MODE>
+// FUSE: kFuseInsertPrev or kFuseInsertPrevProbe.
+template <int MODE, int FUSE>
 __global__ void __launch_bounds__(kR, 8) chain_prev_kernel(const ChainParams p, const PrevParams q) {
-    chain_body<MODE, kFuseInsertPrev>(p, ArrivalParams{}, q);
+    chain_body<MODE, FUSE>(p, ArrivalParams{}, q);
 }
 
 }  // namespace
@@ -370,15 +382,15 @@ __global__ void __launch_bounds__(kR, 8) chain_prev_kernel(const ChainParams p, 
 namespace {
 
 // Launch chain_kernel<mode, FUSE> (chain_arrival_kernel<mode> for kFuseArrival,
-// chain_prev_kernel<mode> for kFuseInsertPrev).
+// chain_prev_kernel<mode, FUSE> for kFuseInsertPrev and kFuseInsertPrevProbe).
 template <int FUSE>
 void launch_chain_kernel(int mode, unsigned grid, cudaStream_t s, const ChainParams &p,
                          const ArrivalParams &a = ArrivalParams{}, const PrevParams &q = PrevParams{}) {
-    if constexpr (FUSE == kFuseInsertPrev) {
+    if constexpr (FUSE == kFuseInsertPrev || FUSE == kFuseInsertPrevProbe) {
         switch (mode) {
-        case KVGOV_UNSALTED: chain_prev_kernel<KVGOV_UNSALTED><<<grid, kR, 0, s>>>(p, q); break;
-        case KVGOV_ROOT: chain_prev_kernel<KVGOV_ROOT><<<grid, kR, 0, s>>>(p, q); break;
-        default: chain_prev_kernel<KVGOV_BOUNDARY><<<grid, kR, 0, s>>>(p, q); break;
+        case KVGOV_UNSALTED: chain_prev_kernel<KVGOV_UNSALTED, FUSE><<<grid, kR, 0, s>>>(p, q); break;
+        case KVGOV_ROOT: chain_prev_kernel<KVGOV_ROOT, FUSE><<<grid, kR, 0, s>>>(p, q); break;
+        default: chain_prev_kernel<KVGOV_BOUNDARY, FUSE><<<grid, kR, 0, s>>>(p, q); break;
         }
     } else if constexpr (FUSE == kFuseArrival) {
         switch (mode) {
@@ -420,7 +432,8 @@ struct FuseArgs {
     const int64_t *prev_blk_off = nullptr;
     int32_t prev_n_req = 0;
     const int32_t *prev_prefix_blocks = nullptr;
-    int32_t *probe_prefix_blocks = nullptr;     // kFuseInsertPrev: probe this batch after the insert
+    int32_t *probe_prefix_blocks = nullptr;     // kFuseInsertPrev: probe this batch after the insert ...
+    bool probe_complete = true;                 // ... to the end (else: leave a lower bound, see launch_chain)
 };
 
 int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
@@ -486,19 +499,36 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     // the chain; there they run as separate launches (same results).
     const DeviceInfo dev = device_info();
     const long long min_fused = 2ll * 32 * 4 * (dev.sms > 0 ? dev.sms : 152);
+    // kFuseInsertPrev with probe_prefix_blocks: the chain launch looks every
+    // block up as it goes (a lower bound, kFuseInsertPrevProbe) and a probe
+    // resumes the walks from there; probe_complete = false leaves that probe
+    // to the caller (kvgov_host::probe_resume), with 0 as the bound where the
+    // launch made no lookups.
     if (f.fuse == kFuseInsertPrev) {
         int rc;
+        bool lower = false;                        // probe_prefix_blocks holds the lookups' lower bound
         if (f.prev_n_req > 0 && n_req >= min_fused) {
-            launch_chain_kernel<kFuseInsertPrev>(mode, grid, s, p, a, q);
+            if (f.probe_prefix_blocks) {
+                p.prefix_blocks = f.probe_prefix_blocks;
+                launch_chain_kernel<kFuseInsertPrevProbe>(mode, grid, s, p, a, q);
+                lower = true;
+            } else {
+                launch_chain_kernel<kFuseInsertPrev>(mode, grid, s, p, a, q);
+            }
             rc = kvgov_host::launch_status();
         } else {                                   // a small batch (or no insert): separate launches
             rc = launch_plain(mode, grid, s, p);
             if (rc == KVGOV_OK && f.prev_n_req > 0) rc = insert_prev();
         }
-        if (rc == KVGOV_OK && f.probe_prefix_blocks)
-            rc = kvgov_probe(f.slots, f.capacity, d_digests, d_blk_off, n_req, f.probe_prefix_blocks, d_status,
-                             stream);
-        return rc;
+        if (rc != KVGOV_OK || !f.probe_prefix_blocks) return rc;
+        if (f.probe_complete)
+            return lower ? kvgov_host::probe_resume(f.slots, f.capacity, d_digests, d_blk_off, n_req,
+                                                    f.probe_prefix_blocks, d_status, stream)
+                         : kvgov_probe(f.slots, f.capacity, d_digests, d_blk_off, n_req, f.probe_prefix_blocks,
+                                       d_status, stream);
+        if (!lower && cudaMemsetAsync(f.probe_prefix_blocks, 0, sizeof(int32_t) * (size_t)n_req, s) != cudaSuccess)
+            return KVGOV_ECUDA;
+        return KVGOV_OK;
     }
     const bool none = f.fuse == kFuseNone;
     const bool fused = !none && n_req >= min_fused;
@@ -569,6 +599,27 @@ extern "C" int kvgov_chain_hash_arrival(int mode, const int32_t *d_tokens, const
                         d_blk_off, d_digests, d_status, f, stream);
 }
 
+namespace {
+
+FuseArgs insert_prev_args(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_prev_digests,
+                          const int64_t *d_prev_blk_off, int32_t prev_n_req, const int32_t *d_prev_prefix_blocks,
+                          int32_t *d_prefix_blocks, unsigned long long *d_n_new, bool probe_complete) {
+    FuseArgs f;
+    f.fuse = kFuseInsertPrev;
+    f.probe_prefix_blocks = d_prefix_blocks;
+    f.probe_complete = probe_complete;
+    f.slots = d_slots;
+    f.capacity = capacity;
+    f.n_new = d_n_new;
+    f.prev_digests = d_prev_digests;
+    f.prev_blk_off = d_prev_blk_off;
+    f.prev_n_req = prev_n_req;
+    f.prev_prefix_blocks = d_prev_prefix_blocks;
+    return f;
+}
+
+}  // namespace
+
 extern "C" int kvgov_chain_hash_insert_prev(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
                                             const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
                                             const int32_t *d_boundary_tok, const int64_t *d_blk_off,
@@ -577,16 +628,26 @@ extern "C" int kvgov_chain_hash_insert_prev(int mode, const int32_t *d_tokens, c
                                             int32_t prev_n_req, const int32_t *d_prev_prefix_blocks,
                                             int32_t *d_prefix_blocks, unsigned long long *d_n_new,
                                             uint32_t *d_status, kvgov_stream_t stream) {
-    FuseArgs f;
-    f.fuse = kFuseInsertPrev;
-    f.probe_prefix_blocks = d_prefix_blocks;
-    f.slots = d_slots;
-    f.capacity = capacity;
-    f.n_new = d_n_new;
-    f.prev_digests = d_prev_digests;
-    f.prev_blk_off = d_prev_blk_off;
-    f.prev_n_req = prev_n_req;
-    f.prev_prefix_blocks = d_prev_prefix_blocks;
     return launch_chain(mode, d_tokens, d_tok_off, n_req, d_principal, d_salts, n_principals, d_boundary_tok,
-                        d_blk_off, d_digests, d_status, f, stream);
+                        d_blk_off, d_digests, d_status,
+                        insert_prev_args(d_slots, capacity, d_prev_digests, d_prev_blk_off, prev_n_req,
+                                         d_prev_prefix_blocks, d_prefix_blocks, d_n_new, true),
+                        stream);
 }
+
+namespace kvgov_host {
+int chain_insert_prev_lower(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                            const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                            const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                            uint8_t *d_slots, uint64_t capacity, const uint8_t *d_prev_digests,
+                            const int64_t *d_prev_blk_off, int32_t prev_n_req, const int32_t *d_prev_prefix_blocks,
+                            int32_t *d_prefix_lower, unsigned long long *d_n_new, uint32_t *d_status,
+                            kvgov_stream_t stream) {
+    if (!d_prefix_lower && n_req > 0) return KVGOV_EINVAL;
+    return launch_chain(mode, d_tokens, d_tok_off, n_req, d_principal, d_salts, n_principals, d_boundary_tok,
+                        d_blk_off, d_digests, d_status,
+                        insert_prev_args(d_slots, capacity, d_prev_digests, d_prev_blk_off, prev_n_req,
+                                         d_prev_prefix_blocks, d_prefix_lower, d_n_new, false),
+                        stream);
+}
+}  // namespace kvgov_host

@@ -46,6 +46,23 @@ int launch_chain_split(int mode, const int32_t *d_tokens, const int64_t *d_tok_o
                        const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
                        uint32_t *d_status, cudaStream_t stream);
 
+// kvgov_probe_resume, arguments already in the library's types (kvgov_table.cu).
+int probe_resume(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests, const int64_t *d_blk_off,
+                 int32_t n_req, int32_t *d_prefix_blocks, uint32_t *d_status, kvgov_stream_t stream);
+
+// kvgov_chain_hash_insert_prev without the probe's completion: d_prefix_lower
+// receives, for every request, a lower bound of its cached prefix on the
+// table after the insert (what the chain launch's own lookups found while
+// the insert ran; 0 where the batch was too small for them), which
+// probe_resume completes (kvgov_chain.cu).
+int chain_insert_prev_lower(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                            const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                            const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                            uint8_t *d_slots, uint64_t capacity, const uint8_t *d_prev_digests,
+                            const int64_t *d_prev_blk_off, int32_t prev_n_req, const int32_t *d_prev_prefix_blocks,
+                            int32_t *d_prefix_lower, unsigned long long *d_n_new, uint32_t *d_status,
+                            kvgov_stream_t stream);
+
 inline int launch_status() {
     return cudaGetLastError() == cudaSuccess ? KVGOV_OK : KVGOV_ECUDA;
 }

@@ -130,11 +130,14 @@ extern "C" int kvgov_pipeline_submit(kvgov_pipeline *pl, const uint8_t *secret, 
     const int32_t *pr = salted ? d_principal : nullptr;
     const uint8_t *sl = salted ? d.d_salts[s] : nullptr;
     const int32_t *bt = d.mode == KVGOV_BOUNDARY ? d_boundary_tok : nullptr;
+    // with the previous batch's insert in the chain launch, that launch also
+    // looks this batch's blocks up (a lower bound of each prefix) and the
+    // probe below resumes the walks from there
     if (q >= 0)
-        KV_TRY(kvgov_chain_hash_insert_prev(d.mode, d_tokens, d_tok_off, n_req, pr, sl, d.n_principals, bt,
-                                            d.d_blk_off[s], d.d_digests[s], d.d_slots, d.capacity, d.d_digests[q],
-                                            d.d_blk_off[q], pl->n_req[q], d.d_prefix[q], nullptr, d.d_n_new,
-                                            d.d_status, cs));
+        KV_TRY(kvgov_host::chain_insert_prev_lower(d.mode, d_tokens, d_tok_off, n_req, pr, sl, d.n_principals, bt,
+                                                   d.d_blk_off[s], d.d_digests[s], d.d_slots, d.capacity,
+                                                   d.d_digests[q], d.d_blk_off[q], pl->n_req[q], d.d_prefix[q],
+                                                   d.d_prefix[s], d.d_n_new, d.d_status, cs));
     else
         KV_TRY(kvgov_chain_hash_probe(d.mode, d_tokens, d_tok_off, n_req, pr, sl, d.n_principals, bt, d.d_blk_off[s],
                                       d.d_digests[s], d.d_slots, d.capacity, d.d_prefix[s], d.d_status, cs));
@@ -146,8 +149,8 @@ extern "C" int kvgov_pipeline_submit(kvgov_pipeline *pl, const uint8_t *secret, 
     if (d.insert_in_chain) {
         if (q >= 0) {                                 // the probe after the insert
             if (table_ev0) KV_TRY(record(table_ev0, cs));
-            KV_TRY(kvgov_probe(d.d_slots, d.capacity, d.d_digests[s], d.d_blk_off[s], n_req, d.d_prefix[s],
-                               d.d_status, cs));
+            KV_TRY(kvgov_host::probe_resume(d.d_slots, d.capacity, d.d_digests[s], d.d_blk_off[s], n_req,
+                                            d.d_prefix[s], d.d_status, cs));
             if (table_ev1) KV_TRY(record(table_ev1, cs));
         }
         KV_TRY(record(d.probed[s], cs));

@@ -132,6 +132,17 @@ __device__ __forceinline__ void probe_range(const int64_t *__restrict__ blk_off,
     }
 }
 
+// Where request r's walk starts: block 0, or (resume) the block its
+// prefix_blocks entry names -- a lower bound of its cached prefix, left there
+// by lookups that ran while the table was still growing -- clamped to
+// [0, nb].
+__device__ __forceinline__ long long probe_start(const int32_t *prefix_blocks, bool resume, long long r,
+                                                 long long nb) {
+    if (!resume || nb <= 0) return 0;
+    const long long s = prefix_blocks[r];
+    return s < 0 ? 0 : (s > nb ? nb : s);
+}
+
 // G lanes per request (32 / G requests per warp).  A request's first round
 // looks up its first `first` blocks; later rounds G, 2G, 4G ... blocks up to
 // G * kPer (kPer lookups per lane, their home slots read together so that
@@ -143,8 +154,8 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
                                                                   unsigned long long mask,
                                                                   const uint4 *__restrict__ digests,
                                                                   const int64_t *__restrict__ blk_off,
-                                                                  int32_t n_req, int32_t *__restrict__ prefix_blocks,
-                                                                  uint32_t *status, int first) {
+                                                                  int32_t n_req, int32_t *prefix_blocks,
+                                                                  uint32_t *status, int first, bool resume) {
     constexpr int kSegs = 32 / G;
     constexpr unsigned kSegMask = G == 32 ? 0xffffffffu : ((1u << G) - 1u);
     const int lane = threadIdx.x & 31, seg = lane / G, sl = lane % G;
@@ -154,9 +165,9 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
         const long long r = wg * kSegs + seg;
         long long base = 0, nb = 0;
         if (r < n_req) probe_range(blk_off, n_req, r, base, nb, sl == 0 ? status : nullptr);
-        long long L = 0;
+        long long L = probe_start(prefix_blocks, resume, r, nb);
         int w = first;
-        bool active = nb > 0;
+        bool active = nb > L;
         while (__any_sync(0xffffffffu, active)) {
             uint4 q0[kPer], q1[kPer], a[kPer], b[kPer], c[kPer], d[kPer];
 #pragma unroll
@@ -230,8 +241,8 @@ __global__ void __launch_bounds__(kProbeThreads) probe_share_kernel(const uint4 
                                                                     unsigned long long mask,
                                                                     const uint4 *__restrict__ digests,
                                                                     const int64_t *__restrict__ blk_off,
-                                                                    int32_t n_req, int32_t *__restrict__ prefix_blocks,
-                                                                    uint32_t *status) {
+                                                                    int32_t n_req, int32_t *prefix_blocks,
+                                                                    uint32_t *status, bool resume) {
     constexpr unsigned kReqMask = (1u << R) - 1u;
     const int lane = threadIdx.x & 31;
     const long long warps_total = (long long)gridDim.x * (kProbeThreads / 32);
@@ -239,8 +250,11 @@ __global__ void __launch_bounds__(kProbeThreads) probe_share_kernel(const uint4 
          wg += warps_total) {                                  // warp-uniform
         const long long r = wg * R + lane;                     // lanes 0..R-1: request r
         long long base = 0, nb = 0, L = 0;
-        if (lane < R && r < n_req) probe_range(blk_off, n_req, r, base, nb, status);
-        unsigned act = __ballot_sync(0xffffffffu, lane < R && nb > 0) & kReqMask;
+        if (lane < R && r < n_req) {
+            probe_range(blk_off, n_req, r, base, nb, status);
+            L = probe_start(prefix_blocks, resume, r, nb);
+        }
+        unsigned act = __ballot_sync(0xffffffffu, lane < R && nb > L) & kReqMask;
         bool first = true;
         while (act) {                                          // warp-uniform
             const int k = __popc(act);
@@ -401,9 +415,12 @@ extern "C" int kvgov_insert(uint8_t *d_slots, uint64_t capacity, const uint8_t *
     return kvgov_host::launch_status();
 }
 
-extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,
-                           const int64_t *d_blk_off, int32_t n_req, int32_t *d_prefix_blocks, uint32_t *d_status,
-                           kvgov_stream_t stream) {
+namespace {
+
+// kvgov_probe, or (resume) its walks continued from each request's
+// prefix_blocks entry (kvgov_host::probe_resume).
+int launch_probe(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests, const int64_t *d_blk_off,
+                 int32_t n_req, int32_t *d_prefix_blocks, uint32_t *d_status, kvgov_stream_t stream, bool resume) {
     using kvgov_host::aligned16;
     if (!d_slots || !aligned16(d_slots) || !kvgov_host::pow2_capacity(capacity) || n_req < 0) return KVGOV_EINVAL;
     if (n_req == 0) return KVGOV_OK;
@@ -412,16 +429,38 @@ extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     if (n_req >= kProbeShareMin)
         probe_share_kernel<kProbeShareR, kProbeSharePair><<<probe_grid(n_req, 32 / kProbeShareR), kProbeThreads, 0, s>>>(
-            slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status);
+            slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, resume);
     else if (n_req >= kProbeMid.min_req)
         probe_seg_kernel<kProbeMid.G, kProbeMid.per, kProbeMid.pair != 0, kProbeMid.coop != 0>
             <<<probe_grid(n_req, kProbeMid.G), kProbeThreads, 0, s>>>(
-                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, kProbeMid.first);
+                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, kProbeMid.first, resume);
     else
         probe_seg_kernel<kProbeFew.G, kProbeFew.per, kProbeFew.pair != 0, kProbeFew.coop != 0>
             <<<probe_grid(n_req, kProbeFew.G), kProbeThreads, 0, s>>>(
-                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, kProbeFew.first);
+                slots, capacity - 1, dig, d_blk_off, n_req, d_prefix_blocks, d_status, kProbeFew.first, resume);
     return kvgov_host::launch_status();
+}
+
+}  // namespace
+
+namespace kvgov_host {
+int probe_resume(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests, const int64_t *d_blk_off,
+                 int32_t n_req, int32_t *d_prefix_blocks, uint32_t *d_status, kvgov_stream_t stream) {
+    return launch_probe(d_slots, capacity, d_digests, d_blk_off, n_req, d_prefix_blocks, d_status, stream, true);
+}
+}  // namespace kvgov_host
+
+extern "C" int kvgov_probe_resume(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,
+                                  const int64_t *d_blk_off, int32_t n_req, int32_t *d_prefix_blocks,
+                                  uint32_t *d_status, kvgov_stream_t stream) {
+    return kvgov_host::probe_resume(d_slots, capacity, d_digests, d_blk_off, n_req, d_prefix_blocks, d_status,
+                                    stream);
+}
+
+extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,
+                           const int64_t *d_blk_off, int32_t n_req, int32_t *d_prefix_blocks, uint32_t *d_status,
+                           kvgov_stream_t stream) {
+    return launch_probe(d_slots, capacity, d_digests, d_blk_off, n_req, d_prefix_blocks, d_status, stream, false);
 }
 
 extern "C" int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,

@@ -80,6 +80,7 @@ def _load():
         L.kvgov_table_init.argtypes = [_p, ctypes.c_uint64, _p]
         L.kvgov_insert.argtypes = [_p, ctypes.c_uint64, _p, ctypes.c_int64, _p, _p, _p]
         L.kvgov_probe.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p]
+        L.kvgov_probe_resume.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p]
         L.kvgov_insert_uncached.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p, _p]
         L.kvgov_owner_init.argtypes = [_p, ctypes.c_uint64, _p]
         L.kvgov_insert_arrival.argtypes = [_p, _p, ctypes.c_uint64, _p, _p, ctypes.c_int32, ctypes.c_uint64, _p, _p,
@@ -103,7 +104,8 @@ def _load():
         L.kvgov_pipeline_destroy.argtypes = [_p]
         L.kvgov_pipeline_destroy.restype = None
         for fn in ("kvgov_block_offsets", "kvgov_count_blocks", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
-                   "kvgov_insert", "kvgov_probe", "kvgov_insert_uncached", "kvgov_chain_hash_probe",
+                   "kvgov_insert", "kvgov_probe", "kvgov_probe_resume", "kvgov_insert_uncached",
+                   "kvgov_chain_hash_probe",
                    "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
                    "kvgov_divergence_boundary", "kvgov_response_key", "kvgov_origami",
                    "kvgov_serve_arrival_static", "kvgov_pipeline_create", "kvgov_pipeline_submit",
@@ -345,6 +347,21 @@ def probe(slots: torch.Tensor, digests: torch.Tensor, blk_off: torch.Tensor,
                              _dev(prefix_blocks, torch.int32, "prefix_blocks"),
                              _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_probe")
+    return prefix_blocks
+
+
+def probe_resume(slots: torch.Tensor, digests: torch.Tensor, blk_off: torch.Tensor, prefix_blocks: torch.Tensor,
+                 status: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """probe, each request's walk starting at prefix_blocks[r] (a lower bound of
+    its prefix on the table as it is now); prefix_blocks is overwritten with
+    the prefix lengths and returned."""
+    n = blk_off.numel() - 1
+    _check(lib().kvgov_probe_resume(_dev(slots, torch.uint8, "slots"), capacity_of(slots),
+                                    _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(blk_off),
+                                    _dev(blk_off, torch.int64, "blk_off"), n,
+                                    _dev(prefix_blocks, torch.int32, "prefix_blocks"),
+                                    _dev(status, torch.int32, "status", True), _stream(stream)),
+           "kvgov_probe_resume")
     return prefix_blocks
 
 

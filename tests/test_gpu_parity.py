@@ -461,6 +461,47 @@ def test_probe_layouts_match_oracle(kv, n_req, max_nb, p_member):
     assert want.max() > (100 if max_nb >= 300 else 0)
 
 
+@pytest.mark.parametrize("n_req,max_nb", [(700, 400), (3000, 70), (40000, 40), (70000, 300)],
+                         ids=["few", "mid", "many", "many_long"])
+def test_probe_resume_from_lower_bounds(kv, n_req, max_nb):
+    """kvgov_probe_resume, every layout: starting each request's walk at any
+    lower bound of its prefix (0, the prefix itself, a random value between,
+    a negative entry, a bound inside a window or at its edge) gives the
+    prefix lengths of the oracle's set (paper section 2.1), as kvgov_probe
+    does from block 0."""
+    rng = np.random.default_rng(3 * n_req + max_nb)
+    pool = keys_np(6000, n_req % 991 + 11)
+    nb = rng.integers(0, max_nb + 1, n_req)
+    nb[:6] = [0, 1, 2, max_nb, max_nb, max_nb]
+    off = np.concatenate([[0], np.cumsum(nb)]).astype(np.int64)
+    digests = pool[rng.integers(0, len(pool), int(off[-1]))]
+    member = rng.random(len(pool)) < 0.97
+    digests[off[3]:off[4]] = pool[np.nonzero(member)[0][:max_nb]]      # request 3: every block cached
+    slots = kv.new_table(1 << 14)
+    st = status_tensor()
+    kv.insert(slots, dev(pool[member]), st)
+    ks = oracle.KeySet(1)
+    ks.insert(pool[member])
+    want = ks.prefix_blocks(digests, off)
+    assert want[3] == max_nb and want.max() > 3
+    d_dig, d_off = dev(digests), dev(off)
+    bounds = {
+        "zero": np.zeros(n_req, np.int32),
+        "exact": want.astype(np.int32),
+        "between": (rng.random(n_req) * (want + 1)).astype(np.int32),
+        "negative": np.where(rng.random(n_req) < 0.5, -rng.integers(1, 5, n_req), want).astype(np.int32),
+        "window_edge": np.minimum(want, 32 * (want // 32)).astype(np.int32),
+    }
+    for name, lower in bounds.items():
+        assert (lower <= want).all()
+        pre = dev(lower)
+        kv.probe_resume(slots, d_dig, d_off, pre, status=st)
+        torch.cuda.synchronize()
+        assert int(st.item()) == 0
+        got = pre.cpu().numpy()
+        assert (got == want).all(), f"{name}: {int((got != want).sum())} of {n_req} prefix lengths differ"
+
+
 @pytest.mark.parametrize("n_req", [500, 5000, 40000], ids=["few", "mid", "many"])
 @pytest.mark.parametrize("cap_log2,n_keys,clustered", [(12, 3686, 0), (12, 2400, 400), (5, 28, 0), (16, 49152, 0)],
                          ids=["load_0.9", "clustered_run", "window_is_table", "load_0.75"])
@@ -686,22 +727,26 @@ def test_chain_hash_insert_prev_matches_separate_calls(kv, mode, n_req, prev_n):
 
 
 @pytest.mark.parametrize("mode", [0, 1, 2])
-@pytest.mark.parametrize("n_req", [180, 40960], ids=["separate_launches", "fused"])
-def test_chain_hash_insert_prev_with_probe(kv, mode, n_req):
+@pytest.mark.parametrize("n_req,stride", [(180, 3), (40960, 3), (40960, 1)],
+                         ids=["separate_launches", "fused", "fused_same_batch"])
+def test_chain_hash_insert_prev_with_probe(kv, mode, n_req, stride):
     """With a prefix output, kvgov_chain_hash_insert_prev gives this batch's
     digests, the previous batch's insert, and this batch's prefix lengths
     against the table after that insert -- the results of kvgov_chain_hash,
     kvgov_insert_uncached and kvgov_probe in sequence.  The previous batch
-    shares keys with this one, so the probe must see the insert."""
-    rng = np.random.default_rng(7 * n_req + mode)
+    shares keys with this one (every third request's blocks, or every
+    request's), so the probe must see the insert: in the fused launch the
+    lookups of a block run while its own key is being inserted, and the
+    resumed probe must make up what they missed."""
+    rng = np.random.default_rng(7 * n_req + mode + stride)
     lengths = list(rng.integers(0, 300, n_req))
     b = W.ragged(23 + mode, lengths)
     salts = oracle.derive_salts(b"probe-after-insert", *W.principal_ids(8))
     ref = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
     blk_ref = oracle.block_offsets(b.tok_off)
-    # the previous batch: this batch's digests of every third request (so its insert makes them hit), plus
+    # the previous batch: this batch's digests of every stride-th request (so its insert makes them hit), plus
     # random keys; its prefix lengths cut some requests short
-    prev_req = np.arange(0, n_req, 3)
+    prev_req = np.arange(0, n_req, stride)
     prev_rows = [ref[blk_ref[r]:blk_ref[r + 1]] for r in prev_req]
     pnb = np.array([len(x) for x in prev_rows], np.int64)
     poff = np.concatenate([[0], np.cumsum(pnb)]).astype(np.int64)
