@@ -132,14 +132,11 @@ __device__ __forceinline__ void probe_range(const int64_t *__restrict__ blk_off,
     }
 }
 
-// Where request r's walk starts: block 0, or (resume) the block its
+// Where request r's walk starts: block 0, or (resume) the block s its
 // prefix_blocks entry names -- a lower bound of its cached prefix, left there
 // by lookups that ran while the table was still growing -- clamped to
-// [0, nb].
-__device__ __forceinline__ long long probe_start(const int32_t *prefix_blocks, bool resume, long long r,
-                                                 long long nb) {
-    if (!resume || nb <= 0) return 0;
-    const long long s = prefix_blocks[r];
+// [0, nb].  The entry is read beside the request's offsets, not after them.
+__device__ __forceinline__ long long probe_start(long long s, long long nb) {
     return s < 0 ? 0 : (s > nb ? nb : s);
 }
 
@@ -163,9 +160,12 @@ __global__ void __launch_bounds__(kProbeThreads) probe_seg_kernel(const uint4 *_
     for (long long wg = ((long long)blockIdx.x * kProbeThreads + threadIdx.x) / 32; wg * kSegs < n_req;
          wg += warps_total) {                                  // warp-uniform
         const long long r = wg * kSegs + seg;
-        long long base = 0, nb = 0;
-        if (r < n_req) probe_range(blk_off, n_req, r, base, nb, sl == 0 ? status : nullptr);
-        long long L = probe_start(prefix_blocks, resume, r, nb);
+        long long base = 0, nb = 0, s0 = 0;
+        if (r < n_req) {
+            if (resume) s0 = prefix_blocks[r];
+            probe_range(blk_off, n_req, r, base, nb, sl == 0 ? status : nullptr);
+        }
+        long long L = probe_start(s0, nb);
         int w = first;
         bool active = nb > L;
         while (__any_sync(0xffffffffu, active)) {
@@ -251,8 +251,9 @@ __global__ void __launch_bounds__(kProbeThreads) probe_share_kernel(const uint4 
         const long long r = wg * R + lane;                     // lanes 0..R-1: request r
         long long base = 0, nb = 0, L = 0;
         if (lane < R && r < n_req) {
+            const long long s0 = resume ? prefix_blocks[r] : 0;
             probe_range(blk_off, n_req, r, base, nb, status);
-            L = probe_start(prefix_blocks, resume, r, nb);
+            L = probe_start(s0, nb);
         }
         unsigned act = __ballot_sync(0xffffffffu, lane < R && nb > L) & kReqMask;
         bool first = true;
