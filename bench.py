@@ -57,8 +57,8 @@ CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain k
 # step's chain kernel from one ncu capture, and the SHA-256 (chain_source_hash)
 # of the sources it was captured from: reported as roofline.traffic only while
 # the kernel's sources still hash to that value.
-CHAIN_TRAFFIC = {"bytes_per_launch": 180044672,
-                 "source_sha256": "899d28ea3ded72913a3263f9e4f86bf540b315b9abdf5d15eda6e46cfe6b9557"}
+CHAIN_TRAFFIC = {"bytes_per_launch": 200526208,
+                 "source_sha256": "c38c045c572c5ac754da09dd5ab1d22c4a1089d672dfffee4a9cafe9cbcee278"}
 
 
 # DRAM bytes per launch of the probe on the probe-heavy workload from one ncu
@@ -67,7 +67,7 @@ TABLE_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_table.cu", "paper_2608_09225
                  "paper_2608_09225_gb300/csrc/kvgov_stash.cuh", "paper_2608_09225_gb300/csrc/kvgov_internal.cuh",
                  "paper_2608_09225_gb300/csrc/kvgov_insert.cuh"]
 TABLE_TRAFFIC = {"probe_share_kernel<16, true>": {
-    "bytes_per_launch": 74625536, "source_sha256": "bf0b4ece69c570d320a286d9ead7225b89e2d3d5c627f682edbce8f44016b5fe"}}
+    "bytes_per_launch": 74626560, "source_sha256": "4813d8c0aabbb808fd422bdbd7f632bf5f9d9f4ed5c8e5a6a8abfd15c8fa9de7"}}
 
 
 def load_peaks() -> dict:
