@@ -58,7 +58,7 @@ CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain k
 # of the sources it was captured from: reported as roofline.traffic only while
 # the kernel's sources still hash to that value.
 CHAIN_TRAFFIC = {"bytes_per_launch": 200526208,
-                 "source_sha256": "c38c045c572c5ac754da09dd5ab1d22c4a1089d672dfffee4a9cafe9cbcee278"}
+                 "source_sha256": "85d072705de98f8ea01e70bcc93f66213122131b53e0fc6a62e5e966b7fa9585"}
 
 
 # DRAM bytes per launch of the probe on the probe-heavy workload from one ncu
@@ -67,7 +67,7 @@ TABLE_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_table.cu", "paper_2608_09225
                  "paper_2608_09225_gb300/csrc/kvgov_stash.cuh", "paper_2608_09225_gb300/csrc/kvgov_internal.cuh",
                  "paper_2608_09225_gb300/csrc/kvgov_insert.cuh"]
 TABLE_TRAFFIC = {"probe_share_kernel<16, true>": {
-    "bytes_per_launch": 74626560, "source_sha256": "4813d8c0aabbb808fd422bdbd7f632bf5f9d9f4ed5c8e5a6a8abfd15c8fa9de7"}}
+    "bytes_per_launch": 74626560, "source_sha256": "de6cb50b8070f52df5d1f6fc0b028f2a93c84958701b43431ccb540876ba6856"}}
 
 
 def load_peaks() -> dict:

@@ -1,7 +1,10 @@
 // kvgov_lookup.cuh -- read-only lookup of a 32-byte key in the prefix-cache
 // table (slot encoding and probe window as described in kvgov_table.cu and
 // include/kvgov.h), shared by the probe kernels and the fused chain + probe
-// kernel.  The table must not change while a lookup runs.
+// kernel.  Exact while the table does not change.  While inserts run (the
+// chain launch that carries the previous batch's insert), a slot only goes
+// from empty to claimed to complete and never changes its key, so a lookup
+// can miss a key that is being inserted but never finds an absent one.
 #pragma once
 #include <cstdint>
 
