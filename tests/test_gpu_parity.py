@@ -796,3 +796,24 @@ def test_probe_empty_and_bad_offsets(kv):
     assert int(st.item()) & kv.F_BADINDEX
     empty = kv.probe(slots, dev(keys_np(1, 7)), dev(np.array([0], np.int64)))
     assert empty.numel() == 0
+
+
+def test_probe_resume_empty_and_bad_offsets(kv):
+    """kvgov_probe_resume, as include/kvgov.h states it: a request whose
+    block range is malformed is flagged and gets 0 whatever its entry; a
+    negative entry reads as the lower bound 0; an entry past the request's
+    blocks is clamped to them (and, being the caller's claim, not checked);
+    an empty batch is a no-op."""
+    keys = keys_np(6, 9)
+    slots = kv.new_table(64)
+    st = status_tensor()
+    kv.insert(slots, dev(keys[:4]), st)
+    off = np.array([0, 4, 2, 6], np.int64)                 # request 1 runs backwards; request 2: rows 2-5
+    pre = dev(np.array([-5, 1, 8], np.int32))
+    kv.probe_resume(slots, dev(keys), dev(off), pre, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & kv.F_BADINDEX
+    assert pre.cpu().numpy().tolist() == [4, 0, 4]
+    empty = torch.zeros(0, dtype=torch.int32, device=DEV)
+    kv.probe_resume(slots, dev(keys[:1]), dev(np.array([0], np.int64)), empty)
+    torch.cuda.synchronize()
