@@ -57,8 +57,9 @@ CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain k
 # step's chain kernel from one ncu capture, and the SHA-256 (chain_source_hash)
 # of the sources it was captured from: reported as roofline.traffic only while
 # the kernel's sources still hash to that value.
-CHAIN_TRAFFIC = {"bytes_per_launch": 200526208,
-                 "source_sha256": "85d072705de98f8ea01e70bcc93f66213122131b53e0fc6a62e5e966b7fa9585"}
+CHAIN_TRAFFIC = {"chain_prev_kernel": {"bytes_per_launch": 200526208,
+                 "source_sha256": "85d072705de98f8ea01e70bcc93f66213122131b53e0fc6a62e5e966b7fa9585"},
+                 "chain_serve_kernel": {"bytes_per_launch": None, "source_sha256": None}}
 
 
 # DRAM bytes per launch of the probe on the probe-heavy workload from one ncu
@@ -112,14 +113,16 @@ def chain_source_hash() -> str:
     return sources_hash(CHAIN_SOURCES)
 
 
-def profiled_traffic():
-    """DRAM bytes per chain-kernel launch from the last ncu capture, if that
-    capture was taken of the chain kernel's current sources; else None."""
-    if CHAIN_TRAFFIC["bytes_per_launch"] is None:
+def profiled_traffic(kernel: str):
+    """DRAM bytes per launch of the step's chain kernel from its last ncu
+    capture, if that capture was taken of the chain kernel's current sources;
+    else None."""
+    rec = CHAIN_TRAFFIC.get(kernel, {})
+    if rec.get("bytes_per_launch") is None:
         return None, "no capture recorded"
-    if CHAIN_TRAFFIC["source_sha256"] != chain_source_hash():
+    if rec.get("source_sha256") != chain_source_hash():
         return None, "the last capture was of other sources"
-    return CHAIN_TRAFFIC["bytes_per_launch"], "ncu capture of the current sources"
+    return rec["bytes_per_launch"], "ncu capture of the current sources"
 
 
 # --------------------------------------------------------------------------- helpers
@@ -458,10 +461,11 @@ def main():
     ap.add_argument("--seed", type=int, default=None, help="base seed (default: fresh per run)")
     ap.add_argument("--cpu-sample", type=int, default=16384, help="requests per oracle step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--schedule", default="insert_in_chain", choices=["insert_in_chain", "inline"],
+    ap.add_argument("--schedule", default="insert_in_chain", choices=["insert_in_chain", "inline", "one_launch"],
                     help="insert_in_chain: each batch's insert runs inside the next batch's chain-hash launch, and "
                          "each batch is probed after its chain hash; inline: chain hash with the fused probe, then "
-                         "the insert")
+                         "the insert; one_launch: each batch's lookups and insert in its own chain-hash launch "
+                         "(kvgov_chain_hash_serve, the table's generations telling the batch's keys from older ones)")
     ap.add_argument("--configs", action="store_true",
                     help="instead of the timed serving step: per-kernel rates on every workload, one JSON line each")
     ap.add_argument("--only", default=None,
@@ -529,7 +533,8 @@ def main():
     # ---- the timed steps: DevicePipeline computes each batch's salts and block
     # offsets on a prep stream beside the previous batch's chain hash
     in_chain = args.schedule == "insert_in_chain"
-    pipe = DevicePipeline(cache, W.BOUNDARY, n_req, n_blocks, insert_in_chain=in_chain)
+    one = args.schedule == "one_launch"
+    pipe = DevicePipeline(cache, W.BOUNDARY, n_req, n_blocks, insert_in_chain=in_chain, one_launch=one)
     epoch = [1]
     launches = [0]
     table_timed = []
@@ -539,12 +544,15 @@ def main():
         epoch[0] += 1
         flushed = flush.before_step()              # load factor would pass 0.5: flush the cache
         pending = pipe.pending
-        if in_chain and (flushed or not pending):
-            tab_ev = None                          # this step runs no probe of its own (chain hash + fused probe)
+        if one or (in_chain and (flushed or not pending)):
+            tab_ev = None                          # this step runs no probe of its own (its chain launch looks up)
         if tab_ev is not None:
             table_timed.append(tab_ev)
         prefix, _ = pipe.submit(db, flushed, ev, tab_ev)
-        if in_chain:
+        if one:
+            # salts, block offsets (2), the chain hash with the batch's lookups and insert (+ table init)
+            launches[0] += 4 + int(flushed)
+        elif in_chain:
             # salts, block offsets (2), then the chain hash with the previous batch's insert and the probe or,
             # after a flush (which runs the pending insert and the table init first), the chain hash with
             # the probe fused in
@@ -641,7 +649,8 @@ def main():
     arrival = arrival_leg(torch, K, W, pool, n_req, n_blocks, cache, args.arrival_steps, chain_ms)
 
     # ---- end to end through the public API with host buffers
-    e2e = e2e_leg(torch, K, W, w0, pool_host[: min(4, args.pool)], args.e2e_steps, world, dist, args.table_slots, in_chain)
+    e2e = e2e_leg(torch, K, W, w0, pool_host[: min(4, args.pool)], args.e2e_steps, world, dist, args.table_slots,
+                  in_chain, one)
 
     # ---- roofline of the chain kernel (integer-pipe bound)
     micro = measure_int_peak(torch, kbuild.PEAK_LIB)
@@ -653,15 +662,18 @@ def main():
     # compressions) register-resident with no memory traffic, the better of two occupancies
     sha_rate = max(micro["sha_msg96"], micro["sha_msg96_8w"])
     peak_tops = n_sm * sha_rate * SM_MAX_MHZ * 1e6 / 1e12
-    traffic, traffic_src = profiled_traffic()
+    traffic, traffic_src = profiled_traffic("chain_serve_kernel" if one else "chain_prev_kernel")
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s (int32)",
                 "frac": achieved / peak_tops, "traffic": traffic,
-                "kernel": ("chain_prev_kernel<BOUNDARY, insert + lookups> (kvgov_chain_hash_insert_prev: the chain "
+                "kernel": ("chain_serve_kernel<BOUNDARY> (kvgov_chain_hash_serve: the chain hash with the batch's "
+                           "own lookups and insert)" if one else
+                           "chain_prev_kernel<BOUNDARY, insert + lookups> (kvgov_chain_hash_insert_prev: the chain "
                            "hash with the previous batch's insert and this batch's lookups)" if in_chain else
                            "chain_kernel<BOUNDARY, probe> (kvgov_chain_hash_probe)"), "ops_per_launch": ops,
                 "kernel_ms": chain_ms, "timed_launches": f"every {timing_every}th step of the timed region",
                 "ops_counted": "SHA-256 ops of the chain only; the fused " +
-                               ("inserts of the previous batch and lookups of this one" if in_chain else "lookups") +
+                               ("lookups and insert of the batch" if one else
+                                "inserts of the previous batch and lookups of this one" if in_chain else "lookups") +
                                " are extra",
                 "algorithmic_bytes_per_launch": 96 * n_blocks,
                 "peak_basis": f"{n_sm} SMs x {sha_rate:.2f} nominal SHA-256 ops per SM per clock x {SM_MAX_MHZ:.0f} MHz:"
@@ -680,7 +692,17 @@ def main():
     # the table kernel of the step (insert of the uncached blocks) against HBM and a random-read ceiling
     gather = measure_gather(torch, kbuild.PEAK_LIB, cache.slots)
     claims = measure_slot_ops(torch, kbuild.PEAK_LIB, cache.slots, int(inserted_per_step))
-    if in_chain:
+    if one:
+        table_roofline = {
+            "kernel": None, "frac": None,
+            "note": "no table kernel of its own: each batch's lookups (blocks 0-4 of every request: 4 hits and a "
+                    "miss) and its insert (blocks 4-7) run inside its chain launch, told apart by the table's "
+                    "generations; the DRAM-bound table case is table_roofline_cfg4",
+            "lookups_in_chain_launch_per_step": 5 * n_req,
+            "keys_inserted_per_step": inserted_per_step,
+            "random_read_microbench": gather,
+            "claim_ceiling_per_s": claims["read_cas_store_per_s"], "slot_op_microbench": claims}
+    elif in_chain:
         # the probe resumes each request's walk where the chain launch's own lookups stopped: they found the 4
         # shared-prefix blocks (L2 hits, as they were hashed), so the probe looks up block 4, a miss walking
         # (1 + 1/(1-a)^2)/2 slots at the table's mean load factor a
@@ -741,7 +763,7 @@ def main():
 
     # gate: no kernel may run above its own ceiling (the paper's section 5.7 gate rejects a result that
     # implies more than 100 % of the GPU's peak)
-    fracs = {"roofline.frac": roofline["frac"], "table_roofline.frac": table_roofline["frac"],
+    fracs = {"roofline.frac": roofline["frac"], "table_roofline.frac": table_roofline["frac"] or 0.0,
              "table_roofline_cfg4.probe.frac": table_cfg4["probe"]["frac"],
              "table_roofline_cfg4.insert.frac": table_cfg4["insert"]["frac"]}
     gate["frac_ok"] = all(f is not None and f <= 1.0 for f in fracs.values())
@@ -762,6 +784,10 @@ def main():
             "tokens_per_s": 16 * value, "chain_digests_per_s": world * n_blocks / (chain_ms / 1e3),
             "host_enqueue_ms_per_step": host_ms / args.steps,
             "schedule": ("DevicePipeline over the library's serving engine (kvgov_pipeline_submit, one call per "
+                         "step), one launch: salts (new epoch) and block offsets of batch i+1 on a prep stream "
+                         "beside the chain launch of batch i, which on a higher-priority compute stream hashes "
+                         "the batch, looks its blocks up and inserts its uncached ones" if one else
+                         "DevicePipeline over the library's serving engine (kvgov_pipeline_submit, one call per "
                          "step), insert in chain: salts (new epoch) and block offsets of batch i+1 on a "
                          "prep stream beside the chain hash of batch i; on a higher-priority compute stream the "
                          "chain hash of batch i with batch i-1's insert in the same launch, then the probe of batch "
@@ -926,7 +952,7 @@ def arrival_leg(torch, K, W, pool, n_req, n_blocks, cache, steps, chain_ms):
             "cache": f"empty {cap}-slot table per batch (re-initialised outside the timed call)"}
 
 
-def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots, in_chain=True):
+def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots, in_chain=True, one_launch=False):
     """Same step with host buffers, through the public HostPipeline: each
     step's inputs are copied from pinned host memory (a copy stream, which
     overlaps the previous step's serving) and its prefix lengths are copied
@@ -941,7 +967,7 @@ def e2e_leg(torch, K, W, w0, hosts, steps, world, dist, table_slots, in_chain=Tr
     n_tok = int(hosts[0].batch.tok_off[-1])
     n_blocks, _ = K.count_blocks(hosts[0].batch.tok_off)
     cache = PrefixCache(table_slots, w0.secret, w0.ids, w0.id_off)
-    pipe = HostPipeline(cache, W.BOUNDARY, n_req, n_tok, insert_in_chain=in_chain)
+    pipe = HostPipeline(cache, W.BOUNDARY, n_req, n_tok, insert_in_chain=in_chain, one_launch=one_launch)
     flush = FlushPolicy(table_slots, 4 * n_req)
     h2d = sum(t.numel() * t.element_size() for t in pinned[0])
     d2h = n_req * 4

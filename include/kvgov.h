@@ -416,6 +416,53 @@ int kvgov_chain_hash_insert_prev(int mode, const int32_t *d_tokens, const int64_
                                  unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream);
 
 /*
+ * kvgov_table_gen_stamp -- the table's generations (the per-key counter that
+ * kvgov_chain_hash_serve keeps beside it): d_gen[h] = value for every handle h
+ * that holds a key -- main slot h, or capacity + 8 + e for live side-store
+ * entry e (the handles of kvgov_insert_arrival) -- and 0 for every other.
+ *   d_gen  [capacity + KVGOV_STASH_SLOTS] u32, owned by the caller.
+ * EINVAL: bad capacity, NULL or misaligned pointer.
+ */
+int kvgov_table_gen_stamp(const uint8_t *d_slots, uint64_t capacity, uint32_t *d_gen, uint32_t value,
+                          kvgov_stream_t stream);
+
+/*
+ * kvgov_chain_hash_serve -- one batch through the whole serving step in one
+ * launch (paper section 2.1: the batch's requests look up their cached
+ * prefixes, then their uncached blocks are cached): kvgov_chain_hash, the
+ * prefix lengths of kvgov_probe against the table as it was before this
+ * call, and kvgov_insert_uncached of the batch after that, with its new keys
+ * given generation `gen`.  The lookups and the insert run in the same
+ * launch: a key counts as cached for this batch only if its generation is in
+ * [gen_floor, gen), and every key this call adds gets generation gen, so the
+ * batch's own keys never count as cached for it, whichever thread gets to a
+ * key first.  A slot this call claims held no key when it began, so its
+ * generation then is below gen_floor whenever the caller keeps the contract:
+ *   - every key in the table has a generation in [gen_floor, gen) (stamp
+ *     the keys of a table filled otherwise with kvgov_table_gen_stamp);
+ *   - every handle that holds no key has a generation below gen_floor
+ *     (zero the array with the table, or raise gen_floor to the first gen
+ *     after each kvgov_table_init);
+ *   - gen grows from one call to the next.
+ *   mode .. d_digests  as for kvgov_chain_hash.
+ *   d_slots, capacity  the table (as for kvgov_insert).
+ *   d_gen  [capacity + KVGOV_STASH_SLOTS] u32 generations (above).
+ *   d_prefix_blocks  [n_req] int32 output, as for kvgov_probe.
+ *   d_n_new, d_status  as for kvgov_insert_uncached (d_status required).
+ * The table must not be read or written by other calls while this one runs.
+ * A batch too small to give every SM sub-partition two warps (n_req < 2 * 32
+ * * 4 * SMs) runs the chain hash, the probe and the insert as separate
+ * launches instead; the results are the same.  EINVAL: as for
+ * kvgov_chain_hash and kvgov_insert_uncached, d_gen NULL, gen_floor > gen.
+ */
+int kvgov_chain_hash_serve(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                           const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                           const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                           uint8_t *d_slots, uint64_t capacity, uint32_t *d_gen, uint32_t gen, uint32_t gen_floor,
+                           int32_t *d_prefix_blocks, unsigned long long *d_n_new, uint32_t *d_status,
+                           kvgov_stream_t stream);
+
+/*
  * Arrival-order serving of one batch -- paper section 2.1 (a lookup matches
  * the longest cached prefix of blocks from position 0) and section 4.2
  * (prefill cost is proportional to the uncached tokens), applied request by

@@ -35,6 +35,13 @@
  *                   is free once the chain launch is done.  With no pending
  *                   batch: kvgov_chain_hash_probe.
  *     insert_in_chain = 0: kvgov_chain_hash_probe, then kvgov_insert_uncached.
+ *     insert_in_chain = 2 (KVGOV_SCHEDULE_ONE_LAUNCH): kvgov_chain_hash_serve,
+ *                   batch i's lookups and insert in one launch, with
+ *                   generation g_i in d_gen: the engine stamps the keys
+ *                   already in the table with generation 1 before its first
+ *                   batch (kvgov_table_gen_stamp), gives batch i generation
+ *                   g_i = i + 2, and after a flush raises the floor to the
+ *                   flushing batch's generation; no insert is left pending.
  *                   records probed[s] after the probe (batch i's prefix
  *                   lengths are then valid in d_prefix[s]).
  * The results equal serving the batches one at a time in order.
@@ -55,12 +62,13 @@ extern "C" {
 typedef struct CUevent_st *kvgov_event_t;
 
 #define KVGOV_PIPELINE_MAX_SLOTS 3
+#define KVGOV_SCHEDULE_ONE_LAUNCH 2   /* kvgov_pipeline_desc.insert_in_chain: see above */
 
 /* What an engine serves with; every pointer and handle is the caller's. */
 typedef struct kvgov_pipeline_desc {
     int mode;                     /* KVGOV_UNSALTED / KVGOV_ROOT / KVGOV_BOUNDARY        */
-    int insert_in_chain;          /* 1: the schedule above (needs 3 slots); 0: 2 slots  */
-    int n_slots;                  /* 3 if insert_in_chain, else 2                        */
+    int insert_in_chain;          /* the schedule above: 1 (3 slots), 0 or 2 (2 slots)   */
+    int n_slots;                  /* 3 if insert_in_chain is 1, else 2                   */
     int32_t max_req;              /* capacity of each slot: requests ...                 */
     int64_t max_blocks;           /* ... and blocks                                      */
     /* the cache */
@@ -85,13 +93,18 @@ typedef struct kvgov_pipeline_desc {
     kvgov_event_t free_ev[KVGOV_PIPELINE_MAX_SLOTS];
     kvgov_stream_t prep_stream;
     kvgov_stream_t compute_stream;
+    /* insert_in_chain = 2 only: the table's generations, [capacity +
+       KVGOV_STASH_SLOTS] u32, zeroed by the caller with the table (or left
+       as an earlier engine of this schedule left them), and used by no
+       other engine while this one is alive */
+    uint32_t *d_gen;
 } kvgov_pipeline_desc;
 
 typedef struct kvgov_pipeline kvgov_pipeline;   /* opaque */
 
 /*
  * kvgov_pipeline_create -- check the description and make an engine.
- * EINVAL: bad mode, slot count not 3 (insert_in_chain) or 2, a NULL buffer,
+ * EINVAL: bad mode, insert_in_chain not 0, 1 or 2, slot count not 3 (insert_in_chain = 1) or 2, a NULL buffer,
  * event or stream, max_req < 0 or max_blocks < 0, a bad capacity, salted
  * mode without ids, misaligned digests or table.
  */

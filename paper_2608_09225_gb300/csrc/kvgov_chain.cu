@@ -97,12 +97,25 @@ struct PrevParams {
     uint32_t spin_limit = 0;
 };
 
+// The generations of kFuseServe: per handle (slot, or capacity + 8 + side-
+// store entry) the generation of the batch that claimed it; a key counts as
+// cached for this batch iff floor <= its generation < g.
+struct GenParams {
+    uint32_t *gen = nullptr;
+    uint32_t g = 0;
+    uint32_t floor = 0;
+    unsigned long long *n_new = nullptr;
+    uint32_t spin_limit = 0;
+};
+
 // What the chain kernel does with each digest besides storing it.
 constexpr int kFuseNone = 0;      // nothing (kvgov_chain_hash)
 constexpr int kFuseProbe = 1;     // look it up (kvgov_chain_hash_probe)
 constexpr int kFuseArrival = 2;   // insert it, arrival order (kvgov_chain_hash_arrival)
 constexpr int kFuseInsertPrev = 3;   // insert the previous batch's uncached blocks (kvgov_chain_hash_insert_prev)
 constexpr int kFuseInsertPrevProbe = 4;   // both: the insert, and a lookup giving a lower bound of the prefix
+constexpr int kFuseServe = 5;        // look it up among older batches' keys, insert it if past the prefix
+                                     // (kvgov_chain_hash_serve)
 
 // Big-endian words of principal pi's 32-byte salt.
 __device__ __forceinline__ void load_salt(const uint8_t *salts, int pi, uint32_t sw[8]) {
@@ -132,9 +145,21 @@ __device__ __forceinline__ void load_salt(const uint8_t *salts, int pi, uint32_t
 // the prefix it leaves is a lower bound of the prefix on the table after the
 // insert, and a probe that resumes each walk where it stopped
 // (kvgov_host::probe_resume) makes it exact.
+// kFuseServe: the batch's own lookups and insert in one launch.  A thread
+// whose blocks 0..j-1 were all cached looks block j up, and counts it as
+// cached only if the generation of the key's slot is in [floor, g): written
+// by an earlier batch since the last flush.  Blocks from the first one that
+// is not on are inserted, and a slot claimed gets generation g, written after
+// the claim.  No ordering between the two is needed: a slot that this launch
+// claims was empty when the launch began, so its generation then was below
+// floor (never written since the flush), and a lookup reads either that or
+// g -- both "not cached", as they should be for a key of this batch; and
+// keys of earlier launches, with their generations, are all visible.  The
+// prefix lengths are those of kvgov_probe before the batch's insert, the
+// table and key count those of kvgov_insert_uncached after it.
 template <int MODE, int FUSE>
 __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalParams &a,
-                                           const PrevParams &q = PrevParams{}) {
+                                           const PrevParams &q = PrevParams{}, const GenParams &gp = GenParams{}) {
     __shared__ __align__(16) uint32_t stage[kStages][kR * kSlotWords];
     __shared__ int s_jmax;
     __shared__ unsigned int s_new, s_flags, s_done;   // kFuseArrival counts
@@ -148,7 +173,8 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
     // against 212 us.  The others need none (next comment).
     constexpr bool kIns = FUSE == kFuseInsertPrev || FUSE == kFuseInsertPrevProbe;   // the previous batch's insert
     constexpr bool kLook = FUSE == kFuseProbe || FUSE == kFuseInsertPrevProbe;        // lookups of this batch
-    constexpr bool kLockstep = FUSE == kFuseArrival || kIns;
+    constexpr bool kServe = FUSE == kFuseServe;
+    constexpr bool kLockstep = FUSE == kFuseArrival || kIns || kServe;
     if (kLockstep && tid == 0) { s_new = 0; s_flags = 0; s_done = 0; s_jmax = 0; }
 
     // Per-request set-up and validation.
@@ -313,6 +339,32 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             dst[0] = q0;
             dst[1] = q1;
             if (kLook && hits == j && lookup(p.slots, p.mask, q0, q1)) hits = j + 1;
+            if (kServe) {
+                bool cached = false;
+                if (hits == j) {
+                    const long long hnd = lookup_handle(p.slots, p.mask, q0, q1);
+                    if (hnd >= 0) {
+                        const uint32_t gv = gp.gen[hnd];
+                        cached = gv >= gp.floor && gv < gp.g;
+                    }
+                }
+                if (cached) {
+                    hits = j + 1;
+                } else {                                 // past the prefix: insert block j
+                    const unsigned long long key[4] = {u64_of(q0.x, q0.y), u64_of(q0.z, q0.w), u64_of(q1.x, q1.y),
+                                                       u64_of(q1.z, q1.w)};
+                    if (key_is_zero(key)) {
+                        my_flags |= KVGOV_F_SENTINEL;
+                    } else {
+                        unsigned long long pos = 0;
+                        const InsertResult res = insert_one(
+                            reinterpret_cast<unsigned long long *>(const_cast<uint4 *>(p.slots)), p.mask, key,
+                            gp.spin_limit, &pos);
+                        count_insert(res, my_new, my_flags);
+                        if (res == kNew) gp.gen[pos] = gp.g;
+                    }
+                }
+            }
             if (FUSE == kFuseArrival) {
                 ak[0] = u64_of(q0.x, q0.y); ak[1] = u64_of(q0.z, q0.w);
                 ak[2] = u64_of(q1.x, q1.y); ak[3] = u64_of(q1.z, q1.w);
@@ -351,12 +403,12 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
         if (kLockstep) __syncthreads();
     }
     cp_async_wait<0>();
-    if (kLook && r < p.n_req) p.prefix_blocks[r] = hits;
+    if ((kLook || kServe) && r < p.n_req) p.prefix_blocks[r] = hits;
     if (kIns)
         while (pleft > 0) prev_insert_one();
-    if (FUSE == kFuseArrival || kIns)
-        publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, FUSE == kFuseArrival ? a.n_new : q.n_new,
-                       p.status);
+    if (FUSE == kFuseArrival || kIns || kServe)
+        publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done,
+                       FUSE == kFuseArrival ? a.n_new : (kServe ? gp.n_new : q.n_new), p.status);
 }
 
 template <int MODE, int FUSE>
@@ -375,6 +427,12 @@ __global__ void __launch_bounds__(kR) chain_arrival_kernel(const ChainParams p, 
 template <int MODE, int FUSE>
 __global__ void __launch_bounds__(kR, 8) chain_prev_kernel(const ChainParams p, const PrevParams q) {
     chain_body<MODE, FUSE>(p, ArrivalParams{}, q);
+}
+
+// kFuseServe; at most 64 registers, as chain_prev_kernel.
+template <int MODE>
+__global__ void __launch_bounds__(kR, 8) chain_serve_kernel(const ChainParams p, const GenParams gp) {
+    chain_body<MODE, kFuseServe>(p, ArrivalParams{}, PrevParams{}, gp);
 }
 
 }  // namespace
@@ -434,6 +492,9 @@ struct FuseArgs {
     const int32_t *prev_prefix_blocks = nullptr;
     int32_t *probe_prefix_blocks = nullptr;     // kFuseInsertPrev: probe this batch after the insert ...
     bool probe_complete = true;                 // ... to the end (else: leave a lower bound, see launch_chain)
+    uint32_t *gen = nullptr;                    // kFuseServe: the table's generations, this batch's, the floor
+    uint32_t g = 0;
+    uint32_t gen_floor = 0;
 };
 
 int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
@@ -468,6 +529,9 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
         return kvgov_insert_uncached(const_cast<uint8_t *>(f.slots), f.capacity, f.prev_digests, f.prev_blk_off,
                                      f.prev_n_req, f.prev_prefix_blocks, f.n_new, d_status, stream);
     };
+    if (f.fuse == kFuseServe && (!f.slots || !aligned16(f.slots) || !kvgov_host::pow2_capacity(f.capacity) ||
+                                 !f.gen || !d_status || (n_req > 0 && !f.prefix_blocks) || f.gen_floor > f.g))
+        return KVGOV_EINVAL;
     if (n_req == 0) return (f.fuse == kFuseInsertPrev && f.prev_n_req > 0) ? insert_prev() : KVGOV_OK;
 
     ChainParams p;
@@ -504,6 +568,31 @@ int launch_chain(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, in
     // resumes the walks from there; probe_complete = false leaves that probe
     // to the caller (kvgov_host::probe_resume), with 0 as the bound where the
     // launch made no lookups.
+    if (f.fuse == kFuseServe) {
+        if (n_req >= min_fused) {
+            GenParams gp;
+            gp.gen = f.gen;
+            gp.g = f.g;
+            gp.floor = f.gen_floor;
+            gp.n_new = f.n_new;
+            gp.spin_limit = kvgov_host::spin_limit();
+            switch (mode) {
+            case KVGOV_UNSALTED: chain_serve_kernel<KVGOV_UNSALTED><<<grid, kR, 0, s>>>(p, gp); break;
+            case KVGOV_ROOT: chain_serve_kernel<KVGOV_ROOT><<<grid, kR, 0, s>>>(p, gp); break;
+            default: chain_serve_kernel<KVGOV_BOUNDARY><<<grid, kR, 0, s>>>(p, gp); break;
+            }
+            return kvgov_host::launch_status();
+        }
+        // a small batch: the chain, the probe (every key in the table is of an
+        // older batch), then the insert with this batch's generation
+        int rc = launch_plain(mode, grid, s, p);
+        if (rc == KVGOV_OK)
+            rc = kvgov_probe(f.slots, f.capacity, d_digests, d_blk_off, n_req, f.prefix_blocks, d_status, stream);
+        if (rc == KVGOV_OK)
+            rc = kvgov_host::insert_uncached_gen(const_cast<uint8_t *>(f.slots), f.capacity, d_digests, d_blk_off,
+                                                 n_req, f.prefix_blocks, f.n_new, d_status, f.gen, f.g, stream);
+        return rc;
+    }
     if (f.fuse == kFuseInsertPrev) {
         int rc;
         bool lower = false;                        // probe_prefix_blocks holds the lookups' lower bound
@@ -651,3 +740,22 @@ int chain_insert_prev_lower(int mode, const int32_t *d_tokens, const int64_t *d_
                         stream);
 }
 }  // namespace kvgov_host
+
+extern "C" int kvgov_chain_hash_serve(int mode, const int32_t *d_tokens, const int64_t *d_tok_off, int32_t n_req,
+                                      const int32_t *d_principal, const uint8_t *d_salts, int32_t n_principals,
+                                      const int32_t *d_boundary_tok, const int64_t *d_blk_off, uint8_t *d_digests,
+                                      uint8_t *d_slots, uint64_t capacity, uint32_t *d_gen, uint32_t gen,
+                                      uint32_t gen_floor, int32_t *d_prefix_blocks, unsigned long long *d_n_new,
+                                      uint32_t *d_status, kvgov_stream_t stream) {
+    FuseArgs f;
+    f.fuse = kFuseServe;
+    f.slots = d_slots;
+    f.capacity = capacity;
+    f.prefix_blocks = d_prefix_blocks;
+    f.n_new = d_n_new;
+    f.gen = d_gen;
+    f.g = gen;
+    f.gen_floor = gen_floor;
+    return launch_chain(mode, d_tokens, d_tok_off, n_req, d_principal, d_salts, n_principals, d_boundary_tok,
+                        d_blk_off, d_digests, d_status, f, stream);
+}

@@ -50,6 +50,12 @@ int launch_chain_split(int mode, const int32_t *d_tokens, const int64_t *d_tok_o
 int probe_resume(const uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests, const int64_t *d_blk_off,
                  int32_t n_req, int32_t *d_prefix_blocks, uint32_t *d_status, kvgov_stream_t stream);
 
+// kvgov_insert_uncached; with d_gen, every slot or side-store entry it claims
+// gets generation `gen` (kvgov_table.cu).
+int insert_uncached_gen(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests, const int64_t *d_blk_off,
+                        int32_t n_req, const int32_t *d_prefix_blocks, unsigned long long *d_n_new,
+                        uint32_t *d_status, uint32_t *d_gen, uint32_t gen, kvgov_stream_t stream);
+
 // kvgov_chain_hash_insert_prev without the probe's completion: d_prefix_lower
 // receives, for every request, a lower bound of its cached prefix on the
 // table after the insert (what the chain launch's own lookups found while

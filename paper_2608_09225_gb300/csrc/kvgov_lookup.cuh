@@ -43,6 +43,26 @@ __device__ __forceinline__ bool lookup(const uint4 *__restrict__ slots, unsigned
     return false;
 }
 
+// lookup() returning the key's handle -- the slot that holds it, or
+// capacity + 8 + its side-store entry -- or -1 if it is absent.
+__device__ __forceinline__ long long lookup_handle(const uint4 *__restrict__ slots, unsigned long long mask, uint4 q0,
+                                                   uint4 q1) {
+    const unsigned long long k0 = u64_of(q0.x, q0.y), k1 = u64_of(q0.z, q0.w);
+    if (key_in_stash(k0, k1, u64_of(q1.x, q1.y), u64_of(q1.z, q1.w)))
+        return stash_lookup_handle(slots, mask, q0, q1);
+    const unsigned long long window = probe_window(mask);
+    unsigned long long pos = k0 & mask;
+    for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
+        const uint4 a = __ldg(slots + 2 * pos);
+        if ((a.x | a.y | a.z | a.w) == 0u) return -1;
+        if (a.x == q0.x && a.y == q0.y && a.z == q0.z && a.w == q0.w) {
+            const uint4 b = __ldg(slots + 2 * pos + 1);
+            if (b.x == q1.x && b.y == q1.y && b.z == q1.z && b.w == q1.w) return (long long)pos;
+        }
+    }
+    return -1;
+}
+
 // The home slot of the key q0 || q1.
 __device__ __forceinline__ unsigned long long home_slot(uint4 q0, unsigned long long mask) {
     return u64_of(q0.x, q0.y) & mask;

@@ -22,6 +22,11 @@ struct kvgov_pipeline {
     int last = -1;                                 // slot of the last batch whose chain launch was queued
     bool used[KVGOV_PIPELINE_MAX_SLOTS] = {};
     int32_t n_req[KVGOV_PIPELINE_MAX_SLOTS] = {};  // the batch in each slot
+    // KVGOV_SCHEDULE_ONE_LAUNCH: the last generation given, the floor, and
+    // whether the table's keys have been stamped with generation 1
+    uint32_t gen = 1;
+    uint32_t gen_floor = 1;
+    bool stamped = false;
 };
 
 namespace {
@@ -52,7 +57,9 @@ int insert_pending(kvgov_pipeline *pl) {
 bool desc_ok(const kvgov_pipeline_desc &d) {
     using kvgov_host::aligned16;
     if (d.mode != KVGOV_UNSALTED && d.mode != KVGOV_ROOT && d.mode != KVGOV_BOUNDARY) return false;
-    if (d.n_slots != (d.insert_in_chain ? 3 : 2)) return false;
+    if (d.insert_in_chain < 0 || d.insert_in_chain > KVGOV_SCHEDULE_ONE_LAUNCH) return false;
+    if (d.n_slots != (d.insert_in_chain == 1 ? 3 : 2)) return false;
+    if (d.insert_in_chain == KVGOV_SCHEDULE_ONE_LAUNCH && !d.d_gen) return false;
     if (d.max_req < 0 || d.max_blocks < 0) return false;
     if (!d.d_slots || !aligned16(d.d_slots) || !kvgov_host::pow2_capacity(d.capacity) || !d.d_status) return false;
     if (d.mode != KVGOV_UNSALTED && (!d.d_ids || !d.d_id_off || d.n_principals <= 0)) return false;
@@ -94,6 +101,7 @@ extern "C" int kvgov_pipeline_submit(kvgov_pipeline *pl, const uint8_t *secret, 
     if ((chain_ev0 == nullptr) != (chain_ev1 == nullptr) || (table_ev0 == nullptr) != (table_ev1 == nullptr))
         return KVGOV_EINVAL;
 
+    if (d.insert_in_chain == KVGOV_SCHEDULE_ONE_LAUNCH && pl->gen == 0xffffffffu) return KVGOV_EINVAL;   // spent
     const int s = (int)(pl->submitted % d.n_slots);
     const kvgov_stream_t ps = d.prep_stream, cs = d.compute_stream;
     const bool salted = d.mode != KVGOV_UNSALTED;
@@ -117,23 +125,36 @@ extern "C" int kvgov_pipeline_submit(kvgov_pipeline *pl, const uint8_t *secret, 
     // compute stream
     if (after) KV_TRY(wait(cs, after));
     KV_TRY(wait(cs, d.prepared[s]));
+    const bool one_launch = d.insert_in_chain == KVGOV_SCHEDULE_ONE_LAUNCH;
     if (flush) {
         KV_TRY(insert_pending(pl));
         KV_TRY(kvgov_table_init(d.d_slots, d.capacity, cs));
+        pl->gen_floor = pl->gen + 1;                  // every generation given so far is below it
+        pl->stamped = true;                           // the table is empty: nothing to stamp
+    }
+    if (one_launch && !pl->stamped) {                 // keys already in the table: generation 1
+        KV_TRY(kvgov_table_gen_stamp(d.d_slots, d.capacity, d.d_gen, 1u, cs));
+        pl->stamped = true;
     }
     if (chain_ev0) KV_TRY(record(chain_ev0, cs));
     // the last command before the chain launch: the next batch's prep starts
     // only once this chain kernel is being placed
     KV_TRY(record(d.chain_start[s], cs));
     pl->last = s;
-    const int q = d.insert_in_chain ? pl->pending : -1;
+    const int q = d.insert_in_chain == 1 ? pl->pending : -1;
     const int32_t *pr = salted ? d_principal : nullptr;
     const uint8_t *sl = salted ? d.d_salts[s] : nullptr;
     const int32_t *bt = d.mode == KVGOV_BOUNDARY ? d_boundary_tok : nullptr;
+    // one launch: the batch's lookups and insert in its chain launch.  Else,
     // with the previous batch's insert in the chain launch, that launch also
     // looks this batch's blocks up (a lower bound of each prefix) and the
     // probe below resumes the walks from there
-    if (q >= 0)
+    if (one_launch) {
+        const uint32_t g = ++pl->gen;
+        KV_TRY(kvgov_chain_hash_serve(d.mode, d_tokens, d_tok_off, n_req, pr, sl, d.n_principals, bt, d.d_blk_off[s],
+                                      d.d_digests[s], d.d_slots, d.capacity, d.d_gen, g, pl->gen_floor,
+                                      d.d_prefix[s], d.d_n_new, d.d_status, cs));
+    } else if (q >= 0)
         KV_TRY(kvgov_host::chain_insert_prev_lower(d.mode, d_tokens, d_tok_off, n_req, pr, sl, d.n_principals, bt,
                                                    d.d_blk_off[s], d.d_digests[s], d.d_slots, d.capacity,
                                                    d.d_digests[q], d.d_blk_off[q], pl->n_req[q], d.d_prefix[q],
@@ -146,7 +167,10 @@ extern "C" int kvgov_pipeline_submit(kvgov_pipeline *pl, const uint8_t *secret, 
         KV_TRY(record(d.free_ev[q], cs));             // the previous batch is cached: its slot is free
         pl->pending = -1;
     }
-    if (d.insert_in_chain) {
+    if (one_launch) {
+        KV_TRY(record(d.probed[s], cs));
+        KV_TRY(record(d.free_ev[s], cs));            // the batch is cached: its slot is free
+    } else if (d.insert_in_chain) {
         if (q >= 0) {                                 // the probe after the insert
             if (table_ev0) KV_TRY(record(table_ev0, cs));
             KV_TRY(kvgov_host::probe_resume(d.d_slots, d.capacity, d.d_digests[s], d.d_blk_off[s], n_req,

@@ -139,4 +139,22 @@ static __device__ __noinline__ bool stash_lookup(const uint4 *slots, unsigned lo
     return false;
 }
 
+// stash_lookup returning the key's handle (capacity + 8 + its entry), or -1.
+static __device__ __noinline__ long long stash_lookup_handle(const uint4 *slots, unsigned long long mask, uint4 q0,
+                                                             uint4 q1) {
+    const uint4 *base = slots + 2 * (mask + 1);
+    const uint32_t *count = reinterpret_cast<const uint32_t *>(base);
+    const uint32_t *state = count + 8;
+    const uint32_t seen = __ldg(count);
+    const int n = seen < (uint32_t)KVGOV_STASH_KEYS ? (int)seen : KVGOV_STASH_KEYS;
+    for (int e = 0; e < n; ++e) {
+        if (__ldg(state + e) != kStashLive) continue;
+        const uint4 a = __ldg(base + 2 * (kStashHeaderSlots + e)), b = __ldg(base + 2 * (kStashHeaderSlots + e) + 1);
+        if (a.x == q0.x && a.y == q0.y && a.z == q0.z && a.w == q0.w && b.x == q1.x && b.y == q1.y && b.z == q1.z &&
+            b.w == q1.w)
+            return (long long)(mask + 1 + kStashHeaderSlots + e);
+    }
+    return -1;
+}
+
 }  // namespace kvgov_dev

@@ -321,7 +321,8 @@ constexpr int kPackReq = 8;
 __global__ void __launch_bounds__(kInsertThreads) insert_uncached_packed_kernel(
     unsigned long long *__restrict__ slots, unsigned long long mask, const uint4 *__restrict__ digests,
     const int64_t *__restrict__ blk_off, int32_t n_req, const int32_t *__restrict__ prefix_blocks,
-    unsigned long long *n_new, uint32_t *status, uint32_t spin_limit) {
+    unsigned long long *n_new, uint32_t *status, uint32_t spin_limit, uint32_t *gen, uint32_t g) {
+    // gen: nullable; a slot (or side-store entry) this launch claims gets generation g
     __shared__ unsigned int s_new, s_flags, s_done;
     if (threadIdx.x == 0) { s_new = 0; s_flags = 0; s_done = 0; }
     __syncthreads();
@@ -374,7 +375,12 @@ __global__ void __launch_bounds__(kInsertThreads) insert_uncached_packed_kernel(
                     mine = false;
                 }
             }
-            if (mine) count_insert(insert_one(slots, mask, key, spin_limit), my_new, my_flags);
+            if (mine) {
+                unsigned long long pos = 0;
+                const InsertResult res = insert_one(slots, mask, key, spin_limit, &pos);
+                count_insert(res, my_new, my_flags);
+                if (gen && res == kNew) gen[pos] = g;
+            }
         }
     }
     publish_counts(my_new, my_flags, &s_new, &s_flags, &s_done, n_new, status);
@@ -467,6 +473,16 @@ extern "C" int kvgov_probe(const uint8_t *d_slots, uint64_t capacity, const uint
 extern "C" int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,
                                      const int64_t *d_blk_off, int32_t n_req, const int32_t *d_prefix_blocks,
                                      unsigned long long *d_n_new, uint32_t *d_status, kvgov_stream_t stream) {
+    return kvgov_host::insert_uncached_gen(d_slots, capacity, d_digests, d_blk_off, n_req, d_prefix_blocks, d_n_new,
+                                           d_status, nullptr, 0, stream);
+}
+
+// kvgov_insert_uncached, a slot it claims getting generation `gen` when
+// d_gen is given (kvgov_chain_hash_serve's small-batch path).
+int kvgov_host::insert_uncached_gen(uint8_t *d_slots, uint64_t capacity, const uint8_t *d_digests,
+                                    const int64_t *d_blk_off, int32_t n_req, const int32_t *d_prefix_blocks,
+                                    unsigned long long *d_n_new, uint32_t *d_status, uint32_t *d_gen, uint32_t gen,
+                                    kvgov_stream_t stream) {
     using kvgov_host::aligned16;
     if (!d_slots || !aligned16(d_slots) || !kvgov_host::pow2_capacity(capacity) || n_req < 0 || !d_status)
         return KVGOV_EINVAL;
@@ -477,7 +493,43 @@ extern "C" int kvgov_insert_uncached(uint8_t *d_slots, uint64_t capacity, const 
     if (grid > 152ll * 64) grid = 152ll * 64;
     insert_uncached_packed_kernel<<<(unsigned)grid, kInsertThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
         reinterpret_cast<unsigned long long *>(d_slots), capacity - 1, reinterpret_cast<const uint4 *>(d_digests),
-        d_blk_off, n_req, d_prefix_blocks, d_n_new, d_status, g_spin_limit.load());
+        d_blk_off, n_req, d_prefix_blocks, d_n_new, d_status, g_spin_limit.load(), d_gen, gen);
+    return kvgov_host::launch_status();
+}
+
+namespace {
+
+// gen[h] = value for every handle h that holds a key (main slots whose first
+// half is not zero, live side-store entries), 0 for every other.
+__global__ void gen_stamp_kernel(const uint4 *__restrict__ slots, unsigned long long capacity,
+                                 uint32_t *__restrict__ gen, uint32_t value) {
+    const unsigned long long n = capacity + KVGOV_STASH_SLOTS;
+    const uint32_t *state = reinterpret_cast<const uint32_t *>(slots + 2 * capacity) + 8;
+    const uint32_t handed = *reinterpret_cast<const uint32_t *>(slots + 2 * capacity);
+    for (unsigned long long h = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; h < n;
+         h += (unsigned long long)gridDim.x * blockDim.x) {
+        bool held;
+        if (h < capacity) {
+            const uint4 a = slots[2 * h];
+            held = (a.x | a.y | a.z | a.w) != 0u;
+        } else {
+            const long long e = (long long)(h - capacity) - kStashHeaderSlots;   // side-store entry
+            held = e >= 0 && e < (long long)handed && e < KVGOV_STASH_KEYS && state[e] == kStashLive;
+        }
+        gen[h] = held ? value : 0u;
+    }
+}
+
+}  // namespace
+
+extern "C" int kvgov_table_gen_stamp(const uint8_t *d_slots, uint64_t capacity, uint32_t *d_gen, uint32_t value,
+                                     kvgov_stream_t stream) {
+    if (!d_slots || !kvgov_host::aligned16(d_slots) || !kvgov_host::pow2_capacity(capacity) || !d_gen)
+        return KVGOV_EINVAL;
+    unsigned long long grid = (capacity + KVGOV_STASH_SLOTS + 255) / 256;
+    if (grid > 152ull * 64) grid = 152ull * 64;
+    gen_stamp_kernel<<<(unsigned)grid, 256, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+        reinterpret_cast<const uint4 *>(d_slots), capacity, d_gen, value);
     return kvgov_host::launch_status();
 }
 

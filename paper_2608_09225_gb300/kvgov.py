@@ -35,6 +35,7 @@ _p = ctypes.c_void_p
 
 
 MAX_SLOTS = 3
+SCHEDULE_ONE_LAUNCH = 2   # kvgov_pipeline_desc.insert_in_chain: KVGOV_SCHEDULE_ONE_LAUNCH
 _S3 = _p * MAX_SLOTS
 
 
@@ -46,7 +47,7 @@ class PipelineDesc(ctypes.Structure):
                 ("d_ids", _p), ("d_id_off", _p), ("n_principals", ctypes.c_int32),
                 ("d_salts", _S3), ("d_blk_off", _S3), ("d_digests", _S3), ("d_prefix", _S3),
                 ("prepared", _S3), ("chain_start", _S3), ("probed", _S3), ("free_ev", _S3),
-                ("prep_stream", _p), ("compute_stream", _p)]
+                ("prep_stream", _p), ("compute_stream", _p), ("d_gen", _p)]
 
 
 class KVGovError(RuntimeError):
@@ -78,6 +79,10 @@ def _load():
                                                    _p, _p, _p, _p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p,
                                                    _p, _p, _p]
         L.kvgov_table_init.argtypes = [_p, ctypes.c_uint64, _p]
+        L.kvgov_table_gen_stamp.argtypes = [_p, ctypes.c_uint64, _p, ctypes.c_uint32, _p]
+        L.kvgov_chain_hash_serve.argtypes = [ctypes.c_int, _p, _p, ctypes.c_int32, _p, _p, ctypes.c_int32, _p, _p, _p,
+                                             _p, ctypes.c_uint64, _p, ctypes.c_uint32, ctypes.c_uint32, _p, _p, _p,
+                                             _p]
         L.kvgov_insert.argtypes = [_p, ctypes.c_uint64, _p, ctypes.c_int64, _p, _p, _p]
         L.kvgov_probe.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p]
         L.kvgov_probe_resume.argtypes = [_p, ctypes.c_uint64, _p, _p, ctypes.c_int32, _p, _p, _p]
@@ -105,6 +110,7 @@ def _load():
         L.kvgov_pipeline_destroy.restype = None
         for fn in ("kvgov_block_offsets", "kvgov_count_blocks", "kvgov_derive_salts", "kvgov_chain_hash", "kvgov_table_init",
                    "kvgov_insert", "kvgov_probe", "kvgov_probe_resume", "kvgov_insert_uncached",
+                   "kvgov_table_gen_stamp", "kvgov_chain_hash_serve",
                    "kvgov_chain_hash_probe",
                    "kvgov_owner_init", "kvgov_insert_arrival", "kvgov_probe_arrival", "kvgov_chain_hash_arrival",
                    "kvgov_divergence_boundary", "kvgov_response_key", "kvgov_origami",
@@ -261,6 +267,50 @@ def chain_hash_probe(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, blk
                                     _dev(prefix_blocks, torch.int32, "prefix_blocks") if n else _dummy(tokens),
                                     _dev(status, torch.int32, "status", True), _stream(stream)),
            "kvgov_chain_hash_probe")
+    return digests, prefix_blocks
+
+
+def new_gen(slots: torch.Tensor) -> torch.Tensor:
+    """A zeroed generation array for a table (kvgov_chain_hash_serve)."""
+    return torch.zeros(slots.shape[0], dtype=torch.int32, device=slots.device)
+
+
+def table_gen_stamp(slots: torch.Tensor, gen: torch.Tensor, value: int, stream=None):
+    """gen[h] = value for every handle holding a key, 0 for the others."""
+    _check(lib().kvgov_table_gen_stamp(_dev(slots, torch.uint8, "slots"), capacity_of(slots),
+                                       _dev(gen, torch.int32, "gen"), int(value), _stream(stream)),
+           "kvgov_table_gen_stamp")
+
+
+def chain_hash_serve(mode: int, tokens: torch.Tensor, tok_off: torch.Tensor, blk_off: torch.Tensor,
+                     slots: torch.Tensor, gen: torch.Tensor, g: int, gen_floor: int, status: torch.Tensor,
+                     principal: torch.Tensor | None = None, salts: torch.Tensor | None = None,
+                     boundary_tok: torch.Tensor | None = None, digests: torch.Tensor | None = None,
+                     n_blocks: int | None = None, n_new: torch.Tensor | None = None,
+                     prefix_blocks: torch.Tensor | None = None, stream=None):
+    """The serving step of one batch in one launch: its digests, its prefix
+    lengths against the keys of generation [gen_floor, g), and its uncached
+    blocks inserted with generation g.  Returns (digests, prefix_blocks)."""
+    L = lib()
+    n = tok_off.numel() - 1
+    if digests is None:
+        if n_blocks is None:
+            n_blocks = int(blk_off[-1].item())
+        digests = torch.empty((n_blocks, 32), dtype=torch.uint8, device=tokens.device)
+    if prefix_blocks is None:
+        prefix_blocks = torch.empty(max(n, 0), dtype=torch.int32, device=tokens.device)
+    if tokens.numel() == 0:
+        tokens = torch.zeros(4, dtype=torch.int32, device=tok_off.device)
+    n_p = 0 if salts is None else salts.shape[0]
+    _check(L.kvgov_chain_hash_serve(
+        int(mode), _dev(tokens, torch.int32, "tokens"), _dev(tok_off, torch.int64, "tok_off"), n,
+        _dev(principal, torch.int32, "principal", True), _dev(salts, torch.uint8, "salts", True), n_p,
+        _dev(boundary_tok, torch.int32, "boundary_tok", True), _dev(blk_off, torch.int64, "blk_off"),
+        _dev(digests, torch.uint8, "digests") if digests.numel() else _dummy(tokens),
+        _dev(slots, torch.uint8, "slots"), capacity_of(slots), _dev(gen, torch.int32, "gen"), int(g), int(gen_floor),
+        _dev(prefix_blocks, torch.int32, "prefix_blocks") if n else _dummy(tokens),
+        _dev(n_new, torch.int64, "n_new", True), _dev(status, torch.int32, "status"), _stream(stream)),
+        "kvgov_chain_hash_serve")
     return digests, prefix_blocks
 
 

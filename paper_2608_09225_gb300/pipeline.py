@@ -70,6 +70,7 @@ class PrefixCache:
         self.slots = torch.empty((self.capacity + K.STASH_SLOTS, 32), dtype=torch.uint8, device=self.device)
         self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
         self.n_new = torch.zeros(1, dtype=torch.int64, device=self.device)
+        self.gen = None        # the table's generations, made by the first one-launch engine on it
         K.table_init(self.slots, self.stream)
         self.derive_salts()
 
@@ -146,6 +147,9 @@ class _Pipelined:
     chain launch (or drain()), and three slots rotate.
     insert_in_chain=False: the chain hash with the probe fused in, then the
     insert; two slots.
+    one_launch=True (overrides insert_in_chain): batch i's lookups and its
+    own insert in its chain launch (kvgov_chain_hash_serve), told apart by
+    the table's generations (cache.gen); two slots, nothing left pending.
 
     Either way every probe sees the table exactly as the previous batch's
     insert left it.  A flush (submit(..., flush=True)) first runs a pending
@@ -153,14 +157,18 @@ class _Pipelined:
     """
 
     def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_blocks: int, device="cuda",
-                 insert_in_chain: bool = True):
+                 insert_in_chain: bool = True, one_launch: bool = False):
         self.cache, self.mode = cache, mode
         self.device = torch.device(device)
-        self.insert_in_chain = insert_in_chain
+        self.one_launch = one_launch
+        self.insert_in_chain = insert_in_chain and not one_launch
+        schedule = K.SCHEDULE_ONE_LAUNCH if one_launch else int(bool(insert_in_chain))
+        if one_launch and getattr(cache, "gen", None) is None:
+            cache.gen = K.new_gen(cache.slots)       # the table's generations, zeroed with it
         self.prep_stream = torch.cuda.Stream(self.device)
         self.compute_stream = torch.cuda.Stream(self.device, priority=-1)
         cache.stream = self.compute_stream
-        n_slots = 3 if insert_in_chain else 2
+        n_slots = 3 if schedule == 1 else 2
         self.slots = []
         for _ in range(n_slots):
             self.slots.append({
@@ -172,7 +180,7 @@ class _Pipelined:
                 "free": torch.cuda.Event(),
             })
         d = K.PipelineDesc()
-        d.mode, d.insert_in_chain, d.n_slots = int(mode), int(insert_in_chain), n_slots
+        d.mode, d.insert_in_chain, d.n_slots = int(mode), schedule, n_slots
         d.max_req, d.max_blocks = int(max_req), int(max_blocks)
         d.d_slots, d.capacity = cache.slots.data_ptr(), cache.capacity
         d.d_status, d.d_n_new = cache.status.data_ptr(), cache.n_new.data_ptr()
@@ -186,6 +194,7 @@ class _Pipelined:
             d.probed[i] = K.event_handle(sl["probed"], cs)
             d.free_ev[i] = K.event_handle(sl["free"], cs)
         d.prep_stream, d.compute_stream = self.prep_stream.cuda_stream, cs.cuda_stream
+        d.d_gen = cache.gen.data_ptr() if one_launch else None
         self.engine = K.Engine(d)
         self._after = [torch.cuda.Event() for _ in self.slots]
         self._i = 0
@@ -255,9 +264,9 @@ class HostPipeline(_Pipelined):
     """
 
     def __init__(self, cache: PrefixCache, mode: int, max_req: int, max_tokens: int, device="cuda",
-                 insert_in_chain: bool = True):
+                 insert_in_chain: bool = True, one_launch: bool = False):
         max_blocks, _ = K.count_blocks([0, max_tokens])        # no batch of max_tokens tokens has more
-        super().__init__(cache, mode, max_req, max_blocks, device, insert_in_chain)
+        super().__init__(cache, mode, max_req, max_blocks, device, insert_in_chain, one_launch)
         self.copy_stream = torch.cuda.Stream(self.device)
         self.out_stream = torch.cuda.Stream(self.device)
         for s in self.slots:

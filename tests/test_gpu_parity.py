@@ -788,6 +788,76 @@ def test_chain_hash_insert_prev_with_probe(kv, mode, n_req, stride):
     assert (want[prev_req][ppre == 0] == (np.diff(blk_ref)[prev_req][ppre == 0])).all()   # inserted: all hit
 
 
+def _repeat_requests(b: W.Batch, idx) -> W.Batch:
+    """The batch of b's requests idx (repeats allowed), in that order."""
+    parts = [b.tokens[b.tok_off[r]:b.tok_off[r + 1]] for r in idx]
+    tok_off = np.concatenate([[0], np.cumsum([len(x) for x in parts])]).astype(np.int64)
+    tokens = np.concatenate(parts + [np.zeros(4, np.int32)]).astype(np.int32)
+    return W.Batch(tokens, tok_off, b.principal[idx].copy(), b.boundary_tok[idx].copy())
+
+
+@pytest.mark.parametrize("mode", [0, 1, 2])
+@pytest.mark.parametrize("n_req", [180, 40960], ids=["separate_launches", "fused"])
+def test_chain_hash_serve_matches_probe_then_insert(kv, mode, n_req):
+    """kvgov_chain_hash_serve over a sequence of batches -- a fresh one, the
+    same one again (every block now cached), a new batch whose requests come
+    in pairs (a key the batch itself adds never counts as cached for it,
+    whichever copy gets there first), then a flush with the floor raised and
+    the first batch twice more -- gives, batch by batch, the digests of
+    kvgov_chain_hash, the prefix lengths of the oracle's set before the
+    batch's insert, and after it the set and key count of inserting every
+    block past the prefix (paper section 2.1).  Keys in the table before the
+    first batch are stamped with generation 1."""
+    rng = np.random.default_rng(11 * n_req + mode)
+    b0 = W.ragged(41 + mode, list(rng.integers(0, 300, n_req)))
+    fresh = W.ragged(43 + mode, list(rng.integers(0, 300, n_req)))
+    pairs = _repeat_requests(fresh, np.repeat(np.arange(n_req // 2), 2))
+    salts = oracle.derive_salts(b"serve", *W.principal_ids(8))
+    d_salts = dev(salts) if mode else None
+    cap = 1 << 22
+    slots = kv.new_table(cap)
+    gen = kv.new_gen(slots)
+    st, n_new = status_tensor(), torch.zeros(1, dtype=torch.int64, device=DEV)
+    ref0 = oracle.chain_hash(mode, b0.tokens, b0.tok_off, b0.principal, salts, b0.boundary_tok)
+    present = ref0[rng.random(len(ref0)) < 0.05]               # a few of the first batch's blocks, cached before
+    kv.insert(slots, dev(present), st)
+    kv.table_gen_stamp(slots, gen, 1)
+    ks = oracle.KeySet(1)
+    ks.insert(present)
+    start_n = ks.n
+    g, floor = 1, 1
+    for step, (b, flush) in enumerate([(b0, False), (b0, False), (pairs, False), (b0, True), (b0, False)]):
+        if flush:                                               # the table emptied; every generation so far below
+            kv.table_init(slots)
+            floor = g + 1
+            ks, start_n = oracle.KeySet(1), 0
+            n_new.zero_()
+        g += 1
+        toks, tok_off = dev(b.tokens, np.int32), dev(b.tok_off, np.int64)
+        blk = kv.block_offsets(tok_off, status=st)
+        pr = dev(b.principal, np.int32) if mode else None
+        bt = dev(b.boundary_tok, np.int32) if mode == 2 else None
+        blk_ref = oracle.block_offsets(b.tok_off)
+        dig, pre = kv.chain_hash_serve(mode, toks, tok_off, blk, slots, gen, g, floor, st, principal=pr,
+                                       salts=d_salts, boundary_tok=bt, n_blocks=int(blk_ref[-1]), n_new=n_new)
+        torch.cuda.synchronize()
+        assert int(st.item()) == 0
+        ref = oracle.chain_hash(mode, b.tokens, b.tok_off, b.principal, salts, b.boundary_tok)
+        assert (dig.cpu().numpy() == ref).all(), f"step {step}: digests differ"
+        want = ks.prefix_blocks(ref, blk_ref)
+        got = pre.cpu().numpy()
+        assert (got == want).all(), f"step {step}: {int((got != want).sum())} of {b.n} prefix lengths differ"
+        rows = np.concatenate([np.arange(blk_ref[r] + want[r], blk_ref[r + 1]) for r in range(b.n)] +
+                              [np.zeros(0, np.int64)]).astype(np.int64)
+        ks.insert(ref[rows])
+        assert int(n_new.item()) == ks.n - start_n, f"step {step}: key count"
+        if step == 1 or step == 4:                              # the same batch again: every block cached
+            assert (want == np.diff(blk_ref)).all()
+        if step == 2:                                           # a new batch in pairs: nothing cached for it
+            assert (want == 0).all() and len(rows) > 0
+    assert table_keys(slots) == {r.tobytes() for r in ks.contents()}
+
+
 def test_probe_empty_and_bad_offsets(kv):
     slots = kv.new_table(64)
     st = status_tensor()

@@ -14,6 +14,14 @@ from tests.pins import run_workload_oracle
 
 pytestmark = pytest.mark.gpu
 
+# the serving engine's schedules: the insert in the next batch's chain launch, the insert after the
+# chain hash and the probe, and the lookups and insert in the batch's own chain launch
+SCHEDULES = ["insert_in_chain", "inline", "one_launch"]
+
+
+def sched(schedule):
+    return {"insert_in_chain": schedule == "insert_in_chain", "one_launch": schedule == "one_launch"}
+
 
 def run_gpu(kv, w: W.Workload, mode: int):
     """Salts, chains, table fill (same content as the oracle's) and probe."""
@@ -185,8 +193,8 @@ def test_full_wide_device_pipeline_matches_oracle(kv):
     assert mins == [0, 4, 8, 8, 4]
 
 
-@pytest.mark.parametrize("in_chain", [True, False], ids=["insert_in_chain", "inline"])
-def test_device_pipeline_empty_and_tiny_batches(kv, in_chain):
+@pytest.mark.parametrize("schedule", SCHEDULES)
+def test_device_pipeline_empty_and_tiny_batches(kv, schedule):
     """Batches of no requests, of one request shorter than a block, and
     ordinary batches, mixed in one stream through the serving engine: the
     empty ones give empty results and leave the cache alone, the others match
@@ -199,7 +207,7 @@ def test_device_pipeline_empty_and_tiny_batches(kv, in_chain):
     short_toks = b.tokens[:7].copy()
     short = DeviceBatch.from_host(short_toks, np.array([0, 7], np.int64), b.principal[:1], b.boundary_tok[:1])
     cache = PrefixCache(1 << 12, w.secret, w.ids, w.id_off)
-    pipe = DevicePipeline(cache, W.ROOT, b.n, full.n_blocks, insert_in_chain=in_chain)
+    pipe = DevicePipeline(cache, W.ROOT, b.n, full.n_blocks, **sched(schedule))
     order = [empty, full, empty, short, full, empty]
     copies = []
     for db in order:
@@ -226,8 +234,8 @@ def test_device_pipeline_empty_and_tiny_batches(kv, in_chain):
     assert int(cache.n_new.item()) == ks.n
 
 
-@pytest.mark.parametrize("in_chain", [True, False], ids=["insert_in_chain", "inline"])
-def test_host_pipeline_matches_device_serving(kv, in_chain):
+@pytest.mark.parametrize("schedule", SCHEDULES)
+def test_host_pipeline_matches_device_serving(kv, schedule):
     """Batches served from pinned host memory through HostPipeline (copies
     overlapping the previous batch's serving; each batch's result read only
     after the next batch is queued) give the prefix lengths of the same
@@ -239,7 +247,7 @@ def test_host_pipeline_matches_device_serving(kv, in_chain):
     dev_cache = PrefixCache(1 << 18, w0.secret, w0.ids, w0.id_off)
     host_cache = PrefixCache(1 << 18, w0.secret, w0.ids, w0.id_off)
     n_tok = int(w0.batch.tok_off[-1])
-    pipe = HostPipeline(host_cache, W.BOUNDARY, w0.batch.n, n_tok, insert_in_chain=in_chain)
+    pipe = HostPipeline(host_cache, W.BOUNDARY, w0.batch.n, n_tok, **sched(schedule))
     order = [0, 1, 2, 0, 3, 1]
     got, want, pending = [], [], None
     for i, k in enumerate(order):
@@ -269,23 +277,23 @@ def test_host_pipeline_matches_device_serving(kv, in_chain):
     assert [int(x.min()) for x in want] == [0, 4, 4, 8, 4, 4]
 
 
-@pytest.mark.parametrize("in_chain", [True, False], ids=["insert_in_chain", "inline"])
+@pytest.mark.parametrize("schedule", SCHEDULES)
 @pytest.mark.parametrize("mode", [W.UNSALTED, W.ROOT, W.BOUNDARY])
-def test_device_pipeline_matches_sequential_serving(kv, mode, in_chain):
+def test_device_pipeline_matches_sequential_serving(kv, mode, schedule):
     """DevicePipeline (salts and block offsets of batch i+1 on a prep stream
     beside batch i's chain hash; batch i's insert inside batch i+1's chain
     launch, or inline) gives the prefix lengths and the key count of serving
     the same batches one by one, across secret changes and a flush of the
     cache between batches."""
-    ws = [W.make("wide", seed=300 + i, n_req=20000) for i in range(3)]
+    ws = [W.make("wide", seed=300 + i, n_req=40960) for i in range(3)]   # the fused launches
     for w in ws[1:]:
         w.batch.tokens.reshape(-1, 128)[:, :64] = ws[0].batch.tokens[:64]
     w0 = ws[0]
     dbs = [DeviceBatch.from_host(w.batch.tokens, w.batch.tok_off, w.batch.principal, w.batch.boundary_tok)
            for w in ws]
-    seq = PrefixCache(1 << 19, w0.secret, w0.ids, w0.id_off)
-    pip = PrefixCache(1 << 19, w0.secret, w0.ids, w0.id_off)
-    pipe = DevicePipeline(pip, mode, w0.batch.n, dbs[0].n_blocks, insert_in_chain=in_chain)
+    seq = PrefixCache(1 << 21, w0.secret, w0.ids, w0.id_off)
+    pip = PrefixCache(1 << 21, w0.secret, w0.ids, w0.id_off)
+    pipe = DevicePipeline(pip, mode, w0.batch.n, dbs[0].n_blocks, **sched(schedule))
     order = [0, 1, 2, 0, 1, 2, 0]
     got, want = [], []
     for i, k in enumerate(order):
@@ -312,9 +320,9 @@ def test_device_pipeline_matches_sequential_serving(kv, mode, in_chain):
         assert int(want[1].min()) == 4
 
 
-@pytest.mark.parametrize("in_chain", [True, False], ids=["insert_in_chain", "inline"])
+@pytest.mark.parametrize("schedule", SCHEDULES)
 @pytest.mark.parametrize("flush_at", [None, 5])
-def test_device_pipeline_back_to_back_matches_oracle(kv, flush_at, in_chain):
+def test_device_pipeline_back_to_back_matches_oracle(kv, flush_at, schedule):
     """Many batches queued without waiting in between (and a cache flush
     queued in the middle): every batch's prefix lengths, copied out on the
     compute stream right after its submit, match the oracle's replay of the
@@ -326,7 +334,7 @@ def test_device_pipeline_back_to_back_matches_oracle(kv, flush_at, in_chain):
     dbs = [DeviceBatch.from_host(w.batch.tokens, w.batch.tok_off, w.batch.principal, w.batch.boundary_tok)
            for w in ws]
     cache = PrefixCache(1 << 17, w0.secret, w0.ids, w0.id_off)
-    pipe = DevicePipeline(cache, W.BOUNDARY, w0.batch.n, dbs[0].n_blocks, insert_in_chain=in_chain)
+    pipe = DevicePipeline(cache, W.BOUNDARY, w0.batch.n, dbs[0].n_blocks, **sched(schedule))
     order = [0, 1, 2, 3, 2, 0, 1, 3]
     copies = []
     for i, k in enumerate(order):

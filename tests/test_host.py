@@ -68,7 +68,8 @@ def _engine_desc(insert_in_chain=1):
     checks below run before any CUDA call)."""
     from paper_2608_09225_gb300.kvgov import PipelineDesc
     d = PipelineDesc()
-    d.mode, d.insert_in_chain, d.n_slots = 2, insert_in_chain, 3 if insert_in_chain else 2
+    d.mode, d.insert_in_chain, d.n_slots = 2, insert_in_chain, 3 if insert_in_chain == 1 else 2
+    d.d_gen = 0x60000 if insert_in_chain == 2 else None
     d.max_req, d.max_blocks = 100, 800
     d.d_slots, d.capacity, d.d_status, d.d_n_new = 0x10000, 1 << 10, 0x20000, 0x30000
     d.d_ids, d.d_id_off, d.n_principals = 0x40000, 0x50000, 4
@@ -103,6 +104,9 @@ def test_serving_engine_checks_its_arguments(libkv):
     d = _engine_desc(); d.probed[1] = 0; bad.append(d)               # missing event
     d = _engine_desc(); d.d_ids = 0; bad.append(d)                   # salted mode without ids
     d = _engine_desc(); d.max_req = -1; bad.append(d)
+    d = _engine_desc(3); d.n_slots = 2; bad.append(d)                # no such schedule
+    d = _engine_desc(2); d.d_gen = None; bad.append(d)              # one launch needs the generations
+    d = _engine_desc(2); d.n_slots = 3; bad.append(d)                # ... and takes 2 slots
     for d in bad:
         assert libkv.kvgov_pipeline_create(ctypes.byref(d), ctypes.byref(h)) == 1
     d = _engine_desc()
@@ -127,6 +131,10 @@ def test_serving_engine_checks_its_arguments(libkv):
     assert libkv.kvgov_pipeline_drain(h) == 0                         # nothing pending: nothing queued
     libkv.kvgov_pipeline_destroy(h)
     libkv.kvgov_pipeline_destroy(None)
+    d = _engine_desc(2)                                               # one launch: generations, 2 slots
+    assert libkv.kvgov_pipeline_create(ctypes.byref(d), ctypes.byref(h)) == 0 and h.value
+    assert submit(n_req=101) == 1 and libkv.kvgov_pipeline_pending(h) == 0
+    libkv.kvgov_pipeline_destroy(h)
 
 
 def test_peak_gather_rejects_bad_arguments():
