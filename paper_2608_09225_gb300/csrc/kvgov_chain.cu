@@ -340,17 +340,13 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
             dst[1] = q1;
             if (kLook && hits == j && lookup(p.slots, p.mask, q0, q1)) hits = j + 1;
             if (kServe) {
-                bool cached = false;
-                if (hits == j) {
-                    const long long hnd = lookup_handle(p.slots, p.mask, q0, q1);
-                    if (hnd >= 0) {
-                        const uint32_t gv = gp.gen[hnd];
-                        cached = gv >= gp.floor && gv < gp.g;
-                    }
-                }
-                if (cached) {
+                // -1 not looked up or not found, 0 found but added by this batch, 1 cached
+                int found = -1;
+                unsigned long long start = 0;            // where the insert's walk may begin
+                if (hits == j) found = lookup_serve(p.slots, p.mask, gp.gen, gp.floor, gp.g, q0, q1, &start);
+                if (found == 1) {
                     hits = j + 1;
-                } else {                                 // past the prefix: insert block j
+                } else if (found < 0) {                  // past the prefix and not in the table yet: insert
                     const unsigned long long key[4] = {u64_of(q0.x, q0.y), u64_of(q0.z, q0.w), u64_of(q1.x, q1.y),
                                                        u64_of(q1.z, q1.w)};
                     if (key_is_zero(key)) {
@@ -359,7 +355,7 @@ __device__ __forceinline__ void chain_body(const ChainParams &p, const ArrivalPa
                         unsigned long long pos = 0;
                         const InsertResult res = insert_one(
                             reinterpret_cast<unsigned long long *>(const_cast<uint4 *>(p.slots)), p.mask, key,
-                            gp.spin_limit, &pos);
+                            gp.spin_limit, &pos, start);
                         count_insert(res, my_new, my_flags);
                         if (res == kNew) gp.gen[pos] = gp.g;
                     }

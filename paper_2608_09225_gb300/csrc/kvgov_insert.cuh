@@ -59,17 +59,21 @@ constexpr uint32_t kSettled = 0x80000000u;
 // kvgov_table.cu; keys the main slots cannot hold go to the side store
 // (kvgov_stash.cuh).  On kNew and kDuplicate, *pos receives the key's handle:
 // the slot that holds it, or capacity + 8 + its side-store entry.
+// start: the walk begins start slots past the home slot -- the caller has
+// seen each slot before it holding a complete first half (both words non-
+// zero) other than the key's, which is final.
 __device__ __forceinline__ InsertResult insert_one(unsigned long long *slots, unsigned long long mask,
                                                    const unsigned long long k[4], uint32_t spin_limit,
-                                                   unsigned long long *pos_out = nullptr) {
+                                                   unsigned long long *pos_out = nullptr,
+                                                   unsigned long long start = 0) {
     if (key_in_stash(k[0], k[1], k[2], k[3])) {
         const StashResult r = stash_insert(slots, mask, k[0], k[1], k[2], k[3], spin_limit);
         if (pos_out && (r.res == kNew || r.res == kDuplicate)) *pos_out = r.pos;
         return static_cast<InsertResult>(r.res);
     }
     const unsigned long long window = probe_window(mask);
-    unsigned long long pos = k[0] & mask;
-    for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
+    unsigned long long pos = (k[0] + start) & mask;
+    for (unsigned long long n = start; n < window; ++n, pos = (pos + 1) & mask) {
         unsigned long long *slot = slots + 4 * pos;
         unsigned long long o0 = 0ull, o1 = 0ull;
         // Look first (measured: it turns the step after a cache flush, where

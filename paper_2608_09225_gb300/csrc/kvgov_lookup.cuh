@@ -63,6 +63,52 @@ __device__ __forceinline__ long long lookup_handle(const uint4 *__restrict__ slo
     return -1;
 }
 
+// The lookup of kvgov_chain_hash_serve: 1 = the key is in the table with a
+// generation in [floor, g) (cached for this batch), 0 = it is in the table
+// with another generation (added by this batch: nothing to insert), -1 = not
+// found.  On -1, *start is where an insert of the key may begin its walk:
+// the offset from the home slot of the first slot not seen holding a
+// complete first half (both words non-zero) other than the key's.  The home
+// slot's generation is read with the home slot, where most keys are found.
+__device__ __forceinline__ int lookup_serve(const uint4 *__restrict__ slots, unsigned long long mask,
+                                            const uint32_t *gen, uint32_t floor, uint32_t g, uint4 q0, uint4 q1,
+                                            unsigned long long *start) {
+    *start = 0;
+    const unsigned long long k0 = u64_of(q0.x, q0.y), k1 = u64_of(q0.z, q0.w);
+    if (key_in_stash(k0, k1, u64_of(q1.x, q1.y), u64_of(q1.z, q1.w))) {
+        const long long h = stash_lookup_handle(slots, mask, q0, q1);
+        if (h < 0) return -1;
+        const uint32_t gv = gen[h];
+        return gv >= floor && gv < g ? 1 : 0;
+    }
+    const unsigned long long window = probe_window(mask);
+    const unsigned long long home = k0 & mask;
+    const uint32_t gv_home = gen[home];
+    bool open = true;                                   // every slot so far: a complete first half, not the key's
+    unsigned long long pos = home;
+    for (unsigned long long n = 0; n < window; ++n, pos = (pos + 1) & mask) {
+        const uint4 a = __ldg(slots + 2 * pos);
+        if ((a.x | a.y | a.z | a.w) == 0u) {
+            if (open) *start = n;
+            return -1;
+        }
+        const bool mine = a.x == q0.x && a.y == q0.y && a.z == q0.z && a.w == q0.w;
+        if (mine) {
+            const uint4 b = __ldg(slots + 2 * pos + 1);
+            if (b.x == q1.x && b.y == q1.y && b.z == q1.z && b.w == q1.w) {
+                const uint32_t gv = n == 0 ? gv_home : gen[pos];
+                return gv >= floor && gv < g ? 1 : 0;
+            }
+        }
+        if (open && (mine || (a.x | a.y) == 0u || (a.z | a.w) == 0u)) {
+            *start = n;                                 // an insert must look at this slot itself
+            open = false;
+        }
+    }
+    if (open) *start = window;
+    return -1;
+}
+
 // The home slot of the key q0 || q1.
 __device__ __forceinline__ unsigned long long home_slot(uint4 q0, unsigned long long mask) {
     return u64_of(q0.x, q0.y) & mask;
