@@ -59,7 +59,8 @@ CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain k
 # the kernel's sources still hash to that value.
 CHAIN_TRAFFIC = {"chain_prev_kernel": {"bytes_per_launch": 200526208,
                  "source_sha256": "85d072705de98f8ea01e70bcc93f66213122131b53e0fc6a62e5e966b7fa9585"},
-                 "chain_serve_kernel": {"bytes_per_launch": None, "source_sha256": None}}
+                 "chain_serve_kernel": {"bytes_per_launch": 200615680,
+                                        "source_sha256": "52af8c54f8c6451df2dbc9061d535a943eddfef2585ff18ad682ffa8e47f2718"}}
 
 
 # DRAM bytes per launch of the probe on the probe-heavy workload from one ncu
@@ -461,7 +462,7 @@ def main():
     ap.add_argument("--seed", type=int, default=None, help="base seed (default: fresh per run)")
     ap.add_argument("--cpu-sample", type=int, default=16384, help="requests per oracle step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--schedule", default="insert_in_chain", choices=["insert_in_chain", "inline", "one_launch"],
+    ap.add_argument("--schedule", default="one_launch", choices=["insert_in_chain", "inline", "one_launch"],
                     help="insert_in_chain: each batch's insert runs inside the next batch's chain-hash launch, and "
                          "each batch is probed after its chain hash; inline: chain hash with the fused probe, then "
                          "the insert; one_launch: each batch's lookups and insert in its own chain-hash launch "
