@@ -229,7 +229,8 @@ class DevicePipeline(_Pipelined):
     submit() returns (prefix_blocks, event) on the device: prefix_blocks is
     valid once event has completed and is overwritten by a later submit (the
     second or third after it).  The batch's uncached blocks are in the table
-    once the next submit's chain launch or drain() has run.  The batch's
+    once the next submit's chain launch or drain() has run (with one_launch,
+    once its own chain launch has: when the event has completed).  The batch's
     tensors are used on the pipeline's streams after the work queued so far
     on the caller's current stream.
     """
