@@ -96,7 +96,9 @@ typedef struct kvgov_pipeline_desc {
     /* insert_in_chain = 2 only: the table's generations, [capacity +
        KVGOV_STASH_SLOTS] u32, zeroed by the caller with the table (or left
        as an earlier engine of this schedule left them), and used by no
-       other engine while this one is alive */
+       other engine while this one is alive.  From the engine's first submit
+       on, the table must change only through it: a key added otherwise has
+       no generation of this engine's and would not count as cached. */
     uint32_t *d_gen;
 } kvgov_pipeline_desc;
 

@@ -150,6 +150,8 @@ class _Pipelined:
     one_launch=True (overrides insert_in_chain): batch i's lookups and its
     own insert in its chain launch (kvgov_chain_hash_serve), told apart by
     the table's generations (cache.gen); two slots, nothing left pending.
+    The keys already in the cache count as cached from the first submit on;
+    after that the cache must change only through this pipeline.
 
     Either way every probe sees the table exactly as the previous batch's
     insert left it.  A flush (submit(..., flush=True)) first runs a pending
