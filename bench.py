@@ -69,7 +69,7 @@ TABLE_SOURCES = ["paper_2608_09225_gb300/csrc/kvgov_table.cu", "paper_2608_09225
                  "paper_2608_09225_gb300/csrc/kvgov_stash.cuh", "paper_2608_09225_gb300/csrc/kvgov_internal.cuh",
                  "paper_2608_09225_gb300/csrc/kvgov_insert.cuh"]
 TABLE_TRAFFIC = {"probe_share_kernel<16, true>": {
-    "bytes_per_launch": 74626560, "source_sha256": "de6cb50b8070f52df5d1f6fc0b028f2a93c84958701b43431ccb540876ba6856"}}
+    "bytes_per_launch": 74561792, "source_sha256": "c4f89d4058529d0c53f612bec5fb827b26dad802c885253c7535f69eebcba2aa"}}
 
 
 def load_peaks() -> dict:
