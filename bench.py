@@ -60,7 +60,7 @@ CHAIN_HEADER = "include/kvgov.h"      # only its #define lines reach the chain k
 CHAIN_TRAFFIC = {"chain_prev_kernel": {"bytes_per_launch": 200526208,
                  "source_sha256": "85d072705de98f8ea01e70bcc93f66213122131b53e0fc6a62e5e966b7fa9585"},
                  "chain_serve_kernel": {"bytes_per_launch": 200615680,
-                                        "source_sha256": "52af8c54f8c6451df2dbc9061d535a943eddfef2585ff18ad682ffa8e47f2718"}}
+                                        "source_sha256": "0619a12914dd648e870c7a6cacd06f92e38e46c2757b83ac2424d8d226fd7827"}}
 
 
 # DRAM bytes per launch of the probe on the probe-heavy workload from one ncu

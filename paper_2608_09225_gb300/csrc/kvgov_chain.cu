@@ -148,9 +148,11 @@ __device__ __forceinline__ void load_salt(const uint8_t *salts, int pi, uint32_t
 // kFuseServe: the batch's own lookups and insert in one launch.  A thread
 // whose blocks 0..j-1 were all cached looks block j up, and counts it as
 // cached only if the generation of the key's slot is in [floor, g): written
-// by an earlier batch since the last flush.  Blocks from the first one that
-// is not on are inserted, and a slot claimed gets generation g, written after
-// the claim.  No ordering between the two is needed: a slot that this launch
+// by an earlier batch since the last flush.  From the first block that is
+// not cached on, the blocks are inserted -- but for one that the lookup found
+// already added by this batch -- and a slot claimed gets generation g, written
+// after the claim; the first such block's insert starts its walk where the
+// lookup's stopped.  No ordering between the two is needed: a slot that this launch
 // claims was empty when the launch began, so its generation then was below
 // floor (never written since the flush), and a lookup reads either that or
 // g -- both "not cached", as they should be for a key of this batch; and
